@@ -1,0 +1,438 @@
+#!/usr/bin/env python
+"""Throughput of the quaternion convolution forward (libquan) on synthetic layers.
+
+One step = one full pass of the hot path (staging, on-chip Hamilton block expansion,
+contraction, bias/IQBN/activation epilogue, store) over one batch of the workload.
+Default workload: the CIFAR-shaped layer N=128, 32x32, 64->64 real channels, 3x3 s1
+p1, fused IQBN + ReLU, bf16 in / fp32 accumulate.  Other workloads: --workload
+c2a | c2b | c3a | c3b (ImageNet / detection-neck layers) | backbone (ResNet-18-style,
+images/s).
+
+Prints one JSON line.  Under torchrun every rank runs its own copy of the workload on
+its own GPU (the batch shards with no exchange step: weak scaling); the timed region
+is bracketed by a barrier and a device synchronisation and the max over ranks is taken.
+--impl reference times the fp64 CPU oracle on the host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "QConv fwd real-equiv TFLOP/s & % bf16 tensor peak (1 GB300); backbone images/s"
+L2_BYTES = 126 * 1024 * 1024
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="c1",
+                    choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target duration of the bounded oracle sample")
+    return ap.parse_args()
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in ("hbm_gbs", "bf16_tflops", "bf16_tflops_sustained")}, \
+            "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2509_05512_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or
+    None when no capture exists or the kernel sources changed since it was taken."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f).get(workload)
+    except (OSError, ValueError):
+        return None
+    if not rec or rec.get("kernel_sha") != kernel_source_hash():
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling while the GPU is busy."""
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.proc = None
+        self.file = tempfile.NamedTemporaryFile(mode="w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", gpu_id, "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = [ln.strip().split(", ") for ln in self.file if ln.strip()]
+        os.unlink(self.file.name)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, r[5:9]):
+                if v.strip() == "Active":
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------- layers
+
+class LayerRunner:
+    """Device buffers for one layer, rotated so that consecutive steps never find their
+    inputs in L2."""
+
+    def __init__(self, spec, torch, quan, inputs):
+        import numpy as np
+        self.spec, self.torch, self.quan = spec, torch, quan
+        d = inputs.layer_inputs(spec)
+        dev = torch.device("cuda")
+
+        def up(a):
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(
+                torch.bfloat16).to(dev)
+
+        self.host = d
+        x0 = up(d["x"])
+        self.w = [up(d[k]) for k in ("wr", "wi", "wj", "wk")]
+        f32 = lambda a: None if a is None else torch.from_numpy(a).to(dev)
+        self.bias, self.scale, self.shift = f32(d["bias"]), f32(d["scale"]), f32(d["shift"])
+        out_elems = spec.N * spec.Ho * spec.Wo * spec.Cout
+        per_set = (x0.numel() + out_elems) * 2
+        self.sets = max(2, min(16, math.ceil(2 * L2_BYTES / per_set)))
+        self.xs = [x0] + [x0.clone() for _ in range(self.sets - 1)]
+        self.outs = [torch.empty((spec.N, spec.Ho, spec.Wo, spec.Cout), dtype=torch.bfloat16,
+                                 device=dev) for _ in range(self.sets)]
+        self.i = 0
+        self.launches_per_step = 1
+        self.footprint = per_set * self.sets
+
+    def step(self, stream):
+        s, q = self.spec, self.quan
+        k = self.i % self.sets
+        self.i += 1
+        q.quan_qconv2d_fwd(self.xs[k], *self.w, self.bias, self.scale, self.shift, s.N, s.H,
+                           s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                           self.outs[k], stream)
+
+    # end to end: pinned host inputs -> device -> kernel -> host
+    def e2e_setup(self):
+        torch = self.torch
+        import numpy as np
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        d = self.host
+        self.h_x = pin(d["x"].view(np.int16))
+        self.h_w = [pin(d[k].view(np.int16)) for k in ("wr", "wi", "wj", "wk")]
+        self.h_p = [pin(d[k]) if d[k] is not None else None for k in ("bias", "scale", "shift")]
+        s = self.spec
+        self.h_out = torch.empty((s.N, s.Ho, s.Wo, s.Cout), dtype=torch.int16).pin_memory()
+        self.e_x = torch.empty_like(self.h_x, device="cuda")
+        self.e_w = [torch.empty_like(t, device="cuda") for t in self.h_w]
+        self.e_p = [torch.empty_like(t, device="cuda") if t is not None else None
+                    for t in self.h_p]
+        self.e_out = torch.empty_like(self.h_out, device="cuda")
+        self.h2d = self.h_x.numel() * 2 + sum(t.numel() * 2 for t in self.h_w) + sum(
+            t.numel() * 4 for t in self.h_p if t is not None)
+        self.d2h = self.h_out.numel() * 2
+
+    def e2e_step(self, stream):
+        s, q = self.spec, self.quan
+        self.e_x.copy_(self.h_x, non_blocking=True)
+        for a, b in zip(self.e_w, self.h_w):
+            a.copy_(b, non_blocking=True)
+        for a, b in zip(self.e_p, self.h_p):
+            if a is not None:
+                a.copy_(b, non_blocking=True)
+        q.quan_qconv2d_fwd(self.e_x, *self.e_w, self.e_p[0], self.e_p[1], self.e_p[2], s.N,
+                           s.H, s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                           self.e_out, stream)
+        self.h_out.copy_(self.e_out, non_blocking=True)
+
+    @property
+    def flops(self):
+        return self.spec.flops
+
+    @property
+    def algorithmic_bytes(self):
+        return self.spec.algorithmic_bytes
+
+
+def cpu_oracle_sample(spec, seconds, inputs):
+    """Time the fp64 oracle on a bounded number of images of the layer."""
+    import oracle
+    d = inputs.layer_inputs(spec, n_images=1)
+    f64 = oracle.bf16_bits_to_f64
+    w = [f64(d[k]) for k in ("wr", "wi", "wj", "wk")]
+
+    def run(n):
+        dd = inputs.layer_inputs(spec, n_images=n)
+        x = f64(dd["x"])
+        t0 = time.perf_counter()
+        oracle.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"],
+                       scale=d["scale"], shift=d["shift"], act=spec.act)
+        return time.perf_counter() - t0
+
+    t1 = run(1)
+    n = max(1, min(spec.N, int(seconds / max(t1, 1e-6))))
+    t = run(n) if n > 1 else t1
+    flop = spec.flops / spec.N * n
+    return {"value": flop / t / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": "%d of %d images of the layer (fp64, %.2f s)" % (n, spec.N, t)}
+
+
+# ---------------------------------------------------------------------------- main
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2509_05512_gb300 import inputs
+
+    if args.impl == "reference":
+        return reference_arm(args, rank, world, inputs)
+
+    import torch
+    from paper_2509_05512_gb300 import build, quan
+
+    torch.cuda.set_device(local_rank)
+    build.build_library()
+    quan.load()
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    if args.workload == "backbone":
+        from paper_2509_05512_gb300 import backbone
+        runner = backbone.BackboneRunner(torch, quan, inputs)
+        unit, per_step_units, dtype = "images/s", runner.N, "bf16"
+        workload_desc = runner.describe()
+    else:
+        spec = inputs.LAYERS[args.workload]
+        runner = LayerRunner(spec, torch, quan, inputs)
+        unit, per_step_units, dtype = "TFLOP/s", spec.flops / 1e12, "bf16"
+        workload_desc = {
+            "c1": "configs[1]: CIFAR-shaped QUAN layer",
+            "c2a": "configs[2] layer a: ImageNet ResNet-stage layer",
+            "c2b": "configs[2] layer b: ImageNet ResNet-stage stride-2 layer",
+            "c3a": "configs[3] layer a: detection-neck pointwise layer",
+            "c3b": "configs[3] layer b: detection-neck 3x3 layer",
+        }[args.workload]
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+
+    # warm-up: at least W steps, and enough untimed steps for the clocks to settle
+    gpu_id = getattr(torch.cuda.get_device_properties(local_rank), "uuid", None)
+    gpu_id = ("GPU-" + str(gpu_id)) if gpu_id is not None else str(local_rank)
+    sampler = ClockSampler(gpu_id) if rank == 0 else None
+    t_end = time.perf_counter() + 1.0
+    n = 0
+    while n < args.warmup or time.perf_counter() < t_end:
+        runner.step(sh)
+        n += 1
+        if n % 64 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+
+    barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        runner.step(sh)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = ev0.elapsed_time(ev1)
+    clocks = sampler.stop() if sampler else None
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    st, bits = quan.quan_device_status(sh)
+    if st != quan.QUAN_OK:
+        raise RuntimeError("kernel reported a timeout (bits 0x%x)" % bits)
+    ms_per_step = ms / args.steps
+    value = per_step_units * args.steps * world / (ms / 1e3)
+
+    # end to end through the public call with host buffers
+    e2e = None
+    if not args.no_e2e:
+        runner.e2e_setup()
+        for _ in range(3):
+            runner.e2e_step(sh)
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            runner.e2e_step(sh)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ems = e0.elapsed_time(e1)
+        if dist is not None:
+            t = torch.tensor([ems], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": per_step_units * args.steps * world / (ems / 1e3), "unit": unit,
+               "h2d_bytes_per_step": int(runner.h2d), "d2h_bytes_per_step": int(runner.d2h)}
+
+    peaks, peak_src = load_peaks()
+    roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        if args.workload == "backbone":
+            cpu = runner.cpu_baseline(args.cpu_seconds)
+        else:
+            cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs)
+
+    if dist is not None:
+        dist.destroy_process_group()
+    if rank != 0:
+        return 0
+    cfg = {"workload": workload_desc, "l2": "inputs larger than L2: %d rotating buffer sets, "
+           "%.0f MB" % (getattr(runner, "sets", 1), runner.footprint / 1e6),
+           "parallelism": "replicas over the batch (dp%d, no collective)" % world}
+    if args.workload != "backbone":
+        s = runner.spec
+        cfg.update({"N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin, "Cout": s.Cout,
+                    "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
+                    "epilogue": "IQBN+ReLU", "flops_per_step": s.flops,
+                    "path": {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")})
+    else:
+        cfg.update(runner.config())
+    line = {"metric": METRIC, "value": round(value, 4), "unit": unit, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
+            "data": "synthetic (seeded; shapes of the paper's workloads)", "config": cfg,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": runner.launches_per_step * args.steps, "clocks": clocks}
+    print(json.dumps(line))
+    return 0
+
+
+def runner_roofline(runner, args, ms_per_step, peaks, peak_src):
+    if args.workload == "backbone":
+        return runner.roofline(peaks, peak_src)
+    flops, nbytes = runner.flops, runner.algorithmic_bytes
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    t = ms_per_step / 1e3  # one kernel launch per step
+    if flops / nbytes >= ridge:
+        achieved, peak, unit, bound = flops / t / 1e12, peaks["bf16_tflops"], "TFLOP/s", "tensor"
+    else:
+        achieved, peak, unit, bound = nbytes / t / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
+    return {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
+            "frac": round(achieved / peak, 4), "traffic": recorded_traffic(args.workload),
+            "kernel": "qconv_tc_kernel", "peak_source": peak_src + " (burst)",
+            "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
+
+
+def reference_arm(args, rank, world, inputs):
+    """The fp64 CPU oracle as the reference arm: each step is a bounded sample of the
+    same workload (rank 0 only)."""
+    if rank != 0:
+        return 0
+    import oracle
+    if args.workload == "backbone":
+        from paper_2509_05512_gb300 import backbone_ref
+        return backbone_ref.reference_arm(args, METRIC)
+    spec = inputs.LAYERS[args.workload]
+    d = inputs.layer_inputs(spec, n_images=1)
+    f64 = oracle.bf16_bits_to_f64
+    x = f64(d["x"])
+    w = [f64(d[k]) for k in ("wr", "wi", "wj", "wk")]
+
+    def step():
+        oracle.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"],
+                       scale=d["scale"], shift=d["shift"], act=spec.act)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    per_step = spec.flops / spec.N  # one image per step
+    value = per_step * args.steps / dt / 1e12
+    cpu = {"value": value, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+           "sample": "1 of %d images of the layer per step (fp64)" % spec.N}
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": args.workload, "N": spec.N, "H": spec.H, "W": spec.W,
+                       "Cin": spec.Cin, "Cout": spec.Cout},
+            "cpu_baseline": cpu,
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

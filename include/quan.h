@@ -1,0 +1,159 @@
+/*
+ * quan.h -- libquan: quaternion convolution forward for NVIDIA GB300 (sm_103a).
+ *
+ * Implements the forward pass of the QUAN quaternion convolution (Grant & Wang,
+ * "Quaternion Approximate Networks for Enhanced Image Classification and Oriented
+ * Object Detection", arXiv 2509.05512):
+ *   - the full Hamilton-product convolution of Sec. III-B, Eq. 5, whose real
+ *     weight is the signed 4x4 block matrix of Eq. 6 built from four letter tensors
+ *     W_r, W_i, W_j, W_k (weight on the left: Y = W (x) X, Hamilton product of Eq. 3);
+ *   - Independent Quaternion Batch Normalization in inference form (Sec. III-C,
+ *     Eq. 11-12), folded by the caller into one scale and one shift per real channel;
+ *   - a split (per real component) activation (ReLU or SiLU, Sec. IV-E ablation);
+ *   - component-wise max pooling (the QSPPF pooling rule of Sec. III-D).
+ *
+ * Conventions shared by every entry point
+ *   Layout      x is NHWC [N][H][W][C_in]; the C_in real channels are four
+ *               component-major blocks [r | i | j | k] of Q_in = C_in / 4 channels, so
+ *               channel c = comp * Q_in + ci.  The output is [N][Ho][Wo][C_out] with
+ *               the same component-major order.  Each letter tensor w_L is
+ *               [Q_out][kh][kw][Q_in], contiguous.  Ho = (H + 2 pad - kh) / stride + 1
+ *               (floor), likewise Wo.
+ *   Convolution "convolution" is a cross-correlation (no kernel flip) with zero padding.
+ *   Epilogue    out = act(scale[c] * (acc + bias[c]) + shift[c] (+ residual)), every
+ *               per-channel vector fp32 [C_out]; a NULL bias is 0, a NULL scale/shift pair
+ *               is the identity (scale and shift must both be NULL or both non-NULL).
+ *   Memory      every tensor pointer is a DEVICE pointer owned by the caller; the library
+ *               keeps no reference after the call and allocates nothing per call.
+ *               `out` must not overlap any input.
+ *   Streams     calls are asynchronous on `stream` (a cudaStream_t; NULL is the legacy
+ *               default stream) and do not synchronise.
+ *   Errors      argument errors are detected on the host before anything is launched and
+ *               return QUAN_ERR_INVALID_ARG or QUAN_ERR_UNSUPPORTED; a launch failure
+ *               returns QUAN_ERR_CUDA.  quan_last_error_message() describes the last error
+ *               of the calling thread.  Kernel-side timeouts are reported by
+ *               quan_device_status().
+ */
+#ifndef QUAN_H_
+#define QUAN_H_
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* quan_stream_t;
+
+typedef enum {
+    QUAN_OK = 0,
+    QUAN_ERR_INVALID_ARG = 1,     /* null pointer, bad size, C % 4 != 0, overlap, ... */
+    QUAN_ERR_UNSUPPORTED = 2,     /* valid arguments no compiled path can run */
+    QUAN_ERR_CUDA = 3,            /* CUDA runtime or launch error */
+    QUAN_ERR_DEVICE_TIMEOUT = 4   /* a kernel's bounded wait ran out (quan_device_status) */
+} quan_status_t;
+
+typedef enum { QUAN_ACT_NONE = 0, QUAN_ACT_RELU = 1, QUAN_ACT_SILU = 2 } quan_act_t;
+
+typedef enum {
+    QUAN_PATH_AUTO = 0, /* tensor-core path when the shape allows it, else CUDA cores */
+    QUAN_PATH_TC = 1,   /* tcgen05 implicit GEMM; UNSUPPORTED if the shape does not allow it */
+    QUAN_PATH_SIMT = 2  /* CUDA-core direct convolution */
+} quan_path_t;
+
+/*
+ * Quaternion convolution forward, bfloat16 tensors, fp32 accumulation.
+ * Sec. III-B Eq. 5 (Hamilton product of Eq. 3 per tap and channel), Eq. 6 block weight,
+ * IQBN inference epilogue of Eq. 11-12.
+ *   x            bf16 [N][H][W][Cin]           (device)
+ *   wr,wi,wj,wk  bf16 [Cout/4][kh][kw][Cin/4]  (device), the letter tensors of Eq. 5
+ *   bias         fp32 [Cout] or NULL           (device)
+ *   iqbn_scale   fp32 [Cout] or NULL           (device)  gamma / sqrt(var + eps)
+ *   iqbn_shift   fp32 [Cout] or NULL           (device)  beta - mean * scale
+ *   N,H,W        batch and input size, >= 1
+ *   Cin, Cout    real channel counts, multiples of 4
+ *   kh,kw        filter size >= 1; stride >= 1; pad >= 0; Ho, Wo >= 1
+ *   act          quan_act_t
+ *   out          bf16 [N][Ho][Wo][Cout]        (device), rounded to nearest even
+ * The tensor-core path needs Cin/4 and Cout/4 to be multiples of 16 and 16-byte aligned
+ * tensor pointers; other shapes run on CUDA cores.  Returns QUAN_OK once launched.
+ */
+quan_status_t quan_qconv2d_fwd(const void* x, const void* wr, const void* wi, const void* wj,
+                               const void* wk, const float* bias, const float* iqbn_scale,
+                               const float* iqbn_shift, int N, int H, int W, int Cin, int Cout,
+                               int kh, int kw, int stride, int pad, int act, void* out,
+                               quan_stream_t stream);
+
+/* Same operation with fp32 x, weights and out (CUDA-core fp32 FFMA path). */
+quan_status_t quan_qconv2d_fwd_f32(const float* x, const float* wr, const float* wi,
+                                   const float* wj, const float* wk, const float* bias,
+                                   const float* iqbn_scale, const float* iqbn_shift, int N, int H,
+                                   int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                   int act, float* out, quan_stream_t stream);
+
+/*
+ * bf16 quaternion convolution that adds `residual` (bf16 [N][Ho][Wo][Cout], device, same
+ * layout as out; may not overlap out) after the IQBN affine and before the activation:
+ *   out = act(scale * (acc + bias) + shift + residual).
+ * This is the second convolution of a residual basic block in the ResNet-style backbone.
+ */
+quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi, const void* wj,
+                                   const void* wk, const float* bias, const float* iqbn_scale,
+                                   const float* iqbn_shift, int N, int H, int W, int Cin,
+                                   int Cout, int kh, int kw, int stride, int pad, int act,
+                                   const void* residual, void* out, quan_stream_t stream);
+
+/*
+ * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,
+ * QSPPF), bf16 NHWC [N][H][W][C] -> [N][Ho][Wo][C], window k x k, stride, zero-size
+ * padding that never wins.  C is any positive count.
+ */
+quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,
+                                 int pad, void* out, quan_stream_t stream);
+
+/* Select the path of later quan_qconv2d_fwd / _res calls in this process (default AUTO). */
+quan_status_t quan_set_path(int path);
+/* Path (quan_path_t, TC or SIMT) the last successful convolution call of this thread ran. */
+int quan_last_path(void);
+
+/*
+ * Tensor-core tile override for later calls (0 = automatic): kappa = quaternion input
+ * channels per K block (16, 32 or 64), bnq = quaternion output channels per tile
+ * (16, 32 or 64), max_ctas = persistent grid size cap.  Values that do not divide the
+ * layer make the call fail with QUAN_ERR_UNSUPPORTED.
+ */
+quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas);
+
+/*
+ * Tensor-core operand reuse (default 0): each input-component tile feeds four
+ * consecutive MMAs (one per output component); with reuse on, the MMA unit keeps it in
+ * its A-operand collector instead of reading shared memory four times.  0 turns the
+ * reuse off (same results, more shared-memory traffic).
+ */
+quan_status_t quan_set_tc_a_reuse(int enable);
+
+/* Time limit of every bounded wait inside the tensor-core kernel, in nanoseconds
+ * (default 2e9).  0 restores the default. */
+quan_status_t quan_set_wait_limit_ns(unsigned long long ns);
+
+/*
+ * Synchronises `stream`, then reads and clears the device status word that kernels set
+ * when a bounded wait runs out.  Returns QUAN_ERR_DEVICE_TIMEOUT if any bit was set
+ * (the bits are stored in *bits when bits != NULL), QUAN_ERR_CUDA on a CUDA error.
+ */
+quan_status_t quan_device_status(quan_stream_t stream, unsigned int* bits);
+
+/* Test hook: when enabled, the tensor-core kernel's MMA role waits on a barrier nothing
+ * arrives on, so every role's bounded wait runs out and the kernel reports a timeout
+ * through quan_device_status() while leaving the context usable. */
+quan_status_t quan_set_fault_injection(int enable);
+
+const char* quan_status_string(quan_status_t status);
+const char* quan_last_error_message(void);
+/* Library version as major * 10000 + minor * 100 + patch. */
+int quan_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QUAN_H_ */

@@ -1,0 +1,60 @@
+// internal.h -- launch interfaces shared by the C-ABI front end (quan_api.cu) and the
+// kernels.  Not part of the public header.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace quan {
+
+// Geometry and epilogue of one quaternion convolution call.  Channels are real
+// channels; Q = C / 4 quaternion channels per component block.
+struct ConvShape {
+    int N, H, W, Cin, Cout, kh, kw, stride, pad, act;
+    int Ho, Wo, Qin, Qout;
+    long long M;  // N * Ho * Wo output pixels
+};
+
+struct EpilogueArgs {
+    const float* bias;   // [Cout] or null
+    const float* scale;  // [Cout] or null (IQBN scale, with shift)
+    const float* shift;  // [Cout] or null
+    const void* residual;  // [M][Cout] (same dtype as out) or null
+};
+
+// Device status word bits (set by kernels whose bounded waits ran out).
+enum : unsigned {
+    STATUS_TIMEOUT_PRODUCER = 1u,
+    STATUS_TIMEOUT_MMA = 2u,
+    STATUS_TIMEOUT_EPILOGUE = 4u,
+    STATUS_TIMEOUT_DRAIN = 8u,
+};
+
+struct TcOptions {
+    int kappa;                    // quaternion input channels per K block (16, 32 or 64); 0 = auto
+    int bnq;                      // quaternion output channels per tile (16, 32 or 64); 0 = auto
+    int max_ctas;                 // persistent grid cap; 0 = number of SMs
+    unsigned long long wait_limit_ns;
+    int inject_stall;             // failure-injection: the MMA role never consumes
+    int a_reuse;                  // reuse each X_p tile from the MMA A collector
+};
+
+// Tensor-core path (tcgen05 + TMA), bf16 in/out, fp32 accumulation.
+bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
+                  const void* residual);
+cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const w[4],
+                            const EpilogueArgs& ep, void* out, const TcOptions& opt,
+                            int num_sms, cudaStream_t stream, char* err, size_t errlen);
+cudaError_t read_and_clear_status(unsigned* status, cudaStream_t stream);
+
+// CUDA-core path, any shape; T = __nv_bfloat16 or float.
+cudaError_t launch_qconv_simt_bf16(const ConvShape& s, const void* x, const void* const w[4],
+                                   const EpilogueArgs& ep, void* out, cudaStream_t stream);
+cudaError_t launch_qconv_simt_f32(const ConvShape& s, const void* x, const void* const w[4],
+                                  const EpilogueArgs& ep, void* out, cudaStream_t stream);
+
+// Per-real-channel max pooling, bf16 NHWC.
+cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
+                                int pad, void* out, int num_sms, cudaStream_t stream);
+
+}  // namespace quan

@@ -1,0 +1,297 @@
+// quan_api.cu -- the C ABI of libquan: argument validation, path selection, launch.
+// See include/quan.h for the contract of every entry point.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <mutex>
+
+#include "internal.h"
+#include "quan.h"
+
+namespace {
+
+thread_local char t_errmsg[512] = "";
+thread_local int t_last_path = 0;
+std::atomic<int> g_path{QUAN_PATH_AUTO};
+std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0};
+std::atomic<unsigned long long> g_wait_limit{2000000000ull};
+std::atomic<int> g_inject{0};
+std::atomic<int> g_a_reuse{0};
+
+constexpr int kMaxDevices = 64;
+int g_num_sms[kMaxDevices] = {0};
+int g_cc[kMaxDevices] = {0};
+std::mutex g_dev_mu;
+
+quan_status_t fail(quan_status_t st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(t_errmsg, sizeof(t_errmsg), fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+quan_status_t cuda_fail(cudaError_t e, const char* what) {
+    return fail(QUAN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Number of SMs and compute capability (major*10+minor) of the current device.
+bool device_info(int* num_sms, int* cc, cudaError_t* err) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        *err = e;
+        return false;
+    }
+    if (dev >= 0 && dev < kMaxDevices) {
+        std::lock_guard<std::mutex> lk(g_dev_mu);
+        if (g_num_sms[dev] == 0) {
+            int sms = 0, maj = 0, mnr = 0;
+            if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) !=
+                    cudaSuccess ||
+                (e = cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev)) !=
+                    cudaSuccess ||
+                (e = cudaDeviceGetAttribute(&mnr, cudaDevAttrComputeCapabilityMinor, dev)) !=
+                    cudaSuccess) {
+                *err = e;
+                return false;
+            }
+            g_num_sms[dev] = sms;
+            g_cc[dev] = maj * 10 + mnr;
+        }
+        *num_sms = g_num_sms[dev];
+        *cc = g_cc[dev];
+        return true;
+    }
+    *err = cudaErrorInvalidDevice;
+    return false;
+}
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+    if (!a || !b) return false;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(a), b0 = reinterpret_cast<uintptr_t>(b);
+    return a0 < b0 + nb && b0 < a0 + na;
+}
+
+quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4],
+                       const float* bias, const float* scale, const float* shift, int N, int H,
+                       int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int act,
+                       const void* residual, const void* out, size_t esize) {
+    if (!x || !w[0] || !w[1] || !w[2] || !w[3] || !out)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if (N < 1 || H < 1 || W < 1 || Cin < 1 || Cout < 1 || kh < 1 || kw < 1 || stride < 1 ||
+        pad < 0)
+        return fail(QUAN_ERR_INVALID_ARG,
+                    "sizes must be positive (N=%d H=%d W=%d Cin=%d Cout=%d kh=%d kw=%d "
+                    "stride=%d) and pad >= 0 (pad=%d)",
+                    N, H, W, Cin, Cout, kh, kw, stride, pad);
+    if (Cin % 4 || Cout % 4)
+        return fail(QUAN_ERR_INVALID_ARG, "Cin=%d and Cout=%d must be multiples of 4", Cin, Cout);
+    if ((scale == nullptr) != (shift == nullptr))
+        return fail(QUAN_ERR_INVALID_ARG, "iqbn_scale and iqbn_shift must both be given or both NULL");
+    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
+    const long long Ho = (static_cast<long long>(H) + 2LL * pad - kh) / stride + 1;
+    const long long Wo = (static_cast<long long>(W) + 2LL * pad - kw) / stride + 1;
+    if (static_cast<long long>(H) + 2LL * pad < kh || static_cast<long long>(W) + 2LL * pad < kw ||
+        Ho < 1 || Wo < 1)
+        return fail(QUAN_ERR_INVALID_ARG, "filter %dx%d larger than the padded input %dx%d", kh,
+                    kw, H + 2 * pad, W + 2 * pad);
+    const long long xin = static_cast<long long>(N) * H * W * Cin;
+    const long long yout = static_cast<long long>(N) * Ho * Wo * Cout;
+    if (xin >= (1LL << 40) || yout >= (1LL << 40) || Ho > 0x7fffffff / Wo)
+        return fail(QUAN_ERR_UNSUPPORTED, "tensor too large");
+    const size_t wbytes = static_cast<size_t>(Cout / 4) * kh * kw * (Cin / 4) * esize;
+    const size_t xbytes = static_cast<size_t>(xin) * esize;
+    const size_t ybytes = static_cast<size_t>(yout) * esize;
+    if (overlaps(out, ybytes, x, xbytes) || overlaps(out, ybytes, w[0], wbytes) ||
+        overlaps(out, ybytes, w[1], wbytes) || overlaps(out, ybytes, w[2], wbytes) ||
+        overlaps(out, ybytes, w[3], wbytes) || overlaps(out, ybytes, residual, ybytes) ||
+        overlaps(out, ybytes, bias, Cout * 4u) || overlaps(out, ybytes, scale, Cout * 4u) ||
+        overlaps(out, ybytes, shift, Cout * 4u))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input");
+    s->N = N; s->H = H; s->W = W; s->Cin = Cin; s->Cout = Cout;
+    s->kh = kh; s->kw = kw; s->stride = stride; s->pad = pad; s->act = act;
+    s->Ho = static_cast<int>(Ho); s->Wo = static_cast<int>(Wo);
+    s->Qin = Cin / 4; s->Qout = Cout / 4;
+    s->M = static_cast<long long>(N) * Ho * Wo;
+    return QUAN_OK;
+}
+
+quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void* wj,
+                       const void* wk, const float* bias, const float* scale, const float* shift,
+                       int N, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                       int act, const void* residual, void* out, quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    quan::ConvShape s;
+    quan_status_t st = validate(&s, x, w, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                                stride, pad, act, residual, out, 2);
+    if (st != QUAN_OK) return st;
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    const int path = g_path.load();
+    const bool tc_ok = cc == 103 && quan::tc_supported(s, x, w, out, residual);
+    bool use_tc;
+    if (path == QUAN_PATH_TC) {
+        if (!tc_ok)
+            return fail(QUAN_ERR_UNSUPPORTED,
+                        "tensor-core path needs sm_103, Cin/4 and Cout/4 multiples of 16 and "
+                        "16-byte aligned tensors (device cc %d, Cin=%d, Cout=%d)",
+                        cc, Cin, Cout);
+        use_tc = true;
+    } else if (path == QUAN_PATH_SIMT) {
+        use_tc = false;
+    } else {
+        use_tc = tc_ok;
+    }
+    const quan::EpilogueArgs ep{bias, scale, shift, residual};
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    if (use_tc) {
+        quan::TcOptions opt;
+        opt.kappa = g_kappa.load();
+        opt.bnq = g_bnq.load();
+        opt.max_ctas = g_max_ctas.load();
+        opt.wait_limit_ns = g_wait_limit.load();
+        opt.inject_stall = g_inject.load();
+        opt.a_reuse = g_a_reuse.load();
+        char err[256] = "";
+        e = quan::launch_qconv_tc(s, x, w, ep, out, opt, num_sms, cs, err, sizeof(err));
+        if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+        if (e != cudaSuccess) return cuda_fail(e, "qconv_tc launch");
+        t_last_path = QUAN_PATH_TC;
+    } else {
+        e = quan::launch_qconv_simt_bf16(s, x, w, ep, out, cs);
+        if (e != cudaSuccess) return cuda_fail(e, "qconv_simt launch");
+        t_last_path = QUAN_PATH_SIMT;
+    }
+    return QUAN_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+quan_status_t quan_qconv2d_fwd(const void* x, const void* wr, const void* wi, const void* wj,
+                               const void* wk, const float* bias, const float* iqbn_scale,
+                               const float* iqbn_shift, int N, int H, int W, int Cin, int Cout,
+                               int kh, int kw, int stride, int pad, int act, void* out,
+                               quan_stream_t stream) {
+    return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                    stride, pad, act, nullptr, out, stream);
+}
+
+quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi, const void* wj,
+                                   const void* wk, const float* bias, const float* iqbn_scale,
+                                   const float* iqbn_shift, int N, int H, int W, int Cin,
+                                   int Cout, int kh, int kw, int stride, int pad, int act,
+                                   const void* residual, void* out, quan_stream_t stream) {
+    if (!residual) return fail(QUAN_ERR_INVALID_ARG, "residual is NULL");
+    return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                    stride, pad, act, residual, out, stream);
+}
+
+quan_status_t quan_qconv2d_fwd_f32(const float* x, const float* wr, const float* wi,
+                                   const float* wj, const float* wk, const float* bias,
+                                   const float* iqbn_scale, const float* iqbn_shift, int N, int H,
+                                   int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                   int act, float* out, quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    quan::ConvShape s;
+    quan_status_t st = validate(&s, x, w, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                                kw, stride, pad, act, nullptr, out, 4);
+    if (st != QUAN_OK) return st;
+    if (g_path.load() == QUAN_PATH_TC)
+        return fail(QUAN_ERR_UNSUPPORTED, "fp32 convolution runs on CUDA cores only");
+    const quan::EpilogueArgs ep{bias, iqbn_scale, iqbn_shift, nullptr};
+    cudaError_t e = quan::launch_qconv_simt_f32(s, x, w, ep, out,
+                                                reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "qconv_simt_f32 launch");
+    t_last_path = QUAN_PATH_SIMT;
+    return QUAN_OK;
+}
+
+quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,
+                                 int pad, void* out, quan_stream_t stream) {
+    if (!x || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if (N < 1 || H < 1 || W < 1 || C < 1 || k < 1 || stride < 1 || pad < 0)
+        return fail(QUAN_ERR_INVALID_ARG, "sizes must be positive and pad >= 0");
+    if (2 * pad > k)
+        return fail(QUAN_ERR_INVALID_ARG, "pad=%d must be at most k/2 (k=%d)", pad, k);
+    if (H + 2 * pad < k || W + 2 * pad < k)
+        return fail(QUAN_ERR_INVALID_ARG, "window larger than the padded input");
+    const long long Ho = (H + 2LL * pad - k) / stride + 1, Wo = (W + 2LL * pad - k) / stride + 1;
+    const size_t xb = static_cast<size_t>(N) * H * W * C * 2;
+    const size_t yb = static_cast<size_t>(N) * Ho * Wo * C * 2;
+    if (overlaps(x, xb, out, yb)) return fail(QUAN_ERR_INVALID_ARG, "out overlaps x");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    e = quan::launch_maxpool_bf16(x, N, H, W, C, k, stride, pad, out, num_sms,
+                                  reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "maxpool launch");
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_path(int path) {
+    if (path < QUAN_PATH_AUTO || path > QUAN_PATH_SIMT)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown path %d", path);
+    g_path.store(path);
+    return QUAN_OK;
+}
+
+int quan_last_path(void) { return t_last_path; }
+
+quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas) {
+    auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };
+    if (!okv(kappa) || !okv(bnq) || max_ctas < 0)
+        return fail(QUAN_ERR_INVALID_ARG, "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0");
+    g_kappa.store(kappa);
+    g_bnq.store(bnq);
+    g_max_ctas.store(max_ctas);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_tc_a_reuse(int enable) {
+    g_a_reuse.store(enable ? 1 : 0);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_wait_limit_ns(unsigned long long ns) {
+    g_wait_limit.store(ns == 0 ? 2000000000ull : ns);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_fault_injection(int enable) {
+    g_inject.store(enable ? 1 : 0);
+    return QUAN_OK;
+}
+
+quan_status_t quan_device_status(quan_stream_t stream, unsigned int* bits) {
+    unsigned v = 0;
+    cudaError_t e = quan::read_and_clear_status(&v, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "device status");
+    if (bits) *bits = v;
+    if (v) return fail(QUAN_ERR_DEVICE_TIMEOUT, "kernel wait timed out (status bits 0x%x)", v);
+    return QUAN_OK;
+}
+
+const char* quan_status_string(quan_status_t status) {
+    switch (status) {
+        case QUAN_OK: return "QUAN_OK";
+        case QUAN_ERR_INVALID_ARG: return "QUAN_ERR_INVALID_ARG";
+        case QUAN_ERR_UNSUPPORTED: return "QUAN_ERR_UNSUPPORTED";
+        case QUAN_ERR_CUDA: return "QUAN_ERR_CUDA";
+        case QUAN_ERR_DEVICE_TIMEOUT: return "QUAN_ERR_DEVICE_TIMEOUT";
+    }
+    return "QUAN_ERR_UNKNOWN";
+}
+
+const char* quan_last_error_message(void) { return t_errmsg; }
+
+int quan_version(void) { return 100; }
+
+}  // extern "C"

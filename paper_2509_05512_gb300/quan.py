@@ -1,0 +1,218 @@
+"""ctypes binding of libquan (include/quan.h).  Argument marshalling only: every
+arithmetic step runs in the library's CUDA kernels.  Tensor arguments may be torch
+tensors (their device pointer is passed), integer device addresses, or None.
+
+The library must have been built (``paper_2509_05512_gb300.build.build_library()``);
+there is no fallback implementation, and a missing library raises immediately.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+
+PKG_DIR = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG_DIR, "libquan.so")
+HEADER = os.path.join(os.path.dirname(PKG_DIR), "include", "quan.h")
+
+QUAN_OK, QUAN_ERR_INVALID_ARG, QUAN_ERR_UNSUPPORTED, QUAN_ERR_CUDA, QUAN_ERR_DEVICE_TIMEOUT = range(5)
+QUAN_ACT_NONE, QUAN_ACT_RELU, QUAN_ACT_SILU = 0, 1, 2
+QUAN_PATH_AUTO, QUAN_PATH_TC, QUAN_PATH_SIMT = 0, 1, 2
+
+_lock = threading.Lock()
+_lib = None
+
+_vp = ctypes.c_void_p
+_i = ctypes.c_int
+_conv_args = [_vp] * 8 + [_i] * 10
+
+
+class QuanError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__("%s: %s" % (_status_name(status), message))
+        self.status = status
+
+
+def _status_name(st: int) -> str:
+    names = ["QUAN_OK", "QUAN_ERR_INVALID_ARG", "QUAN_ERR_UNSUPPORTED", "QUAN_ERR_CUDA",
+             "QUAN_ERR_DEVICE_TIMEOUT"]
+    return names[st] if 0 <= st < len(names) else "QUAN_ERR_%d" % st
+
+
+def header_functions() -> list:
+    """Names of the functions include/quan.h declares."""
+    with open(HEADER) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(quan_[a-z0-9_]+)\s*\(", text)))
+
+
+def load():
+    """Load libquan.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libquan.so is not built; run "
+                               "paper_2509_05512_gb300.build.build_library() first")
+        lib = ctypes.CDLL(LIB_PATH)
+        lib.quan_qconv2d_fwd.argtypes = _conv_args + [_vp, _vp]
+        lib.quan_qconv2d_fwd_f32.argtypes = _conv_args + [_vp, _vp]
+        lib.quan_qconv2d_fwd_res.argtypes = _conv_args + [_vp, _vp, _vp]
+        lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
+        lib.quan_set_path.argtypes = [_i]
+        lib.quan_last_path.argtypes = []
+        lib.quan_set_tc_tiles.argtypes = [_i, _i, _i]
+        lib.quan_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
+        lib.quan_set_tc_a_reuse.argtypes = [_i]
+        lib.quan_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_uint)]
+        lib.quan_set_fault_injection.argtypes = [_i]
+        lib.quan_status_string.argtypes = [_i]
+        lib.quan_status_string.restype = ctypes.c_char_p
+        lib.quan_last_error_message.argtypes = []
+        lib.quan_last_error_message.restype = ctypes.c_char_p
+        lib.quan_version.argtypes = []
+        for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
+                     "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
+                     "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
+                     "quan_set_tc_a_reuse"):
+            getattr(lib, name).restype = _i
+        lib.quan_last_path.restype = _i
+        lib.quan_version.restype = _i
+        _lib = lib
+        return lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(st: int):
+    if st != QUAN_OK:
+        msg = load().quan_last_error_message().decode(errors="replace")
+        raise QuanError(st, msg)
+
+
+def quan_qconv2d_fwd(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                     stride, pad, act, out, stream=None) -> None:
+    _check(load().quan_qconv2d_fwd(_ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), _ptr(bias),
+                                   _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W, Cin, Cout, kh, kw,
+                                   stride, pad, act, _ptr(out), _stream(stream)))
+
+
+def quan_qconv2d_fwd_f32(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                         kw, stride, pad, act, out, stream=None) -> None:
+    _check(load().quan_qconv2d_fwd_f32(_ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk),
+                                       _ptr(bias), _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W,
+                                       Cin, Cout, kh, kw, stride, pad, act, _ptr(out),
+                                       _stream(stream)))
+
+
+def quan_qconv2d_fwd_res(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                         kw, stride, pad, act, residual, out, stream=None) -> None:
+    _check(load().quan_qconv2d_fwd_res(_ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk),
+                                       _ptr(bias), _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W,
+                                       Cin, Cout, kh, kw, stride, pad, act, _ptr(residual),
+                                       _ptr(out), _stream(stream)))
+
+
+def quan_maxpool2d_fwd(x, N, H, W, C, k, stride, pad, out, stream=None) -> None:
+    _check(load().quan_maxpool2d_fwd(_ptr(x), N, H, W, C, k, stride, pad, _ptr(out),
+                                     _stream(stream)))
+
+
+def quan_set_path(path: int) -> None:
+    _check(load().quan_set_path(path))
+
+
+def quan_last_path() -> int:
+    return load().quan_last_path()
+
+
+def quan_set_tc_tiles(kappa: int = 0, bnq: int = 0, max_ctas: int = 0) -> None:
+    _check(load().quan_set_tc_tiles(kappa, bnq, max_ctas))
+
+
+def quan_set_tc_a_reuse(enable: bool) -> None:
+    _check(load().quan_set_tc_a_reuse(1 if enable else 0))
+
+
+def quan_set_wait_limit_ns(ns: int) -> None:
+    _check(load().quan_set_wait_limit_ns(ns))
+
+
+def quan_set_fault_injection(enable: bool) -> None:
+    _check(load().quan_set_fault_injection(1 if enable else 0))
+
+
+def quan_device_status(stream=None) -> tuple:
+    """Returns (status, bits); does not raise on QUAN_ERR_DEVICE_TIMEOUT."""
+    bits = ctypes.c_uint(0)
+    st = load().quan_device_status(_stream(stream), ctypes.byref(bits))
+    if st not in (QUAN_OK, QUAN_ERR_DEVICE_TIMEOUT):
+        _check(st)
+    return st, bits.value
+
+
+def quan_status_string(status: int) -> str:
+    return load().quan_status_string(status).decode()
+
+
+def quan_version() -> int:
+    return load().quan_version()
+
+
+# ------------------------------------------------------------------ tensor helpers
+
+def out_size(n: int, k: int, stride: int, pad: int) -> int:
+    return (n + 2 * pad - k) // stride + 1
+
+
+def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=None,
+            act=QUAN_ACT_NONE, residual=None, out=None, stream=None):
+    """Allocate the output (torch, same dtype/device as x) and run the convolution.
+    x: [N, H, W, Cin] (bf16 or fp32, CUDA); w*: [Cout/4, kh, kw, Cin/4]."""
+    import torch
+    N, H, W, Cin = x.shape
+    Qout, kh, kw, _ = wr.shape
+    Cout = 4 * Qout
+    Ho, Wo = out_size(H, kh, stride, pad), out_size(W, kw, stride, pad)
+    if out is None:
+        out = torch.empty((N, Ho, Wo, Cout), dtype=x.dtype, device=x.device)
+    if x.dtype == torch.float32:
+        if residual is not None:
+            raise ValueError("the fp32 entry point has no residual input")
+        quan_qconv2d_fwd_f32(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                             stride, pad, act, out, stream)
+    elif residual is not None:
+        quan_qconv2d_fwd_res(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                             stride, pad, act, residual, out, stream)
+    else:
+        quan_qconv2d_fwd(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                         stride, pad, act, out, stream)
+    return out
+
+
+def maxpool2d(x, *, k=3, stride=2, pad=1, out=None, stream=None):
+    import torch
+    N, H, W, C = x.shape
+    Ho, Wo = out_size(H, k, stride, pad), out_size(W, k, stride, pad)
+    if out is None:
+        out = torch.empty((N, Ho, Wo, C), dtype=x.dtype, device=x.device)
+    quan_maxpool2d_fwd(x, N, H, W, C, k, stride, pad, out, stream)
+    return out

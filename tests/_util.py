@@ -1,0 +1,70 @@
+"""Shared helpers for the tests: device upload of generated inputs and the
+tolerance checks stated for this method (fp64 oracle as the reference)."""
+import numpy as np
+
+from oracle import bf16_bits_to_f64
+
+# bf16 layers: relative L2 error <= 5e-3 and max-abs error <= 3e-2 * RMS(reference);
+# fp32 layers: max-abs error <= 1e-4 * RMS(reference).
+BF16_REL_L2 = 5e-3
+BF16_MAX_ABS_RMS = 3e-2
+F32_MAX_ABS_RMS = 1e-4
+
+
+def to_dev(a, dtype):
+    import torch
+    if a is None:
+        return None
+    if dtype == "bf16":
+        t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.cuda()
+
+
+def to_dev_f32(a):
+    import torch
+    if a is None:
+        return None
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).cuda()
+
+
+def host_f64(a, dtype):
+    """Inputs as the oracle reads them (bf16 bits -> exact float64)."""
+    if a is None:
+        return None
+    if dtype == "bf16":
+        return bf16_bits_to_f64(a)
+    return np.asarray(a, dtype=np.float64)
+
+
+def out_f64(t):
+    import torch
+    return t.detach().to(torch.float64).cpu().numpy()
+
+
+def errors(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    diff = got - ref
+    rms = float(np.sqrt(np.mean(ref * ref))) if ref.size else 0.0
+    rel_l2 = float(np.linalg.norm(diff) / max(np.linalg.norm(ref), 1e-300))
+    max_abs = float(np.abs(diff).max()) if diff.size else 0.0
+    return rel_l2, max_abs, rms
+
+
+def assert_bf16_close(got, ref, what=""):
+    rel_l2, max_abs, rms = errors(got, ref)
+    assert np.isfinite(got).all(), what + ": non-finite output"
+    assert rel_l2 <= BF16_REL_L2, "%s: rel-L2 %.3e > %.1e" % (what, rel_l2, BF16_REL_L2)
+    assert max_abs <= BF16_MAX_ABS_RMS * rms, "%s: max-abs %.3e > %.1e * RMS %.3e" % (
+        what, max_abs, BF16_MAX_ABS_RMS, rms)
+    return rel_l2, max_abs, rms
+
+
+def assert_f32_close(got, ref, what=""):
+    rel_l2, max_abs, rms = errors(got, ref)
+    assert np.isfinite(got).all(), what + ": non-finite output"
+    assert max_abs <= F32_MAX_ABS_RMS * rms, "%s: max-abs %.3e > %.1e * RMS %.3e" % (
+        what, max_abs, F32_MAX_ABS_RMS, rms)
+    return rel_l2, max_abs, rms

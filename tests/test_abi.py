@@ -1,0 +1,81 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds, loads and
+exports every function include/quan.h declares, and argument errors are rejected on
+the host before anything is launched."""
+import ctypes
+
+import pytest
+
+from paper_2509_05512_gb300 import build, quan
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build_library()
+    return quan.load()
+
+
+def test_exports_every_header_function(lib):
+    names = quan.header_functions()
+    assert "quan_qconv2d_fwd" in names and "quan_maxpool2d_fwd" in names
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_version(lib):
+    assert quan.quan_status_string(quan.QUAN_OK) == "QUAN_OK"
+    assert quan.quan_status_string(quan.QUAN_ERR_DEVICE_TIMEOUT) == "QUAN_ERR_DEVICE_TIMEOUT"
+    assert quan.quan_status_string(99) == "QUAN_ERR_UNKNOWN"
+    assert quan.quan_version() >= 100
+
+
+FAKE = 0x10000  # never dereferenced: every case below fails validation first
+
+
+def _call(lib, **kw):
+    a = dict(x=FAKE, wr=FAKE + 0x1000, wi=FAKE + 0x2000, wj=FAKE + 0x3000, wk=FAKE + 0x4000,
+             bias=None, scale=None, shift=None, N=1, H=8, W=8, Cin=64, Cout=64, kh=3, kw=3,
+             stride=1, pad=1, act=1, out=0x7000000, stream=None)
+    a.update(kw)
+    return lib.quan_qconv2d_fwd(a["x"], a["wr"], a["wi"], a["wj"], a["wk"], a["bias"], a["scale"],
+                                a["shift"], a["N"], a["H"], a["W"], a["Cin"], a["Cout"], a["kh"],
+                                a["kw"], a["stride"], a["pad"], a["act"], a["out"], a["stream"])
+
+
+@pytest.mark.parametrize("bad", [
+    dict(x=None), dict(wk=None), dict(out=None),
+    dict(Cin=6), dict(Cout=10), dict(N=0), dict(H=-1), dict(stride=0), dict(pad=-1),
+    dict(kh=0), dict(act=7), dict(kh=11, pad=1),
+    dict(scale=0x9000000),            # scale without shift
+    dict(shift=0x9000000),            # shift without scale
+    dict(out=FAKE),                   # out overlaps x
+])
+def test_invalid_arguments(lib, bad):
+    assert _call(lib, **bad) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_last_error_message()
+
+
+def test_maxpool_and_setters_validate(lib):
+    assert lib.quan_maxpool2d_fwd(None, 1, 4, 4, 8, 3, 2, 1, FAKE, None) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_maxpool2d_fwd(FAKE, 1, 4, 4, 8, 3, 2, 2, FAKE * 64, None) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_path(5) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_tiles(24, 0, 0) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_tiles(0, 0, 0) == quan.QUAN_OK
+    assert lib.quan_set_path(0) == quan.QUAN_OK
+    assert lib.quan_set_wait_limit_ns(0) == quan.QUAN_OK
+
+
+def test_f32_entry_point_validates(lib):
+    f = lib.quan_qconv2d_fwd_f32
+    assert f(None, FAKE, FAKE, FAKE, FAKE, None, None, None, 1, 4, 4, 4, 4, 3, 3, 1, 1, 0,
+             FAKE * 16, None) == quan.QUAN_ERR_INVALID_ARG
+    r = lib.quan_qconv2d_fwd_res
+    assert r(FAKE, FAKE, FAKE, FAKE, FAKE, None, None, None, 1, 4, 4, 4, 4, 3, 3, 1, 1, 0,
+             None, FAKE * 16, None) == quan.QUAN_ERR_INVALID_ARG
+
+
+def test_no_python_fallback_when_library_missing(monkeypatch, tmp_path):
+    # The binding must fail loudly, never compute elsewhere, if libquan.so is absent.
+    monkeypatch.setattr(quan, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(quan, "_lib", None)
+    with pytest.raises(RuntimeError, match="not built"):
+        quan.load()

@@ -1,0 +1,41 @@
+"""The seeded generators: bf16 rounding agrees with torch's round-to-nearest-even
+conversion, draws are deterministic, and a smaller batch is a prefix of the full one."""
+import numpy as np
+import torch
+
+from paper_2509_05512_gb300 import inputs
+
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(0)
+    a = np.concatenate([rng.standard_normal(100000).astype(np.float32),
+                        np.array([0.0, -0.0, 1.0, 1.00390625, 1.01171875, 3.0e38, -1e-38],
+                                 dtype=np.float32)])
+    ours = inputs.to_bf16_bits(a)
+    ref = torch.from_numpy(a).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(ours, ref)
+
+
+def test_layer_inputs_deterministic_and_prefix():
+    spec = inputs.small_layer("t", 4, 5, 6, 16, 32, 3, 1, 1, bias=True)
+    a = inputs.layer_inputs(spec)
+    b = inputs.layer_inputs(spec)
+    c = inputs.layer_inputs(spec, n_images=2)
+    for k in ("x", "wr", "wi", "wj", "wk", "bias", "scale", "shift"):
+        np.testing.assert_array_equal(a[k], b[k])
+    np.testing.assert_array_equal(a["x"][:2], c["x"])
+    np.testing.assert_array_equal(a["wk"], c["wk"])
+    assert a["x"].shape == (4, 5, 6, 16) and a["wr"].shape == (8, 3, 3, 4)
+
+
+def test_config_shapes_and_flops():
+    L = inputs.LAYERS
+    assert (L["c2b"].Ho, L["c2b"].Wo) == (28, 28)
+    assert abs(L["c1"].flops - 9.66e9) / 9.66e9 < 1e-3
+    assert abs(L["c3b"].flops - 483.2e9) / 483.2e9 < 1e-3
+    layers = inputs.backbone_layers()
+    convs = [l for l in layers if l.kind == "conv"]
+    assert len(convs) == 20
+    assert sum(l.kind == "maxpool" for l in layers) == 1
+    total = sum(l.spec.flops for l in convs)
+    assert 9.0e11 < total < 1.0e12

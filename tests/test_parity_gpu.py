@@ -1,0 +1,307 @@
+"""GPU parity: libquan (through the C ABI) against the fp64 oracle on identical seeded
+inputs.  Small layers are compared element by element over several tiles with a
+ragged tail; the full-size layers of the five configurations are compared on sampled
+output pixels (first/last pixels, tile boundaries, random picks) plus quaternion
+identities that hold at any size."""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+from paper_2509_05512_gb300 import build, inputs, quan
+from tests._util import (assert_bf16_close, assert_f32_close, host_f64, out_f64, to_dev,
+                         to_dev_f32)
+
+pytestmark = pytest.mark.gpu
+
+NEEDS_GPU = not torch.cuda.is_available()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if NEEDS_GPU:
+        pytest.skip("no CUDA device")
+    build.build_library()
+    lib = quan.load()
+    yield lib
+    quan.quan_set_path(quan.QUAN_PATH_AUTO)
+    quan.quan_set_tc_tiles(0, 0, 0)
+
+
+@pytest.fixture(autouse=True)
+def _reset_paths():
+    yield
+    quan.quan_set_path(quan.QUAN_PATH_AUTO)
+    quan.quan_set_tc_tiles(0, 0, 0)
+    quan.quan_set_fault_injection(False)
+    quan.quan_set_wait_limit_ns(0)
+    quan.quan_set_tc_a_reuse(False)
+
+
+def run_gpu(d, path=quan.QUAN_PATH_AUTO, guard=True):
+    """Upload a generated layer, run it through the C ABI, return float64 output."""
+    spec = d["spec"]
+    dt = spec.dtype
+    x = to_dev(d["x"], dt)
+    w = [to_dev(d[k], dt) for k in ("wr", "wi", "wj", "wk")]
+    bias, scale, shift = (to_dev_f32(d[k]) for k in ("bias", "scale", "shift"))
+    res = to_dev(d["residual"], dt) if d["residual"] is not None else None
+    tdt = torch.bfloat16 if dt == "bf16" else torch.float32
+    n_out = spec.N * spec.Ho * spec.Wo * spec.Cout
+    pad = 4096
+    buf = torch.full((n_out + 2 * pad,), float("nan"), dtype=tdt, device="cuda")
+    out = buf[pad:pad + n_out].view(spec.N, spec.Ho, spec.Wo, spec.Cout)
+    quan.quan_set_path(path)
+    quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=bias, scale=scale, shift=shift,
+                 act=spec.act, residual=res, out=out)
+    torch.cuda.synchronize()
+    if guard:  # guard bands on both sides of the output stay untouched
+        assert torch.isnan(buf[:pad].float()).all() and torch.isnan(buf[pad + n_out:].float()).all()
+    st, bits = quan.quan_device_status()
+    assert st == quan.QUAN_OK, bits
+    return out_f64(out), quan.quan_last_path()
+
+
+def oracle_full(d):
+    spec = d["spec"]
+    dt = spec.dtype
+    return oracle.qconv2d(host_f64(d["x"], dt), *(host_f64(d[k], dt) for k in ("wr", "wi", "wj", "wk")),
+                          stride=spec.stride, pad=spec.pad, bias=d["bias"], scale=d["scale"],
+                          shift=d["shift"], residual=host_f64(d["residual"], dt), act=spec.act)
+
+
+def check(spec, path=quan.QUAN_PATH_AUTO, expect_path=None, **kw):
+    d = inputs.layer_inputs(spec)
+    got, used = run_gpu(d, path)
+    if expect_path is not None:
+        assert used == expect_path
+    ref = oracle_full(d)
+    if spec.dtype == "bf16":
+        return assert_bf16_close(got, ref, spec.name)
+    return assert_f32_close(got, ref, spec.name)
+
+
+# ------------------------------------------------------------------ configs 0 and 1 in full
+
+def test_config0_fp32_full():
+    check(inputs.LAYERS["c0"], expect_path=quan.QUAN_PATH_SIMT)
+
+
+@pytest.mark.parametrize("path", [quan.QUAN_PATH_TC, quan.QUAN_PATH_SIMT])
+def test_config1_full(path):
+    check(inputs.LAYERS["c1"], path=path, expect_path=path)
+
+
+# ------------------------------------------------------------------ tensor-core small layers
+
+SMALL_TC = [
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra
+    ("ragged", 3, 13, 11, 64, 64, 3, 1, 1, {}),
+    ("stride2", 2, 15, 17, 64, 128, 3, 2, 1, {}),
+    ("pointwise", 2, 12, 10, 128, 256, 1, 1, 0, {}),
+    ("pointwise_s2", 2, 14, 14, 64, 128, 1, 2, 0, {"act": quan.QUAN_ACT_NONE}),
+    ("tiny_image", 1, 1, 1, 64, 64, 3, 1, 1, {}),
+    ("stem_like_7x7", 1, 20, 18, 64, 64, 7, 2, 3, {}),
+    ("wide_q", 1, 9, 9, 256, 256, 3, 1, 1, {}),
+    ("qin48", 2, 7, 9, 192, 64, 3, 1, 1, {}),
+    ("bias_silu", 2, 9, 8, 64, 128, 3, 1, 1, {"bias": True, "act": quan.QUAN_ACT_SILU}),
+    ("no_iqbn", 2, 9, 8, 64, 64, 3, 1, 1, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
+    ("residual", 2, 10, 9, 128, 128, 3, 1, 1, {"residual": True}),
+    ("pad2_5x5", 1, 11, 12, 64, 64, 5, 1, 2, {}),
+]
+
+
+@pytest.mark.parametrize("case", SMALL_TC, ids=[c[0] for c in SMALL_TC])
+def test_tc_small_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(200, len(name)), **extra)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+@pytest.mark.parametrize("a_reuse", [1, 0])
+@pytest.mark.parametrize("kappa,bnq", [(16, 16), (16, 64), (32, 32), (64, 16), (64, 64),
+                                       (32, 64)])
+def test_tc_tile_variants(kappa, bnq, a_reuse):
+    spec = inputs.small_layer("tiles", 2, 11, 13, 256, 256, 3, 1, 1, seed=(201, kappa + bnq))
+    quan.quan_set_tc_tiles(kappa, bnq, 0)
+    quan.quan_set_tc_a_reuse(bool(a_reuse))
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+def test_tc_few_ctas_many_tiles():
+    # a small persistent grid walks many tiles per CTA (accumulator double buffering,
+    # ring wrap-around many times)
+    spec = inputs.small_layer("few_ctas", 4, 16, 16, 64, 128, 3, 1, 1, seed=(202, 0))
+    quan.quan_set_tc_tiles(0, 16, 3)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+def test_tc_nonsquare_kernel():
+    spec = inputs.small_layer("k3x1", 2, 9, 10, 64, 64, 3, 1, 1, kw=1, seed=(203, 0))
+    # pad 1 on both sides with kw = 1 widens the output; valid for the oracle too
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+# ------------------------------------------------------------------ CUDA-core path
+
+SMALL_SIMT = [
+    ("q3", 2, 7, 6, 12, 8, 3, 1, 1, {}),
+    ("stem", 2, 23, 21, 4, 64, 7, 2, 3, {}),
+    ("q1_to_q1", 1, 5, 5, 4, 4, 3, 1, 1, {"act": quan.QUAN_ACT_SILU, "bias": True}),
+    ("residual", 1, 6, 6, 8, 8, 3, 1, 1, {"residual": True}),
+]
+
+
+@pytest.mark.parametrize("case", SMALL_SIMT, ids=[c[0] for c in SMALL_SIMT])
+def test_simt_small_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(300, len(name)), **extra)
+    check(spec, expect_path=quan.QUAN_PATH_SIMT)
+
+
+def test_simt_fp32_shapes():
+    spec = inputs.small_layer("f32", 2, 9, 7, 8, 12, 3, 2, 1, dtype="f32", bias=True,
+                              act=quan.QUAN_ACT_RELU, seed=(301, 0))
+    check(spec, expect_path=quan.QUAN_PATH_SIMT)
+
+
+def test_misaligned_pointer_demotes_to_simt():
+    spec = inputs.small_layer("mis", 1, 6, 6, 64, 64, 3, 1, 1, seed=(302, 0))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    xs = torch.empty(x.numel() + 8, dtype=torch.bfloat16, device="cuda")
+    xs[1:1 + x.numel()] = x.flatten()
+    xm = xs[1:1 + x.numel()].view_as(x)          # 2-byte aligned only
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
+    with pytest.raises(quan.QuanError) as ei:
+        quan.quan_set_path(quan.QUAN_PATH_TC)
+        quan.qconv2d(xm, *w, stride=1, pad=1, scale=sc, shift=sh, act=spec.act)
+    assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+    quan.quan_set_path(quan.QUAN_PATH_AUTO)
+    y = quan.qconv2d(xm, *w, stride=1, pad=1, scale=sc, shift=sh, act=spec.act)
+    torch.cuda.synchronize()
+    assert quan.quan_last_path() == quan.QUAN_PATH_SIMT
+    assert_bf16_close(out_f64(y), oracle_full(d), "misaligned")
+
+
+# ------------------------------------------------------------------ full-size layers, sampled
+
+def sample_points(spec, n_random, seed):
+    rng = np.random.default_rng(seed)
+    M = spec.N * spec.Ho * spec.Wo
+    idx = set([0, 1, M - 1, M - 2, 127, 128, 129, (M // 128) * 128 - 1])
+    idx.update(int(i) for i in rng.integers(0, M, n_random))
+    idx = sorted(i for i in idx if 0 <= i < M)
+    hw = spec.Ho * spec.Wo
+    return [(i // hw, (i % hw) // spec.Wo, i % spec.Wo) for i in idx]
+
+
+@pytest.mark.parametrize("name", ["c1", "c2a", "c2b", "c3a", "c3b"])
+def test_full_size_layer_sampled(name):
+    spec = inputs.LAYERS[name]
+    d = inputs.layer_inputs(spec)
+    got, used = run_gpu(d, guard=True)
+    assert used == quan.QUAN_PATH_TC
+    pts = sample_points(spec, 384, 7)
+    images = sorted(set(p[0] for p in pts))
+    remap = {n: i for i, n in enumerate(images)}
+    xs = host_f64(d["x"][images], "bf16")
+    w = [host_f64(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    ref = oracle.qconv2d_points(xs, *w, [(remap[n], h, ww) for n, h, ww in pts],
+                                stride=spec.stride, pad=spec.pad, bias=d["bias"],
+                                scale=d["scale"], shift=d["shift"], act=spec.act)
+    g = np.stack([got[n, h, ww] for n, h, ww in pts])
+    assert_bf16_close(g, ref, name)
+    # whole-output sanity: finite, ReLU non-negative, not all zero
+    assert np.isfinite(got).all() and (got >= 0).all() and (got > 0).mean() > 0.2
+
+
+def _left_mul_unit(wl, unit):
+    """Letters of u (x) W for a basis unit u (exact in bf16: a signed permutation)."""
+    wr, wi, wj, wk = wl
+    if unit == "i":
+        return [-wi, wr, -wk, wj]
+    if unit == "j":
+        return [-wj, wk, wr, -wi]
+    return [-wk, -wj, wi, wr]
+
+
+def _left_mul_out(y, unit, Q):
+    r, i, j, k = (y[..., m * Q:(m + 1) * Q] for m in range(4))
+    if unit == "i":
+        parts = [-i, r, -k, j]
+    elif unit == "j":
+        parts = [-j, k, r, -i]
+    else:
+        parts = [-k, -j, i, r]
+    return np.concatenate(parts, axis=-1)
+
+
+@pytest.mark.parametrize("name,unit", [("c2a", "i"), ("c3a", "j"), ("c2b", "k")])
+def test_full_size_left_multiplication_identity(name, unit):
+    # u (x) (W (x) X) = (u (x) W) (x) X for a constant quaternion u (associativity of
+    # Eq. 3, lifted to the convolution by linearity); with u a basis unit both sides
+    # are exact signed permutations, so the check covers the whole output.
+    # The signed permutations used here: i (x) (a + bi + cj + dk) = -b + ai - dj + ck, etc.
+    spec = inputs.LAYERS[name]
+    d = inputs.layer_inputs(spec)
+    dd = dict(d)
+    dd["scale"] = dd["shift"] = None
+    base_spec = dataclasses.replace(spec, iqbn=False, act=quan.QUAN_ACT_NONE)
+    dd["spec"] = base_spec
+    y, _ = run_gpu(dd)
+    wl = [d[k] for k in ("wr", "wi", "wj", "wk")]
+    # negate bf16 by flipping the sign bit (exact)
+    neg = lambda b: (b ^ np.uint16(0x8000)).astype(np.uint16)
+    mapping = {"i": [("wi", 1), ("wr", 0), ("wk", 1), ("wj", 0)],
+               "j": [("wj", 1), ("wk", 0), ("wr", 0), ("wi", 1)],
+               "k": [("wk", 1), ("wj", 1), ("wi", 0), ("wr", 0)]}[unit]
+    d2 = dict(dd)
+    for L, (src, negate) in zip(("wr", "wi", "wj", "wk"), mapping):
+        d2[L] = neg(d[src]) if negate else d[src]
+    y2, _ = run_gpu(d2)
+    lhs = _left_mul_out(y, unit, spec.Cout // 4)
+    rel = np.linalg.norm(y2 - lhs) / np.linalg.norm(lhs)
+    assert rel < 1e-3, rel
+
+
+# ------------------------------------------------------------------ pooling
+
+@pytest.mark.parametrize("shape", [(2, 9, 8, 64, 3, 2, 1), (1, 7, 7, 12, 3, 2, 1),
+                                   (2, 112, 112, 64, 3, 2, 1)])
+def test_maxpool(shape):
+    N, H, W, C, k, s, p = shape
+    rng = np.random.default_rng(sum(shape))
+    bits = inputs.to_bf16_bits(rng.standard_normal((N, H, W, C)).astype(np.float32))
+    x = to_dev(bits, "bf16")
+    y = quan.maxpool2d(x, k=k, stride=s, pad=p)
+    torch.cuda.synchronize()
+    ref = oracle.maxpool2d(host_f64(bits, "bf16"), k=k, stride=s, pad=p)
+    np.testing.assert_array_equal(out_f64(y), ref)
+
+
+# ------------------------------------------------------------------ failure detection
+
+def test_bounded_wait_timeout_reports_status_and_context_survives():
+    spec = inputs.small_layer("inject", 1, 16, 16, 64, 64, 3, 1, 1, seed=(400, 0))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
+    quan.quan_set_path(quan.QUAN_PATH_TC)
+    quan.quan_set_wait_limit_ns(5_000_000)          # 5 ms
+    quan.quan_set_fault_injection(True)
+    quan.qconv2d(x, *w, stride=1, pad=1, scale=sc, shift=sh, act=spec.act)
+    st, bits = quan.quan_device_status()
+    assert st == quan.QUAN_ERR_DEVICE_TIMEOUT and bits != 0
+    quan.quan_set_fault_injection(False)
+    quan.quan_set_wait_limit_ns(0)
+    st, bits = quan.quan_device_status()            # cleared
+    assert st == quan.QUAN_OK
+    y = quan.qconv2d(x, *w, stride=1, pad=1, scale=sc, shift=sh, act=spec.act)
+    torch.cuda.synchronize()
+    assert_bf16_close(out_f64(y), oracle_full(d), "after-timeout")
