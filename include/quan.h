@@ -118,18 +118,14 @@ int quan_last_path(void);
 /*
  * Tensor-core tile override for later calls (0 = automatic): kappa = quaternion input
  * channels per K block (16, 32 or 64), bnq = quaternion output channels per tile
- * (16, 32 or 64), max_ctas = persistent grid size cap.  Values that do not divide the
- * layer make the call fail with QUAN_ERR_UNSUPPORTED.
+ * (16, 32 or 64), max_ctas = persistent grid size cap, mode = MMA decomposition
+ * (1: one MMA per output/input component pair, N = bnq; 2: output components paired,
+ * N = 2 bnq; 3: weight-stationary, the whole signed block weight expanded once per CTA
+ * in shared memory, only for Cin = Cout = 64 and at most 9 taps).  Values that do not
+ * divide the layer, or a tile that does not fit in shared memory, make the call fail
+ * with QUAN_ERR_UNSUPPORTED.
  */
-quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas);
-
-/*
- * Tensor-core operand reuse (default 0): each input-component tile feeds four
- * consecutive MMAs (one per output component); with reuse on, the MMA unit keeps it in
- * its A-operand collector instead of reading shared memory four times.  0 turns the
- * reuse off (same results, more shared-memory traffic).
- */
-quan_status_t quan_set_tc_a_reuse(int enable);
+quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode);
 
 /* Time limit of every bounded wait inside the tensor-core kernel, in nanoseconds
  * (default 2e9).  0 restores the default. */

@@ -34,9 +34,9 @@ struct TcOptions {
     int kappa;                    // quaternion input channels per K block (16, 32 or 64); 0 = auto
     int bnq;                      // quaternion output channels per tile (16, 32 or 64); 0 = auto
     int max_ctas;                 // persistent grid cap; 0 = number of SMs
+    int mode;                     // 0 auto, 1 one MMA per (q, p), 2 paired output components
     unsigned long long wait_limit_ns;
     int inject_stall;             // failure-injection: the MMA role never consumes
-    int a_reuse;                  // reuse each X_p tile from the MMA A collector
 };
 
 // Tensor-core path (tcgen05 + TMA), bf16 in/out, fp32 accumulation.

@@ -16,10 +16,9 @@ namespace {
 thread_local char t_errmsg[512] = "";
 thread_local int t_last_path = 0;
 std::atomic<int> g_path{QUAN_PATH_AUTO};
-std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0};
+std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0};
 std::atomic<unsigned long long> g_wait_limit{2000000000ull};
 std::atomic<int> g_inject{0};
-std::atomic<int> g_a_reuse{0};
 
 constexpr int kMaxDevices = 64;
 int g_num_sms[kMaxDevices] = {0};
@@ -155,9 +154,9 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         opt.kappa = g_kappa.load();
         opt.bnq = g_bnq.load();
         opt.max_ctas = g_max_ctas.load();
+        opt.mode = g_mode.load();
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
-        opt.a_reuse = g_a_reuse.load();
         char err[256] = "";
         e = quan::launch_qconv_tc(s, x, w, ep, out, opt, num_sms, cs, err, sizeof(err));
         if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
@@ -245,18 +244,15 @@ quan_status_t quan_set_path(int path) {
 
 int quan_last_path(void) { return t_last_path; }
 
-quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas) {
+quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };
-    if (!okv(kappa) || !okv(bnq) || max_ctas < 0)
-        return fail(QUAN_ERR_INVALID_ARG, "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0");
+    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 3)
+        return fail(QUAN_ERR_INVALID_ARG,
+                    "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 3");
     g_kappa.store(kappa);
     g_bnq.store(bnq);
     g_max_ctas.store(max_ctas);
-    return QUAN_OK;
-}
-
-quan_status_t quan_set_tc_a_reuse(int enable) {
-    g_a_reuse.store(enable ? 1 : 0);
+    g_mode.store(mode);
     return QUAN_OK;
 }
 

@@ -64,9 +64,8 @@ def load():
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
         lib.quan_set_path.argtypes = [_i]
         lib.quan_last_path.argtypes = []
-        lib.quan_set_tc_tiles.argtypes = [_i, _i, _i]
+        lib.quan_set_tc_tiles.argtypes = [_i, _i, _i, _i]
         lib.quan_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
-        lib.quan_set_tc_a_reuse.argtypes = [_i]
         lib.quan_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_uint)]
         lib.quan_set_fault_injection.argtypes = [_i]
         lib.quan_status_string.argtypes = [_i]
@@ -76,8 +75,7 @@ def load():
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
-                     "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
-                     "quan_set_tc_a_reuse"):
+                     "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection"):
             getattr(lib, name).restype = _i
         lib.quan_last_path.restype = _i
         lib.quan_version.restype = _i
@@ -144,12 +142,8 @@ def quan_last_path() -> int:
     return load().quan_last_path()
 
 
-def quan_set_tc_tiles(kappa: int = 0, bnq: int = 0, max_ctas: int = 0) -> None:
-    _check(load().quan_set_tc_tiles(kappa, bnq, max_ctas))
-
-
-def quan_set_tc_a_reuse(enable: bool) -> None:
-    _check(load().quan_set_tc_a_reuse(1 if enable else 0))
+def quan_set_tc_tiles(kappa: int = 0, bnq: int = 0, max_ctas: int = 0, mode: int = 0) -> None:
+    _check(load().quan_set_tc_tiles(kappa, bnq, max_ctas, mode))
 
 
 def quan_set_wait_limit_ns(ns: int) -> None:

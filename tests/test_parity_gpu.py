@@ -28,17 +28,16 @@ def lib():
     lib = quan.load()
     yield lib
     quan.quan_set_path(quan.QUAN_PATH_AUTO)
-    quan.quan_set_tc_tiles(0, 0, 0)
+    quan.quan_set_tc_tiles(0, 0, 0, 0)
 
 
 @pytest.fixture(autouse=True)
 def _reset_paths():
     yield
     quan.quan_set_path(quan.QUAN_PATH_AUTO)
-    quan.quan_set_tc_tiles(0, 0, 0)
+    quan.quan_set_tc_tiles(0, 0, 0, 0)
     quan.quan_set_fault_injection(False)
     quan.quan_set_wait_limit_ns(0)
-    quan.quan_set_tc_a_reuse(False)
 
 
 def run_gpu(d, path=quan.QUAN_PATH_AUTO, guard=True):
@@ -95,6 +94,28 @@ def test_config1_full(path):
     check(inputs.LAYERS["c1"], path=path, expect_path=path)
 
 
+@pytest.mark.parametrize("mode", [1, 2, 3])
+def test_config1_full_every_mode(mode):
+    quan.quan_set_tc_tiles(0, 0, 0, mode)
+    check(inputs.LAYERS["c1"], path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+WS_CASES = [
+    ("ws_ragged", 3, 13, 11, 64, 64, 3, 1, 1, {}),
+    ("ws_stride2", 2, 15, 17, 64, 64, 3, 2, 1, {"residual": True}),
+    ("ws_1x1", 2, 9, 7, 64, 64, 1, 1, 0, {"bias": True, "act": quan.QUAN_ACT_SILU}),
+    ("ws_5x1", 1, 9, 8, 64, 64, 5, 1, 2, {"kw": 1}),
+]
+
+
+@pytest.mark.parametrize("case", WS_CASES, ids=[c[0] for c in WS_CASES])
+def test_tc_weight_stationary_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(205, len(name)), **extra)
+    quan.quan_set_tc_tiles(0, 0, 0, 3)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
 # ------------------------------------------------------------------ tensor-core small layers
 
 SMALL_TC = [
@@ -121,13 +142,24 @@ def test_tc_small_layers(case):
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
-@pytest.mark.parametrize("a_reuse", [1, 0])
-@pytest.mark.parametrize("kappa,bnq", [(16, 16), (16, 64), (32, 32), (64, 16), (64, 64),
-                                       (32, 64)])
-def test_tc_tile_variants(kappa, bnq, a_reuse):
+# every (kappa, bnq, mode) whose stages fit in shared memory (64 x 64 does not)
+TILE_CASES = [(k, b, m) for m in (1, 2) for k in (16, 32, 64) for b in (16, 32, 64)
+              if not (k == 64 and b == 64)]
+
+
+@pytest.mark.parametrize("kappa,bnq,mode", TILE_CASES)
+def test_tc_tile_variants(kappa, bnq, mode):
     spec = inputs.small_layer("tiles", 2, 11, 13, 256, 256, 3, 1, 1, seed=(201, kappa + bnq))
-    quan.quan_set_tc_tiles(kappa, bnq, 0)
-    quan.quan_set_tc_a_reuse(bool(a_reuse))
+    quan.quan_set_tc_tiles(kappa, bnq, 0, mode)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+@pytest.mark.parametrize("mode", [1, 2])
+def test_tc_pair_mode_layers(mode):
+    # stride-2, ragged tail, residual and both modes on the same layer
+    spec = inputs.small_layer("pairs", 3, 15, 13, 128, 256, 3, 2, 1, residual=True,
+                              seed=(204, mode))
+    quan.quan_set_tc_tiles(0, 0, 0, mode)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
@@ -135,7 +167,7 @@ def test_tc_few_ctas_many_tiles():
     # a small persistent grid walks many tiles per CTA (accumulator double buffering,
     # ring wrap-around many times)
     spec = inputs.small_layer("few_ctas", 4, 16, 16, 64, 128, 3, 1, 1, seed=(202, 0))
-    quan.quan_set_tc_tiles(0, 16, 3)
+    quan.quan_set_tc_tiles(0, 16, 3, 0)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
