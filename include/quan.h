@@ -127,6 +127,15 @@ int quan_last_path(void);
  */
 quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode);
 
+/*
+ * Weight-stationary pixel staging (default 1): for stride-1 layers whose output keeps the
+ * input size and whose width is a multiple of 8 (at most 128), a tile is a block of whole
+ * output rows and one TMA box per horizontal filter offset holds those rows plus their
+ * vertical halo, shared by the vertical filter offsets.  0 stages one im2col box per
+ * filter tap instead (same results).
+ */
+quan_status_t quan_set_tc_halo(int enable);
+
 /* Time limit of every bounded wait inside the tensor-core kernel, in nanoseconds
  * (default 2e9).  0 restores the default. */
 quan_status_t quan_set_wait_limit_ns(unsigned long long ns);

@@ -34,7 +34,10 @@ struct TcOptions {
     int kappa;                    // quaternion input channels per K block (16, 32 or 64); 0 = auto
     int bnq;                      // quaternion output channels per tile (16, 32 or 64); 0 = auto
     int max_ctas;                 // persistent grid cap; 0 = number of SMs
-    int mode;                     // 0 auto, 1 one MMA per (q, p), 2 paired output components
+    int mode;                     // 0 auto, 1 one MMA per (q, p), 2 paired output components,
+                                  // 3 weight-stationary
+    int ws_halo;                  // weight-stationary: stage row blocks with halos (1) when
+                                  // the shape allows it, else one im2col box per tap (0)
     unsigned long long wait_limit_ns;
     int inject_stall;             // failure-injection: the MMA role never consumes
 };

@@ -200,6 +200,43 @@ __device__ __forceinline__ void tma_store_2d(const void* map, uint32_t src, int 
         : "memory");
 }
 
+__device__ __forceinline__ void tma_store_3d(const void* map, uint32_t src, int x, int y, int z) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(x), "r"(y), "r"(z), "r"(src)
+        : "memory");
+}
+
+// 4-D tiled load (coordinates may be negative or past the end: the box is zero-filled).
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const void* map, uint32_t bar, int c,
+                                            int w, int h, int n, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        ".L2::cache_hint [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c), "r"(w), "r"(h), "r"(n), "r"(bar),
+        "l"(policy)
+        : "memory");
+}
+
+// Prefetch a tiled box (4-D) or an im2col box into L2 only (no shared memory).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const void* map, int c, int w, int h, int n) {
+    asm volatile(
+        "cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(c), "r"(w), "r"(h), "r"(n)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch_l2_im2col_4d(const void* map, int c, int w, int h,
+                                                          int n, uint16_t off_w, uint16_t off_h) {
+    asm volatile(
+        "cp.async.bulk.prefetch.tensor.4d.L2.global.im2col [%0, {%1, %2, %3, %4}], {%5, %6};" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(c), "r"(w), "r"(h), "r"(n), "h"(off_w), "h"(off_h)
+        : "memory");
+}
+
 __device__ __forceinline__ void bulk_commit_group() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }

@@ -4,47 +4,37 @@
 //   Y[pixel][q, co] = sum_{tap, p, ci} X[pixel + tap][p, ci] * B[tap][p, ci][q, co]
 // whose weight B is the signed 4x4 block (Hamilton) matrix of Eq. 6 built from four
 // compact letter tensors W_r, W_i, W_j, W_k.  The block weight is never written to
-// global memory: each K block stages the four input-component tiles X_p and the
-// compact letter tiles, and the signed block structure is produced by choosing, per
-// MMA, which letter tile the B descriptor points at and the instruction's negate bit.
-// Weight traffic is therefore 1/4 of the real-equivalent layer.
+// global memory: the signed block structure is produced on chip, so weight traffic
+// is 1/4 of the real-equivalent layer.  Three MMA decompositions:
 //
-// Two MMA decompositions (template MODE):
 //   MODE_QUAD  16 MMAs per 16-wide K step, one per (output q, input p):
 //                D_q += sign(q, p) * X_p * W_{q xor p}^T            (N = BNQ)
+//              the letter is chosen by the B descriptor and the sign by the
+//              instruction descriptor's negate bit.
 //   MODE_PAIR  8 MMAs per K step, each covering two output components:
 //                [D_r | D_i] and [D_j | D_k] += +-X_p * S^T         (N = 2 BNQ)
 //              where S is a stack of two letter blocks.  The four stacks Eq. 6 needs,
 //              [W_r; W_i], [-W_i; W_r], [W_j; W_k], [W_k; -W_j] (up to an overall sign),
 //              are all windows of the two 3-block sequences
 //                [-W_i | W_r | W_i]  and  [W_j | W_k | -W_j],
-//              so a stage holds 6 letter blocks (W_i and W_j are loaded twice) and a
-//              helper warp flips the sign bits of the two negated copies.  The larger N
-//              keeps the tensor pipe busy (an M=128 MMA costs at least ~45 cycles on
-//              this part, a full N=64 one is 32 cycles of work, N=128 is 64).
+//              so a stage holds 6 letter blocks; TMA loads the 4 letters and a helper
+//              warp writes the two negated copies.  The larger N keeps the tensor pipe
+//              busy (an M=128 MMA costs at least ~45 cycles on this part, a full N=64 one
+//              is 32 cycles of work, N=128 is 64).
+//   MODE_WS    (16 -> 16 quaternion channels, at most 9 taps; qconv_ws.cuh)
+//              weight-stationary: every CTA expands the whole signed block weight once
+//              into shared memory and streams only pixels; N = 64 MMAs cover all four
+//              output components.
 //
-//   MODE_WS    (16 -> 16 quaternion channels, at most 9 taps) weight-stationary: every CTA
-//              expands the whole signed block weight of Eq. 6 into shared memory once
-//              (read from the compact letters, 72 KB for 3x3), then streams one im2col
-//              box per tap that holds all four input components (64 channels, 128-byte
-//              rows); 4 MMAs of N = 64 per tap cover all four output components.
-//
-// Structure (one persistent CTA per SM, 12 warps):
+// Structure of the QUAD/PAIR kernel (one persistent CTA per SM, 12 warps):
 //   warps 0, 3  TMA producers: per K block (tap, chunk of KAPPA quaternion input channels)
 //               warp 0 issues the 4 im2col loads of X (zero padding comes from
 //               out-of-bounds fill) and warp 3 the letter tiles, into a STAGES-deep ring
-//               (a single thread issues TMA copies at a limited rate);
+//               (one thread issues TMA copies at a limited rate);
 //   warp 1      owns TMEM (2 accumulator buffers x 4 components x BNQ columns); one lane
 //               issues the tcgen05.mma / tcgen05.commit stream;
-//   warp 2      MODE_PAIR only: writes the two sign-flipped letter copies of each stage;
-//   warps 4..11 epilogue, two warps per TMEM lane quadrant, each half of them owning two
-//               output components: tcgen05.ld TMEM -> registers,
-//               act(scale*(acc+bias)+shift+res) (IQBN inference form of Eq. 11-12) with
-//               the per-channel vectors staged in shared memory, bf16 round-to-nearest
-//               into a swizzled shared-memory tile, TMA store into the component-major
-//               NHWC output (rows past the last pixel are clipped by the tensor map).
-//               Double-buffered accumulators let the epilogue of tile i overlap the
-//               main loop of tile i+1.
+//   warp 2      MODE_PAIR: writes the two sign-flipped letter copies of each stage;
+//   warps 4..11 epilogue (tc_common.cuh), overlapping the next tile's main loop.
 // Every mbarrier wait is bounded in time; a wait that runs out sets a bit in the device
 // status word, raises a CTA-wide abort flag, drains the copies and MMAs still in flight,
 // frees TMEM and returns.
@@ -58,137 +48,59 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "tc_common.cuh"
 
 namespace quan {
-
-__device__ unsigned int g_status;
-
 namespace {
 
-constexpr int BM = 128;           // output pixels per tile (MMA M)
-constexpr int NUM_THREADS = 384;  // 12 warps
+using namespace tc;
+
 constexpr int MODE_QUAD = 0;
 constexpr int MODE_PAIR = 1;
 constexpr int MODE_WS = 2;
 constexpr int WS_MAX_TAPS = 9;
-constexpr int EPI_WARP0 = 4;
-constexpr int UMMA_K = 16;        // K of one kind::f16 MMA
-
-// Output component q takes input component p through letter L = q xor p, read off Eq. 5:
-//   y_r: +W_r X_r  -W_i X_i  -W_j X_j  -W_k X_k
-//   y_i: +W_i X_r  +W_r X_i  -W_k X_j  +W_j X_k
-//   y_j: +W_j X_r  +W_k X_i  +W_r X_j  -W_i X_k
-//   y_k: +W_k X_r  -W_j X_i  +W_i X_j  +W_r X_k
-// Bit (4 q + p) of NEG_MASK marks the negative terms.
-constexpr uint32_t NEG_MASK = (1u << 1) | (1u << 2) | (1u << 3)  // y_r: X_i, X_j, X_k
-                              | (1u << 6)                        // y_i: X_j
-                              | (1u << 11)                       // y_j: X_k
-                              | (1u << 13);                      // y_k: X_i
+constexpr int MAX_STAGES = 8;
 
 struct TcParams {
     ConvShape s;
     EpilogueArgs ep;
-    __nv_bfloat16* out;
     int kchunks;      // Qin / KAPPA
     int ktiles;       // kh * kw * kchunks K blocks per tile
     int num_n_tiles;  // Qout / BNQ
     int num_tiles;
     unsigned long long wait_limit_ns;
     int inject_stall;
-    const __nv_bfloat16* w[4];  // compact letter tensors (read directly by MODE_WS)
 };
 
 template <int KAPPA, int BNQ, int MODE>
 struct Cfg {
-    // pixel-tile row: KAPPA channels of one component, or all four components (WS)
-    static constexpr int A_ROW_BYTES = (MODE == MODE_WS ? 4 * KAPPA : KAPPA) * 2;
-    static constexpr int A_TILE = BM * A_ROW_BYTES;
-    static constexpr int A_TILES = MODE == MODE_WS ? 1 : 4;
-    static constexpr int B_TILE = BNQ * KAPPA * 2;  // one letter block of the weight tile
-    static constexpr int B_SLOTS = MODE == MODE_PAIR ? 6 : (MODE == MODE_QUAD ? 4 : 0);
-    static constexpr int STAGE_BYTES = A_TILES * A_TILE + B_SLOTS * B_TILE;
-    // bytes the TMA copies per stage (pair mode writes two slots itself)
-    static constexpr int STAGE_TX = A_TILES * A_TILE + (B_SLOTS ? 4 : 0) * B_TILE;
-    // resident expanded weight (WS): per tap a [4 BNQ rows x 4 KAPPA] K-major tile
-    static constexpr int WSB_TAP = MODE == MODE_WS ? 4 * BNQ * 4 * KAPPA * 2 : 0;
-    static constexpr int WSB_BYTES = MODE == MODE_WS ? WS_MAX_TAPS * WSB_TAP : 0;
-    static constexpr int OUT_TILE = BM * BNQ * 2;        // one output component block, bf16
-    static constexpr int STAGING_BYTES = 2 * OUT_TILE;   // one block per epilogue half
-    static constexpr int PARAM_BYTES = 3 * 4 * BNQ * 4;  // bias, scale, shift of a tile
-    static constexpr int FIXED_BYTES = 1024 + WSB_BYTES + STAGING_BYTES + PARAM_BYTES + 512;
+    static constexpr int A_ROW_BYTES = KAPPA * 2;
+    static constexpr int A_TILE = BM * A_ROW_BYTES;  // one component of the pixel tile
+    static constexpr int B_TILE = BNQ * KAPPA * 2;   // one letter block of the weight tile
+    static constexpr int B_SLOTS = MODE == MODE_PAIR ? 6 : 4;
+    static constexpr int STAGE_BYTES = 4 * A_TILE + B_SLOTS * B_TILE;
+    static constexpr int TX_A = 4 * A_TILE;          // bytes TMA writes per stage: pixels
+    static constexpr int TX_W = 4 * B_TILE;          //                               letters
+    using E = EpiSmem<BNQ>;
+    static constexpr int FIXED_BYTES = 1024 + E::STAGING_BYTES + E::PARAM_BYTES + 512;
     static constexpr int STAGES_RAW = (227 * 1024 - FIXED_BYTES) / STAGE_BYTES;
-    static constexpr int STAGES = STAGES_RAW > 8 ? 8 : (STAGES_RAW < 2 ? 2 : STAGES_RAW);
+    static constexpr int STAGES =
+        STAGES_RAW > MAX_STAGES ? MAX_STAGES : (STAGES_RAW < 2 ? 2 : STAGES_RAW);
     static constexpr int TILES_BYTES = STAGES * STAGE_BYTES;
-    static constexpr int WSB_OFF = TILES_BYTES;
-    static constexpr int STAGING_OFF = WSB_OFF + WSB_BYTES;
-    static constexpr int PARAM_OFF = STAGING_OFF + STAGING_BYTES;
-    static constexpr int BAR_OFF = PARAM_OFF + PARAM_BYTES;
-    // output staging swizzle: rows of BNQ bf16 (128, 64 or 32 bytes)
-    static constexpr uint32_t OUT_ROW = BNQ * 2;
-    static constexpr uint32_t OUT_SW_MASK = BNQ == 64 ? 7u : (BNQ == 32 ? 3u : 1u);
+    static constexpr int STAGING_OFF = TILES_BYTES;
+    static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
+    static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
     // full (pixels), full (letters), empty, ready (negated copies done), acc_full[2],
-    // acc_empty[2], drain, expanded weight ready (WS)
-    static constexpr int NUM_BARS = 4 * STAGES + 6;
+    // acc_empty[2], drain
+    static constexpr int NUM_BARS = 4 * STAGES + 5;
     static constexpr int SMEM_BYTES = 1024 + BAR_OFF + NUM_BARS * 8 + 16;
     static constexpr bool FITS = SMEM_BYTES <= 227 * 1024;
     static constexpr uint32_t TMEM_COLS = 8 * BNQ;  // 2 buffers x 4 components x BNQ fp32 columns
     static constexpr int KSTEPS = KAPPA / UMMA_K;
-    static constexpr uint32_t SBO = 8 * A_ROW_BYTES;  // pitch of 8-row core-matrix groups
-    // smem descriptor layout type: 128B, 64B or 32B swizzle
-    static constexpr uint64_t LAYOUT = A_ROW_BYTES == 128 ? 2ull : (A_ROW_BYTES == 64 ? 4ull : 6ull);
-    // high 32 bits of every operand descriptor: SBO, descriptor version, swizzle mode
-    static constexpr uint32_t DESC_HI =
-        (SBO >> 4) | (1u << 14) | (static_cast<uint32_t>(LAYOUT) << 29);
+    static constexpr uint32_t DESC_HI = desc_hi(8 * A_ROW_BYTES, desc_layout(A_ROW_BYTES));
     static_assert(KAPPA == 16 || KAPPA == 32 || KAPPA == 64, "KAPPA");
     static_assert(BNQ == 16 || BNQ == 32 || BNQ == 64, "BNQ");
-    static_assert(MODE != MODE_WS || (KAPPA == 16 && BNQ == 16), "WS tile");
 };
-
-// tcgen05 shared-memory matrix descriptors (K-major, swizzled operand tiles) are built
-// as two 32-bit words: the low word holds the start address >> 4 (bits 0-13) and the
-// leading byte offset (bits 16-29, unused for these layouts, set to 1); the high word
-// holds the stride byte offset >> 4 (pitch of 8-row core-matrix groups), the
-// descriptor version (bit 46) and the swizzle mode (bits 61-63).
-// Low 32 bits of the descriptor: start address and the (unused) leading byte offset.
-__device__ __forceinline__ uint32_t desc_lo(uint32_t saddr) {
-    return ((saddr & 0x3FFFFu) >> 4) | (1u << 16);
-}
-
-// Instruction descriptor, kind::f16: bf16 A and B, fp32 D, both operands K-major.
-__host__ __device__ constexpr uint32_t make_idesc(int M, int N, int negate) {
-    return (1u << 4)                                   // D format: f32
-           | (1u << 7)                                 // A format: bf16
-           | (1u << 10)                                // B format: bf16
-           | (static_cast<uint32_t>(negate) << 13)     // negate A
-           | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
-           | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
-}
-
-__device__ __forceinline__ float activate(float z, int act) {
-    if (act == 1) return fmaxf(z, 0.0f);
-    if (act == 2) return z / (1.0f + __expf(-z));
-    return z;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uint64_t limit,
-                                              volatile int* abort_flag, unsigned code) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = global_timer_ns();
-    while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if (global_timer_ns() - t0 > limit) {
-            atomicOr(&g_status, code);
-            *abort_flag = 1;
-            return false;
-        }
-    }
-}
 
 template <int KAPPA, int BNQ, int MODE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
@@ -212,10 +124,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
     auto ready_bar = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
     auto fullw_bar = [&](int s) { return bar0 + 8u * (3 * STAGES + s); };
-    auto accf_bar = [&](int b) { return bar0 + 8u * (4 * STAGES + b); };
-    auto acce_bar = [&](int b) { return bar0 + 8u * (4 * STAGES + 2 + b); };
+    const uint32_t accf0 = bar0 + 8u * (4 * STAGES);
+    const uint32_t acce0 = bar0 + 8u * (4 * STAGES + 2);
     const uint32_t drain_bar = bar0 + 8u * (4 * STAGES + 4);
-    const uint32_t wsready_bar = bar0 + 8u * (4 * STAGES + 5);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
@@ -229,11 +140,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             mbar_init(ready_bar(i), 1);
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(accf_bar(b), 1);
-            mbar_init(acce_bar(b), 8 * 32);
+            mbar_init(accf0 + 8u * b, 1);
+            mbar_init(acce0 + 8u * b, 8 * 32);
         }
         mbar_init(drain_bar, 1);
-        mbar_init(wsready_bar, NUM_THREADS / 32 - 2);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -255,68 +165,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint32_t tmem_base = *tmem_slot;
     const int hw = s.Ho * s.Wo;
 
-    if constexpr (MODE == MODE_WS) {
-        if (warp >= 2) {
-            // Expand the signed block weight of Eq. 6 once (warps 2..11, while the producer
-            // already streams pixels): for tap t, row n = (q, co) and K index k = (p, ci)
-            // the value is sign(q, p) * W_{q xor p}[co][t][ci]; rows are 128 bytes (all four
-            // input components) in the 128-byte swizzled K-major layout.
-            constexpr int EXP_THREADS = NUM_THREADS - 64;
-            constexpr int MAX_CHUNKS = WS_MAX_TAPS * 4 * BNQ * 8;
-            constexpr int PER_THREAD = (MAX_CHUNKS + EXP_THREADS - 1) / EXP_THREADS;
-            const int taps = s.kh * s.kw;
-            const int chunks = taps * (4 * BNQ) * 8;  // 16-byte chunks
-            const int et = threadIdx.x - 64;
-            uint4 v[PER_THREAD];
-#pragma unroll
-            for (int k = 0; k < PER_THREAD; ++k) {
-                const int idx = et + k * EXP_THREADS;
-                if (idx < chunks) {
-                    const int ch = idx & 7;                // chunk of the row: p = ch / 2
-                    const int n = (idx >> 3) % (4 * BNQ);  // row: q = n / BNQ, co = n % BNQ
-                    const int t = (idx >> 3) / (4 * BNQ);  // tap
-                    const int q = n / BNQ, co = n % BNQ, pc = ch >> 1, ci0 = (ch & 1) * 8;
-                    v[k] = __ldg(reinterpret_cast<const uint4*>(
-                        p.w[q ^ pc] + (static_cast<size_t>(co) * taps + t) * KAPPA + ci0));
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < PER_THREAD; ++k) {
-                const int idx = et + k * EXP_THREADS;
-                if (idx < chunks) {
-                    const int ch = idx & 7;
-                    const int n = (idx >> 3) % (4 * BNQ);
-                    const int t = (idx >> 3) / (4 * BNQ);
-                    const int q = n / BNQ, pc = ch >> 1;
-                    uint4 u = v[k];
-                    if ((NEG_MASK >> (4 * q + pc)) & 1u) {
-                        u.x ^= 0x80008000u; u.y ^= 0x80008000u; u.z ^= 0x80008000u; u.w ^= 0x80008000u;
-                    }
-                    const uint32_t off = static_cast<uint32_t>(
-                        C::WSB_OFF + t * C::WSB_TAP + n * 128 + ((ch ^ (n & 7)) << 4));
-                    *reinterpret_cast<uint4*>(smem + off) = u;
-                }
-            }
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(wsready_bar);
-        }
-    }
-
     if (warp == 0 || warp == 3) {
         // ------------------------------------------------------------ TMA producers
-        // One thread can only issue TMA copies at a limited rate, so two warps share the
-        // work: warp 0 stages the pixel tiles and warp 3 the letter tiles of each K block
-        // (WS mode: the two alternate K blocks).
         if (lane == 0) {
-            const int role = warp == 0 ? 0 : 1;
+            const int role = warp == 0 ? 0 : 1;  // 0: pixels, 1: letters
             const uint64_t pol_x = l2_policy_evict_normal();
             const uint64_t pol_w = l2_policy_evict_last();
             int stage = 0;
             uint32_t phase = 0;
-            uint32_t filled = 0, fill_parity = 0;  // per-stage: ever filled, parity of last fill
+            uint32_t filled = 0, fill_parity = 0;  // per stage: ever filled, parity of last fill
             bool ok = true;
-            int kt_all = 0;
             for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
                 const int m_tile = tile / p.num_n_tiles;
                 const int n_tile = tile - m_tile * p.num_n_tiles;
@@ -328,35 +186,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 for (int kt = 0; kt < p.ktiles; ++kt) {
                     const int tap = kt / p.kchunks, chunk = kt - tap * p.kchunks;
                     const int dh = tap / s.kw, dw = tap - (tap / s.kw) * s.kw;
-                    if (MODE == MODE_WS && (kt_all++ & 1) != role) {
-                        if (++stage == STAGES) {
-                            stage = 0;
-                            phase ^= 1u;
-                        }
-                        continue;
-                    }
                     if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                        STATUS_TIMEOUT_PRODUCER)) {
                         ok = false;
                         break;
                     }
                     // pixels complete full_bar, letters complete fullw_bar
-                    const uint32_t fb = role == 0 || MODE == MODE_WS ? full_bar(stage)
-                                                                     : fullw_bar(stage);
-                    mbar_arrive_expect_tx(fb, MODE == MODE_WS ? C::STAGE_TX
-                                              : (role == 0 ? C::A_TILES * C::A_TILE
-                                                           : C::STAGE_TX - C::A_TILES * C::A_TILE));
+                    const uint32_t fb = role == 0 ? full_bar(stage) : fullw_bar(stage);
+                    mbar_arrive_expect_tx(fb, role == 0 ? C::TX_A : C::TX_W);
                     filled |= 1u << stage;
                     fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
                     const uint32_t a0 = sbase + stage * C::STAGE_BYTES;
-                    const uint32_t b0 = a0 + C::A_TILES * C::A_TILE;
+                    const uint32_t b0 = a0 + 4 * C::A_TILE;
                     const int cin0 = chunk * KAPPA;
-                    if constexpr (MODE == MODE_WS) {
-                        // all four components of the pixel (channels 0 .. 4 KAPPA) at once
-                        tma_load_im2col_4d(a0, &tmap_x, fb, 0, wbase, hbase, img,
-                                           static_cast<uint16_t>(dw), static_cast<uint16_t>(dh),
-                                           pol_x);
-                    } else if (role == 0) {
+                    if (role == 0) {
 #pragma unroll
                         for (int comp = 0; comp < 4; ++comp)
                             tma_load_im2col_4d(a0 + comp * C::A_TILE, &tmap_x, fb,
@@ -386,26 +229,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
             }
-            if (!ok) {
-                // Copies already issued complete on their own; wait for each stage's most
-                // recent fill so that no copy targets this CTA's memory after it exits.
-                for (int i = 0; i < STAGES; ++i) {
-                    if (!(filled & (1u << i))) continue;
-                    const uint32_t own = role == 0 || MODE == MODE_WS ? full_bar(i) : fullw_bar(i);
-                    const uint64_t t0 = global_timer_ns();
-                    while (!mbar_try_wait(own, (fill_parity >> i) & 1u)) {
-                        if (global_timer_ns() - t0 > limit) {
-                            atomicOr(&g_status, STATUS_TIMEOUT_DRAIN);
-                            break;
-                        }
-                    }
-                }
-            }
+            if (!ok)
+                drain_fills(role == 0 ? full_bar(0) : fullw_bar(0), STAGES, filled, fill_parity,
+                            limit);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
-            constexpr int NMMA = MODE == MODE_PAIR ? 2 * BNQ : (MODE == MODE_WS ? 4 * BNQ : BNQ);
+            constexpr int NMMA = MODE == MODE_PAIR ? 2 * BNQ : BNQ;
             constexpr uint32_t IDESC_POS = make_idesc(BM, NMMA, 0);
             constexpr uint32_t IDESC_NEG = make_idesc(BM, NMMA, 1);
             int stage = 0;
@@ -415,17 +246,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (p.inject_stall) {
                 // Failure injection: wait on a barrier nothing arrives on, so that every
                 // role runs into its bounded wait and the kernel reports a timeout.
-                ok = wait_or_abort(drain_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
+                wait_or_abort(drain_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
                 ok = false;
-            }
-            if constexpr (MODE == MODE_WS) {
-                if (ok) ok = wait_or_abort(wsready_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
             }
             int local = 0;
             for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
                 const int buf = local & 1;
                 const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
-                if (!wait_or_abort(acce_bar(buf), use ^ 1u, limit, abort_flag,
+                if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA)) {
                     ok = false;
                     break;
@@ -435,31 +263,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 for (int kt = 0; kt < p.ktiles; ++kt) {
                     // pixels, then the letter tiles (pair mode: with their negated copies)
                     if (!wait_or_abort(full_bar(stage), phase, limit, abort_flag,
-                                       STATUS_TIMEOUT_MMA)) {
+                                       STATUS_TIMEOUT_MMA) ||
+                        !wait_or_abort(MODE == MODE_PAIR ? ready_bar(stage) : fullw_bar(stage),
+                                       phase, limit, abort_flag, STATUS_TIMEOUT_MMA)) {
                         ok = false;
                         break;
-                    }
-                    if constexpr (MODE != MODE_WS) {
-                        const uint32_t wb = MODE == MODE_PAIR ? ready_bar(stage) : fullw_bar(stage);
-                        if (!wait_or_abort(wb, phase, limit, abort_flag, STATUS_TIMEOUT_MMA)) {
-                            ok = false;
-                            break;
-                        }
                     }
                     tc_fence_after();
                     // descriptor low words of this stage's first X_p and W_L tiles; every
                     // sub-MMA below only adds a compile-time offset to them
                     const uint32_t a_lo0 = desc_lo(sbase + stage * C::STAGE_BYTES);
-                    const uint32_t first = kt != 0 ? 1u : 0u;
-                    if constexpr (MODE == MODE_WS) {
-                        // K step p = input component p (32 bytes into the 128-byte rows)
-                        const uint32_t b_lo0 = desc_lo(sbase + C::WSB_OFF + kt * C::WSB_TAP);
-#pragma unroll
-                        for (int pc = 0; pc < 4; ++pc)
-                            umma_f16_w(dbase, a_lo0 + pc * 2, C::DESC_HI, b_lo0 + pc * 2,
-                                       C::DESC_HI, IDESC_POS, pc != 0 ? 1u : first);
-                    } else {
                     const uint32_t b_lo0 = a_lo0 + (4 * C::A_TILE >> 4);
+                    const uint32_t first = kt != 0 ? 1u : 0u;
 #pragma unroll
                     for (int pc = 0; pc < 4; ++pc) {
 #pragma unroll
@@ -493,7 +308,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             }
                         }
                     }
-                    }
                     ++issued;
                     umma_commit(empty_bar(stage));  // frees the stage when these MMAs finish
                     if (++stage == STAGES) {
@@ -502,7 +316,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
                 if (!ok) break;
-                umma_commit(accf_bar(buf));  // accumulator buffer ready for the epilogue
+                umma_commit(accf0 + 8u * buf);  // accumulator buffer ready for the epilogue
             }
             if (!ok && issued > 0) {
                 // Let every MMA already issued finish before TMEM is released.
@@ -541,14 +355,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     uint4* s5 = reinterpret_cast<uint4*>(b0 + 5 * C::B_TILE);
 #pragma unroll 4
                     for (int i = lane; i < WORDS; i += 32) {
-                        uint4 a = s2[i], b = s3[i];
-                        a.x ^= 0x80008000u; a.y ^= 0x80008000u; a.z ^= 0x80008000u; a.w ^= 0x80008000u;
-                        b.x ^= 0x80008000u; b.y ^= 0x80008000u; b.z ^= 0x80008000u; b.w ^= 0x80008000u;
-                        s0[i] = a;
-                        s5[i] = b;
+                        s0[i] = negate_bf16x8(s2[i]);
+                        s5[i] = negate_bf16x8(s3[i]);
                     }
                     // make the generic-proxy writes visible to the tensor core (async proxy)
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(ready_bar(stage));
                     if (++stage == STAGES) {
@@ -560,116 +371,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
     } else if (warp >= EPI_WARP0) {
         // ------------------------------------------------------------ epilogue
-        const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
-        const int half = (warp - EPI_WARP0) >> 2;  // output components 2*half, 2*half+1
-        const int row = quad * 32 + lane;
-        const bool leader = (warp == EPI_WARP0 + 4 * half) && lane == 0;
-        const int etid = threadIdx.x - EPI_WARP0 * 32;  // 0..255
-        const int Cout = s.Cout;
-        const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(p.ep.residual);
-        float* prm_s = reinterpret_cast<float*>(smem + C::PARAM_OFF);  // [3][4*BNQ]
-        uint8_t* stg = smem + C::STAGING_OFF + half * C::OUT_TILE;
-        const uint32_t stg_addr = smem_u32(stg);
-        int cached_n = -1;
-        int local = 0;
-        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++local) {
-            const int buf = local & 1;
-            const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
-            const bool ok = wait_or_abort(accf_bar(buf), use, limit, abort_flag,
-                                          STATUS_TIMEOUT_EPILOGUE);
-            // leave together: a warp that gave up must not strand the others at a barrier
-            if (named_bar_or(1, 256, !ok)) break;
-            tc_fence_after();
-            const int m_tile = tile / p.num_n_tiles;
-            const int n_tile = tile - m_tile * p.num_n_tiles;
-            if (n_tile != cached_n) {
-                // per-channel vectors of this tile's 4 x BNQ channels -> shared memory
-                named_bar_sync(1, 256);
-                for (int i = etid; i < 4 * BNQ; i += 256) {
-                    const int c = (i / BNQ) * s.Qout + n_tile * BNQ + (i % BNQ);
-                    prm_s[i] = p.ep.bias ? __ldg(p.ep.bias + c) : 0.0f;
-                    prm_s[4 * BNQ + i] = p.ep.scale ? __ldg(p.ep.scale + c) : 1.0f;
-                    prm_s[8 * BNQ + i] = p.ep.scale ? __ldg(p.ep.shift + c) : 0.0f;
-                }
-                named_bar_sync(1, 256);
-                cached_n = n_tile;
-            }
-            const long long m = static_cast<long long>(m_tile) * BM + row;
-            const bool valid = m < s.M;
-            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                                   static_cast<uint32_t>(buf * 4 * BNQ);
-#pragma unroll
-            for (int qq = 0; qq < 2; ++qq) {
-                const int q = 2 * half + qq;
-                // the staging block is free once the previous store has read it
-                if (leader) bulk_wait_group_read<0>();
-                named_bar_sync(2 + half, 128);
-                constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
-#pragma unroll
-                for (int j0 = 0; j0 < BNQ; j0 += CH) {
-                    uint32_t v[32];
-                    if constexpr (CH == 32) {
-                        tmem_ld_32x32b_x32(taddr + q * BNQ + j0, v);
-                    } else {
-                        uint32_t (&v16)[16] = *reinterpret_cast<uint32_t(*)[16]>(v);
-                        tmem_ld_32x32b_x16(taddr + q * BNQ + j0, v16);
-                    }
-                    float rz[CH];
-                    if (res != nullptr && valid) {
-                        const uint4* rp = reinterpret_cast<const uint4*>(
-                            res + m * Cout + q * s.Qout + n_tile * BNQ + j0);
-#pragma unroll
-                        for (int u = 0; u < CH / 8; ++u) {
-                            const uint4 r4 = __ldg(rp + u);
-                            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r4);
-#pragma unroll
-                            for (int t = 0; t < 4; ++t) {
-                                const float2 f = __bfloat1622float2(h[t]);
-                                rz[8 * u + 2 * t] = f.x;
-                                rz[8 * u + 2 * t + 1] = f.y;
-                            }
-                        }
-                    } else {
-#pragma unroll
-                        for (int t = 0; t < CH; ++t) rz[t] = 0.0f;
-                    }
-                    tmem_ld_wait();
-                    const float* pb = prm_s + q * BNQ + j0;
-                    const float* ps = prm_s + 4 * BNQ + q * BNQ + j0;
-                    const float* ph = prm_s + 8 * BNQ + q * BNQ + j0;
-#pragma unroll
-                    for (int u = 0; u < CH / 8; ++u) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int t = 0; t < 4; ++t) {
-                            const int e = 8 * u + 2 * t;
-                            float z0 = __uint_as_float(v[e]) + pb[e];
-                            float z1 = __uint_as_float(v[e + 1]) + pb[e + 1];
-                            z0 = fmaf(ps[e], z0, ph[e]) + rz[e];
-                            z1 = fmaf(ps[e + 1], z1, ph[e + 1]) + rz[e + 1];
-                            w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
-                        }
-                        // 16-byte chunk (j0/8 + u) of this row, swizzled like the TMA map
-                        const uint32_t chunk = static_cast<uint32_t>(j0 / 8 + u);
-                        const uint32_t off = static_cast<uint32_t>(row) * C::OUT_ROW +
-                                             ((chunk ^ ((static_cast<uint32_t>(row) *
-                                                         C::OUT_ROW >> 7) & C::OUT_SW_MASK))
-                                              << 4);
-                        *reinterpret_cast<uint4*>(stg + off) = make_uint4(w[0], w[1], w[2], w[3]);
-                    }
-                }
-                fence_proxy_async_smem();
-                named_bar_sync(2 + half, 128);
-                if (leader) {
-                    tma_store_2d(&tmap_y, stg_addr, q * s.Qout + n_tile * BNQ,
-                                 static_cast<int>(m_tile) * BM);
-                    bulk_commit_group();
-                }
-            }
-            tc_fence_before();
-            mbar_arrive(acce_bar(buf));
-        }
-        if (leader) bulk_wait_group<0>();
+        const int num_n = p.num_n_tiles;
+        const long long M = s.M;
+        epilogue_role<BNQ, false>(
+            s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
+            reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
+            abort_flag, [num_n, M](int tile) {
+                EpiTile g;
+                const int m_tile = tile / num_n;
+                g.n_tile = tile - m_tile * num_n;
+                g.m0 = static_cast<long long>(m_tile) * BM;
+                const long long left = M - g.m0;
+                g.rows = left < BM ? static_cast<int>(left) : BM;
+                g.sy = static_cast<int>(g.m0);
+                g.sz = 0;
+                return g;
+            });
     }
 
     tc_fence_before();
@@ -680,6 +397,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tmem_dealloc(tmem_base, C::TMEM_COLS);
     }
 }
+
+#include "qconv_ws.cuh"
 
 // ---------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
@@ -703,12 +422,14 @@ bool load_encoders() {
     return g_encode_tiled != nullptr && g_encode_im2col != nullptr;
 }
 
-CUtensorMapSwizzle swizzle_for(int kappa) {
-    return kappa == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
-                       : (kappa == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B);
+CUtensorMapSwizzle swizzle_for_row(int row_bytes) {
+    return row_bytes == 128 ? CU_TENSOR_MAP_SWIZZLE_128B
+                            : (row_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                               : CU_TENSOR_MAP_SWIZZLE_32B);
 }
 
-bool encode_x(CUtensorMap* map, const ConvShape& s, const void* x, int kappa) {
+// Activation im2col map: boxes of BM output pixels x `channels` channels.
+bool encode_x_im2col(CUtensorMap* map, const ConvShape& s, const void* x, int channels) {
     const cuuint64_t dims[4] = {static_cast<cuuint64_t>(s.Cin), static_cast<cuuint64_t>(s.W),
                                 static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(s.Cin) * 2,
@@ -722,8 +443,27 @@ bool encode_x(CUtensorMap* map, const ConvShape& s, const void* x, int kappa) {
                                 static_cast<cuuint32_t>(s.stride), 1};
     const CUresult r = g_encode_im2col(
         map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, lower,
-        upper, static_cast<cuuint32_t>(kappa), BM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-        swizzle_for(kappa), CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        upper, static_cast<cuuint32_t>(channels), BM, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+        swizzle_for_row(channels * 2), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// Activation tiled map for halo boxes: `channels` x Wo columns x `rows` rows of one image.
+bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int channels,
+                   int rows) {
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(s.Cin), static_cast<cuuint64_t>(s.W),
+                                static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(s.Cin) * 2,
+                                   static_cast<cuuint64_t>(s.Cin) * 2 * s.W,
+                                   static_cast<cuuint64_t>(s.Cin) * 2 * s.W * s.H};
+    const cuuint32_t box[4] = {static_cast<cuuint32_t>(channels), static_cast<cuuint32_t>(s.Wo),
+                               static_cast<cuuint32_t>(rows), 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = g_encode_tiled(
+        map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
+        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(channels * 2),
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
 
@@ -735,26 +475,57 @@ bool encode_w(CUtensorMap* map, const ConvShape& s, const void* w, int kappa, in
     const cuuint32_t estr[2] = {1, 1};
     const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                                       const_cast<void*>(w), dims, strides, box, estr,
-                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(kappa),
+                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(kappa * 2),
                                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
 
-// Output [M rows][Cout] bf16, stored in boxes of 128 rows x BNQ channels.
-bool encode_y(CUtensorMap* map, const ConvShape& s, const void* y, int bnq) {
+// Output [M rows][Cout] bf16, stored in boxes of BM rows x BNQ channels.
+bool encode_y_2d(CUtensorMap* map, const ConvShape& s, const void* y, int bnq) {
     const cuuint64_t dims[2] = {static_cast<cuuint64_t>(s.Cout), static_cast<cuuint64_t>(s.M)};
     const cuuint64_t strides[1] = {static_cast<cuuint64_t>(s.Cout) * 2};
     const cuuint32_t box[2] = {static_cast<cuuint32_t>(bnq), static_cast<cuuint32_t>(BM)};
     const cuuint32_t estr[2] = {1, 1};
-    const CUtensorMapSwizzle sw = bnq == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
-                                            : (bnq == 32 ? CU_TENSOR_MAP_SWIZZLE_64B
-                                                         : CU_TENSOR_MAP_SWIZZLE_32B);
-    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(y),
-                                      dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                                      const_cast<void*>(y), dims, strides, box, estr,
+                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(bnq * 2),
                                       CU_TENSOR_MAP_L2_PROMOTION_NONE,
                                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+// Output viewed as [N][Ho*Wo][Cout], stored in boxes of `rows` pixels of one image, so a
+// partial last row block of an image is clipped at the image end.
+bool encode_y_3d(CUtensorMap* map, const ConvShape& s, const void* y, int bnq, int rows) {
+    const cuuint64_t hw = static_cast<cuuint64_t>(s.Ho) * s.Wo;
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(s.Cout), hw,
+                                static_cast<cuuint64_t>(s.N)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(s.Cout) * 2,
+                                   static_cast<cuuint64_t>(s.Cout) * 2 * hw};
+    const cuuint32_t box[3] = {static_cast<cuuint32_t>(bnq), static_cast<cuuint32_t>(rows), 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                                      const_cast<void*>(y), dims, strides, box, estr,
+                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(bnq * 2),
+                                      CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// The shared-memory opt-in is per device and kernel; set it once for each.
+template <typename K>
+cudaError_t set_smem_once(K kern, int bytes, std::atomic<unsigned long long>& done) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(done.load() & bit)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        if (e != cudaSuccess) return e;
+        done.fetch_or(bit);
+    }
+    return cudaSuccess;
 }
 
 template <int KAPPA, int BNQ, int MODE>
@@ -764,22 +535,13 @@ cudaError_t launch_cfg(const CUtensorMap maps[6], const TcParams& prm, int grid,
     if constexpr (!C::FITS) {
         return cudaErrorInvalidValue;
     } else {
-    auto kern = qconv_tc_kernel<KAPPA, BNQ, MODE>;
-    // The shared-memory opt-in is per device; set it once for each.
-    static std::atomic<unsigned long long> attr_done{0};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    const unsigned long long bit = 1ull << (dev & 63);
-    if (!(attr_done.load() & bit)) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 C::SMEM_BYTES);
+        auto kern = qconv_tc_kernel<KAPPA, BNQ, MODE>;
+        static std::atomic<unsigned long long> attr_done{0};
+        cudaError_t e = set_smem_once(kern, C::SMEM_BYTES, attr_done);
         if (e != cudaSuccess) return e;
-        attr_done.fetch_or(bit);
-    }
-    kern<<<grid, NUM_THREADS, C::SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3],
-                                                       maps[4], maps[5], prm);
-    return cudaGetLastError();
+        kern<<<grid, NUM_THREADS, C::SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3],
+                                                           maps[4], maps[5], prm);
+        return cudaGetLastError();
     }
 }
 
@@ -789,16 +551,16 @@ constexpr bool cfg_fits() {
 }
 
 // Encoded tensor maps of recent calls, keyed by every value that goes into them, so a
-// layer called repeatedly on the same buffers skips the five host-side encodes.
+// layer called repeatedly on the same buffers skips the host-side encodes.
 struct MapKey {
     const void* ptr[6];
-    int N, H, W, Cin, Cout, kh, kw, stride, pad, kappa, bnq;
+    int N, H, W, Cin, Cout, kh, kw, stride, pad, kappa, bnq, variant;
     bool operator==(const MapKey& o) const {
         for (int i = 0; i < 6; ++i)
             if (ptr[i] != o.ptr[i]) return false;
         return N == o.N && H == o.H && W == o.W && Cin == o.Cin && Cout == o.Cout &&
                kh == o.kh && kw == o.kw && stride == o.stride && pad == o.pad &&
-               kappa == o.kappa && bnq == o.bnq;
+               kappa == o.kappa && bnq == o.bnq && variant == o.variant;
     }
 };
 
@@ -813,6 +575,37 @@ MapEntry g_map_cache[kMapCacheSize];
 int g_map_next = 0;
 std::mutex g_map_mu;
 
+bool cache_lookup(const MapKey& key, CUtensorMap* maps) {
+    std::lock_guard<std::mutex> lk(g_map_mu);
+    for (int i = 0; i < kMapCacheSize; ++i)
+        if (g_map_cache[i].valid && g_map_cache[i].key == key) {
+            for (int l = 0; l < 6; ++l) maps[l] = g_map_cache[i].maps[l];
+            return true;
+        }
+    return false;
+}
+
+void cache_store(const MapKey& key, const CUtensorMap* maps) {
+    std::lock_guard<std::mutex> lk(g_map_mu);
+    MapEntry& e = g_map_cache[g_map_next];
+    g_map_next = (g_map_next + 1) % kMapCacheSize;
+    e.key = key;
+    for (int l = 0; l < 6; ++l) e.maps[l] = maps[l];
+    e.valid = true;
+}
+
+MapKey make_key(const ConvShape& s, const void* x, const void* const w[4], const void* out,
+                int kappa, int bnq, int variant) {
+    MapKey key;
+    key.ptr[0] = x;
+    for (int l = 0; l < 4; ++l) key.ptr[1 + l] = w[l];
+    key.ptr[5] = out;
+    key.N = s.N; key.H = s.H; key.W = s.W; key.Cin = s.Cin; key.Cout = s.Cout;
+    key.kh = s.kh; key.kw = s.kw; key.stride = s.stride; key.pad = s.pad;
+    key.kappa = kappa; key.bnq = bnq; key.variant = variant;
+    return key;
+}
+
 int pick_kappa(int Qin, int req) {
     if (req == 16 || req == 32 || req == 64) return Qin % req == 0 ? req : 0;
     if (Qin % 32 == 0) return 32;
@@ -824,6 +617,88 @@ int pick_bnq(int Qout, int req) {
     if (Qout % 64 == 0) return 64;
     if (Qout % 32 == 0) return 32;
     return 16;
+}
+
+int grid_for(const TcOptions& opt, int num_sms, int num_tiles) {
+    int grid = opt.max_ctas > 0 ? opt.max_ctas : num_sms;
+    if (grid > num_tiles) grid = num_tiles;
+    return grid < 1 ? 1 : grid;
+}
+
+cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
+                      const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
+                      cudaStream_t stream, char* err, size_t errlen) {
+    WsParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.taps = s.kh * s.kw;
+    const bool halo = ws_halo_ok(s) && opt.ws_halo != 0;
+    prm.halo = halo ? 1 : 0;
+    long long tiles;
+    if (halo) {
+        prm.R = BM / s.Wo;
+        prm.tpi = (s.Ho + prm.R - 1) / prm.R;
+        prm.kblocks = s.kw;
+        prm.box_bytes = s.Wo * (prm.R + s.kh - 1) * WS_ROW_BYTES;
+        tiles = static_cast<long long>(s.N) * prm.tpi;
+    } else {
+        prm.R = 0;
+        prm.tpi = 0;
+        prm.kblocks = prm.taps;
+        prm.box_bytes = BM * WS_ROW_BYTES;
+        tiles = (s.M + BM - 1) / BM;
+    }
+    if (tiles > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many tiles");
+        return cudaErrorInvalidValue;
+    }
+    prm.num_tiles = static_cast<int>(tiles);
+    prm.stage_bytes = (prm.box_bytes + 1023) & ~1023;
+    int stages = WsCfg::RING_BYTES / prm.stage_bytes;
+    if (stages > MAX_STAGES) stages = MAX_STAGES;
+    if (stages < 2) {
+        snprintf(err, errlen, "weight-stationary pixel box of %d bytes does not fit",
+                 prm.box_bytes);
+        return cudaErrorInvalidValue;
+    }
+    prm.stages = stages;
+
+    const MapKey key = make_key(s, x, w, out, 16, 16, halo ? 3 : 2);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        const bool okx = halo ? encode_x_halo(&maps[0], s, x, 4 * 16, prm.R + s.kh - 1)
+                              : encode_x_im2col(&maps[0], s, x, 4 * 16);
+        if (!okx) {
+            snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        // one store box covers the whole 64-channel output row (wide epilogue)
+        const bool oky = halo ? encode_y_3d(&maps[1], s, out, 64, prm.R * s.Wo)
+                              : encode_y_2d(&maps[1], s, out, 64);
+        if (!oky) {
+            snprintf(err, errlen, "tensor-map encode failed for the output tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 2; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    const int grid = grid_for(opt, num_sms, prm.num_tiles);
+    static std::atomic<unsigned long long> done_h{0}, done_t{0};
+    if (halo) {
+        auto kern = qconv_ws_kernel<true>;
+        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+    } else {
+        auto kern = qconv_ws_kernel<false>;
+        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+    }
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -850,12 +725,12 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
         snprintf(err, errlen, "tensor-map encoders unavailable from the CUDA driver");
         return cudaErrorNotSupported;
     }
-    int kappa = pick_kappa(s.Qin, opt.kappa);
-    int bnq = pick_bnq(s.Qout, opt.bnq);
     // Weight-stationary for 16 -> 16 quaternion channels (the whole expanded weight fits);
     // pair mode (N = 2 BNQ per MMA) otherwise, unless the tile is so narrow that even
     // pairs stay far below the tensor pipe's per-instruction cost.
     const bool ws_ok = s.Qin == 16 && s.Qout == 16 && s.kh * s.kw <= WS_MAX_TAPS;
+    int kappa = pick_kappa(s.Qin, opt.kappa);
+    const int bnq = pick_bnq(s.Qout, opt.bnq);
     int mode;
     if (opt.mode == 1) mode = MODE_QUAD;
     else if (opt.mode == 2) mode = MODE_PAIR;
@@ -867,79 +742,17 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                      WS_MAX_TAPS);
             return cudaErrorInvalidValue;
         }
-        kappa = 16;
-        bnq = 16;
+        return launch_ws(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     }
-    // A 6-slot stage of 64 x 64 letter blocks plus 64-channel pixel tiles does not fit
-    // twice in shared memory; use 32-channel K blocks then.
-    if (mode == MODE_PAIR && kappa == 64 && bnq == 64 && opt.kappa == 0) kappa = 32;
     if (kappa == 0 || bnq == 0) {
         snprintf(err, errlen, "requested tile (kappa=%d, bnq=%d) does not divide Qin=%d/Qout=%d",
                  opt.kappa, opt.bnq, s.Qin, s.Qout);
         return cudaErrorInvalidValue;
     }
-    MapKey key;
-    key.ptr[0] = x;
-    for (int l = 0; l < 4; ++l) key.ptr[1 + l] = w[l];
-    key.ptr[5] = out;
-    key.N = s.N; key.H = s.H; key.W = s.W; key.Cin = s.Cin; key.Cout = s.Cout;
-    key.kh = s.kh; key.kw = s.kw; key.stride = s.stride; key.pad = s.pad;
-    key.kappa = mode == MODE_WS ? -kappa : kappa; key.bnq = bnq;
-    CUtensorMap maps[6];
-    bool hit = false;
+    // A 6-slot stage of 64 x 64 letter blocks plus 64-channel pixel tiles does not fit
+    // twice in shared memory; use 32-channel K blocks then.
+    if (mode == MODE_PAIR && kappa == 64 && bnq == 64 && opt.kappa == 0) kappa = 32;
     {
-        std::lock_guard<std::mutex> lk(g_map_mu);
-        for (int i = 0; i < kMapCacheSize; ++i)
-            if (g_map_cache[i].valid && g_map_cache[i].key == key) {
-                for (int l = 0; l < 6; ++l) maps[l] = g_map_cache[i].maps[l];
-                hit = true;
-                break;
-            }
-    }
-    if (!hit) {
-        if (!encode_x(&maps[0], s, x, mode == MODE_WS ? 4 * kappa : kappa)) {
-            snprintf(err, errlen, "cuTensorMapEncodeIm2col failed for the activation tensor");
-            return cudaErrorInvalidValue;
-        }
-        for (int l = 0; l < 4; ++l)
-            if (!encode_w(&maps[1 + l], s, w[l], kappa, bnq)) {
-                snprintf(err, errlen, "cuTensorMapEncodeTiled failed for weight letter %d", l);
-                return cudaErrorInvalidValue;
-            }
-        if (!encode_y(&maps[5], s, out, bnq)) {
-            snprintf(err, errlen, "cuTensorMapEncodeTiled failed for the output tensor");
-            return cudaErrorInvalidValue;
-        }
-        std::lock_guard<std::mutex> lk(g_map_mu);
-        MapEntry& e = g_map_cache[g_map_next];
-        g_map_next = (g_map_next + 1) % kMapCacheSize;
-        e.key = key;
-        for (int l = 0; l < 6; ++l) e.maps[l] = maps[l];
-        e.valid = true;
-    }
-    TcParams prm;
-    prm.s = s;
-    prm.ep = ep;
-    prm.out = static_cast<__nv_bfloat16*>(out);
-    prm.kchunks = s.Qin / kappa;
-    prm.ktiles = s.kh * s.kw * prm.kchunks;
-    prm.num_n_tiles = s.Qout / bnq;
-    const long long m_tiles = (s.M + BM - 1) / BM;
-    const long long tiles = m_tiles * prm.num_n_tiles;
-    if (tiles > 0x7fffffffLL) {
-        snprintf(err, errlen, "too many tiles");
-        return cudaErrorInvalidValue;
-    }
-    prm.num_tiles = static_cast<int>(tiles);
-    prm.wait_limit_ns = opt.wait_limit_ns;
-    prm.inject_stall = opt.inject_stall;
-    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
-    int grid = opt.max_ctas > 0 ? opt.max_ctas : num_sms;
-    if (grid > prm.num_tiles) grid = prm.num_tiles;
-    if (grid < 1) grid = 1;
-
-    static_assert(Cfg<16, 16, MODE_WS>::FITS, "weight-stationary tile must fit");
-    if (mode != MODE_WS) {
         bool fits = true;
 #define QUAN_FIT_CASE(K, B)                                                        \
     if (kappa == K && bnq == B)                                                    \
@@ -954,7 +767,41 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
             return cudaErrorInvalidValue;
         }
     }
-    if (mode == MODE_WS) return launch_cfg<16, 16, MODE_WS>(maps, prm, grid, stream);
+    const MapKey key = make_key(s, x, w, out, kappa, bnq, 0);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_im2col(&maps[0], s, x, kappa)) {
+            snprintf(err, errlen, "cuTensorMapEncodeIm2col failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 0; l < 4; ++l)
+            if (!encode_w(&maps[1 + l], s, w[l], kappa, bnq)) {
+                snprintf(err, errlen, "cuTensorMapEncodeTiled failed for weight letter %d", l);
+                return cudaErrorInvalidValue;
+            }
+        if (!encode_y_2d(&maps[5], s, out, bnq)) {
+            snprintf(err, errlen, "cuTensorMapEncodeTiled failed for the output tensor");
+            return cudaErrorInvalidValue;
+        }
+        cache_store(key, maps);
+    }
+    TcParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    prm.kchunks = s.Qin / kappa;
+    prm.ktiles = s.kh * s.kw * prm.kchunks;
+    prm.num_n_tiles = s.Qout / bnq;
+    const long long m_tiles = (s.M + BM - 1) / BM;
+    const long long tiles = m_tiles * prm.num_n_tiles;
+    if (tiles > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many tiles");
+        return cudaErrorInvalidValue;
+    }
+    prm.num_tiles = static_cast<int>(tiles);
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    const int grid = grid_for(opt, num_sms, prm.num_tiles);
+
 #define QUAN_TC_CASE(K, B)                                                       \
     if (kappa == K && bnq == B)                                                  \
         return mode == MODE_PAIR ? launch_cfg<K, B, MODE_PAIR>(maps, prm, grid, stream) \

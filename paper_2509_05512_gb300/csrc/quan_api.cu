@@ -16,7 +16,7 @@ namespace {
 thread_local char t_errmsg[512] = "";
 thread_local int t_last_path = 0;
 std::atomic<int> g_path{QUAN_PATH_AUTO};
-std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0};
+std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1};
 std::atomic<unsigned long long> g_wait_limit{2000000000ull};
 std::atomic<int> g_inject{0};
 
@@ -155,6 +155,7 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         opt.bnq = g_bnq.load();
         opt.max_ctas = g_max_ctas.load();
         opt.mode = g_mode.load();
+        opt.ws_halo = g_ws_halo.load();
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -253,6 +254,11 @@ quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     g_bnq.store(bnq);
     g_max_ctas.store(max_ctas);
     g_mode.store(mode);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_tc_halo(int enable) {
+    g_ws_halo.store(enable ? 1 : 0);
     return QUAN_OK;
 }
 

@@ -1,0 +1,304 @@
+// tc_common.cuh -- pieces shared by the tensor-core quaternion convolution kernels
+// (qconv_tc.cu is the only translation unit that includes this file): constants, the
+// device status word, descriptor helpers, bounded waits and the 8-warp epilogue.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace quan {
+
+// Device status word: bits set by kernels whose bounded waits ran out.
+__device__ unsigned int g_status;
+
+namespace tc {
+
+constexpr int BM = 128;           // rows (output pixels) of the MMA tile
+constexpr int NUM_THREADS = 384;  // 12 warps
+constexpr int EPI_WARP0 = 4;      // warps 4..11: epilogue
+constexpr int UMMA_K = 16;        // K of one kind::f16 MMA
+
+// Output component q takes input component p through letter L = q xor p, read off Eq. 5:
+//   y_r: +W_r X_r  -W_i X_i  -W_j X_j  -W_k X_k
+//   y_i: +W_i X_r  +W_r X_i  -W_k X_j  +W_j X_k
+//   y_j: +W_j X_r  +W_k X_i  +W_r X_j  -W_i X_k
+//   y_k: +W_k X_r  -W_j X_i  +W_i X_j  +W_r X_k
+// Bit (4 q + p) of NEG_MASK marks the negative terms.
+constexpr uint32_t NEG_MASK = (1u << 1) | (1u << 2) | (1u << 3)  // y_r: X_i, X_j, X_k
+                              | (1u << 6)                        // y_i: X_j
+                              | (1u << 11)                       // y_j: X_k
+                              | (1u << 13);                      // y_k: X_i
+
+// tcgen05 shared-memory matrix descriptors (K-major, swizzled operand tiles) are built
+// as two 32-bit words: the low word holds the start address >> 4 (bits 0-13) and the
+// leading byte offset (bits 16-29, unused for these layouts, set to 1); the high word
+// holds the stride byte offset >> 4 (pitch of 8-row core-matrix groups), the
+// descriptor version (bit 46) and the swizzle mode (bits 61-63).
+__device__ __forceinline__ uint32_t desc_lo(uint32_t saddr) {
+    return ((saddr & 0x3FFFFu) >> 4) | (1u << 16);
+}
+
+constexpr uint32_t desc_hi(uint32_t sbo_bytes, uint32_t layout) {
+    return (sbo_bytes >> 4) | (1u << 14) | (layout << 29);
+}
+
+// swizzle mode of the descriptor for K-major rows of `row_bytes` (128, 64 or 32)
+constexpr uint32_t desc_layout(int row_bytes) {
+    return row_bytes == 128 ? 2u : (row_bytes == 64 ? 4u : 6u);
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B, fp32 D, both operands K-major.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N, int negate) {
+    return (1u << 4)                                   // D format: f32
+           | (1u << 7)                                 // A format: bf16
+           | (1u << 10)                                // B format: bf16
+           | (static_cast<uint32_t>(negate) << 13)     // negate A
+           | (static_cast<uint32_t>(N >> 3) << 17)     // N / 8
+           | (static_cast<uint32_t>(M >> 4) << 24);    // M / 16
+}
+
+__device__ __forceinline__ float activate(float z, int act) {
+    if (act == 1) return fmaxf(z, 0.0f);
+    if (act == 2) return z / (1.0f + __expf(-z));
+    return z;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ uint4 negate_bf16x8(uint4 v) {
+    v.x ^= 0x80008000u;
+    v.y ^= 0x80008000u;
+    v.z ^= 0x80008000u;
+    v.w ^= 0x80008000u;
+    return v;
+}
+
+// Bounded wait: false once the CTA-wide abort flag is up or `limit` ns have passed (then
+// the status bit is recorded and the abort flag raised).
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uint64_t limit,
+                                              volatile int* abort_flag, unsigned code) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (global_timer_ns() - t0 > limit) {
+            atomicOr(&g_status, code);
+            *abort_flag = 1;
+            return false;
+        }
+    }
+}
+
+// Wait for the most recent fill of each stage a producer armed, so that no copy still
+// targets this CTA's shared memory when it exits after an abort.
+__device__ __forceinline__ void drain_fills(uint32_t bar0, int stages, uint32_t filled,
+                                            uint32_t parity, uint64_t limit) {
+    for (int i = 0; i < stages; ++i) {
+        if (!(filled & (1u << i))) continue;
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(bar0 + 8u * i, (parity >> i) & 1u)) {
+            if (global_timer_ns() - t0 > limit) {
+                atomicOr(&g_status, STATUS_TIMEOUT_DRAIN);
+                break;
+            }
+        }
+    }
+}
+
+// Geometry of one output tile as the epilogue sees it.
+struct EpiTile {
+    long long m0;  // linear index of the pixel in TMEM lane 0
+    int rows;      // valid lanes (pixels) of the tile
+    int n_tile;    // quaternion output channel block
+    int sy, sz;    // TMA store coordinates after the channel one (2-D: sy = m0)
+};
+
+// Shared-memory resources of the epilogue: two staging blocks of 128 x BNQ bf16 (one per
+// half; with WIDE, two blocks of 128 x 4 BNQ, one per tile parity) and the per-channel
+// vectors [3][4 BNQ].
+template <int BNQ, bool WIDE = false>
+struct EpiSmem {
+    static constexpr int OUT_TILE = BM * BNQ * 2;
+    static constexpr int STAGING_BYTES = WIDE ? 2 * 4 * OUT_TILE : 2 * OUT_TILE;
+    static constexpr int PARAM_BYTES = 3 * 4 * BNQ * 4;
+    static constexpr uint32_t OUT_ROW = BNQ * 2;
+    static constexpr uint32_t OUT_SW_MASK = BNQ == 64 ? 7u : (BNQ == 32 ? 3u : 1u);
+};
+
+// The epilogue role (warps 4..11, two per TMEM lane quadrant; the first four warps
+// handle output components r, i and the last four j, k).  For each tile of this CTA:
+// wait for its accumulator buffer, apply act(scale*(acc+bias)+shift+residual) (IQBN
+// inference form of Eq. 11-12), round to bf16, write a swizzled shared-memory block per
+// component and store it with TMA (rows outside the tensor are clipped by the map).
+// With WIDE (4 BNQ = 64 channels = the whole output row, BNQ == Qout) all four
+// components go into one 128-byte-row block and a single TMA store per tile, the block
+// alternating between two buffers so the store overlaps the next tile.
+// Accumulator buffer b of a tile lives at TMEM columns [4 BNQ b, 4 BNQ (b+1)), component
+// q at offset q BNQ.
+template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false>
+__device__ __forceinline__ void epilogue_role(const ConvShape& s, const EpilogueArgs& ep,
+                                              const CUtensorMap* tmap_y, uint32_t tmem_base,
+                                              uint8_t* staging, float* prm_s,
+                                              uint32_t accf0, uint32_t acce0, int num_tiles,
+                                              uint64_t limit, volatile int* abort_flag,
+                                              Geo geo) {
+    using E = EpiSmem<BNQ, WIDE>;
+    static_assert(!WIDE || BNQ == 16, "wide stores need 64-channel rows");
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
+    const int half = (warp - EPI_WARP0) >> 2;  // output components 2*half, 2*half+1
+    const int row = quad * 32 + lane;
+    const bool leader = (warp == EPI_WARP0 + 4 * half) && lane == 0;
+    const int etid = threadIdx.x - EPI_WARP0 * 32;  // 0..255
+    const int Cout = s.Cout;
+    const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(ep.residual);
+    uint8_t* stg = staging + (WIDE ? 0 : half * E::OUT_TILE);
+    uint32_t stg_addr = smem_u32(stg);
+    int cached_n = -1;
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+        const int buf = local & 1;
+        const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        // one lane per warp polls the barrier (256 pollers would crowd the shared-memory
+        // pipe that TMA and the barriers themselves use), then broadcasts the result
+        bool ok = true;
+        if (lane == 0)
+            ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        // leave together: a warp that gave up must not strand the others at a barrier
+        if (named_bar_or(1, 256, !ok)) break;
+        tc_fence_after();
+        const EpiTile g = geo(tile);
+        if (g.n_tile != cached_n) {
+            // per-channel vectors of this tile's 4 x BNQ channels -> shared memory
+            named_bar_sync(1, 256);
+            for (int i = etid; i < 4 * BNQ; i += 256) {
+                const int c = (i / BNQ) * s.Qout + g.n_tile * BNQ + (i % BNQ);
+                prm_s[i] = ep.bias ? __ldg(ep.bias + c) : 0.0f;
+                prm_s[4 * BNQ + i] = ep.scale ? __ldg(ep.scale + c) : 1.0f;
+                prm_s[8 * BNQ + i] = ep.scale ? __ldg(ep.shift + c) : 0.0f;
+            }
+            named_bar_sync(1, 256);
+            cached_n = g.n_tile;
+        }
+        const long long m = g.m0 + row;
+        const bool valid = row < g.rows;
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                               static_cast<uint32_t>(buf * 4 * BNQ);
+        if constexpr (WIDE) {
+            // block of this tile parity; free once the store of two tiles ago has read it
+            stg = staging + buf * 4 * E::OUT_TILE;
+            stg_addr = smem_u32(stg);
+            if (threadIdx.x == EPI_WARP0 * 32) bulk_wait_group_read<1>();
+            named_bar_sync(1, 256);
+        }
+#pragma unroll
+        for (int qq = 0; qq < 2; ++qq) {
+            const int q = 2 * half + qq;
+            if constexpr (!WIDE) {
+                // the staging block is free once the previous store has read it
+                if (leader) bulk_wait_group_read<0>();
+                named_bar_sync(2 + half, 128);
+            }
+            constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
+#pragma unroll
+            for (int j0 = 0; j0 < BNQ; j0 += CH) {
+                uint32_t v[32];
+                if constexpr (CH == 32) {
+                    tmem_ld_32x32b_x32(taddr + q * BNQ + j0, v);
+                } else {
+                    uint32_t(&v16)[16] = *reinterpret_cast<uint32_t(*)[16]>(v);
+                    tmem_ld_32x32b_x16(taddr + q * BNQ + j0, v16);
+                }
+                float rz[CH];
+                if (res != nullptr && valid) {
+                    const uint4* rp = reinterpret_cast<const uint4*>(
+                        res + m * Cout + q * s.Qout + g.n_tile * BNQ + j0);
+#pragma unroll
+                    for (int u = 0; u < CH / 8; ++u) {
+                        const uint4 r4 = __ldg(rp + u);
+                        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r4);
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const float2 f = __bfloat1622float2(h[t]);
+                            rz[8 * u + 2 * t] = f.x;
+                            rz[8 * u + 2 * t + 1] = f.y;
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int t = 0; t < CH; ++t) rz[t] = 0.0f;
+                }
+                tmem_ld_wait();
+                const float* pb = prm_s + q * BNQ + j0;
+                const float* ps = prm_s + 4 * BNQ + q * BNQ + j0;
+                const float* ph = prm_s + 8 * BNQ + q * BNQ + j0;
+#pragma unroll
+                for (int u = 0; u < CH / 8; ++u) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const int e = 8 * u + 2 * t;
+                        float z0 = __uint_as_float(v[e]) + pb[e];
+                        float z1 = __uint_as_float(v[e + 1]) + pb[e + 1];
+                        z0 = fmaf(ps[e], z0, ph[e]) + rz[e];
+                        z1 = fmaf(ps[e + 1], z1, ph[e + 1]) + rz[e + 1];
+                        w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                    }
+                    if constexpr (WIDE) {
+                        // 128-byte row of all four components, 128-byte swizzle
+                        const uint32_t chunk = static_cast<uint32_t>(q * (BNQ / 8) + j0 / 8 + u);
+                        const uint32_t off = static_cast<uint32_t>(row) * 128 +
+                                             ((chunk ^ (static_cast<uint32_t>(row) & 7u)) << 4);
+                        *reinterpret_cast<uint4*>(stg + off) = make_uint4(w[0], w[1], w[2], w[3]);
+                    } else {
+                        // 16-byte chunk (j0/8 + u) of this row, swizzled like the TMA map
+                        const uint32_t chunk = static_cast<uint32_t>(j0 / 8 + u);
+                        const uint32_t off = static_cast<uint32_t>(row) * E::OUT_ROW +
+                                             ((chunk ^ ((static_cast<uint32_t>(row) * E::OUT_ROW >>
+                                                         7) & E::OUT_SW_MASK))
+                                              << 4);
+                        *reinterpret_cast<uint4*>(stg + off) = make_uint4(w[0], w[1], w[2], w[3]);
+                    }
+                }
+            }
+            if constexpr (!WIDE) {
+                fence_proxy_async_smem();
+                named_bar_sync(2 + half, 128);
+                if (leader) {
+                    const int c0 = q * s.Qout + g.n_tile * BNQ;
+                    if constexpr (STORE3D)
+                        tma_store_3d(tmap_y, stg_addr, c0, g.sy, g.sz);
+                    else
+                        tma_store_2d(tmap_y, stg_addr, c0, g.sy);
+                    bulk_commit_group();
+                }
+            }
+        }
+        if constexpr (WIDE) {
+            fence_proxy_async_smem();
+            named_bar_sync(1, 256);
+            if (threadIdx.x == EPI_WARP0 * 32) {
+                if constexpr (STORE3D)
+                    tma_store_3d(tmap_y, stg_addr, 0, g.sy, g.sz);
+                else
+                    tma_store_2d(tmap_y, stg_addr, 0, g.sy);
+                bulk_commit_group();
+            }
+        }
+        tc_fence_before();
+        mbar_arrive(acce0 + 8u * buf);
+    }
+    if (leader || (WIDE && threadIdx.x == EPI_WARP0 * 32)) bulk_wait_group<0>();
+}
+
+}  // namespace tc
+}  // namespace quan

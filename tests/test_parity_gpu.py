@@ -38,6 +38,7 @@ def _reset_paths():
     quan.quan_set_tc_tiles(0, 0, 0, 0)
     quan.quan_set_fault_injection(False)
     quan.quan_set_wait_limit_ns(0)
+    quan.quan_set_tc_halo(True)
 
 
 def run_gpu(d, path=quan.QUAN_PATH_AUTO, guard=True):
@@ -105,15 +106,30 @@ WS_CASES = [
     ("ws_stride2", 2, 15, 17, 64, 64, 3, 2, 1, {"residual": True}),
     ("ws_1x1", 2, 9, 7, 64, 64, 1, 1, 0, {"bias": True, "act": quan.QUAN_ACT_SILU}),
     ("ws_5x1", 1, 9, 8, 64, 64, 5, 1, 2, {"kw": 1}),
+    # row-block halo staging: partial last block (R = 5), 112-row tiles, 1x1, valid conv
+    ("ws_halo_24", 2, 24, 24, 64, 64, 3, 1, 1, {"residual": True}),
+    ("ws_halo_56", 1, 56, 56, 64, 64, 3, 1, 1, {}),
+    ("ws_halo_1x1", 2, 16, 16, 64, 64, 1, 1, 0, {"act": quan.QUAN_ACT_NONE}),
+    ("ws_halo_valid", 2, 18, 18, 64, 64, 3, 1, 0, {"bias": True}),
+    ("ws_halo_1x3", 1, 12, 16, 64, 64, 1, 1, 0, {"kw": 3}),
 ]
 
 
+@pytest.mark.parametrize("halo", [1, 0])
 @pytest.mark.parametrize("case", WS_CASES, ids=[c[0] for c in WS_CASES])
-def test_tc_weight_stationary_layers(case):
+def test_tc_weight_stationary_layers(case, halo):
     name, N, H, W, Cin, Cout, k, s, p, extra = case
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(205, len(name)), **extra)
     quan.quan_set_tc_tiles(0, 0, 0, 3)
+    quan.quan_set_tc_halo(bool(halo))
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+@pytest.mark.parametrize("halo", [1, 0])
+def test_config1_weight_stationary_staging(halo):
+    quan.quan_set_tc_tiles(0, 0, 0, 3)
+    quan.quan_set_tc_halo(bool(halo))
+    check(inputs.LAYERS["c1"], path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
 # ------------------------------------------------------------------ tensor-core small layers
@@ -317,6 +333,29 @@ def test_maxpool(shape):
 
 
 # ------------------------------------------------------------------ failure detection
+
+@pytest.mark.parametrize("mode", [2, 3])
+def test_bounded_wait_timeout_every_kernel(mode):
+    # the failure-injection path of the pair-mode and weight-stationary kernels
+    spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    quan.quan_set_path(quan.QUAN_PATH_TC)
+    quan.quan_set_tc_tiles(0, 16 if mode == 2 else 0, 0, mode)
+    quan.quan_set_wait_limit_ns(5_000_000)
+    quan.quan_set_fault_injection(True)
+    quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act)
+    st, bits = quan.quan_device_status()
+    assert st == quan.QUAN_ERR_DEVICE_TIMEOUT and bits != 0
+    quan.quan_set_fault_injection(False)
+    quan.quan_set_wait_limit_ns(0)
+    y = quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    d2 = dict(d); d2["scale"] = d2["shift"] = None
+    assert_bf16_close(out_f64(y), oracle_full(d2), "after-timeout-%d" % mode)
+
 
 def test_bounded_wait_timeout_reports_status_and_context_survives():
     spec = inputs.small_layer("inject", 1, 16, 16, 64, 64, 3, 1, 1, seed=(400, 0))
