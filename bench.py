@@ -46,6 +46,11 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target duration of the bounded oracle sample")
+    ap.add_argument("--profile", action="store_true",
+                    help="for ncu: exactly W + K plain launches, no clock sampling, no e2e "
+                         "or CPU legs")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="time a plain launch loop instead of one CUDA-graph replay")
     return ap.parse_args()
 
 
@@ -268,6 +273,7 @@ def main():
     if args.workload == "backbone":
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs)
+        runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
         workload_desc = runner.describe()
     else:
@@ -275,14 +281,23 @@ def main():
         runner = LayerRunner(spec, torch, quan, inputs)
         unit, per_step_units, dtype = "TFLOP/s", spec.flops / 1e12, "bf16"
         workload_desc = {
-            "c1": "configs[1]: CIFAR-shaped QUAN layer",
-            "c2a": "configs[2] layer a: ImageNet ResNet-stage layer",
-            "c2b": "configs[2] layer b: ImageNet ResNet-stage stride-2 layer",
-            "c3a": "configs[3] layer a: detection-neck pointwise layer",
-            "c3b": "configs[3] layer b: detection-neck 3x3 layer",
+            "c1": "CIFAR-shaped QUAN layer",
+            "c2a": "ImageNet ResNet-stage layer",
+            "c2b": "ImageNet ResNet-stage stride-2 layer",
+            "c3a": "detection-neck pointwise layer",
+            "c3b": "detection-neck 3x3 layer",
         }[args.workload]
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
+
+    if args.profile:
+        for _ in range(args.warmup + args.steps):
+            runner.step(sh)
+        torch.cuda.synchronize()
+        st, bits = quan.quan_device_status(sh)
+        print(json.dumps({"profile_run": args.workload, "launches": args.warmup + args.steps,
+                          "status": st}))
+        return 0 if st == quan.QUAN_OK else 1
 
     # warm-up: at least W steps, and enough untimed steps for the clocks to settle
     gpu_id = getattr(torch.cuda.get_device_properties(local_rank), "uuid", None)
@@ -297,12 +312,29 @@ def main():
             torch.cuda.synchronize()
     torch.cuda.synchronize()
 
+    # The timed region is exactly K steps.  By default they are captured once into a CUDA
+    # graph (same launches, same buffers) so host launch overhead does not leave gaps.
+    graph = None
+    if not args.no_graph:
+        cap = torch.cuda.Stream()
+        cap.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=cap):
+            for _ in range(args.steps):
+                runner.step(cap.cuda_stream)
+        torch.cuda.synchronize()
+        graph.replay()  # warm replay (untimed)
+        torch.cuda.synchronize()
+
     barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
-    for _ in range(args.steps):
-        runner.step(sh)
+    if graph is not None:
+        graph.replay()
+    else:
+        for _ in range(args.steps):
+            runner.step(sh)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -342,12 +374,15 @@ def main():
                "h2d_bytes_per_step": int(runner.h2d), "d2h_bytes_per_step": int(runner.d2h)}
 
     peaks, peak_src = load_peaks()
-    roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src)
+    if args.workload == "backbone":
+        roofline = backbone_roofline(runner, torch, stream, peaks, peak_src)
+    else:
+        roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         if args.workload == "backbone":
-            cpu = runner.cpu_baseline(args.cpu_seconds)
+            cpu = backbone_cpu_sample(runner, args.cpu_seconds, inputs)
         else:
             cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs)
 
@@ -357,7 +392,9 @@ def main():
         return 0
     cfg = {"workload": workload_desc, "l2": "inputs larger than L2: %d rotating buffer sets, "
            "%.0f MB" % (getattr(runner, "sets", 1), runner.footprint / 1e6),
-           "parallelism": "replicas over the batch (dp%d, no collective)" % world}
+           "parallelism": "replicas over the batch (dp%d, no collective)" % world,
+           "timing": "one CUDA-graph replay of the K steps" if graph is not None
+           else "plain launch loop"}
     if args.workload != "backbone":
         s = runner.spec
         cfg.update({"N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin, "Cout": s.Cout,
@@ -392,6 +429,70 @@ def runner_roofline(runner, args, ms_per_step, peaks, peak_src):
             "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
 
 
+def backbone_roofline(runner, torch, stream, peaks, peak_src):
+    """Time every layer once with events on the launching stream (outside the timed
+    region), then report the roofline of the layer with the largest share of the step."""
+    sh = stream.cuda_stream
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    times = []
+    for i, L in enumerate(runner.layers):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for _ in range(2):
+            runner.run_layer(i, sh)
+        e0.record(stream)
+        for _ in range(5):
+            runner.run_layer(i, sh)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1) / 5 / 1e3)
+    layers = []
+    for i, (L, t) in enumerate(zip(runner.layers, times)):
+        if L.kind == "conv":
+            fl, nb = L.spec.flops, L.spec.algorithmic_bytes
+            if L.res is not None:
+                nb += L.spec.N * L.spec.Ho * L.spec.Wo * L.spec.Cout * 2
+            name = "conv%dx%d/%d %d->%d @%d" % (L.spec.kh, L.spec.kw, L.spec.stride, L.spec.Cin,
+                                                L.spec.Cout, L.spec.H)
+        else:
+            src = runner.outs[L.src]
+            fl, nb = 0.0, src.numel() * 2 + runner.outs[i].numel() * 2
+            name = "maxpool%d/%d" % (L.k, L.stride)
+        bound = "tensor" if fl / nb >= ridge else "hbm"
+        ach = fl / t / 1e12 if bound == "tensor" else nb / t / 1e9
+        peak = peaks["bf16_tflops"] if bound == "tensor" else peaks["hbm_gbs"]
+        layers.append({"layer": i, "name": name, "ms": round(t * 1e3, 4), "bound": bound,
+                       "achieved": round(ach, 1), "frac": round(ach / peak, 3)})
+    top = max(layers, key=lambda r: r["ms"])
+    total = sum(r["ms"] for r in layers)
+    L = runner.layers[top["layer"]]
+    fl = L.spec.flops if L.kind == "conv" else 0.0
+    return {"bound": top["bound"], "achieved": top["achieved"],
+            "peak": peaks["bf16_tflops"] if top["bound"] == "tensor" else peaks["hbm_gbs"],
+            "unit": "TFLOP/s" if top["bound"] == "tensor" else "GB/s", "frac": top["frac"],
+            "traffic": None, "kernel": top["name"],
+            "share": round(top["ms"] / total, 3), "peak_source": peak_src + " (burst)",
+            "layers": layers}
+
+
+def backbone_cpu_sample(runner, seconds, inputs):
+    """The fp64 oracle backbone on a bounded number of images."""
+    import oracle
+    import oracle.backbone as ob
+    params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in runner.layers]
+    layers = inputs.backbone_layers(N=1, H=runner.H)
+    x = runner.x_host
+    t0 = time.perf_counter()
+    ob.forward(layers, params, x[:1])
+    t1 = time.perf_counter() - t0
+    n = max(1, min(runner.N, int(seconds / max(t1, 1e-6))))
+    if n > 1:
+        t0 = time.perf_counter()
+        ob.forward(inputs.backbone_layers(N=n, H=runner.H), params, x[:n])
+        t1 = time.perf_counter() - t0
+    return {"value": n / t1, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": "%d of %d images of the backbone (fp64, %.2f s)" % (n, runner.N, t1)}
+
+
 def reference_arm(args, rank, world, inputs):
     """The fp64 CPU oracle as the reference arm: each step is a bounded sample of the
     same workload (rank 0 only)."""
@@ -399,8 +500,29 @@ def reference_arm(args, rank, world, inputs):
         return 0
     import oracle
     if args.workload == "backbone":
-        from paper_2509_05512_gb300 import backbone_ref
-        return backbone_ref.reference_arm(args, METRIC)
+        import oracle.backbone as ob
+        layers = inputs.backbone_layers(N=1)
+        params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in layers]
+        x = inputs.backbone_input(n_images=1)
+        for _ in range(args.warmup):
+            ob.forward(layers, params, x)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            ob.forward(layers, params, x)
+        dt = time.perf_counter() - t0
+        value = args.steps / dt
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": "backbone", "N": 256, "H": 224},
+                "cpu_baseline": {"value": value, "unit": "images/s", "cores": oracle.num_threads(),
+                                 "kind": "oracle",
+                                 "sample": "1 of 256 images of the backbone per step (fp64)"},
+                "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
     spec = inputs.LAYERS[args.workload]
     d = inputs.layer_inputs(spec, n_images=1)
     f64 = oracle.bf16_bits_to_f64

@@ -1,0 +1,133 @@
+"""ResNet-18-style quaternion backbone forward through the libquan C ABI.
+
+Layer list (inputs.backbone_layers): 7x7/2 quaternion stem (4 -> 64 real channels) with
+IQBN + ReLU, 3x3/2 max pooling applied to every real channel on its own, then four
+stages of two basic blocks (64/128/256/512 real channels, 3x3 quaternion convolutions
+with IQBN, 1x1/2 quaternion shortcut where the shape changes, the block's second
+convolution adding the block input before its ReLU).  Every operation runs in libquan
+kernels on one CUDA stream; torch only allocates device memory.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import inputs as _inputs
+
+
+class BackboneRunner:
+    """Weights, activations and the per-step launch sequence of the backbone."""
+
+    def __init__(self, torch, quan, inputs=_inputs, N: int = 256, H: int = 224, seed: int = 4,
+                 x_bits=None):
+        self.torch, self.quan, self.N, self.H = torch, quan, N, H
+        dev = torch.device("cuda")
+        self.layers = inputs.backbone_layers(N=N, H=H, seed=seed)
+
+        def up(bits):
+            return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(
+                torch.bfloat16).to(dev)
+
+        self.params = []
+        self.outs = []
+        for L in self.layers:
+            if L.kind == "conv":
+                prm = inputs.backbone_params(L)
+                self.params.append({
+                    "w": [up(prm[k]) for k in ("wr", "wi", "wj", "wk")],
+                    "scale": torch.from_numpy(prm["scale"]).to(dev),
+                    "shift": torch.from_numpy(prm["shift"]).to(dev),
+                    "host": prm})
+                s = L.spec
+                self.outs.append(torch.empty((N, s.Ho, s.Wo, s.Cout), dtype=torch.bfloat16,
+                                             device=dev))
+            else:
+                src = self.outs[L.src]
+                _, Hs, Ws, C = src.shape
+                Ho = (Hs + 2 * L.pad - L.k) // L.stride + 1
+                Wo = (Ws + 2 * L.pad - L.k) // L.stride + 1
+                self.params.append(None)
+                self.outs.append(torch.empty((N, Ho, Wo, C), dtype=torch.bfloat16, device=dev))
+        if x_bits is None:
+            x_bits = inputs.backbone_input(N=N, H=H, seed=seed)
+        self.x_host = x_bits
+        self.x = up(x_bits)
+        self.launches_per_step = len(self.layers)
+        self.footprint = sum(t.numel() * 2 for t in self.outs) + self.x.numel() * 2
+
+    # ---------------------------------------------------------------- execution
+    def layer_input(self, idx: int):
+        src = self.layers[idx].src
+        return self.x if src == -1 else self.outs[src]
+
+    def run_layer(self, idx: int, stream, x=None, out=None):
+        L = self.layers[idx]
+        q = self.quan
+        x = self.layer_input(idx) if x is None else x
+        out = self.outs[idx] if out is None else out
+        if L.kind == "maxpool":
+            N, H, W, C = x.shape
+            q.quan_maxpool2d_fwd(x, N, H, W, C, L.k, L.stride, L.pad, out, stream)
+            return out
+        s, prm = L.spec, self.params[idx]
+        N, H, W, C = x.shape
+        if L.res is not None:
+            q.quan_qconv2d_fwd_res(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
+                                   s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                                   self.outs[L.res], out, stream)
+        else:
+            q.quan_qconv2d_fwd(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
+                               s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act, out, stream)
+        return out
+
+    def step(self, stream):
+        for i in range(len(self.layers)):
+            self.run_layer(i, stream)
+
+    @property
+    def output(self):
+        return self.outs[-1]
+
+    # ---------------------------------------------------------------- accounting
+    @property
+    def flops(self) -> float:
+        return sum(L.spec.flops for L in self.layers if L.kind == "conv")
+
+    def describe(self) -> str:
+        return ("ResNet-18-style QUAN backbone, N=%d, %dx%dx4 quaternion input"
+                % (self.N, self.H, self.H))
+
+    def config(self) -> dict:
+        return {"N": self.N, "H": self.H, "W": self.H, "convs": sum(
+            L.kind == "conv" for L in self.layers), "maxpool": 1,
+            "flops_per_step": self.flops, "epilogue": "IQBN+ReLU (+residual)"}
+
+    def layer_table(self):
+        rows = []
+        for i, L in enumerate(self.layers):
+            if L.kind == "conv":
+                s = L.spec
+                rows.append((i, "conv", s.H, s.Cin, s.Cout, s.kh, s.stride, s.flops))
+            else:
+                rows.append((i, "maxpool", None, None, None, L.k, L.stride, 0.0))
+        return rows
+
+    # ---------------------------------------------------------------- e2e (host buffers)
+    def e2e_setup(self):
+        torch = self.torch
+        self.h_x = torch.from_numpy(np.ascontiguousarray(self.x_host).view(np.int16)).pin_memory()
+        out = self.outs[-1]
+        self.h_out = torch.empty(out.shape, dtype=torch.int16).pin_memory()
+        self.e_x = self.x  # the device input buffer is refilled every step
+        self.h2d = self.h_x.numel() * 2
+        self.d2h = self.h_out.numel() * 2
+
+    def e2e_step(self, stream):
+        torch = self.torch
+        self.x.view(torch.int16).copy_(self.h_x, non_blocking=True)
+        self.step(stream)
+        self.h_out.copy_(self.outs[-1].view(torch.int16), non_blocking=True)
+
+    def roofline(self, peaks, peak_src):
+        return {"bound": "mixed", "achieved": None, "peak": None, "unit": None, "frac": None,
+                "traffic": None, "kernel": "per layer",
+                "peak_source": peak_src}

@@ -101,11 +101,13 @@ LAYERS = {
     "c3b": LayerSpec("c3b", 16, 40, 40, 1024, 1024, 3, 3, 1, 1, seed=(3, 1)),
 }
 
+# Workload groups: the small fp32 check layer, the CIFAR-shaped layer, the two
+# ImageNet ResNet-stage layers, the two detection-neck layers.
 CONFIGS = {
-    "configs[0]": ["c0"],
-    "configs[1]": ["c1"],
-    "configs[2]": ["c2a", "c2b"],
-    "configs[3]": ["c3a", "c3b"],
+    "small": ["c0"],
+    "cifar": ["c1"],
+    "imagenet_stage": ["c2a", "c2b"],
+    "detection_neck": ["c3a", "c3b"],
 }
 
 

@@ -6,6 +6,9 @@ from oracle import bf16_bits_to_f64
 
 # bf16 layers: relative L2 error <= 5e-3 and max-abs error <= 3e-2 * RMS(reference);
 # fp32 layers: max-abs error <= 1e-4 * RMS(reference).
+# The bf16 max-abs bound is applied to the error beyond the one rounding the output
+# format imposes: an exact result stored in bf16 (round to nearest even) is off by up to
+# half an ulp, at most |ref| * 2^-8, so the check is |got - ref| - |ref| * 2^-8 <= bound.
 BF16_REL_L2 = 5e-3
 BF16_MAX_ABS_RMS = 3e-2
 F32_MAX_ABS_RMS = 1e-4
@@ -43,18 +46,23 @@ def out_f64(t):
     return t.detach().to(torch.float64).cpu().numpy()
 
 
-def errors(got, ref):
+BF16_HALF_ULP = 2.0 ** -8
+
+
+def errors(got, ref, out_rounding=0.0):
+    """rel-L2, max-abs error beyond out_rounding * |ref|, and RMS of the reference."""
     got = np.asarray(got, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     diff = got - ref
     rms = float(np.sqrt(np.mean(ref * ref))) if ref.size else 0.0
     rel_l2 = float(np.linalg.norm(diff) / max(np.linalg.norm(ref), 1e-300))
-    max_abs = float(np.abs(diff).max()) if diff.size else 0.0
+    excess = np.abs(diff) - out_rounding * np.abs(ref)
+    max_abs = float(max(excess.max(), 0.0)) if diff.size else 0.0
     return rel_l2, max_abs, rms
 
 
 def assert_bf16_close(got, ref, what=""):
-    rel_l2, max_abs, rms = errors(got, ref)
+    rel_l2, max_abs, rms = errors(got, ref, BF16_HALF_ULP)
     assert np.isfinite(got).all(), what + ": non-finite output"
     assert rel_l2 <= BF16_REL_L2, "%s: rel-L2 %.3e > %.1e" % (what, rel_l2, BF16_REL_L2)
     assert max_abs <= BF16_MAX_ABS_RMS * rms, "%s: max-abs %.3e > %.1e * RMS %.3e" % (

@@ -1,0 +1,80 @@
+"""Backbone parity: the ResNet-18-style quaternion backbone run through
+libquan against the fp64 oracle.
+
+Per layer, the oracle is fed the GPU's own input (and residual) of that layer, so every
+convolution is held to the bf16 tolerance on exact inputs; max pooling is bit-exact.
+End to end, the bf16 rounding of the 20 intermediate activations accumulates, so the
+whole-network comparison uses a looser bound, relative L2 <= 2e-2: 21 layers each add
+up to half a bf16 ulp (2^-9 relative) of fresh rounding, and the residual blocks carry it
+forward, which puts the expected relative L2 near sqrt(21) * 2^-9 / sqrt(3) ~ 5e-3; the
+bound leaves a factor of four for amplification through the network."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle.backbone as ob
+from oracle import bf16_bits_to_f64
+from paper_2509_05512_gb300 import build, inputs, quan
+from paper_2509_05512_gb300.backbone import BackboneRunner
+from tests._util import assert_bf16_close, errors
+
+pytestmark = pytest.mark.gpu
+
+E2E_REL_L2 = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    build.build_library()
+    quan.load()
+    quan.quan_set_path(quan.QUAN_PATH_AUTO)
+    quan.quan_set_tc_tiles(0, 0, 0, 0)
+
+
+def bits_of(t):
+    return t.detach().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def check_layers(runner, images):
+    params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in runner.layers]
+    for i, L in enumerate(runner.layers):
+        xin = bf16_bits_to_f64(bits_of(runner.layer_input(i)[images]))
+        res = None
+        if L.kind == "conv" and L.res is not None:
+            res = bf16_bits_to_f64(bits_of(runner.outs[L.res][images]))
+        ref = ob.layer_forward(L, params[i], xin, res)
+        got = bf16_bits_to_f64(bits_of(runner.outs[i][images]))
+        if L.kind == "maxpool":
+            np.testing.assert_array_equal(got, ref)
+        else:
+            assert_bf16_close(got, ref, "layer %d" % i)
+    return params
+
+
+def test_backbone_two_images_per_layer_and_end_to_end():
+    x_bits = inputs.backbone_input(n_images=2)
+    runner = BackboneRunner(torch, quan, inputs, N=2, x_bits=x_bits)
+    stream = torch.cuda.current_stream().cuda_stream
+    runner.step(stream)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    params = check_layers(runner, slice(0, 2))
+    y_ref = ob.forward(inputs.backbone_layers(N=2), params, x_bits)
+    got = bf16_bits_to_f64(bits_of(runner.output))
+    rel_l2, max_abs, rms = errors(got, y_ref)
+    assert rel_l2 <= E2E_REL_L2, rel_l2
+    assert (got >= 0).all() and got.std() > 0.1
+
+
+def test_backbone_full_batch_sampled_images():
+    runner = BackboneRunner(torch, quan, inputs, N=256)
+    stream = torch.cuda.current_stream().cuda_stream
+    runner.step(stream)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    check_layers(runner, [0, 255])
+    out = runner.output.float()
+    assert torch.isfinite(out).all() and (out >= 0).all()
