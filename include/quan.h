@@ -74,8 +74,11 @@ typedef enum {
  *   kh,kw        filter size >= 1; stride >= 1; pad >= 0; Ho, Wo >= 1
  *   act          quan_act_t
  *   out          bf16 [N][Ho][Wo][Cout]        (device), rounded to nearest even
- * The tensor-core path needs Cin/4 and Cout/4 to be multiples of 16 and 16-byte aligned
- * tensor pointers; other shapes run on CUDA cores.  Returns QUAN_OK once launched.
+ * The tensor-core path needs 16-byte aligned tensor pointers, fewer than 2^31 output
+ * pixels and either Cin/4 and Cout/4 multiples of 16, or Cin = 4, Cout = 64, stride 2
+ * and an even W (the 4-channel stem; at most 32 16-byte K units, i.e.
+ * kh * ceil((kw + pad mod 2) / 2) <= 32); other shapes run on CUDA cores.  Returns
+ * QUAN_OK once launched.
  */
 quan_status_t quan_qconv2d_fwd(const void* x, const void* wr, const void* wi, const void* wj,
                                const void* wk, const float* bias, const float* iqbn_scale,
@@ -121,7 +124,9 @@ int quan_last_path(void);
  * (16, 32 or 64), max_ctas = persistent grid size cap, mode = MMA decomposition
  * (1: one MMA per output/input component pair, N = bnq; 2: output components paired,
  * N = 2 bnq; 3: weight-stationary, the whole signed block weight expanded once per CTA
- * in shared memory, only for Cin = Cout = 64 and at most 9 taps).  Values that do not
+ * in shared memory, only for Cin = Cout = 64 and at most 9 taps; 4: pixel-pair gather,
+ * weight-stationary with the pixel tile built from 16-byte pairs of adjacent input
+ * pixels, only for the Cin = 4 stem shapes above; mode 0 picks it for those).  Values that do not
  * divide the layer, or a tile that does not fit in shared memory, make the call fail
  * with QUAN_ERR_UNSUPPORTED.
  */

@@ -25,6 +25,9 @@
 //              weight-stationary: every CTA expands the whole signed block weight once
 //              into shared memory and streams only pixels; N = 64 MMAs cover all four
 //              output components.
+//   gather     (1 -> 16 quaternion channels, stride 2: the 4-channel stem;
+//              qconv_gather.cuh) weight-stationary like MODE_WS, with the A tile built by
+//              16-byte cp.async copies of horizontal pixel pairs instead of TMA.
 //
 // Structure of the QUAD/PAIR kernel (one persistent CTA per SM, 12 warps):
 //   warps 0, 3  TMA producers: per K block (tap, chunk of KAPPA quaternion input channels)
@@ -399,6 +402,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 #include "qconv_ws.cuh"
+#include "qconv_gather.cuh"
 
 // ---------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
@@ -701,12 +705,64 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     return cudaGetLastError();
 }
 
+cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
+                          const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
+                          cudaStream_t stream, char* err, size_t errlen) {
+    GatherParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    prm.x = static_cast<const __nv_bfloat16*>(x);
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.lead = s.pad & 1;
+    prm.nsp = (s.kw + prm.lead + 1) / 2;
+    const int real_units = s.kh * prm.nsp;
+    prm.units = real_units + (real_units & 1);
+    prm.ksteps = prm.units / 2;
+    prm.W2 = s.W / 2;
+    prm.stage_bytes = BM * prm.units * 16;
+    int stages = GaCfg::RING_BYTES / prm.stage_bytes;
+    if (stages > MAX_STAGES) stages = MAX_STAGES;
+    if (stages < 2 || prm.units > GA_MAX_UNITS) {
+        snprintf(err, errlen, "pixel-pair gather: %d K units do not fit", prm.units);
+        return cudaErrorInvalidValue;
+    }
+    prm.stages = stages;
+    const long long tiles = (s.M + BM - 1) / BM;
+    if (tiles > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many tiles");
+        return cudaErrorInvalidValue;
+    }
+    prm.num_tiles = static_cast<int>(tiles);
+
+    const MapKey key = make_key(s, x, w, out, 1, 16, 4);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        // one store box covers the whole 64-channel output row (wide epilogue)
+        if (!encode_y_2d(&maps[0], s, out, 64)) {
+            snprintf(err, errlen, "tensor-map encode failed for the output tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    const int grid = grid_for(opt, num_sms, prm.num_tiles);
+    static std::atomic<unsigned long long> done{0};
+    cudaError_t e = set_smem_once(qconv_gather_kernel, GaCfg::SMEM_BYTES, done);
+    if (e != cudaSuccess) return e;
+    qconv_gather_kernel<<<grid, GA_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
                   const void* residual) {
     auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
-    if (s.Qin % 16 != 0 || s.Qout % 16 != 0) return false;
+    if ((s.Qin % 16 != 0 || s.Qout % 16 != 0) && !gather_ok(s)) return false;
+    // TMA coordinates of the output (pixel index) are 32-bit
+    if (s.M > 0x7fffffffLL) return false;
     if (!al16(x) || !al16(out) || !al16(w[0]) || !al16(w[1]) || !al16(w[2]) || !al16(w[3]))
         return false;
     if (residual && !al16(residual)) return false;
@@ -724,6 +780,14 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     if (!load_encoders()) {
         snprintf(err, errlen, "tensor-map encoders unavailable from the CUDA driver");
         return cudaErrorNotSupported;
+    }
+    if (gather_ok(s) && (opt.mode == 0 || opt.mode == 4))
+        return launch_gather(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+    if (opt.mode == 4) {
+        snprintf(err, errlen,
+                 "pixel-pair gather mode needs Cin = 4, Cout = 64, stride 2, even W and at "
+                 "most %d K units", GA_MAX_UNITS);
+        return cudaErrorInvalidValue;
     }
     // Weight-stationary for 16 -> 16 quaternion channels (the whole expanded weight fits);
     // pair mode (N = 2 BNQ per MMA) otherwise, unless the tile is so narrow that even

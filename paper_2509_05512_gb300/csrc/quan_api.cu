@@ -138,8 +138,9 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
     if (path == QUAN_PATH_TC) {
         if (!tc_ok)
             return fail(QUAN_ERR_UNSUPPORTED,
-                        "tensor-core path needs sm_103, Cin/4 and Cout/4 multiples of 16 and "
-                        "16-byte aligned tensors (device cc %d, Cin=%d, Cout=%d)",
+                        "tensor-core path needs sm_103, Cin/4 and Cout/4 multiples of 16 (or "
+                        "Cin = 4, Cout = 64, stride 2, even W) and 16-byte aligned tensors "
+                        "(device cc %d, Cin=%d, Cout=%d)",
                         cc, Cin, Cout);
         use_tc = true;
     } else if (path == QUAN_PATH_SIMT) {
@@ -247,9 +248,9 @@ int quan_last_path(void) { return t_last_path; }
 
 quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };
-    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 3)
+    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 4)
         return fail(QUAN_ERR_INVALID_ARG,
-                    "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 3");
+                    "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 4");
     g_kappa.store(kappa);
     g_bnq.store(bnq);
     g_max_ctas.store(max_ctas);

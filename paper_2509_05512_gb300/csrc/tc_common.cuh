@@ -122,12 +122,13 @@ struct EpiTile {
 };
 
 // Shared-memory resources of the epilogue: two staging blocks of 128 x BNQ bf16 (one per
-// half; with WIDE, two blocks of 128 x 4 BNQ, one per tile parity) and the per-channel
-// vectors [3][4 BNQ].
-template <int BNQ, bool WIDE = false>
+// half; with WIDE, WBUFS blocks of 128 x 4 BNQ, one per tile parity when WBUFS = 2) and
+// the per-channel vectors [3][4 BNQ].
+template <int BNQ, bool WIDE = false, int WBUFS = 2>
 struct EpiSmem {
+    static_assert(WBUFS == 1 || WBUFS == 2, "one or two wide staging blocks");
     static constexpr int OUT_TILE = BM * BNQ * 2;
-    static constexpr int STAGING_BYTES = WIDE ? 2 * 4 * OUT_TILE : 2 * OUT_TILE;
+    static constexpr int STAGING_BYTES = WIDE ? WBUFS * 4 * OUT_TILE : 2 * OUT_TILE;
     static constexpr int PARAM_BYTES = 3 * 4 * BNQ * 4;
     static constexpr uint32_t OUT_ROW = BNQ * 2;
     static constexpr uint32_t OUT_SW_MASK = BNQ == 64 ? 7u : (BNQ == 32 ? 3u : 1u);
@@ -139,18 +140,19 @@ struct EpiSmem {
 // inference form of Eq. 11-12), round to bf16, write a swizzled shared-memory block per
 // component and store it with TMA (rows outside the tensor are clipped by the map).
 // With WIDE (4 BNQ = 64 channels = the whole output row, BNQ == Qout) all four
-// components go into one 128-byte-row block and a single TMA store per tile, the block
-// alternating between two buffers so the store overlaps the next tile.
+// components go into one 128-byte-row block and a single TMA store per tile; with
+// WBUFS = 2 the block alternates between two buffers so the store overlaps the next
+// tile, with WBUFS = 1 the next tile waits until the store has read the block.
 // Accumulator buffer b of a tile lives at TMEM columns [4 BNQ b, 4 BNQ (b+1)), component
 // q at offset q BNQ.
-template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false>
+template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false, int WBUFS = 2>
 __device__ __forceinline__ void epilogue_role(const ConvShape& s, const EpilogueArgs& ep,
                                               const CUtensorMap* tmap_y, uint32_t tmem_base,
                                               uint8_t* staging, float* prm_s,
                                               uint32_t accf0, uint32_t acce0, int num_tiles,
                                               uint64_t limit, volatile int* abort_flag,
                                               Geo geo) {
-    using E = EpiSmem<BNQ, WIDE>;
+    using E = EpiSmem<BNQ, WIDE, WBUFS>;
     static_assert(!WIDE || BNQ == 16, "wide stores need 64-channel rows");
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
@@ -194,10 +196,10 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                static_cast<uint32_t>(buf * 4 * BNQ);
         if constexpr (WIDE) {
-            // block of this tile parity; free once the store of two tiles ago has read it
-            stg = staging + buf * 4 * E::OUT_TILE;
+            // block of this tile parity; free once the store of WBUFS tiles ago has read it
+            stg = staging + (WBUFS == 2 ? buf : 0) * 4 * E::OUT_TILE;
             stg_addr = smem_u32(stg);
-            if (threadIdx.x == EPI_WARP0 * 32) bulk_wait_group_read<1>();
+            if (threadIdx.x == EPI_WARP0 * 32) bulk_wait_group_read<WBUFS - 1>();
             named_bar_sync(1, 256);
         }
 #pragma unroll

@@ -187,6 +187,44 @@ def test_tc_few_ctas_many_tiles():
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
+# ------------------------------------------------------------------ pixel-pair gather (Cin = 4)
+
+GATHER_CASES = [
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra
+    ("stem_7x7", 2, 32, 32, 4, 64, 7, 2, 3, {}),             # 512 pixels, 4 whole tiles
+    ("stem_ragged", 2, 22, 22, 4, 64, 7, 2, 3, {}),          # 242 pixels, ragged tail
+    ("stem_rect_res", 3, 19, 30, 4, 64, 7, 2, 3,             # odd H, residual, SiLU
+     {"residual": True, "act": quan.QUAN_ACT_SILU}),
+    ("even_pad_5x5", 2, 18, 16, 4, 64, 5, 2, 2, {"bias": True}),  # 15 units + 1 zero unit
+    ("k3_pad1", 2, 20, 14, 4, 64, 3, 2, 1, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
+    ("k4x2_valid", 1, 17, 12, 4, 64, 4, 2, 0, {"kw": 2}),     # one pair per filter row
+    ("tiny", 1, 2, 2, 4, 64, 7, 2, 3, {}),                   # a single output pixel
+]
+
+
+@pytest.mark.parametrize("case", GATHER_CASES, ids=[c[0] for c in GATHER_CASES])
+def test_tc_pixel_pair_gather_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(206, len(name)), **extra)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+def test_tc_pixel_pair_gather_few_ctas():
+    # 32 tiles on 3 CTAs: every CTA wraps the stage ring and both accumulators many times
+    spec = inputs.small_layer("gather_few", 4, 64, 64, 4, 64, 7, 2, 3, seed=(207, 0))
+    quan.quan_set_tc_tiles(0, 0, 3, 4)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+def test_tc_pixel_pair_gather_mode_rejects_other_shapes():
+    spec = inputs.small_layer("not_stem", 1, 8, 8, 64, 64, 3, 1, 1, seed=(208, 0))
+    d = inputs.layer_inputs(spec)
+    quan.quan_set_tc_tiles(0, 0, 0, 4)
+    with pytest.raises(quan.QuanError) as ei:
+        run_gpu(d, path=quan.QUAN_PATH_TC)
+    assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+
+
 def test_tc_nonsquare_kernel():
     spec = inputs.small_layer("k3x1", 2, 9, 10, 64, 64, 3, 1, 1, kw=1, seed=(203, 0))
     # pad 1 on both sides with kw = 1 widens the output; valid for the oracle too
@@ -334,10 +372,13 @@ def test_maxpool(shape):
 
 # ------------------------------------------------------------------ failure detection
 
-@pytest.mark.parametrize("mode", [2, 3])
+@pytest.mark.parametrize("mode", [2, 3, 4])
 def test_bounded_wait_timeout_every_kernel(mode):
-    # the failure-injection path of the pair-mode and weight-stationary kernels
-    spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
+    # the failure-injection path of the pair-mode, weight-stationary and gather kernels
+    if mode == 4:
+        spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
+    else:
+        spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
     d = inputs.layer_inputs(spec)
     x = to_dev(d["x"], "bf16")
     w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
@@ -345,12 +386,12 @@ def test_bounded_wait_timeout_every_kernel(mode):
     quan.quan_set_tc_tiles(0, 16 if mode == 2 else 0, 0, mode)
     quan.quan_set_wait_limit_ns(5_000_000)
     quan.quan_set_fault_injection(True)
-    quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act)
+    quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, act=spec.act)
     st, bits = quan.quan_device_status()
     assert st == quan.QUAN_ERR_DEVICE_TIMEOUT and bits != 0
     quan.quan_set_fault_injection(False)
     quan.quan_set_wait_limit_ns(0)
-    y = quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act)
+    y = quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, act=spec.act)
     torch.cuda.synchronize()
     assert quan.quan_device_status()[0] == quan.QUAN_OK
     d2 = dict(d); d2["scale"] = d2["shift"] = None
