@@ -245,6 +245,48 @@ def cpu_oracle_sample(spec, seconds, inputs):
 
 # ---------------------------------------------------------------------------- main
 
+WORKLOAD_DESC = {
+    "c1": "CIFAR-shaped QUAN layer",
+    "c2a": "ImageNet ResNet-stage layer",
+    "c2b": "ImageNet ResNet-stage stride-2 layer",
+    "c3a": "detection-neck pointwise layer",
+    "c3b": "detection-neck 3x3 layer",
+    "backbone": "ResNet-18-style QUAN backbone",
+}
+
+
+def workload_config(workload: str, inputs) -> dict:
+    """The workload part of the JSON line's config, shared by both arms."""
+    if workload == "backbone":
+        layers = inputs.backbone_layers()
+        convs = [L.spec for L in layers if L.kind == "conv"]
+        c0 = convs[0]
+        return {"workload": "%s, N=%d, %dx%dx4 quaternion input" % (
+                    WORKLOAD_DESC[workload], c0.N, c0.H, c0.W),
+                "N": c0.N, "H": c0.H, "W": c0.W, "convs": len(convs), "maxpool": 1,
+                "flops_per_step": sum(c.flops for c in convs),
+                "epilogue": "IQBN+ReLU (+residual)"}
+    s = inputs.LAYERS[workload]
+    return {"workload": WORKLOAD_DESC[workload], "N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin,
+            "Cout": s.Cout, "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
+            "epilogue": "IQBN+ReLU", "flops_per_step": s.flops}
+
+
+def max_over_ranks(ms: float, dist, torch, device: str) -> float:
+    """Slowest rank's time: every rank runs the same replica workload, the job ends when
+    the last one does.  No-op without a process group."""
+    if dist is None:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(units_per_step: float, steps: int, world: int, ms: float) -> float:
+    """Whole-job rate: every rank processes units_per_step per step (weak scaling)."""
+    return units_per_step * steps * world / (ms / 1e3)
+
+
 def main():
     args = parse_args()
     rank = int(os.environ.get("RANK", "0"))
@@ -275,18 +317,10 @@ def main():
         runner = backbone.BackboneRunner(torch, quan, inputs)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
-        workload_desc = runner.describe()
     else:
         spec = inputs.LAYERS[args.workload]
         runner = LayerRunner(spec, torch, quan, inputs)
         unit, per_step_units, dtype = "TFLOP/s", spec.flops / 1e12, "bf16"
-        workload_desc = {
-            "c1": "CIFAR-shaped QUAN layer",
-            "c2a": "ImageNet ResNet-stage layer",
-            "c2b": "ImageNet ResNet-stage stride-2 layer",
-            "c3a": "detection-neck pointwise layer",
-            "c3b": "detection-neck 3x3 layer",
-        }[args.workload]
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
 
@@ -311,6 +345,7 @@ def main():
         if n % 64 == 0:
             torch.cuda.synchronize()
     torch.cuda.synchronize()
+    kernel_name = quan.quan_last_kernel() if args.workload != "backbone" else None
 
     # The timed region is exactly K steps.  By default they are captured once into a CUDA
     # graph (same launches, same buffers) so host launch overhead does not leave gaps.
@@ -340,15 +375,12 @@ def main():
     barrier()
     ms = ev0.elapsed_time(ev1)
     clocks = sampler.stop() if sampler else None
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dist, torch, "cuda")
     st, bits = quan.quan_device_status(sh)
     if st != quan.QUAN_OK:
         raise RuntimeError("kernel reported a timeout (bits 0x%x)" % bits)
     ms_per_step = ms / args.steps
-    value = per_step_units * args.steps * world / (ms / 1e3)
+    value = job_throughput(per_step_units, args.steps, world, ms)
 
     # end to end through the public call with host buffers
     e2e = None
@@ -365,19 +397,15 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        ems = e0.elapsed_time(e1)
-        if dist is not None:
-            t = torch.tensor([ems], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": per_step_units * args.steps * world / (ems / 1e3), "unit": unit,
+        ems = max_over_ranks(e0.elapsed_time(e1), dist, torch, "cuda")
+        e2e = {"value": job_throughput(per_step_units, args.steps, world, ems), "unit": unit,
                "h2d_bytes_per_step": int(runner.h2d), "d2h_bytes_per_step": int(runner.d2h)}
 
     peaks, peak_src = load_peaks()
     if args.workload == "backbone":
         roofline = backbone_roofline(runner, torch, stream, peaks, peak_src)
     else:
-        roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src)
+        roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -390,19 +418,14 @@ def main():
         dist.destroy_process_group()
     if rank != 0:
         return 0
-    cfg = {"workload": workload_desc, "l2": "inputs larger than L2: %d rotating buffer sets, "
-           "%.0f MB" % (getattr(runner, "sets", 1), runner.footprint / 1e6),
-           "parallelism": "replicas over the batch (dp%d, no collective)" % world,
-           "timing": "one CUDA-graph replay of the K steps" if graph is not None
-           else "plain launch loop"}
+    cfg = workload_config(args.workload, inputs)
+    cfg.update({"l2": "inputs larger than L2: %d rotating buffer sets, %.0f MB" % (
+                    getattr(runner, "sets", 1), runner.footprint / 1e6),
+                "parallelism": "replicas over the batch (dp%d, no collective)" % world,
+                "timing": "one CUDA-graph replay of the K steps" if graph is not None
+                else "plain launch loop"})
     if args.workload != "backbone":
-        s = runner.spec
-        cfg.update({"N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin, "Cout": s.Cout,
-                    "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
-                    "epilogue": "IQBN+ReLU", "flops_per_step": s.flops,
-                    "path": {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")})
-    else:
-        cfg.update(runner.config())
+        cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     line = {"metric": METRIC, "value": round(value, 4), "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
@@ -413,9 +436,7 @@ def main():
     return 0
 
 
-def runner_roofline(runner, args, ms_per_step, peaks, peak_src):
-    if args.workload == "backbone":
-        return runner.roofline(peaks, peak_src)
+def runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name):
     flops, nbytes = runner.flops, runner.algorithmic_bytes
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     t = ms_per_step / 1e3  # one kernel launch per step
@@ -425,7 +446,7 @@ def runner_roofline(runner, args, ms_per_step, peaks, peak_src):
         achieved, peak, unit, bound = nbytes / t / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
     return {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
             "frac": round(achieved / peak, 4), "traffic": recorded_traffic(args.workload),
-            "kernel": "qconv_tc_kernel", "peak_source": peak_src + " (burst)",
+            "kernel": kernel_name, "peak_source": peak_src + " (burst)",
             "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
 
 
@@ -434,11 +455,12 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
     region), then report the roofline of the layer with the largest share of the step."""
     sh = stream.cuda_stream
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    times = []
+    times, kernels = [], []
     for i, L in enumerate(runner.layers):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         for _ in range(2):
             runner.run_layer(i, sh)
+        kernels.append(runner.quan.quan_last_kernel() if L.kind == "conv" else "maxpool_kernel")
         e0.record(stream)
         for _ in range(5):
             runner.run_layer(i, sh)
@@ -460,8 +482,8 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
         bound = "tensor" if fl / nb >= ridge else "hbm"
         ach = fl / t / 1e12 if bound == "tensor" else nb / t / 1e9
         peak = peaks["bf16_tflops"] if bound == "tensor" else peaks["hbm_gbs"]
-        layers.append({"layer": i, "name": name, "ms": round(t * 1e3, 4), "bound": bound,
-                       "achieved": round(ach, 1), "frac": round(ach / peak, 3)})
+        layers.append({"layer": i, "name": name, "kernel": kernels[i], "ms": round(t * 1e3, 4),
+                       "bound": bound, "achieved": round(ach, 1), "frac": round(ach / peak, 3)})
     top = max(layers, key=lambda r: r["ms"])
     total = sum(r["ms"] for r in layers)
     L = runner.layers[top["layer"]]
@@ -469,7 +491,7 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
     return {"bound": top["bound"], "achieved": top["achieved"],
             "peak": peaks["bf16_tflops"] if top["bound"] == "tensor" else peaks["hbm_gbs"],
             "unit": "TFLOP/s" if top["bound"] == "tensor" else "GB/s", "frac": top["frac"],
-            "traffic": None, "kernel": top["name"],
+            "traffic": None, "kernel": "%s (%s)" % (top["kernel"], top["name"]),
             "share": round(top["ms"] / total, 3), "peak_source": peak_src + " (burst)",
             "layers": layers}
 
@@ -499,6 +521,8 @@ def reference_arm(args, rank, world, inputs):
     if rank != 0:
         return 0
     import oracle
+    ref_cfg = workload_config(args.workload, inputs)
+    ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
     if args.workload == "backbone":
         import oracle.backbone as ob
         layers = inputs.backbone_layers(N=1)
@@ -515,7 +539,7 @@ def reference_arm(args, rank, world, inputs):
                 "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-                "config": {"workload": "backbone", "N": 256, "H": 224},
+                "config": ref_cfg,
                 "cpu_baseline": {"value": value, "unit": "images/s", "cores": oracle.num_threads(),
                                  "kind": "oracle",
                                  "sample": "1 of 256 images of the backbone per step (fp64)"},
@@ -547,8 +571,7 @@ def reference_arm(args, rank, world, inputs):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": args.workload, "N": spec.N, "H": spec.H, "W": spec.W,
-                       "Cin": spec.Cin, "Cout": spec.Cout},
+            "config": ref_cfg,
             "cpu_baseline": cpu,
             "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}

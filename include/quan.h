@@ -117,6 +117,10 @@ quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int 
 quan_status_t quan_set_path(int path);
 /* Path (quan_path_t, TC or SIMT) the last successful convolution call of this thread ran. */
 int quan_last_path(void);
+/* Name of the kernel (with its template variant) the last successful convolution call of
+ * this thread launched, e.g. "qconv_ws_kernel<halo>"; "" before the first call.  The
+ * string is owned by the library and stays valid until the thread's next call. */
+const char* quan_last_kernel(void);
 
 /*
  * Tensor-core tile override for later calls (0 = automatic): kappa = quaternion input

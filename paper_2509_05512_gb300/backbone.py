@@ -92,15 +92,6 @@ class BackboneRunner:
     def flops(self) -> float:
         return sum(L.spec.flops for L in self.layers if L.kind == "conv")
 
-    def describe(self) -> str:
-        return ("ResNet-18-style QUAN backbone, N=%d, %dx%dx4 quaternion input"
-                % (self.N, self.H, self.H))
-
-    def config(self) -> dict:
-        return {"N": self.N, "H": self.H, "W": self.H, "convs": sum(
-            L.kind == "conv" for L in self.layers), "maxpool": 1,
-            "flops_per_step": self.flops, "epilogue": "IQBN+ReLU (+residual)"}
-
     def layer_table(self):
         rows = []
         for i, L in enumerate(self.layers):
@@ -126,8 +117,3 @@ class BackboneRunner:
         self.x.view(torch.int16).copy_(self.h_x, non_blocking=True)
         self.step(stream)
         self.h_out.copy_(self.outs[-1].view(torch.int16), non_blocking=True)
-
-    def roofline(self, peaks, peak_src):
-        return {"bound": "mixed", "achieved": None, "peak": None, "unit": None, "frac": None,
-                "traffic": None, "kernel": "per layer",
-                "peak_source": peak_src}

@@ -49,6 +49,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                             const EpilogueArgs& ep, void* out, const TcOptions& opt,
                             int num_sms, cudaStream_t stream, char* err, size_t errlen);
 cudaError_t read_and_clear_status(unsigned* status, cudaStream_t stream);
+// Name of the tensor-core kernel the calling thread's last launch_qconv_tc used.
+const char* last_tc_kernel();
 
 // CUDA-core path, any shape; T = __nv_bfloat16 or float.
 cudaError_t launch_qconv_simt_bf16(const ConvShape& s, const void* x, const void* const w[4],

@@ -58,6 +58,12 @@ namespace {
 
 using namespace tc;
 
+thread_local char t_kernel_name[64] = "";
+
+void set_kernel_name(const char* fmt, int a = 0, int b = 0) {
+    snprintf(t_kernel_name, sizeof(t_kernel_name), fmt, a, b);
+}
+
 constexpr int MODE_QUAD = 0;
 constexpr int MODE_PAIR = 1;
 constexpr int MODE_WS = 2;
@@ -691,6 +697,7 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
     static std::atomic<unsigned long long> done_h{0}, done_t{0};
+    set_kernel_name(halo ? "qconv_ws_kernel<halo>" : "qconv_ws_kernel<im2col>");
     if (halo) {
         auto kern = qconv_ws_kernel<true>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
@@ -749,6 +756,7 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
     static std::atomic<unsigned long long> done{0};
+    set_kernel_name("qconv_gather_kernel");
     cudaError_t e = set_smem_once(qconv_gather_kernel, GaCfg::SMEM_BYTES, done);
     if (e != cudaSuccess) return e;
     qconv_gather_kernel<<<grid, GA_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
@@ -865,6 +873,9 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
+    set_kernel_name(mode == MODE_PAIR ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
+                                      : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
+                    kappa, bnq);
 
 #define QUAN_TC_CASE(K, B)                                                       \
     if (kappa == K && bnq == B)                                                  \
@@ -883,6 +894,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     snprintf(err, errlen, "no kernel instance for kappa=%d bnq=%d mode=%d", kappa, bnq, mode);
     return cudaErrorInvalidValue;
 }
+
+const char* last_tc_kernel() { return t_kernel_name; }
 
 cudaError_t read_and_clear_status(unsigned* status, cudaStream_t stream) {
     cudaError_t e = cudaMemcpyFromSymbolAsync(status, g_status, sizeof(unsigned), 0,

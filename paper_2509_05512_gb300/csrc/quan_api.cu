@@ -15,6 +15,7 @@ namespace {
 
 thread_local char t_errmsg[512] = "";
 thread_local int t_last_path = 0;
+thread_local const char* t_last_kernel = "";
 std::atomic<int> g_path{QUAN_PATH_AUTO};
 std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1};
 std::atomic<unsigned long long> g_wait_limit{2000000000ull};
@@ -164,10 +165,12 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
         if (e != cudaSuccess) return cuda_fail(e, "qconv_tc launch");
         t_last_path = QUAN_PATH_TC;
+        t_last_kernel = quan::last_tc_kernel();
     } else {
         e = quan::launch_qconv_simt_bf16(s, x, w, ep, out, cs);
         if (e != cudaSuccess) return cuda_fail(e, "qconv_simt launch");
         t_last_path = QUAN_PATH_SIMT;
+        t_last_kernel = "qconv_simt_kernel<bf16>";
     }
     return QUAN_OK;
 }
@@ -212,6 +215,7 @@ quan_status_t quan_qconv2d_fwd_f32(const float* x, const float* wr, const float*
                                                 reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "qconv_simt_f32 launch");
     t_last_path = QUAN_PATH_SIMT;
+    t_last_kernel = "qconv_simt_kernel<f32>";
     return QUAN_OK;
 }
 
@@ -245,6 +249,8 @@ quan_status_t quan_set_path(int path) {
 }
 
 int quan_last_path(void) { return t_last_path; }
+
+const char* quan_last_kernel(void) { return t_last_kernel; }
 
 quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };

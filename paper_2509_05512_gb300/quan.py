@@ -64,6 +64,8 @@ def load():
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
         lib.quan_set_path.argtypes = [_i]
         lib.quan_last_path.argtypes = []
+        lib.quan_last_kernel.argtypes = []
+        lib.quan_last_kernel.restype = ctypes.c_char_p
         lib.quan_set_tc_tiles.argtypes = [_i, _i, _i, _i]
         lib.quan_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
         lib.quan_set_tc_halo.argtypes = [_i]
@@ -142,6 +144,10 @@ def quan_set_path(path: int) -> None:
 
 def quan_last_path() -> int:
     return load().quan_last_path()
+
+
+def quan_last_kernel() -> str:
+    return load().quan_last_kernel().decode()
 
 
 def quan_set_tc_tiles(kappa: int = 0, bnq: int = 0, max_ctas: int = 0, mode: int = 0) -> None:

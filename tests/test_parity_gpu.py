@@ -123,6 +123,7 @@ def test_tc_weight_stationary_layers(case, halo):
     quan.quan_set_tc_tiles(0, 0, 0, 3)
     quan.quan_set_tc_halo(bool(halo))
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel().startswith("qconv_ws_kernel<")
 
 
 @pytest.mark.parametrize("halo", [1, 0])
@@ -168,6 +169,8 @@ def test_tc_tile_variants(kappa, bnq, mode):
     spec = inputs.small_layer("tiles", 2, 11, 13, 256, 256, 3, 1, 1, seed=(201, kappa + bnq))
     quan.quan_set_tc_tiles(kappa, bnq, 0, mode)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_tc_kernel<%s,kappa=%d,bnq=%d>" % (
+        "quad" if mode == 1 else "pair", kappa, bnq)
 
 
 @pytest.mark.parametrize("mode", [1, 2])
@@ -207,6 +210,7 @@ def test_tc_pixel_pair_gather_layers(case):
     name, N, H, W, Cin, Cout, k, s, p, extra = case
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(206, len(name)), **extra)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_gather_kernel"
 
 
 def test_tc_pixel_pair_gather_few_ctas():
