@@ -76,9 +76,9 @@ typedef enum {
  *   out          bf16 [N][Ho][Wo][Cout]        (device), rounded to nearest even
  * The tensor-core path needs 16-byte aligned tensor pointers, fewer than 2^31 output
  * pixels and either Cin/4 and Cout/4 multiples of 16, or Cin = 4, Cout = 64, stride 2
- * and an even W (the 4-channel stem; at most 32 16-byte K units, i.e.
- * kh * ceil((kw + pad mod 2) / 2) <= 32); other shapes run on CUDA cores.  Returns
- * QUAN_OK once launched.
+ * and an even W (the 4-channel stem: kh * P <= 32, where P = ceil((kw + pad mod 2) / 2)
+ * rounded up to even is the number of 2-pixel pairs a filter row spans); other shapes
+ * run on CUDA cores.  Returns QUAN_OK once launched.
  */
 quan_status_t quan_qconv2d_fwd(const void* x, const void* wr, const void* wi, const void* wj,
                                const void* wk, const float* bias, const float* iqbn_scale,
@@ -128,9 +128,10 @@ const char* quan_last_kernel(void);
  * (16, 32 or 64), max_ctas = persistent grid size cap, mode = MMA decomposition
  * (1: one MMA per output/input component pair, N = bnq; 2: output components paired,
  * N = 2 bnq; 3: weight-stationary, the whole signed block weight expanded once per CTA
- * in shared memory, only for Cin = Cout = 64 and at most 9 taps; 4: pixel-pair gather,
- * weight-stationary with the pixel tile built from 16-byte pairs of adjacent input
- * pixels, only for the Cin = 4 stem shapes above; mode 0 picks it for those).  Values that do not
+ * in shared memory, only for Cin = Cout = 64 and at most 9 taps; 4: pixel pairs,
+ * weight-stationary with the input loaded as 16-byte pairs of adjacent pixels, one TMA
+ * box per filter row, only for the Cin = 4 stem shapes above; mode 0 picks it for
+ * those).  Values that do not
  * divide the layer, or a tile that does not fit in shared memory, make the call fail
  * with QUAN_ERR_UNSUPPORTED.
  */

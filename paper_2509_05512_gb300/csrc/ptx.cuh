@@ -252,26 +252,6 @@ __device__ __forceinline__ void bulk_wait_group() {
     asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
 }
 
-// 16-byte global -> shared copy through L1 (non-bulk cp.async); the last 16 - src_bytes
-// bytes of the destination are zero-filled, so src_bytes = 0 writes 16 zero bytes and
-// reads nothing.
-__device__ __forceinline__ void cp_async_16_zfill(uint32_t dst, const void* src,
-                                                  uint32_t src_bytes) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
-                 "r"(src_bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void cp_async_commit() {
-    asm volatile("cp.async.commit_group;" ::: "memory");
-}
-
-// Wait until at most N committed cp.async groups of this thread are still in flight.
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }

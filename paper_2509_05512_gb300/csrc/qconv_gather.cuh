@@ -2,56 +2,64 @@
 // input channel (the 4-channel stem of the backbone), included by qconv_tc.cu inside its
 // anonymous namespace.
 //
-// With Q_in = 1 a pixel holds only 4 bf16 (8 bytes): too narrow for the tensor-map loads
-// of the other kernels (a TMA row must be a multiple of 16 bytes) and far too narrow for
-// a 16-wide K step per tap.  For stride-2 layers on inputs of even width, two horizontally
-// adjacent pixels form an aligned 16-byte "pixel pair" [x_{2s}: r i j k | x_{2s+1}: r i j k],
-// and the 7x7/2 filter window of an output pixel at column wo covers nsp = 4 consecutive
-// pairs per filter row, starting at pair wo - (pad + lead) / 2 (lead = pad mod 2 is a
-// filter column -1 whose weight is zero).  One 16-byte K unit is one (filter row, pair)
-// and a pixel's im2col row is kh x nsp units (28 for the 7x7 stem: K = 224, 14 MMA K steps).
+// With Q_in = 1 a pixel holds only 4 bf16 (8 bytes): too narrow for a 16-wide K step per
+// tap and for the pixel-tile maps of the other kernels.  For stride-2 layers on inputs of
+// even width, two horizontally adjacent pixels form an aligned 16-byte "pixel pair"
+// [x_{2s}: r i j k | x_{2s+1}: r i j k], and in pair coordinates the horizontal stride is
+// 1: output column wo reads pairs wo - shift + j, j = 0 .. nsp - 1, where
+// shift = (pad + lead) / 2, lead = pad mod 2 is a leading filter column -1 of zero weight,
+// and nsp (rounded up to even, 4 for the 7x7 stem) is the number of pairs per filter row.
 //
-//   warps 12..15  gather: one thread per pixel row of the 128-pixel tile issues its
-//                 units as 16-byte cp.async copies straight into the K-major 32-byte-
-//                 swizzled A tile (pairs outside the image are zero-filled by the copy),
-//                 through L1 so that the 4-7 fold reuse of input pairs between filter
-//                 taps and neighbouring pixels stays on chip; a stage is handed to the
-//                 MMA once the next one has been issued (one group of copies in flight
-//                 behind the one being completed).
-//   warp 1        TMEM owner and MMA issuer: 14 MMAs of M = 128, N = 64 per tile.
-//   warps 0, 2..11  expand the signed block weight of Eq. 6 once per CTA:
+// Tile = 128 consecutive output columns of one output row (one MMA of M = 128; columns
+// past the row end are computed and never stored).  For each filter row ky one tiled TMA
+// box holds the 128 + nsp - 1 pairs of input row 2 ho - pad + ky the tile reads, zero
+// filled outside the image.  The A operand of the K step (ky, pairs 2t, 2t + 1) is that
+// box read as a K-major, non-swizzled matrix whose row m starts at pair m + 2t: 16-byte
+// rows, 8-row groups 128 bytes apart (stride byte offset) and the second 8-element K half
+// one pair (16 bytes) further on (leading byte offset) -- the overlapping rows of an
+// im2col matrix come from the descriptor, so the pixels are read from global memory once
+// per filter row and never copied on chip.
+//
+//   warp 0        TMA producer: kh boxes per tile into a ring of stages.
+//   warp 1        TMEM owner and MMA issuer: kh * nsp / 2 MMAs of M = 128, N = 64 per
+//                 tile (14 for the stem, K = 224).
+//   warps 2..11   expand the signed block weight of Eq. 6 once per CTA:
 //                 B[(q, co)][(ky, pair, e, p)] = sign(q, p) W_{q xor p}[co][ky][2 pair - lead + e]
-//                 (zero outside the filter); then warps 4..11 run the wide epilogue.
+//                 (zero outside the filter), K-major with a 32-byte swizzle; then warps
+//                 4..11 run the wide epilogue (one 3-D TMA store per tile, clipped at the
+//                 end of the output row).
 // The zero-weight columns read real input pixels, which only matters for non-finite
 // inputs (0 * inf); finite inputs give exactly the convolution of Eq. 5.
 
 constexpr int GA_MAX_UNITS = 32;  // K <= 256
-constexpr int GA_THREADS = 512;
-constexpr int GA_GATHER_WARP0 = 12;
+constexpr int GA_TILE_W = 128;    // output columns per tile
 
 struct GatherParams {
     ConvShape s;
     EpilogueArgs ep;
-    const __nv_bfloat16* x;
     const __nv_bfloat16* w[4];  // letter tensors [16][kh][kw][1]
     unsigned long long wait_limit_ns;
     int inject_stall;
-    int nsp;          // pixel pairs per filter row
+    int nsp;          // pixel pairs per filter row (even)
     int lead;         // pad mod 2: zero-weight filter column before the first pair
-    int units;        // 16-byte K units per pixel row: kh * nsp rounded up to even
-    int ksteps;       // units / 2
-    int W2;           // W / 2 pairs per input row
-    int stage_bytes;  // BM rows x units x 16 bytes
+    int shift;        // (pad + lead) / 2: first pair of output column 0 is -shift
+    int boxw;         // pairs per box: GA_TILE_W + nsp - 1
+    int box_stride;   // bytes between the boxes of one stage (128-byte multiple)
+    int box_bytes;    // boxw * 16
+    int stage_bytes;
     int stages;
+    int segs;         // tiles per output row
     int num_tiles;
 };
 
 struct GaCfg {
-    static constexpr int CHUNK_A = BM * 32;  // one K step of the A tile: 128 rows x 32 bytes
     static constexpr int CHUNK_B = 64 * 32;  // one K step of the weight: 64 rows x 32 bytes
     static constexpr int B_BYTES = (GA_MAX_UNITS / 2) * CHUNK_B;
-    using E = EpiSmem<16, true, 1>;
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 6;  // full, empty, accf[2], acce[2], drain, bready
+    using E = EpiSmem<16, true, 2>;
+    // accumulator buffers in TMEM: enough that neither the MMAs' completion latency nor
+    // the epilogue's turnaround stalls the MMA issue
+    static constexpr int NACC = 4;
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + 2;  // full, empty, accf, acce, drain, bready
     static constexpr int TAIL_BYTES = B_BYTES + E::STAGING_BYTES + E::PARAM_BYTES +
                                       NUM_BARS * 8 + 16;
     static constexpr int SMEM_BYTES = 227 * 1024;
@@ -60,26 +68,42 @@ struct GaCfg {
     static constexpr int STAGING_OFF = B_OFF + B_BYTES;
     static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
     static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
-    static constexpr uint32_t DESC_HI = desc_hi(8 * 32, desc_layout(32));
-    static constexpr uint32_t TMEM_COLS = 128;  // 2 buffers x 64 columns
-    static constexpr int EXP_WARPS = 11;        // warps 0, 2..11
-    static constexpr int GATHER_WARPS = 4;
+    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
+    // A: K-major, no swizzle, 8-row groups 128 bytes apart (the leading byte offset of
+    // one pair, 16 bytes, is the low word's default); B: K-major rows of 32 bytes.
+    static constexpr uint32_t A_DESC_HI = desc_hi(8 * 16, 0);
+    static constexpr uint32_t B_DESC_HI = desc_hi(8 * 32, desc_layout(32));
+    static constexpr uint32_t TMEM_COLS = 64 * NACC;
+    static constexpr int EXP_WARPS = 10;        // warps 2..11
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "gather shared memory");
-    static_assert(GA_GATHER_WARP0 + GATHER_WARPS == GA_THREADS / 32, "warp roles");
 };
 
-// Shapes the pixel-pair gather covers: one quaternion input channel, 16 quaternion
-// output channels, stride 2, even input width, K within the weight region.
-bool gather_ok(const ConvShape& s) {
-    if (s.Qin != 1 || s.Qout != 16 || s.stride != 2 || (s.W & 1)) return false;
+// nsp of a shape: pairs covering lead + kw filter columns, rounded up to even.
+int gather_nsp(const ConvShape& s) {
     const int lead = s.pad & 1;
     const int nsp = (s.kw + lead + 1) / 2;
-    const long long units = static_cast<long long>(s.kh) * nsp;
-    return units + (units & 1) <= GA_MAX_UNITS;
+    return nsp + (nsp & 1);
 }
 
-__global__ void __launch_bounds__(GA_THREADS, 1)
-    qconv_gather_kernel(const __grid_constant__ CUtensorMap tmap_y, const GatherParams p) {
+// Shapes the pixel-pair kernel covers: one quaternion input channel, 16 quaternion output
+// channels, stride 2, even input width, K within the weight region.
+bool gather_ok(const ConvShape& s) {
+    if (s.Qin != 1 || s.Qout != 16 || s.stride != 2 || (s.W & 1)) return false;
+    return static_cast<long long>(s.kh) * gather_nsp(s) <= GA_MAX_UNITS;
+}
+
+// Bytes between the pair boxes of one stage for nsp pairs per filter row.
+__host__ __device__ constexpr int gather_box_stride(int nsp) {
+    return ((GA_TILE_W + nsp - 1) * 16 + 127) & ~127;
+}
+
+// KH, NSP > 0: the filter height and pairs per filter row known at compile time, so the
+// MMA issue loop is fully unrolled with constant descriptor offsets; 0 = from the
+// parameters at run time.
+template <int KH, int NSP>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    qconv_pairs_kernel(const __grid_constant__ CUtensorMap tmap_x,
+                       const __grid_constant__ CUtensorMap tmap_y, const GatherParams p) {
     using C = GaCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -92,9 +116,9 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (MAX_STAGES + s); };
     const uint32_t accf0 = bar0 + 8u * (2 * MAX_STAGES);
-    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + 2);
-    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 4);
-    const uint32_t bready_bar = bar0 + 8u * (2 * MAX_STAGES + 5);
+    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + C::NACC);
+    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
+    const uint32_t bready_bar = drain_bar + 8u;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
@@ -103,10 +127,10 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
-            mbar_init(full_bar(i), C::GATHER_WARPS);
+            mbar_init(full_bar(i), 1);
             mbar_init(empty_bar(i), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::NACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
             mbar_init(acce0 + 8u * b, 8 * 32);
         }
@@ -115,7 +139,10 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap_y);
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmap_x);
+        tma_prefetch_desc(&tmap_y);
+    }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
         tmem_relinquish();
@@ -125,80 +152,37 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (warp >= GA_GATHER_WARP0) {
-        // ------------------------------------------------------------ pixel-pair gather
-        const int m = (warp - GA_GATHER_WARP0) * 32 + lane;  // pixel row of the tile
-        const int hw = s.Ho * s.Wo;
-        const int s_shift = (s.pad + p.lead) / 2;
-        // byte offset of (row m, unit u) in a stage: K step u / 2, 16-byte half u % 2,
-        // 32-byte swizzle (the half flips on rows 4..7 of each 8-row group)
-        const uint32_t row_off = static_cast<uint32_t>(m) * 32;
-        const uint32_t sw = (static_cast<uint32_t>(m) >> 2) & 1u;
-        const uint8_t* xb = reinterpret_cast<const uint8_t*>(p.x);
-        int stage = 0, prev = -1;
-        uint32_t phase = 0;
-        bool aborted = false;
-        for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
-            // lane 0 waits for the stage and the warp follows it, so the warp stays
-            // converged for the __syncwarp of the hand-off even when the wait gives up
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t pol_x = l2_policy_evict_normal();
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
-            if (lane == 0)
-                ok = wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
-                                   STATUS_TIMEOUT_PRODUCER);
-            if (__shfl_sync(0xffffffffu, ok ? 1 : 0, 0) == 0) {
-                aborted = true;
-                break;
-            }
-            const long long pix = static_cast<long long>(tile) * BM + m;
-            const bool valid = pix < s.M;
-            int img = 0, ho = 0, wo = 0;
-            if (valid) {
-                img = static_cast<int>(pix / hw);
-                const int rem = static_cast<int>(pix - static_cast<long long>(img) * hw);
-                ho = rem / s.Wo;
-                wo = rem - ho * s.Wo;
-            }
-            const int iy0 = ho * 2 - s.pad;
-            const int s0 = wo - s_shift;
-            const uint32_t dst0 = sbase + stage * p.stage_bytes + row_off;
-            int u = 0;
-            for (int ky = 0; ky < s.kh; ++ky) {
-                const int iy = iy0 + ky;
-                const bool row_ok = valid && iy >= 0 && iy < s.H;
-                const long long rbase = (static_cast<long long>(img) * s.H + iy) * p.W2;
-                for (int j = 0; j < p.nsp; ++j, ++u) {
-                    const int sp = s0 + j;
-                    const bool ok = row_ok && sp >= 0 && sp < p.W2;
-                    const uint8_t* src = ok ? xb + (rbase + sp) * 16 : xb;
-                    const uint32_t dst = dst0 + (u >> 1) * C::CHUNK_A +
-                                         ((static_cast<uint32_t>(u & 1) ^ sw) << 4);
-                    cp_async_16_zfill(dst, src, ok ? 16u : 0u);
+            const uint32_t tx = static_cast<uint32_t>(s.kh * p.box_bytes);
+            for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
+                const int row = tile / p.segs, seg = tile - (tile / p.segs) * p.segs;
+                const int img = row / s.Ho, ho = row - (row / s.Ho) * s.Ho;
+                if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
+                                   STATUS_TIMEOUT_PRODUCER)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t fb = full_bar(stage);
+                mbar_arrive_expect_tx(fb, tx);
+                filled |= 1u << stage;
+                fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
+                const uint32_t dst = sbase + stage * p.stage_bytes;
+                const int x0 = seg * GA_TILE_W - p.shift, y0 = ho * 2 - s.pad;
+                for (int ky = 0; ky < s.kh; ++ky)
+                    tma_load_4d(dst + ky * p.box_stride, &tmap_x, fb, 0, x0, y0 + ky, img, pol_x);
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
-            for (; u < p.units; ++u) {
-                const uint32_t dst = dst0 + (u >> 1) * C::CHUNK_A +
-                                     ((static_cast<uint32_t>(u & 1) ^ sw) << 4);
-                cp_async_16_zfill(dst, xb, 0u);
-            }
-            cp_async_commit();
-            if (prev >= 0) {
-                // the previous stage's copies have landed: publish it to the tensor cores
-                cp_async_wait<1>();
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(full_bar(prev));
-            }
-            prev = stage;
-            if (++stage == STAGES) {
-                stage = 0;
-                phase ^= 1u;
-            }
-        }
-        cp_async_wait<0>();
-        if (prev >= 0 && !aborted) {
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(full_bar(prev));
+            if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -215,10 +199,11 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
             }
             tc_fence_after();
             const uint32_t b_lo0 = desc_lo(sbase + C::B_OFF);
+            const int half = p.nsp / 2;
             int local = 0;
             for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
-                const int buf = local & 1;
-                const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+                const int buf = local % C::NACC;
+                const uint32_t use = static_cast<uint32_t>(local / C::NACC) & 1u;
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA) ||
                     !wait_or_abort(full_bar(stage), phase, limit, abort_flag,
@@ -229,10 +214,26 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * 64);
                 const uint32_t a_lo0 = desc_lo(sbase + stage * p.stage_bytes);
-                for (int c = 0; c < p.ksteps; ++c)
-                    umma_f16_w(d, a_lo0 + ((c * C::CHUNK_A) >> 4), C::DESC_HI,
-                               b_lo0 + ((c * C::CHUNK_B) >> 4), C::DESC_HI, IDESC,
-                               c != 0 ? 1u : 0u);
+                if constexpr (KH > 0) {
+                    constexpr uint32_t BOX_LO = gather_box_stride(NSP) >> 4;
+#pragma unroll
+                    for (int ky = 0; ky < KH; ++ky)
+#pragma unroll
+                        for (int t = 0; t < NSP / 2; ++t) {
+                            const int c = ky * (NSP / 2) + t;
+                            umma_f16_w(d, a_lo0 + ky * BOX_LO + 2 * t, C::A_DESC_HI,
+                                       b_lo0 + ((c * C::CHUNK_B) >> 4), C::B_DESC_HI, IDESC,
+                                       c != 0 ? 1u : 0u);
+                        }
+                } else {
+                    const uint32_t box_lo = static_cast<uint32_t>(p.box_stride) >> 4;
+                    int c = 0;
+                    for (int ky = 0; ky < s.kh; ++ky)
+                        for (int t = 0; t < half; ++t, ++c)
+                            umma_f16_w(d, a_lo0 + ky * box_lo + 2 * t, C::A_DESC_HI,
+                                       b_lo0 + ((c * C::CHUNK_B) >> 4), C::B_DESC_HI, IDESC,
+                                       c != 0 ? 1u : 0u);
+                }
                 ++issued;
                 umma_commit(empty_bar(stage));
                 umma_commit(accf0 + 8u * buf);
@@ -254,21 +255,21 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
         }
     } else {
         // ------------------------------------------------------------ weight expansion
-        // warps 0, 2..11: one 16-byte K unit (filter row ky, pair j) of output row
+        // warps 2..11: one 16-byte K unit (filter row ky, pair j) of output row
         // n = (q, co) per item: 8 values, pixel e of the pair major, input component p minor.
-        const int et = warp == 0 ? lane : (warp - 1) * 32 + lane;  // 0 .. 351
+        const int et = (warp - 2) * 32 + lane;  // 0 .. 319
         constexpr int ET = C::EXP_WARPS * 32;
         const int taps = s.kh * s.kw;
-        const int real_units = s.kh * p.nsp;
-        for (int i = et; i < 64 * p.units; i += ET) {
-            const int n = i / p.units, u = i - (i / p.units) * p.units;
+        const int units = s.kh * p.nsp;
+        for (int i = et; i < 64 * units; i += ET) {
+            const int n = i / units, u = i - (i / units) * units;
             const int q = n >> 4, co = n & 15;
             const int ky = u / p.nsp, j = u - (u / p.nsp) * p.nsp;
             uint32_t packed[4];
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 const int kx = 2 * j - p.lead + e;
-                const bool in = u < real_units && kx >= 0 && kx < s.kw;
+                const bool in = kx >= 0 && kx < s.kw;
                 float v[4];
 #pragma unroll
                 for (int pc = 0; pc < 4; ++pc) {
@@ -283,9 +284,10 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
                 packed[2 * e] = pack_bf16x2(v[0], v[1]);
                 packed[2 * e + 1] = pack_bf16x2(v[2], v[3]);
             }
-            const uint32_t off = static_cast<uint32_t>(C::B_OFF + (u >> 1) * C::CHUNK_B + n * 32) +
-                                 ((static_cast<uint32_t>(u & 1) ^ ((static_cast<uint32_t>(n) >> 2) & 1u))
-                                  << 4);
+            // K step u / 2, 16-byte half u % 2 of the 32-byte row, 32-byte swizzle
+            const uint32_t off =
+                static_cast<uint32_t>(C::B_OFF + (u >> 1) * C::CHUNK_B + n * 32) +
+                ((static_cast<uint32_t>(u & 1) ^ ((static_cast<uint32_t>(n) >> 2) & 1u)) << 4);
             *reinterpret_cast<uint4*>(smem + off) =
                 make_uint4(packed[0], packed[1], packed[2], packed[3]);
         }
@@ -295,18 +297,19 @@ __global__ void __launch_bounds__(GA_THREADS, 1)
 
         if (warp >= EPI_WARP0) {
             // -------------------------------------------------------- epilogue
-            const long long M = s.M;
-            auto geo = [M](int tile) {
+            const int segs = p.segs, Wo = s.Wo;
+            auto geo = [segs, Wo](int tile) {
                 EpiTile g;
                 g.n_tile = 0;
-                g.m0 = static_cast<long long>(tile) * BM;
-                const long long left = M - g.m0;
-                g.rows = left < BM ? static_cast<int>(left) : BM;
-                g.sy = static_cast<int>(g.m0);
-                g.sz = 0;
+                const int row = tile / segs, seg = tile - (tile / segs) * segs;
+                g.m0 = static_cast<long long>(row) * Wo + seg * GA_TILE_W;
+                const int left = Wo - seg * GA_TILE_W;
+                g.rows = left < GA_TILE_W ? left : GA_TILE_W;
+                g.sy = seg * GA_TILE_W;
+                g.sz = row;
                 return g;
             };
-            epilogue_role<16, false, decltype(geo), true, 1>(
+            epilogue_role<16, true, decltype(geo), true, 2, C::NACC>(
                 s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
                 reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
                 abort_flag, geo);

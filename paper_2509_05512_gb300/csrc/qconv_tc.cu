@@ -25,9 +25,10 @@
 //              weight-stationary: every CTA expands the whole signed block weight once
 //              into shared memory and streams only pixels; N = 64 MMAs cover all four
 //              output components.
-//   gather     (1 -> 16 quaternion channels, stride 2: the 4-channel stem;
-//              qconv_gather.cuh) weight-stationary like MODE_WS, with the A tile built by
-//              16-byte cp.async copies of horizontal pixel pairs instead of TMA.
+//   pairs      (1 -> 16 quaternion channels, stride 2: the 4-channel stem;
+//              qconv_gather.cuh) weight-stationary like MODE_WS; pixels are loaded as
+//              16-byte horizontal pairs, one TMA box per filter row, and the filter taps
+//              are descriptor offsets into those boxes.
 //
 // Structure of the QUAD/PAIR kernel (one persistent CTA per SM, 12 warps):
 //   warps 0, 3  TMA producers: per K block (tap, chunk of KAPPA quaternion input channels)
@@ -99,6 +100,7 @@ struct Cfg {
     static constexpr int STAGING_OFF = TILES_BYTES;
     static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
     static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
+    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
     // full (pixels), full (letters), empty, ready (negated copies done), acc_full[2],
     // acc_empty[2], drain
     static constexpr int NUM_BARS = 4 * STAGES + 5;
@@ -238,7 +240,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
             }
-            if (!ok)
+            // after an abort anywhere in the CTA, let every copy still in flight land
+            // before the CTA can exit
+            if (!ok || *abort_flag)
                 drain_fills(role == 0 ? full_bar(0) : fullw_bar(0), STAGES, filled, fill_parity,
                             limit);
         }
@@ -477,6 +481,39 @@ bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int chan
     return r == CUDA_SUCCESS;
 }
 
+// Input of a 4-channel layer viewed as 16-byte pixel pairs: [N][H][W/2][8], boxes of
+// `boxw` pairs of one input row, no swizzle (dense 16-byte rows in shared memory).
+bool encode_x_pairs(CUtensorMap* map, const ConvShape& s, const void* x, int boxw) {
+    const cuuint64_t W2 = static_cast<cuuint64_t>(s.W / 2);
+    const cuuint64_t dims[4] = {8, W2, static_cast<cuuint64_t>(s.H),
+                                static_cast<cuuint64_t>(s.N)};
+    const cuuint64_t strides[3] = {16, 16 * W2, 16 * W2 * s.H};
+    const cuuint32_t box[4] = {8, static_cast<cuuint32_t>(boxw), 1, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = g_encode_tiled(
+        map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
+        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+// Output of a 64-channel layer viewed as [N*Ho][Wo][64], stored in boxes of up to
+// `cols` output columns of one row (128-byte rows, 128-byte swizzle); a box reaching past
+// the end of the row is clipped there.
+bool encode_y_rows(CUtensorMap* map, const ConvShape& s, const void* y, int cols) {
+    const cuuint64_t dims[3] = {64, static_cast<cuuint64_t>(s.Wo),
+                                static_cast<cuuint64_t>(s.N) * s.Ho};
+    const cuuint64_t strides[2] = {128, 128 * static_cast<cuuint64_t>(s.Wo)};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(cols), 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
+                                      const_cast<void*>(y), dims, strides, box, estr,
+                                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                      CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 bool encode_w(CUtensorMap* map, const ConvShape& s, const void* w, int kappa, int bnq) {
     const cuuint64_t kw_cols = static_cast<cuuint64_t>(s.kh) * s.kw * s.Qin;
     const cuuint64_t dims[2] = {kw_cols, static_cast<cuuint64_t>(s.Qout)};
@@ -696,15 +733,20 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    static std::atomic<unsigned long long> done_h{0}, done_t{0};
+    static std::atomic<unsigned long long> done_h3{0}, done_h{0}, done_t{0};
     set_kernel_name(halo ? "qconv_ws_kernel<halo>" : "qconv_ws_kernel<im2col>");
-    if (halo) {
-        auto kern = qconv_ws_kernel<true>;
+    if (halo && s.kh == 3) {
+        auto kern = qconv_ws_kernel<true, 3>;
+        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h3);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+    } else if (halo) {
+        auto kern = qconv_ws_kernel<true, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
         if (e != cudaSuccess) return e;
         kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
     } else {
-        auto kern = qconv_ws_kernel<false>;
+        auto kern = qconv_ws_kernel<false, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
         if (e != cudaSuccess) return e;
         kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
@@ -718,48 +760,60 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     GatherParams prm;
     prm.s = s;
     prm.ep = ep;
-    prm.x = static_cast<const __nv_bfloat16*>(x);
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     prm.lead = s.pad & 1;
-    prm.nsp = (s.kw + prm.lead + 1) / 2;
-    const int real_units = s.kh * prm.nsp;
-    prm.units = real_units + (real_units & 1);
-    prm.ksteps = prm.units / 2;
-    prm.W2 = s.W / 2;
-    prm.stage_bytes = BM * prm.units * 16;
+    prm.nsp = gather_nsp(s);
+    prm.shift = (s.pad + prm.lead) / 2;
+    prm.boxw = GA_TILE_W + prm.nsp - 1;
+    prm.box_bytes = prm.boxw * 16;
+    prm.box_stride = gather_box_stride(prm.nsp);
+    prm.stage_bytes = (s.kh * prm.box_stride + 1023) & ~1023;
     int stages = GaCfg::RING_BYTES / prm.stage_bytes;
     if (stages > MAX_STAGES) stages = MAX_STAGES;
-    if (stages < 2 || prm.units > GA_MAX_UNITS) {
-        snprintf(err, errlen, "pixel-pair gather: %d K units do not fit", prm.units);
+    if (stages < 2 || s.kh * prm.nsp > GA_MAX_UNITS || prm.boxw > 256) {
+        snprintf(err, errlen, "pixel-pair kernel: kh=%d kw=%d does not fit", s.kh, s.kw);
         return cudaErrorInvalidValue;
     }
     prm.stages = stages;
-    const long long tiles = (s.M + BM - 1) / BM;
+    prm.segs = (s.Wo + GA_TILE_W - 1) / GA_TILE_W;
+    const long long rows = static_cast<long long>(s.N) * s.Ho;
+    const long long tiles = rows * prm.segs;
     if (tiles > 0x7fffffffLL) {
         snprintf(err, errlen, "too many tiles");
         return cudaErrorInvalidValue;
     }
     prm.num_tiles = static_cast<int>(tiles);
 
-    const MapKey key = make_key(s, x, w, out, 1, 16, 4);
+    const MapKey key = make_key(s, x, w, out, 1, 16, 5);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        // one store box covers the whole 64-channel output row (wide epilogue)
-        if (!encode_y_2d(&maps[0], s, out, 64)) {
+        if (!encode_x_pairs(&maps[0], s, x, prm.boxw)) {
+            snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        if (!encode_y_rows(&maps[1], s, out, s.Wo < GA_TILE_W ? s.Wo : GA_TILE_W)) {
             snprintf(err, errlen, "tensor-map encode failed for the output tensor");
             return cudaErrorInvalidValue;
         }
-        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        for (int l = 2; l < 6; ++l) maps[l] = maps[0];
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    static std::atomic<unsigned long long> done{0};
-    set_kernel_name("qconv_gather_kernel");
-    cudaError_t e = set_smem_once(qconv_gather_kernel, GaCfg::SMEM_BYTES, done);
-    if (e != cudaSuccess) return e;
-    qconv_gather_kernel<<<grid, GA_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+    static std::atomic<unsigned long long> done_74{0}, done_any{0};
+    set_kernel_name("qconv_pairs_kernel");
+    if (s.kh == 7 && prm.nsp == 4) {  // the 7x7 stem
+        auto kern = qconv_pairs_kernel<7, 4>;
+        cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+    } else {
+        auto kern = qconv_pairs_kernel<0, 0>;
+        cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_any);
+        if (e != cudaSuccess) return e;
+        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+    }
     return cudaGetLastError();
 }
 

@@ -41,7 +41,10 @@ struct WsCfg {
     static constexpr int TAP_BYTES = 64 * WS_ROW_BYTES;  // expanded weight of one tap
     static constexpr int WSB_BYTES = WS_MAX_TAPS * TAP_BYTES;
     using E = EpiSmem<16, true>;
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 6;  // full, empty, accf[2], acce[2], drain, wsready
+    // accumulator buffers in TMEM: enough that neither the MMAs' completion latency nor
+    // the epilogue's turnaround stalls the MMA issue
+    static constexpr int NACC = 4;
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + 2;  // full, empty, accf, acce, drain, wsready
     static constexpr int TAIL_BYTES =
         WSB_BYTES + E::STAGING_BYTES + E::PARAM_BYTES + NUM_BARS * 8 + 16;
     static constexpr int SMEM_BYTES = 227 * 1024;
@@ -50,8 +53,9 @@ struct WsCfg {
     static constexpr int STAGING_OFF = WSB_OFF + WSB_BYTES;
     static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
     static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
+    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
     static constexpr uint32_t DESC_HI = desc_hi(8 * WS_ROW_BYTES, desc_layout(WS_ROW_BYTES));
-    static constexpr uint32_t TMEM_COLS = 128;  // 2 buffers x 64 columns
+    static constexpr uint32_t TMEM_COLS = 64 * NACC;
     static constexpr int EXP_WARPS = 9;          // warps 2, 4..11 expand the weight
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "WS shared memory");
 };
@@ -64,7 +68,9 @@ bool ws_halo_ok(const ConvShape& s) {
     return 2 * stage <= WsCfg::RING_BYTES;
 }
 
-template <bool HALO>
+// KH > 0: the filter height, known at compile time (halo staging), so the MMA issue
+// loop is fully unrolled; 0 = from the shape at run time.
+template <bool HALO, int KH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_y, const WsParams p) {
@@ -80,9 +86,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (MAX_STAGES + s); };
     const uint32_t accf0 = bar0 + 8u * (2 * MAX_STAGES);
-    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + 2);
-    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 4);
-    const uint32_t wsready_bar = bar0 + 8u * (2 * MAX_STAGES + 5);
+    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + C::NACC);
+    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
+    const uint32_t wsready_bar = drain_bar + 8u;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
@@ -94,7 +100,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             mbar_init(full_bar(i), 1);
             mbar_init(empty_bar(i), 1);
         }
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < C::NACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
             mbar_init(acce0 + 8u * b, 8 * 32);
         }
@@ -191,7 +197,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
             }
-            if (!ok) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
+            if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -209,9 +215,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tc_fence_after();
             const uint32_t wsb_lo = desc_lo(sbase + C::WSB_OFF);
             int local = 0;
+            const uint32_t row_lo = (s.Wo * WS_ROW_BYTES) >> 4;  // one output row of pixels
             for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
-                const int buf = local & 1;
-                const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+                const int buf = local % C::NACC;
+                const uint32_t use = static_cast<uint32_t>(local / C::NACC) & 1u;
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA)) {
                     ok = false;
@@ -227,10 +234,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                     tc_fence_after();
                     const uint32_t a_lo0 = desc_lo(sbase + stage * p.stage_bytes);
-                    if constexpr (HALO) {
+                    if constexpr (HALO && KH > 0) {
+                        const uint32_t b_lo0 = wsb_lo + ((kb * C::TAP_BYTES) >> 4);
+                        const uint32_t b_row = (s.kw * C::TAP_BYTES) >> 4;
+#pragma unroll
+                        for (int dh = 0; dh < KH; ++dh) {
+#pragma unroll
+                            for (int pc = 0; pc < 4; ++pc)
+                                umma_f16_w(d, a_lo0 + dh * row_lo + pc * 2, C::DESC_HI,
+                                           b_lo0 + dh * b_row + pc * 2, C::DESC_HI, IDESC,
+                                           (kb | dh | pc) != 0 ? 1u : 0u);
+                        }
+                    } else if constexpr (HALO) {
                         for (int dh = 0; dh < s.kh; ++dh) {
                             const int tap = dh * s.kw + kb;
-                            const uint32_t a_lo = a_lo0 + ((dh * s.Wo * WS_ROW_BYTES) >> 4);
+                            const uint32_t a_lo = a_lo0 + dh * row_lo;
                             const uint32_t b_lo = wsb_lo + ((tap * C::TAP_BYTES) >> 4);
 #pragma unroll
                             for (int pc = 0; pc < 4; ++pc)
@@ -318,7 +336,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                     return g;
                 };
-            epilogue_role<16, HALO, decltype(geo), true>(
+            epilogue_role<16, HALO, decltype(geo), true, 2, C::NACC>(
                 s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
                 reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
                 abort_flag, geo);

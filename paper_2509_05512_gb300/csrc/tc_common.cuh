@@ -123,13 +123,14 @@ struct EpiTile {
 
 // Shared-memory resources of the epilogue: two staging blocks of 128 x BNQ bf16 (one per
 // half; with WIDE, WBUFS blocks of 128 x 4 BNQ, one per tile parity when WBUFS = 2) and
-// the per-channel vectors [3][4 BNQ].
+// the per-channel vectors [2][4 BNQ] (16-byte aligned): the IQBN scale and the shift with
+// the bias folded in.
 template <int BNQ, bool WIDE = false, int WBUFS = 2>
 struct EpiSmem {
     static_assert(WBUFS == 1 || WBUFS == 2, "one or two wide staging blocks");
     static constexpr int OUT_TILE = BM * BNQ * 2;
     static constexpr int STAGING_BYTES = WIDE ? WBUFS * 4 * OUT_TILE : 2 * OUT_TILE;
-    static constexpr int PARAM_BYTES = 3 * 4 * BNQ * 4;
+    static constexpr int PARAM_BYTES = 2 * 4 * BNQ * 4;
     static constexpr uint32_t OUT_ROW = BNQ * 2;
     static constexpr uint32_t OUT_SW_MASK = BNQ == 64 ? 7u : (BNQ == 32 ? 3u : 1u);
 };
@@ -139,13 +140,17 @@ struct EpiSmem {
 // wait for its accumulator buffer, apply act(scale*(acc+bias)+shift+residual) (IQBN
 // inference form of Eq. 11-12), round to bf16, write a swizzled shared-memory block per
 // component and store it with TMA (rows outside the tensor are clipped by the map).
+// The affine step is evaluated as fma(scale, acc, scale*bias + shift): the folded shift
+// is formed once per channel, and the two vectors are read as float4 broadcasts (the
+// shared-memory pipe is shared with the tensor cores' operand reads, so the epilogue
+// keeps its own shared-memory traffic small).
 // With WIDE (4 BNQ = 64 channels = the whole output row, BNQ == Qout) all four
 // components go into one 128-byte-row block and a single TMA store per tile; with
 // WBUFS = 2 the block alternates between two buffers so the store overlaps the next
 // tile, with WBUFS = 1 the next tile waits until the store has read the block.
-// Accumulator buffer b of a tile lives at TMEM columns [4 BNQ b, 4 BNQ (b+1)), component
-// q at offset q BNQ.
-template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false, int WBUFS = 2>
+// Accumulator buffer b (of NACC, used round robin) of a tile lives at TMEM columns
+// [4 BNQ b, 4 BNQ (b+1)), component q at offset q BNQ.
+template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false, int WBUFS = 2, int NACC = 2>
 __device__ __forceinline__ void epilogue_role(const ConvShape& s, const EpilogueArgs& ep,
                                               const CUtensorMap* tmap_y, uint32_t tmem_base,
                                               uint8_t* staging, float* prm_s,
@@ -167,8 +172,8 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
     int cached_n = -1;
     int local = 0;
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
-        const int buf = local & 1;
-        const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        const int buf = local % NACC;
+        const uint32_t use = static_cast<uint32_t>(local / NACC) & 1u;
         // one lane per warp polls the barrier (256 pollers would crowd the shared-memory
         // pipe that TMA and the barriers themselves use), then broadcasts the result
         bool ok = true;
@@ -184,9 +189,11 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
             named_bar_sync(1, 256);
             for (int i = etid; i < 4 * BNQ; i += 256) {
                 const int c = (i / BNQ) * s.Qout + g.n_tile * BNQ + (i % BNQ);
-                prm_s[i] = ep.bias ? __ldg(ep.bias + c) : 0.0f;
-                prm_s[4 * BNQ + i] = ep.scale ? __ldg(ep.scale + c) : 1.0f;
-                prm_s[8 * BNQ + i] = ep.scale ? __ldg(ep.shift + c) : 0.0f;
+                const float b = ep.bias ? __ldg(ep.bias + c) : 0.0f;
+                const float sc = ep.scale ? __ldg(ep.scale + c) : 1.0f;
+                const float sh = ep.scale ? __ldg(ep.shift + c) : 0.0f;
+                prm_s[i] = sc;
+                prm_s[4 * BNQ + i] = fmaf(sc, b, sh);
             }
             named_bar_sync(1, 256);
             cached_n = g.n_tile;
@@ -196,8 +203,9 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                static_cast<uint32_t>(buf * 4 * BNQ);
         if constexpr (WIDE) {
-            // block of this tile parity; free once the store of WBUFS tiles ago has read it
-            stg = staging + (WBUFS == 2 ? buf : 0) * 4 * E::OUT_TILE;
+            // block of this tile's parity (by tile count, not accumulator buffer); free once
+            // the store of WBUFS tiles ago has read it
+            stg = staging + (local % WBUFS) * 4 * E::OUT_TILE;
             stg_addr = smem_u32(stg);
             if (threadIdx.x == EPI_WARP0 * 32) bulk_wait_group_read<WBUFS - 1>();
             named_bar_sync(1, 256);
@@ -240,19 +248,21 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
                     for (int t = 0; t < CH; ++t) rz[t] = 0.0f;
                 }
                 tmem_ld_wait();
-                const float* pb = prm_s + q * BNQ + j0;
-                const float* ps = prm_s + 4 * BNQ + q * BNQ + j0;
-                const float* ph = prm_s + 8 * BNQ + q * BNQ + j0;
+                const float4* ps4 = reinterpret_cast<const float4*>(prm_s + q * BNQ + j0);
+                const float4* ph4 = reinterpret_cast<const float4*>(prm_s + 4 * BNQ + q * BNQ + j0);
 #pragma unroll
                 for (int u = 0; u < CH / 8; ++u) {
+                    const float4 sa = ps4[2 * u], sb = ps4[2 * u + 1];
+                    const float4 ha = ph4[2 * u], hb = ph4[2 * u + 1];
+                    const float sc[8] = {sa.x, sa.y, sa.z, sa.w, sb.x, sb.y, sb.z, sb.w};
+                    const float sh[8] = {ha.x, ha.y, ha.z, ha.w, hb.x, hb.y, hb.z, hb.w};
                     uint32_t w[4];
 #pragma unroll
                     for (int t = 0; t < 4; ++t) {
                         const int e = 8 * u + 2 * t;
-                        float z0 = __uint_as_float(v[e]) + pb[e];
-                        float z1 = __uint_as_float(v[e + 1]) + pb[e + 1];
-                        z0 = fmaf(ps[e], z0, ph[e]) + rz[e];
-                        z1 = fmaf(ps[e + 1], z1, ph[e + 1]) + rz[e + 1];
+                        const float z0 = fmaf(sc[2 * t], __uint_as_float(v[e]), sh[2 * t]) + rz[e];
+                        const float z1 =
+                            fmaf(sc[2 * t + 1], __uint_as_float(v[e + 1]), sh[2 * t + 1]) + rz[e + 1];
                         w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
                     }
                     if constexpr (WIDE) {

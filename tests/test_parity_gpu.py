@@ -127,6 +127,17 @@ def test_tc_weight_stationary_layers(case, halo):
 
 
 @pytest.mark.parametrize("halo", [1, 0])
+def test_tc_weight_stationary_few_ctas(halo):
+    # 96 tiles on 3 CTAs: the accumulator ring, the stage ring and the epilogue's staging
+    # blocks all wrap many times
+    spec = inputs.small_layer("ws_few", 12, 32, 32, 64, 64, 3, 1, 1, residual=True,
+                              seed=(209, halo))
+    quan.quan_set_tc_tiles(0, 0, 3, 3)
+    quan.quan_set_tc_halo(bool(halo))
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+@pytest.mark.parametrize("halo", [1, 0])
 def test_config1_weight_stationary_staging(halo):
     quan.quan_set_tc_tiles(0, 0, 0, 3)
     quan.quan_set_tc_halo(bool(halo))
@@ -202,6 +213,8 @@ GATHER_CASES = [
     ("k3_pad1", 2, 20, 14, 4, 64, 3, 2, 1, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
     ("k4x2_valid", 1, 17, 12, 4, 64, 4, 2, 0, {"kw": 2}),     # one pair per filter row
     ("tiny", 1, 2, 2, 4, 64, 7, 2, 3, {}),                   # a single output pixel
+    ("wide_rows", 1, 6, 300, 4, 64, 7, 2, 3, {}),            # Wo = 150: two tiles per row
+    ("odd_kw", 2, 12, 20, 4, 64, 3, 2, 2, {"kw": 5}),        # 3x5, pad 2: zero pair slot
 ]
 
 
@@ -210,7 +223,7 @@ def test_tc_pixel_pair_gather_layers(case):
     name, N, H, W, Cin, Cout, k, s, p, extra = case
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(206, len(name)), **extra)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
-    assert quan.quan_last_kernel() == "qconv_gather_kernel"
+    assert quan.quan_last_kernel() == "qconv_pairs_kernel"
 
 
 def test_tc_pixel_pair_gather_few_ctas():
