@@ -51,6 +51,9 @@ def parse_args():
                          "or CPU legs")
     ap.add_argument("--no-graph", action="store_true",
                     help="time a plain launch loop instead of one CUDA-graph replay")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="with --profile: run the workload at this batch size (a smaller "
+                         "case for multi-pass ncu captures)")
     return ap.parse_args()
 
 
@@ -76,9 +79,10 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload: str):
+def recorded_traffic(workload: str, kernel: str | None = None):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or
-    None when no capture exists or the kernel sources changed since it was taken."""
+    None when no capture exists, it is of another kernel, or the kernel sources changed
+    since it was taken."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
@@ -86,6 +90,8 @@ def recorded_traffic(workload: str):
     except (OSError, ValueError):
         return None
     if not rec or rec.get("kernel_sha") != kernel_source_hash():
+        return None
+    if kernel is not None and not kernel.startswith(rec.get("kernel", "").split("<")[0]):
         return None
     return rec.get("dram_bytes_per_launch")
 
@@ -312,13 +318,18 @@ def main():
         if dist is not None:
             dist.barrier()
 
+    if args.batch and not args.profile:
+        raise SystemExit("--batch is for --profile runs only")
     if args.workload == "backbone":
         from paper_2509_05512_gb300 import backbone
-        runner = backbone.BackboneRunner(torch, quan, inputs)
+        runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
     else:
         spec = inputs.LAYERS[args.workload]
+        if args.batch:
+            import dataclasses
+            spec = dataclasses.replace(spec, N=args.batch)
         runner = LayerRunner(spec, torch, quan, inputs)
         unit, per_step_units, dtype = "TFLOP/s", spec.flops / 1e12, "bf16"
     stream = torch.cuda.current_stream()
@@ -445,7 +456,8 @@ def runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name):
     else:
         achieved, peak, unit, bound = nbytes / t / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
     return {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
-            "frac": round(achieved / peak, 4), "traffic": recorded_traffic(args.workload),
+            "frac": round(achieved / peak, 4),
+            "traffic": recorded_traffic(args.workload, kernel_name),
             "kernel": kernel_name, "peak_source": peak_src + " (burst)",
             "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
 
@@ -491,7 +503,8 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
     return {"bound": top["bound"], "achieved": top["achieved"],
             "peak": peaks["bf16_tflops"] if top["bound"] == "tensor" else peaks["hbm_gbs"],
             "unit": "TFLOP/s" if top["bound"] == "tensor" else "GB/s", "frac": top["frac"],
-            "traffic": None, "kernel": "%s (%s)" % (top["kernel"], top["name"]),
+            "traffic": recorded_traffic("backbone", top["kernel"]),
+            "kernel": "%s (%s)" % (top["kernel"], top["name"]),
             "share": round(top["ms"] / total, 3), "peak_source": peak_src + " (burst)",
             "layers": layers}
 

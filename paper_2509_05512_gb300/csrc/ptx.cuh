@@ -46,6 +46,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Same test, but a thread whose phase is not complete is suspended in hardware until the
+// phase completes or about `suspend_ns` nanoseconds have passed, instead of spinning (a
+// spinning waiter takes issue slots from the warps doing the work on its scheduler).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity,
+                                                    uint32_t suspend_ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(suspend_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait on an mbarrier phase.  Returns false once `limit_ns` of global time
 // has passed without the phase completing; the caller records the failure.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,

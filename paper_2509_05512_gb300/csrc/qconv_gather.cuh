@@ -11,23 +11,34 @@
 // and nsp (rounded up to even, 4 for the 7x7 stem) is the number of pairs per filter row.
 //
 // Tile = 128 consecutive output columns of one output row (one MMA of M = 128; columns
-// past the row end are computed and never stored).  For each filter row ky one tiled TMA
-// box holds the 128 + nsp - 1 pairs of input row 2 ho - pad + ky the tile reads, zero
-// filled outside the image.  The A operand of the K step (ky, pairs 2t, 2t + 1) is that
-// box read as a K-major, non-swizzled matrix whose row m starts at pair m + 2t: 16-byte
-// rows, 8-row groups 128 bytes apart (stride byte offset) and the second 8-element K half
-// one pair (16 bytes) further on (leading byte offset) -- the overlapping rows of an
-// im2col matrix come from the descriptor, so the pixels are read from global memory once
-// per filter row and never copied on chip.
+// past the row end are computed and never stored).  One 3-D TMA box per tile holds, for
+// the kh consecutive input rows 2 ho - pad .. 2 ho - pad + kh - 1, the 128 + nsp - 1 pairs
+// the tile reads, zero filled outside the image.  The box addresses the input in groups
+// of G pairs (128-byte elements for W a multiple of 16), since the TMA unit's cost grows
+// with the number of inner-dimension elements: 16-byte elements made a box 917 requests
+// and its latency several microseconds.  The tile's first pair then sits d0 = (-shift)
+// mod G pairs into the box.  The A operand of the K step
+// (ky, pairs 2t, 2t + 1) is that box's row ky read as a K-major, non-swizzled matrix whose
+// row m starts at pair m + 2t: 16-byte rows, 8-row groups 128 bytes apart (stride byte
+// offset) and the second 8-element K half one pair (16 bytes) further on (leading byte
+// offset) -- the overlapping rows of an im2col matrix come from the descriptor, so the
+// pixels are read from global memory once per filter row and never copied on chip, and a
+// tile costs one TMA instruction (the per-box issue cost of the TMA unit, not its bytes,
+// limits boxes this narrow).
 //
-//   warp 0        TMA producer: kh boxes per tile into a ring of stages.
-//   warp 1        TMEM owner and MMA issuer: kh * nsp / 2 MMAs of M = 128, N = 64 per
-//                 tile (14 for the stem, K = 224).
+//   warp 0        TMA producer: one box per tile into a ring of stages.
+//   warps 1..3    MMA issuers, one lane each, taking the CTA's tiles round robin: each
+//                 waits for its tile's stage and accumulator buffer and issues the
+//                 kh * nsp / 2 MMAs of M = 128, N = 64 (14 for the stem, K = 224) in one
+//                 unrolled run.  The tensor pipe keeps almost no queue and the issuing
+//                 thread's own waits and branches cost hundreds of cycles while its MMAs
+//                 are in flight, so three issuers are needed to keep the pipe busy.
+//                 Warp 1 also owns TMEM (8 accumulator buffers of 64 columns).
 //   warps 2..11   expand the signed block weight of Eq. 6 once per CTA:
 //                 B[(q, co)][(ky, pair, e, p)] = sign(q, p) W_{q xor p}[co][ky][2 pair - lead + e]
 //                 (zero outside the filter), K-major with a 32-byte swizzle; then warps
-//                 4..11 run the wide epilogue (one 3-D TMA store per tile, clipped at the
-//                 end of the output row).
+//                 4..11 run the direct epilogue (tc_common.cuh: no shared memory, coalesced
+//                 global stores, columns past the end of the output row not stored).
 // The zero-weight columns read real input pixels, which only matters for non-finite
 // inputs (0 * inf); finite inputs give exactly the convolution of Eq. 5.
 
@@ -38,14 +49,17 @@ struct GatherParams {
     ConvShape s;
     EpilogueArgs ep;
     const __nv_bfloat16* w[4];  // letter tensors [16][kh][kw][1]
+    void* y;                    // output [N][Ho][Wo][64]
     unsigned long long wait_limit_ns;
     int inject_stall;
     int nsp;          // pixel pairs per filter row (even)
     int lead;         // pad mod 2: zero-weight filter column before the first pair
     int shift;        // (pad + lead) / 2: first pair of output column 0 is -shift
-    int boxw;         // pairs per box: GA_TILE_W + nsp - 1
-    int box_stride;   // bytes between the boxes of one stage (128-byte multiple)
-    int box_bytes;    // boxw * 16
+    int group;        // G: pairs per TMA element (1, 2, 4 or 8)
+    int d0;           // pairs from the box start to the tile's first pair
+    int boxg;         // G-pair elements per filter row of the box
+    int box_stride;   // bytes between filter rows in the box: boxg * 16 G
+    int box_bytes;    // bytes of one filter row: boxg * 16 G
     int stage_bytes;
     int stages;
     int segs;         // tiles per output row
@@ -55,20 +69,20 @@ struct GatherParams {
 struct GaCfg {
     static constexpr int CHUNK_B = 64 * 32;  // one K step of the weight: 64 rows x 32 bytes
     static constexpr int B_BYTES = (GA_MAX_UNITS / 2) * CHUNK_B;
-    using E = EpiSmem<16, true, 2>;
+    // the letter tensors during the weight expansion (4 x 16 x taps x 2 bytes, taps <= 64)
+    static constexpr int SCRATCH_BYTES = 8 * 1024;
     // accumulator buffers in TMEM: enough that neither the MMAs' completion latency nor
     // the epilogue's turnaround stalls the MMA issue
-    static constexpr int NACC = 4;
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + 2;  // full, empty, accf, acce, drain, bready
-    static constexpr int TAIL_BYTES = B_BYTES + E::STAGING_BYTES + E::PARAM_BYTES +
-                                      NUM_BARS * 8 + 16;
+    static constexpr int NACC = 8;
+    static constexpr int ISSUERS = 3;  // warps 1..3
+    // full, empty, accf, acce, drain (one per issuer), bready
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + ISSUERS + 1;
+    static constexpr int TAIL_BYTES = B_BYTES + SCRATCH_BYTES + NUM_BARS * 8 + 16;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr int RING_BYTES = ((SMEM_BYTES - 1024 - TAIL_BYTES) / 1024) * 1024;
     static constexpr int B_OFF = RING_BYTES;
-    static constexpr int STAGING_OFF = B_OFF + B_BYTES;
-    static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
-    static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
-    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
+    static constexpr int SCRATCH_OFF = B_OFF + B_BYTES;
+    static constexpr int BAR_OFF = SCRATCH_OFF + SCRATCH_BYTES;
     // A: K-major, no swizzle, 8-row groups 128 bytes apart (the leading byte offset of
     // one pair, 16 bytes, is the low word's default); B: K-major rows of 32 bytes.
     static constexpr uint32_t A_DESC_HI = desc_hi(8 * 16, 0);
@@ -85,6 +99,16 @@ int gather_nsp(const ConvShape& s) {
     return nsp + (nsp & 1);
 }
 
+// Weight expansion, run by warps 2..11 (EXP_WARPS): the signed block weight of Eq. 6 as
+// K-major rows of 32-byte K steps with a 32-byte swizzle,
+//   B[(q, co)][(ky, pair j, pixel e, component p)] = sign(q, p) W_{q xor p}[co][ky][2 j - lead + e]
+// (zero outside the filter).  The four letter tensors are first copied to shared memory
+// (a scratch area) with every thread's 16-byte loads in flight at once, then expanded
+// shared -> shared.
+__device__ __forceinline__ void expand_block_weight(const ConvShape& s, const GatherParams& p,
+                                                    uint8_t* smem, int warp, int lane,
+                                                    uint32_t bready_bar);
+
 // Shapes the pixel-pair kernel covers: one quaternion input channel, 16 quaternion output
 // channels, stride 2, even input width, K within the weight region.
 bool gather_ok(const ConvShape& s) {
@@ -92,9 +116,74 @@ bool gather_ok(const ConvShape& s) {
     return static_cast<long long>(s.kh) * gather_nsp(s) <= GA_MAX_UNITS;
 }
 
-// Bytes between the pair boxes of one stage for nsp pairs per filter row.
-__host__ __device__ constexpr int gather_box_stride(int nsp) {
-    return ((GA_TILE_W + nsp - 1) * 16 + 127) & ~127;
+
+__device__ __forceinline__ void expand_block_weight(const ConvShape& s, const GatherParams& p,
+                                                    uint8_t* smem, int warp, int lane,
+                                                    uint32_t bready_bar) {
+    using C = GaCfg;
+    const int et = (warp - 2) * 32 + lane;  // 0 .. 319
+    constexpr int ET = C::EXP_WARPS * 32;
+    const int taps = s.kh * s.kw;
+    // 1. letters [16][kh][kw][1] -> shared memory, 2 * taps 16-byte chunks per letter
+    const int lchunks = 2 * taps, nchunks = 4 * lchunks;
+    uint8_t* wl = smem + C::SCRATCH_OFF;
+    {
+        uint4 v[2];
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            const int i = et + r * ET;
+            if (i < nchunks) {
+                const int L = i / lchunks;
+                v[r] = __ldg(reinterpret_cast<const uint4*>(p.w[L]) + (i - L * lchunks));
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r)
+            if (et + r * ET < nchunks) reinterpret_cast<uint4*>(wl)[et + r * ET] = v[r];
+        for (int i = et + 2 * ET; i < nchunks; i += ET) {
+            const int L = i / lchunks;
+            reinterpret_cast<uint4*>(wl)[i] =
+                __ldg(reinterpret_cast<const uint4*>(p.w[L]) + (i - L * lchunks));
+        }
+    }
+    named_bar_sync(5, ET);
+    const __nv_bfloat16* wls = reinterpret_cast<const __nv_bfloat16*>(wl);
+    // 2. one 16-byte K unit (filter row ky, pair j) of output row n = (q, co) per item:
+    //    8 values, pixel e of the pair major, input component p minor
+    const int units = s.kh * p.nsp;
+    for (int i = et; i < 64 * units; i += ET) {
+        const int n = i / units, u = i - (i / units) * units;
+        const int q = n >> 4, co = n & 15;
+        const int ky = u / p.nsp, j = u - (u / p.nsp) * p.nsp;
+        uint32_t packed[4];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            const int kx = 2 * j - p.lead + e;
+            const bool in = kx >= 0 && kx < s.kw;
+            float v[4];
+#pragma unroll
+            for (int pc = 0; pc < 4; ++pc) {
+                float wv = 0.0f;
+                if (in) {
+                    const int L = q ^ pc;
+                    wv = __bfloat162float(wls[(L * 16 + co) * taps + ky * s.kw + kx]);
+                    if ((NEG_MASK >> (4 * q + pc)) & 1u) wv = -wv;
+                }
+                v[pc] = wv;
+            }
+            packed[2 * e] = pack_bf16x2(v[0], v[1]);
+            packed[2 * e + 1] = pack_bf16x2(v[2], v[3]);
+        }
+        // K step u / 2, 16-byte half u % 2 of the 32-byte row, 32-byte swizzle
+        const uint32_t off =
+            static_cast<uint32_t>(C::B_OFF + (u >> 1) * C::CHUNK_B + n * 32) +
+            ((static_cast<uint32_t>(u & 1) ^ ((static_cast<uint32_t>(n) >> 2) & 1u)) << 4);
+        *reinterpret_cast<uint4*>(smem + off) =
+            make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bready_bar);
 }
 
 // KH, NSP > 0: the filter height and pairs per filter row known at compile time, so the
@@ -102,8 +191,7 @@ __host__ __device__ constexpr int gather_box_stride(int nsp) {
 // parameters at run time.
 template <int KH, int NSP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    qconv_pairs_kernel(const __grid_constant__ CUtensorMap tmap_x,
-                       const __grid_constant__ CUtensorMap tmap_y, const GatherParams p) {
+    qconv_pairs_kernel(const __grid_constant__ CUtensorMap tmap_x, const GatherParams p) {
     using C = GaCfg;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -117,8 +205,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     auto empty_bar = [&](int s) { return bar0 + 8u * (MAX_STAGES + s); };
     const uint32_t accf0 = bar0 + 8u * (2 * MAX_STAGES);
     const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + C::NACC);
-    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
-    const uint32_t bready_bar = drain_bar + 8u;
+    const uint32_t drain0 = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
+    const uint32_t bready_bar = drain0 + 8u * C::ISSUERS;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
@@ -132,17 +220,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         for (int b = 0; b < C::NACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
-            mbar_init(acce0 + 8u * b, 8 * 32);
+            mbar_init(acce0 + 8u * b, EPI2_ACCE_COUNT);
         }
-        mbar_init(drain_bar, 1);
+        for (int i = 0; i < C::ISSUERS; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(bready_bar, C::EXP_WARPS);
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&tmap_x);
-        tma_prefetch_desc(&tmap_y);
-    }
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap_x);
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
         tmem_relinquish();
@@ -174,9 +259,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 filled |= 1u << stage;
                 fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
                 const uint32_t dst = sbase + stage * p.stage_bytes;
-                const int x0 = seg * GA_TILE_W - p.shift, y0 = ho * 2 - s.pad;
-                for (int ky = 0; ky < s.kh; ++ky)
-                    tma_load_4d(dst + ky * p.box_stride, &tmap_x, fb, 0, x0, y0 + ky, img, pol_x);
+                tma_load_4d(dst, &tmap_x, fb, 0, (seg * GA_TILE_W - p.shift - p.d0) / p.group,
+                            ho * 2 - s.pad, img, pol_x);
                 if (++stage == STAGES) {
                     stage = 0;
                     phase ^= 1u;
@@ -184,15 +268,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+    }
+    if (warp >= 1 && warp <= C::ISSUERS) {
+        // ------------------------------------------------------------ MMA issuers
+        // (warps 2 and 3 first help with the weight expansion below)
+        if (warp >= 2) expand_block_weight(s, p, smem, warp, lane, bready_bar);
         if (lane == 0) {
             constexpr uint32_t IDESC = make_idesc(BM, 64, 0);
-            int stage = 0;
-            uint32_t phase = 0;
+            const int me = warp - 1;
+            const uint32_t drain_bar = drain0 + 8u * me;
             bool ok = wait_or_abort(bready_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
             int issued = 0;
-            if (p.inject_stall) {
+            if (p.inject_stall && me == 0) {
                 // Failure injection: wait on a barrier nothing arrives on.
                 wait_or_abort(drain_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
                 ok = false;
@@ -200,10 +287,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tc_fence_after();
             const uint32_t b_lo0 = desc_lo(sbase + C::B_OFF);
             const int half = p.nsp / 2;
-            int local = 0;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
-                const int buf = local % C::NACC;
-                const uint32_t use = static_cast<uint32_t>(local / C::NACC) & 1u;
+            // local tile k of this CTA is tile blockIdx.x + k * gridDim.x; it uses stage
+            // k mod STAGES and accumulator buffer k mod NACC
+            for (int k = me, tile = blockIdx.x + me * gridDim.x; ok && tile < p.num_tiles;
+                 k += C::ISSUERS, tile += C::ISSUERS * gridDim.x) {
+                const int buf = k % C::NACC;
+                const uint32_t use = static_cast<uint32_t>(k / C::NACC) & 1u;
+                const int stage = k % STAGES;
+                const uint32_t phase = static_cast<uint32_t>(k / STAGES) & 1u;
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA) ||
                     !wait_or_abort(full_bar(stage), phase, limit, abort_flag,
@@ -213,20 +304,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * 64);
-                const uint32_t a_lo0 = desc_lo(sbase + stage * p.stage_bytes);
+                const uint32_t a_lo0 = desc_lo(sbase + stage * p.stage_bytes) + p.d0;
+                const uint32_t box_lo = static_cast<uint32_t>(p.box_stride) >> 4;
                 if constexpr (KH > 0) {
-                    constexpr uint32_t BOX_LO = gather_box_stride(NSP) >> 4;
 #pragma unroll
                     for (int ky = 0; ky < KH; ++ky)
 #pragma unroll
                         for (int t = 0; t < NSP / 2; ++t) {
                             const int c = ky * (NSP / 2) + t;
-                            umma_f16_w(d, a_lo0 + ky * BOX_LO + 2 * t, C::A_DESC_HI,
+                            umma_f16_w(d, a_lo0 + ky * box_lo + 2 * t, C::A_DESC_HI,
                                        b_lo0 + ((c * C::CHUNK_B) >> 4), C::B_DESC_HI, IDESC,
                                        c != 0 ? 1u : 0u);
                         }
                 } else {
-                    const uint32_t box_lo = static_cast<uint32_t>(p.box_stride) >> 4;
                     int c = 0;
                     for (int ky = 0; ky < s.kh; ++ky)
                         for (int t = 0; t < half; ++t, ++c)
@@ -237,12 +327,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 ++issued;
                 umma_commit(empty_bar(stage));
                 umma_commit(accf0 + 8u * buf);
-                if (++stage == STAGES) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
             }
             if (!ok && issued > 0) {
+                // let this issuer's MMAs finish before TMEM is released
                 umma_commit(drain_bar);
                 const uint64_t t0 = global_timer_ns();
                 while (!mbar_try_wait(drain_bar, 0u)) {
@@ -253,49 +340,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
             }
         }
-    } else {
-        // ------------------------------------------------------------ weight expansion
-        // warps 2..11: one 16-byte K unit (filter row ky, pair j) of output row
-        // n = (q, co) per item: 8 values, pixel e of the pair major, input component p minor.
-        const int et = (warp - 2) * 32 + lane;  // 0 .. 319
-        constexpr int ET = C::EXP_WARPS * 32;
-        const int taps = s.kh * s.kw;
-        const int units = s.kh * p.nsp;
-        for (int i = et; i < 64 * units; i += ET) {
-            const int n = i / units, u = i - (i / units) * units;
-            const int q = n >> 4, co = n & 15;
-            const int ky = u / p.nsp, j = u - (u / p.nsp) * p.nsp;
-            uint32_t packed[4];
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int kx = 2 * j - p.lead + e;
-                const bool in = kx >= 0 && kx < s.kw;
-                float v[4];
-#pragma unroll
-                for (int pc = 0; pc < 4; ++pc) {
-                    float wv = 0.0f;
-                    if (in) {
-                        const int L = q ^ pc;
-                        wv = __bfloat162float(p.w[L][co * taps + ky * s.kw + kx]);
-                        if ((NEG_MASK >> (4 * q + pc)) & 1u) wv = -wv;
-                    }
-                    v[pc] = wv;
-                }
-                packed[2 * e] = pack_bf16x2(v[0], v[1]);
-                packed[2 * e + 1] = pack_bf16x2(v[2], v[3]);
-            }
-            // K step u / 2, 16-byte half u % 2 of the 32-byte row, 32-byte swizzle
-            const uint32_t off =
-                static_cast<uint32_t>(C::B_OFF + (u >> 1) * C::CHUNK_B + n * 32) +
-                ((static_cast<uint32_t>(u & 1) ^ ((static_cast<uint32_t>(n) >> 2) & 1u)) << 4);
-            *reinterpret_cast<uint4*>(smem + off) =
-                make_uint4(packed[0], packed[1], packed[2], packed[3]);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(bready_bar);
-
-        if (warp >= EPI_WARP0) {
+    } else if (warp >= EPI_WARP0) {
+        expand_block_weight(s, p, smem, warp, lane, bready_bar);
+        {
             // -------------------------------------------------------- epilogue
             const int segs = p.segs, Wo = s.Wo;
             auto geo = [segs, Wo](int tile) {
@@ -309,10 +356,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 g.sz = row;
                 return g;
             };
-            epilogue_role<16, true, decltype(geo), true, 2, C::NACC>(
-                s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
-                reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
-                abort_flag, geo);
+            epilogue_direct64<decltype(geo), C::NACC>(s, p.ep, p.y, tmem_base, accf0, acce0,
+                                                      p.num_tiles, limit, abort_flag, geo);
         }
     }
 

@@ -481,36 +481,22 @@ bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int chan
     return r == CUDA_SUCCESS;
 }
 
-// Input of a 4-channel layer viewed as 16-byte pixel pairs: [N][H][W/2][8], boxes of
-// `boxw` pairs of one input row, no swizzle (dense 16-byte rows in shared memory).
-bool encode_x_pairs(CUtensorMap* map, const ConvShape& s, const void* x, int boxw) {
-    const cuuint64_t W2 = static_cast<cuuint64_t>(s.W / 2);
-    const cuuint64_t dims[4] = {8, W2, static_cast<cuuint64_t>(s.H),
+// Input of a 4-channel layer viewed as groups of G pixel pairs (16 G bytes):
+// [N][H][W/(2G)][8 G], boxes of `boxg` groups x kh input rows of one image, no swizzle
+// (dense rows in shared memory).
+bool encode_x_pairs(CUtensorMap* map, const ConvShape& s, const void* x, int group, int boxg) {
+    const cuuint64_t WG = static_cast<cuuint64_t>(s.W / (2 * group));
+    const cuuint64_t eb = 16ull * group;
+    const cuuint64_t dims[4] = {8ull * group, WG, static_cast<cuuint64_t>(s.H),
                                 static_cast<cuuint64_t>(s.N)};
-    const cuuint64_t strides[3] = {16, 16 * W2, 16 * W2 * s.H};
-    const cuuint32_t box[4] = {8, static_cast<cuuint32_t>(boxw), 1, 1};
+    const cuuint64_t strides[3] = {eb, eb * WG, eb * WG * s.H};
+    const cuuint32_t box[4] = {8u * group, static_cast<cuuint32_t>(boxg),
+                               static_cast<cuuint32_t>(s.kh), 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     const CUresult r = g_encode_tiled(
         map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
-
-// Output of a 64-channel layer viewed as [N*Ho][Wo][64], stored in boxes of up to
-// `cols` output columns of one row (128-byte rows, 128-byte swizzle); a box reaching past
-// the end of the row is clipped there.
-bool encode_y_rows(CUtensorMap* map, const ConvShape& s, const void* y, int cols) {
-    const cuuint64_t dims[3] = {64, static_cast<cuuint64_t>(s.Wo),
-                                static_cast<cuuint64_t>(s.N) * s.Ho};
-    const cuuint64_t strides[2] = {128, 128 * static_cast<cuuint64_t>(s.Wo)};
-    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(cols), 1};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
-                                      const_cast<void*>(y), dims, strides, box, estr,
-                                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                                      CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
 
@@ -761,18 +747,23 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     prm.s = s;
     prm.ep = ep;
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     prm.lead = s.pad & 1;
     prm.nsp = gather_nsp(s);
     prm.shift = (s.pad + prm.lead) / 2;
-    prm.boxw = GA_TILE_W + prm.nsp - 1;
-    prm.box_bytes = prm.boxw * 16;
-    prm.box_stride = gather_box_stride(prm.nsp);
+    const int W2 = s.W / 2;
+    prm.group = W2 % 8 == 0 ? 8 : (W2 % 4 == 0 ? 4 : (W2 % 2 == 0 ? 2 : 1));
+    prm.d0 = ((-prm.shift) % prm.group + prm.group) % prm.group;
+    const int boxw = GA_TILE_W + prm.nsp - 1;  // pairs a tile reads per filter row
+    prm.boxg = (prm.d0 + boxw + prm.group - 1) / prm.group;
+    prm.box_bytes = prm.boxg * 16 * prm.group;
+    prm.box_stride = prm.box_bytes;
     prm.stage_bytes = (s.kh * prm.box_stride + 1023) & ~1023;
     int stages = GaCfg::RING_BYTES / prm.stage_bytes;
     if (stages > MAX_STAGES) stages = MAX_STAGES;
-    if (stages < 2 || s.kh * prm.nsp > GA_MAX_UNITS || prm.boxw > 256) {
+    if (stages < 2 || s.kh * prm.nsp > GA_MAX_UNITS || prm.boxg > 256 || s.kh > 256) {
         snprintf(err, errlen, "pixel-pair kernel: kh=%d kw=%d does not fit", s.kh, s.kw);
         return cudaErrorInvalidValue;
     }
@@ -786,18 +777,14 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     }
     prm.num_tiles = static_cast<int>(tiles);
 
-    const MapKey key = make_key(s, x, w, out, 1, 16, 5);
+    const MapKey key = make_key(s, x, w, out, 1, 16, 6);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        if (!encode_x_pairs(&maps[0], s, x, prm.boxw)) {
+        if (!encode_x_pairs(&maps[0], s, x, prm.group, prm.boxg)) {
             snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
             return cudaErrorInvalidValue;
         }
-        if (!encode_y_rows(&maps[1], s, out, s.Wo < GA_TILE_W ? s.Wo : GA_TILE_W)) {
-            snprintf(err, errlen, "tensor-map encode failed for the output tensor");
-            return cudaErrorInvalidValue;
-        }
-        for (int l = 2; l < 6; ++l) maps[l] = maps[0];
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
@@ -807,12 +794,12 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         auto kern = qconv_pairs_kernel<7, 4>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else {
         auto kern = qconv_pairs_kernel<0, 0>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_any);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     }
     return cudaGetLastError();
 }
