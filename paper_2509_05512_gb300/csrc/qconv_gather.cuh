@@ -32,8 +32,9 @@
 //                 kh * nsp / 2 MMAs of M = 128, N = 64 (14 for the stem, K = 224) in one
 //                 unrolled run.  The tensor pipe keeps almost no queue and the issuing
 //                 thread's own waits and branches cost hundreds of cycles while its MMAs
-//                 are in flight, so three issuers are needed to keep the pipe busy.
-//                 Warp 1 also owns TMEM (8 accumulator buffers of 64 columns).
+//                 are in flight, so three issuers are needed to keep the pipe busy.  Each
+//                 issuer owns its stages and two accumulator buffers (issuer_stage,
+//                 issuer_acc in tc_common.cuh).  Warp 1 also owns TMEM.
 //   warps 2..11   expand the signed block weight of Eq. 6 once per CTA:
 //                 B[(q, co)][(ky, pair, e, p)] = sign(q, p) W_{q xor p}[co][ky][2 pair - lead + e]
 //                 (zero outside the filter), K-major with a 32-byte swizzle; then warps
@@ -61,7 +62,7 @@ struct GatherParams {
     int box_stride;   // bytes between filter rows in the box: boxg * 16 G
     int box_bytes;    // bytes of one filter row: boxg * 16 G
     int stage_bytes;
-    int stages;
+    int per;          // stages owned by each issuer
     int segs;         // tiles per output row
     int num_tiles;
 };
@@ -71,12 +72,10 @@ struct GaCfg {
     static constexpr int B_BYTES = (GA_MAX_UNITS / 2) * CHUNK_B;
     // the letter tensors during the weight expansion (4 x 16 x taps x 2 bytes, taps <= 64)
     static constexpr int SCRATCH_BYTES = 8 * 1024;
-    // accumulator buffers in TMEM: enough that neither the MMAs' completion latency nor
-    // the epilogue's turnaround stalls the MMA issue
-    static constexpr int NACC = 8;
-    static constexpr int ISSUERS = 3;  // warps 1..3
+    static constexpr int MAX_PER = 4;                // stages per issuer at most
+    static constexpr int NSTAGE = ISSUERS * MAX_PER;  // stage barriers
     // full, empty, accf, acce, drain (one per issuer), bready
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + ISSUERS + 1;
+    static constexpr int NUM_BARS = 2 * NSTAGE + 2 * ISSUER_ACC + ISSUERS + 1;
     static constexpr int TAIL_BYTES = B_BYTES + SCRATCH_BYTES + NUM_BARS * 8 + 16;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr int RING_BYTES = ((SMEM_BYTES - 1024 - TAIL_BYTES) / 1024) * 1024;
@@ -87,7 +86,7 @@ struct GaCfg {
     // one pair, 16 bytes, is the low word's default); B: K-major rows of 32 bytes.
     static constexpr uint32_t A_DESC_HI = desc_hi(8 * 16, 0);
     static constexpr uint32_t B_DESC_HI = desc_hi(8 * 32, desc_layout(32));
-    static constexpr uint32_t TMEM_COLS = 64 * NACC;
+    static constexpr uint32_t TMEM_COLS = 512;  // ISSUER_ACC buffers of 64 columns
     static constexpr int EXP_WARPS = 10;        // warps 2..11
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "gather shared memory");
 };
@@ -202,27 +201,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (MAX_STAGES + s); };
-    const uint32_t accf0 = bar0 + 8u * (2 * MAX_STAGES);
-    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + C::NACC);
-    const uint32_t drain0 = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
-    const uint32_t bready_bar = drain0 + 8u * C::ISSUERS;
+    auto empty_bar = [&](int s) { return bar0 + 8u * (C::NSTAGE + s); };
+    const uint32_t accf0 = bar0 + 8u * (2 * C::NSTAGE);
+    const uint32_t acce0 = bar0 + 8u * (2 * C::NSTAGE + ISSUER_ACC);
+    const uint32_t drain0 = bar0 + 8u * (2 * C::NSTAGE + 2 * ISSUER_ACC);
+    const uint32_t bready_bar = drain0 + 8u * ISSUERS;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
     const uint64_t limit = p.wait_limit_ns;
-    const int STAGES = p.stages;
+    const int STAGES = ISSUERS * p.per;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(full_bar(i), 1);
             mbar_init(empty_bar(i), 1);
         }
-        for (int b = 0; b < C::NACC; ++b) {
+        for (int b = 0; b < ISSUER_ACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
             mbar_init(acce0 + 8u * b, EPI2_ACCE_COUNT);
         }
-        for (int i = 0; i < C::ISSUERS; ++i) mbar_init(drain0 + 8u * i, 1);
+        for (int i = 0; i < ISSUERS; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(bready_bar, C::EXP_WARPS);
         *abort_flag = 0;
         fence_barrier_init();
@@ -241,14 +240,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t pol_x = l2_policy_evict_normal();
-            int stage = 0;
-            uint32_t phase = 0;
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
             const uint32_t tx = static_cast<uint32_t>(s.kh * p.box_bytes);
-            for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
+            int k = 0;
+            for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++k) {
                 const int row = tile / p.segs, seg = tile - (tile / p.segs) * p.segs;
                 const int img = row / s.Ho, ho = row - (row / s.Ho) * s.Ho;
+                // local tile k -> issuer k % ISSUERS, its (k / ISSUERS)-th stage use
+                int stage;
+                uint32_t phase;
+                issuer_stage(k % ISSUERS, k / ISSUERS, p.per, stage, phase);
                 if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_PRODUCER)) {
                     ok = false;
@@ -261,15 +263,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const uint32_t dst = sbase + stage * p.stage_bytes;
                 tma_load_4d(dst, &tmap_x, fb, 0, (seg * GA_TILE_W - p.shift - p.d0) / p.group,
                             ho * 2 - s.pad, img, pol_x);
-                if (++stage == STAGES) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
             }
             if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
         }
     }
-    if (warp >= 1 && warp <= C::ISSUERS) {
+    if (warp >= 1 && warp <= ISSUERS) {
         // ------------------------------------------------------------ MMA issuers
         // (warps 2 and 3 first help with the weight expansion below)
         if (warp >= 2) expand_block_weight(s, p, smem, warp, lane, bready_bar);
@@ -287,14 +285,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tc_fence_after();
             const uint32_t b_lo0 = desc_lo(sbase + C::B_OFF);
             const int half = p.nsp / 2;
-            // local tile k of this CTA is tile blockIdx.x + k * gridDim.x; it uses stage
-            // k mod STAGES and accumulator buffer k mod NACC
-            for (int k = me, tile = blockIdx.x + me * gridDim.x; ok && tile < p.num_tiles;
-                 k += C::ISSUERS, tile += C::ISSUERS * gridDim.x) {
-                const int buf = k % C::NACC;
-                const uint32_t use = static_cast<uint32_t>(k / C::NACC) & 1u;
-                const int stage = k % STAGES;
-                const uint32_t phase = static_cast<uint32_t>(k / STAGES) & 1u;
+            // local tile k of this CTA is tile blockIdx.x + k * gridDim.x; this issuer's
+            // j-th tile is k = me + j * ISSUERS
+            for (int k = me, j = 0, tile = blockIdx.x + me * gridDim.x; ok && tile < p.num_tiles;
+                 k += ISSUERS, ++j, tile += ISSUERS * gridDim.x) {
+                int buf, stage;
+                uint32_t use, phase;
+                issuer_acc(k, buf, use);
+                issuer_stage(me, j, p.per, stage, phase);
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA) ||
                     !wait_or_abort(full_bar(stage), phase, limit, abort_flag,
@@ -356,8 +354,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 g.sz = row;
                 return g;
             };
-            epilogue_direct64<decltype(geo), C::NACC>(s, p.ep, p.y, tmem_base, accf0, acce0,
-                                                      p.num_tiles, limit, abort_flag, geo);
+            epilogue_direct64<decltype(geo)>(s, p.ep, p.y, tmem_base, accf0, acce0,
+                                             p.num_tiles, limit, abort_flag, geo);
         }
     }
 

@@ -528,24 +528,6 @@ bool encode_y_2d(CUtensorMap* map, const ConvShape& s, const void* y, int bnq) {
     return r == CUDA_SUCCESS;
 }
 
-// Output viewed as [N][Ho*Wo][Cout], stored in boxes of `rows` pixels of one image, so a
-// partial last row block of an image is clipped at the image end.
-bool encode_y_3d(CUtensorMap* map, const ConvShape& s, const void* y, int bnq, int rows) {
-    const cuuint64_t hw = static_cast<cuuint64_t>(s.Ho) * s.Wo;
-    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(s.Cout), hw,
-                                static_cast<cuuint64_t>(s.N)};
-    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(s.Cout) * 2,
-                                   static_cast<cuuint64_t>(s.Cout) * 2 * hw};
-    const cuuint32_t box[3] = {static_cast<cuuint32_t>(bnq), static_cast<cuuint32_t>(rows), 1};
-    const cuuint32_t estr[3] = {1, 1, 1};
-    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3,
-                                      const_cast<void*>(y), dims, strides, box, estr,
-                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(bnq * 2),
-                                      CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
-
 // The shared-memory opt-in is per device and kernel; set it once for each.
 template <typename K>
 cudaError_t set_smem_once(K kern, int bytes, std::atomic<unsigned long long>& done) {
@@ -665,6 +647,7 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     prm.s = s;
     prm.ep = ep;
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     prm.taps = s.kh * s.kw;
@@ -690,14 +673,14 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     }
     prm.num_tiles = static_cast<int>(tiles);
     prm.stage_bytes = (prm.box_bytes + 1023) & ~1023;
-    int stages = WsCfg::RING_BYTES / prm.stage_bytes;
-    if (stages > MAX_STAGES) stages = MAX_STAGES;
-    if (stages < 2) {
+    int per = WsCfg::RING_BYTES / prm.stage_bytes / ISSUERS;
+    if (per > WsCfg::MAX_PER) per = WsCfg::MAX_PER;
+    if (per < 1) {
         snprintf(err, errlen, "weight-stationary pixel box of %d bytes does not fit",
                  prm.box_bytes);
         return cudaErrorInvalidValue;
     }
-    prm.stages = stages;
+    prm.per = per;
 
     const MapKey key = make_key(s, x, w, out, 16, 16, halo ? 3 : 2);
     CUtensorMap maps[6];
@@ -708,14 +691,7 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
             snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
             return cudaErrorInvalidValue;
         }
-        // one store box covers the whole 64-channel output row (wide epilogue)
-        const bool oky = halo ? encode_y_3d(&maps[1], s, out, 64, prm.R * s.Wo)
-                              : encode_y_2d(&maps[1], s, out, 64);
-        if (!oky) {
-            snprintf(err, errlen, "tensor-map encode failed for the output tensor");
-            return cudaErrorInvalidValue;
-        }
-        for (int l = 2; l < 6; ++l) maps[l] = maps[0];
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
@@ -725,17 +701,17 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         auto kern = qconv_ws_kernel<true, 3>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h3);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else if (halo) {
         auto kern = qconv_ws_kernel<true, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else {
         auto kern = qconv_ws_kernel<false, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], maps[1], prm);
+        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     }
     return cudaGetLastError();
 }
@@ -761,13 +737,13 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     prm.box_bytes = prm.boxg * 16 * prm.group;
     prm.box_stride = prm.box_bytes;
     prm.stage_bytes = (s.kh * prm.box_stride + 1023) & ~1023;
-    int stages = GaCfg::RING_BYTES / prm.stage_bytes;
-    if (stages > MAX_STAGES) stages = MAX_STAGES;
-    if (stages < 2 || s.kh * prm.nsp > GA_MAX_UNITS || prm.boxg > 256 || s.kh > 256) {
+    int per = GaCfg::RING_BYTES / prm.stage_bytes / ISSUERS;
+    if (per > GaCfg::MAX_PER) per = GaCfg::MAX_PER;
+    if (per < 1 || s.kh * prm.nsp > GA_MAX_UNITS || prm.boxg > 256 || s.kh > 256) {
         snprintf(err, errlen, "pixel-pair kernel: kh=%d kw=%d does not fit", s.kh, s.kw);
         return cudaErrorInvalidValue;
     }
-    prm.stages = stages;
+    prm.per = per;
     prm.segs = (s.Wo + GA_TILE_W - 1) / GA_TILE_W;
     const long long rows = static_cast<long long>(s.N) * s.Ho;
     const long long tiles = rows * prm.segs;

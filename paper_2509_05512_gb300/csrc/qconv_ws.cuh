@@ -17,6 +17,18 @@
 //            vertical offsets dh are descriptor offsets of dh * Wo rows into that box,
 //            so kw boxes replace kh * kw.
 //   per tap  otherwise: one im2col box of 128 pixels per filter tap.
+//
+// Roles (12 warps):
+//   warp 0       TMA producer: the K blocks of each group of ISSUERS consecutive local
+//                tiles interleaved (block 0 of each tile, then block 1, ...), each into
+//                the next stage of the issuer that owns the tile.
+//   warps 1..3   MMA issuers taking the CTA's local tiles round robin, each waiting only
+//                for its own stages and accumulator buffers (issuer_stage, issuer_acc in
+//                tc_common.cuh; the tensor pipe keeps almost no queue and an issuing
+//                thread's own waits and branches cost hundreds of cycles while its MMAs
+//                are in flight).  Warp 1 owns TMEM.
+//   warps 2..11  expand the signed block weight once per CTA; then warps 4..11 run the
+//                shared-memory-free direct epilogue (tc_common.cuh).
 
 constexpr int WS_ROW_BYTES = 128;  // 64 channels x bf16: all four components of a pixel
 
@@ -24,6 +36,7 @@ struct WsParams {
     ConvShape s;
     EpilogueArgs ep;
     const __nv_bfloat16* w[4];  // compact letter tensors [16][kh][kw][16]
+    void* y;                    // output [N][Ho][Wo][64]
     unsigned long long wait_limit_ns;
     int inject_stall;
     int taps;         // kh * kw
@@ -33,31 +46,27 @@ struct WsParams {
     int kblocks;      // K blocks per tile: kw (halo) or taps
     int box_bytes;    // pixel box of one K block
     int stage_bytes;  // box rounded up to the 1024-byte swizzle period
-    int stages;       // ring depth (<= MAX_STAGES)
+    int per;          // stages owned by each issuer
     int num_tiles;
 };
 
 struct WsCfg {
     static constexpr int TAP_BYTES = 64 * WS_ROW_BYTES;  // expanded weight of one tap
     static constexpr int WSB_BYTES = WS_MAX_TAPS * TAP_BYTES;
-    using E = EpiSmem<16, true>;
-    // accumulator buffers in TMEM: enough that neither the MMAs' completion latency nor
-    // the epilogue's turnaround stalls the MMA issue
-    static constexpr int NACC = 4;
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * NACC + 2;  // full, empty, accf, acce, drain, wsready
-    static constexpr int TAIL_BYTES =
-        WSB_BYTES + E::STAGING_BYTES + E::PARAM_BYTES + NUM_BARS * 8 + 16;
+    static constexpr int MAX_PER = 4;                // stages per issuer at most
+    static constexpr int NSTAGE = ISSUERS * MAX_PER;  // stage barriers
+    // full, empty, accf, acce, drain (one per issuer), wsready
+    static constexpr int NUM_BARS = 2 * NSTAGE + 2 * ISSUER_ACC + ISSUERS + 1;
+    static constexpr int TAIL_BYTES = WSB_BYTES + NUM_BARS * 8 + 16;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr int RING_BYTES = ((SMEM_BYTES - 1024 - TAIL_BYTES) / 1024) * 1024;
     static constexpr int WSB_OFF = RING_BYTES;
-    static constexpr int STAGING_OFF = WSB_OFF + WSB_BYTES;
-    static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
-    static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
-    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
+    static constexpr int BAR_OFF = WSB_OFF + WSB_BYTES;
     static constexpr uint32_t DESC_HI = desc_hi(8 * WS_ROW_BYTES, desc_layout(WS_ROW_BYTES));
-    static constexpr uint32_t TMEM_COLS = 64 * NACC;
-    static constexpr int EXP_WARPS = 9;          // warps 2, 4..11 expand the weight
+    static constexpr uint32_t TMEM_COLS = 512;  // ISSUER_ACC buffers of 64 columns
+    static constexpr int EXP_WARPS = 10;  // warps 2..11 expand the weight
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "WS shared memory");
+    static_assert(4 * WS_MAX_TAPS * 32 <= 4 * EXP_WARPS * 32, "expansion in four rounds");
 };
 
 bool ws_halo_ok(const ConvShape& s) {
@@ -65,16 +74,59 @@ bool ws_halo_ok(const ConvShape& s) {
     const int R = BM / s.Wo;
     const long long box = static_cast<long long>(s.Wo) * (R + s.kh - 1) * WS_ROW_BYTES;
     const long long stage = (box + 1023) & ~1023LL;
-    return 2 * stage <= WsCfg::RING_BYTES;
+    return ISSUERS * stage <= WsCfg::RING_BYTES;
+}
+
+// Weight expansion by warps 2..11: for tap t, row n = (q, co) and K index k = (p, ci) the
+// value is sign(q, p) * W_{q xor p}[co][t][ci], rows of 128 bytes, 128-byte swizzle.  Each
+// 16-byte chunk of a compact letter L is read once from global memory (all of a thread's
+// chunks in flight together) and written to its four places (p = 0..3, q = L xor p).
+__device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int warp,
+                                          int lane, uint32_t wsready_bar) {
+    using C = WsCfg;
+    const int et = (warp - 2) * 32 + lane;  // 0 .. 319
+    constexpr int ET = C::EXP_WARPS * 32;
+    const int taps = p.taps;
+    const int letter_chunks = taps * 32;  // 16-byte chunks of one letter (16 x taps x 16)
+    const int total = 4 * letter_chunks;
+    uint4 v[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        const int i = et + r * ET;
+        if (i < total) {
+            const int L = i / letter_chunks;
+            v[r] = __ldg(reinterpret_cast<const uint4*>(p.w[L]) + (i - L * letter_chunks));
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        const int i = et + r * ET;
+        if (i >= total) continue;
+        const int L = i / letter_chunks, off = i - L * letter_chunks;
+        // chunk `off` of letter L holds W_L[co][t][ci0 .. ci0 + 7]
+        const int co = off / (taps * 2), rem = off - co * (taps * 2);
+        const int t = rem >> 1, half_ci = rem & 1;
+#pragma unroll
+        for (int pc = 0; pc < 4; ++pc) {
+            const int q = L ^ pc;
+            const int n = q * 16 + co, ch = pc * 2 + half_ci;
+            const uint4 u = ((NEG_MASK >> (4 * q + pc)) & 1u) ? negate_bf16x8(v[r]) : v[r];
+            *reinterpret_cast<uint4*>(smem + C::WSB_OFF + t * C::TAP_BYTES + n * WS_ROW_BYTES +
+                                      ((ch ^ (n & 7)) << 4)) = u;
+        }
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(wsready_bar);
 }
 
 // KH > 0: the filter height, known at compile time (halo staging), so the MMA issue
 // loop is fully unrolled; 0 = from the shape at run time.
 template <bool HALO, int KH>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x,
-                    const __grid_constant__ CUtensorMap tmap_y, const WsParams p) {
+    qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x, const WsParams p) {
     using C = WsCfg;
+    constexpr int NI = ISSUERS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -84,35 +136,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (MAX_STAGES + s); };
-    const uint32_t accf0 = bar0 + 8u * (2 * MAX_STAGES);
-    const uint32_t acce0 = bar0 + 8u * (2 * MAX_STAGES + C::NACC);
-    const uint32_t drain_bar = bar0 + 8u * (2 * MAX_STAGES + 2 * C::NACC);
-    const uint32_t wsready_bar = drain_bar + 8u;
+    auto empty_bar = [&](int s) { return bar0 + 8u * (C::NSTAGE + s); };
+    const uint32_t accf0 = bar0 + 8u * (2 * C::NSTAGE);
+    const uint32_t acce0 = bar0 + 8u * (2 * C::NSTAGE + ISSUER_ACC);
+    const uint32_t drain0 = bar0 + 8u * (2 * C::NSTAGE + 2 * ISSUER_ACC);
+    const uint32_t wsready_bar = drain0 + 8u * NI;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
     const uint64_t limit = p.wait_limit_ns;
-    const int STAGES = p.stages;
+    const int STAGES = NI * p.per;
+    // this CTA's local tiles: blockIdx.x + k * gridDim.x, k < kt
+    const int kt = (p.num_tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                   static_cast<int>(gridDim.x);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(full_bar(i), 1);
             mbar_init(empty_bar(i), 1);
         }
-        for (int b = 0; b < C::NACC; ++b) {
+        for (int b = 0; b < ISSUER_ACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
-            mbar_init(acce0 + 8u * b, 8 * 32);
+            mbar_init(acce0 + 8u * b, EPI2_ACCE_COUNT);
         }
-        mbar_init(drain_bar, 1);
+        for (int i = 0; i < NI; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(wsready_bar, C::EXP_WARPS);
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&tmap_x);
-        tma_prefetch_desc(&tmap_y);
-    }
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap_x);
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
         tmem_relinquish();
@@ -122,41 +174,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const int hw = s.Ho * s.Wo;
+    // pixel rows of a tile: halo -> (image, first input row); per tap -> first pixel
+    auto tile_base = [&](int tile, int& img, int& hbase, int& wbase) {
+        if constexpr (HALO) {
+            img = tile / p.tpi;
+            const int r0 = (tile - img * p.tpi) * p.R;
+            hbase = r0 - s.pad;
+            wbase = -s.pad;
+        } else {
+            const long long m0 = static_cast<long long>(tile) * BM;
+            img = static_cast<int>(m0 / hw);
+            const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
+            const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
+            wbase = wo * s.stride - s.pad;
+            hbase = ho * s.stride - s.pad;
+        }
+    };
 
-    if (warp == 0 || warp == 3) {
-        // ------------------------------------------------------------ TMA producers
-        // the two producer threads take alternate K blocks
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
-            const int role = warp == 0 ? 0 : 1;
             const uint64_t pol_x = l2_policy_evict_normal();
-            int stage = 0;
-            uint32_t phase = 0;
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
-            int kb_all = 0;
-            // pixel rows of a tile: halo -> (image, first input row); per tap -> first pixel
-            auto tile_base = [&](int tile, int& img, int& hbase, int& wbase) {
-                if constexpr (HALO) {
-                    img = tile / p.tpi;
-                    const int r0 = (tile - img * p.tpi) * p.R;
-                    hbase = r0 - s.pad;
-                    wbase = -s.pad;
-                } else {
-                    const long long m0 = static_cast<long long>(tile) * BM;
-                    img = static_cast<int>(m0 / hw);
-                    const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
-                    const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
-                    wbase = wo * s.stride - s.pad;
-                    hbase = ho * s.stride - s.pad;
-                }
-            };
             // Cold pixels come from DRAM with a latency far above what the ring covers, so
-            // the first producer asks L2 for this CTA's tiles PF tiles ahead of the ring.
-            constexpr int PF = 2;
-            auto prefetch_tile = [&](int tile) {
-                if (role != 0 || tile >= p.num_tiles) return;
+            // the producer asks L2 for the tiles two groups ahead.
+            auto prefetch_tile = [&](int k) {
+                if (k >= kt) return;
                 int pimg, ph, pw;
-                tile_base(tile, pimg, ph, pw);
+                tile_base(static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x), pimg, ph, pw);
                 if constexpr (HALO)
                     tma_prefetch_l2_4d(&tmap_x, 0, pw + s.pad, ph, pimg);
                 else
@@ -164,13 +210,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                               static_cast<uint16_t>(s.kw / 2),
                                               static_cast<uint16_t>(s.kh / 2));
             };
-            for (int k = 0; k < PF; ++k) prefetch_tile(blockIdx.x + k * gridDim.x);
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
-                int img, hbase, wbase;
-                tile_base(tile, img, hbase, wbase);
-                prefetch_tile(tile + PF * gridDim.x);
-                for (int kb = 0; kb < p.kblocks; ++kb, ++kb_all) {
-                    if ((kb_all & 1) == role) {
+            for (int k = 0; k < 2 * NI; ++k) prefetch_tile(k);
+            for (int g0 = 0; ok && g0 < kt; g0 += NI) {
+                const int ng = kt - g0 < NI ? kt - g0 : NI;
+                for (int k = g0 + 2 * NI; k < g0 + 3 * NI; ++k) prefetch_tile(k);
+                int img[NI], hbase[NI], wbase[NI];
+#pragma unroll
+                for (int i = 0; i < NI; ++i)
+                    if (i < ng)
+                        tile_base(static_cast<int>(blockIdx.x) + (g0 + i) * static_cast<int>(gridDim.x),
+                                  img[i], hbase[i], wbase[i]);
+                for (int kb = 0; ok && kb < p.kblocks; ++kb) {
+#pragma unroll
+                    for (int i = 0; i < NI; ++i) {
+                        if (i >= ng) break;
+                        // K block kb of local tile g0 + i: use (g0 / NI) * kblocks + kb of issuer i
+                        int stage;
+                        uint32_t phase;
+                        issuer_stage(i, (g0 / NI) * p.kblocks + kb, p.per, stage, phase);
                         if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                            STATUS_TIMEOUT_PRODUCER)) {
                             ok = false;
@@ -183,42 +240,40 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         const uint32_t dst = sbase + stage * p.stage_bytes;
                         if constexpr (HALO) {
                             // K block kb = horizontal filter offset dw
-                            tma_load_4d(dst, &tmap_x, fb, 0, wbase + kb, hbase, img, pol_x);
+                            tma_load_4d(dst, &tmap_x, fb, 0, wbase[i] + kb, hbase[i], img[i], pol_x);
                         } else {
                             const int dh = kb / s.kw, dw = kb - (kb / s.kw) * s.kw;
-                            tma_load_im2col_4d(dst, &tmap_x, fb, 0, wbase, hbase, img,
+                            tma_load_im2col_4d(dst, &tmap_x, fb, 0, wbase[i], hbase[i], img[i],
                                                static_cast<uint16_t>(dw),
                                                static_cast<uint16_t>(dh), pol_x);
                         }
-                    }
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
                     }
                 }
             }
             if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
+    } else if (warp <= NI) {
+        // ------------------------------------------------------------ MMA issuers
+        if (warp >= 2) ws_expand(p, smem, warp, lane, wsready_bar);
         if (lane == 0) {
             constexpr uint32_t IDESC = make_idesc(BM, 64, 0);
-            int stage = 0;
-            uint32_t phase = 0;
+            const int me = warp - 1;
+            const uint32_t drain_bar = drain0 + 8u * me;
             bool ok = wait_or_abort(wsready_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
             int issued = 0;
-            if (p.inject_stall) {
+            if (p.inject_stall && me == 0) {
                 // Failure injection: wait on a barrier nothing arrives on.
                 wait_or_abort(drain_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
                 ok = false;
             }
             tc_fence_after();
             const uint32_t wsb_lo = desc_lo(sbase + C::WSB_OFF);
-            int local = 0;
             const uint32_t row_lo = (s.Wo * WS_ROW_BYTES) >> 4;  // one output row of pixels
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
-                const int buf = local % C::NACC;
-                const uint32_t use = static_cast<uint32_t>(local / C::NACC) & 1u;
+            const uint32_t b_row = (s.kw * C::TAP_BYTES) >> 4;    // one filter row of taps
+            for (int k = me, j = 0; ok && k < kt; k += NI, ++j) {
+                int buf;
+                uint32_t use;
+                issuer_acc(k, buf, use);
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA)) {
                     ok = false;
@@ -227,6 +282,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * 64);
                 for (int kb = 0; kb < p.kblocks; ++kb) {
+                    int stage;
+                    uint32_t phase;
+                    issuer_stage(me, j * p.kblocks + kb, p.per, stage, phase);
                     if (!wait_or_abort(full_bar(stage), phase, limit, abort_flag,
                                        STATUS_TIMEOUT_MMA)) {
                         ok = false;
@@ -236,7 +294,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     const uint32_t a_lo0 = desc_lo(sbase + stage * p.stage_bytes);
                     if constexpr (HALO && KH > 0) {
                         const uint32_t b_lo0 = wsb_lo + ((kb * C::TAP_BYTES) >> 4);
-                        const uint32_t b_row = (s.kw * C::TAP_BYTES) >> 4;
 #pragma unroll
                         for (int dh = 0; dh < KH; ++dh) {
 #pragma unroll
@@ -248,12 +305,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     } else if constexpr (HALO) {
                         for (int dh = 0; dh < s.kh; ++dh) {
                             const int tap = dh * s.kw + kb;
-                            const uint32_t a_lo = a_lo0 + dh * row_lo;
                             const uint32_t b_lo = wsb_lo + ((tap * C::TAP_BYTES) >> 4);
 #pragma unroll
                             for (int pc = 0; pc < 4; ++pc)
-                                umma_f16_w(d, a_lo + pc * 2, C::DESC_HI, b_lo + pc * 2,
-                                           C::DESC_HI, IDESC, (kb | dh | pc) != 0 ? 1u : 0u);
+                                umma_f16_w(d, a_lo0 + dh * row_lo + pc * 2, C::DESC_HI,
+                                           b_lo + pc * 2, C::DESC_HI, IDESC,
+                                           (kb | dh | pc) != 0 ? 1u : 0u);
                         }
                     } else {
                         const uint32_t b_lo = wsb_lo + ((kb * C::TAP_BYTES) >> 4);
@@ -264,15 +321,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                     ++issued;
                     umma_commit(empty_bar(stage));
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
                 }
                 if (!ok) break;
                 umma_commit(accf0 + 8u * buf);
             }
             if (!ok && issued > 0) {
+                // let this issuer's MMAs finish before TMEM is released
                 umma_commit(drain_bar);
                 const uint64_t t0 = global_timer_ns();
                 while (!mbar_try_wait(drain_bar, 0u)) {
@@ -284,63 +338,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
         }
     } else {
-        // ------------------------------------------------------------ weight expansion
-        // warps 2 and 4..11 write the signed block weight: for tap t, row n = (q, co) and K
-        // index k = (p, ci) the value is sign(q, p) * W_{q xor p}[co][t][ci], rows of 128
-        // bytes, 128-byte swizzle.  Each 16-byte chunk of a compact letter L is read once
-        // from global memory and written to its four places (p = 0..3, q = L xor p).
-        const int et = warp == 2 ? lane : (warp - 3) * 32 + lane;  // 0 .. 287
-        constexpr int ET = C::EXP_WARPS * 32;
-        const int taps = p.taps;
-        const int letter_chunks = taps * 32;  // 16-byte chunks of one letter (16 x taps x 16)
-        for (int i = et; i < 4 * letter_chunks; i += ET) {
-            const int L = i / letter_chunks, off = i - L * letter_chunks;
-            const uint4 v = __ldg(reinterpret_cast<const uint4*>(p.w[L]) + off);
-            // chunk `off` of letter L holds W_L[co][t][ci0 .. ci0 + 7]
-            const int co = off / (taps * 2), rem = off - co * (taps * 2);
-            const int t = rem >> 1, half_ci = rem & 1;
-#pragma unroll
-            for (int pc = 0; pc < 4; ++pc) {
-                const int q = L ^ pc;
-                const int n = q * 16 + co, ch = pc * 2 + half_ci;
-                const uint4 u = ((NEG_MASK >> (4 * q + pc)) & 1u) ? negate_bf16x8(v) : v;
-                *reinterpret_cast<uint4*>(smem + C::WSB_OFF + t * C::TAP_BYTES +
-                                          n * WS_ROW_BYTES + ((ch ^ (n & 7)) << 4)) = u;
+        ws_expand(p, smem, warp, lane, wsready_bar);
+        // -------------------------------------------------------- epilogue (warps 4..11)
+        const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
+        const long long M = s.M;
+        auto geo = [tpi, R, Ho, Wo, M](int tile) {
+            EpiTile g;
+            g.n_tile = 0;
+            if constexpr (HALO) {
+                const int img = tile / tpi;
+                const int r0 = (tile - img * tpi) * R;
+                g.m0 = (static_cast<long long>(img) * Ho + r0) * Wo;
+                const int nr = Ho - r0 < R ? Ho - r0 : R;
+                g.rows = nr * Wo;
+            } else {
+                g.m0 = static_cast<long long>(tile) * BM;
+                const long long left = M - g.m0;
+                g.rows = left < BM ? static_cast<int>(left) : BM;
             }
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(wsready_bar);
-
-        if (warp >= EPI_WARP0) {
-            // -------------------------------------------------------- epilogue
-            const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
-            const long long M = s.M;
-            auto geo = [tpi, R, Ho, Wo, M](int tile) {
-                    EpiTile g;
-                    g.n_tile = 0;
-                    if constexpr (HALO) {
-                        const int img = tile / tpi;
-                        const int r0 = (tile - img * tpi) * R;
-                        g.m0 = (static_cast<long long>(img) * Ho + r0) * Wo;
-                        const int nr = Ho - r0 < R ? Ho - r0 : R;
-                        g.rows = nr * Wo;
-                        g.sy = r0 * Wo;
-                        g.sz = img;
-                    } else {
-                        g.m0 = static_cast<long long>(tile) * BM;
-                        const long long left = M - g.m0;
-                        g.rows = left < BM ? static_cast<int>(left) : BM;
-                        g.sy = static_cast<int>(g.m0);
-                        g.sz = 0;
-                    }
-                    return g;
-                };
-            epilogue_role<16, HALO, decltype(geo), true, 2, C::NACC>(
-                s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
-                reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
-                abort_flag, geo);
-        }
+            g.sy = g.sz = 0;
+            return g;
+        };
+        epilogue_direct64<decltype(geo)>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles,
+                                         limit, abort_flag, geo);
     }
 
     tc_fence_before();

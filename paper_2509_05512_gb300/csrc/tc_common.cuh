@@ -330,8 +330,32 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
 //      Eq. 11-12) with the 8 channels' vectors held in registers, rounds to bf16 and
 //      writes 16 bytes per lane per row: every store instruction writes four whole
 //      128-byte output rows, the residual is read the same way.
-// Accumulator buffers are used round robin over NACC.
+// Accumulator buffers follow issuer_acc.
 constexpr int EPI2_ACCE_COUNT = 128;
+
+// Tiles of a CTA are issued round robin by ISSUERS threads (local tile k by issuer
+// k % ISSUERS).  mbarrier parity waits only tell a phase from its neighbours, so a waiter
+// must never get two phases ahead of a barrier; that is guaranteed by letting every stage
+// and accumulator buffer be used by one issuer only, whose program order then orders the
+// uses:
+//   - issuer i owns stages i * per .. i * per + per - 1; its n-th stage use (counting its
+//     K blocks in order) is stage i * per + n % per in round n / per;
+//   - issuer i owns accumulator buffers i and i + ISSUERS, alternating over its tiles;
+//     a buffer's tiles all have the same parity, so one epilogue group drains it.
+constexpr int ISSUERS = 3;
+constexpr int ISSUER_ACC = 2 * ISSUERS;  // accumulator buffers in use
+
+__device__ __forceinline__ void issuer_stage(int i, int n, int per, int& stage,
+                                             uint32_t& phase) {
+    stage = i * per + n % per;
+    phase = static_cast<uint32_t>(n / per) & 1u;
+}
+
+__device__ __forceinline__ void issuer_acc(int k, int& buf, uint32_t& use) {
+    const int j = k / ISSUERS;
+    buf = (k - j * ISSUERS) + ISSUERS * (j & 1);
+    use = static_cast<uint32_t>(j >> 1) & 1u;
+}
 
 // One transpose stage: lanes i and i ^ K exchange the chunks whose index differs from the
 // lane in bit K (E[j] for bit_K(j) != bit_K(i), partner's E[j ^ K] in return).
@@ -353,7 +377,7 @@ __device__ __forceinline__ void chunk_transpose_stage(float (&E)[8][8], int i) {
     }
 }
 
-template <typename Geo, int NACC>
+template <typename Geo>
 __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const EpilogueArgs& ep,
                                                   void* y, uint32_t tmem_base, uint32_t accf0,
                                                   uint32_t acce0, int num_tiles, uint64_t limit,
@@ -377,8 +401,9 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
     int local = grp;
     for (int tile = blockIdx.x + grp * gridDim.x; tile < num_tiles;
          tile += 2 * gridDim.x, local += 2) {
-        const int buf = local % NACC;
-        const uint32_t use = static_cast<uint32_t>(local / NACC) & 1u;
+        int buf;
+        uint32_t use;
+        issuer_acc(local, buf, use);
         bool ok = true;
         if (lane == 0)
             ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
