@@ -35,10 +35,10 @@
 //                 are in flight, so three issuers are needed to keep the pipe busy.  Each
 //                 issuer owns its stages and two accumulator buffers (issuer_stage,
 //                 issuer_acc in tc_common.cuh).  Warp 1 also owns TMEM.
-//   warps 2..11   expand the signed block weight of Eq. 6 once per CTA:
+//   warps 2..15   expand the signed block weight of Eq. 6 once per CTA:
 //                 B[(q, co)][(ky, pair, e, p)] = sign(q, p) W_{q xor p}[co][ky][2 pair - lead + e]
 //                 (zero outside the filter), K-major with a 32-byte swizzle; then warps
-//                 4..11 run the direct epilogue (tc_common.cuh: no shared memory, coalesced
+//                 4..15 run the direct epilogue (tc_common.cuh: no shared memory, coalesced
 //                 global stores, columns past the end of the output row not stored).
 // The zero-weight columns read real input pixels, which only matters for non-finite
 // inputs (0 * inf); finite inputs give exactly the convolution of Eq. 5.
@@ -87,7 +87,7 @@ struct GaCfg {
     static constexpr uint32_t A_DESC_HI = desc_hi(8 * 16, 0);
     static constexpr uint32_t B_DESC_HI = desc_hi(8 * 32, desc_layout(32));
     static constexpr uint32_t TMEM_COLS = 512;  // ISSUER_ACC buffers of 64 columns
-    static constexpr int EXP_WARPS = 10;        // warps 2..11
+    static constexpr int EXP_WARPS = 14;        // warps 2..15
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "gather shared memory");
 };
 
@@ -98,7 +98,7 @@ int gather_nsp(const ConvShape& s) {
     return nsp + (nsp & 1);
 }
 
-// Weight expansion, run by warps 2..11 (EXP_WARPS): the signed block weight of Eq. 6 as
+// Weight expansion, run by warps 2..15 (EXP_WARPS): the signed block weight of Eq. 6 as
 // K-major rows of 32-byte K steps with a 32-byte swizzle,
 //   B[(q, co)][(ky, pair j, pixel e, component p)] = sign(q, p) W_{q xor p}[co][ky][2 j - lead + e]
 // (zero outside the filter).  The four letter tensors are first copied to shared memory
@@ -120,7 +120,7 @@ __device__ __forceinline__ void expand_block_weight(const ConvShape& s, const Ga
                                                     uint8_t* smem, int warp, int lane,
                                                     uint32_t bready_bar) {
     using C = GaCfg;
-    const int et = (warp - 2) * 32 + lane;  // 0 .. 319
+    const int et = (warp - 2) * 32 + lane;  // 0 .. 447
     constexpr int ET = C::EXP_WARPS * 32;
     const int taps = s.kh * s.kw;
     // 1. letters [16][kh][kw][1] -> shared memory, 2 * taps 16-byte chunks per letter
@@ -189,7 +189,7 @@ __device__ __forceinline__ void expand_block_weight(const ConvShape& s, const Ga
 // MMA issue loop is fully unrolled with constant descriptor offsets; 0 = from the
 // parameters at run time.
 template <int KH, int NSP>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_pairs_kernel(const __grid_constant__ CUtensorMap tmap_x, const GatherParams p) {
     using C = GaCfg;
     extern __shared__ uint8_t smem_raw[];

@@ -701,17 +701,17 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         auto kern = qconv_ws_kernel<true, 3>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h3);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else if (halo) {
         auto kern = qconv_ws_kernel<true, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else {
         auto kern = qconv_ws_kernel<false, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     }
     return cudaGetLastError();
 }
@@ -770,12 +770,12 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         auto kern = qconv_pairs_kernel<7, 4>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        kern<<<grid, WIDE_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     } else {
         auto kern = qconv_pairs_kernel<0, 0>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_any);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        kern<<<grid, WIDE_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
     }
     return cudaGetLastError();
 }

@@ -18,7 +18,7 @@
 //            so kw boxes replace kh * kw.
 //   per tap  otherwise: one im2col box of 128 pixels per filter tap.
 //
-// Roles (12 warps):
+// Roles (16 warps):
 //   warp 0       TMA producer: the K blocks of each group of ISSUERS consecutive local
 //                tiles interleaved (block 0 of each tile, then block 1, ...), each into
 //                the next stage of the issuer that owns the tile.
@@ -27,7 +27,7 @@
 //                tc_common.cuh; the tensor pipe keeps almost no queue and an issuing
 //                thread's own waits and branches cost hundreds of cycles while its MMAs
 //                are in flight).  Warp 1 owns TMEM.
-//   warps 2..11  expand the signed block weight once per CTA; then warps 4..11 run the
+//   warps 2..15  expand the signed block weight once per CTA; then warps 4..15 run the
 //                shared-memory-free direct epilogue (tc_common.cuh).
 
 constexpr int WS_ROW_BYTES = 128;  // 64 channels x bf16: all four components of a pixel
@@ -64,7 +64,7 @@ struct WsCfg {
     static constexpr int BAR_OFF = WSB_OFF + WSB_BYTES;
     static constexpr uint32_t DESC_HI = desc_hi(8 * WS_ROW_BYTES, desc_layout(WS_ROW_BYTES));
     static constexpr uint32_t TMEM_COLS = 512;  // ISSUER_ACC buffers of 64 columns
-    static constexpr int EXP_WARPS = 10;  // warps 2..11 expand the weight
+    static constexpr int EXP_WARPS = 14;  // warps 2..15 expand the weight
     static_assert(BAR_OFF + NUM_BARS * 8 + 16 + 1024 <= SMEM_BYTES, "WS shared memory");
     static_assert(4 * WS_MAX_TAPS * 32 <= 4 * EXP_WARPS * 32, "expansion in four rounds");
 };
@@ -77,14 +77,14 @@ bool ws_halo_ok(const ConvShape& s) {
     return ISSUERS * stage <= WsCfg::RING_BYTES;
 }
 
-// Weight expansion by warps 2..11: for tap t, row n = (q, co) and K index k = (p, ci) the
+// Weight expansion by warps 2..15: for tap t, row n = (q, co) and K index k = (p, ci) the
 // value is sign(q, p) * W_{q xor p}[co][t][ci], rows of 128 bytes, 128-byte swizzle.  Each
 // 16-byte chunk of a compact letter L is read once from global memory (all of a thread's
 // chunks in flight together) and written to its four places (p = 0..3, q = L xor p).
 __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int warp,
                                           int lane, uint32_t wsready_bar) {
     using C = WsCfg;
-    const int et = (warp - 2) * 32 + lane;  // 0 .. 319
+    const int et = (warp - 2) * 32 + lane;  // 0 .. 447
     constexpr int ET = C::EXP_WARPS * 32;
     const int taps = p.taps;
     const int letter_chunks = taps * 32;  // 16-byte chunks of one letter (16 x taps x 16)
@@ -123,7 +123,7 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
 // KH > 0: the filter height, known at compile time (halo staging), so the MMA issue
 // loop is fully unrolled; 0 = from the shape at run time.
 template <bool HALO, int KH>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+__global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x, const WsParams p) {
     using C = WsCfg;
     constexpr int NI = ISSUERS;
@@ -197,23 +197,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint64_t pol_x = l2_policy_evict_normal();
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
-            // Cold pixels come from DRAM with a latency far above what the ring covers, so
-            // the producer asks L2 for the tiles two groups ahead.
-            auto prefetch_tile = [&](int k) {
-                if (k >= kt) return;
-                int pimg, ph, pw;
-                tile_base(static_cast<int>(blockIdx.x) + k * static_cast<int>(gridDim.x), pimg, ph, pw);
-                if constexpr (HALO)
-                    tma_prefetch_l2_4d(&tmap_x, 0, pw + s.pad, ph, pimg);
-                else
-                    tma_prefetch_l2_im2col_4d(&tmap_x, 0, pw, ph, pimg,
-                                              static_cast<uint16_t>(s.kw / 2),
-                                              static_cast<uint16_t>(s.kh / 2));
-            };
-            for (int k = 0; k < 2 * NI; ++k) prefetch_tile(k);
             for (int g0 = 0; ok && g0 < kt; g0 += NI) {
                 const int ng = kt - g0 < NI ? kt - g0 : NI;
-                for (int k = g0 + 2 * NI; k < g0 + 3 * NI; ++k) prefetch_tile(k);
                 int img[NI], hbase[NI], wbase[NI];
 #pragma unroll
                 for (int i = 0; i < NI; ++i)
@@ -339,7 +324,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
     } else {
         ws_expand(p, smem, warp, lane, wsready_bar);
-        // -------------------------------------------------------- epilogue (warps 4..11)
+        // -------------------------------------------------------- epilogue (warps 4..15)
         const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
         const long long M = s.M;
         auto geo = [tpi, R, Ho, Wo, M](int tile) {

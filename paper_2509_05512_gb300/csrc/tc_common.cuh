@@ -317,21 +317,23 @@ __device__ __forceinline__ void epilogue_role(const ConvShape& s, const Epilogue
 }
 
 // Direct epilogue for 64-channel outputs (Qout = 16: one output-channel tile), used by the
-// weight-stationary and pixel-pair kernels.  The tensor cores' operand reads keep the
-// shared-memory pipe saturated, so this epilogue touches no shared memory: each of the 8
-// warps works on its own, warps 4..7 on the CTA's even local tiles and 8..11 on the odd
-// ones, each warp on the 32 TMEM lanes (output pixels) of its quadrant.  Per tile a warp
-//   1. loads its 32 rows x 64 columns (4 components x 16 channels) with two 32-column
-//      tcgen05.ld and releases the accumulator buffer (acce, 128 arrivals per tile);
-//   2. transposes, within each group of 8 lanes, the 8 x 8 matrix of 8-channel chunks
-//      (rows x chunks) with three shfl_xor stages, so lane i of group g holds channels
-//      8i .. 8i+7 of the group's 8 rows;
+// weight-stationary and pixel-pair kernels (16 warps: producer, 3 issuers, 12 epilogue).
+// The tensor cores' operand reads keep the shared-memory pipe saturated, so this epilogue
+// touches no shared memory.  Warps 4..15 form three groups of four (one warp per TMEM lane
+// quadrant); group g takes the CTA's local tiles k with k % 3 == g, the tiles issuer g
+// produced, so three tiles are in flight.  Per tile and per 32-channel half a warp
+//   1. loads its 32 rows x 32 columns with one tcgen05.ld (once the second half is in
+//      registers it releases the accumulator buffer, acce, 128 arrivals per tile);
+//   2. transposes, within each group of 4 lanes, the 4 x 4 matrix of 8-channel chunks
+//      (rows x chunks) with two shfl_xor stages, so lane i of lane group r holds
+//      channels 32 half + 8i .. +7 of that group's 4 rows;
 //   3. applies act(scale * (acc + bias) + shift + residual) (IQBN inference form of
-//      Eq. 11-12) with the 8 channels' vectors held in registers, rounds to bf16 and
-//      writes 16 bytes per lane per row: every store instruction writes four whole
-//      128-byte output rows, the residual is read the same way.
-// Accumulator buffers follow issuer_acc.
-constexpr int EPI2_ACCE_COUNT = 128;
+//      Eq. 11-12) with its channels' vectors held in registers, rounds to bf16 and
+//      writes 16 bytes per lane per row: every store instruction writes 64-byte halves of
+//      8 whole output rows; the residual is read the same way.
+constexpr int EPI_GROUPS = 3;
+constexpr int WIDE_THREADS = 512;  // block size of the kernels using this epilogue
+constexpr int EPI2_ACCE_COUNT = 128;  // the 4 warps of one group arrive once per tile
 
 // Tiles of a CTA are issued round robin by ISSUERS threads (local tile k by issuer
 // k % ISSUERS).  mbarrier parity waits only tell a phase from its neighbours, so a waiter
@@ -359,11 +361,11 @@ __device__ __forceinline__ void issuer_acc(int k, int& buf, uint32_t& use) {
 
 // One transpose stage: lanes i and i ^ K exchange the chunks whose index differs from the
 // lane in bit K (E[j] for bit_K(j) != bit_K(i), partner's E[j ^ K] in return).
-template <int K>
-__device__ __forceinline__ void chunk_transpose_stage(float (&E)[8][8], int i) {
+template <int K, int NCH>
+__device__ __forceinline__ void chunk_transpose_stage(float (&E)[NCH][8], int i) {
     const bool hi = (i & K) != 0;
 #pragma unroll
-    for (int j0 = 0; j0 < 8; ++j0) {
+    for (int j0 = 0; j0 < NCH; ++j0) {
         if (j0 & K) continue;
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -382,25 +384,28 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
                                                   void* y, uint32_t tmem_base, uint32_t accf0,
                                                   uint32_t acce0, int num_tiles, uint64_t limit,
                                                   volatile int* abort_flag, Geo geo) {
+    static_assert(EPI_GROUPS == ISSUERS, "each epilogue group drains one issuer's buffers");
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int quad = warp & 3;                // TMEM lane quadrant this warp may access
-    const int grp = (warp - EPI_WARP0) >> 2;  // 0: even local tiles, 1: odd
-    const int ci = lane & 7;                  // this lane's 8-channel chunk after the transpose
-    const int rg = lane >> 3;                 // group of 8 rows (8 lanes) within the warp
-    // the chunk's per-channel vectors, in registers for the whole kernel
-    float sc[8], sh[8];
+    const int grp = (warp - EPI_WARP0) >> 2;  // local tiles k with k % 3 == grp
+    const int ci = lane & 3;                  // this lane's chunk after the transpose
+    const int rg = lane >> 2;                 // group of 4 rows (4 lanes) within the warp
+    // the chunks' per-channel vectors (channels 8 ci + 32 h + e), in registers
+    float sc[2][8], sh[2][8];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const int c = 8 * ci + e;
-        const float b = ep.bias ? __ldg(ep.bias + c) : 0.0f;
-        sc[e] = ep.scale ? __ldg(ep.scale + c) : 1.0f;
-        sh[e] = fmaf(sc[e], b, ep.scale ? __ldg(ep.shift + c) : 0.0f);
-    }
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int c = 32 * h + 8 * ci + e;
+            const float b = ep.bias ? __ldg(ep.bias + c) : 0.0f;
+            sc[h][e] = ep.scale ? __ldg(ep.scale + c) : 1.0f;
+            sh[h][e] = fmaf(sc[h][e], b, ep.scale ? __ldg(ep.shift + c) : 0.0f);
+        }
     const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(ep.residual);
     __nv_bfloat16* out = static_cast<__nv_bfloat16*>(y);
     int local = grp;
     for (int tile = blockIdx.x + grp * gridDim.x; tile < num_tiles;
-         tile += 2 * gridDim.x, local += 2) {
+         tile += EPI_GROUPS * gridDim.x, local += EPI_GROUPS) {
         int buf;
         uint32_t use;
         issuer_acc(local, buf, use);
@@ -411,60 +416,65 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
         tc_fence_after();
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                static_cast<uint32_t>(buf * 64);
-        uint32_t v[64];  // column (= output channel) c of this lane's row
-        tmem_ld_32x32b_x32(taddr, *reinterpret_cast<uint32_t(*)[32]>(v));
-        tmem_ld_32x32b_x32(taddr + 32, *reinterpret_cast<uint32_t(*)[32]>(v + 32));
         const EpiTile g = geo(tile);
-        // this lane's rows after the transpose: quad*32 + 8 rg + k, k = 0..7
-        const int row0 = quad * 32 + 8 * rg;
-        uint4 r4[8];
-        if (res != nullptr) {
+        // this lane's rows after the transpose: quad*32 + 4 rg + k, k = 0..3
+        const int row0 = quad * 32 + 4 * rg;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                r4[k] = make_uint4(0u, 0u, 0u, 0u);
-                if (row0 + k < g.rows)
-                    r4[k] = __ldg(reinterpret_cast<const uint4*>(res + (g.m0 + row0 + k) * 64 +
-                                                                 8 * ci));
+        for (int h = 0; h < 2; ++h) {
+            uint32_t v[32];  // channel 32 h + c of this lane's row
+            tmem_ld_32x32b_x32(taddr + 32 * h, v);
+            tmem_ld_wait();
+            if (h == 1) {
+                // the accumulator is in registers: hand the buffer back to the MMA issuer
+                tc_fence_before();
+                mbar_arrive(acce0 + 8u * buf);
             }
-        }
-        tmem_ld_wait();
-        // the accumulator is in registers: hand the buffer back to the MMA issuers
-        tc_fence_before();
-        mbar_arrive(acce0 + 8u * buf);
-        float E[8][8];  // E[j][e]: channel 8j + e of this lane's row
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-#pragma unroll
-            for (int e = 0; e < 8; ++e) E[j][e] = __uint_as_float(v[8 * j + e]);
-        chunk_transpose_stage<4>(E, ci);
-        chunk_transpose_stage<2>(E, ci);
-        chunk_transpose_stage<1>(E, ci);
-        // now E[k][e] = channel 8 ci + e of row row0 + k
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            float rz[8];
+            const int c0 = 32 * h + 8 * ci;
+            uint4 r4[4];
             if (res != nullptr) {
-                const __nv_bfloat162* rh = reinterpret_cast<const __nv_bfloat162*>(&r4[k]);
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    r4[k] = make_uint4(0u, 0u, 0u, 0u);
+                    if (row0 + k < g.rows)
+                        r4[k] = __ldg(
+                            reinterpret_cast<const uint4*>(res + (g.m0 + row0 + k) * 64 + c0));
+                }
+            }
+            float E[4][8];  // E[j][e]: channel 32 h + 8j + e of this lane's row
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+                for (int e = 0; e < 8; ++e) E[j][e] = __uint_as_float(v[8 * j + e]);
+            chunk_transpose_stage<2, 4>(E, ci);
+            chunk_transpose_stage<1, 4>(E, ci);
+            // now E[k][e] = channel c0 + e of row row0 + k
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                float rz[8];
+                if (res != nullptr) {
+                    const __nv_bfloat162* rh = reinterpret_cast<const __nv_bfloat162*>(&r4[k]);
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const float2 f = __bfloat1622float2(rh[t]);
+                        rz[2 * t] = f.x;
+                        rz[2 * t + 1] = f.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) rz[e] = 0.0f;
+                }
+                uint32_t w[4];
 #pragma unroll
                 for (int t = 0; t < 4; ++t) {
-                    const float2 f = __bfloat1622float2(rh[t]);
-                    rz[2 * t] = f.x;
-                    rz[2 * t + 1] = f.y;
+                    const float z0 = fmaf(sc[h][2 * t], E[k][2 * t], sh[h][2 * t]) + rz[2 * t];
+                    const float z1 =
+                        fmaf(sc[h][2 * t + 1], E[k][2 * t + 1], sh[h][2 * t + 1]) + rz[2 * t + 1];
+                    w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
                 }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) rz[e] = 0.0f;
+                if (row0 + k < g.rows)
+                    *reinterpret_cast<uint4*>(out + (g.m0 + row0 + k) * 64 + c0) =
+                        make_uint4(w[0], w[1], w[2], w[3]);
             }
-            uint32_t w[4];
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-                const float z0 = fmaf(sc[2 * t], E[k][2 * t], sh[2 * t]) + rz[2 * t];
-                const float z1 = fmaf(sc[2 * t + 1], E[k][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
-                w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
-            }
-            if (row0 + k < g.rows)
-                *reinterpret_cast<uint4*>(out + (g.m0 + row0 + k) * 64 + 8 * ci) =
-                    make_uint4(w[0], w[1], w[2], w[3]);
         }
     }
 }
