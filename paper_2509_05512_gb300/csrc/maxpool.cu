@@ -61,6 +61,50 @@ __global__ void __launch_bounds__(256) maxpool_kernel(const __nv_bfloat16* __res
     }
 }
 
+// One CTA per output row (n, ho); thread t covers column wo = t / cv and channels
+// 8 (t % cv) .. +7 (cv = C / 8), with a block-stride loop when Wo * cv exceeds the block.
+// All index arithmetic is 32-bit and done once per output; neighbouring columns share
+// their input columns through L1.
+__global__ void __launch_bounds__(512) maxpool_rows_kernel(const __nv_bfloat16* __restrict__ x,
+                                                           int H, int W, int C, int k,
+                                                           int stride, int pad, int Ho, int Wo,
+                                                           __nv_bfloat16* __restrict__ y) {
+    const int cv = C / 8;
+    const int row = blockIdx.x;  // n * Ho + ho
+    const int n = row / Ho, ho = row - (row / Ho) * Ho;
+    const uint4* xr = reinterpret_cast<const uint4*>(x) + static_cast<long long>(n) * H * W * cv;
+    uint4* yr = reinterpret_cast<uint4*>(y) + static_cast<long long>(row) * Wo * cv;
+    const int h0 = ho * stride - pad;
+    for (int t = threadIdx.x; t < Wo * cv; t += blockDim.x) {
+        const int wo = t / cv, c = t - (t / cv) * cv;
+        const int w0 = wo * stride - pad;
+        float m[8];
+#pragma unroll
+        for (int v = 0; v < 8; ++v) m[v] = -INFINITY;
+        for (int dh = 0; dh < k; ++dh) {
+            const int h = h0 + dh;
+            if (h < 0 || h >= H) continue;
+            for (int dw = 0; dw < k; ++dw) {
+                const int w = w0 + dw;
+                if (w < 0 || w >= W) continue;
+                const uint4 raw = __ldg(xr + (h * W + w) * cv + c);
+                const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
+#pragma unroll
+                for (int v = 0; v < 4; ++v) {
+                    const float2 f = __bfloat1622float2(b2[v]);
+                    m[2 * v] = fmaxf(m[2 * v], f.x);
+                    m[2 * v + 1] = fmaxf(m[2 * v + 1], f.y);
+                }
+            }
+        }
+        uint4 raw;
+        __nv_bfloat162* b2 = reinterpret_cast<__nv_bfloat162*>(&raw);
+#pragma unroll
+        for (int v = 0; v < 4; ++v) b2[v] = __floats2bfloat162_rn(m[2 * v], m[2 * v + 1]);
+        yr[t] = raw;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
@@ -77,6 +121,15 @@ cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k
     if (blocks > cap) blocks = cap;
     const auto* xb = static_cast<const __nv_bfloat16*>(x);
     auto* yb = static_cast<__nv_bfloat16*>(out);
+    const long long rows = static_cast<long long>(N) * Ho;
+    // 32-bit per-image offsets for the row kernel
+    if (vec && rows <= 0x7fffffffLL && static_cast<long long>(H) * W * (C / 8) <= 0x7fffffffLL) {
+        const int work = Wo * (C / 8);
+        const int t = work >= 512 ? 512 : ((work + 31) / 32) * 32;
+        maxpool_rows_kernel<<<static_cast<unsigned>(rows), t, 0, stream>>>(
+            xb, H, W, C, k, stride, pad, Ho, Wo, yb);
+        return cudaGetLastError();
+    }
     if (vec)
         maxpool_kernel<8><<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
             xb, N, H, W, C, k, stride, pad, Ho, Wo, yb);

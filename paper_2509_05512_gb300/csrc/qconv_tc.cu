@@ -37,7 +37,8 @@
 //               (one thread issues TMA copies at a limited rate);
 //   warp 1      owns TMEM (2 accumulator buffers x 4 components x BNQ columns); one lane
 //               issues the tcgen05.mma / tcgen05.commit stream;
-//   warp 2      MODE_PAIR: writes the two sign-flipped letter copies of each stage;
+//   warp 2      waits for both fills of each stage (MODE_PAIR: writes the two
+//               sign-flipped letter copies) and hands it to the issuer with one barrier;
 //   warps 4..11 epilogue (tc_common.cuh), overlapping the next tile's main loop.
 // Every mbarrier wait is bounded in time; a wait that runs out sets a bit in the device
 // status word, raises a CTA-wide abort flag, drains the copies and MMAs still in flight,
@@ -274,11 +275,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 tc_fence_after();
                 const uint32_t dbase = tmem_base + static_cast<uint32_t>(buf * 4 * BNQ);
                 for (int kt = 0; kt < p.ktiles; ++kt) {
-                    // pixels, then the letter tiles (pair mode: with their negated copies)
-                    if (!wait_or_abort(full_bar(stage), phase, limit, abort_flag,
-                                       STATUS_TIMEOUT_MMA) ||
-                        !wait_or_abort(MODE == MODE_PAIR ? ready_bar(stage) : fullw_bar(stage),
-                                       phase, limit, abort_flag, STATUS_TIMEOUT_MMA)) {
+                    // pixels and letter tiles landed (pair mode: with the negated copies)
+                    if (!wait_or_abort(ready_bar(stage), phase, limit, abort_flag,
+                                       STATUS_TIMEOUT_MMA)) {
                         ok = false;
                         break;
                     }
@@ -344,23 +343,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
         }
     } else if (warp == 2) {
-        // ------------------------------------------------------------ sign flips
-        if constexpr (MODE == MODE_PAIR) {
-            // Write -W_i (slot 0) and -W_j (slot 5) of every stage from its copies of W_i
-            // and W_j (slots 2, 3) once they have landed, then hand the stage to the MMA
-            // issuer.  Slot sizes are multiples of the swizzle period, so a raw copy keeps
-            // the layout.
-            constexpr int WORDS = C::B_TILE / 16;  // uint4 per slot
-            int stage = 0;
-            uint32_t phase = 0;
-            bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
-                for (int kt = 0; kt < p.ktiles; ++kt) {
-                    if (!wait_or_abort(fullw_bar(stage), phase, limit, abort_flag,
-                                       STATUS_TIMEOUT_PRODUCER)) {
-                        ok = false;
-                        break;
-                    }
+        // ------------------------------------------------------------ stage hand-off
+        // Waits for both fills of every stage (and in pair mode writes -W_i (slot 0) and
+        // -W_j (slot 5) from its copies of W_i and W_j (slots 2, 3); slot sizes are
+        // multiples of the swizzle period, so a raw copy keeps the layout), then hands
+        // the stage to the MMA issuer through one barrier: every mbarrier wait the issuing
+        // thread itself performs stalls the tensor pipe for hundreds of cycles.
+        constexpr int WORDS = C::B_TILE / 16;  // uint4 per slot
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+            for (int kt = 0; kt < p.ktiles; ++kt) {
+                if (!wait_or_abort(fullw_bar(stage), phase, limit, abort_flag,
+                                   STATUS_TIMEOUT_PRODUCER)) {
+                    ok = false;
+                    break;
+                }
+                if constexpr (MODE == MODE_PAIR) {
                     uint8_t* b0 = smem + stage * C::STAGE_BYTES + 4 * C::A_TILE;
                     const uint4* s2 = reinterpret_cast<const uint4*>(b0 + 2 * C::B_TILE);
                     const uint4* s3 = reinterpret_cast<const uint4*>(b0 + 3 * C::B_TILE);
@@ -373,12 +373,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                     // make the generic-proxy writes visible to the tensor core (async proxy)
                     fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(ready_bar(stage));
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
+                }
+                if (!wait_or_abort(full_bar(stage), phase, limit, abort_flag,
+                                   STATUS_TIMEOUT_PRODUCER)) {
+                    ok = false;
+                    break;
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(ready_bar(stage));
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
             }
         }
