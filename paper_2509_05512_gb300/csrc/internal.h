@@ -58,6 +58,26 @@ cudaError_t launch_qconv_simt_bf16(const ConvShape& s, const void* x, const void
 cudaError_t launch_qconv_simt_f32(const ConvShape& s, const void* x, const void* const w[4],
                                   const EpilogueArgs& ep, void* out, cudaStream_t stream);
 
+// Launch with programmatic stream serialization: the kernel may start while the previous
+// kernel in the stream is finishing (once all of that grid's CTAs have signalled), runs its
+// prologue (barriers, TMEM, descriptor prefetch) and waits with griddepcontrol.wait before
+// its first global access.  Every kernel of this library follows that rule.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream);

@@ -14,6 +14,8 @@ __global__ void __launch_bounds__(256) maxpool_kernel(const __nv_bfloat16* __res
                                                       int H, int W, int C, int k, int stride,
                                                       int pad, int Ho, int Wo,
                                                       __nv_bfloat16* __restrict__ y) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs from the previous kernel
     const int cv = C / VEC;
     const long long total = static_cast<long long>(N) * Ho * Wo * cv;
     for (long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -69,6 +71,8 @@ __global__ void __launch_bounds__(512) maxpool_rows_kernel(const __nv_bfloat16* 
                                                            int H, int W, int C, int k,
                                                            int stride, int pad, int Ho, int Wo,
                                                            __nv_bfloat16* __restrict__ y) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs from the previous kernel
     const int cv = C / 8;
     const int row = blockIdx.x;  // n * Ho + ho
     const int n = row / Ho, ho = row - (row / Ho) * Ho;
@@ -126,17 +130,14 @@ cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k
     if (vec && rows <= 0x7fffffffLL && static_cast<long long>(H) * W * (C / 8) <= 0x7fffffffLL) {
         const int work = Wo * (C / 8);
         const int t = work >= 512 ? 512 : ((work + 31) / 32) * 32;
-        maxpool_rows_kernel<<<static_cast<unsigned>(rows), t, 0, stream>>>(
-            xb, H, W, C, k, stride, pad, Ho, Wo, yb);
-        return cudaGetLastError();
+        return launch_pdl(maxpool_rows_kernel, dim3(static_cast<unsigned>(rows)), dim3(t), 0,
+                          stream, xb, H, W, C, k, stride, pad, Ho, Wo, yb);
     }
     if (vec)
-        maxpool_kernel<8><<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-            xb, N, H, W, C, k, stride, pad, Ho, Wo, yb);
-    else
-        maxpool_kernel<1><<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-            xb, N, H, W, C, k, stride, pad, Ho, Wo, yb);
-    return cudaGetLastError();
+        return launch_pdl(maxpool_kernel<8>, dim3(static_cast<unsigned>(blocks)), dim3(threads),
+                          0, stream, xb, N, H, W, C, k, stride, pad, Ho, Wo, yb);
+    return launch_pdl(maxpool_kernel<1>, dim3(static_cast<unsigned>(blocks)), dim3(threads), 0,
+                      stream, xb, N, H, W, C, k, stride, pad, Ho, Wo, yb);
 }
 
 }  // namespace quan

@@ -296,4 +296,31 @@ __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// ------------------------------------------------------------------ shared-memory flags
+// A release store and an acquire load of one shared-memory word: the hand-off between a
+// helper warp and an MMA-issuing thread.  One acquire load costs the issuing thread about
+// a third of an mbarrier wait, and the tensor pipe keeps almost no queue while it stalls.
+__device__ __forceinline__ uint32_t ld_acquire_shared(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_release_shared(uint32_t addr, uint32_t v) {
+    asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+// ------------------------------------------------------------------ dependent launch
+// Programmatic dependent launch: the next kernel in the stream (launched with the
+// programmatic-serialization attribute) may start once every CTA of this grid has called
+// launch_dependents, and griddep_wait returns once the previous grid has completed and its
+// memory is visible.  A kernel reads and writes no global data before griddep_wait.
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ void griddep_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 }  // namespace quan

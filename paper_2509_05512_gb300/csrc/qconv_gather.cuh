@@ -212,6 +212,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
     const uint64_t limit = p.wait_limit_ns;
     const int STAGES = ISSUERS * p.per;
 
+    griddep_launch_dependents();
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(full_bar(i), 1);
@@ -235,6 +236,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    griddep_wait();  // the previous kernel's output (this layer's input) is complete
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer

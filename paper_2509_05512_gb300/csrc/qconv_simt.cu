@@ -35,6 +35,8 @@ __global__ void __launch_bounds__(256) qconv_simt_kernel(ConvShape s, const T* _
                                                          const T* __restrict__ wj,
                                                          const T* __restrict__ wk,
                                                          EpilogueArgs ep, T* __restrict__ out) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs from the previous kernel
     const long long total = s.M * s.Qout;
     const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= total) return;
@@ -93,10 +95,10 @@ cudaError_t launch(const ConvShape& s, const void* x, const void* const w[4],
     const int threads = 256;
     const long long blocks = (total + threads - 1) / threads;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    qconv_simt_kernel<T><<<static_cast<unsigned>(blocks), threads, 0, stream>>>(
-        s, static_cast<const T*>(x), static_cast<const T*>(w[0]), static_cast<const T*>(w[1]),
-        static_cast<const T*>(w[2]), static_cast<const T*>(w[3]), ep, static_cast<T*>(out));
-    return cudaGetLastError();
+    return launch_pdl(qconv_simt_kernel<T>, dim3(static_cast<unsigned>(blocks)), dim3(threads),
+                      0, stream, s, static_cast<const T*>(x), static_cast<const T*>(w[0]),
+                      static_cast<const T*>(w[1]), static_cast<const T*>(w[2]),
+                      static_cast<const T*>(w[3]), ep, static_cast<T*>(out));
 }
 
 }  // namespace

@@ -38,7 +38,8 @@
 //   warp 1      owns TMEM (2 accumulator buffers x 4 components x BNQ columns); one lane
 //               issues the tcgen05.mma / tcgen05.commit stream;
 //   warp 2      waits for both fills of each stage (MODE_PAIR: writes the two
-//               sign-flipped letter copies) and hands it to the issuer with one barrier;
+//               sign-flipped letter copies) and hands it to the issuer by a release store
+//               of the stage's sequence word, which the issuer reads with an acquire load;
 //   warps 4..11 epilogue (tc_common.cuh), overlapping the next tile's main loop.
 // Every mbarrier wait is bounded in time; a wait that runs out sets a bit in the device
 // status word, raises a CTA-wide abort flag, drains the copies and MMAs still in flight,
@@ -102,10 +103,10 @@ struct Cfg {
     static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
     static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
     static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
-    // full (pixels), full (letters), empty, ready (negated copies done), acc_full[2],
-    // acc_empty[2], drain
-    static constexpr int NUM_BARS = 4 * STAGES + 5;
-    static constexpr int SMEM_BYTES = 1024 + BAR_OFF + NUM_BARS * 8 + 16;
+    // full (pixels), empty, full (letters), acc_full[2], acc_empty[2], drain; then the
+    // TMEM address, the abort flag and one ready sequence word per stage
+    static constexpr int NUM_BARS = 3 * STAGES + 5;
+    static constexpr int SMEM_BYTES = 1024 + BAR_OFF + NUM_BARS * 8 + 16 + 4 * STAGES;
     static constexpr bool FITS = SMEM_BYTES <= 227 * 1024;
     static constexpr uint32_t TMEM_COLS = 8 * BNQ;  // 2 buffers x 4 components x BNQ fp32 columns
     static constexpr int KSTEPS = KAPPA / UMMA_K;
@@ -131,25 +132,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::BAR_OFF);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NUM_BARS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    uint32_t* ready_seq = tmem_slot + 4;  // per stage: fills handed to the issuer so far
     const uint32_t bar0 = smem_u32(bars);
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-    auto ready_bar = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
-    auto fullw_bar = [&](int s) { return bar0 + 8u * (3 * STAGES + s); };
-    const uint32_t accf0 = bar0 + 8u * (4 * STAGES);
-    const uint32_t acce0 = bar0 + 8u * (4 * STAGES + 2);
-    const uint32_t drain_bar = bar0 + 8u * (4 * STAGES + 4);
+    auto fullw_bar = [&](int s) { return bar0 + 8u * (2 * STAGES + s); };
+    auto ready_word = [&](int s) { return smem_u32(ready_seq + s); };
+    const uint32_t accf0 = bar0 + 8u * (3 * STAGES);
+    const uint32_t acce0 = bar0 + 8u * (3 * STAGES + 2);
+    const uint32_t drain_bar = bar0 + 8u * (3 * STAGES + 4);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
     const uint64_t limit = p.wait_limit_ns;
 
+    griddep_launch_dependents();
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(full_bar(i), 1);
             mbar_init(fullw_bar(i), 1);
             mbar_init(empty_bar(i), 1);
-            mbar_init(ready_bar(i), 1);
+            ready_seq[i] = 0;
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(accf0 + 8u * b, 1);
@@ -176,6 +179,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const int hw = s.Ho * s.Wo;
+    griddep_wait();  // the previous kernel's output (this layer's input) is complete
 
     if (warp == 0 || warp == 3) {
         // ------------------------------------------------------------ TMA producers
@@ -254,7 +258,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             constexpr uint32_t IDESC_POS = make_idesc(BM, NMMA, 0);
             constexpr uint32_t IDESC_NEG = make_idesc(BM, NMMA, 1);
             int stage = 0;
-            uint32_t phase = 0;
+            uint32_t round = 0;  // completed passes over the stage ring
             bool ok = true;
             int issued = 0;
             if (p.inject_stall) {
@@ -276,8 +280,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const uint32_t dbase = tmem_base + static_cast<uint32_t>(buf * 4 * BNQ);
                 for (int kt = 0; kt < p.ktiles; ++kt) {
                     // pixels and letter tiles landed (pair mode: with the negated copies)
-                    if (!wait_or_abort(ready_bar(stage), phase, limit, abort_flag,
-                                       STATUS_TIMEOUT_MMA)) {
+                    if (!flag_wait_or_abort(ready_word(stage), round + 1u, limit, abort_flag,
+                                            STATUS_TIMEOUT_MMA)) {
                         ok = false;
                         break;
                     }
@@ -324,7 +328,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     umma_commit(empty_bar(stage));  // frees the stage when these MMAs finish
                     if (++stage == STAGES) {
                         stage = 0;
-                        phase ^= 1u;
+                        ++round;
                     }
                 }
                 if (!ok) break;
@@ -347,11 +351,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // Waits for both fills of every stage (and in pair mode writes -W_i (slot 0) and
         // -W_j (slot 5) from its copies of W_i and W_j (slots 2, 3); slot sizes are
         // multiples of the swizzle period, so a raw copy keeps the layout), then hands
-        // the stage to the MMA issuer through one barrier: every mbarrier wait the issuing
-        // thread itself performs stalls the tensor pipe for hundreds of cycles.
+        // the stage to the MMA issuer through its ready sequence word: every mbarrier wait
+        // the issuing thread itself performs stalls the tensor pipe for hundreds of cycles,
+        // an acquire load of that word for about a third of that.
         constexpr int WORDS = C::B_TILE / 16;  // uint4 per slot
         int stage = 0;
-        uint32_t phase = 0;
+        uint32_t phase = 0, round = 0;
         bool ok = true;
         for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
             for (int kt = 0; kt < p.ktiles; ++kt) {
@@ -380,10 +385,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     break;
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(ready_bar(stage));
+                if (lane == 0) st_release_shared(ready_word(stage), round + 1u);
                 if (++stage == STAGES) {
                     stage = 0;
                     phase ^= 1u;
+                    ++round;
                 }
             }
         }
@@ -559,9 +565,8 @@ cudaError_t launch_cfg(const CUtensorMap maps[6], const TcParams& prm, int grid,
         static std::atomic<unsigned long long> attr_done{0};
         cudaError_t e = set_smem_once(kern, C::SMEM_BYTES, attr_done);
         if (e != cudaSuccess) return e;
-        kern<<<grid, NUM_THREADS, C::SMEM_BYTES, stream>>>(maps[0], maps[1], maps[2], maps[3],
-                                                           maps[4], maps[5], prm);
-        return cudaGetLastError();
+        return launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, stream, maps[0],
+                          maps[1], maps[2], maps[3], maps[4], maps[5], prm);
     }
 }
 
@@ -706,19 +711,21 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         auto kern = qconv_ws_kernel<true, 3>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h3);
         if (e != cudaSuccess) return e;
-        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
     } else if (halo) {
         auto kern = qconv_ws_kernel<true, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
         if (e != cudaSuccess) return e;
-        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
     } else {
         auto kern = qconv_ws_kernel<false, 0>;
         cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
         if (e != cudaSuccess) return e;
-        kern<<<grid, WIDE_THREADS, WsCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
     }
-    return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
@@ -775,14 +782,15 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         auto kern = qconv_pairs_kernel<7, 4>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74);
         if (e != cudaSuccess) return e;
-        kern<<<grid, WIDE_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
     } else {
         auto kern = qconv_pairs_kernel<0, 0>;
         cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_any);
         if (e != cudaSuccess) return e;
-        kern<<<grid, WIDE_THREADS, GaCfg::SMEM_BYTES, stream>>>(maps[0], prm);
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
     }
-    return cudaGetLastError();
 }
 
 }  // namespace

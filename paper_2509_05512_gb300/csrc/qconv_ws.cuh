@@ -150,6 +150,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
     const int kt = (p.num_tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                    static_cast<int>(gridDim.x);
 
+    griddep_launch_dependents();
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(full_bar(i), 1);
@@ -174,6 +175,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const int hw = s.Ho * s.Wo;
+    griddep_wait();  // the previous kernel's output (this layer's input) is complete
     // pixel rows of a tile: halo -> (image, first input row); per tap -> first pixel
     auto tile_base = [&](int tile, int& img, int& hbase, int& wbase) {
         if constexpr (HALO) {

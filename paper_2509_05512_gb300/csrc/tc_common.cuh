@@ -101,6 +101,25 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, uin
     }
 }
 
+// Bounded wait for a sequence word in shared memory (written with st_release_shared) to
+// reach `target` (wrap-safe comparison).  Same failure handling as wait_or_abort.
+__device__ __forceinline__ bool flag_wait_or_abort(uint32_t addr, uint32_t target,
+                                                   uint64_t limit, volatile int* abort_flag,
+                                                   unsigned code) {
+    if (static_cast<int>(ld_acquire_shared(addr) - target) >= 0) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+        if (static_cast<int>(ld_acquire_shared(addr) - target) >= 0) return true;
+        if (*abort_flag) return false;
+        if (global_timer_ns() - t0 > limit) {
+            atomicOr(&g_status, code);
+            *abort_flag = 1;
+            return false;
+        }
+        __nanosleep(32);
+    }
+}
+
 // Wait for the most recent fill of each stage a producer armed, so that no copy still
 // targets this CTA's shared memory when it exits after an abort.
 __device__ __forceinline__ void drain_fills(uint32_t bar0, int stages, uint32_t filled,
