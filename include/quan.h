@@ -74,7 +74,8 @@ typedef enum {
  *   kh,kw        filter size >= 1; stride >= 1; pad >= 0; Ho, Wo >= 1
  *   act          quan_act_t
  *   out          bf16 [N][Ho][Wo][Cout]        (device), rounded to nearest even
- * The tensor-core path needs 16-byte aligned tensor pointers, fewer than 2^31 output
+ * The tensor-core path needs 16-byte aligned pointers (every tensor, the residual and the
+ * per-channel vectors), fewer than 2^31 output
  * pixels and either Cin/4 and Cout/4 multiples of 16, or Cin = 4, Cout = 64, stride 2
  * and an even W (the 4-channel stem: kh * P <= 32, where P = ceil((kw + pad mod 2) / 2)
  * rounded up to even is the number of 2-pixel pairs a filter row spans); other shapes
@@ -145,6 +146,15 @@ quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode);
  * filter tap instead (same results).
  */
 quan_status_t quan_set_tc_halo(int enable);
+
+/*
+ * MMA-issuing threads of the weight-stationary kernel (16 -> 16 quaternion channels):
+ * 0 (default) chooses three when that still leaves every issuer as many pixel stages as
+ * a tile has K blocks (at most three), else two; 2 or 3 force the count.  Any other
+ * value returns QUAN_ERR_INVALID_ARG.  Results do not depend on it.  Process-wide, like
+ * the other tile options.
+ */
+quan_status_t quan_set_tc_issuers(int issuers);
 
 /* Time limit of every bounded wait inside the tensor-core kernel, in nanoseconds
  * (default 2e9).  0 restores the default. */

@@ -38,13 +38,14 @@ struct TcOptions {
                                   // 3 weight-stationary
     int ws_halo;                  // weight-stationary: stage row blocks with halos (1) when
                                   // the shape allows it, else one im2col box per tap (0)
+    int ws_issuers;               // weight-stationary MMA issuers: 0 auto, 2 or 3
     unsigned long long wait_limit_ns;
     int inject_stall;             // failure-injection: the MMA role never consumes
 };
 
 // Tensor-core path (tcgen05 + TMA), bf16 in/out, fp32 accumulation.
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
-                  const void* residual);
+                  const EpilogueArgs& ep);
 cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const w[4],
                             const EpilogueArgs& ep, void* out, const TcOptions& opt,
                             int num_sms, cudaStream_t stream, char* err, size_t errlen);

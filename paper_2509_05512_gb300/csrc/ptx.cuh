@@ -296,6 +296,23 @@ __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// ------------------------------------------------------------------ streaming global access
+// Output stores and residual loads of the epilogues bypass L1 allocation, so the small L1
+// left beside a full shared-memory carve-out keeps the per-channel vectors.
+__device__ __forceinline__ void st_global_na(void* p, uint4 v) {
+    asm volatile("st.global.L1::no_allocate.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x),
+                 "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_global_na(const void* p) {
+    uint4 v;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p));
+    return v;
+}
+
 // ------------------------------------------------------------------ shared-memory flags
 // A release store and an acquire load of one shared-memory word: the hand-off between a
 // helper warp and an MMA-issuing thread.  One acquire load costs the issuing thread about

@@ -352,8 +352,6 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
                 g.m0 = static_cast<long long>(row) * Wo + seg * GA_TILE_W;
                 const int left = Wo - seg * GA_TILE_W;
                 g.rows = left < GA_TILE_W ? left : GA_TILE_W;
-                g.sy = seg * GA_TILE_W;
-                g.sz = row;
                 return g;
             };
             epilogue_direct64<decltype(geo)>(s, p.ep, p.y, tmem_base, accf0, acce0,

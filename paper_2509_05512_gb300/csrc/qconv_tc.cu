@@ -80,6 +80,7 @@ struct TcParams {
     int ktiles;       // kh * kw * kchunks K blocks per tile
     int num_n_tiles;  // Qout / BNQ
     int num_tiles;
+    void* y;          // output [M][Cout]
     unsigned long long wait_limit_ns;
     int inject_stall;
 };
@@ -93,20 +94,19 @@ struct Cfg {
     static constexpr int STAGE_BYTES = 4 * A_TILE + B_SLOTS * B_TILE;
     static constexpr int TX_A = 4 * A_TILE;          // bytes TMA writes per stage: pixels
     static constexpr int TX_W = 4 * B_TILE;          //                               letters
-    using E = EpiSmem<BNQ>;
-    static constexpr int FIXED_BYTES = 1024 + E::STAGING_BYTES + E::PARAM_BYTES + 512;
+    // 1024 bytes of alignment slack, then the stage ring and the barrier area (the
+    // epilogue needs no shared memory)
+    static constexpr int FIXED_BYTES = 1024 + 384;
     static constexpr int STAGES_RAW = (227 * 1024 - FIXED_BYTES) / STAGE_BYTES;
     static constexpr int STAGES =
         STAGES_RAW > MAX_STAGES ? MAX_STAGES : (STAGES_RAW < 2 ? 2 : STAGES_RAW);
     static constexpr int TILES_BYTES = STAGES * STAGE_BYTES;
-    static constexpr int STAGING_OFF = TILES_BYTES;
-    static constexpr int PARAM_OFF = STAGING_OFF + E::STAGING_BYTES;
-    static constexpr int BAR_OFF = PARAM_OFF + E::PARAM_BYTES;
-    static_assert(PARAM_OFF % 16 == 0, "float4 reads of the epilogue vectors");
+    static constexpr int BAR_OFF = TILES_BYTES;
     // full (pixels), empty, full (letters), acc_full[2], acc_empty[2], drain; then the
     // TMEM address, the abort flag and one ready sequence word per stage
     static constexpr int NUM_BARS = 3 * STAGES + 5;
     static constexpr int SMEM_BYTES = 1024 + BAR_OFF + NUM_BARS * 8 + 16 + 4 * STAGES;
+    static_assert(NUM_BARS * 8 + 16 + 4 * STAGES <= FIXED_BYTES - 1024, "barrier area");
     static constexpr bool FITS = SMEM_BYTES <= 227 * 1024;
     static constexpr uint32_t TMEM_COLS = 8 * BNQ;  // 2 buffers x 4 components x BNQ fp32 columns
     static constexpr int KSTEPS = KAPPA / UMMA_K;
@@ -121,8 +121,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     const __grid_constant__ CUtensorMap tmap_wr,
                     const __grid_constant__ CUtensorMap tmap_wi,
                     const __grid_constant__ CUtensorMap tmap_wj,
-                    const __grid_constant__ CUtensorMap tmap_wk,
-                    const __grid_constant__ CUtensorMap tmap_y, const TcParams p) {
+                    const __grid_constant__ CUtensorMap tmap_wk, const TcParams p) {
     using C = Cfg<KAPPA, BNQ, MODE>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -168,7 +167,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tma_prefetch_desc(&tmap_wi);
         tma_prefetch_desc(&tmap_wj);
         tma_prefetch_desc(&tmap_wk);
-        tma_prefetch_desc(&tmap_y);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
@@ -397,18 +395,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // ------------------------------------------------------------ epilogue
         const int num_n = p.num_n_tiles;
         const long long M = s.M;
-        epilogue_role<BNQ, false>(
-            s, p.ep, &tmap_y, tmem_base, smem + C::STAGING_OFF,
-            reinterpret_cast<float*>(smem + C::PARAM_OFF), accf0, acce0, p.num_tiles, limit,
-            abort_flag, [num_n, M](int tile) {
+        epilogue_direct_pair<BNQ>(
+            s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit, abort_flag,
+            [num_n, M](int tile) {
                 EpiTile g;
                 const int m_tile = tile / num_n;
                 g.n_tile = tile - m_tile * num_n;
                 g.m0 = static_cast<long long>(m_tile) * BM;
                 const long long left = M - g.m0;
                 g.rows = left < BM ? static_cast<int>(left) : BM;
-                g.sy = static_cast<int>(g.m0);
-                g.sz = 0;
                 return g;
             });
     }
@@ -525,20 +520,6 @@ bool encode_w(CUtensorMap* map, const ConvShape& s, const void* w, int kappa, in
     return r == CUDA_SUCCESS;
 }
 
-// Output [M rows][Cout] bf16, stored in boxes of BM rows x BNQ channels.
-bool encode_y_2d(CUtensorMap* map, const ConvShape& s, const void* y, int bnq) {
-    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(s.Cout), static_cast<cuuint64_t>(s.M)};
-    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(s.Cout) * 2};
-    const cuuint32_t box[2] = {static_cast<cuuint32_t>(bnq), static_cast<cuuint32_t>(BM)};
-    const cuuint32_t estr[2] = {1, 1};
-    const CUresult r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
-                                      const_cast<void*>(y), dims, strides, box, estr,
-                                      CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(bnq * 2),
-                                      CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
-
 // The shared-memory opt-in is per device and kernel; set it once for each.
 template <typename K>
 cudaError_t set_smem_once(K kern, int bytes, std::atomic<unsigned long long>& done) {
@@ -566,7 +547,7 @@ cudaError_t launch_cfg(const CUtensorMap maps[6], const TcParams& prm, int grid,
         cudaError_t e = set_smem_once(kern, C::SMEM_BYTES, attr_done);
         if (e != cudaSuccess) return e;
         return launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, stream, maps[0],
-                          maps[1], maps[2], maps[3], maps[4], maps[5], prm);
+                          maps[1], maps[2], maps[3], maps[4], prm);
     }
 }
 
@@ -650,6 +631,16 @@ int grid_for(const TcOptions& opt, int num_sms, int num_tiles) {
     return grid < 1 ? 1 : grid;
 }
 
+template <bool HALO, int KH, int NI>
+cudaError_t launch_ws_kernel(const CUtensorMap& map, const WsParams& prm, int grid,
+                             cudaStream_t stream) {
+    auto kern = qconv_ws_kernel<HALO, KH, NI>;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, attr_done);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream, map, prm);
+}
+
 cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
                       const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
                       cudaStream_t stream, char* err, size_t errlen) {
@@ -683,11 +674,14 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     }
     prm.num_tiles = static_cast<int>(tiles);
     prm.stage_bytes = (prm.box_bytes + 1023) & ~1023;
-    int per = WsCfg::RING_BYTES / prm.stage_bytes / ISSUERS;
-    if (per > WsCfg::MAX_PER) per = WsCfg::MAX_PER;
+    const int ni = opt.ws_issuers == 2 || opt.ws_issuers == ISSUERS
+                       ? opt.ws_issuers
+                       : ws_issuers(prm.stage_bytes, prm.kblocks);
+    int per = WsCfg::RING_BYTES / prm.stage_bytes / ni;
+    if (per > WsCfg::NSTAGE / ni) per = WsCfg::NSTAGE / ni;
     if (per < 1) {
-        snprintf(err, errlen, "weight-stationary pixel box of %d bytes does not fit",
-                 prm.box_bytes);
+        snprintf(err, errlen, "weight-stationary pixel box of %d bytes does not fit %d issuers",
+                 prm.box_bytes, ni);
         return cudaErrorInvalidValue;
     }
     prm.per = per;
@@ -705,27 +699,16 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    static std::atomic<unsigned long long> done_h3{0}, done_h{0}, done_t{0};
-    set_kernel_name(halo ? "qconv_ws_kernel<halo>" : "qconv_ws_kernel<im2col>");
-    if (halo && s.kh == 3) {
-        auto kern = qconv_ws_kernel<true, 3>;
-        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h3);
-        if (e != cudaSuccess) return e;
-        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
-                          maps[0], prm);
-    } else if (halo) {
-        auto kern = qconv_ws_kernel<true, 0>;
-        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_h);
-        if (e != cudaSuccess) return e;
-        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
-                          maps[0], prm);
-    } else {
-        auto kern = qconv_ws_kernel<false, 0>;
-        cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, done_t);
-        if (e != cudaSuccess) return e;
-        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream,
-                          maps[0], prm);
+    set_kernel_name(halo ? "qconv_ws_kernel<halo,issuers=%d>" : "qconv_ws_kernel<im2col,issuers=%d>",
+                    ni);
+    if (ni == 2) {
+        if (halo && s.kh == 3) return launch_ws_kernel<true, 3, 2>(maps[0], prm, grid, stream);
+        if (halo) return launch_ws_kernel<true, 0, 2>(maps[0], prm, grid, stream);
+        return launch_ws_kernel<false, 0, 2>(maps[0], prm, grid, stream);
     }
+    if (halo && s.kh == 3) return launch_ws_kernel<true, 3, ISSUERS>(maps[0], prm, grid, stream);
+    if (halo) return launch_ws_kernel<true, 0, ISSUERS>(maps[0], prm, grid, stream);
+    return launch_ws_kernel<false, 0, ISSUERS>(maps[0], prm, grid, stream);
 }
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
@@ -796,14 +779,18 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
 }  // namespace
 
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
-                  const void* residual) {
+                  const EpilogueArgs& ep) {
     auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
     if ((s.Qin % 16 != 0 || s.Qout % 16 != 0) && !gather_ok(s)) return false;
     // TMA coordinates of the output (pixel index) are 32-bit
     if (s.M > 0x7fffffffLL) return false;
     if (!al16(x) || !al16(out) || !al16(w[0]) || !al16(w[1]) || !al16(w[2]) || !al16(w[3]))
         return false;
-    if (residual && !al16(residual)) return false;
+    // the epilogues read the residual and the per-channel vectors 16 bytes at a time
+    if (ep.residual && !al16(ep.residual)) return false;
+    if ((ep.bias && !al16(ep.bias)) || (ep.scale && !al16(ep.scale)) ||
+        (ep.shift && !al16(ep.shift)))
+        return false;
     if (s.stride > 8) return false;
     // im2col bounding-box corner offsets must fit the 4-D encoding range [-128, 127]
     if (s.pad > 127 || s.pad - (s.kh - 1) < -128 || s.pad - (s.kw - 1) < -128) return false;
@@ -851,8 +838,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                  opt.kappa, opt.bnq, s.Qin, s.Qout);
         return cudaErrorInvalidValue;
     }
-    // A 6-slot stage of 64 x 64 letter blocks plus 64-channel pixel tiles does not fit
-    // twice in shared memory; use 32-channel K blocks then.
+    // Only two 6-slot stages of 64 x 64 letter blocks plus 64-channel pixel tiles fit in
+    // shared memory; 32-channel K blocks give four.
     if (mode == MODE_PAIR && kappa == 64 && bnq == 64 && opt.kappa == 0) kappa = 32;
     {
         bool fits = true;
@@ -881,10 +868,7 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                 snprintf(err, errlen, "cuTensorMapEncodeTiled failed for weight letter %d", l);
                 return cudaErrorInvalidValue;
             }
-        if (!encode_y_2d(&maps[5], s, out, bnq)) {
-            snprintf(err, errlen, "cuTensorMapEncodeTiled failed for the output tensor");
-            return cudaErrorInvalidValue;
-        }
+        maps[5] = maps[0];
         cache_store(key, maps);
     }
     TcParams prm;
@@ -893,6 +877,7 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     prm.kchunks = s.Qin / kappa;
     prm.ktiles = s.kh * s.kw * prm.kchunks;
     prm.num_n_tiles = s.Qout / bnq;
+    prm.y = out;
     const long long m_tiles = (s.M + BM - 1) / BM;
     const long long tiles = m_tiles * prm.num_n_tiles;
     if (tiles > 0x7fffffffLL) {

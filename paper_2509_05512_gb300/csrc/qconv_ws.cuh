@@ -19,16 +19,21 @@
 //   per tap  otherwise: one im2col box of 128 pixels per filter tap.
 //
 // Roles (16 warps):
-//   warp 0       TMA producer: the K blocks of each group of ISSUERS consecutive local
-//                tiles interleaved (block 0 of each tile, then block 1, ...), each into
-//                the next stage of the issuer that owns the tile.
-//   warps 1..3   MMA issuers taking the CTA's local tiles round robin, each waiting only
-//                for its own stages and accumulator buffers (issuer_stage, issuer_acc in
+//   warp 0       TMA producer: the K blocks of each group of NI consecutive local tiles
+//                interleaved (block 0 of each tile, then block 1, ...), each into the next
+//                stage of the issuer that owns the tile.
+//   warps 1..NI  MMA issuers taking the CTA's local tiles round robin, each waiting only
+//                for its own stages and accumulator buffers (issuer_stage, issuer_acc_n in
 //                tc_common.cuh; the tensor pipe keeps almost no queue and an issuing
 //                thread's own waits and branches cost hundreds of cycles while its MMAs
-//                are in flight).  Warp 1 owns TMEM.
-//   warps 2..15  expand the signed block weight once per CTA; then warps 4..15 run the
-//                shared-memory-free direct epilogue (tc_common.cuh).
+//                are in flight).  Warp 1 owns TMEM.  NI = 3 hides those stalls best; NI = 2
+//                gives each issuer half of the stage ring instead of a third, for pixel
+//                boxes so large that three issuers would hold fewer stages than a tile
+//                has K blocks (the third block's load then waits for the first block's
+//                MMAs and its latency is exposed).
+//   warps 2..15  expand the signed block weight once per CTA; then warps 4 .. 4 + 4 NI - 1
+//                run the shared-memory-free direct epilogue (tc_common.cuh), one group of
+//                four per issuer.
 
 constexpr int WS_ROW_BYTES = 128;  // 64 channels x bf16: all four components of a pixel
 
@@ -74,7 +79,15 @@ bool ws_halo_ok(const ConvShape& s) {
     const int R = BM / s.Wo;
     const long long box = static_cast<long long>(s.Wo) * (R + s.kh - 1) * WS_ROW_BYTES;
     const long long stage = (box + 1023) & ~1023LL;
-    return ISSUERS * stage <= WsCfg::RING_BYTES;
+    return 2 * stage <= WsCfg::RING_BYTES;
+}
+
+// Issuers for a pixel stage of `stage_bytes` and `kblocks` K blocks per tile: three while
+// that leaves each at least min(kblocks, 3) stages, else two.
+int ws_issuers(int stage_bytes, int kblocks) {
+    const int stages = WsCfg::RING_BYTES / stage_bytes;
+    const int want = kblocks < 3 ? kblocks : 3;
+    return stages / 3 >= want ? 3 : 2;
 }
 
 // Weight expansion by warps 2..15: for tap t, row n = (q, co) and K index k = (p, ci) the
@@ -121,12 +134,12 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
 }
 
 // KH > 0: the filter height, known at compile time (halo staging), so the MMA issue
-// loop is fully unrolled; 0 = from the shape at run time.
-template <bool HALO, int KH>
+// loop is fully unrolled; 0 = from the shape at run time.  NI: MMA issuers (2 or 3).
+template <bool HALO, int KH, int NI>
 __global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x, const WsParams p) {
     using C = WsCfg;
-    constexpr int NI = ISSUERS;
+    static_assert(NI == 2 || NI == ISSUERS, "two or three issuers");
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -260,7 +273,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             for (int k = me, j = 0; ok && k < kt; k += NI, ++j) {
                 int buf;
                 uint32_t use;
-                issuer_acc(k, buf, use);
+                issuer_acc_n<NI>(k, buf, use);
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA)) {
                     ok = false;
@@ -326,7 +339,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
         }
     } else {
         ws_expand(p, smem, warp, lane, wsready_bar);
-        // -------------------------------------------------------- epilogue (warps 4..15)
+        // ------------------------------------------- epilogue (warps 4 .. 4 + 4 NI - 1)
         const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
         const long long M = s.M;
         auto geo = [tpi, R, Ho, Wo, M](int tile) {
@@ -343,11 +356,11 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
                 const long long left = M - g.m0;
                 g.rows = left < BM ? static_cast<int>(left) : BM;
             }
-            g.sy = g.sz = 0;
             return g;
         };
-        epilogue_direct64<decltype(geo)>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles,
-                                         limit, abort_flag, geo);
+        if (warp >= EPI_WARP0)
+            epilogue_direct64<decltype(geo), NI>(s, p.ep, p.y, tmem_base, accf0, acce0,
+                                                 p.num_tiles, limit, abort_flag, geo);
     }
 
     tc_fence_before();

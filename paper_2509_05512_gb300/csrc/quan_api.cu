@@ -17,7 +17,7 @@ thread_local char t_errmsg[512] = "";
 thread_local int t_last_path = 0;
 thread_local const char* t_last_kernel = "";
 std::atomic<int> g_path{QUAN_PATH_AUTO};
-std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1};
+std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1}, g_ws_issuers{0};
 std::atomic<unsigned long long> g_wait_limit{2000000000ull};
 std::atomic<int> g_inject{0};
 
@@ -134,7 +134,8 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
     const int path = g_path.load();
-    const bool tc_ok = cc == 103 && quan::tc_supported(s, x, w, out, residual);
+    const quan::EpilogueArgs ep{bias, scale, shift, residual};
+    const bool tc_ok = cc == 103 && quan::tc_supported(s, x, w, out, ep);
     bool use_tc;
     if (path == QUAN_PATH_TC) {
         if (!tc_ok)
@@ -149,7 +150,6 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
     } else {
         use_tc = tc_ok;
     }
-    const quan::EpilogueArgs ep{bias, scale, shift, residual};
     cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
     if (use_tc) {
         quan::TcOptions opt;
@@ -158,6 +158,7 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         opt.max_ctas = g_max_ctas.load();
         opt.mode = g_mode.load();
         opt.ws_halo = g_ws_halo.load();
+        opt.ws_issuers = g_ws_issuers.load();
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -266,6 +267,13 @@ quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
 
 quan_status_t quan_set_tc_halo(int enable) {
     g_ws_halo.store(enable ? 1 : 0);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_tc_issuers(int issuers) {
+    if (issuers != 0 && issuers != 2 && issuers != 3)
+        return fail(QUAN_ERR_INVALID_ARG, "issuers must be 0 (automatic), 2 or 3");
+    g_ws_issuers.store(issuers);
     return QUAN_OK;
 }
 

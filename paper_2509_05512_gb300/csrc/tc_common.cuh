@@ -141,199 +141,7 @@ struct EpiTile {
     long long m0;  // linear index of the pixel in TMEM lane 0
     int rows;      // valid lanes (pixels) of the tile
     int n_tile;    // quaternion output channel block
-    int sy, sz;    // TMA store coordinates after the channel one (2-D: sy = m0)
 };
-
-// Shared-memory resources of the epilogue: two staging blocks of 128 x BNQ bf16 (one per
-// half; with WIDE, WBUFS blocks of 128 x 4 BNQ, one per tile parity when WBUFS = 2) and
-// the per-channel vectors [2][4 BNQ] (16-byte aligned): the IQBN scale and the shift with
-// the bias folded in.
-template <int BNQ, bool WIDE = false, int WBUFS = 2>
-struct EpiSmem {
-    static_assert(WBUFS == 1 || WBUFS == 2, "one or two wide staging blocks");
-    static constexpr int OUT_TILE = BM * BNQ * 2;
-    static constexpr int STAGING_BYTES = WIDE ? WBUFS * 4 * OUT_TILE : 2 * OUT_TILE;
-    static constexpr int PARAM_BYTES = 2 * 4 * BNQ * 4;
-    static constexpr uint32_t OUT_ROW = BNQ * 2;
-    static constexpr uint32_t OUT_SW_MASK = BNQ == 64 ? 7u : (BNQ == 32 ? 3u : 1u);
-};
-
-// The epilogue role (warps 4..11, two per TMEM lane quadrant; the first four warps
-// handle output components r, i and the last four j, k).  For each tile of this CTA:
-// wait for its accumulator buffer, apply act(scale*(acc+bias)+shift+residual) (IQBN
-// inference form of Eq. 11-12), round to bf16, write a swizzled shared-memory block per
-// component and store it with TMA (rows outside the tensor are clipped by the map).
-// The affine step is evaluated as fma(scale, acc, scale*bias + shift): the folded shift
-// is formed once per channel, and the two vectors are read as float4 broadcasts (the
-// shared-memory pipe is shared with the tensor cores' operand reads, so the epilogue
-// keeps its own shared-memory traffic small).
-// With WIDE (4 BNQ = 64 channels = the whole output row, BNQ == Qout) all four
-// components go into one 128-byte-row block and a single TMA store per tile; with
-// WBUFS = 2 the block alternates between two buffers so the store overlaps the next
-// tile, with WBUFS = 1 the next tile waits until the store has read the block.
-// Accumulator buffer b (of NACC, used round robin) of a tile lives at TMEM columns
-// [4 BNQ b, 4 BNQ (b+1)), component q at offset q BNQ.
-template <int BNQ, bool STORE3D, typename Geo, bool WIDE = false, int WBUFS = 2, int NACC = 2>
-__device__ __forceinline__ void epilogue_role(const ConvShape& s, const EpilogueArgs& ep,
-                                              const CUtensorMap* tmap_y, uint32_t tmem_base,
-                                              uint8_t* staging, float* prm_s,
-                                              uint32_t accf0, uint32_t acce0, int num_tiles,
-                                              uint64_t limit, volatile int* abort_flag,
-                                              Geo geo) {
-    using E = EpiSmem<BNQ, WIDE, WBUFS>;
-    static_assert(!WIDE || BNQ == 16, "wide stores need 64-channel rows");
-    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
-    const int half = (warp - EPI_WARP0) >> 2;  // output components 2*half, 2*half+1
-    const int row = quad * 32 + lane;
-    const bool leader = (warp == EPI_WARP0 + 4 * half) && lane == 0;
-    const int etid = threadIdx.x - EPI_WARP0 * 32;  // 0..255
-    const int Cout = s.Cout;
-    const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(ep.residual);
-    uint8_t* stg = staging + (WIDE ? 0 : half * E::OUT_TILE);
-    uint32_t stg_addr = smem_u32(stg);
-    int cached_n = -1;
-    int local = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
-        const int buf = local % NACC;
-        const uint32_t use = static_cast<uint32_t>(local / NACC) & 1u;
-        // one lane per warp polls the barrier (256 pollers would crowd the shared-memory
-        // pipe that TMA and the barriers themselves use), then broadcasts the result
-        bool ok = true;
-        if (lane == 0)
-            ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
-        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-        // leave together: a warp that gave up must not strand the others at a barrier
-        if (named_bar_or(1, 256, !ok)) break;
-        tc_fence_after();
-        const EpiTile g = geo(tile);
-        if (g.n_tile != cached_n) {
-            // per-channel vectors of this tile's 4 x BNQ channels -> shared memory
-            named_bar_sync(1, 256);
-            for (int i = etid; i < 4 * BNQ; i += 256) {
-                const int c = (i / BNQ) * s.Qout + g.n_tile * BNQ + (i % BNQ);
-                const float b = ep.bias ? __ldg(ep.bias + c) : 0.0f;
-                const float sc = ep.scale ? __ldg(ep.scale + c) : 1.0f;
-                const float sh = ep.scale ? __ldg(ep.shift + c) : 0.0f;
-                prm_s[i] = sc;
-                prm_s[4 * BNQ + i] = fmaf(sc, b, sh);
-            }
-            named_bar_sync(1, 256);
-            cached_n = g.n_tile;
-        }
-        const long long m = g.m0 + row;
-        const bool valid = row < g.rows;
-        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                               static_cast<uint32_t>(buf * 4 * BNQ);
-        if constexpr (WIDE) {
-            // block of this tile's parity (by tile count, not accumulator buffer); free once
-            // the store of WBUFS tiles ago has read it
-            stg = staging + (local % WBUFS) * 4 * E::OUT_TILE;
-            stg_addr = smem_u32(stg);
-            if (threadIdx.x == EPI_WARP0 * 32) bulk_wait_group_read<WBUFS - 1>();
-            named_bar_sync(1, 256);
-        }
-#pragma unroll
-        for (int qq = 0; qq < 2; ++qq) {
-            const int q = 2 * half + qq;
-            if constexpr (!WIDE) {
-                // the staging block is free once the previous store has read it
-                if (leader) bulk_wait_group_read<0>();
-                named_bar_sync(2 + half, 128);
-            }
-            constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
-#pragma unroll
-            for (int j0 = 0; j0 < BNQ; j0 += CH) {
-                uint32_t v[32];
-                if constexpr (CH == 32) {
-                    tmem_ld_32x32b_x32(taddr + q * BNQ + j0, v);
-                } else {
-                    uint32_t(&v16)[16] = *reinterpret_cast<uint32_t(*)[16]>(v);
-                    tmem_ld_32x32b_x16(taddr + q * BNQ + j0, v16);
-                }
-                float rz[CH];
-                if (res != nullptr && valid) {
-                    const uint4* rp = reinterpret_cast<const uint4*>(
-                        res + m * Cout + q * s.Qout + g.n_tile * BNQ + j0);
-#pragma unroll
-                    for (int u = 0; u < CH / 8; ++u) {
-                        const uint4 r4 = __ldg(rp + u);
-                        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r4);
-#pragma unroll
-                        for (int t = 0; t < 4; ++t) {
-                            const float2 f = __bfloat1622float2(h[t]);
-                            rz[8 * u + 2 * t] = f.x;
-                            rz[8 * u + 2 * t + 1] = f.y;
-                        }
-                    }
-                } else {
-#pragma unroll
-                    for (int t = 0; t < CH; ++t) rz[t] = 0.0f;
-                }
-                tmem_ld_wait();
-                const float4* ps4 = reinterpret_cast<const float4*>(prm_s + q * BNQ + j0);
-                const float4* ph4 = reinterpret_cast<const float4*>(prm_s + 4 * BNQ + q * BNQ + j0);
-#pragma unroll
-                for (int u = 0; u < CH / 8; ++u) {
-                    const float4 sa = ps4[2 * u], sb = ps4[2 * u + 1];
-                    const float4 ha = ph4[2 * u], hb = ph4[2 * u + 1];
-                    const float sc[8] = {sa.x, sa.y, sa.z, sa.w, sb.x, sb.y, sb.z, sb.w};
-                    const float sh[8] = {ha.x, ha.y, ha.z, ha.w, hb.x, hb.y, hb.z, hb.w};
-                    uint32_t w[4];
-#pragma unroll
-                    for (int t = 0; t < 4; ++t) {
-                        const int e = 8 * u + 2 * t;
-                        const float z0 = fmaf(sc[2 * t], __uint_as_float(v[e]), sh[2 * t]) + rz[e];
-                        const float z1 =
-                            fmaf(sc[2 * t + 1], __uint_as_float(v[e + 1]), sh[2 * t + 1]) + rz[e + 1];
-                        w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
-                    }
-                    if constexpr (WIDE) {
-                        // 128-byte row of all four components, 128-byte swizzle
-                        const uint32_t chunk = static_cast<uint32_t>(q * (BNQ / 8) + j0 / 8 + u);
-                        const uint32_t off = static_cast<uint32_t>(row) * 128 +
-                                             ((chunk ^ (static_cast<uint32_t>(row) & 7u)) << 4);
-                        *reinterpret_cast<uint4*>(stg + off) = make_uint4(w[0], w[1], w[2], w[3]);
-                    } else {
-                        // 16-byte chunk (j0/8 + u) of this row, swizzled like the TMA map
-                        const uint32_t chunk = static_cast<uint32_t>(j0 / 8 + u);
-                        const uint32_t off = static_cast<uint32_t>(row) * E::OUT_ROW +
-                                             ((chunk ^ ((static_cast<uint32_t>(row) * E::OUT_ROW >>
-                                                         7) & E::OUT_SW_MASK))
-                                              << 4);
-                        *reinterpret_cast<uint4*>(stg + off) = make_uint4(w[0], w[1], w[2], w[3]);
-                    }
-                }
-            }
-            if constexpr (!WIDE) {
-                fence_proxy_async_smem();
-                named_bar_sync(2 + half, 128);
-                if (leader) {
-                    const int c0 = q * s.Qout + g.n_tile * BNQ;
-                    if constexpr (STORE3D)
-                        tma_store_3d(tmap_y, stg_addr, c0, g.sy, g.sz);
-                    else
-                        tma_store_2d(tmap_y, stg_addr, c0, g.sy);
-                    bulk_commit_group();
-                }
-            }
-        }
-        if constexpr (WIDE) {
-            fence_proxy_async_smem();
-            named_bar_sync(1, 256);
-            if (threadIdx.x == EPI_WARP0 * 32) {
-                if constexpr (STORE3D)
-                    tma_store_3d(tmap_y, stg_addr, 0, g.sy, g.sz);
-                else
-                    tma_store_2d(tmap_y, stg_addr, 0, g.sy);
-                bulk_commit_group();
-            }
-        }
-        tc_fence_before();
-        mbar_arrive(acce0 + 8u * buf);
-    }
-    if (leader || (WIDE && threadIdx.x == EPI_WARP0 * 32)) bulk_wait_group<0>();
-}
 
 // Direct epilogue for 64-channel outputs (Qout = 16: one output-channel tile), used by the
 // weight-stationary and pixel-pair kernels (16 warps: producer, 3 issuers, 12 epilogue).
@@ -354,17 +162,18 @@ constexpr int EPI_GROUPS = 3;
 constexpr int WIDE_THREADS = 512;  // block size of the kernels using this epilogue
 constexpr int EPI2_ACCE_COUNT = 128;  // the 4 warps of one group arrive once per tile
 
-// Tiles of a CTA are issued round robin by ISSUERS threads (local tile k by issuer
-// k % ISSUERS).  mbarrier parity waits only tell a phase from its neighbours, so a waiter
-// must never get two phases ahead of a barrier; that is guaranteed by letting every stage
-// and accumulator buffer be used by one issuer only, whose program order then orders the
+// Tiles of a CTA are issued round robin by NI threads (local tile k by issuer k % NI;
+// NI = ISSUERS = 3, or 2 where three issuers would leave each with too few stages).
+// mbarrier parity waits only tell a phase from its neighbours, so a waiter must never get
+// two phases ahead of a barrier; that is guaranteed by letting every stage and
+// accumulator buffer be used by one issuer only, whose program order then orders the
 // uses:
 //   - issuer i owns stages i * per .. i * per + per - 1; its n-th stage use (counting its
 //     K blocks in order) is stage i * per + n % per in round n / per;
-//   - issuer i owns accumulator buffers i and i + ISSUERS, alternating over its tiles;
+//   - issuer i owns accumulator buffers i and i + NI, alternating over its tiles;
 //     a buffer's tiles all have the same parity, so one epilogue group drains it.
 constexpr int ISSUERS = 3;
-constexpr int ISSUER_ACC = 2 * ISSUERS;  // accumulator buffers in use
+constexpr int ISSUER_ACC = 2 * ISSUERS;  // accumulator buffer barriers (64 columns each)
 
 __device__ __forceinline__ void issuer_stage(int i, int n, int per, int& stage,
                                              uint32_t& phase) {
@@ -372,10 +181,15 @@ __device__ __forceinline__ void issuer_stage(int i, int n, int per, int& stage,
     phase = static_cast<uint32_t>(n / per) & 1u;
 }
 
-__device__ __forceinline__ void issuer_acc(int k, int& buf, uint32_t& use) {
-    const int j = k / ISSUERS;
-    buf = (k - j * ISSUERS) + ISSUERS * (j & 1);
+template <int NI>
+__device__ __forceinline__ void issuer_acc_n(int k, int& buf, uint32_t& use) {
+    const int j = k / NI;
+    buf = (k - j * NI) + NI * (j & 1);
     use = static_cast<uint32_t>(j >> 1) & 1u;
+}
+
+__device__ __forceinline__ void issuer_acc(int k, int& buf, uint32_t& use) {
+    issuer_acc_n<ISSUERS>(k, buf, use);
 }
 
 // One transpose stage: lanes i and i ^ K exchange the chunks whose index differs from the
@@ -398,15 +212,178 @@ __device__ __forceinline__ void chunk_transpose_stage(float (&E)[NCH][8], int i)
     }
 }
 
-template <typename Geo>
+// v[0..7] = p[c .. c + 7] (p 16-byte aligned, c a multiple of 4), or `fill` if p is null.
+__device__ __forceinline__ void load8(const float* p, int c, float fill, float (&v)[8]) {
+    if (p == nullptr) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = fill;
+        return;
+    }
+    const float4 a = __ldg(reinterpret_cast<const float4*>(p + c));
+    const float4 b = __ldg(reinterpret_cast<const float4*>(p + c + 4));
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+// Direct epilogue of the QUAD/PAIR kernel (warps 4..11, two per TMEM lane quadrant;
+// warps 4..7 take output components r and i of every tile, warps 8..11 components j and k).
+// Accumulator buffer b (of two, used round robin over the CTA's tiles) lives at TMEM
+// columns [4 BNQ b, 4 BNQ (b+1)), component q at offset q BNQ.  A warp's share of a tile
+// is NB = 2 BNQ / CH blocks of its 32 rows x CH = min(BNQ, 32) columns; for each block it
+//   1. loads the block with one tcgen05.ld (after the last load of a tile it releases the
+//      accumulator buffer: acce, 256 arrivals per tile);
+//   2. transposes, within each group of NCH = CH / 8 lanes, the NCH x NCH matrix of
+//      8-channel chunks (rows x chunks) with shfl_xor, so every lane holds one chunk of
+//      NCH rows;
+//   3. applies act(scale * (acc + bias) + shift + residual) (IQBN inference form of
+//      Eq. 11-12; the affine step as fma(scale, acc, scale * bias + shift)), rounds to
+//      bf16 and writes 16 bytes per lane per row: each store instruction covers CH * 2
+//      contiguous bytes of 32 / NCH output rows.
+// The blocks are software-pipelined: the TMEM load and the per-channel vectors of block
+// b + 1 are requested before block b is processed, so their latency (hundreds of cycles
+// each, with the tensor cores busy on the other buffer) overlaps the work on block b.
+// No shared memory is touched (the tensor cores' operand reads keep that pipe busy); the
+// per-channel vectors are read through the L1 cache, 16 bytes at a time.
+template <int BNQ, typename Geo>
+__device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const EpilogueArgs& ep,
+                                                     void* y, uint32_t tmem_base,
+                                                     uint32_t accf0, uint32_t acce0,
+                                                     int num_tiles, uint64_t limit,
+                                                     volatile int* abort_flag, Geo geo) {
+    constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
+    constexpr int NCH = CH / 8;              // 8-channel chunks per load: 2 or 4
+    constexpr int SLICES = BNQ / CH;
+    constexpr int NB = 2 * SLICES;           // blocks per warp and tile
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
+    const int half = (warp - EPI_WARP0) >> 2;  // output components 2 half, 2 half + 1
+    const int ci = lane % NCH;                 // this lane's chunk after the transpose
+    const int row0 = quad * 32 + NCH * (lane / NCH);  // its rows: row0 .. row0 + NCH - 1
+    const long long Cout = s.Cout;
+    const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(ep.residual);
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(y);
+    // block b of this warp: component 2 half + b / SLICES, columns (b % SLICES) CH ..
+    auto tmem_col = [&](int b) { return (2 * half + b / SLICES) * BNQ + (b % SLICES) * CH; };
+    auto load_block = [&](uint32_t taddr, int b, uint32_t(&v)[CH]) {
+        if constexpr (CH == 32)
+            tmem_ld_32x32b_x32(taddr + tmem_col(b), v);
+        else
+            tmem_ld_32x32b_x16(taddr + tmem_col(b), v);
+    };
+    // the per-channel vectors of this lane's 8 channels of block b
+    auto load_vectors = [&](int cb, float(&sc)[8], float(&sh)[8]) {
+        float bi[8];
+        load8(ep.scale, cb, 1.0f, sc);
+        load8(ep.shift, cb, 0.0f, sh);
+        load8(ep.bias, cb, 0.0f, bi);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) sh[e] = fmaf(sc[e], bi[e], sh[e]);
+    };
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+        const int buf = local & 1;
+        const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        bool ok = true;
+        if (lane == 0)
+            ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        // leave together: a warp that gave up must not strand the others at a barrier
+        if (named_bar_or(1, 256, !ok)) break;
+        tc_fence_after();
+        const EpiTile g = geo(tile);
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                               static_cast<uint32_t>(buf * 4 * BNQ);
+        const int c_tile = g.n_tile * BNQ + 8 * ci;  // + q Qout + slice offset: lane's channel
+        uint32_t va[CH], vb[CH];
+        float sca[8], sha[8], scb[8], shb[8];
+        load_block(taddr, 0, va);
+        load_vectors(c_tile + (2 * half) * s.Qout, sca, sha);
+        tmem_ld_wait();
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            uint32_t(&v)[CH] = (b & 1) ? vb : va;
+            uint32_t(&vn)[CH] = (b & 1) ? va : vb;
+            float(&sc)[8] = (b & 1) ? scb : sca;
+            float(&sh)[8] = (b & 1) ? shb : sha;
+            float(&scn)[8] = (b & 1) ? sca : scb;
+            float(&shn)[8] = (b & 1) ? sha : shb;
+            const int q = 2 * half + b / SLICES;
+            const int cb = c_tile + q * s.Qout + (b % SLICES) * CH;
+            if (b + 1 < NB) {
+                // next block in flight while this one is processed
+                load_block(taddr, b + 1, vn);
+                load_vectors(c_tile + (2 * half + (b + 1) / SLICES) * s.Qout +
+                                 ((b + 1) % SLICES) * CH,
+                             scn, shn);
+            } else {
+                // the tile's accumulator is in registers: hand the buffer back
+                tc_fence_before();
+                mbar_arrive(acce0 + 8u * buf);
+            }
+            uint4 r4[NCH];
+            if (res != nullptr) {
+#pragma unroll
+                for (int k = 0; k < NCH; ++k) {
+                    r4[k] = make_uint4(0u, 0u, 0u, 0u);
+                    if (row0 + k < g.rows)
+                        r4[k] = ld_global_na(res + (g.m0 + row0 + k) * Cout + cb);
+                }
+            }
+            float E[NCH][8];  // E[j][e]: channel 8 j + e of this lane's row
+#pragma unroll
+            for (int j = 0; j < NCH; ++j)
+#pragma unroll
+                for (int e = 0; e < 8; ++e) E[j][e] = __uint_as_float(v[8 * j + e]);
+            if constexpr (NCH == 4) {
+                chunk_transpose_stage<2, 4>(E, ci);
+                chunk_transpose_stage<1, 4>(E, ci);
+            } else {
+                chunk_transpose_stage<1, 2>(E, ci);
+            }
+            // now E[k][e] = channel cb + e of row row0 + k
+#pragma unroll
+            for (int k = 0; k < NCH; ++k) {
+                float rz[8];
+                if (res != nullptr) {
+                    const __nv_bfloat162* rh = reinterpret_cast<const __nv_bfloat162*>(&r4[k]);
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const float2 f = __bfloat1622float2(rh[t]);
+                        rz[2 * t] = f.x;
+                        rz[2 * t + 1] = f.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) rz[e] = 0.0f;
+                }
+                uint32_t w[4];
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                    const float z0 = fmaf(sc[2 * t], E[k][2 * t], sh[2 * t]) + rz[2 * t];
+                    const float z1 =
+                        fmaf(sc[2 * t + 1], E[k][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
+                    w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                }
+                if (row0 + k < g.rows)
+                    st_global_na(out + (g.m0 + row0 + k) * Cout + cb,
+                                 make_uint4(w[0], w[1], w[2], w[3]));
+            }
+            if (b + 1 < NB) tmem_ld_wait();
+        }
+    }
+}
+
+// NG epilogue groups, one per MMA issuer (warps 4 + 4 NG .. 15 take no part).
+template <typename Geo, int NG = EPI_GROUPS>
 __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const EpilogueArgs& ep,
                                                   void* y, uint32_t tmem_base, uint32_t accf0,
                                                   uint32_t acce0, int num_tiles, uint64_t limit,
                                                   volatile int* abort_flag, Geo geo) {
-    static_assert(EPI_GROUPS == ISSUERS, "each epilogue group drains one issuer's buffers");
+    static_assert(NG >= 1 && NG <= EPI_GROUPS, "each epilogue group drains one issuer's buffers");
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int quad = warp & 3;                // TMEM lane quadrant this warp may access
-    const int grp = (warp - EPI_WARP0) >> 2;  // local tiles k with k % 3 == grp
+    const int grp = (warp - EPI_WARP0) >> 2;  // local tiles k with k % NG == grp
+    if (grp >= NG) return;
     const int ci = lane & 3;                  // this lane's chunk after the transpose
     const int rg = lane >> 2;                 // group of 4 rows (4 lanes) within the warp
     // the chunks' per-channel vectors (channels 8 ci + 32 h + e), in registers
@@ -424,10 +401,10 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
     __nv_bfloat16* out = static_cast<__nv_bfloat16*>(y);
     int local = grp;
     for (int tile = blockIdx.x + grp * gridDim.x; tile < num_tiles;
-         tile += EPI_GROUPS * gridDim.x, local += EPI_GROUPS) {
+         tile += NG * gridDim.x, local += NG) {
         int buf;
         uint32_t use;
-        issuer_acc(local, buf, use);
+        issuer_acc_n<NG>(local, buf, use);
         bool ok = true;
         if (lane == 0)
             ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);

@@ -69,6 +69,7 @@ def load():
         lib.quan_set_tc_tiles.argtypes = [_i, _i, _i, _i]
         lib.quan_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
         lib.quan_set_tc_halo.argtypes = [_i]
+        lib.quan_set_tc_issuers.argtypes = [_i]
         lib.quan_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_uint)]
         lib.quan_set_fault_injection.argtypes = [_i]
         lib.quan_status_string.argtypes = [_i]
@@ -79,7 +80,7 @@ def load():
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
-                     "quan_set_tc_halo"):
+                     "quan_set_tc_halo", "quan_set_tc_issuers"):
             getattr(lib, name).restype = _i
         lib.quan_last_path.restype = _i
         lib.quan_version.restype = _i
@@ -156,6 +157,10 @@ def quan_set_tc_tiles(kappa: int = 0, bnq: int = 0, max_ctas: int = 0, mode: int
 
 def quan_set_tc_halo(enable: bool) -> None:
     _check(load().quan_set_tc_halo(1 if enable else 0))
+
+
+def quan_set_tc_issuers(issuers: int = 0) -> None:
+    _check(load().quan_set_tc_issuers(issuers))
 
 
 def quan_set_wait_limit_ns(ns: int) -> None:

@@ -62,6 +62,10 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_set_tc_tiles(0, 0, 0, 5) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_tiles(0, 0, 0, 4) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 0) == quan.QUAN_OK
+    assert lib.quan_set_tc_issuers(1) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_issuers(4) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_issuers(2) == quan.QUAN_OK
+    assert lib.quan_set_tc_issuers(0) == quan.QUAN_OK
     assert lib.quan_set_path(0) == quan.QUAN_OK
     assert lib.quan_set_wait_limit_ns(0) == quan.QUAN_OK
 

@@ -39,6 +39,7 @@ def _reset_paths():
     quan.quan_set_fault_injection(False)
     quan.quan_set_wait_limit_ns(0)
     quan.quan_set_tc_halo(True)
+    quan.quan_set_tc_issuers(0)
 
 
 def run_gpu(d, path=quan.QUAN_PATH_AUTO, guard=True):
@@ -115,32 +116,41 @@ WS_CASES = [
 ]
 
 
+@pytest.mark.parametrize("issuers", [0, 2, 3])
 @pytest.mark.parametrize("halo", [1, 0])
 @pytest.mark.parametrize("case", WS_CASES, ids=[c[0] for c in WS_CASES])
-def test_tc_weight_stationary_layers(case, halo):
+def test_tc_weight_stationary_layers(case, halo, issuers):
     name, N, H, W, Cin, Cout, k, s, p, extra = case
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(205, len(name)), **extra)
     quan.quan_set_tc_tiles(0, 0, 0, 3)
     quan.quan_set_tc_halo(bool(halo))
+    quan.quan_set_tc_issuers(issuers)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
-    assert quan.quan_last_kernel().startswith("qconv_ws_kernel<")
+    kernel = quan.quan_last_kernel()
+    assert kernel.startswith("qconv_ws_kernel<")
+    if issuers:
+        assert kernel.endswith("issuers=%d>" % issuers)
 
 
+@pytest.mark.parametrize("issuers", [2, 3])
 @pytest.mark.parametrize("halo", [1, 0])
-def test_tc_weight_stationary_few_ctas(halo):
-    # 96 tiles on 3 CTAs: the accumulator ring, the stage ring and the epilogue's staging
-    # blocks all wrap many times
+def test_tc_weight_stationary_few_ctas(halo, issuers):
+    # 96 tiles on 3 CTAs: the accumulator buffers and every issuer's stages wrap many
+    # times
     spec = inputs.small_layer("ws_few", 12, 32, 32, 64, 64, 3, 1, 1, residual=True,
                               seed=(209, halo))
     quan.quan_set_tc_tiles(0, 0, 3, 3)
     quan.quan_set_tc_halo(bool(halo))
+    quan.quan_set_tc_issuers(issuers)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
+@pytest.mark.parametrize("issuers", [2, 3])
 @pytest.mark.parametrize("halo", [1, 0])
-def test_config1_weight_stationary_staging(halo):
+def test_config1_weight_stationary_staging(halo, issuers):
     quan.quan_set_tc_tiles(0, 0, 0, 3)
     quan.quan_set_tc_halo(bool(halo))
+    quan.quan_set_tc_issuers(issuers)
     check(inputs.LAYERS["c1"], path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
@@ -170,9 +180,8 @@ def test_tc_small_layers(case):
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
 
 
-# every (kappa, bnq, mode) whose stages fit in shared memory (64 x 64 does not)
-TILE_CASES = [(k, b, m) for m in (1, 2) for k in (16, 32, 64) for b in (16, 32, 64)
-              if not (k == 64 and b == 64)]
+# every (kappa, bnq, mode)
+TILE_CASES = [(k, b, m) for m in (1, 2) for k in (16, 32, 64) for b in (16, 32, 64)]
 
 
 @pytest.mark.parametrize("kappa,bnq,mode", TILE_CASES)
@@ -291,6 +300,27 @@ def test_misaligned_pointer_demotes_to_simt():
     assert_bf16_close(out_f64(y), oracle_full(d), "misaligned")
 
 
+def test_misaligned_channel_vector_demotes_to_simt():
+    # the tensor-core epilogues read the per-channel vectors 16 bytes at a time
+    spec = inputs.small_layer("mis_vec", 1, 6, 6, 64, 64, 3, 1, 1, seed=(302, 1))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
+    buf = torch.empty(sc.numel() + 4, dtype=torch.float32, device="cuda")
+    buf[1:1 + sc.numel()] = sc
+    scm = buf[1:1 + sc.numel()]                   # 4-byte aligned only
+    with pytest.raises(quan.QuanError) as ei:
+        quan.quan_set_path(quan.QUAN_PATH_TC)
+        quan.qconv2d(x, *w, stride=1, pad=1, scale=scm, shift=sh, act=spec.act)
+    assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+    quan.quan_set_path(quan.QUAN_PATH_AUTO)
+    y = quan.qconv2d(x, *w, stride=1, pad=1, scale=scm, shift=sh, act=spec.act)
+    torch.cuda.synchronize()
+    assert quan.quan_last_path() == quan.QUAN_PATH_SIMT
+    assert_bf16_close(out_f64(y), oracle_full(d), "misaligned-vector")
+
+
 # ------------------------------------------------------------------ full-size layers, sampled
 
 def sample_points(spec, n_random, seed):
@@ -389,9 +419,10 @@ def test_maxpool(shape):
 
 # ------------------------------------------------------------------ failure detection
 
-@pytest.mark.parametrize("mode", [2, 3, 4])
-def test_bounded_wait_timeout_every_kernel(mode):
-    # the failure-injection path of the pair-mode, weight-stationary and gather kernels
+@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0)])
+def test_bounded_wait_timeout_every_kernel(mode, issuers):
+    # the failure-injection path of the pair-mode, weight-stationary (two and three
+    # issuers) and gather kernels
     if mode == 4:
         spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
     else:
@@ -401,6 +432,7 @@ def test_bounded_wait_timeout_every_kernel(mode):
     w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
     quan.quan_set_path(quan.QUAN_PATH_TC)
     quan.quan_set_tc_tiles(0, 16 if mode == 2 else 0, 0, mode)
+    quan.quan_set_tc_issuers(issuers)
     quan.quan_set_wait_limit_ns(5_000_000)
     quan.quan_set_fault_injection(True)
     quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, act=spec.act)
