@@ -103,17 +103,29 @@ class BackboneRunner:
         return rows
 
     # ---------------------------------------------------------------- e2e (host buffers)
-    def e2e_setup(self):
+    # Buffer set b of the end-to-end pipeline is an input image batch and a copy of the
+    # last layer's output; the intermediate activations are shared, which is safe because
+    # every step's kernels run in order on one stream.
+    def e2e_setup(self, nbuf: int = 2):
         torch = self.torch
-        self.h_x = torch.from_numpy(np.ascontiguousarray(self.x_host).view(np.int16)).pin_memory()
+        self.h_x = torch.from_numpy(
+            np.ascontiguousarray(self.x_host).reshape(-1).view(np.uint8)).pin_memory()
         out = self.outs[-1]
-        self.h_out = torch.empty(out.shape, dtype=torch.int16).pin_memory()
-        self.e_x = self.x  # the device input buffer is refilled every step
-        self.h2d = self.h_x.numel() * 2
-        self.d2h = self.h_out.numel() * 2
+        self.h_out = [torch.empty(out.numel() * 2, dtype=torch.uint8).pin_memory()
+                      for _ in range(nbuf)]
+        self.e_x = [torch.empty_like(self.x) for _ in range(nbuf)]
+        self.e_out = [torch.empty_like(out) for _ in range(nbuf)]
+        self.h2d = self.h_x.numel()
+        self.d2h = self.h_out[0].numel()
 
-    def e2e_step(self, stream):
-        torch = self.torch
-        self.x.view(torch.int16).copy_(self.h_x, non_blocking=True)
-        self.step(stream)
-        self.h_out.copy_(self.outs[-1].view(torch.int16), non_blocking=True)
+    def e2e_in(self, b):
+        return [(self.e_x[b].view(-1).view(self.torch.uint8), self.h_x)]
+
+    def e2e_out(self, b):
+        return [(self.h_out[b], self.e_out[b].view(-1).view(self.torch.uint8))]
+
+    def e2e_compute(self, b, stream):
+        last = len(self.layers) - 1
+        for i in range(len(self.layers)):
+            x = self.e_x[b] if self.layers[i].src == -1 else None
+            self.run_layer(i, stream, x=x, out=self.e_out[b] if i == last else None)
