@@ -1,6 +1,7 @@
 // tc_common.cuh -- pieces shared by the tensor-core quaternion convolution kernels
 // (qconv_tc.cu is the only translation unit that includes this file): constants, the
-// device status word, descriptor helpers, bounded waits and the 8-warp epilogue.
+// device status word, descriptor helpers, bounded waits, the issuer bookkeeping and the
+// register-only epilogues.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
