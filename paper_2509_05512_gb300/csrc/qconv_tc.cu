@@ -701,12 +701,13 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
     set_kernel_name(halo ? "qconv_ws_kernel<halo,issuers=%d>" : "qconv_ws_kernel<im2col,issuers=%d>",
                     ni);
+    const bool k3x3 = s.kh == 3 && s.kw == 3;
     if (ni == 2) {
-        if (halo && s.kh == 3) return launch_ws_kernel<true, 3, 2>(maps[0], prm, grid, stream);
+        if (halo && k3x3) return launch_ws_kernel<true, 3, 2>(maps[0], prm, grid, stream);
         if (halo) return launch_ws_kernel<true, 0, 2>(maps[0], prm, grid, stream);
         return launch_ws_kernel<false, 0, 2>(maps[0], prm, grid, stream);
     }
-    if (halo && s.kh == 3) return launch_ws_kernel<true, 3, ISSUERS>(maps[0], prm, grid, stream);
+    if (halo && k3x3) return launch_ws_kernel<true, 3, ISSUERS>(maps[0], prm, grid, stream);
     if (halo) return launch_ws_kernel<true, 0, ISSUERS>(maps[0], prm, grid, stream);
     return launch_ws_kernel<false, 0, ISSUERS>(maps[0], prm, grid, stream);
 }

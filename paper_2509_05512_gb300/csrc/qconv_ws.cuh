@@ -94,12 +94,16 @@ int ws_issuers(int stage_bytes, int kblocks) {
 // value is sign(q, p) * W_{q xor p}[co][t][ci], rows of 128 bytes, 128-byte swizzle.  Each
 // 16-byte chunk of a compact letter L is read once from global memory (all of a thread's
 // chunks in flight together) and written to its four places (p = 0..3, q = L xor p).
+// TAPS > 0: the tap count known at compile time, so the chunk index splits with constant
+// divisions (the expansion sits on every launch's critical path and is bound by its
+// integer work); 0 = from the parameters.
+template <int TAPS>
 __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int warp,
                                           int lane, uint32_t wsready_bar) {
     using C = WsCfg;
     const int et = (warp - 2) * 32 + lane;  // 0 .. 447
     constexpr int ET = C::EXP_WARPS * 32;
-    const int taps = p.taps;
+    const int taps = TAPS > 0 ? TAPS : p.taps;
     const int letter_chunks = taps * 32;  // 16-byte chunks of one letter (16 x taps x 16)
     const int total = 4 * letter_chunks;
     uint4 v[4];
@@ -119,13 +123,14 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
         // chunk `off` of letter L holds W_L[co][t][ci0 .. ci0 + 7]
         const int co = off / (taps * 2), rem = off - co * (taps * 2);
         const int t = rem >> 1, half_ci = rem & 1;
+        const uint32_t signs = (LETTER_SIGNS >> (4 * L)) & 15u;
+        uint8_t* row = smem + C::WSB_OFF + t * C::TAP_BYTES + co * WS_ROW_BYTES;
+        const int sw = co & 7;  // the row's 128-byte swizzle phase (q * 16 keeps it)
 #pragma unroll
         for (int pc = 0; pc < 4; ++pc) {
-            const int q = L ^ pc;
-            const int n = q * 16 + co, ch = pc * 2 + half_ci;
-            const uint4 u = ((NEG_MASK >> (4 * q + pc)) & 1u) ? negate_bf16x8(v[r]) : v[r];
-            *reinterpret_cast<uint4*>(smem + C::WSB_OFF + t * C::TAP_BYTES + n * WS_ROW_BYTES +
-                                      ((ch ^ (n & 7)) << 4)) = u;
+            const int q = L ^ pc, ch = pc * 2 + half_ci;
+            const uint4 u = ((signs >> pc) & 1u) ? negate_bf16x8(v[r]) : v[r];
+            *reinterpret_cast<uint4*>(row + q * 16 * WS_ROW_BYTES + ((ch ^ sw) << 4)) = u;
         }
     }
     fence_proxy_async_smem();
@@ -133,8 +138,9 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
     if (lane == 0) mbar_arrive(wsready_bar);
 }
 
-// KH > 0: the filter height, known at compile time (halo staging), so the MMA issue
-// loop is fully unrolled; 0 = from the shape at run time.  NI: MMA issuers (2 or 3).
+// KH = 3: a 3x3 filter with halo staging, known at compile time, so the MMA issue loop is
+// fully unrolled and the expansion's tap count is a constant; 0 = from the shape at run
+// time.  NI: MMA issuers (2 or 3).
 template <bool HALO, int KH, int NI>
 __global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x, const WsParams p) {
@@ -254,7 +260,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
         }
     } else if (warp <= NI) {
         // ------------------------------------------------------------ MMA issuers
-        if (warp >= 2) ws_expand(p, smem, warp, lane, wsready_bar);
+        if (warp >= 2) ws_expand<KH == 3 ? 9 : 0>(p, smem, warp, lane, wsready_bar);
         if (lane == 0) {
             constexpr uint32_t IDESC = make_idesc(BM, 64, 0);
             const int me = warp - 1;
@@ -338,7 +344,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             }
         }
     } else {
-        ws_expand(p, smem, warp, lane, wsready_bar);
+        ws_expand<KH == 3 ? 9 : 0>(p, smem, warp, lane, wsready_bar);
         // ------------------------------------------- epilogue (warps 4 .. 4 + 4 NI - 1)
         const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
         const long long M = s.M;

@@ -34,6 +34,16 @@ constexpr uint32_t NEG_MASK = (1u << 1) | (1u << 2) | (1u << 3)  // y_r: X_i, X_
                               | (1u << 11)                       // y_j: X_k
                               | (1u << 13);                      // y_k: X_i
 
+// The same signs indexed by letter: bit (4 L + p) is set when letter L enters through input
+// component p (output component L xor p) with a minus sign.
+constexpr uint32_t letter_sign_table() {
+    uint32_t t = 0;
+    for (int L = 0; L < 4; ++L)
+        for (int p = 0; p < 4; ++p) t |= ((NEG_MASK >> (4 * (L ^ p) + p)) & 1u) << (4 * L + p);
+    return t;
+}
+constexpr uint32_t LETTER_SIGNS = letter_sign_table();
+
 // tcgen05 shared-memory matrix descriptors (K-major, swizzled operand tiles) are built
 // as two 32-bit words: the low word holds the start address >> 4 (bits 0-13) and the
 // leading byte offset (bits 16-29, unused for these layouts, set to 1); the high word
