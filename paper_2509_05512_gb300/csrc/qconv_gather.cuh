@@ -245,14 +245,18 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
             const uint32_t tx = static_cast<uint32_t>(s.kh * p.box_bytes);
-            int k = 0;
-            for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x, ++k) {
+            StageCursor cur(p.per);  // advanced once per round of ISSUERS tiles
+            int ki = 0;              // local tile k % ISSUERS
+            for (int tile = blockIdx.x; tile < p.num_tiles; tile += gridDim.x) {
                 const int row = tile / p.segs, seg = tile - (tile / p.segs) * p.segs;
                 const int img = row / s.Ho, ho = row - (row / s.Ho) * s.Ho;
                 // local tile k -> issuer k % ISSUERS, its (k / ISSUERS)-th stage use
-                int stage;
-                uint32_t phase;
-                issuer_stage(k % ISSUERS, k / ISSUERS, p.per, stage, phase);
+                const int stage = cur.stage(ki);
+                const uint32_t phase = cur.phase;
+                if (++ki == ISSUERS) {
+                    ki = 0;
+                    cur.next();
+                }
                 if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_PRODUCER)) {
                     ok = false;
@@ -288,13 +292,16 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             const uint32_t b_lo0 = desc_lo(sbase + C::B_OFF);
             const int half = p.nsp / 2;
             // local tile k of this CTA is tile blockIdx.x + k * gridDim.x; this issuer's
-            // j-th tile is k = me + j * ISSUERS
-            for (int k = me, j = 0, tile = blockIdx.x + me * gridDim.x; ok && tile < p.num_tiles;
-                 k += ISSUERS, ++j, tile += ISSUERS * gridDim.x) {
-                int buf, stage;
-                uint32_t use, phase;
+            // tiles are k = me, me + ISSUERS, ...
+            StageCursor cur(p.per);
+            for (int k = me, tile = blockIdx.x + me * gridDim.x; ok && tile < p.num_tiles;
+                 k += ISSUERS, tile += ISSUERS * gridDim.x) {
+                int buf;
+                uint32_t use;
                 issuer_acc(k, buf, use);
-                issuer_stage(me, j, p.per, stage, phase);
+                const int stage = cur.stage(me);  // this issuer's (k / ISSUERS)-th stage use
+                const uint32_t phase = cur.phase;
+                cur.next();
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA) ||
                     !wait_or_abort(full_bar(stage), phase, limit, abort_flag,

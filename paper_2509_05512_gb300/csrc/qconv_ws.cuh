@@ -218,6 +218,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             const uint64_t pol_x = l2_policy_evict_normal();
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
+            StageCursor cur(p.per);
             for (int g0 = 0; ok && g0 < kt; g0 += NI) {
                 const int ng = kt - g0 < NI ? kt - g0 : NI;
                 int img[NI], hbase[NI], wbase[NI];
@@ -226,14 +227,14 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
                     if (i < ng)
                         tile_base(static_cast<int>(blockIdx.x) + (g0 + i) * static_cast<int>(gridDim.x),
                                   img[i], hbase[i], wbase[i]);
-                for (int kb = 0; ok && kb < p.kblocks; ++kb) {
+                for (int kb = 0; ok && kb < p.kblocks; ++kb, cur.next()) {
 #pragma unroll
                     for (int i = 0; i < NI; ++i) {
                         if (i >= ng) break;
-                        // K block kb of local tile g0 + i: use (g0 / NI) * kblocks + kb of issuer i
-                        int stage;
-                        uint32_t phase;
-                        issuer_stage(i, (g0 / NI) * p.kblocks + kb, p.per, stage, phase);
+                        // K block kb of local tile g0 + i: use (g0 / NI) * kblocks + kb of
+                        // issuer i, the same use count for every issuer of the group
+                        const int stage = cur.stage(i);
+                        const uint32_t phase = cur.phase;
                         if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                            STATUS_TIMEOUT_PRODUCER)) {
                             ok = false;
@@ -276,7 +277,8 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             const uint32_t wsb_lo = desc_lo(sbase + C::WSB_OFF);
             const uint32_t row_lo = (s.Wo * WS_ROW_BYTES) >> 4;  // one output row of pixels
             const uint32_t b_row = (s.kw * C::TAP_BYTES) >> 4;    // one filter row of taps
-            for (int k = me, j = 0; ok && k < kt; k += NI, ++j) {
+            StageCursor cur(p.per);
+            for (int k = me; ok && k < kt; k += NI) {
                 int buf;
                 uint32_t use;
                 issuer_acc_n<NI>(k, buf, use);
@@ -288,9 +290,10 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * 64);
                 for (int kb = 0; kb < p.kblocks; ++kb) {
-                    int stage;
-                    uint32_t phase;
-                    issuer_stage(me, j * p.kblocks + kb, p.per, stage, phase);
+                    // use (k / NI) * kblocks + kb of this issuer
+                    const int stage = cur.stage(me);
+                    const uint32_t phase = cur.phase;
+                    cur.next();
                     if (!wait_or_abort(full_bar(stage), phase, limit, abort_flag,
                                        STATUS_TIMEOUT_MMA)) {
                         ok = false;

@@ -192,6 +192,23 @@ __device__ __forceinline__ void issuer_stage(int i, int n, int per, int& stage,
     phase = static_cast<uint32_t>(n / per) & 1u;
 }
 
+// The same mapping walked one use at a time, without the division by `per` (an issuing
+// thread's integer work between MMAs is idle tensor time): after n calls of next(),
+// stage(i) and phase equal issuer_stage(i, n, ...).  One cursor serves every issuer whose
+// use counts advance together.
+struct StageCursor {
+    int per, idx;
+    uint32_t phase;
+    __device__ __forceinline__ explicit StageCursor(int per_) : per(per_), idx(0), phase(0u) {}
+    __device__ __forceinline__ int stage(int i) const { return i * per + idx; }
+    __device__ __forceinline__ void next() {
+        if (++idx == per) {
+            idx = 0;
+            phase ^= 1u;
+        }
+    }
+};
+
 template <int NI>
 __device__ __forceinline__ void issuer_acc_n(int k, int& buf, uint32_t& use) {
     const int j = k / NI;
