@@ -197,9 +197,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
                 const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
                 const int wbase = wo * s.stride - s.pad, hbase = ho * s.stride - s.pad;
+                // K block kt = (tap, chunk), tap = dh * kw + dw: walked without divisions
+                int chunk = 0, tap = 0, dh = 0, dw = 0;
                 for (int kt = 0; kt < p.ktiles; ++kt) {
-                    const int tap = kt / p.kchunks, chunk = kt - tap * p.kchunks;
-                    const int dh = tap / s.kw, dw = tap - (tap / s.kw) * s.kw;
+                    if (kt > 0 && ++chunk == p.kchunks) {
+                        chunk = 0;
+                        ++tap;
+                        if (++dw == s.kw) {
+                            dw = 0;
+                            ++dh;
+                        }
+                    }
                     if (!wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
                                        STATUS_TIMEOUT_PRODUCER)) {
                         ok = false;
