@@ -42,6 +42,9 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c1",
                     choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone"])
+    ap.add_argument("--variant", choices=["full", "separable"], default="full",
+                    help="layer workloads: the full Hamilton form (Eq. 5/6) or the separable "
+                         "form of Eq. 7 (a quarter of the multiply-adds)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -189,9 +192,11 @@ class LayerRunner:
     """Device buffers for one layer, rotated so that consecutive steps never find their
     inputs in L2."""
 
-    def __init__(self, spec, torch, quan, inputs):
+    def __init__(self, spec, torch, quan, inputs, separable=False):
         import numpy as np
         self.spec, self.torch, self.quan = spec, torch, quan
+        self.separable = separable
+        self.conv = quan.quan_qconv2d_sep_fwd if separable else quan.quan_qconv2d_fwd
         d = inputs.layer_inputs(spec)
         dev = torch.device("cuda")
 
@@ -215,12 +220,11 @@ class LayerRunner:
         self.footprint = per_set * self.sets
 
     def step(self, stream):
-        s, q = self.spec, self.quan
+        s = self.spec
         k = self.i % self.sets
         self.i += 1
-        q.quan_qconv2d_fwd(self.xs[k], *self.w, self.bias, self.scale, self.shift, s.N, s.H,
-                           s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
-                           self.outs[k], stream)
+        self.conv(self.xs[k], *self.w, self.bias, self.scale, self.shift, s.N, s.H, s.W, s.Cin,
+                  s.Cout, s.kh, s.kw, s.stride, s.pad, s.act, self.outs[k], stream)
 
     # end to end: pinned host inputs -> device -> kernel -> host, with E2E_BUFFERS device
     # buffer sets so that one step's copies overlap another step's kernel (e2e_pipeline).
@@ -269,39 +273,40 @@ class LayerRunner:
 
         w = [view(k, torch.bfloat16) for k in ("wr", "wi", "wj", "wk")]
         out = self.e_out[b].view(torch.bfloat16).view(s.N, s.Ho, s.Wo, s.Cout)
-        q.quan_qconv2d_fwd(view("x", torch.bfloat16), *w, view("bias", torch.float32),
-                           view("scale", torch.float32), view("shift", torch.float32), s.N,
-                           s.H, s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act, out,
-                           stream)
+        self.conv(view("x", torch.bfloat16), *w, view("bias", torch.float32),
+                  view("scale", torch.float32), view("shift", torch.float32), s.N, s.H, s.W,
+                  s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act, out, stream)
 
     @property
     def flops(self):
-        return self.spec.flops
+        # the separable form keeps the 4 diagonal component convolutions of the 16
+        return self.spec.flops / 4 if self.separable else self.spec.flops
 
     @property
     def algorithmic_bytes(self):
         return self.spec.algorithmic_bytes
 
 
-def cpu_oracle_sample(spec, seconds, inputs):
+def cpu_oracle_sample(spec, seconds, inputs, separable=False):
     """Time the fp64 oracle on a bounded number of images of the layer."""
     import oracle
     d = inputs.layer_inputs(spec, n_images=1)
     f64 = oracle.bf16_bits_to_f64
     w = [f64(d[k]) for k in ("wr", "wi", "wj", "wk")]
+    conv = oracle.qconv2d_separable if separable else oracle.qconv2d
 
     def run(n):
         dd = inputs.layer_inputs(spec, n_images=n)
         x = f64(dd["x"])
         t0 = time.perf_counter()
-        oracle.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"],
-                       scale=d["scale"], shift=d["shift"], act=spec.act)
+        conv(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"], scale=d["scale"],
+             shift=d["shift"], act=spec.act)
         return time.perf_counter() - t0
 
     t1 = run(1)
     n = max(1, min(spec.N, int(seconds / max(t1, 1e-6))))
     t = run(n) if n > 1 else t1
-    flop = spec.flops / spec.N * n
+    flop = spec.flops / spec.N * n / (4 if separable else 1)
     return {"value": flop / t / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(),
             "kind": "oracle",
             "sample": "%d of %d images of the layer (fp64, %.2f s)" % (n, spec.N, t)}
@@ -319,7 +324,7 @@ WORKLOAD_DESC = {
 }
 
 
-def workload_config(workload: str, inputs) -> dict:
+def workload_config(workload: str, inputs, variant: str = "full") -> dict:
     """The workload part of the JSON line's config, shared by both arms."""
     if workload == "backbone":
         layers = inputs.backbone_layers()
@@ -331,9 +336,13 @@ def workload_config(workload: str, inputs) -> dict:
                 "flops_per_step": sum(c.flops for c in convs),
                 "epilogue": "IQBN+ReLU (+residual)"}
     s = inputs.LAYERS[workload]
-    return {"workload": WORKLOAD_DESC[workload], "N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin,
-            "Cout": s.Cout, "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
-            "epilogue": "IQBN+ReLU", "flops_per_step": s.flops}
+    cfg = {"workload": WORKLOAD_DESC[workload], "N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin,
+           "Cout": s.Cout, "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
+           "epilogue": "IQBN+ReLU", "flops_per_step": s.flops}
+    if variant == "separable":
+        cfg["workload"] += ", separable form (Eq. 7)"
+        cfg["flops_per_step"] = s.flops / 4
+    return cfg
 
 
 def max_over_ranks(ms: float, dist, torch, device: str) -> float:
@@ -379,6 +388,8 @@ def main():
     if args.batch and not args.profile:
         raise SystemExit("--batch is for --profile runs only")
     if args.workload == "backbone":
+        if args.variant != "full":
+            raise SystemExit("--variant applies to the single-layer workloads")
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256)
         runner.sets = 1
@@ -388,8 +399,8 @@ def main():
         if args.batch:
             import dataclasses
             spec = dataclasses.replace(spec, N=args.batch)
-        runner = LayerRunner(spec, torch, quan, inputs)
-        unit, per_step_units, dtype = "TFLOP/s", spec.flops / 1e12, "bf16"
+        runner = LayerRunner(spec, torch, quan, inputs, separable=args.variant == "separable")
+        unit, per_step_units, dtype = "TFLOP/s", runner.flops / 1e12, "bf16"
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
 
@@ -479,13 +490,14 @@ def main():
         if args.workload == "backbone":
             cpu = backbone_cpu_sample(runner, args.cpu_seconds, inputs)
         else:
-            cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs)
+            cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs,
+                                    separable=runner.separable)
 
     if dist is not None:
         dist.destroy_process_group()
     if rank != 0:
         return 0
-    cfg = workload_config(args.workload, inputs)
+    cfg = workload_config(args.workload, inputs, args.variant)
     cfg.update({"l2": "inputs larger than L2: %d rotating buffer sets, %.0f MB" % (
                     getattr(runner, "sets", 1), runner.footprint / 1e6),
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
@@ -513,7 +525,8 @@ def runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name):
         achieved, peak, unit, bound = nbytes / t / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
     return {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
             "frac": round(achieved / peak, 4),
-            "traffic": recorded_traffic(args.workload, kernel_name),
+            "traffic": recorded_traffic(args.workload + (":sep" if args.variant == "separable"
+                                                         else ""), kernel_name),
             "kernel": kernel_name, "peak_source": peak_src + " (burst)",
             "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
 
@@ -590,7 +603,7 @@ def reference_arm(args, rank, world, inputs):
     if rank != 0:
         return 0
     import oracle
-    ref_cfg = workload_config(args.workload, inputs)
+    ref_cfg = workload_config(args.workload, inputs, args.variant)
     ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
     if args.workload == "backbone":
         import oracle.backbone as ob
@@ -622,9 +635,12 @@ def reference_arm(args, rank, world, inputs):
     x = f64(d["x"])
     w = [f64(d[k]) for k in ("wr", "wi", "wj", "wk")]
 
+    sep = args.variant == "separable"
+    conv = oracle.qconv2d_separable if sep else oracle.qconv2d
+
     def step():
-        oracle.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"],
-                       scale=d["scale"], shift=d["shift"], act=spec.act)
+        conv(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"], scale=d["scale"],
+             shift=d["shift"], act=spec.act)
 
     for _ in range(args.warmup):
         step()
@@ -632,7 +648,7 @@ def reference_arm(args, rank, world, inputs):
     for _ in range(args.steps):
         step()
     dt = time.perf_counter() - t0
-    per_step = spec.flops / spec.N  # one image per step
+    per_step = spec.flops / spec.N / (4 if sep else 1)  # one image per step
     value = per_step * args.steps / dt / 1e12
     cpu = {"value": value, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
            "sample": "1 of %d images of the layer per step (fp64)" % spec.N}

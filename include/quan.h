@@ -107,6 +107,23 @@ quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi
                                    const void* residual, void* out, quan_stream_t stream);
 
 /*
+ * The separable QUAN convolution of Eq. 7 (Sec. III-B), bf16, same arguments, layouts,
+ * epilogue and errors as quan_qconv2d_fwd.  Each output component is a signed sum of the
+ * four per-component convolutions c_p = W_p (*) x_p (p = r, i, j, k):
+ *   y_r = c_r - c_i - c_j - c_k,   y_i = c_r + c_i + c_j - c_k,
+ *   y_j = c_r - c_i + c_j + c_k,   y_k = c_r + c_i - c_j + c_k,
+ * a quarter of the full form's multiply-adds (the cross-component terms W_L x_p, L != p,
+ * are dropped, as the paper describes).  The tensor-core path needs Cin/4 and Cout/4
+ * multiples of 16 and 16-byte aligned pointers; other shapes run on CUDA cores.  MMA-mode
+ * overrides (quan_set_tc_tiles' mode) must be 0: UNSUPPORTED otherwise.
+ */
+quan_status_t quan_qconv2d_sep_fwd(const void* x, const void* wr, const void* wi,
+                                   const void* wj, const void* wk, const float* bias,
+                                   const float* iqbn_scale, const float* iqbn_shift, int N, int H,
+                                   int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                   int act, void* out, quan_stream_t stream);
+
+/*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,
  * QSPPF), bf16 NHWC [N][H][W][C] -> [N][Ho][Wo][C], window k x k, stride, zero-size
  * padding that never wins.  C is any positive count.

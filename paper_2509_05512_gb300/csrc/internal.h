@@ -13,6 +13,7 @@ struct ConvShape {
     int N, H, W, Cin, Cout, kh, kw, stride, pad, act;
     int Ho, Wo, Qin, Qout;
     long long M;  // N * Ho * Wo output pixels
+    int sep;      // 1: the separable form of Eq. 7 (per-component convolutions, sign mix)
 };
 
 struct EpilogueArgs {

@@ -10,6 +10,10 @@
 //   y_k = W_r x_k + W_i x_j - W_j x_i + W_k x_r
 // summed over taps and input quaternion channels, followed by the fused epilogue
 // act(scale * (acc + bias) + shift + residual) (IQBN inference form of Eq. 11-12).
+// The separable form of Eq. 7 (s.sep) keeps only the diagonal convolutions
+// c_p = W_p x_p and mixes them with that equation's signs:
+//   y_r = c_r - c_i - c_j - c_k,  y_i = c_r + c_i + c_j - c_k,
+//   y_j = c_r - c_i + c_j + c_k,  y_k = c_r + c_i - c_j + c_k.
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -61,6 +65,16 @@ __global__ void __launch_bounds__(256) qconv_simt_kernel(ConvShape s, const T* _
             const T* pi = wi + wofs * Qin;
             const T* pj = wj + wofs * Qin;
             const T* pk = wk + wofs * Qin;
+            if (s.sep) {
+                // c_r .. c_k accumulate in ar .. ak
+                for (int ci = 0; ci < Qin; ++ci) {
+                    ar = fmaf(to_f32(__ldg(pr + ci)), to_f32(xp[ci]), ar);
+                    ai = fmaf(to_f32(__ldg(pi + ci)), to_f32(xp[Qin + ci]), ai);
+                    aj = fmaf(to_f32(__ldg(pj + ci)), to_f32(xp[2 * Qin + ci]), aj);
+                    ak = fmaf(to_f32(__ldg(pk + ci)), to_f32(xp[3 * Qin + ci]), ak);
+                }
+                continue;
+            }
             for (int ci = 0; ci < Qin; ++ci) {
                 const float xr = to_f32(xp[ci]), xi = to_f32(xp[Qin + ci]);
                 const float xj = to_f32(xp[2 * Qin + ci]), xk = to_f32(xp[3 * Qin + ci]);
@@ -73,7 +87,13 @@ __global__ void __launch_bounds__(256) qconv_simt_kernel(ConvShape s, const T* _
             }
         }
     }
-    const float acc[4] = {ar, ai, aj, ak};
+    float acc[4] = {ar, ai, aj, ak};
+    if (s.sep) {
+        acc[0] = ar - ai - aj - ak;
+        acc[1] = ar + ai + aj - ak;
+        acc[2] = ar - ai + aj + ak;
+        acc[3] = ar + ai - aj + ak;
+    }
     T* op = out + m * s.Cout;
     const T* rp = ep.residual ? static_cast<const T*>(ep.residual) + m * s.Cout : nullptr;
 #pragma unroll

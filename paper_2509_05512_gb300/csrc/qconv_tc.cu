@@ -21,6 +21,9 @@
 //              warp writes the two negated copies.  The larger N keeps the tensor pipe
 //              busy (an M=128 MMA costs at least ~45 cycles on this part, a full N=64 one
 //              is 32 cycles of work, N=128 is 64).
+//   MODE_SEP   the separable form of Eq. 7: 4 MMAs per K step, D_p += X_p * W_p^T
+//              (N = BNQ), one per input component; the epilogue mixes the four D_p
+//              with the signs of Eq. 7 (epilogue_direct_sep), so no negated letters.
 //   MODE_WS    (16 -> 16 quaternion channels, at most 9 taps; qconv_ws.cuh)
 //              weight-stationary: every CTA expands the whole signed block weight once
 //              into shared memory and streams only pixels; N = 64 MMAs cover all four
@@ -70,6 +73,7 @@ void set_kernel_name(const char* fmt, int a = 0, int b = 0) {
 constexpr int MODE_QUAD = 0;
 constexpr int MODE_PAIR = 1;
 constexpr int MODE_WS = 2;
+constexpr int MODE_SEP = 3;
 constexpr int WS_MAX_TAPS = 9;
 constexpr int MAX_STAGES = 8;
 
@@ -317,6 +321,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                            NEG1[pc] ? IDESC_NEG : IDESC_POS, acc);
                                 umma_f16_w(dbase + 2 * BNQ, a_lo, C::DESC_HI, b2, C::DESC_HI,
                                            IDESC_POS, acc);
+                            } else if constexpr (MODE == MODE_SEP) {
+                                // D_pc += X_pc * W_pc^T (letter pc sits in slot pc); D_pc's
+                                // first MMA of a tile is its own ks = 0 of K block 0
+                                const uint32_t b_lo =
+                                    b_lo0 + ((pc * C::B_TILE + ks * (UMMA_K * 2)) >> 4);
+                                umma_f16_w(dbase + pc * BNQ, a_lo, C::DESC_HI, b_lo, C::DESC_HI,
+                                           IDESC_POS, ks != 0 ? 1u : first);
                             } else {
 #pragma unroll
                                 for (int q = 0; q < 4; ++q) {
@@ -403,17 +414,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // ------------------------------------------------------------ epilogue
         const int num_n = p.num_n_tiles;
         const long long M = s.M;
-        epilogue_direct_pair<BNQ>(
-            s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit, abort_flag,
-            [num_n, M](int tile) {
-                EpiTile g;
-                const int m_tile = tile / num_n;
-                g.n_tile = tile - m_tile * num_n;
-                g.m0 = static_cast<long long>(m_tile) * BM;
-                const long long left = M - g.m0;
-                g.rows = left < BM ? static_cast<int>(left) : BM;
-                return g;
-            });
+        auto geo = [num_n, M](int tile) {
+            EpiTile g;
+            const int m_tile = tile / num_n;
+            g.n_tile = tile - m_tile * num_n;
+            g.m0 = static_cast<long long>(m_tile) * BM;
+            const long long left = M - g.m0;
+            g.rows = left < BM ? static_cast<int>(left) : BM;
+            return g;
+        };
+        if constexpr (MODE == MODE_SEP)
+            epilogue_direct_sep<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit,
+                                     abort_flag, geo);
+        else
+            epilogue_direct_pair<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit,
+                                      abort_flag, geo);
     }
 
     tc_fence_before();
@@ -707,8 +722,14 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    set_kernel_name(halo ? "qconv_ws_kernel<halo,issuers=%d>" : "qconv_ws_kernel<im2col,issuers=%d>",
-                    ni);
+    if (s.sep)
+        set_kernel_name(halo ? "qconv_ws_kernel<halo,issuers=%d,sep>"
+                             : "qconv_ws_kernel<im2col,issuers=%d,sep>",
+                        ni);
+    else
+        set_kernel_name(halo ? "qconv_ws_kernel<halo,issuers=%d>"
+                             : "qconv_ws_kernel<im2col,issuers=%d>",
+                        ni);
     const bool k3x3 = s.kh == 3 && s.kw == 3;
     if (ni == 2) {
         if (halo && k3x3) return launch_ws_kernel<true, 3, 2>(maps[0], prm, grid, stream);
@@ -790,7 +811,7 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
                   const EpilogueArgs& ep) {
     auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
-    if ((s.Qin % 16 != 0 || s.Qout % 16 != 0) && !gather_ok(s)) return false;
+    if ((s.Qin % 16 != 0 || s.Qout % 16 != 0) && (s.sep || !gather_ok(s))) return false;
     // TMA coordinates of the output (pixel index) are 32-bit
     if (s.M > 0x7fffffffLL) return false;
     if (!al16(x) || !al16(out) || !al16(w[0]) || !al16(w[1]) || !al16(w[2]) || !al16(w[3]))
@@ -815,7 +836,11 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
         snprintf(err, errlen, "tensor-map encoders unavailable from the CUDA driver");
         return cudaErrorNotSupported;
     }
-    if (gather_ok(s) && (opt.mode == 0 || opt.mode == 4))
+    if (s.sep && opt.mode != 0) {
+        snprintf(err, errlen, "MMA-mode overrides apply to the full Hamilton form only");
+        return cudaErrorInvalidValue;
+    }
+    if (!s.sep && gather_ok(s) && (opt.mode == 0 || opt.mode == 4))
         return launch_gather(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     if (opt.mode == 4) {
         snprintf(err, errlen,
@@ -830,7 +855,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     int kappa = pick_kappa(s.Qin, opt.kappa);
     const int bnq = pick_bnq(s.Qout, opt.bnq);
     int mode;
-    if (opt.mode == 1) mode = MODE_QUAD;
+    if (s.sep) mode = ws_ok ? MODE_WS : MODE_SEP;
+    else if (opt.mode == 1) mode = MODE_QUAD;
     else if (opt.mode == 2) mode = MODE_PAIR;
     else if (opt.mode == 3) mode = MODE_WS;
     else mode = ws_ok ? MODE_WS : (bnq >= 32 ? MODE_PAIR : MODE_QUAD);
@@ -854,7 +880,9 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
         bool fits = true;
 #define QUAN_FIT_CASE(K, B)                                                        \
     if (kappa == K && bnq == B)                                                    \
-        fits = mode == MODE_PAIR ? cfg_fits<K, B, MODE_PAIR>() : cfg_fits<K, B, MODE_QUAD>();
+        fits = mode == MODE_PAIR ? cfg_fits<K, B, MODE_PAIR>()                     \
+             : mode == MODE_SEP  ? cfg_fits<K, B, MODE_SEP>()                      \
+                                 : cfg_fits<K, B, MODE_QUAD>();
         QUAN_FIT_CASE(16, 16) QUAN_FIT_CASE(16, 32) QUAN_FIT_CASE(16, 64)
         QUAN_FIT_CASE(32, 16) QUAN_FIT_CASE(32, 32) QUAN_FIT_CASE(32, 64)
         QUAN_FIT_CASE(64, 16) QUAN_FIT_CASE(64, 32) QUAN_FIT_CASE(64, 64)
@@ -897,14 +925,16 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    set_kernel_name(mode == MODE_PAIR ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
-                                      : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
+    set_kernel_name(mode == MODE_PAIR  ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
+                    : mode == MODE_SEP ? "qconv_tc_kernel<sep,kappa=%d,bnq=%d>"
+                                       : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
                     kappa, bnq);
 
 #define QUAN_TC_CASE(K, B)                                                       \
     if (kappa == K && bnq == B)                                                  \
-        return mode == MODE_PAIR ? launch_cfg<K, B, MODE_PAIR>(maps, prm, grid, stream) \
-                                 : launch_cfg<K, B, MODE_QUAD>(maps, prm, grid, stream);
+        return mode == MODE_PAIR  ? launch_cfg<K, B, MODE_PAIR>(maps, prm, grid, stream) \
+               : mode == MODE_SEP ? launch_cfg<K, B, MODE_SEP>(maps, prm, grid, stream)  \
+                                  : launch_cfg<K, B, MODE_QUAD>(maps, prm, grid, stream);
     QUAN_TC_CASE(16, 16)
     QUAN_TC_CASE(16, 32)
     QUAN_TC_CASE(16, 64)

@@ -9,6 +9,10 @@
 // so one 16-wide K step of an MMA is one input component p, and an MMA of N = 64 covers
 // all four output components.
 //
+// The separable form of Eq. 7 runs here too: its block weight has sign * W_p in every row
+// block of column block p (ws_expand<.., true>), so the MMAs and the epilogue are those of
+// the full form and the sign mix comes with the weight.
+//
 // Pixel staging, per tile of 128 output pixels:
 //   halo     (stride 1, output width Wo a multiple of 8, at most 128): the tile is
 //            R = 128 / Wo whole output rows of one image; for each horizontal filter
@@ -96,8 +100,10 @@ int ws_issuers(int stage_bytes, int kblocks) {
 // chunks in flight together) and written to its four places (p = 0..3, q = L xor p).
 // TAPS > 0: the tap count known at compile time, so the chunk index splits with constant
 // divisions (the expansion sits on every launch's critical path and is bound by its
-// integer work); 0 = from the parameters.
-template <int TAPS>
+// integer work); 0 = from the parameters.  SEP: the separable form of Eq. 7 instead, whose
+// block weight has letter p in every row block of column block p (sign * W_p), so the
+// same MMAs compute it with the sign mix folded into the weight.
+template <int TAPS, bool SEP>
 __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int warp,
                                           int lane, uint32_t wsready_bar) {
     using C = WsCfg;
@@ -123,13 +129,14 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
         // chunk `off` of letter L holds W_L[co][t][ci0 .. ci0 + 7]
         const int co = off / (taps * 2), rem = off - co * (taps * 2);
         const int t = rem >> 1, half_ci = rem & 1;
-        const uint32_t signs = (LETTER_SIGNS >> (4 * L)) & 15u;
+        const uint32_t signs = ((SEP ? SEP_LETTER_SIGNS : LETTER_SIGNS) >> (4 * L)) & 15u;
         uint8_t* row = smem + C::WSB_OFF + t * C::TAP_BYTES + co * WS_ROW_BYTES;
         const int sw = co & 7;  // the row's 128-byte swizzle phase (q * 16 keeps it)
 #pragma unroll
-        for (int pc = 0; pc < 4; ++pc) {
-            const int q = L ^ pc, ch = pc * 2 + half_ci;
-            const uint4 u = ((signs >> pc) & 1u) ? negate_bf16x8(v[r]) : v[r];
+        for (int j = 0; j < 4; ++j) {
+            // Hamilton: row block L xor j, column block j; separable: row block j, column L
+            const int q = SEP ? j : L ^ j, ch = (SEP ? L : j) * 2 + half_ci;
+            const uint4 u = ((signs >> j) & 1u) ? negate_bf16x8(v[r]) : v[r];
             *reinterpret_cast<uint4*>(row + q * 16 * WS_ROW_BYTES + ((ch ^ sw) << 4)) = u;
         }
     }
@@ -261,7 +268,10 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
         }
     } else if (warp <= NI) {
         // ------------------------------------------------------------ MMA issuers
-        if (warp >= 2) ws_expand<KH == 3 ? 9 : 0>(p, smem, warp, lane, wsready_bar);
+        if (warp >= 2) {
+            if (s.sep) ws_expand<KH == 3 ? 9 : 0, true>(p, smem, warp, lane, wsready_bar);
+            else ws_expand<KH == 3 ? 9 : 0, false>(p, smem, warp, lane, wsready_bar);
+        }
         if (lane == 0) {
             constexpr uint32_t IDESC = make_idesc(BM, 64, 0);
             const int me = warp - 1;
@@ -347,7 +357,8 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             }
         }
     } else {
-        ws_expand<KH == 3 ? 9 : 0>(p, smem, warp, lane, wsready_bar);
+        if (s.sep) ws_expand<KH == 3 ? 9 : 0, true>(p, smem, warp, lane, wsready_bar);
+        else ws_expand<KH == 3 ? 9 : 0, false>(p, smem, warp, lane, wsready_bar);
         // ------------------------------------------- epilogue (warps 4 .. 4 + 4 NI - 1)
         const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
         const long long M = s.M;

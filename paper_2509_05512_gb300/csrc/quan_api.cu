@@ -118,18 +118,21 @@ quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4]
     s->Ho = static_cast<int>(Ho); s->Wo = static_cast<int>(Wo);
     s->Qin = Cin / 4; s->Qout = Cout / 4;
     s->M = static_cast<long long>(N) * Ho * Wo;
+    s->sep = 0;
     return QUAN_OK;
 }
 
 quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void* wj,
                        const void* wk, const float* bias, const float* scale, const float* shift,
                        int N, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
-                       int act, const void* residual, void* out, quan_stream_t stream) {
+                       int act, const void* residual, void* out, quan_stream_t stream,
+                       bool separable = false) {
     const void* w[4] = {wr, wi, wj, wk};
     quan::ConvShape s;
     quan_status_t st = validate(&s, x, w, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
                                 stride, pad, act, residual, out, 2);
     if (st != QUAN_OK) return st;
+    s.sep = separable ? 1 : 0;
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
@@ -140,9 +143,9 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
     if (path == QUAN_PATH_TC) {
         if (!tc_ok)
             return fail(QUAN_ERR_UNSUPPORTED,
-                        "tensor-core path needs sm_103, Cin/4 and Cout/4 multiples of 16 (or "
-                        "Cin = 4, Cout = 64, stride 2, even W) and 16-byte aligned tensors "
-                        "(device cc %d, Cin=%d, Cout=%d)",
+                        "tensor-core path needs sm_103, Cin/4 and Cout/4 multiples of 16 (or, "
+                        "for the full form, Cin = 4, Cout = 64, stride 2, even W) and 16-byte "
+                        "aligned tensors (device cc %d, Cin=%d, Cout=%d)",
                         cc, Cin, Cout);
         use_tc = true;
     } else if (path == QUAN_PATH_SIMT) {
@@ -171,7 +174,7 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         e = quan::launch_qconv_simt_bf16(s, x, w, ep, out, cs);
         if (e != cudaSuccess) return cuda_fail(e, "qconv_simt launch");
         t_last_path = QUAN_PATH_SIMT;
-        t_last_kernel = "qconv_simt_kernel<bf16>";
+        t_last_kernel = s.sep ? "qconv_simt_kernel<bf16,sep>" : "qconv_simt_kernel<bf16>";
     }
     return QUAN_OK;
 }
@@ -197,6 +200,15 @@ quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi
     if (!residual) return fail(QUAN_ERR_INVALID_ARG, "residual is NULL");
     return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
                     stride, pad, act, residual, out, stream);
+}
+
+quan_status_t quan_qconv2d_sep_fwd(const void* x, const void* wr, const void* wi,
+                                   const void* wj, const void* wk, const float* bias,
+                                   const float* iqbn_scale, const float* iqbn_shift, int N, int H,
+                                   int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                   int act, void* out, quan_stream_t stream) {
+    return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                    stride, pad, act, nullptr, out, stream, true);
 }
 
 quan_status_t quan_qconv2d_fwd_f32(const float* x, const float* wr, const float* wi,

@@ -44,6 +44,23 @@ constexpr uint32_t letter_sign_table() {
 }
 constexpr uint32_t LETTER_SIGNS = letter_sign_table();
 
+// The separable form of Eq. 7: output component m = sum over p of sign * (W_p conv x_p),
+// bit (4 m + p) of SEP_NEG marking the negative terms,
+//   y_r = +r -i -j -k,  y_i = +r +i +j -k,  y_j = +r -i +j +k,  y_k = +r +i -j +k.
+// As a block weight it is row block m, column block p = sign * W_p; SEP_LETTER_SIGNS holds
+// letter p's signs down its column, bit (4 p + m).
+constexpr uint32_t SEP_NEG = (1u << 1) | (1u << 2) | (1u << 3)  // y_r: -i -j -k
+                             | (1u << 7)                        // y_i: -k
+                             | (1u << 9)                        // y_j: -i
+                             | (1u << 14);                      // y_k: -j
+constexpr uint32_t sep_letter_sign_table() {
+    uint32_t t = 0;
+    for (int p = 0; p < 4; ++p)
+        for (int m = 0; m < 4; ++m) t |= ((SEP_NEG >> (4 * m + p)) & 1u) << (4 * p + m);
+    return t;
+}
+constexpr uint32_t SEP_LETTER_SIGNS = sep_letter_sign_table();
+
 // tcgen05 shared-memory matrix descriptors (K-major, swizzled operand tiles) are built
 // as two 32-bit words: the low word holds the start address >> 4 (bits 0-13) and the
 // leading byte offset (bits 16-29, unused for these layouts, set to 1); the high word
@@ -397,6 +414,109 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
                                  make_uint4(w[0], w[1], w[2], w[3]));
             }
             if (b + 1 < NB) tmem_ld_wait();
+        }
+    }
+}
+
+// Epilogue of the separable form (Eq. 7, MODE_SEP of the QUAD/PAIR kernel).  The
+// accumulator holds the four per-component convolutions D_p = W_p (*) X_p (component p at
+// TMEM column offset p BNQ); output component m is the signed sum
+//   y_r = D_r - D_i - D_j - D_k,  y_i = D_r + D_i + D_j - D_k,
+//   y_j = D_r - D_i + D_j + D_k,  y_k = D_r + D_i - D_j + D_k,
+// followed by the same act(scale * (y + bias) + shift).  Warps 4..7 take the first half of
+// the tile's BNQ channels, warps 8..11 the second; every warp loads the four D_p of its 32
+// rows for SS = min(BNQ / 2, 16) channels at a time, mixes them in registers and writes
+// the four output components (a 2x2 chunk transpose across lane pairs when SS = 16, so a
+// store instruction covers 32-byte pieces of 16 rows).  No shared memory; the per-channel
+// vectors through L1.
+template <int BNQ, typename Geo>
+__device__ __forceinline__ void epilogue_direct_sep(const ConvShape& s, const EpilogueArgs& ep,
+                                                    void* y, uint32_t tmem_base,
+                                                    uint32_t accf0, uint32_t acce0,
+                                                    int num_tiles, uint64_t limit,
+                                                    volatile int* abort_flag, Geo geo) {
+    constexpr int CS = BNQ / 2;             // channels per half (per warp group)
+    constexpr int SS = CS < 16 ? CS : 16;   // channels per TMEM load
+    constexpr int NSUB = CS / SS;
+    constexpr int NCH = SS / 8;             // 8-channel chunks per load: 1 or 2
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int quad = warp & 3;
+    const int half = (warp - EPI_WARP0) >> 2;
+    const int ci = lane % NCH;
+    const int row0 = quad * 32 + NCH * (lane / NCH);
+    const long long Cout = s.Cout;
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(y);
+    int local = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+        const int buf = local & 1;
+        const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        bool ok = true;
+        if (lane == 0)
+            ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (named_bar_or(1, 256, !ok)) break;
+        tc_fence_after();
+        const EpiTile g = geo(tile);
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                               static_cast<uint32_t>(buf * 4 * BNQ);
+#pragma unroll
+        for (int sub = 0; sub < NSUB; ++sub) {
+            const int col0 = half * CS + sub * SS;  // column within a component block
+            uint32_t d[4][SS];
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+                if constexpr (SS == 16)
+                    tmem_ld_32x32b_x16(taddr + p * BNQ + col0, d[p]);
+                else
+                    tmem_ld_32x32b_x8(taddr + p * BNQ + col0, d[p]);
+            }
+            tmem_ld_wait();
+            if (sub == NSUB - 1) {
+                // the tile's accumulator is in registers: hand the buffer back
+                tc_fence_before();
+                mbar_arrive(acce0 + 8u * buf);
+            }
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                float E[NCH][8];  // E[j][e]: channel col0 + 8 j + e of this lane's row
+#pragma unroll
+                for (int j = 0; j < NCH; ++j)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        float z = 0.0f;
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) {
+                            const float dp = __uint_as_float(d[p][8 * j + e]);
+                            z = ((SEP_NEG >> (4 * m + p)) & 1u) ? z - dp : z + dp;
+                        }
+                        E[j][e] = z;
+                    }
+                if constexpr (NCH == 2) chunk_transpose_stage<1, 2>(E, ci);
+                // now E[k][e] = channel cb + e of row row0 + k
+                const int cb = m * s.Qout + g.n_tile * BNQ + col0 + 8 * ci;
+                float sc[8], sh[8];
+                {
+                    float bi[8];
+                    load8(ep.scale, cb, 1.0f, sc);
+                    load8(ep.shift, cb, 0.0f, sh);
+                    load8(ep.bias, cb, 0.0f, bi);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) sh[e] = fmaf(sc[e], bi[e], sh[e]);
+                }
+#pragma unroll
+                for (int k = 0; k < NCH; ++k) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const float z0 = fmaf(sc[2 * t], E[k][2 * t], sh[2 * t]);
+                        const float z1 = fmaf(sc[2 * t + 1], E[k][2 * t + 1], sh[2 * t + 1]);
+                        w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                    }
+                    if (row0 + k < g.rows)
+                        st_global_na(out + (g.m0 + row0 + k) * Cout + cb,
+                                     make_uint4(w[0], w[1], w[2], w[3]));
+                }
+            }
         }
     }
 }

@@ -61,6 +61,7 @@ def load():
         lib.quan_qconv2d_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_qconv2d_fwd_f32.argtypes = _conv_args + [_vp, _vp]
         lib.quan_qconv2d_fwd_res.argtypes = _conv_args + [_vp, _vp, _vp]
+        lib.quan_qconv2d_sep_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
         lib.quan_set_path.argtypes = [_i]
         lib.quan_last_path.argtypes = []
@@ -78,6 +79,7 @@ def load():
         lib.quan_last_error_message.restype = ctypes.c_char_p
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
+                     "quan_qconv2d_sep_fwd",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
                      "quan_set_tc_halo", "quan_set_tc_issuers"):
@@ -188,6 +190,14 @@ def quan_version() -> int:
     return load().quan_version()
 
 
+def quan_qconv2d_sep_fwd(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                         kw, stride, pad, act, out, stream=None) -> None:
+    _check(load().quan_qconv2d_sep_fwd(_ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk),
+                                       _ptr(bias), _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W,
+                                       Cin, Cout, kh, kw, stride, pad, act, _ptr(out),
+                                       _stream(stream)))
+
+
 # ------------------------------------------------------------------ tensor helpers
 
 def out_size(n: int, k: int, stride: int, pad: int) -> int:
@@ -195,9 +205,10 @@ def out_size(n: int, k: int, stride: int, pad: int) -> int:
 
 
 def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=None,
-            act=QUAN_ACT_NONE, residual=None, out=None, stream=None):
+            act=QUAN_ACT_NONE, residual=None, out=None, stream=None, separable=False):
     """Allocate the output (torch, same dtype/device as x) and run the convolution.
-    x: [N, H, W, Cin] (bf16 or fp32, CUDA); w*: [Cout/4, kh, kw, Cin/4]."""
+    x: [N, H, W, Cin] (bf16 or fp32, CUDA); w*: [Cout/4, kh, kw, Cin/4].  separable=True
+    runs the separable form of Eq. 7 (bf16 only, no residual)."""
     import torch
     N, H, W, Cin = x.shape
     Qout, kh, kw, _ = wr.shape
@@ -205,7 +216,12 @@ def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=
     Ho, Wo = out_size(H, kh, stride, pad), out_size(W, kw, stride, pad)
     if out is None:
         out = torch.empty((N, Ho, Wo, Cout), dtype=x.dtype, device=x.device)
-    if x.dtype == torch.float32:
+    if separable:
+        if x.dtype != torch.bfloat16 or residual is not None:
+            raise ValueError("the separable form takes bf16 tensors and no residual")
+        quan_qconv2d_sep_fwd(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                             stride, pad, act, out, stream)
+    elif x.dtype == torch.float32:
         if residual is not None:
             raise ValueError("the fp32 entry point has no residual input")
         quan_qconv2d_fwd_f32(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
