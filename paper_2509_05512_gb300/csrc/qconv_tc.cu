@@ -654,14 +654,27 @@ int grid_for(const TcOptions& opt, int num_sms, int num_tiles) {
     return grid < 1 ? 1 : grid;
 }
 
-template <bool HALO, int KH, int NI>
+template <bool HALO, int KH, int NI, bool SEP>
 cudaError_t launch_ws_kernel(const CUtensorMap& map, const WsParams& prm, int grid,
                              cudaStream_t stream) {
-    auto kern = qconv_ws_kernel<HALO, KH, NI>;
+    auto kern = qconv_ws_kernel<HALO, KH, NI, SEP>;
     static std::atomic<unsigned long long> attr_done{0};
     cudaError_t e = set_smem_once(kern, WsCfg::SMEM_BYTES, attr_done);
     if (e != cudaSuccess) return e;
     return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), WsCfg::SMEM_BYTES, stream, map, prm);
+}
+
+template <bool SEP>
+cudaError_t launch_ws_form(const CUtensorMap& map, const WsParams& prm, int grid, bool halo,
+                           bool k3x3, int ni, cudaStream_t stream) {
+    if (ni == 2) {
+        if (halo && k3x3) return launch_ws_kernel<true, 3, 2, SEP>(map, prm, grid, stream);
+        if (halo) return launch_ws_kernel<true, 0, 2, SEP>(map, prm, grid, stream);
+        return launch_ws_kernel<false, 0, 2, SEP>(map, prm, grid, stream);
+    }
+    if (halo && k3x3) return launch_ws_kernel<true, 3, ISSUERS, SEP>(map, prm, grid, stream);
+    if (halo) return launch_ws_kernel<true, 0, ISSUERS, SEP>(map, prm, grid, stream);
+    return launch_ws_kernel<false, 0, ISSUERS, SEP>(map, prm, grid, stream);
 }
 
 cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
@@ -731,14 +744,8 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
                              : "qconv_ws_kernel<im2col,issuers=%d>",
                         ni);
     const bool k3x3 = s.kh == 3 && s.kw == 3;
-    if (ni == 2) {
-        if (halo && k3x3) return launch_ws_kernel<true, 3, 2>(maps[0], prm, grid, stream);
-        if (halo) return launch_ws_kernel<true, 0, 2>(maps[0], prm, grid, stream);
-        return launch_ws_kernel<false, 0, 2>(maps[0], prm, grid, stream);
-    }
-    if (halo && k3x3) return launch_ws_kernel<true, 3, ISSUERS>(maps[0], prm, grid, stream);
-    if (halo) return launch_ws_kernel<true, 0, ISSUERS>(maps[0], prm, grid, stream);
-    return launch_ws_kernel<false, 0, ISSUERS>(maps[0], prm, grid, stream);
+    return s.sep ? launch_ws_form<true>(maps[0], prm, grid, halo, k3x3, ni, stream)
+                 : launch_ws_form<false>(maps[0], prm, grid, halo, k3x3, ni, stream);
 }
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],

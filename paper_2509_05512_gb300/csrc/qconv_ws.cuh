@@ -147,8 +147,8 @@ __device__ __forceinline__ void ws_expand(const WsParams& p, uint8_t* smem, int 
 
 // KH = 3: a 3x3 filter with halo staging, known at compile time, so the MMA issue loop is
 // fully unrolled and the expansion's tap count is a constant; 0 = from the shape at run
-// time.  NI: MMA issuers (2 or 3).
-template <bool HALO, int KH, int NI>
+// time.  NI: MMA issuers (2 or 3).  SEP: the separable block weight of Eq. 7.
+template <bool HALO, int KH, int NI, bool SEP>
 __global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_ws_kernel(const __grid_constant__ CUtensorMap tmap_x, const WsParams p) {
     using C = WsCfg;
@@ -268,10 +268,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
         }
     } else if (warp <= NI) {
         // ------------------------------------------------------------ MMA issuers
-        if (warp >= 2) {
-            if (s.sep) ws_expand<KH == 3 ? 9 : 0, true>(p, smem, warp, lane, wsready_bar);
-            else ws_expand<KH == 3 ? 9 : 0, false>(p, smem, warp, lane, wsready_bar);
-        }
+        if (warp >= 2) ws_expand<KH == 3 ? 9 : 0, SEP>(p, smem, warp, lane, wsready_bar);
         if (lane == 0) {
             constexpr uint32_t IDESC = make_idesc(BM, 64, 0);
             const int me = warp - 1;
@@ -357,8 +354,7 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
             }
         }
     } else {
-        if (s.sep) ws_expand<KH == 3 ? 9 : 0, true>(p, smem, warp, lane, wsready_bar);
-        else ws_expand<KH == 3 ? 9 : 0, false>(p, smem, warp, lane, wsready_bar);
+        ws_expand<KH == 3 ? 9 : 0, SEP>(p, smem, warp, lane, wsready_bar);
         // ------------------------------------------- epilogue (warps 4 .. 4 + 4 NI - 1)
         const int tpi = p.tpi, R = p.R, Ho = s.Ho, Wo = s.Wo;
         const long long M = s.M;
