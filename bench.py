@@ -41,7 +41,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c1",
-                    choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone"])
+                    choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone", "poincare"])
     ap.add_argument("--variant", choices=["full", "separable"], default="full",
                     help="layer workloads: the full Hamilton form (Eq. 5/6) or the separable "
                          "form of Eq. 7 (a quarter of the multiply-adds)")
@@ -321,11 +321,84 @@ WORKLOAD_DESC = {
     "c3a": "detection-neck pointwise layer",
     "c3b": "detection-neck 3x3 layer",
     "backbone": "ResNet-18-style QUAN backbone",
+    "poincare": "Poincare RGB -> quaternion input mapping (Eq. 4)",
 }
+
+POINCARE_SHAPE = (256, 224, 224)  # the backbone's input batch: N, H, W
+
+
+class PoincareRunner:
+    """The Eq. 4 input mapping of an image batch, fp32 RGB -> bf16 quaternion pixels, on
+    rotating buffer sets larger than L2."""
+
+    def __init__(self, torch, quan, N, H, W):
+        import numpy as np
+        self.torch, self.quan, self.N = torch, quan, N
+        self.npix = N * H * W
+        rng = np.random.default_rng(44)
+        self.host_rgb = rng.uniform(0.0, 1.0, size=(N, H, W, 3)).astype(np.float32)
+        rgb0 = torch.from_numpy(self.host_rgb).cuda()
+        per_set = self.npix * 20
+        self.sets = max(2, min(8, math.ceil(2 * L2_BYTES / per_set)))
+        self.rgb = [rgb0] + [rgb0.clone() for _ in range(self.sets - 1)]
+        self.out = [torch.empty((N, H, W, 4), dtype=torch.bfloat16, device="cuda")
+                    for _ in range(self.sets)]
+        self.i = 0
+        self.launches_per_step = 1
+        self.footprint = per_set * self.sets
+        self.flops = 0.0
+        self.algorithmic_bytes = float(per_set)  # 12 bytes read, 8 written per pixel
+        self.separable = False
+
+    def step(self, stream):
+        k = self.i % self.sets
+        self.i += 1
+        self.quan.quan_poincare_fwd(self.rgb[k], self.npix, self.out[k], stream)
+
+    def e2e_setup(self):
+        torch = self.torch
+        self.h_in = torch.from_numpy(self.host_rgb.reshape(-1)).pin_memory()
+        self.h_out = [torch.empty(self.npix * 4, dtype=torch.bfloat16).pin_memory()
+                      for _ in range(E2E_BUFFERS)]
+        self.e_in = [torch.empty_like(self.h_in, device="cuda") for _ in range(E2E_BUFFERS)]
+        self.e_out = [torch.empty_like(t, device="cuda") for t in self.h_out]
+        self.h2d = self.npix * 12
+        self.d2h = self.npix * 8
+
+    def e2e_in(self, b):
+        return [(self.e_in[b], self.h_in)]
+
+    def e2e_out(self, b):
+        return [(self.h_out[b], self.e_out[b])]
+
+    def e2e_compute(self, b, stream):
+        self.quan.quan_poincare_fwd(self.e_in[b], self.npix, self.e_out[b], stream)
+
+
+def poincare_cpu_sample(runner, seconds):
+    """Time the fp64 oracle mapping on a bounded number of images of the batch."""
+    import numpy as np
+    import oracle
+    img = runner.host_rgb[0].astype(np.float64)
+    t0 = time.perf_counter()
+    oracle.poincare(img)
+    t1 = max(time.perf_counter() - t0, 1e-6)
+    n = max(1, min(runner.N, int(seconds / t1)))
+    t0 = time.perf_counter()
+    for i in range(n):
+        oracle.poincare(runner.host_rgb[i].astype(np.float64))
+    t = time.perf_counter() - t0
+    return {"value": n / t, "unit": "images/s", "cores": 1, "kind": "oracle",
+            "sample": "%d of %d images of the batch (fp64, %.2f s)" % (n, runner.N, t)}
 
 
 def workload_config(workload: str, inputs, variant: str = "full") -> dict:
     """The workload part of the JSON line's config, shared by both arms."""
+    if workload == "poincare":
+        N, H, W = POINCARE_SHAPE
+        return {"workload": "%s, N=%d, %dx%d fp32 RGB -> bf16 quaternion pixels" % (
+                    WORKLOAD_DESC[workload], N, H, W), "N": N, "H": H, "W": W,
+                "bytes_per_step": N * H * W * 20}
     if workload == "backbone":
         layers = inputs.backbone_layers()
         convs = [L.spec for L in layers if L.kind == "conv"]
@@ -387,9 +460,12 @@ def main():
 
     if args.batch and not args.profile:
         raise SystemExit("--batch is for --profile runs only")
-    if args.workload == "backbone":
-        if args.variant != "full":
-            raise SystemExit("--variant applies to the single-layer workloads")
+    if args.workload in ("backbone", "poincare") and args.variant != "full":
+        raise SystemExit("--variant applies to the convolution layer workloads")
+    if args.workload == "poincare":
+        runner = PoincareRunner(torch, quan, *POINCARE_SHAPE)
+        unit, per_step_units, dtype = "images/s", runner.N, "f32->bf16"
+    elif args.workload == "backbone":
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256)
         runner.sets = 1
@@ -425,7 +501,8 @@ def main():
         if n % 64 == 0:
             torch.cuda.synchronize()
     torch.cuda.synchronize()
-    kernel_name = quan.quan_last_kernel() if args.workload != "backbone" else None
+    kernel_name = (None if args.workload == "backbone" else
+                   "poincare_kernel" if args.workload == "poincare" else quan.quan_last_kernel())
 
     # The timed region is exactly K steps.  By default they are captured once into a CUDA
     # graph (same launches, same buffers) so host launch overhead does not leave gaps.
@@ -489,6 +566,8 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         if args.workload == "backbone":
             cpu = backbone_cpu_sample(runner, args.cpu_seconds, inputs)
+        elif args.workload == "poincare":
+            cpu = poincare_cpu_sample(runner, args.cpu_seconds)
         else:
             cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs,
                                     separable=runner.separable)
@@ -503,7 +582,7 @@ def main():
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
                 "timing": "one CUDA-graph replay of the K steps" if graph is not None
                 else "plain launch loop"})
-    if args.workload != "backbone":
+    if args.workload not in ("backbone", "poincare"):
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     line = {"metric": METRIC, "value": round(value, 4), "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
@@ -605,6 +684,29 @@ def reference_arm(args, rank, world, inputs):
     import oracle
     ref_cfg = workload_config(args.workload, inputs, args.variant)
     ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
+    if args.workload == "poincare":
+        import numpy as np
+        N, H, W = POINCARE_SHAPE
+        img = np.random.default_rng(44).uniform(0.0, 1.0, size=(H, W, 3))
+        for _ in range(args.warmup):
+            oracle.poincare(img)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.poincare(img)
+        dt = time.perf_counter() - t0
+        value = args.steps / dt
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": ref_cfg,
+                "cpu_baseline": {"value": value, "unit": "images/s", "cores": 1,
+                                 "kind": "oracle",
+                                 "sample": "1 of %d images of the batch per step (fp64)" % N},
+                "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
     if args.workload == "backbone":
         import oracle.backbone as ob
         layers = inputs.backbone_layers(N=1)

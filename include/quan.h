@@ -124,6 +124,20 @@ quan_status_t quan_qconv2d_sep_fwd(const void* x, const void* wr, const void* wi
                                    int act, void* out, quan_stream_t stream);
 
 /*
+ * Poincare mapping of RGB pixels onto the unit quaternion sphere (Eq. 4, Sec. III-A), the
+ * input mapping in front of the quaternion stem:
+ *   n2 = r^2 + g^2 + b^2,   q = ((1 - n2), 2 r, 2 g, 2 b) / (1 + n2),
+ * computed in fp32 and rounded to bf16 (nearest even).
+ *   rgb   fp32 [npix][3] (device; e.g. NHWC with C = 3, npix = N H W), 4-byte aligned
+ *   out   bf16 [npix][4] (device): channels [r|i|j|k] of one quaternion channel, the
+ *         layout quan_qconv2d_fwd reads for Cin = 4; must not overlap rgb
+ * npix = 0 is a no-op; npix < 0, a NULL pointer or a misaligned pointer returns
+ * QUAN_ERR_INVALID_ARG.
+ */
+quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
+                                quan_stream_t stream);
+
+/*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,
  * QSPPF), bf16 NHWC [N][H][W][C] -> [N][Ho][Wo][C], window k x k, stride, zero-size
  * padding that never wins.  C is any positive count.

@@ -80,6 +80,10 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// Poincare RGB -> quaternion mapping (Eq. 4): fp32 [npix][3] -> bf16 [npix][4].
+cudaError_t launch_poincare(const float* rgb, long long npix, void* out, int num_sms,
+                            cudaStream_t stream);
+
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream);

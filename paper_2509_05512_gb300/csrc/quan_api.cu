@@ -232,6 +232,24 @@ quan_status_t quan_qconv2d_fwd_f32(const float* x, const float* wr, const float*
     return QUAN_OK;
 }
 
+quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
+                                quan_stream_t stream) {
+    if (npix < 0) return fail(QUAN_ERR_INVALID_ARG, "npix must be >= 0");
+    if (npix == 0) return QUAN_OK;
+    if (!rgb || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if (npix > (1LL << 40)) return fail(QUAN_ERR_UNSUPPORTED, "tensor too large");
+    if (reinterpret_cast<uintptr_t>(rgb) % 4 != 0 || reinterpret_cast<uintptr_t>(out) % 2 != 0)
+        return fail(QUAN_ERR_INVALID_ARG, "rgb must be 4-byte and out 2-byte aligned");
+    if (overlaps(rgb, static_cast<size_t>(npix) * 12, out, static_cast<size_t>(npix) * 8))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps rgb");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    e = quan::launch_poincare(rgb, npix, out, num_sms, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "poincare launch");
+    return QUAN_OK;
+}
+
 quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,
                                  int pad, void* out, quan_stream_t stream) {
     if (!x || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");

@@ -63,6 +63,7 @@ def load():
         lib.quan_qconv2d_fwd_res.argtypes = _conv_args + [_vp, _vp, _vp]
         lib.quan_qconv2d_sep_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
+        lib.quan_poincare_fwd.argtypes = [_vp, ctypes.c_longlong, _vp, _vp]
         lib.quan_set_path.argtypes = [_i]
         lib.quan_last_path.argtypes = []
         lib.quan_last_kernel.argtypes = []
@@ -79,7 +80,7 @@ def load():
         lib.quan_last_error_message.restype = ctypes.c_char_p
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
-                     "quan_qconv2d_sep_fwd",
+                     "quan_qconv2d_sep_fwd", "quan_poincare_fwd",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
                      "quan_set_tc_halo", "quan_set_tc_issuers"):
@@ -232,6 +233,21 @@ def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=
     else:
         quan_qconv2d_fwd(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
                          stride, pad, act, out, stream)
+    return out
+
+
+def quan_poincare_fwd(rgb, npix, out, stream=None) -> None:
+    _check(load().quan_poincare_fwd(_ptr(rgb), npix, _ptr(out), _stream(stream)))
+
+
+def poincare(rgb, *, out=None, stream=None):
+    """Eq. 4 on the GPU: fp32 rgb [..., 3] (CUDA) -> bf16 quaternion pixels [..., 4]."""
+    import torch
+    if rgb.dtype != torch.float32 or rgb.shape[-1] != 3:
+        raise ValueError("rgb must be float32 with a last dimension of 3")
+    if out is None:
+        out = torch.empty(rgb.shape[:-1] + (4,), dtype=torch.bfloat16, device=rgb.device)
+    quan_poincare_fwd(rgb, rgb.numel() // 3, out, stream)
     return out
 
 

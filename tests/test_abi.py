@@ -62,6 +62,11 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_set_tc_tiles(0, 0, 0, 5) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_tiles(0, 0, 0, 4) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 0) == quan.QUAN_OK
+    assert lib.quan_poincare_fwd(None, 4, FAKE, None) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_poincare_fwd(FAKE, -1, FAKE * 64, None) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_poincare_fwd(FAKE + 1, 4, FAKE * 64, None) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_poincare_fwd(FAKE, 4, FAKE + 8, None) == quan.QUAN_ERR_INVALID_ARG  # overlap
+    assert lib.quan_poincare_fwd(None, 0, None, None) == quan.QUAN_OK
     assert lib.quan_set_tc_issuers(1) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_issuers(4) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_issuers(2) == quan.QUAN_OK
