@@ -308,6 +308,102 @@ int oracle_maxpool2d(const double *x, int N, int H, int W, int C, int k, int str
     return 0;
 }
 
+/* ---------------------------------------------------------------- backward pass
+ * Gradients of the convolution of Eq. 5 before its epilogue, y = sum over taps and input
+ * quaternion channels of W (x) X, given dy = dL/dy (same layout as y).  Both are written
+ * from the Jacobians of the Hamilton product (Eq. 3) taken literally:
+ *   d(W (x) X)_q / dX_p = (W (x) e_p)_q,    d(W (x) X)_q / dW_L = (e_L (x) X)_q,
+ * e_m the quaternion basis element m, each evaluated with oracle_qmul. */
+static const double BASIS[4][4] = {{1, 0, 0, 0}, {0, 1, 0, 0}, {0, 0, 1, 0}, {0, 0, 0, 1}};
+
+/* dx [N][H][W][C_in]: every output pixel and tap that reads input pixel (h, w) adds
+ * sum_q (W (x) e_p)_q dy_q to dx_p.  Returns 0, or -1 on invalid arguments. */
+int oracle_qconv2d_bwd_data(const double *dy, const double *wr, const double *wi,
+                            const double *wj, const double *wk, int N, int H, int W, int Cin,
+                            int Cout, int kh, int kw, int stride, int pad, double *dx) {
+    qconv_args a = {dy, wr, wi, wj, wk, NULL, NULL, NULL, NULL,
+                    N, H, W, Cin, Cout, kh, kw, stride, pad, ACT_NONE, 0, 0};
+    if (stride <= 0 || !dx) return -1;
+    a.Ho = out_dim(H, kh, stride, pad);
+    a.Wo = out_dim(W, kw, stride, pad);
+    if (check_args(&a)) return -1;
+    const int Qin = Cin / 4, Qout = Cout / 4;
+    memset(dx, 0, sizeof(double) * (size_t)N * H * W * Cin);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int n = 0; n < N; ++n) {          /* one image per thread: no shared dx entry */
+        for (int ho = 0; ho < a.Ho; ++ho)
+            for (int wo = 0; wo < a.Wo; ++wo) {
+                const double *g = dy + (((size_t)n * a.Ho + ho) * a.Wo + wo) * Cout;
+                for (int dh = 0; dh < kh; ++dh) {
+                    const int h = ho * stride - pad + dh;
+                    if (h < 0 || h >= H) continue;
+                    for (int dw = 0; dw < kw; ++dw) {
+                        const int w = wo * stride - pad + dw;
+                        if (w < 0 || w >= W) continue;
+                        double *d = dx + (((size_t)n * H + h) * W + w) * Cin;
+                        for (int co = 0; co < Qout; ++co)
+                            for (int ci = 0; ci < Qin; ++ci) {
+                                const size_t widx = (((size_t)co * kh + dh) * kw + dw) * Qin + ci;
+                                const double wq[4] = {wr[widx], wi[widx], wj[widx], wk[widx]};
+                                for (int p = 0; p < 4; ++p) {
+                                    double col[4];
+                                    oracle_qmul(wq, BASIS[p], col);
+                                    for (int q = 0; q < 4; ++q)
+                                        d[p * Qin + ci] += col[q] * g[q * Qout + co];
+                                }
+                            }
+                    }
+                }
+            }
+    }
+    return 0;
+}
+
+/* dW_L [Q_out][kh][kw][Q_in] for L = r, i, j, k: the sum over output pixels of
+ * sum_q (e_L (x) X)_q dy_q, X the input quaternion the tap reads.  Returns 0 or -1. */
+int oracle_qconv2d_bwd_weight(const double *x, const double *dy, int N, int H, int W, int Cin,
+                              int Cout, int kh, int kw, int stride, int pad, double *dwr,
+                              double *dwi, double *dwj, double *dwk) {
+    const double dummy = 0.0;
+    qconv_args a = {x, &dummy, &dummy, &dummy, &dummy, NULL, NULL, NULL, NULL,
+                    N, H, W, Cin, Cout, kh, kw, stride, pad, ACT_NONE, 0, 0};
+    if (stride <= 0 || !dy || !dwr || !dwi || !dwj || !dwk) return -1;
+    a.Ho = out_dim(H, kh, stride, pad);
+    a.Wo = out_dim(W, kw, stride, pad);
+    if (check_args(&a)) return -1;
+    const int Qin = Cin / 4, Qout = Cout / 4;
+    double *dwl[4] = {dwr, dwi, dwj, dwk};
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int co = 0; co < Qout; ++co)       /* one output channel per thread */
+        for (int dh = 0; dh < kh; ++dh)
+            for (int dw = 0; dw < kw; ++dw)
+                for (int ci = 0; ci < Qin; ++ci) {
+                    double acc[4] = {0, 0, 0, 0};
+                    for (int n = 0; n < N; ++n)
+                        for (int ho = 0; ho < a.Ho; ++ho) {
+                            const int h = ho * stride - pad + dh;
+                            if (h < 0 || h >= H) continue;
+                            for (int wo = 0; wo < a.Wo; ++wo) {
+                                const int w = wo * stride - pad + dw;
+                                if (w < 0 || w >= W) continue;
+                                const double *xp = x + (((size_t)n * H + h) * W + w) * Cin;
+                                const double *g =
+                                    dy + (((size_t)n * a.Ho + ho) * a.Wo + wo) * Cout;
+                                const double xq[4] = {xp[ci], xp[Qin + ci], xp[2 * Qin + ci],
+                                                      xp[3 * Qin + ci]};
+                                for (int L = 0; L < 4; ++L) {
+                                    double t[4];
+                                    oracle_qmul(BASIS[L], xq, t);
+                                    for (int q = 0; q < 4; ++q) acc[L] += t[q] * g[q * Qout + co];
+                                }
+                            }
+                        }
+                    const size_t widx = (((size_t)co * kh + dh) * kw + dw) * Qin + ci;
+                    for (int L = 0; L < 4; ++L) dwl[L][widx] = acc[L];
+                }
+    return 0;
+}
+
 /* Poincare mapping of Eq. 4 (Sec. III-A): rgb [npix][3] -> q [npix][4] as
  * (q_r, q_i, q_j, q_k) = ((1 - n^2), 2r, 2g, 2b) / (1 + n^2), n^2 = r^2 + g^2 + b^2. */
 void oracle_poincare(const double *rgb, long long npix, double *q) {

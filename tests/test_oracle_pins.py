@@ -260,3 +260,72 @@ def test_separable_eq7_against_eq9_mixing_matrix():
         base = _torch_conv(_comp(x, p, Cin // 4), w[p], 1, 1)
         for q in range(4):
             np.testing.assert_allclose(_comp(y, q, Cout // 4), M[p, q] * base, atol=1e-12)
+
+
+# ----------------------------------------------------------------- backward pass
+# The convolution before its epilogue is linear in x and in each letter, so its gradients
+# are the adjoints of the forward map: <dy, F(x, W)> = <dx(dy), x> = sum_L <dW_L(x, dy), W_L>
+# exactly (up to fp64 rounding).  The forward oracle is pinned above.
+
+BWD_CASES = [
+    # N, H, W, Cin, Cout, kh, kw, stride, pad
+    (2, 6, 7, 8, 12, 3, 3, 1, 1),
+    (1, 9, 8, 4, 8, 3, 3, 2, 1),
+    (2, 7, 7, 8, 4, 5, 3, 2, 2),
+    (1, 5, 6, 12, 8, 1, 1, 1, 0),
+    (1, 8, 9, 4, 4, 7, 7, 2, 3),
+]
+
+
+@pytest.mark.parametrize("case", BWD_CASES)
+def test_backward_is_the_adjoint_of_the_forward(case):
+    N, H, W, Cin, Cout, kh, kw, s, p = case
+    rng = np.random.default_rng(sum(case))
+    x, w = _rand_layer(rng, N, H, W, Cin, Cout, kh, kw)
+    y = oracle.qconv2d(x, *w, stride=s, pad=p)
+    dy = rng.standard_normal(y.shape)
+    lhs = float(np.sum(dy * y))
+    dx = oracle.qconv2d_bwd_data(dy, *w, H=H, W=W, stride=s, pad=p)
+    dw = oracle.qconv2d_bwd_weight(x, dy, kh=kh, kw=kw, stride=s, pad=p)
+    assert dx.shape == x.shape and all(g.shape == t.shape for g, t in zip(dw, w))
+    np.testing.assert_allclose(float(np.sum(dx * x)), lhs, rtol=1e-11)
+    np.testing.assert_allclose(sum(float(np.sum(g * t)) for g, t in zip(dw, w)), lhs,
+                               rtol=1e-11)
+
+
+def test_backward_finite_differences():
+    # one perturbed entry at a time: the forward map is linear, so the difference quotient
+    # is the gradient entry up to rounding
+    rng = np.random.default_rng(31)
+    N, H, W, Cin, Cout, kh, kw, s, p = 1, 5, 5, 8, 8, 3, 3, 2, 1
+    x, w = _rand_layer(rng, N, H, W, Cin, Cout, kh, kw)
+    y0 = oracle.qconv2d(x, *w, stride=s, pad=p)
+    dy = rng.standard_normal(y0.shape)
+    dx = oracle.qconv2d_bwd_data(dy, *w, H=H, W=W, stride=s, pad=p)
+    dw = oracle.qconv2d_bwd_weight(x, dy, kh=kh, kw=kw, stride=s, pad=p)
+    eps = 0.5
+    for idx in [(0, 0, 0, 0), (0, 2, 3, 5), (0, 4, 4, 7), (0, 1, 2, 2)]:
+        xp = x.copy()
+        xp[idx] += eps
+        fd = np.sum(dy * (oracle.qconv2d(xp, *w, stride=s, pad=p) - y0)) / eps
+        np.testing.assert_allclose(fd, dx[idx], rtol=1e-10, atol=1e-12)
+    for L in range(4):
+        for idx in [(0, 0, 0, 0), (1, 2, 1, 1), (0, 1, 2, 1)]:
+            wp = [t.copy() for t in w]
+            wp[L][idx] += eps
+            fd = np.sum(dy * (oracle.qconv2d(x, *wp, stride=s, pad=p) - y0)) / eps
+            np.testing.assert_allclose(fd, dw[L][idx], rtol=1e-10, atol=1e-12)
+
+
+def test_backward_single_pixel_is_conjugate_multiplication():
+    # 1x1 kernel, one quaternion channel, one pixel: y = w (x) x, so the input gradient is
+    # conj(w) (x) dy and the weight gradient is dy (x) conj(x) (quaternion algebra)
+    rng = np.random.default_rng(32)
+    wq, xq, g = rng.standard_normal(4), rng.standard_normal(4), rng.standard_normal(4)
+    conj = lambda q: q * np.array([1.0, -1, -1, -1])
+    w = [np.full((1, 1, 1, 1), wq[m]) for m in range(4)]
+    dx = oracle.qconv2d_bwd_data(g.reshape(1, 1, 1, 4), *w, H=1, W=1)
+    np.testing.assert_allclose(dx.reshape(4), oracle.qmul(conj(wq), g), rtol=1e-14, atol=1e-15)
+    dw = oracle.qconv2d_bwd_weight(xq.reshape(1, 1, 1, 4), g.reshape(1, 1, 1, 4), kh=1, kw=1)
+    np.testing.assert_allclose(np.array([t.item() for t in dw]), oracle.qmul(g, conj(xq)),
+                               rtol=1e-14, atol=1e-15)
