@@ -1,7 +1,7 @@
 /*
- * quan.h -- libquan: quaternion convolution forward for NVIDIA GB300 (sm_103a).
+ * quan.h -- libquan: quaternion convolution for NVIDIA GB300 (sm_103a).
  *
- * Implements the forward pass of the QUAN quaternion convolution (Grant & Wang,
+ * Implements the QUAN quaternion convolution (Grant & Wang,
  * "Quaternion Approximate Networks for Enhanced Image Classification and Oriented
  * Object Detection", arXiv 2509.05512):
  *   - the full Hamilton-product convolution of Sec. III-B, Eq. 5, whose real
@@ -10,7 +10,10 @@
  *   - Independent Quaternion Batch Normalization in inference form (Sec. III-C,
  *     Eq. 11-12), folded by the caller into one scale and one shift per real channel;
  *   - a split (per real component) activation (ReLU or SiLU, Sec. IV-E ablation);
- *   - component-wise max pooling (the QSPPF pooling rule of Sec. III-D).
+ *   - component-wise max pooling (the QSPPF pooling rule of Sec. III-D);
+ *   - the Poincare RGB mapping of Eq. 4 (Sec. III-A);
+ *   - the separable form of Eq. 7 and its backward pass (Eq. 8-10), and the backward
+ *     pass of the full form (input and weight gradients before the epilogue).
  *
  * Conventions shared by every entry point
  *   Layout      x is NHWC [N][H][W][C_in]; the C_in real channels are four
@@ -36,6 +39,8 @@
  */
 #ifndef QUAN_H_
 #define QUAN_H_
+
+#include <stddef.h>
 
 #ifdef __cplusplus
 extern "C" {
@@ -136,6 +141,75 @@ quan_status_t quan_qconv2d_sep_fwd(const void* x, const void* wr, const void* wi
  */
 quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
                                 quan_stream_t stream);
+
+/*
+ * Backward pass of the convolution before its epilogue.  dy is dL/d(acc), the gradient of
+ * the convolution's accumulator (the caller applies the activation, IQBN scale and bias
+ * gradients first).  Layouts as in quan_qconv2d_fwd; dy is bf16 [N][Ho][Wo][Cout].
+ *
+ * Full form (Eq. 5): from the Jacobians of the Hamilton product (Eq. 3), per tap and
+ * channel pair, dL/dX = conj(W) (x) dy and dL/dW = dy (x) conj(X), with
+ * conj(q) = (q_r, -q_i, -q_j, -q_k).
+ * Separable form (Eq. 7): Eq. 8-10.  The output gradients are mixed by the matrix M of
+ * Eq. 9, g_p = sum_m M[p][m] dy_m (M transposed is Eq. 7's sign table), and then
+ * dL/dx_p is the transposed convolution of g_p with W_p and dL/dW_p the correlation of g_p
+ * with x_p, per component p.
+ */
+
+/*
+ * Bytes of device workspace quan_qconv2d_bwd_data and quan_qconv2d_sep_bwd_data need:
+ * the four transformed letter tensors, 4 * (Cin/4) * kh * kw * (Cout/4) bf16.  Returns 0
+ * for sizes that are not positive or channel counts that are not multiples of 4.
+ */
+size_t quan_qconv2d_bwd_data_workspace_size(int Cin, int Cout, int kh, int kw);
+
+/*
+ * Input gradient dx = dL/dx, bf16 [N][H][W][Cin] (device), rounded to nearest even from an
+ * fp32 accumulation.  N..pad are the FORWARD convolution's arguments.
+ *   workspace        device scratch of at least quan_qconv2d_bwd_data_workspace_size
+ *                    bytes, 16-byte aligned for the tensor-core path, owned by the caller;
+ *                    NULL or too small returns QUAN_ERR_INVALID_ARG.  Its contents are
+ *                    overwritten; concurrent calls need separate workspaces.
+ * dx must not overlap dy, the weights or the workspace.  For stride 1, a square filter,
+ * pad < kh and Cin/4, Cout/4 multiples of 16 on sm_103, the tensor-core path runs: one
+ * kernel writes conj(W) with its channel axes swapped and the filter rotated by 180
+ * degrees into the workspace, then the forward tensor-core kernel convolves dy with it
+ * (padding kh - 1 - pad).  Other shapes run a direct CUDA-core kernel.
+ * quan_set_path(QUAN_PATH_TC) makes a shape the tensor-core path cannot run fail with
+ * QUAN_ERR_UNSUPPORTED.
+ */
+quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* wi,
+                                    const void* wj, const void* wk, int N, int H, int W, int Cin,
+                                    int Cout, int kh, int kw, int stride, int pad,
+                                    void* workspace, size_t workspace_bytes, void* dx,
+                                    quan_stream_t stream);
+
+/* Separable form (Eq. 8-9) of the input gradient; same arguments.  Runs on CUDA cores
+ * (the workspace is checked but not used). */
+quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const void* wi,
+                                        const void* wj, const void* wk, int N, int H, int W,
+                                        int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                        void* workspace, size_t workspace_bytes, void* dx,
+                                        quan_stream_t stream);
+
+/*
+ * Weight gradients dwr..dwk = dL/dW_L, fp32 [Cout/4][kh][kw][Cin/4] each (device, 4-byte
+ * aligned, pairwise disjoint and disjoint from x and dy): zeroed on the stream, then
+ * accumulated over all N * Ho * Wo output pixels on CUDA cores (fp32 partial sums added
+ * with atomics, so the summation order, and the last bits, vary from run to run).
+ * x is the forward input, bf16 [N][H][W][Cin].  quan_set_path(QUAN_PATH_TC) returns
+ * QUAN_ERR_UNSUPPORTED.
+ */
+quan_status_t quan_qconv2d_bwd_weight(const void* x, const void* dy, int N, int H, int W,
+                                      int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                      float* dwr, float* dwi, float* dwj, float* dwk,
+                                      quan_stream_t stream);
+
+/* Separable form (Eq. 10) of the weight gradients; same arguments. */
+quan_status_t quan_qconv2d_sep_bwd_weight(const void* x, const void* dy, int N, int H, int W,
+                                          int Cin, int Cout, int kh, int kw, int stride,
+                                          int pad, float* dwr, float* dwi, float* dwj,
+                                          float* dwk, quan_stream_t stream);
 
 /*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,

@@ -17,7 +17,9 @@ Passages followed (Grant & Wang, arXiv 2509.05512):
   * separable variant ........... Eq. 7 (Sec. III-B)
   * backward pass ............... the input and weight gradients of Eq. 5 (the
                                   pre-epilogue convolution), from the Jacobians of
-                                  Eq. 3; Eq. 8-10 state the separable form's
+                                  Eq. 3
+  * separable backward .......... Eq. 8-10 (Sec. III-B): mixing matrix M of Eq. 9,
+                                  then per-component convolution gradients
   * IQBN, inference form ........ Eq. 11-12 (Sec. III-C), folded to scale/shift
   * component-wise pooling ...... QSPPF (Sec. III-D)
 """
@@ -80,6 +82,11 @@ def _load():
             lib.oracle_qconv2d_bwd_data.restype = ctypes.c_int
             lib.oracle_qconv2d_bwd_weight.argtypes = [_dp] * 2 + [ctypes.c_int] * 9 + [_dp] * 4
             lib.oracle_qconv2d_bwd_weight.restype = ctypes.c_int
+            lib.oracle_qconv2d_sep_bwd_data.argtypes = [_dp] * 5 + [ctypes.c_int] * 9 + [_dp]
+            lib.oracle_qconv2d_sep_bwd_data.restype = ctypes.c_int
+            lib.oracle_qconv2d_sep_bwd_weight.argtypes = ([_dp] * 2 + [ctypes.c_int] * 9 +
+                                                          [_dp] * 4)
+            lib.oracle_qconv2d_sep_bwd_weight.restype = ctypes.c_int
             lib.oracle_poincare.argtypes = [_dp, ctypes.c_longlong, _dp]
             lib.oracle_poincare.restype = None
             lib.oracle_num_threads.argtypes = []
@@ -254,6 +261,40 @@ def qconv2d_bwd_weight(x, dy, *, kh, kw, stride=1, pad=0):
                                            stride, pad, *(_ptr(t) for t in dw))
     if rc != 0:
         raise ValueError("oracle_qconv2d_bwd_weight: invalid arguments")
+    return tuple(dw)
+
+
+def qconv2d_sep_bwd_data(dy, wr, wi, wj, wk, *, H, W, stride=1, pad=0) -> np.ndarray:
+    """Input gradient of the separable convolution (Eq. 7) before its epilogue, by Eq. 8-9:
+    dy [N, Ho, Wo, C_out] -> dx [N, H, W, C_in]."""
+    dy, wr, wi, wj, wk = map(_f64, (dy, wr, wi, wj, wk))
+    N, Ho, Wo, Cout = dy.shape
+    Qout, kh, kw, Qin = wr.shape
+    Cin = 4 * Qin
+    if (out_size(H, kh, stride, pad), out_size(W, kw, stride, pad)) != (Ho, Wo):
+        raise ValueError("dy does not match the forward output size")
+    dx = np.zeros((N, H, W, Cin))
+    rc = _load().oracle_qconv2d_sep_bwd_data(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk),
+                                             N, H, W, Cin, Cout, kh, kw, stride, pad, _ptr(dx))
+    if rc != 0:
+        raise ValueError("oracle_qconv2d_sep_bwd_data: invalid arguments")
+    return dx
+
+
+def qconv2d_sep_bwd_weight(x, dy, *, kh, kw, stride=1, pad=0):
+    """Weight gradients of the separable convolution (Eq. 7) before its epilogue, by
+    Eq. 9-10: (dW_r, dW_i, dW_j, dW_k), each [C_out/4, kh, kw, C_in/4]."""
+    x, dy = map(_f64, (x, dy))
+    N, H, W, Cin = x.shape
+    Cout = dy.shape[-1]
+    if dy.shape[:3] != (N, out_size(H, kh, stride, pad), out_size(W, kw, stride, pad)):
+        raise ValueError("dy does not match the forward output size")
+    shape = (Cout // 4, kh, kw, Cin // 4)
+    dw = [np.zeros(shape) for _ in range(4)]
+    rc = _load().oracle_qconv2d_sep_bwd_weight(_ptr(x), _ptr(dy), N, H, W, Cin, Cout, kh, kw,
+                                               stride, pad, *(_ptr(t) for t in dw))
+    if rc != 0:
+        raise ValueError("oracle_qconv2d_sep_bwd_weight: invalid arguments")
     return tuple(dw)
 
 

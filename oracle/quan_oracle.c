@@ -404,6 +404,108 @@ int oracle_qconv2d_bwd_weight(const double *x, const double *dy, int N, int H, i
     return 0;
 }
 
+/* ---------------------------------------------------------------- separable backward
+ * Gradients of the separable convolution of Eq. 7 before its epilogue, by Eq. 8-10:
+ * the output gradients are mixed by the matrix M of Eq. 9,
+ *     [  1  1  1  1 ]
+ *     [ -1  1 -1  1 ]
+ *     [ -1  1  1 -1 ]
+ *     [ -1 -1  1  1 ],
+ * row p giving the weights of dy_r, dy_i, dy_j, dy_k for input component p, and each
+ * component p then takes the plain convolution gradients with its own letter W_p:
+ *     dx_p = sum_m M[p][m] (dy_m correlated back through W_p),
+ *     dW_p = sum_m M[p][m] (dy_m correlated with x_p).
+ * (Eq. 8 and 10 print the same letter q on the sum and inside it; this is the reading
+ * that makes them the gradient of Eq. 7, whose sign table is M transposed.) */
+static const double MIX_EQ9[4][4] = {
+    {+1, +1, +1, +1},
+    {-1, +1, -1, +1},
+    {-1, +1, +1, -1},
+    {-1, -1, +1, +1},
+};
+
+/* dx [N][H][W][C_in] of the separable form.  Returns 0, or -1 on invalid arguments. */
+int oracle_qconv2d_sep_bwd_data(const double *dy, const double *wr, const double *wi,
+                                const double *wj, const double *wk, int N, int H, int W,
+                                int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                double *dx) {
+    qconv_args a = {dy, wr, wi, wj, wk, NULL, NULL, NULL, NULL,
+                    N, H, W, Cin, Cout, kh, kw, stride, pad, ACT_NONE, 0, 0};
+    if (stride <= 0 || !dx) return -1;
+    a.Ho = out_dim(H, kh, stride, pad);
+    a.Wo = out_dim(W, kw, stride, pad);
+    if (check_args(&a)) return -1;
+    const int Qin = Cin / 4, Qout = Cout / 4;
+    const double *wl[4] = {wr, wi, wj, wk};
+    memset(dx, 0, sizeof(double) * (size_t)N * H * W * Cin);
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int n = 0; n < N; ++n) {          /* one image per thread: no shared dx entry */
+        for (int ho = 0; ho < a.Ho; ++ho)
+            for (int wo = 0; wo < a.Wo; ++wo) {
+                const double *g = dy + (((size_t)n * a.Ho + ho) * a.Wo + wo) * Cout;
+                for (int dh = 0; dh < kh; ++dh) {
+                    const int h = ho * stride - pad + dh;
+                    if (h < 0 || h >= H) continue;
+                    for (int dw = 0; dw < kw; ++dw) {
+                        const int w = wo * stride - pad + dw;
+                        if (w < 0 || w >= W) continue;
+                        double *d = dx + (((size_t)n * H + h) * W + w) * Cin;
+                        for (int co = 0; co < Qout; ++co)
+                            for (int ci = 0; ci < Qin; ++ci) {
+                                const size_t widx = (((size_t)co * kh + dh) * kw + dw) * Qin + ci;
+                                for (int p = 0; p < 4; ++p)
+                                    for (int m = 0; m < 4; ++m)
+                                        d[p * Qin + ci] +=
+                                            MIX_EQ9[p][m] * wl[p][widx] * g[m * Qout + co];
+                            }
+                    }
+                }
+            }
+    }
+    return 0;
+}
+
+/* dW_p [Q_out][kh][kw][Q_in] of the separable form.  Returns 0 or -1. */
+int oracle_qconv2d_sep_bwd_weight(const double *x, const double *dy, int N, int H, int W,
+                                  int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                  double *dwr, double *dwi, double *dwj, double *dwk) {
+    const double dummy = 0.0;
+    qconv_args a = {x, &dummy, &dummy, &dummy, &dummy, NULL, NULL, NULL, NULL,
+                    N, H, W, Cin, Cout, kh, kw, stride, pad, ACT_NONE, 0, 0};
+    if (stride <= 0 || !dy || !dwr || !dwi || !dwj || !dwk) return -1;
+    a.Ho = out_dim(H, kh, stride, pad);
+    a.Wo = out_dim(W, kw, stride, pad);
+    if (check_args(&a)) return -1;
+    const int Qin = Cin / 4, Qout = Cout / 4;
+    double *dwl[4] = {dwr, dwi, dwj, dwk};
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int co = 0; co < Qout; ++co)       /* one output channel per thread */
+        for (int dh = 0; dh < kh; ++dh)
+            for (int dw = 0; dw < kw; ++dw)
+                for (int ci = 0; ci < Qin; ++ci) {
+                    double acc[4] = {0, 0, 0, 0};
+                    for (int n = 0; n < N; ++n)
+                        for (int ho = 0; ho < a.Ho; ++ho) {
+                            const int h = ho * stride - pad + dh;
+                            if (h < 0 || h >= H) continue;
+                            for (int wo = 0; wo < a.Wo; ++wo) {
+                                const int w = wo * stride - pad + dw;
+                                if (w < 0 || w >= W) continue;
+                                const double *xp = x + (((size_t)n * H + h) * W + w) * Cin;
+                                const double *g =
+                                    dy + (((size_t)n * a.Ho + ho) * a.Wo + wo) * Cout;
+                                for (int p = 0; p < 4; ++p)
+                                    for (int m = 0; m < 4; ++m)
+                                        acc[p] += MIX_EQ9[p][m] * g[m * Qout + co] *
+                                                  xp[p * Qin + ci];
+                            }
+                        }
+                    const size_t widx = (((size_t)co * kh + dh) * kw + dw) * Qin + ci;
+                    for (int p = 0; p < 4; ++p) dwl[p][widx] = acc[p];
+                }
+    return 0;
+}
+
 /* Poincare mapping of Eq. 4 (Sec. III-A): rgb [npix][3] -> q [npix][4] as
  * (q_r, q_i, q_j, q_k) = ((1 - n^2), 2r, 2g, 2b) / (1 + n^2), n^2 = r^2 + g^2 + b^2. */
 void oracle_poincare(const double *rgb, long long npix, double *q) {

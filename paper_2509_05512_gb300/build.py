@@ -13,7 +13,8 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libquan.so")
-SOURCES = ["quan_api.cu", "qconv_tc.cu", "qconv_simt.cu", "maxpool.cu", "poincare.cu"]
+SOURCES = ["quan_api.cu", "qconv_tc.cu", "qconv_simt.cu", "qconv_bwd.cu", "maxpool.cu",
+           "poincare.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -84,6 +84,20 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
 cudaError_t launch_poincare(const float* rgb, long long npix, void* out, int num_sms,
                             cudaStream_t stream);
 
+// Backward of the pre-epilogue convolution (s.sep selects the separable form, Eq. 8-10).
+// Bytes of the transformed letters bwd_transform writes: 4 x [Qin][kh][kw][Qout] bf16.
+size_t bwd_data_workspace_bytes(int Cin, int Cout, int kh, int kw);
+// out_L[ci][kh-1-dh][kw-1-dw][co] = (L == r ? +1 : -1) * w_L[co][dh][dw][ci], the four
+// letters one after the other: the forward weights of the stride-1 input gradient.
+cudaError_t launch_bwd_transform(int Cin, int Cout, int kh, int kw, const void* const w[4],
+                                 void* out, int num_sms, cudaStream_t stream);
+// dx [N][H][W][Cin] from dy [N][Ho][Wo][Cout] on CUDA cores, any stride.
+cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void* const w[4],
+                                 void* dx, cudaStream_t stream);
+// dW_L fp32 [Qout][kh][kw][Qin] (zeroed, then accumulated) on CUDA cores.
+cudaError_t launch_bwd_weight_simt(const ConvShape& s, const void* x, const void* dy,
+                                   float* const dw[4], int num_sms, cudaStream_t stream);
+
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream);

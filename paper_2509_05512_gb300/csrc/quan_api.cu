@@ -76,12 +76,9 @@ bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
     return a0 < b0 + nb && b0 < a0 + na;
 }
 
-quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4],
-                       const float* bias, const float* scale, const float* shift, int N, int H,
-                       int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int act,
-                       const void* residual, const void* out, size_t esize) {
-    if (!x || !w[0] || !w[1] || !w[2] || !w[3] || !out)
-        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+// Checks the sizes of one convolution and fills *s (epilogue-free, full form).
+quan_status_t geometry(quan::ConvShape* s, int N, int H, int W, int Cin, int Cout, int kh,
+                       int kw, int stride, int pad) {
     if (N < 1 || H < 1 || W < 1 || Cin < 1 || Cout < 1 || kh < 1 || kw < 1 || stride < 1 ||
         pad < 0)
         return fail(QUAN_ERR_INVALID_ARG,
@@ -90,10 +87,6 @@ quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4]
                     N, H, W, Cin, Cout, kh, kw, stride, pad);
     if (Cin % 4 || Cout % 4)
         return fail(QUAN_ERR_INVALID_ARG, "Cin=%d and Cout=%d must be multiples of 4", Cin, Cout);
-    if ((scale == nullptr) != (shift == nullptr))
-        return fail(QUAN_ERR_INVALID_ARG, "iqbn_scale and iqbn_shift must both be given or both NULL");
-    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
-        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
     const long long Ho = (static_cast<long long>(H) + 2LL * pad - kh) / stride + 1;
     const long long Wo = (static_cast<long long>(W) + 2LL * pad - kw) / stride + 1;
     if (static_cast<long long>(H) + 2LL * pad < kh || static_cast<long long>(W) + 2LL * pad < kw ||
@@ -104,21 +97,46 @@ quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4]
     const long long yout = static_cast<long long>(N) * Ho * Wo * Cout;
     if (xin >= (1LL << 40) || yout >= (1LL << 40) || Ho > 0x7fffffff / Wo)
         return fail(QUAN_ERR_UNSUPPORTED, "tensor too large");
-    const size_t wbytes = static_cast<size_t>(Cout / 4) * kh * kw * (Cin / 4) * esize;
-    const size_t xbytes = static_cast<size_t>(xin) * esize;
-    const size_t ybytes = static_cast<size_t>(yout) * esize;
+    s->N = N; s->H = H; s->W = W; s->Cin = Cin; s->Cout = Cout;
+    s->kh = kh; s->kw = kw; s->stride = stride; s->pad = pad; s->act = QUAN_ACT_NONE;
+    s->Ho = static_cast<int>(Ho); s->Wo = static_cast<int>(Wo);
+    s->Qin = Cin / 4; s->Qout = Cout / 4;
+    s->M = static_cast<long long>(N) * Ho * Wo;
+    s->sep = 0;
+    return QUAN_OK;
+}
+
+size_t x_bytes(const quan::ConvShape& s, size_t esize) {
+    return static_cast<size_t>(s.N) * s.H * s.W * s.Cin * esize;
+}
+size_t y_bytes(const quan::ConvShape& s, size_t esize) {
+    return static_cast<size_t>(s.M) * s.Cout * esize;
+}
+size_t w_bytes(const quan::ConvShape& s, size_t esize) {
+    return static_cast<size_t>(s.Qout) * s.kh * s.kw * s.Qin * esize;
+}
+
+quan_status_t validate(quan::ConvShape* s, const void* x, const void* const w[4],
+                       const float* bias, const float* scale, const float* shift, int N, int H,
+                       int W, int Cin, int Cout, int kh, int kw, int stride, int pad, int act,
+                       const void* residual, const void* out, size_t esize) {
+    if (!x || !w[0] || !w[1] || !w[2] || !w[3] || !out)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    quan_status_t st = geometry(s, N, H, W, Cin, Cout, kh, kw, stride, pad);
+    if (st != QUAN_OK) return st;
+    if ((scale == nullptr) != (shift == nullptr))
+        return fail(QUAN_ERR_INVALID_ARG, "iqbn_scale and iqbn_shift must both be given or both NULL");
+    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
+    const size_t wbytes = w_bytes(*s, esize), xbytes = x_bytes(*s, esize);
+    const size_t ybytes = y_bytes(*s, esize);
     if (overlaps(out, ybytes, x, xbytes) || overlaps(out, ybytes, w[0], wbytes) ||
         overlaps(out, ybytes, w[1], wbytes) || overlaps(out, ybytes, w[2], wbytes) ||
         overlaps(out, ybytes, w[3], wbytes) || overlaps(out, ybytes, residual, ybytes) ||
         overlaps(out, ybytes, bias, Cout * 4u) || overlaps(out, ybytes, scale, Cout * 4u) ||
         overlaps(out, ybytes, shift, Cout * 4u))
         return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input");
-    s->N = N; s->H = H; s->W = W; s->Cin = Cin; s->Cout = Cout;
-    s->kh = kh; s->kw = kw; s->stride = stride; s->pad = pad; s->act = act;
-    s->Ho = static_cast<int>(Ho); s->Wo = static_cast<int>(Wo);
-    s->Qin = Cin / 4; s->Qout = Cout / 4;
-    s->M = static_cast<long long>(N) * Ho * Wo;
-    s->sep = 0;
+    s->act = act;
     return QUAN_OK;
 }
 
@@ -176,6 +194,107 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         t_last_path = QUAN_PATH_SIMT;
         t_last_kernel = s.sep ? "qconv_simt_kernel<bf16,sep>" : "qconv_simt_kernel<bf16>";
     }
+    return QUAN_OK;
+}
+
+// Input gradient of the pre-epilogue convolution (full form or separable).
+quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H, int W, int Cin,
+                           int Cout, int kh, int kw, int stride, int pad, bool separable,
+                           void* workspace, size_t workspace_bytes, void* dx,
+                           quan_stream_t stream) {
+    if (!dy || !w[0] || !w[1] || !w[2] || !w[3] || !dx)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    quan::ConvShape s;
+    quan_status_t st = geometry(&s, N, H, W, Cin, Cout, kh, kw, stride, pad);
+    if (st != QUAN_OK) return st;
+    s.sep = separable ? 1 : 0;
+    const size_t need = quan::bwd_data_workspace_bytes(Cin, Cout, kh, kw);
+    if (!workspace || workspace_bytes < need)
+        return fail(QUAN_ERR_INVALID_ARG, "workspace must hold %zu bytes (got %zu%s)", need,
+                    workspace_bytes, workspace ? "" : ", NULL");
+    const size_t dxb = x_bytes(s, 2), dyb = y_bytes(s, 2), wb = w_bytes(s, 2);
+    for (int L = 0; L < 4; ++L)
+        if (overlaps(dx, dxb, w[L], wb) || overlaps(workspace, need, w[L], wb))
+            return fail(QUAN_ERR_INVALID_ARG, "dx or workspace overlaps a weight tensor");
+    if (overlaps(dx, dxb, dy, dyb) || overlaps(workspace, need, dy, dyb) ||
+        overlaps(workspace, need, dx, dxb))
+        return fail(QUAN_ERR_INVALID_ARG, "dx, dy and workspace must not overlap");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    // The stride-1 full form is a forward convolution of dy with the transformed letters
+    // (output channels Cin, input channels Cout, padding kh - 1 - pad).
+    quan::ConvShape t;
+    const quan::EpilogueArgs none{nullptr, nullptr, nullptr, nullptr};
+    const size_t per = need / 4;
+    const void* tw[4];
+    for (int L = 0; L < 4; ++L) tw[L] = static_cast<const char*>(workspace) + L * per;
+    bool tc_ok = !separable && stride == 1 && kh == kw && pad <= kh - 1 && cc == 103 &&
+                 geometry(&t, N, s.Ho, s.Wo, Cout, Cin, kh, kw, 1, kh - 1 - pad) == QUAN_OK &&
+                 quan::tc_supported(t, dy, tw, dx, none);
+    const int path = g_path.load();
+    if (path == QUAN_PATH_TC && !tc_ok)
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "tensor-core input gradient needs the full form, stride 1, a square filter, "
+                    "pad < kh, sm_103 and Cin/4, Cout/4 multiples of 16 with 16-byte aligned "
+                    "tensors");
+    if (tc_ok && path != QUAN_PATH_SIMT) {
+        e = quan::launch_bwd_transform(Cin, Cout, kh, kw, w, workspace, num_sms, cs);
+        if (e != cudaSuccess) return cuda_fail(e, "bwd_transform launch");
+        quan::TcOptions opt;
+        opt.kappa = g_kappa.load();
+        opt.bnq = g_bnq.load();
+        opt.max_ctas = g_max_ctas.load();
+        opt.mode = g_mode.load();
+        opt.ws_halo = g_ws_halo.load();
+        opt.ws_issuers = g_ws_issuers.load();
+        opt.wait_limit_ns = g_wait_limit.load();
+        opt.inject_stall = g_inject.load();
+        char err[256] = "";
+        e = quan::launch_qconv_tc(t, dy, tw, none, dx, opt, num_sms, cs, err, sizeof(err));
+        if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+        if (e != cudaSuccess) return cuda_fail(e, "qconv_tc launch");
+        t_last_path = QUAN_PATH_TC;
+        t_last_kernel = quan::last_tc_kernel();
+        return QUAN_OK;
+    }
+    e = quan::launch_bwd_data_simt(s, dy, w, dx, cs);
+    if (e != cudaSuccess) return cuda_fail(e, "bwd_data_simt launch");
+    t_last_path = QUAN_PATH_SIMT;
+    t_last_kernel = separable ? "bwd_data_simt_kernel<sep>" : "bwd_data_simt_kernel";
+    return QUAN_OK;
+}
+
+// Weight gradients of the pre-epilogue convolution (full form or separable).
+quan_status_t run_bwd_weight(const void* x, const void* dy, int N, int H, int W, int Cin,
+                             int Cout, int kh, int kw, int stride, int pad, bool separable,
+                             float* const dw[4], quan_stream_t stream) {
+    if (!x || !dy || !dw[0] || !dw[1] || !dw[2] || !dw[3])
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    quan::ConvShape s;
+    quan_status_t st = geometry(&s, N, H, W, Cin, Cout, kh, kw, stride, pad);
+    if (st != QUAN_OK) return st;
+    s.sep = separable ? 1 : 0;
+    const size_t xb = x_bytes(s, 2), dyb = y_bytes(s, 2), wb = w_bytes(s, 4);
+    for (int L = 0; L < 4; ++L) {
+        if (overlaps(dw[L], wb, x, xb) || overlaps(dw[L], wb, dy, dyb))
+            return fail(QUAN_ERR_INVALID_ARG, "a weight gradient overlaps x or dy");
+        for (int K = 0; K < L; ++K)
+            if (overlaps(dw[L], wb, dw[K], wb))
+                return fail(QUAN_ERR_INVALID_ARG, "the weight gradients overlap");
+        if (reinterpret_cast<uintptr_t>(dw[L]) % 4 != 0)
+            return fail(QUAN_ERR_INVALID_ARG, "weight gradients must be 4-byte aligned");
+    }
+    if (g_path.load() == QUAN_PATH_TC)
+        return fail(QUAN_ERR_UNSUPPORTED, "the weight gradient runs on CUDA cores only");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    e = quan::launch_bwd_weight_simt(s, x, dy, dw, num_sms, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "bwd_weight_simt launch");
+    t_last_path = QUAN_PATH_SIMT;
+    t_last_kernel = separable ? "bwd_weight_simt_kernel<sep>" : "bwd_weight_simt_kernel";
     return QUAN_OK;
 }
 
@@ -248,6 +367,47 @@ quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
     e = quan::launch_poincare(rgb, npix, out, num_sms, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "poincare launch");
     return QUAN_OK;
+}
+
+size_t quan_qconv2d_bwd_data_workspace_size(int Cin, int Cout, int kh, int kw) {
+    if (Cin < 4 || Cout < 4 || kh < 1 || kw < 1 || Cin % 4 || Cout % 4) return 0;
+    return quan::bwd_data_workspace_bytes(Cin, Cout, kh, kw);
+}
+
+quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* wi,
+                                    const void* wj, const void* wk, int N, int H, int W, int Cin,
+                                    int Cout, int kh, int kw, int stride, int pad,
+                                    void* workspace, size_t workspace_bytes, void* dx,
+                                    quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    return run_bwd_data(dy, w, N, H, W, Cin, Cout, kh, kw, stride, pad, false, workspace,
+                        workspace_bytes, dx, stream);
+}
+
+quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const void* wi,
+                                        const void* wj, const void* wk, int N, int H, int W,
+                                        int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                        void* workspace, size_t workspace_bytes, void* dx,
+                                        quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    return run_bwd_data(dy, w, N, H, W, Cin, Cout, kh, kw, stride, pad, true, workspace,
+                        workspace_bytes, dx, stream);
+}
+
+quan_status_t quan_qconv2d_bwd_weight(const void* x, const void* dy, int N, int H, int W,
+                                      int Cin, int Cout, int kh, int kw, int stride, int pad,
+                                      float* dwr, float* dwi, float* dwj, float* dwk,
+                                      quan_stream_t stream) {
+    float* const dw[4] = {dwr, dwi, dwj, dwk};
+    return run_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, false, dw, stream);
+}
+
+quan_status_t quan_qconv2d_sep_bwd_weight(const void* x, const void* dy, int N, int H, int W,
+                                          int Cin, int Cout, int kh, int kw, int stride,
+                                          int pad, float* dwr, float* dwi, float* dwj,
+                                          float* dwk, quan_stream_t stream) {
+    float* const dw[4] = {dwr, dwi, dwj, dwk};
+    return run_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, true, dw, stream);
 }
 
 quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,

@@ -14,7 +14,8 @@ Recipe (the paper's data sets are not available; these stand in for them):
   * numpy PCG64 generators seeded with (config, layer, 0) for the activations
     (images drawn in batch order, so a smaller batch is a prefix of the full one)
     and (config, layer, 1) for the parameters, drawn in the order
-    W_r, W_i, W_j, W_k, bias, scale, shift; a residual input uses (config, layer, 7).
+    W_r, W_i, W_j, W_k, bias, scale, shift; a residual input uses (config, layer, 7),
+    the output gradient of the backward pass ~ N(0, 1) uses (config, layer, 9).
 Shapes follow the paper's workloads: CIFAR 32x32, ImageNet ResNet stages at
 56/28/14/7, and a 640-px detector neck at stride 8/16.
 """
@@ -150,6 +151,15 @@ def layer_inputs(spec: LayerSpec, n_images: int | None = None) -> dict:
     else:
         out["residual"] = None
     return out
+
+
+def grad_output(spec: LayerSpec, n_images: int | None = None) -> np.ndarray:
+    """The output gradient dy [N, Ho, Wo, C_out] for the backward pass of one layer, as
+    bf16 bits (a prefix of the full batch for a smaller ``n_images``)."""
+    N = spec.N if n_images is None else n_images
+    rng = np.random.default_rng(spec.seed + (9,))
+    dy = rng.standard_normal((N, spec.Ho, spec.Wo, spec.Cout), dtype=np.float32)
+    return to_bf16_bits(dy)
 
 
 def small_layer(name: str, N: int, H: int, W: int, Cin: int, Cout: int, k: int, stride: int,

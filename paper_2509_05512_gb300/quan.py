@@ -64,6 +64,14 @@ def load():
         lib.quan_qconv2d_sep_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
         lib.quan_poincare_fwd.argtypes = [_vp, ctypes.c_longlong, _vp, _vp]
+        _bwd_data_args = [_vp] * 5 + [_i] * 9 + [_vp, ctypes.c_size_t, _vp, _vp]
+        lib.quan_qconv2d_bwd_data.argtypes = _bwd_data_args
+        lib.quan_qconv2d_sep_bwd_data.argtypes = _bwd_data_args
+        lib.quan_qconv2d_bwd_data_workspace_size.argtypes = [_i] * 4
+        lib.quan_qconv2d_bwd_data_workspace_size.restype = ctypes.c_size_t
+        _bwd_weight_args = [_vp] * 2 + [_i] * 9 + [_vp] * 5
+        lib.quan_qconv2d_bwd_weight.argtypes = _bwd_weight_args
+        lib.quan_qconv2d_sep_bwd_weight.argtypes = _bwd_weight_args
         lib.quan_set_path.argtypes = [_i]
         lib.quan_last_path.argtypes = []
         lib.quan_last_kernel.argtypes = []
@@ -80,7 +88,9 @@ def load():
         lib.quan_last_error_message.restype = ctypes.c_char_p
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
-                     "quan_qconv2d_sep_fwd", "quan_poincare_fwd",
+                     "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
+                     "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
+                     "quan_qconv2d_sep_bwd_weight",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
                      "quan_set_tc_halo", "quan_set_tc_issuers"):
@@ -248,6 +258,74 @@ def poincare(rgb, *, out=None, stream=None):
     if out is None:
         out = torch.empty(rgb.shape[:-1] + (4,), dtype=torch.bfloat16, device=rgb.device)
     quan_poincare_fwd(rgb, rgb.numel() // 3, out, stream)
+    return out
+
+
+def quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw) -> int:
+    return load().quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw)
+
+
+def quan_qconv2d_bwd_data(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad, workspace,
+                          workspace_bytes, dx, stream=None) -> None:
+    _check(load().quan_qconv2d_bwd_data(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), N, H,
+                                        W, Cin, Cout, kh, kw, stride, pad, _ptr(workspace),
+                                        workspace_bytes, _ptr(dx), _stream(stream)))
+
+
+def quan_qconv2d_sep_bwd_data(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad,
+                              workspace, workspace_bytes, dx, stream=None) -> None:
+    _check(load().quan_qconv2d_sep_bwd_data(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), N,
+                                            H, W, Cin, Cout, kh, kw, stride, pad,
+                                            _ptr(workspace), workspace_bytes, _ptr(dx),
+                                            _stream(stream)))
+
+
+def quan_qconv2d_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, dwr, dwi, dwj, dwk,
+                            stream=None) -> None:
+    _check(load().quan_qconv2d_bwd_weight(_ptr(x), _ptr(dy), N, H, W, Cin, Cout, kh, kw, stride,
+                                          pad, _ptr(dwr), _ptr(dwi), _ptr(dwj), _ptr(dwk),
+                                          _stream(stream)))
+
+
+def quan_qconv2d_sep_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, dwr, dwi, dwj,
+                                dwk, stream=None) -> None:
+    _check(load().quan_qconv2d_sep_bwd_weight(_ptr(x), _ptr(dy), N, H, W, Cin, Cout, kh, kw,
+                                              stride, pad, _ptr(dwr), _ptr(dwi), _ptr(dwj),
+                                              _ptr(dwk), _stream(stream)))
+
+
+def qconv2d_backward_data(dy, wr, wi, wj, wk, *, H, W, stride=1, pad=0, separable=False,
+                          workspace=None, out=None, stream=None):
+    """Input gradient of the pre-epilogue convolution: dy [N, Ho, Wo, Cout] (bf16, CUDA) ->
+    dx [N, H, W, Cin] bf16.  `workspace` (a uint8 CUDA tensor of at least
+    quan_qconv2d_bwd_data_workspace_size bytes) is allocated when not given."""
+    import torch
+    N, Ho, Wo, Cout = dy.shape
+    Qout, kh, kw, Qin = wr.shape
+    Cin = 4 * Qin
+    need = quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dy.device)
+    if out is None:
+        out = torch.empty((N, H, W, Cin), dtype=torch.bfloat16, device=dy.device)
+    fn = quan_qconv2d_sep_bwd_data if separable else quan_qconv2d_bwd_data
+    fn(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad, workspace,
+       workspace.numel() * workspace.element_size(), out, stream)
+    return out
+
+
+def qconv2d_backward_weight(x, dy, *, kh, kw, stride=1, pad=0, separable=False, out=None,
+                            stream=None):
+    """Weight gradients of the pre-epilogue convolution: x [N, H, W, Cin], dy
+    [N, Ho, Wo, Cout] (bf16, CUDA) -> (dW_r, dW_i, dW_j, dW_k), fp32 [Cout/4, kh, kw, Cin/4]."""
+    import torch
+    N, H, W, Cin = x.shape
+    Cout = dy.shape[-1]
+    if out is None:
+        out = tuple(torch.empty((Cout // 4, kh, kw, Cin // 4), dtype=torch.float32,
+                                device=x.device) for _ in range(4))
+    fn = quan_qconv2d_sep_bwd_weight if separable else quan_qconv2d_bwd_weight
+    fn(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, *out, stream)
     return out
 
 

@@ -90,3 +90,64 @@ def test_no_python_fallback_when_library_missing(monkeypatch, tmp_path):
     monkeypatch.setattr(quan, "_lib", None)
     with pytest.raises(RuntimeError, match="not built"):
         quan.load()
+
+
+def _bwd_data(lib, sep=False, **kw):
+    a = dict(dy=FAKE, wr=FAKE + 0x1000, wi=FAKE + 0x2000, wj=FAKE + 0x3000, wk=FAKE + 0x4000,
+             N=1, H=8, W=8, Cin=64, Cout=128, kh=3, kw=3, stride=1, pad=1,
+             ws=0x8000000, ws_bytes=36864, dx=0x7000000)
+    a.update(kw)
+    f = lib.quan_qconv2d_sep_bwd_data if sep else lib.quan_qconv2d_bwd_data
+    return f(a["dy"], a["wr"], a["wi"], a["wj"], a["wk"], a["N"], a["H"], a["W"], a["Cin"],
+             a["Cout"], a["kh"], a["kw"], a["stride"], a["pad"], a["ws"], a["ws_bytes"], a["dx"],
+             None)
+
+
+def _bwd_weight(lib, sep=False, **kw):
+    a = dict(x=FAKE, dy=FAKE * 16, N=1, H=8, W=8, Cin=64, Cout=128, kh=3, kw=3, stride=1,
+             pad=1, dwr=0x7000000, dwi=0x7100000, dwj=0x7200000, dwk=0x7300000)
+    a.update(kw)
+    f = lib.quan_qconv2d_sep_bwd_weight if sep else lib.quan_qconv2d_bwd_weight
+    return f(a["x"], a["dy"], a["N"], a["H"], a["W"], a["Cin"], a["Cout"], a["kh"], a["kw"],
+             a["stride"], a["pad"], a["dwr"], a["dwi"], a["dwj"], a["dwk"], None)
+
+
+def test_backward_workspace_size(lib):
+    # four transformed letters of (Cin/4) * kh * kw * (Cout/4) bf16 values
+    assert lib.quan_qconv2d_bwd_data_workspace_size(64, 128, 3, 3) == 4 * 16 * 9 * 32 * 2
+    assert lib.quan_qconv2d_bwd_data_workspace_size(4, 64, 7, 7) == 4 * 1 * 49 * 16 * 2
+    assert lib.quan_qconv2d_bwd_data_workspace_size(6, 64, 3, 3) == 0
+    assert lib.quan_qconv2d_bwd_data_workspace_size(64, 64, 0, 3) == 0
+
+
+@pytest.mark.parametrize("sep", [False, True])
+@pytest.mark.parametrize("bad", [
+    dict(dy=None), dict(wj=None), dict(dx=None), dict(Cin=6), dict(stride=0), dict(kh=11),
+    dict(ws=None), dict(ws_bytes=36863),   # workspace missing or one byte short
+    dict(dx=FAKE),                         # dx overlaps dy
+    dict(ws=FAKE + 0x2000),                # workspace overlaps a weight tensor
+    dict(ws=0x7000000 + 64),               # workspace overlaps dx
+])
+def test_backward_data_invalid_arguments(lib, sep, bad):
+    assert _bwd_data(lib, sep, **bad) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_last_error_message()
+
+
+@pytest.mark.parametrize("sep", [False, True])
+@pytest.mark.parametrize("bad", [
+    dict(x=None), dict(dwk=None), dict(Cout=10), dict(pad=-1),
+    dict(dwi=0x7000000 + 4),               # two weight gradients overlap
+    dict(dwr=FAKE),                        # a weight gradient overlaps x
+    dict(dwj=0x7200002),                   # misaligned fp32 output
+])
+def test_backward_weight_invalid_arguments(lib, sep, bad):
+    assert _bwd_weight(lib, sep, **bad) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_last_error_message()
+
+
+def test_backward_weight_has_no_tensor_core_path(lib):
+    assert lib.quan_set_path(quan.QUAN_PATH_TC) == quan.QUAN_OK
+    try:
+        assert _bwd_weight(lib) == quan.QUAN_ERR_UNSUPPORTED
+    finally:
+        assert lib.quan_set_path(quan.QUAN_PATH_AUTO) == quan.QUAN_OK

@@ -329,3 +329,52 @@ def test_backward_single_pixel_is_conjugate_multiplication():
     dw = oracle.qconv2d_bwd_weight(xq.reshape(1, 1, 1, 4), g.reshape(1, 1, 1, 4), kh=1, kw=1)
     np.testing.assert_allclose(np.array([t.item() for t in dw]), oracle.qmul(g, conj(xq)),
                                rtol=1e-14, atol=1e-15)
+
+
+# ----------------------------------------------------------------- separable backward
+# Eq. 8-10: the same adjoint identities against the separable forward (Eq. 7), and the
+# per-component reduction to PyTorch's own convolution gradients with Eq. 9's M.
+
+EQ9_M = np.array([[1, 1, 1, 1], [-1, 1, -1, 1], [-1, 1, 1, -1], [-1, -1, 1, 1]], dtype=float)
+
+
+@pytest.mark.parametrize("case", BWD_CASES)
+def test_separable_backward_is_the_adjoint_of_eq7(case):
+    N, H, W, Cin, Cout, kh, kw, s, p = case
+    rng = np.random.default_rng(100 + sum(case))
+    x, w = _rand_layer(rng, N, H, W, Cin, Cout, kh, kw)
+    y = oracle.qconv2d_separable(x, *w, stride=s, pad=p)
+    dy = rng.standard_normal(y.shape)
+    lhs = float(np.sum(dy * y))
+    dx = oracle.qconv2d_sep_bwd_data(dy, *w, H=H, W=W, stride=s, pad=p)
+    dw = oracle.qconv2d_sep_bwd_weight(x, dy, kh=kh, kw=kw, stride=s, pad=p)
+    assert dx.shape == x.shape and all(g.shape == t.shape for g, t in zip(dw, w))
+    np.testing.assert_allclose(float(np.sum(dx * x)), lhs, rtol=1e-11)
+    np.testing.assert_allclose(sum(float(np.sum(g * t)) for g, t in zip(dw, w)), lhs,
+                               rtol=1e-11)
+
+
+@pytest.mark.parametrize("case", [(1, 7, 6, 8, 12, 3, 3, 1, 1), (2, 9, 8, 8, 4, 3, 3, 2, 1)])
+def test_separable_backward_matches_torch_gradients(case):
+    # component p: dx_p = conv2d_input(sum_m M[p][m] dy_m, W_p) and
+    # dW_p = conv2d_weight(x_p, ..., sum_m M[p][m] dy_m), PyTorch fp64 on the CPU
+    N, H, W, Cin, Cout, kh, kw, s, p = case
+    rng = np.random.default_rng(200 + sum(case))
+    x, w = _rand_layer(rng, N, H, W, Cin, Cout, kh, kw)
+    Qin, Qout = Cin // 4, Cout // 4
+    Ho, Wo = (H + 2 * p - kh) // s + 1, (W + 2 * p - kw) // s + 1
+    dy = rng.standard_normal((N, Ho, Wo, Cout))
+    dx = oracle.qconv2d_sep_bwd_data(dy, *w, H=H, W=W, stride=s, pad=p)
+    dw = oracle.qconv2d_sep_bwd_weight(x, dy, kh=kh, kw=kw, stride=s, pad=p)
+    nchw = lambda a: torch.from_numpy(np.ascontiguousarray(a)).permute(0, 3, 1, 2)
+    for comp in range(4):
+        g = sum(EQ9_M[comp, m] * _comp(dy, m, Qout) for m in range(4))
+        wt = nchw(w[comp])  # [Qout][Qin][kh][kw]
+        ref_dx = torch.nn.grad.conv2d_input((N, Qin, H, W), wt, nchw(g), stride=s, padding=p)
+        np.testing.assert_allclose(_comp(dx, comp, Qin), ref_dx.permute(0, 2, 3, 1).numpy(),
+                                   rtol=1e-12, atol=1e-12)
+        ref_dw = torch.nn.grad.conv2d_weight(nchw(_comp(x, comp, Qin)), (Qout, Qin, kh, kw),
+                                             nchw(g), stride=s, padding=p)
+        np.testing.assert_allclose(dw[comp], ref_dw.permute(0, 2, 3, 1).numpy(), rtol=1e-12,
+                                   atol=1e-12)
+
