@@ -32,6 +32,7 @@ if ROOT not in sys.path:
 METRIC = "QConv fwd real-equiv TFLOP/s & % bf16 tensor peak (1 GB300); backbone images/s"
 L2_BYTES = 126 * 1024 * 1024
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.070e9 / 1e12  # FFMA: SMs x lanes x 2 FLOP x max clock
 
 
 def parse_args():
@@ -42,6 +43,10 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c1",
                     choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone", "poincare"])
+    ap.add_argument("--pass", dest="direction", choices=["fwd", "bwd"], default="fwd",
+                    help="layer workloads: the forward convolution, or its backward pass "
+                         "(input and weight gradients before the epilogue, from a seeded "
+                         "output gradient)")
     ap.add_argument("--variant", choices=["full", "separable"], default="full",
                     help="layer workloads: the full Hamilton form (Eq. 5/6) or the separable "
                          "form of Eq. 7 (a quarter of the multiply-adds)")
@@ -287,6 +292,196 @@ class LayerRunner:
         return self.spec.algorithmic_bytes
 
 
+class BwdRunner:
+    """Backward pass of one layer: dx (quan_qconv2d[_sep]_bwd_data) and dW
+    (quan_qconv2d[_sep]_bwd_weight) from a seeded output gradient, with rotating buffer
+    sets like LayerRunner."""
+
+    def __init__(self, spec, torch, quan, inputs, separable=False):
+        import numpy as np
+        self.spec, self.torch, self.quan = spec, torch, quan
+        self.separable = separable
+        self.bwd_data = quan.quan_qconv2d_sep_bwd_data if separable else quan.quan_qconv2d_bwd_data
+        self.bwd_weight = (quan.quan_qconv2d_sep_bwd_weight if separable
+                           else quan.quan_qconv2d_bwd_weight)
+        d = inputs.layer_inputs(spec)
+        d["dy"] = inputs.grad_output(spec)
+        dev = torch.device("cuda")
+
+        def up(a):
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(
+                torch.bfloat16).to(dev)
+
+        self.host = d
+        x0, dy0 = up(d["x"]), up(d["dy"])
+        self.w = [up(d[k]) for k in ("wr", "wi", "wj", "wk")]
+        per_set = (2 * x0.numel() + 2 * dy0.numel()) * 2  # x, dy read; dx written
+        self.sets = max(2, min(16, math.ceil(2 * L2_BYTES / per_set)))
+        self.xs = [x0] + [x0.clone() for _ in range(self.sets - 1)]
+        self.dys = [dy0] + [dy0.clone() for _ in range(self.sets - 1)]
+        self.dxs = [torch.empty_like(x0) for _ in range(self.sets)]
+        wshape = (spec.Cout // 4, spec.kh, spec.kw, spec.Cin // 4)
+        self.dws = [torch.empty(wshape, dtype=torch.float32, device=dev) for _ in range(4)]
+        self.ws_bytes = quan.quan_qconv2d_bwd_data_workspace_size(spec.Cin, spec.Cout,
+                                                                  spec.kh, spec.kw)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=dev)
+        self.i = 0
+        self.footprint = per_set * self.sets
+        self.launches_per_step = None  # set by count_launches()
+
+    def data(self, k, stream):
+        s = self.spec
+        self.bwd_data(self.dys[k], *self.w, s.N, s.H, s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride,
+                      s.pad, self.ws, self.ws_bytes, self.dxs[k], stream)
+
+    def weight(self, k, stream):
+        s = self.spec
+        self.bwd_weight(self.xs[k], self.dys[k], s.N, s.H, s.W, s.Cin, s.Cout, s.kh, s.kw,
+                        s.stride, s.pad, *self.dws, stream)
+
+    def step(self, stream):
+        k = self.i % self.sets
+        self.i += 1
+        self.data(k, stream)
+        self.weight(k, stream)
+
+    def count_launches(self, stream):
+        """Kernels of this library one step launches (the tensor-core input gradient is a
+        weight transform plus one convolution kernel; the weight gradient one kernel)."""
+        self.data(0, stream)
+        n = 2 if self.quan.quan_last_path() == self.quan.QUAN_PATH_TC else 1
+        self.data_kernel = self.quan.quan_last_kernel()
+        self.weight(0, stream)
+        self.weight_kernel = self.quan.quan_last_kernel()
+        self.launches_per_step = n + 1
+
+    def e2e_setup(self):
+        torch = self.torch
+        import numpy as np
+        d = self.host
+        parts = [("x", d["x"].view(np.uint8)), ("dy", d["dy"].view(np.uint8))]
+        parts += [(k, d[k].view(np.uint8)) for k in ("wr", "wi", "wj", "wk")]
+        self.e2e_layout, off = {}, 0
+        for name, a in parts:
+            self.e2e_layout[name] = (off, a.nbytes)
+            off += (a.nbytes + 255) // 256 * 256
+        host = np.zeros(off, dtype=np.uint8)
+        for name, a in parts:
+            o, n = self.e2e_layout[name]
+            host[o:o + n] = np.ascontiguousarray(a).reshape(-1)
+        self.h_in = torch.from_numpy(host).pin_memory()
+        s = self.spec
+        dx_bytes = s.N * s.H * s.W * s.Cin * 2
+        dw_bytes = s.Cout * s.Cin * s.kh * s.kw // 4 * 4  # four fp32 letters
+        self.out_layout = (dx_bytes, (dx_bytes + 255) // 256 * 256)
+        out_total = self.out_layout[1] + dw_bytes
+        self.h_out = [torch.empty(out_total, dtype=torch.uint8).pin_memory()
+                      for _ in range(E2E_BUFFERS)]
+        self.e_in = [torch.empty_like(self.h_in, device="cuda") for _ in range(E2E_BUFFERS)]
+        self.e_out = [torch.empty_like(t, device="cuda") for t in self.h_out]
+        self.h2d = sum(n for _, n in self.e2e_layout.values())
+        self.d2h = dx_bytes + dw_bytes
+
+    def e2e_in(self, b):
+        return [(self.e_in[b], self.h_in)]
+
+    def e2e_out(self, b):
+        return [(self.h_out[b], self.e_out[b])]
+
+    def e2e_compute(self, b, stream):
+        torch, s = self.torch, self.spec
+
+        def view(name):
+            o, n = self.e2e_layout[name]
+            return self.e_in[b][o:o + n].view(torch.bfloat16)
+
+        dx_bytes, dw_off = self.out_layout
+        dx = self.e_out[b][:dx_bytes]
+        per = s.Cout * s.Cin * s.kh * s.kw // 16 * 4
+        dw = [self.e_out[b][dw_off + L * per:dw_off + (L + 1) * per].view(torch.float32)
+              for L in range(4)]
+        w = [view(k) for k in ("wr", "wi", "wj", "wk")]
+        self.bwd_data(view("dy"), *w, s.N, s.H, s.W, s.Cin, s.Cout, s.kh, s.kw, s.stride,
+                      s.pad, self.ws, self.ws_bytes, dx, stream)
+        self.bwd_weight(view("x"), view("dy"), s.N, s.H, s.W, s.Cin, s.Cout, s.kh, s.kw,
+                        s.stride, s.pad, *dw, stream)
+
+    @property
+    def flops(self):
+        # input and weight gradients, each as many multiply-adds as the forward
+        return 2 * self.spec.flops / (4 if self.separable else 1)
+
+    def kernel_times(self, torch, stream, reps=5):
+        """Average duration of the input-gradient and weight-gradient calls, timed apart
+        with events on the launching stream (outside the timed region)."""
+        sh = stream.cuda_stream
+        out = []
+        for fn in (self.data, self.weight):
+            for k in range(2):
+                fn(k % self.sets, sh)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for r in range(reps):
+                fn(r % self.sets, sh)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) / reps / 1e3)
+        return out
+
+
+def bwd_roofline(runner, torch, stream, peaks, peak_src, direction_key):
+    """Roofline of the slower of the two gradient calls.  Tensor-core input gradient:
+    FLOPs against the bf16 peak; CUDA-core gradients: FLOPs against the fp32 FFMA peak
+    (152 SMs x 128 lanes x 2 FLOP x 2.07 GHz maximum clock)."""
+    t_data, t_weight = runner.kernel_times(torch, stream)
+    half = runner.flops / 2
+    rows = []
+    for name, t, kernel in (("dx", t_data, runner.data_kernel),
+                            ("dW", t_weight, runner.weight_kernel)):
+        tc = kernel.startswith("qconv_")
+        peak = peaks["bf16_tflops"] if tc else FP32_ALU_TFLOPS
+        ach = half / t / 1e12
+        rows.append({"grad": name, "kernel": kernel, "ms": round(t * 1e3, 4),
+                     "bound": "tensor" if tc else "alu", "achieved": round(ach, 2),
+                     "peak": peak, "frac": round(ach / peak, 4)})
+    top = max(rows, key=lambda r: r["ms"])
+    src = (peak_src + " (burst)" if top["bound"] == "tensor"
+           else "derived: 152 SMs x 128 FP32 lanes x 2 FLOP x 2070 MHz")
+    return {"bound": top["bound"], "achieved": top["achieved"], "peak": top["peak"],
+            "unit": "TFLOP/s", "frac": top["frac"],
+            "traffic": recorded_traffic(direction_key, top["kernel"]),
+            "kernel": "%s (%s)" % (top["kernel"], top["grad"]),
+            "share": round(top["ms"] / (rows[0]["ms"] + rows[1]["ms"]), 3),
+            "peak_source": src, "algorithmic_flops": half, "gradients": rows}
+
+
+def cpu_bwd_sample(spec, seconds, inputs, separable=False):
+    """Time the fp64 oracle's two gradients on a bounded number of images."""
+    import oracle
+    d = inputs.layer_inputs(spec, n_images=1)
+    f64 = oracle.bf16_bits_to_f64
+    w = [f64(d[k]) for k in ("wr", "wi", "wj", "wk")]
+    bd = oracle.qconv2d_sep_bwd_data if separable else oracle.qconv2d_bwd_data
+    bw = oracle.qconv2d_sep_bwd_weight if separable else oracle.qconv2d_bwd_weight
+
+    def run(n):
+        x = f64(inputs.layer_inputs(spec, n_images=n)["x"])
+        dy = f64(inputs.grad_output(spec, n_images=n))
+        t0 = time.perf_counter()
+        bd(dy, *w, H=spec.H, W=spec.W, stride=spec.stride, pad=spec.pad)
+        bw(x, dy, kh=spec.kh, kw=spec.kw, stride=spec.stride, pad=spec.pad)
+        return time.perf_counter() - t0
+
+    t1 = run(1)
+    n = max(1, min(spec.N, int(seconds / max(t1, 1e-6))))
+    t = run(n) if n > 1 else t1
+    flop = 2 * spec.flops / spec.N * n / (4 if separable else 1)
+    return {"value": flop / t / 1e12, "unit": "TFLOP/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": "input and weight gradients of %d of %d images of the layer (fp64, "
+                      "%.2f s)" % (n, spec.N, t)}
+
+
 def cpu_oracle_sample(spec, seconds, inputs, separable=False):
     """Time the fp64 oracle on a bounded number of images of the layer."""
     import oracle
@@ -392,7 +587,7 @@ def poincare_cpu_sample(runner, seconds):
             "sample": "%d of %d images of the batch (fp64, %.2f s)" % (n, runner.N, t)}
 
 
-def workload_config(workload: str, inputs, variant: str = "full") -> dict:
+def workload_config(workload: str, inputs, variant: str = "full", direction: str = "fwd") -> dict:
     """The workload part of the JSON line's config, shared by both arms."""
     if workload == "poincare":
         N, H, W = POINCARE_SHAPE
@@ -415,6 +610,11 @@ def workload_config(workload: str, inputs, variant: str = "full") -> dict:
     if variant == "separable":
         cfg["workload"] += ", separable form (Eq. 7)"
         cfg["flops_per_step"] = s.flops / 4
+    if direction == "bwd":
+        cfg["workload"] += ", backward: input and weight gradients before the epilogue" + (
+            " (Eq. 8-10)" if variant == "separable" else "")
+        cfg["flops_per_step"] *= 2
+        cfg["epilogue"] = "none (gradient of the convolution's accumulator)"
     return cfg
 
 
@@ -460,8 +660,9 @@ def main():
 
     if args.batch and not args.profile:
         raise SystemExit("--batch is for --profile runs only")
-    if args.workload in ("backbone", "poincare") and args.variant != "full":
-        raise SystemExit("--variant applies to the convolution layer workloads")
+    if args.workload in ("backbone", "poincare") and (args.variant != "full" or
+                                                       args.direction != "fwd"):
+        raise SystemExit("--variant and --pass apply to the convolution layer workloads")
     if args.workload == "poincare":
         runner = PoincareRunner(torch, quan, *POINCARE_SHAPE)
         unit, per_step_units, dtype = "images/s", runner.N, "f32->bf16"
@@ -475,7 +676,10 @@ def main():
         if args.batch:
             import dataclasses
             spec = dataclasses.replace(spec, N=args.batch)
-        runner = LayerRunner(spec, torch, quan, inputs, separable=args.variant == "separable")
+        cls = BwdRunner if args.direction == "bwd" else LayerRunner
+        runner = cls(spec, torch, quan, inputs, separable=args.variant == "separable")
+        if args.direction == "bwd":
+            runner.count_launches(torch.cuda.current_stream().cuda_stream)
         unit, per_step_units, dtype = "TFLOP/s", runner.flops / 1e12, "bf16"
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
@@ -559,6 +763,8 @@ def main():
     peaks, peak_src = load_peaks()
     if args.workload == "backbone":
         roofline = backbone_roofline(runner, torch, stream, peaks, peak_src)
+    elif args.direction == "bwd":
+        roofline = bwd_roofline(runner, torch, stream, peaks, peak_src, traffic_key(args))
     else:
         roofline = runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name)
 
@@ -568,6 +774,9 @@ def main():
             cpu = backbone_cpu_sample(runner, args.cpu_seconds, inputs)
         elif args.workload == "poincare":
             cpu = poincare_cpu_sample(runner, args.cpu_seconds)
+        elif args.direction == "bwd":
+            cpu = cpu_bwd_sample(runner.spec, args.cpu_seconds, inputs,
+                                 separable=runner.separable)
         else:
             cpu = cpu_oracle_sample(runner.spec, args.cpu_seconds, inputs,
                                     separable=runner.separable)
@@ -576,14 +785,16 @@ def main():
         dist.destroy_process_group()
     if rank != 0:
         return 0
-    cfg = workload_config(args.workload, inputs, args.variant)
+    cfg = workload_config(args.workload, inputs, args.variant, args.direction)
     cfg.update({"l2": "inputs larger than L2: %d rotating buffer sets, %.0f MB" % (
                     getattr(runner, "sets", 1), runner.footprint / 1e6),
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
                 "timing": "one CUDA-graph replay of the K steps" if graph is not None
                 else "plain launch loop"})
-    if args.workload not in ("backbone", "poincare"):
+    if args.workload not in ("backbone", "poincare") and args.direction == "fwd":
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
+    if args.direction == "bwd":
+        cfg["kernels"] = {"dx": runner.data_kernel, "dW": runner.weight_kernel}
     line = {"metric": METRIC, "value": round(value, 4), "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
@@ -592,6 +803,12 @@ def main():
             "gpu_launches": runner.launches_per_step * args.steps, "clocks": clocks}
     print(json.dumps(line))
     return 0
+
+
+def traffic_key(args) -> str:
+    """Key of the workload in the recorded ncu traffic table."""
+    return (args.workload + (":bwd" if args.direction == "bwd" else "") +
+            (":sep" if args.variant == "separable" else ""))
 
 
 def runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name):
@@ -604,8 +821,7 @@ def runner_roofline(runner, args, ms_per_step, peaks, peak_src, kernel_name):
         achieved, peak, unit, bound = nbytes / t / 1e9, peaks["hbm_gbs"], "GB/s", "hbm"
     return {"bound": bound, "achieved": round(achieved, 2), "peak": peak, "unit": unit,
             "frac": round(achieved / peak, 4),
-            "traffic": recorded_traffic(args.workload + (":sep" if args.variant == "separable"
-                                                         else ""), kernel_name),
+            "traffic": recorded_traffic(traffic_key(args), kernel_name),
             "kernel": kernel_name, "peak_source": peak_src + " (burst)",
             "algorithmic_flops": flops, "algorithmic_bytes": nbytes}
 
@@ -682,7 +898,7 @@ def reference_arm(args, rank, world, inputs):
     if rank != 0:
         return 0
     import oracle
-    ref_cfg = workload_config(args.workload, inputs, args.variant)
+    ref_cfg = workload_config(args.workload, inputs, args.variant, args.direction)
     ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
     if args.workload == "poincare":
         import numpy as np
@@ -739,8 +955,17 @@ def reference_arm(args, rank, world, inputs):
 
     sep = args.variant == "separable"
     conv = oracle.qconv2d_separable if sep else oracle.qconv2d
+    bwd = args.direction == "bwd"
+    if bwd:
+        dy = f64(inputs.grad_output(spec, n_images=1))
+        bd = oracle.qconv2d_sep_bwd_data if sep else oracle.qconv2d_bwd_data
+        bw = oracle.qconv2d_sep_bwd_weight if sep else oracle.qconv2d_bwd_weight
 
     def step():
+        if bwd:
+            bd(dy, *w, H=spec.H, W=spec.W, stride=spec.stride, pad=spec.pad)
+            bw(x, dy, kh=spec.kh, kw=spec.kw, stride=spec.stride, pad=spec.pad)
+            return
         conv(x, *w, stride=spec.stride, pad=spec.pad, bias=d["bias"], scale=d["scale"],
              shift=d["shift"], act=spec.act)
 
@@ -750,10 +975,11 @@ def reference_arm(args, rank, world, inputs):
     for _ in range(args.steps):
         step()
     dt = time.perf_counter() - t0
-    per_step = spec.flops / spec.N / (4 if sep else 1)  # one image per step
+    per_step = spec.flops / spec.N / (4 if sep else 1) * (2 if bwd else 1)  # one image
     value = per_step * args.steps / dt / 1e12
     cpu = {"value": value, "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
-           "sample": "1 of %d images of the layer per step (fp64)" % spec.N}
+           "sample": "1 of %d images of the layer per step (fp64%s)" % (
+               spec.N, ", input and weight gradients" if bwd else "")}
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
