@@ -184,6 +184,30 @@ quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* 
                                     void* workspace, size_t workspace_bytes, void* dx,
                                     quan_stream_t stream);
 
+/*
+ * quan_qconv2d_bwd_data without the workspace argument, for callers that cannot allocate
+ * device memory: code running where cudaMalloc is off limits (its implicit device-wide
+ * synchronisation would stall other work, or a framework owns all device memory through
+ * its own pool), or a plain C caller with no allocator at hand.  The paper has no
+ * counterpart.  The transformed letters go to a scratch buffer of 2 MiB (2097152 bytes)
+ * that the library keeps in static device memory: every GPU that loads the library holds
+ * it until the process exits; the call itself allocates and frees nothing.
+ * Same arguments (minus the workspace), paths, results and errors as
+ * quan_qconv2d_bwd_data, plus QUAN_ERR_UNSUPPORTED when
+ * quan_qconv2d_bwd_data_workspace_size exceeds 2 MiB (e.g. 1024 -> 1024 real channels
+ * with a 3x3 filter: use quan_qconv2d_bwd_data with a workspace there).
+ *   Sharing  every call on a device uses the same buffer, which keeps the last call's
+ *            contents (each call rewrites all of it that it reads, so nothing has to start
+ *            at zero).  Calls whose kernels overlap on the GPU (other streams, other host
+ *            threads) race on it: order them (one stream, or events).
+ *   Set-up   the first call on each device looks up the buffer's device address, with
+ *            that device current; make that first call before any stream capture.
+ */
+quan_status_t quan_qconv2d_bwd_data_static(const void* dy, const void* wr, const void* wi,
+                                           const void* wj, const void* wk, int N, int H, int W,
+                                           int Cin, int Cout, int kh, int kw, int stride,
+                                           int pad, void* dx, quan_stream_t stream);
+
 /* Separable form (Eq. 8-9) of the input gradient; same arguments.  Runs on CUDA cores
  * (the workspace is checked but not used). */
 quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const void* wi,

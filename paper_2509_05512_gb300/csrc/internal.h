@@ -94,6 +94,10 @@ cudaError_t launch_bwd_transform(int Cin, int Cout, int kh, int kw, const void* 
 // dx [N][H][W][Cin] from dy [N][Ho][Wo][Cout] on CUDA cores, any stride.
 cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void* const w[4],
                                  void* dx, cudaStream_t stream);
+// Library-owned device scratch of quan_qconv2d_bwd_data_static (one per device, in the
+// module's static device memory): its size, and its address on the current device.
+constexpr size_t BWD_STATIC_SCRATCH_BYTES = size_t(2) << 20;
+cudaError_t bwd_static_scratch_address(void** ptr);
 // dW_L fp32 [Qout][kh][kw][Qin] (zeroed, then accumulated) on CUDA cores.
 cudaError_t launch_bwd_weight_simt(const ConvShape& s, const void* x, const void* dy,
                                    float* const dw[4], int num_sms, cudaStream_t stream);

@@ -183,7 +183,20 @@ __global__ void __launch_bounds__(256) bwd_weight_simt_kernel(
     atomicAdd(dwk + o, a3);
 }
 
+// Scratch of quan_qconv2d_bwd_data_static, the entry point for callers that cannot
+// allocate device memory: the transformed letters of one call live here instead of in a
+// caller workspace.  Every call writes all of the region it then reads, so nothing in it
+// has to start at zero; calls that overlap on the GPU share it and race.  Host code must
+// not pass this name to a kernel: on the host it is a stand-in, not a device address.
+static __device__ __align__(256) unsigned char g_bwd_static_scratch[BWD_STATIC_SCRATCH_BYTES];
+
 }  // namespace
+
+// Device address of the scratch on the current device (called once per device, with
+// that device current, by the entry point's first call there).
+cudaError_t bwd_static_scratch_address(void** ptr) {
+    return cudaGetSymbolAddress(ptr, g_bwd_static_scratch);
+}
 
 size_t bwd_data_workspace_bytes(int Cin, int Cout, int kh, int kw) {
     return static_cast<size_t>(4) * (Cin / 4) * kh * kw * (Cout / 4) * 2;

@@ -24,6 +24,7 @@ std::atomic<int> g_inject{0};
 constexpr int kMaxDevices = 64;
 int g_num_sms[kMaxDevices] = {0};
 int g_cc[kMaxDevices] = {0};
+void* g_static_scratch[kMaxDevices] = {nullptr};  // quan_qconv2d_bwd_data_static, per device
 std::mutex g_dev_mu;
 
 quan_status_t fail(quan_status_t st, const char* fmt, ...) {
@@ -382,6 +383,44 @@ quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* 
     const void* w[4] = {wr, wi, wj, wk};
     return run_bwd_data(dy, w, N, H, W, Cin, Cout, kh, kw, stride, pad, false, workspace,
                         workspace_bytes, dx, stream);
+}
+
+quan_status_t quan_qconv2d_bwd_data_static(const void* dy, const void* wr, const void* wi,
+                                           const void* wj, const void* wk, int N, int H, int W,
+                                           int Cin, int Cout, int kh, int kw, int stride,
+                                           int pad, void* dx, quan_stream_t stream) {
+    quan::ConvShape s;
+    quan_status_t st = geometry(&s, N, H, W, Cin, Cout, kh, kw, stride, pad);
+    if (st != QUAN_OK) return st;
+    if (!dy || !wr || !wi || !wj || !wk || !dx)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    const size_t need = quan::bwd_data_workspace_bytes(Cin, Cout, kh, kw);
+    if (need > quan::BWD_STATIC_SCRATCH_BYTES)
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "the transformed letters (%zu bytes) exceed the %zu-byte static scratch; "
+                    "use quan_qconv2d_bwd_data with a workspace",
+                    need, quan::BWD_STATIC_SCRATCH_BYTES);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    if (dev < 0 || dev >= kMaxDevices) return cuda_fail(cudaErrorInvalidDevice, "device query");
+    void* scratch = nullptr;
+    {
+        std::lock_guard<std::mutex> lk(g_dev_mu);
+        if (!g_static_scratch[dev]) {
+            // once per device, with that device current
+            void* p = nullptr;
+            e = quan::bwd_static_scratch_address(&p);
+            if (e != cudaSuccess || !p)
+                return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol,
+                                 "static scratch address");
+            g_static_scratch[dev] = p;
+        }
+        scratch = g_static_scratch[dev];
+    }
+    const void* w[4] = {wr, wi, wj, wk};
+    return run_bwd_data(dy, w, N, H, W, Cin, Cout, kh, kw, stride, pad, false, scratch,
+                        quan::BWD_STATIC_SCRATCH_BYTES, dx, stream);
 }
 
 quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const void* wi,

@@ -67,6 +67,7 @@ def load():
         _bwd_data_args = [_vp] * 5 + [_i] * 9 + [_vp, ctypes.c_size_t, _vp, _vp]
         lib.quan_qconv2d_bwd_data.argtypes = _bwd_data_args
         lib.quan_qconv2d_sep_bwd_data.argtypes = _bwd_data_args
+        lib.quan_qconv2d_bwd_data_static.argtypes = [_vp] * 5 + [_i] * 9 + [_vp, _vp]
         lib.quan_qconv2d_bwd_data_workspace_size.argtypes = [_i] * 4
         lib.quan_qconv2d_bwd_data_workspace_size.restype = ctypes.c_size_t
         _bwd_weight_args = [_vp] * 2 + [_i] * 9 + [_vp] * 5
@@ -90,6 +91,7 @@ def load():
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
                      "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
                      "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
+                     "quan_qconv2d_bwd_data_static",
                      "quan_qconv2d_sep_bwd_weight",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
@@ -270,6 +272,13 @@ def quan_qconv2d_bwd_data(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride
     _check(load().quan_qconv2d_bwd_data(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), N, H,
                                         W, Cin, Cout, kh, kw, stride, pad, _ptr(workspace),
                                         workspace_bytes, _ptr(dx), _stream(stream)))
+
+
+def quan_qconv2d_bwd_data_static(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad,
+                                 dx, stream=None) -> None:
+    _check(load().quan_qconv2d_bwd_data_static(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj),
+                                               _ptr(wk), N, H, W, Cin, Cout, kh, kw, stride,
+                                               pad, _ptr(dx), _stream(stream)))
 
 
 def quan_qconv2d_sep_bwd_data(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad,
