@@ -98,6 +98,13 @@ cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void*
 // module's static device memory): its size, and its address on the current device.
 constexpr size_t BWD_STATIC_SCRATCH_BYTES = size_t(2) << 20;
 cudaError_t bwd_static_scratch_address(void** ptr);
+// Tensor-core weight gradient of the full form (stride 1, Cin and Cout multiples of 64,
+// Cout <= 256 or a multiple of 256, 16-byte aligned x and dy).  Zeroes dW_L, then adds.
+bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy);
+cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* dy,
+                                 float* const dw[4], int num_sms,
+                                 unsigned long long wait_limit_ns, cudaStream_t stream,
+                                 char* err, size_t errlen);
 // dW_L fp32 [Qout][kh][kw][Qin] (zeroed, then accumulated) on CUDA cores.
 cudaError_t launch_bwd_weight_simt(const ConvShape& s, const void* x, const void* dy,
                                    float* const dw[4], int num_sms, cudaStream_t stream);

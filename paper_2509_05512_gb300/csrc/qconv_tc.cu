@@ -442,6 +442,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
 #include "qconv_ws.cuh"
 #include "qconv_gather.cuh"
+#include "qconv_dw.cuh"
 
 // ---------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 g_encode_tiled = nullptr;
@@ -813,6 +814,91 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     }
 }
 
+// ---------------------------------------------------------------- weight gradient
+constexpr int DW_SMEM_MAX = 232448;  // dynamic shared memory a CTA may opt into
+
+// Tiling of the tensor-core weight gradient (see qconv_dw.cuh); false if the shape has none.
+bool dw_plan(const ConvShape& s, int num_sms, dwk::DwParams* p) {
+    if (s.sep || s.stride != 1 || s.Cin % 64 != 0 || s.Cout % 64 != 0) return false;
+    if (s.Cout > 256 && s.Cout % 256 != 0) return false;
+    dwk::DwParams q = {};
+    q.Ho = s.Ho; q.Wo = s.Wo; q.Qin = s.Qin; q.Qout = s.Qout;
+    q.kh = s.kh; q.kw = s.kw; q.pad = s.pad; q.taps = s.kh * s.kw;
+    q.nxc = s.Cin / 64;
+    q.units = q.taps * q.nxc;
+    q.npairs = (q.units + 1) / 2;
+    q.ncols = s.Cout <= 256 ? s.Cout : 256;
+    q.nyb = q.ncols / 64;
+    int a_max = 512 / q.ncols;
+    if (a_max > dwk::MAX_PAIRS) a_max = dwk::MAX_PAIRS;
+    if (a_max > q.npairs) a_max = q.npairs;
+    // the most unit pairs per CTA for which some pixel block fits; for those, the block
+    // shape (Ht rows x Wbox columns, Wbox a multiple of 8 so a block is whole 1024-byte
+    // swizzle atoms) with the least padding, preferring three or more pipeline stages
+    bool found = false;
+    for (int a_per = a_max; a_per >= 1 && !found; --a_per) {
+        double best = 1e30;
+        const int wcand[2] = {(s.Wo + 7) / 8 * 8, (s.Wo + 15) / 16 * 16};
+        for (int wc = 0; wc < 2; ++wc) {
+            const int Wbox = wcand[wc];
+            if (Wbox > 256) continue;
+            for (int Ht = 1; Ht <= 8; ++Ht) {
+                const int P = Wbox * Ht;
+                if (P % 16 != 0 || P > 256) continue;
+                const long long stage =
+                    static_cast<long long>(2 * a_per + q.nyb) * P * dwk::BOX_ROW;
+                long long stages =
+                    (DW_SMEM_MAX - 1024 - dwk::BAR_BYTES - dwk::tail_bytes(P)) / stage;
+                if (stages > dwk::MAX_STAGES) stages = dwk::MAX_STAGES;
+                if (stages < 2) continue;
+                const int rb = (s.Ho + Ht - 1) / Ht;
+                double score = static_cast<double>(P) * rb / (static_cast<double>(s.Wo) * s.Ho);
+                if (stages < 3) score *= 1.15;
+                if (P < 32) score *= 1.2;
+                if (score < best) {
+                    best = score;
+                    q.a_per = a_per;
+                    q.Wbox = Wbox; q.Ht = Ht; q.P = P; q.rblocks = rb;
+                    q.stages = static_cast<int>(stages);
+                    q.stage_bytes = static_cast<uint32_t>(stage);
+                }
+            }
+        }
+        found = best < 1e29;
+    }
+    if (!found) return false;
+    q.pair_groups = (q.npairs + q.a_per - 1) / q.a_per;
+    q.groups = q.pair_groups * (s.Cout / q.ncols);
+    q.kblocks = static_cast<long long>(s.N) * q.rblocks;
+    long long splits = num_sms / q.groups;
+    if (splits < 1) splits = 1;
+    if (splits > q.kblocks) splits = q.kblocks;
+    q.splits = static_cast<int>(splits);
+    if (static_cast<long long>(q.groups) * q.splits > 0x7fffffffLL) return false;
+    uint32_t cols = 32;
+    while (cols < static_cast<uint32_t>(q.a_per * q.ncols)) cols <<= 1;
+    q.tmem_cols = cols;
+    *p = q;
+    return true;
+}
+
+// [N][H][W][C] bf16, boxes of 64 channels x Wbox columns x Ht rows of one image, SW128.
+bool encode_dw_map(CUtensorMap* map, const void* t, int C, int W, int H, int N, int Wbox,
+                   int Ht) {
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(C), static_cast<cuuint64_t>(W),
+                                static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(N)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(C) * 2,
+                                   static_cast<cuuint64_t>(C) * 2 * W,
+                                   static_cast<cuuint64_t>(C) * 2 * W * H};
+    const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(Wbox), static_cast<cuuint32_t>(Ht), 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = g_encode_tiled(
+        map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(t), dims, strides, box, estr,
+        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
@@ -954,6 +1040,51 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
 #undef QUAN_TC_CASE
     snprintf(err, errlen, "no kernel instance for kappa=%d bnq=%d mode=%d", kappa, bnq, mode);
     return cudaErrorInvalidValue;
+}
+
+bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy) {
+    dwk::DwParams p;
+    return dw_plan(s, 152, &p) && reinterpret_cast<uintptr_t>(x) % 16 == 0 &&
+           reinterpret_cast<uintptr_t>(dy) % 16 == 0;
+}
+
+cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* dy,
+                                 float* const dw[4], int num_sms,
+                                 unsigned long long wait_limit_ns, cudaStream_t stream,
+                                 char* err, size_t errlen) {
+    dwk::DwParams p;
+    if (!dw_plan(s, num_sms, &p) || !bwd_weight_tc_supported(s, x, dy)) {
+        snprintf(err, errlen, "no tensor-core weight-gradient tiling for this shape");
+        return cudaErrorInvalidValue;
+    }
+    if (!load_encoders()) {
+        snprintf(err, errlen, "cuTensorMapEncodeTiled is not available");
+        return cudaErrorInvalidValue;
+    }
+    CUtensorMap mx, mdy;
+    if (!encode_dw_map(&mx, x, s.Cin, s.W, s.H, s.N, p.Wbox, p.Ht) ||
+        !encode_dw_map(&mdy, dy, s.Cout, s.Wo, s.Ho, s.N, p.Wbox, p.Ht)) {
+        snprintf(err, errlen, "tensor-map encode failed for the weight gradient");
+        return cudaErrorInvalidValue;
+    }
+    const size_t bytes = static_cast<size_t>(s.Qout) * s.kh * s.kw * s.Qin * sizeof(float);
+    for (int L = 0; L < 4; ++L) {
+        cudaError_t e = cudaMemsetAsync(dw[L], 0, bytes, stream);
+        if (e != cudaSuccess) return e;
+    }
+    p.wait_limit_ns = wait_limit_ns;
+    p.dwr = dw[0];
+    p.dwi = dw[1];
+    p.dwj = dw[2];
+    p.dwk = dw[3];
+    const int smem = p.stages * static_cast<int>(p.stage_bytes) + dwk::BAR_BYTES +
+                     dwk::tail_bytes(p.P) + 1024;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(dwk::qconv_dw_kernel, DW_SMEM_MAX, attr_done);
+    if (e != cudaSuccess) return e;
+    set_kernel_name("qconv_dw_kernel<pairs=%d,n=%d>", p.a_per, p.ncols);
+    return launch_pdl(dwk::qconv_dw_kernel, dim3(static_cast<unsigned>(p.groups * p.splits)),
+                      dim3(dwk::THREADS), static_cast<size_t>(smem), stream, mx, mdy, p);
 }
 
 const char* last_tc_kernel() { return t_kernel_name; }

@@ -287,12 +287,31 @@ quan_status_t run_bwd_weight(const void* x, const void* dy, int N, int H, int W,
         if (reinterpret_cast<uintptr_t>(dw[L]) % 4 != 0)
             return fail(QUAN_ERR_INVALID_ARG, "weight gradients must be 4-byte aligned");
     }
-    if (g_path.load() == QUAN_PATH_TC)
-        return fail(QUAN_ERR_UNSUPPORTED, "the weight gradient runs on CUDA cores only");
+    // tensor cores for the full form at stride 1 (the shape checks need no device)
+    const bool tc_shape = !separable && quan::bwd_weight_tc_supported(s, x, dy);
+    const int path = g_path.load();
+    if (path == QUAN_PATH_TC && !tc_shape)
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "tensor-core weight gradient needs the full form, stride 1, Cin and Cout "
+                    "multiples of 64 (Cout <= 256 or a multiple of 256) and 16-byte aligned x "
+                    "and dy");
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
-    e = quan::launch_bwd_weight_simt(s, x, dy, dw, num_sms, reinterpret_cast<cudaStream_t>(stream));
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    if (path == QUAN_PATH_TC && cc != 103)
+        return fail(QUAN_ERR_UNSUPPORTED, "tensor-core weight gradient needs sm_103 (cc %d)", cc);
+    if (tc_shape && cc == 103 && path != QUAN_PATH_SIMT) {
+        char err[256] = "";
+        e = quan::launch_bwd_weight_tc(s, x, dy, dw, num_sms, g_wait_limit.load(), cs, err,
+                                       sizeof(err));
+        if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+        if (e != cudaSuccess) return cuda_fail(e, "qconv_dw launch");
+        t_last_path = QUAN_PATH_TC;
+        t_last_kernel = quan::last_tc_kernel();
+        return QUAN_OK;
+    }
+    e = quan::launch_bwd_weight_simt(s, x, dy, dw, num_sms, cs);
     if (e != cudaSuccess) return cuda_fail(e, "bwd_weight_simt launch");
     t_last_path = QUAN_PATH_SIMT;
     t_last_kernel = separable ? "bwd_weight_simt_kernel<sep>" : "bwd_weight_simt_kernel";

@@ -56,8 +56,9 @@ def gpu_bwd_data(d, separable=False, path=quan.QUAN_PATH_AUTO):
     return out_f64(dx), quan.quan_last_path(), quan.quan_last_kernel()
 
 
-def gpu_bwd_weight(d, separable=False):
+def gpu_bwd_weight(d, separable=False, path=quan.QUAN_PATH_AUTO):
     spec = d["spec"]
+    quan.quan_set_path(path)
     x, dy = to_dev(d["x"], "bf16"), to_dev(d["dy"], "bf16")
     # the outputs start as garbage: the call zeroes them itself
     out = tuple(torch.full((spec.Cout // 4, spec.kh, spec.kw, spec.Cin // 4), 7.0,
@@ -83,12 +84,24 @@ def oracle_bwd_weight(d, separable=False):
               stride=spec.stride, pad=spec.pad)
 
 
-def check_weight(d, separable=False):
-    got, kernel = gpu_bwd_weight(d, separable)
-    assert kernel == ("bwd_weight_simt_kernel<sep>" if separable else "bwd_weight_simt_kernel")
+def tc_weight_shape(spec):
+    return (spec.stride == 1 and spec.Cin % 64 == 0 and spec.Cout % 64 == 0 and
+            (spec.Cout <= 256 or spec.Cout % 256 == 0))
+
+
+def check_weight(d, separable=False, path=quan.QUAN_PATH_AUTO):
+    got, kernel = gpu_bwd_weight(d, separable, path)
+    spec = d["spec"]
+    if separable:
+        assert kernel == "bwd_weight_simt_kernel<sep>"
+    elif path != quan.QUAN_PATH_SIMT and tc_weight_shape(spec):
+        assert kernel.startswith("qconv_dw_kernel<"), kernel
+    else:
+        assert kernel == "bwd_weight_simt_kernel", kernel
     ref = oracle_bwd_weight(d, separable)
     for L in range(4):
-        assert_f32_close(got[L], ref[L], "%s dW[%d]" % (d["spec"].name, L))
+        assert_f32_close(got[L], ref[L], "%s dW[%d] (%s)" % (spec.name, L, kernel))
+    return got
 
 
 TC_CASES = [
@@ -188,6 +201,36 @@ def test_bwd_weight(case):
     name, N, H, W, Cin, Cout, k, s, p = case
     check_weight(layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p,
                                           seed=(607, len(name)))))
+
+
+TC_WEIGHT_CASES = [
+    # name, N, H, W, Cin, Cout, k, stride, pad: the tensor-core weight gradient
+    ("dw_odd_units", 2, 13, 11, 64, 64, 3, 1, 1),    # 9 taps: the last unit pair repeats
+    ("dw_cout128", 2, 12, 10, 64, 128, 3, 1, 1),
+    ("dw_cin256", 1, 9, 13, 256, 64, 3, 1, 1),       # 8 unit pairs per CTA, 3 pair groups
+    ("dw_c192", 1, 7, 9, 192, 192, 3, 1, 1),
+    ("dw_pointwise", 2, 10, 9, 128, 256, 1, 1, 0),
+    ("dw_pad0", 2, 11, 12, 64, 128, 3, 1, 0),
+    ("dw_k5", 1, 12, 11, 64, 64, 5, 1, 2),
+    ("dw_cout512", 1, 6, 7, 64, 512, 3, 1, 1),       # two output-channel groups
+    ("dw_tiny", 1, 1, 1, 64, 64, 3, 1, 1),
+    ("dw_wide_row", 1, 3, 200, 64, 64, 3, 1, 1),     # 200 columns: one row per block
+]
+
+
+@pytest.mark.parametrize("case", TC_WEIGHT_CASES, ids=[c[0] for c in TC_WEIGHT_CASES])
+def test_bwd_weight_tensor_cores(case):
+    name, N, H, W, Cin, Cout, k, s, p = case
+    d = layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(610, len(name))))
+    check_weight(d, path=quan.QUAN_PATH_TC)
+
+
+def test_bwd_weight_paths_agree():
+    d = layer(inputs.small_layer("dw_both", 2, 9, 10, 64, 128, 3, 1, 1, seed=(611, 0)))
+    tc = check_weight(d, path=quan.QUAN_PATH_TC)
+    simt = check_weight(d, path=quan.QUAN_PATH_SIMT)
+    for L in range(4):
+        assert_f32_close(tc[L], simt[L], "tc vs simt dW[%d]" % L)
 
 
 SEP_CASES = [
