@@ -200,12 +200,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc_fence_after();
         if (ok && !*abort_flag) {
             const int row = 32 * q + lane;  // x channel within the unit pair
+            const long long wstride = static_cast<long long>(p.taps) * p.Qin;  // one co step
             for (int a = 0; a < npair; ++a) {
                 const int u = 2 * (pair0 + a) + row / 64;
                 const bool live = u < p.units;  // the repeated last unit is not written
                 const int tap = (live ? u : 0) / p.nxc;
                 const int c = ((live ? u : 0) - tap * p.nxc) * 64 + row % 64;
                 const int pc = c / p.Qin, ci = c - pc * p.Qin;
+                const long long row_off = static_cast<long long>(tap) * p.Qin + ci;
                 for (int j0 = 0; j0 < p.ncols; j0 += 32) {
                     uint32_t v[32];
                     tmem_ld_32x32b_x32(
@@ -214,16 +216,19 @@ __global__ void __launch_bounds__(THREADS, 1)
                         v);
                     tmem_ld_wait();
                     if (!live) continue;
+                    // 16 columns never straddle two output components (Qout is a multiple
+                    // of 16): letter, sign and base address are fixed per half
 #pragma unroll
-                    for (int jj = 0; jj < 32; ++jj) {
-                        const int d = cg * p.ncols + j0 + jj;
-                        const int m = d / p.Qout, co = d - m * p.Qout;
-                        const int L = m ^ pc;
-                        float val = __uint_as_float(v[jj]);
-                        if ((NEG_MASK >> (4 * m + pc)) & 1u) val = -val;
-                        atomicAdd(letter_ptr(p, L) +
-                                      (static_cast<long long>(co) * p.taps + tap) * p.Qin + ci,
-                                  val);
+                    for (int h = 0; h < 2; ++h) {
+                        const int d0 = cg * p.ncols + j0 + 16 * h;
+                        const int m = d0 / p.Qout, co0 = d0 - m * p.Qout;
+                        const bool neg = (NEG_MASK >> (4 * m + pc)) & 1u;
+                        float* dst = letter_ptr(p, m ^ pc) + co0 * wstride + row_off;
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) {
+                            const float val = __uint_as_float(v[16 * h + jj]);
+                            atomicAdd(dst + jj * wstride, neg ? -val : val);
+                        }
                     }
                 }
             }
