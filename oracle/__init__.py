@@ -21,6 +21,8 @@ Passages followed (Grant & Wang, arXiv 2509.05512):
   * separable backward .......... Eq. 8-10 (Sec. III-B): mixing matrix M of Eq. 9,
                                   then per-component convolution gradients
   * IQBN, inference form ........ Eq. 11-12 (Sec. III-C), folded to scale/shift
+  * IQBN, training mode ......... Eq. 11 batch statistics (biased variance), Eq. 12
+                                  normalisation and affine
   * component-wise pooling ...... QSPPF (Sec. III-D)
 """
 from __future__ import annotations
@@ -87,6 +89,12 @@ def _load():
             lib.oracle_qconv2d_sep_bwd_weight.argtypes = ([_dp] * 2 + [ctypes.c_int] * 9 +
                                                           [_dp] * 4)
             lib.oracle_qconv2d_sep_bwd_weight.restype = ctypes.c_int
+            lib.oracle_iqbn_batch_stats.argtypes = [_dp, ctypes.c_longlong, ctypes.c_int, _dp,
+                                                    _dp]
+            lib.oracle_iqbn_batch_stats.restype = ctypes.c_int
+            lib.oracle_iqbn_train.argtypes = [_dp, ctypes.c_longlong, ctypes.c_int, _dp, _dp,
+                                              ctypes.c_double, ctypes.c_int, _dp]
+            lib.oracle_iqbn_train.restype = ctypes.c_int
             lib.oracle_poincare.argtypes = [_dp, ctypes.c_longlong, _dp]
             lib.oracle_poincare.restype = None
             lib.oracle_num_threads.argtypes = []
@@ -296,6 +304,30 @@ def qconv2d_sep_bwd_weight(x, dy, *, kh, kw, stride=1, pad=0):
     if rc != 0:
         raise ValueError("oracle_qconv2d_sep_bwd_weight: invalid arguments")
     return tuple(dw)
+
+
+def iqbn_batch_stats(x):
+    """Batch statistics of Eq. 11 per real channel: x [..., C] -> (mean, biased var), each
+    [C], over every leading index (N, H, W)."""
+    x = _f64(x)
+    C = x.shape[-1]
+    npix = x.size // C
+    mean, var = np.zeros(C), np.zeros(C)
+    if _load().oracle_iqbn_batch_stats(_ptr(x), npix, C, _ptr(mean), _ptr(var)) != 0:
+        raise ValueError("oracle_iqbn_batch_stats: invalid arguments")
+    return mean, var
+
+
+def iqbn_train(x, gamma, beta, *, eps=1e-5, act=ACT_NONE):
+    """Training-mode IQBN (Eq. 11-12) with the batch's own statistics, then the split
+    activation: x [..., C] -> same shape."""
+    x, gamma, beta = map(_f64, (x, gamma, beta))
+    C = x.shape[-1]
+    y = np.zeros_like(x)
+    if _load().oracle_iqbn_train(_ptr(x), x.size // C, C, _ptr(gamma), _ptr(beta), float(eps),
+                                 act, _ptr(y)) != 0:
+        raise ValueError("oracle_iqbn_train: invalid arguments")
+    return y
 
 
 def poincare(rgb) -> np.ndarray:

@@ -26,6 +26,7 @@
  *   - activations are split (elementwise per real component).
  */
 #include <math.h>
+#include <stdlib.h>
 #include <stddef.h>
 #include <stdint.h>
 #include <string.h>
@@ -503,6 +504,56 @@ int oracle_qconv2d_sep_bwd_weight(const double *x, const double *dy, int N, int 
                     const size_t widx = (((size_t)co * kh + dh) * kw + dw) * Qin + ci;
                     for (int p = 0; p < 4; ++p) dwl[p][widx] = acc[p];
                 }
+    return 0;
+}
+
+/* ---------------------------------------------------------------- IQBN, training mode
+ * Batch statistics of Eq. 11 (Sec. III-C), one real channel at a time: over the N H W
+ * values of channel c (one component of one quaternion channel),
+ *     mu_c = E[x_c],   sigma2_c = E[(x_c - mu_c)^2]      (two passes, biased variance).
+ * x is [npix][C] (NHWC flattened).  Returns 0, or -1 on invalid arguments. */
+int oracle_iqbn_batch_stats(const double *x, long long npix, int C, double *mean,
+                            double *var) {
+    if (!x || !mean || !var || npix < 1 || C < 1) return -1;
+#pragma omp parallel for schedule(static)
+    for (int c = 0; c < C; ++c) {
+        double s = 0.0;
+        for (long long p = 0; p < npix; ++p) s += x[(size_t)p * C + c];
+        const double mu = s / (double)npix;
+        double s2 = 0.0;
+        for (long long p = 0; p < npix; ++p) {
+            const double d = x[(size_t)p * C + c] - mu;
+            s2 += d * d;
+        }
+        mean[c] = mu;
+        var[c] = s2 / (double)npix;
+    }
+    return 0;
+}
+
+/* Training-mode IQBN output of Eq. 11-12: x_hat = (x - mu) / sqrt(sigma2 + eps) with the
+ * batch statistics above, then x_hat * gamma + beta per real channel, then the split
+ * activation.  Returns 0 or -1. */
+int oracle_iqbn_train(const double *x, long long npix, int C, const double *gamma,
+                      const double *beta, double eps, int act, double *y) {
+    if (!x || !gamma || !beta || !y || npix < 1 || C < 1 || eps < 0.0) return -1;
+    if (act < ACT_NONE || act > ACT_SILU) return -1;
+    double *mean = (double *)malloc(sizeof(double) * (size_t)C);
+    double *var = (double *)malloc(sizeof(double) * (size_t)C);
+    if (!mean || !var) {
+        free(mean);
+        free(var);
+        return -1;
+    }
+    oracle_iqbn_batch_stats(x, npix, C, mean, var);
+#pragma omp parallel for schedule(static)
+    for (long long p = 0; p < npix; ++p)
+        for (int c = 0; c < C; ++c) {
+            const double xh = (x[(size_t)p * C + c] - mean[c]) / sqrt(var[c] + eps);
+            y[(size_t)p * C + c] = apply_act(xh * gamma[c] + beta[c], act);
+        }
+    free(mean);
+    free(var);
     return 0;
 }
 

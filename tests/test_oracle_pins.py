@@ -378,3 +378,69 @@ def test_separable_backward_matches_torch_gradients(case):
         np.testing.assert_allclose(dw[comp], ref_dw.permute(0, 2, 3, 1).numpy(), rtol=1e-12,
                                    atol=1e-12)
 
+
+
+# ----------------------------------------------------------------- IQBN, training mode
+# Eq. 11: per real channel, mu = E[x], sigma^2 = E[(x - mu)^2] over N, H, W; Eq. 12: the
+# normalised value times gamma plus beta.
+
+def test_iqbn_stats_hand_example():
+    # channel 0: 1, 2, 3, 6 -> mu = 12 / 4 = 3, sigma^2 = (4 + 1 + 0 + 9) / 4 = 3.5;
+    # channel 1: constant -2 -> mu = -2, sigma^2 = 0
+    x = np.array([[1.0, -2.0], [2.0, -2.0], [3.0, -2.0], [6.0, -2.0]]).reshape(2, 1, 2, 2)
+    mean, var = oracle.iqbn_batch_stats(x)
+    np.testing.assert_array_equal(mean, [3.0, -2.0])
+    np.testing.assert_array_equal(var, [3.5, 0.0])
+
+
+def test_iqbn_stats_large_offset_is_exact():
+    # 1e6 + (0, 1, 2, 3): mu = 1e6 + 1.5, sigma^2 = 1.25 exactly (two-pass definition; the
+    # one-pass E[x^2] - mu^2 loses every digit here)
+    x = (1e6 + np.arange(4.0)).reshape(4, 1)
+    mean, var = oracle.iqbn_batch_stats(x)
+    assert mean[0] == 1e6 + 1.5 and var[0] == 1.25
+
+
+def test_iqbn_stats_affine_and_channel_independence():
+    rng = np.random.default_rng(50)
+    x = rng.standard_normal((3, 5, 4, 8))
+    mean, var = oracle.iqbn_batch_stats(x)
+    a = np.linspace(-2.0, 3.0, 8)
+    b = np.linspace(5.0, -1.0, 8)
+    m2, v2 = oracle.iqbn_batch_stats(a * x + b)
+    np.testing.assert_allclose(m2, a * mean + b, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(v2, a * a * var, rtol=1e-12, atol=1e-14)
+    y = x.copy()
+    y[..., 3] *= 7.0
+    m3, v3 = oracle.iqbn_batch_stats(y)
+    keep = np.arange(8) != 3
+    np.testing.assert_array_equal(m3[keep], mean[keep])
+    np.testing.assert_array_equal(v3[keep], var[keep])
+
+
+def test_iqbn_train_normalised_moments():
+    # gamma = 1, beta = 0: every channel of the output has mean 0 and mean square
+    # sigma^2 / (sigma^2 + eps); with gamma, beta the output is their affine image
+    rng = np.random.default_rng(51)
+    x = rng.standard_normal((2, 6, 5, 12)) * np.linspace(0.1, 4.0, 12) + np.linspace(-3, 3, 12)
+    eps = 1e-3
+    ones, zeros = np.ones(12), np.zeros(12)
+    xh = oracle.iqbn_train(x, ones, zeros, eps=eps)
+    _, var = oracle.iqbn_batch_stats(x)
+    np.testing.assert_allclose(xh.reshape(-1, 12).mean(0), 0.0, atol=1e-12)
+    np.testing.assert_allclose((xh ** 2).reshape(-1, 12).mean(0), var / (var + eps), rtol=1e-12)
+    g, b = np.linspace(0.5, 1.5, 12), np.linspace(-0.2, 0.2, 12)
+    np.testing.assert_allclose(oracle.iqbn_train(x, g, b, eps=eps), xh * g + b, rtol=1e-12,
+                               atol=1e-12)
+
+
+def test_iqbn_train_constant_channel_and_activations():
+    # a constant channel normalises to 0, so the output is act(beta)
+    x = np.full((4, 3), 2.5)
+    g, b = np.array([1.3, 0.7, 2.0]), np.array([-0.5, 0.25, 1.0])
+    np.testing.assert_array_equal(oracle.iqbn_train(x, g, b), np.broadcast_to(b, (4, 3)))
+    np.testing.assert_array_equal(oracle.iqbn_train(x, g, b, act=oracle.ACT_RELU),
+                                  np.broadcast_to([0.0, 0.25, 1.0], (4, 3)))
+    silu = b / (1.0 + np.exp(-b))
+    np.testing.assert_allclose(oracle.iqbn_train(x, g, b, act=oracle.ACT_SILU)[0], silu,
+                               rtol=1e-15)
