@@ -42,7 +42,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c1",
-                    choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone", "poincare"])
+                    choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone", "poincare", "iqbn"])
     ap.add_argument("--pass", dest="direction", choices=["fwd", "bwd"], default="fwd",
                     help="layer workloads: the forward convolution, or its backward pass "
                          "(input and weight gradients before the epilogue, from a seeded "
@@ -517,9 +517,135 @@ WORKLOAD_DESC = {
     "c3b": "detection-neck 3x3 layer",
     "backbone": "ResNet-18-style QUAN backbone",
     "poincare": "Poincare RGB -> quaternion input mapping (Eq. 4)",
+    "iqbn": "training-mode IQBN (Eq. 11-12): batch statistics, then normalisation + ReLU",
 }
 
 POINCARE_SHAPE = (256, 224, 224)  # the backbone's input batch: N, H, W
+IQBN_SHAPE = (64, 56, 56, 256)    # the ImageNet-stage layer's output: N, H, W, C
+
+
+class IqbnRunner:
+    """Training-mode IQBN of one activation tensor (bf16 NHWC): quan_iqbn_batch_stats, then
+    quan_iqbn_train_fwd with ReLU into a separate output, on rotating buffer sets larger
+    than L2."""
+
+    def __init__(self, torch, quan, inputs, N, H, W, C):
+        import numpy as np
+        self.torch, self.quan, self.N, self.C = torch, quan, N, C
+        self.npix = N * H * W
+        rng = np.random.default_rng(45)
+        x = rng.standard_normal((N, H, W, C), dtype=np.float32) + np.float32(0.5)
+        self.host_x = inputs.to_bf16_bits(x)
+        self.host_gamma = rng.uniform(0.5, 1.5, C).astype(np.float32)
+        self.host_beta = (rng.standard_normal(C, dtype=np.float32) * np.float32(0.1))
+        x0 = torch.from_numpy(self.host_x.view(np.int16)).view(torch.bfloat16).cuda()
+        per_set = self.npix * C * 4  # x and out
+        self.sets = max(2, min(8, math.ceil(2 * L2_BYTES / per_set)))
+        self.xs = [x0] + [x0.clone() for _ in range(self.sets - 1)]
+        self.outs = [torch.empty_like(x0) for _ in range(self.sets)]
+        self.gamma = torch.from_numpy(self.host_gamma).cuda()
+        self.beta = torch.from_numpy(self.host_beta).cuda()
+        self.mean = torch.empty(C, dtype=torch.float32, device="cuda")
+        self.var = torch.empty(C, dtype=torch.float32, device="cuda")
+        self.ws_bytes = quan.quan_iqbn_batch_stats_workspace_size(C)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device="cuda")
+        self.i = 0
+        self.launches_per_step = 3  # statistics, finalisation, normalisation
+        self.footprint = per_set * self.sets
+        self.flops = 0.0
+        self.stats_bytes = float(self.npix * C * 2)      # x read once
+        self.apply_bytes = float(self.npix * C * 4)      # x read, out written
+        self.algorithmic_bytes = self.stats_bytes + self.apply_bytes
+        self.separable = False
+
+    def stats(self, k, stream):
+        self.quan.quan_iqbn_batch_stats(self.xs[k], self.npix, self.C, self.ws, self.ws_bytes,
+                                        self.mean, self.var, stream)
+
+    def apply(self, k, stream):
+        self.quan.quan_iqbn_train_fwd(self.xs[k], self.npix, self.C, self.mean, self.var,
+                                      self.gamma, self.beta, 1e-5, self.quan.QUAN_ACT_RELU,
+                                      self.outs[k], stream)
+
+    def step(self, stream):
+        k = self.i % self.sets
+        self.i += 1
+        self.stats(k, stream)
+        self.apply(k, stream)
+
+    def kernel_times(self, torch, stream, reps=5):
+        sh = stream.cuda_stream
+        out = []
+        for fn in (self.stats, self.apply):
+            for k in range(2):
+                fn(k % self.sets, sh)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for r in range(reps):
+                fn(r % self.sets, sh)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            out.append(e0.elapsed_time(e1) / reps / 1e3)
+        return out
+
+    def e2e_setup(self):
+        torch = self.torch
+        import numpy as np
+        self.h_in = torch.from_numpy(self.host_x.view(np.int16).reshape(-1)).pin_memory()
+        self.h_out = [torch.empty(self.npix * self.C, dtype=torch.int16).pin_memory()
+                      for _ in range(E2E_BUFFERS)]
+        self.e_in = [torch.empty_like(self.h_in, device="cuda") for _ in range(E2E_BUFFERS)]
+        self.e_out = [torch.empty_like(t, device="cuda") for t in self.h_out]
+        self.h2d = self.npix * self.C * 2
+        self.d2h = self.npix * self.C * 2
+
+    def e2e_in(self, b):
+        return [(self.e_in[b], self.h_in)]
+
+    def e2e_out(self, b):
+        return [(self.h_out[b], self.e_out[b])]
+
+    def e2e_compute(self, b, stream):
+        q = self.quan
+        q.quan_iqbn_batch_stats(self.e_in[b], self.npix, self.C, self.ws, self.ws_bytes,
+                                self.mean, self.var, stream)
+        q.quan_iqbn_train_fwd(self.e_in[b], self.npix, self.C, self.mean, self.var, self.gamma,
+                              self.beta, 1e-5, q.QUAN_ACT_RELU, self.e_out[b], stream)
+
+
+def iqbn_roofline(runner, torch, stream, peaks, peak_src):
+    """HBM roofline of the slower of the two kernels, timed apart with events."""
+    t_stats, t_apply = runner.kernel_times(torch, stream)
+    rows = [{"kernel": "iqbn_stats_kernel (+ finalize)", "ms": round(t_stats * 1e3, 4),
+             "achieved": round(runner.stats_bytes / t_stats / 1e9, 1)},
+            {"kernel": "iqbn_apply_kernel", "ms": round(t_apply * 1e3, 4),
+             "achieved": round(runner.apply_bytes / t_apply / 1e9, 1)}]
+    for r in rows:
+        r["frac"] = round(r["achieved"] / peaks["hbm_gbs"], 4)
+    top = max(rows, key=lambda r: r["ms"])
+    return {"bound": "hbm", "achieved": top["achieved"], "peak": peaks["hbm_gbs"],
+            "unit": "GB/s", "frac": top["frac"],
+            "traffic": recorded_traffic("iqbn", top["kernel"].split()[0]),
+            "kernel": top["kernel"], "share": round(top["ms"] / (rows[0]["ms"] + rows[1]["ms"]), 3),
+            "peak_source": peak_src + " (burst)", "kernels": rows}
+
+
+def iqbn_cpu_sample(runner, seconds):
+    """The fp64 oracle's training-mode IQBN on a bounded number of images of the batch."""
+    import oracle
+    f64 = oracle.bf16_bits_to_f64
+    g, b = runner.host_gamma.astype("float64"), runner.host_beta.astype("float64")
+    t0 = time.perf_counter()
+    oracle.iqbn_train(f64(runner.host_x[:1]), g, b, act=oracle.ACT_RELU)
+    t1 = max(time.perf_counter() - t0, 1e-6)
+    n = max(1, min(runner.N, int(seconds / t1)))
+    x = f64(runner.host_x[:n])
+    t0 = time.perf_counter()
+    oracle.iqbn_train(x, g, b, act=oracle.ACT_RELU)
+    t = time.perf_counter() - t0
+    return {"value": n / t, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": "statistics and normalisation of %d of %d images of the batch (fp64, "
+                      "%.2f s)" % (n, runner.N, t)}
 
 
 class PoincareRunner:
@@ -594,6 +720,10 @@ def workload_config(workload: str, inputs, variant: str = "full", direction: str
         return {"workload": "%s, N=%d, %dx%d fp32 RGB -> bf16 quaternion pixels" % (
                     WORKLOAD_DESC[workload], N, H, W), "N": N, "H": H, "W": W,
                 "bytes_per_step": N * H * W * 20}
+    if workload == "iqbn":
+        N, H, W, C = IQBN_SHAPE
+        return {"workload": "%s, N=%d, %dx%d, C=%d bf16" % (WORKLOAD_DESC[workload], N, H, W, C),
+                "N": N, "H": H, "W": W, "C": C, "bytes_per_step": N * H * W * C * 6}
     if workload == "backbone":
         layers = inputs.backbone_layers()
         convs = [L.spec for L in layers if L.kind == "conv"]
@@ -660,12 +790,15 @@ def main():
 
     if args.batch and not args.profile:
         raise SystemExit("--batch is for --profile runs only")
-    if args.workload in ("backbone", "poincare") and (args.variant != "full" or
+    if args.workload in ("backbone", "poincare", "iqbn") and (args.variant != "full" or
                                                        args.direction != "fwd"):
         raise SystemExit("--variant and --pass apply to the convolution layer workloads")
     if args.workload == "poincare":
         runner = PoincareRunner(torch, quan, *POINCARE_SHAPE)
         unit, per_step_units, dtype = "images/s", runner.N, "f32->bf16"
+    elif args.workload == "iqbn":
+        runner = IqbnRunner(torch, quan, inputs, *IQBN_SHAPE)
+        unit, per_step_units, dtype = "images/s", runner.N, "bf16 (fp32 statistics)"
     elif args.workload == "backbone":
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256)
@@ -705,7 +838,7 @@ def main():
         if n % 64 == 0:
             torch.cuda.synchronize()
     torch.cuda.synchronize()
-    kernel_name = (None if args.workload == "backbone" else
+    kernel_name = (None if args.workload in ("backbone", "iqbn") else
                    "poincare_kernel" if args.workload == "poincare" else quan.quan_last_kernel())
 
     # The timed region is exactly K steps.  By default they are captured once into a CUDA
@@ -763,6 +896,8 @@ def main():
     peaks, peak_src = load_peaks()
     if args.workload == "backbone":
         roofline = backbone_roofline(runner, torch, stream, peaks, peak_src)
+    elif args.workload == "iqbn":
+        roofline = iqbn_roofline(runner, torch, stream, peaks, peak_src)
     elif args.direction == "bwd":
         roofline = bwd_roofline(runner, torch, stream, peaks, peak_src, traffic_key(args))
     else:
@@ -774,6 +909,8 @@ def main():
             cpu = backbone_cpu_sample(runner, args.cpu_seconds, inputs)
         elif args.workload == "poincare":
             cpu = poincare_cpu_sample(runner, args.cpu_seconds)
+        elif args.workload == "iqbn":
+            cpu = iqbn_cpu_sample(runner, args.cpu_seconds)
         elif args.direction == "bwd":
             cpu = cpu_bwd_sample(runner.spec, args.cpu_seconds, inputs,
                                  separable=runner.separable)
@@ -791,7 +928,7 @@ def main():
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
                 "timing": "one CUDA-graph replay of the K steps" if graph is not None
                 else "plain launch loop"})
-    if args.workload not in ("backbone", "poincare") and args.direction == "fwd":
+    if args.workload not in ("backbone", "poincare", "iqbn") and args.direction == "fwd":
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     if args.direction == "bwd":
         cfg["kernels"] = {"dx": runner.data_kernel, "dW": runner.weight_kernel}
@@ -918,6 +1055,31 @@ def reference_arm(args, rank, world, inputs):
                 "config": ref_cfg,
                 "cpu_baseline": {"value": value, "unit": "images/s", "cores": 1,
                                  "kind": "oracle",
+                                 "sample": "1 of %d images of the batch per step (fp64)" % N},
+                "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
+    if args.workload == "iqbn":
+        N, H, W, C = IQBN_SHAPE
+        import numpy as np
+        rng = np.random.default_rng(45)
+        x = rng.standard_normal((1, H, W, C)) + 0.5
+        g, b = rng.uniform(0.5, 1.5, C), rng.standard_normal(C) * 0.1
+        for _ in range(args.warmup):
+            oracle.iqbn_train(x, g, b, act=oracle.ACT_RELU)
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            oracle.iqbn_train(x, g, b, act=oracle.ACT_RELU)
+        dt = time.perf_counter() - t0
+        value = args.steps / dt
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",
+                "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": ref_cfg,
+                "cpu_baseline": {"value": value, "unit": "images/s",
+                                 "cores": oracle.num_threads(), "kind": "oracle",
                                  "sample": "1 of %d images of the batch per step (fp64)" % N},
                 "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}

@@ -13,7 +13,8 @@
  *   - component-wise max pooling (the QSPPF pooling rule of Sec. III-D);
  *   - the Poincare RGB mapping of Eq. 4 (Sec. III-A);
  *   - the separable form of Eq. 7 and its backward pass (Eq. 8-10), and the backward
- *     pass of the full form (input and weight gradients before the epilogue).
+ *     pass of the full form (input and weight gradients before the epilogue);
+ *   - IQBN in training mode: batch statistics (Eq. 11) and normalisation (Eq. 12).
  *
  * Conventions shared by every entry point
  *   Layout      x is NHWC [N][H][W][C_in]; the C_in real channels are four
@@ -234,6 +235,37 @@ quan_status_t quan_qconv2d_sep_bwd_weight(const void* x, const void* dy, int N, 
                                           int Cin, int Cout, int kh, int kw, int stride,
                                           int pad, float* dwr, float* dwi, float* dwj,
                                           float* dwk, quan_stream_t stream);
+
+/*
+ * Independent Quaternion Batch Normalization in training mode (Sec. III-C, Eq. 11-12):
+ * every real channel (one component of one quaternion channel) is normalised with its own
+ * statistics over the batch and the spatial positions.  x is bf16 [npix][C] (NHWC with
+ * npix = N H W), device.  The CUDA-core kernels take C a multiple of 8 up to 2048 with
+ * 16-byte aligned x (and out), or any C up to 256; other C return QUAN_ERR_UNSUPPORTED.
+ *
+ * quan_iqbn_batch_stats: mean[c] = E[x_c] and var[c] = E[(x_c - mean[c])^2] (the biased
+ * variance of Eq. 11; the unbiased running estimate is var * npix / (npix - 1)), fp32 [C]
+ * each, device, 4-byte aligned, disjoint from each other and from x.  `workspace` is
+ * device scratch of at least quan_iqbn_batch_stats_workspace_size(C) bytes (4-byte
+ * aligned, owned by the caller, overwritten; NULL or too small is QUAN_ERR_INVALID_ARG):
+ * one row of per-block partial sums, added in a fixed order, so repeated calls on the
+ * same input give the same bits.
+ */
+size_t quan_iqbn_batch_stats_workspace_size(int C);
+quan_status_t quan_iqbn_batch_stats(const void* x, long long npix, int C, void* workspace,
+                                    size_t workspace_bytes, float* mean, float* var,
+                                    quan_stream_t stream);
+
+/*
+ * quan_iqbn_train_fwd: out = act(gamma[c] (x - mean[c]) / sqrt(var[c] + eps) + beta[c])
+ * (Eq. 12 followed by the split activation), bf16 [npix][C], rounded to nearest even.
+ * mean and var are typically quan_iqbn_batch_stats' outputs; gamma and beta fp32 [C] or
+ * NULL (1 and 0).  out may be x itself (in place) but must not overlap it otherwise.
+ * eps must be finite and >= 0.
+ */
+quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const float* mean,
+                                  const float* var, const float* gamma, const float* beta,
+                                  float eps, int act, void* out, quan_stream_t stream);
 
 /*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,

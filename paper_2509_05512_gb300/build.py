@@ -14,7 +14,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libquan.so")
 SOURCES = ["quan_api.cu", "qconv_tc.cu", "qconv_simt.cu", "qconv_bwd.cu", "maxpool.cu",
-           "poincare.cu"]
+           "poincare.cu", "iqbn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -109,6 +109,19 @@ cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* 
 cudaError_t launch_bwd_weight_simt(const ConvShape& s, const void* x, const void* dy,
                                    float* const dw[4], int num_sms, cudaStream_t stream);
 
+// Training-mode IQBN (Eq. 11-12) over bf16 [npix][C].  The 16-byte vector path needs C a
+// multiple of 8 (at most 2048) and 16-byte aligned tensors; otherwise C <= 256.
+bool iqbn_vec_ok(int C, const void* a, const void* b);
+bool iqbn_supported(int C, const void* a, const void* b);
+// Partial sums of at most IQBN_MAX_PARTIALS blocks: workspace fp32 [blocks][2][C].
+constexpr int IQBN_MAX_PARTIALS = 1024;
+size_t iqbn_stats_workspace_bytes(int C);
+cudaError_t launch_iqbn_stats(const void* x, long long npix, int C, void* workspace,
+                              float* mean, float* var, int num_sms, cudaStream_t stream);
+cudaError_t launch_iqbn_apply(const void* x, long long npix, int C, const float* mean,
+                              const float* var, const float* gamma, const float* beta, float eps,
+                              int act, void* out, int num_sms, cudaStream_t stream);
+
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream);

@@ -5,6 +5,7 @@
 #include <atomic>
 #include <cstdarg>
 #include <cstdint>
+#include <cmath>
 #include <cstdio>
 #include <mutex>
 
@@ -466,6 +467,72 @@ quan_status_t quan_qconv2d_sep_bwd_weight(const void* x, const void* dy, int N, 
                                           float* dwk, quan_stream_t stream) {
     float* const dw[4] = {dwr, dwi, dwj, dwk};
     return run_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, true, dw, stream);
+}
+
+size_t quan_iqbn_batch_stats_workspace_size(int C) { return quan::iqbn_stats_workspace_bytes(C); }
+
+quan_status_t quan_iqbn_batch_stats(const void* x, long long npix, int C, void* workspace,
+                                    size_t workspace_bytes, float* mean, float* var,
+                                    quan_stream_t stream) {
+    if (!x || !mean || !var) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if (npix < 1 || C < 1) return fail(QUAN_ERR_INVALID_ARG, "npix and C must be >= 1");
+    if (npix > (1LL << 40) / C) return fail(QUAN_ERR_UNSUPPORTED, "tensor too large");
+    const size_t need = quan::iqbn_stats_workspace_bytes(C);
+    if (!workspace || workspace_bytes < need)
+        return fail(QUAN_ERR_INVALID_ARG, "workspace must hold %zu bytes (got %zu%s)", need,
+                    workspace_bytes, workspace ? "" : ", NULL");
+    if (reinterpret_cast<uintptr_t>(x) % 2 != 0 || reinterpret_cast<uintptr_t>(mean) % 4 != 0 ||
+        reinterpret_cast<uintptr_t>(var) % 4 != 0 ||
+        reinterpret_cast<uintptr_t>(workspace) % 4 != 0)
+        return fail(QUAN_ERR_INVALID_ARG,
+                    "x must be 2-byte, mean, var and the workspace 4-byte aligned");
+    const size_t xb = static_cast<size_t>(npix) * C * 2, vb = static_cast<size_t>(C) * 4;
+    if (overlaps(mean, vb, var, vb) || overlaps(mean, vb, x, xb) || overlaps(var, vb, x, xb) ||
+        overlaps(workspace, need, x, xb) || overlaps(workspace, need, mean, vb) ||
+        overlaps(workspace, need, var, vb))
+        return fail(QUAN_ERR_INVALID_ARG, "mean, var, the workspace and x must not overlap");
+    if (!quan::iqbn_supported(C, x, x))
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "C=%d: needs C <= 256, or C a multiple of 8 up to 2048 with x 16-byte "
+                    "aligned", C);
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    e = quan::launch_iqbn_stats(x, npix, C, workspace, mean, var, num_sms,
+                                reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "iqbn_stats launch");
+    return QUAN_OK;
+}
+
+quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const float* mean,
+                                  const float* var, const float* gamma, const float* beta,
+                                  float eps, int act, void* out, quan_stream_t stream) {
+    if (!x || !mean || !var || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if (npix < 1 || C < 1) return fail(QUAN_ERR_INVALID_ARG, "npix and C must be >= 1");
+    if (!(eps >= 0.0f) || !std::isfinite(eps))
+        return fail(QUAN_ERR_INVALID_ARG, "eps must be finite and >= 0");
+    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
+    if (npix > (1LL << 40) / C) return fail(QUAN_ERR_UNSUPPORTED, "tensor too large");
+    if (reinterpret_cast<uintptr_t>(x) % 2 != 0 || reinterpret_cast<uintptr_t>(out) % 2 != 0)
+        return fail(QUAN_ERR_INVALID_ARG, "x and out must be 2-byte aligned");
+    const size_t xb = static_cast<size_t>(npix) * C * 2, vb = static_cast<size_t>(C) * 4;
+    if (out != x && overlaps(out, xb, x, xb))
+        return fail(QUAN_ERR_INVALID_ARG, "out must be x itself or not overlap it");
+    if (overlaps(out, xb, mean, vb) || overlaps(out, xb, var, vb) ||
+        overlaps(out, xb, gamma, vb) || overlaps(out, xb, beta, vb))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps a per-channel vector");
+    if (!quan::iqbn_supported(C, x, out))
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "C=%d: needs C <= 256, or C a multiple of 8 up to 2048 with x and out "
+                    "16-byte aligned", C);
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    e = quan::launch_iqbn_apply(x, npix, C, mean, var, gamma, beta, eps, act, out, num_sms,
+                                reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "iqbn_apply launch");
+    return QUAN_OK;
 }
 
 quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,

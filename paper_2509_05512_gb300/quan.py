@@ -67,6 +67,12 @@ def load():
         _bwd_data_args = [_vp] * 5 + [_i] * 9 + [_vp, ctypes.c_size_t, _vp, _vp]
         lib.quan_qconv2d_bwd_data.argtypes = _bwd_data_args
         lib.quan_qconv2d_sep_bwd_data.argtypes = _bwd_data_args
+        lib.quan_iqbn_batch_stats.argtypes = [_vp, ctypes.c_longlong, _i, _vp, ctypes.c_size_t,
+                                              _vp, _vp, _vp]
+        lib.quan_iqbn_batch_stats_workspace_size.argtypes = [_i]
+        lib.quan_iqbn_batch_stats_workspace_size.restype = ctypes.c_size_t
+        lib.quan_iqbn_train_fwd.argtypes = ([_vp, ctypes.c_longlong, _i] + [_vp] * 4 +
+                                            [ctypes.c_float, _i, _vp, _vp])
         lib.quan_qconv2d_bwd_data_static.argtypes = [_vp] * 5 + [_i] * 9 + [_vp, _vp]
         lib.quan_qconv2d_bwd_data_workspace_size.argtypes = [_i] * 4
         lib.quan_qconv2d_bwd_data_workspace_size.restype = ctypes.c_size_t
@@ -91,7 +97,8 @@ def load():
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
                      "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
                      "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
-                     "quan_qconv2d_bwd_data_static",
+                     "quan_qconv2d_bwd_data_static", "quan_iqbn_batch_stats",
+                     "quan_iqbn_train_fwd",
                      "quan_qconv2d_sep_bwd_weight",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
@@ -336,6 +343,50 @@ def qconv2d_backward_weight(x, dy, *, kh, kw, stride=1, pad=0, separable=False, 
     fn = quan_qconv2d_sep_bwd_weight if separable else quan_qconv2d_bwd_weight
     fn(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, *out, stream)
     return out
+
+
+def quan_iqbn_batch_stats_workspace_size(C) -> int:
+    return load().quan_iqbn_batch_stats_workspace_size(C)
+
+
+def quan_iqbn_batch_stats(x, npix, C, workspace, workspace_bytes, mean, var,
+                          stream=None) -> None:
+    _check(load().quan_iqbn_batch_stats(_ptr(x), npix, C, _ptr(workspace), workspace_bytes,
+                                        _ptr(mean), _ptr(var), _stream(stream)))
+
+
+def quan_iqbn_train_fwd(x, npix, C, mean, var, gamma, beta, eps, act, out, stream=None) -> None:
+    _check(load().quan_iqbn_train_fwd(_ptr(x), npix, C, _ptr(mean), _ptr(var), _ptr(gamma),
+                                      _ptr(beta), eps, act, _ptr(out), _stream(stream)))
+
+
+def iqbn_batch_stats(x, *, workspace=None, stream=None):
+    """Eq. 11 on the GPU: bf16 x [..., C] (CUDA) -> (mean, biased var), fp32 [C] each.
+    `workspace` (a CUDA tensor of at least quan_iqbn_batch_stats_workspace_size(C) bytes)
+    is allocated when not given."""
+    import torch
+    C = x.shape[-1]
+    if workspace is None:
+        workspace = torch.empty(quan_iqbn_batch_stats_workspace_size(C), dtype=torch.uint8,
+                                device=x.device)
+    mean = torch.empty(C, dtype=torch.float32, device=x.device)
+    var = torch.empty(C, dtype=torch.float32, device=x.device)
+    quan_iqbn_batch_stats(x, x.numel() // C, C, workspace,
+                          workspace.numel() * workspace.element_size(), mean, var, stream)
+    return mean, var
+
+
+def iqbn_train(x, gamma=None, beta=None, *, eps=1e-5, act=QUAN_ACT_NONE, out=None,
+               stream=None):
+    """Training-mode IQBN (Eq. 11-12) with the batch's statistics, then the activation:
+    bf16 x [..., C] -> bf16, same shape; returns (out, mean, var)."""
+    import torch
+    mean, var = iqbn_batch_stats(x, stream=stream)
+    if out is None:
+        out = torch.empty_like(x)
+    C = x.shape[-1]
+    quan_iqbn_train_fwd(x, x.numel() // C, C, mean, var, gamma, beta, eps, act, out, stream)
+    return out, mean, var
 
 
 def maxpool2d(x, *, k=3, stride=2, pad=1, out=None, stream=None):

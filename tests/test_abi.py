@@ -157,3 +157,32 @@ def test_backward_weight_tensor_core_shapes(lib):
         assert _bwd_weight(lib, x=FAKE + 8) == quan.QUAN_ERR_UNSUPPORTED  # misaligned for TMA
     finally:
         assert lib.quan_set_path(quan.QUAN_PATH_AUTO) == quan.QUAN_OK
+
+
+def test_iqbn_entry_points_validate(lib):
+    st, tr = lib.quan_iqbn_batch_stats, lib.quan_iqbn_train_fwd
+    bad = quan.QUAN_ERR_INVALID_ARG
+    ws, wsb = 0x8000000, lib.quan_iqbn_batch_stats_workspace_size(64)
+    assert wsb == 1024 * 2 * 64 * 4 and lib.quan_iqbn_batch_stats_workspace_size(0) == 0
+    args = lambda **k: [k.get("x", FAKE), k.get("npix", 16), k.get("C", 64), k.get("ws", ws),
+                        k.get("wsb", wsb), k.get("mean", 0x7000000), k.get("var", 0x7100000),
+                        None]
+    assert st(*args(x=None)) == bad
+    assert st(*args(npix=0)) == bad
+    assert st(*args(C=0)) == bad
+    assert st(*args(ws=None)) == bad
+    assert st(*args(wsb=wsb - 1)) == bad
+    assert st(*args(var=0x7000000 + 8)) == bad          # mean overlaps var
+    assert st(*args(mean=FAKE + 64)) == bad             # mean overlaps x
+    assert st(*args(mean=0x7000002)) == bad             # misaligned mean
+    assert st(*args(ws=0x7100000 - 64)) == bad          # workspace overlaps var
+    assert st(*args(C=260, wsb=lib.quan_iqbn_batch_stats_workspace_size(260))) == \
+        quan.QUAN_ERR_UNSUPPORTED
+    v = (FAKE, 16, 64, 0x7000000, 0x7100000, None, None)
+    assert tr(*v, ctypes.c_float(1e-5), 7, 0x7200000, None) == bad      # unknown activation
+    assert tr(*v, ctypes.c_float(-1.0), 0, 0x7200000, None) == bad      # negative eps
+    assert tr(*v, ctypes.c_float(float("nan")), 0, 0x7200000, None) == bad
+    assert tr(*v, ctypes.c_float(1e-5), 0, FAKE + 2, None) == bad       # partial overlap
+    assert tr(*v, ctypes.c_float(1e-5), 0, 0x7000000, None) == bad      # out overlaps mean
+    assert tr(FAKE, 16, 260, 0x7000000, 0x7100000, None, None, ctypes.c_float(1e-5), 0,
+              0x7200000, None) == quan.QUAN_ERR_UNSUPPORTED
