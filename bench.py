@@ -50,6 +50,11 @@ def parse_args():
     ap.add_argument("--variant", choices=["full", "separable"], default="full",
                     help="layer workloads: the full Hamilton form (Eq. 5/6) or the separable "
                          "form of Eq. 7 (a quarter of the multiply-adds)")
+    ap.add_argument("--act", choices=["relu", "silu"], default="relu",
+                    help="backbone: the activation of its convolutions (ReLU as configured, "
+                         "or SiLU as in YOLO-style detectors)")
+    ap.add_argument("--no-fuse", action="store_true",
+                    help="backbone: run the stem and its max pool as two calls")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -713,7 +718,12 @@ def poincare_cpu_sample(runner, seconds):
             "sample": "%d of %d images of the batch (fp64, %.2f s)" % (n, runner.N, t)}
 
 
-def workload_config(workload: str, inputs, variant: str = "full", direction: str = "fwd") -> dict:
+def act_code(name: str) -> int:
+    return {"relu": 1, "silu": 2}[name]
+
+
+def workload_config(workload: str, inputs, variant: str = "full", direction: str = "fwd",
+                    act: str = "relu") -> dict:
     """The workload part of the JSON line's config, shared by both arms."""
     if workload == "poincare":
         N, H, W = POINCARE_SHAPE
@@ -725,14 +735,15 @@ def workload_config(workload: str, inputs, variant: str = "full", direction: str
         return {"workload": "%s, N=%d, %dx%d, C=%d bf16" % (WORKLOAD_DESC[workload], N, H, W, C),
                 "N": N, "H": H, "W": W, "C": C, "bytes_per_step": N * H * W * C * 6}
     if workload == "backbone":
-        layers = inputs.backbone_layers()
+        layers = inputs.backbone_layers(act=act_code(act))
         convs = [L.spec for L in layers if L.kind == "conv"]
         c0 = convs[0]
         return {"workload": "%s, N=%d, %dx%dx4 quaternion input" % (
                     WORKLOAD_DESC[workload], c0.N, c0.H, c0.W),
                 "N": c0.N, "H": c0.H, "W": c0.W, "convs": len(convs), "maxpool": 1,
                 "flops_per_step": sum(c.flops for c in convs),
-                "epilogue": "IQBN+ReLU (+residual)"}
+                "epilogue": "IQBN+%s (+residual)" % ("SiLU" if act == "silu" else "ReLU"),
+                "fusions": "stem conv + 3x3/2 max pool (horizontal max in the stem epilogue)"}
     s = inputs.LAYERS[workload]
     cfg = {"workload": WORKLOAD_DESC[workload], "N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin,
            "Cout": s.Cout, "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
@@ -793,6 +804,8 @@ def main():
     if args.workload in ("backbone", "poincare", "iqbn") and (args.variant != "full" or
                                                        args.direction != "fwd"):
         raise SystemExit("--variant and --pass apply to the convolution layer workloads")
+    if args.workload != "backbone" and args.act != "relu":
+        raise SystemExit("--act applies to the backbone workload")
     if args.workload == "poincare":
         runner = PoincareRunner(torch, quan, *POINCARE_SHAPE)
         unit, per_step_units, dtype = "images/s", runner.N, "f32->bf16"
@@ -801,7 +814,9 @@ def main():
         unit, per_step_units, dtype = "images/s", runner.N, "bf16 (fp32 statistics)"
     elif args.workload == "backbone":
         from paper_2509_05512_gb300 import backbone
-        runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256)
+        runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256,
+                                         act=act_code(args.act),
+                                         fuse_stem_pool=not args.no_fuse)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
     else:
@@ -922,12 +937,14 @@ def main():
         dist.destroy_process_group()
     if rank != 0:
         return 0
-    cfg = workload_config(args.workload, inputs, args.variant, args.direction)
+    cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act)
     cfg.update({"l2": "inputs larger than L2: %d rotating buffer sets, %.0f MB" % (
                     getattr(runner, "sets", 1), runner.footprint / 1e6),
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
                 "timing": "one CUDA-graph replay of the K steps" if graph is not None
                 else "plain launch loop"})
+    if args.workload == "backbone" and not getattr(runner, "fused", False):
+        cfg["fusions"] = "none"
     if args.workload not in ("backbone", "poincare", "iqbn") and args.direction == "fwd":
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     if args.direction == "bwd":
@@ -981,13 +998,22 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1) / 5 / 1e3)
     layers = []
+    fused = getattr(runner, "fused", False)
     for i, (L, t) in enumerate(zip(runner.layers, times)):
+        if fused and L.kind == "maxpool" and L.src == 0:
+            continue  # part of the stem's fused call (layer 0)
         if L.kind == "conv":
             fl, nb = L.spec.flops, L.spec.algorithmic_bytes
             if L.res is not None:
                 nb += L.spec.N * L.spec.Ho * L.spec.Wo * L.spec.Cout * 2
             name = "conv%dx%d/%d %d->%d @%d" % (L.spec.kh, L.spec.kw, L.spec.stride, L.spec.Cin,
                                                 L.spec.Cout, L.spec.H)
+            if fused and i == 0:
+                # stem + 3x3/2 max pool: the pooled output replaces the stem's
+                s0 = L.spec
+                nb += (runner.outs[1].numel() - s0.N * s0.Ho * s0.Wo * s0.Cout) * 2
+                name += " + maxpool3/2 (fused)"
+                kernels[i] = kernels[i] + " + vpool_rows_kernel"
         else:
             src = runner.outs[L.src]
             fl, nb = 0.0, src.numel() * 2 + runner.outs[i].numel() * 2
@@ -1015,7 +1041,7 @@ def backbone_cpu_sample(runner, seconds, inputs):
     import oracle
     import oracle.backbone as ob
     params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in runner.layers]
-    layers = inputs.backbone_layers(N=1, H=runner.H)
+    layers = inputs.backbone_layers(N=1, H=runner.H, act=runner.act)
     x = runner.x_host
     t0 = time.perf_counter()
     ob.forward(layers, params, x[:1])
@@ -1023,7 +1049,7 @@ def backbone_cpu_sample(runner, seconds, inputs):
     n = max(1, min(runner.N, int(seconds / max(t1, 1e-6))))
     if n > 1:
         t0 = time.perf_counter()
-        ob.forward(inputs.backbone_layers(N=n, H=runner.H), params, x[:n])
+        ob.forward(inputs.backbone_layers(N=n, H=runner.H, act=runner.act), params, x[:n])
         t1 = time.perf_counter() - t0
     return {"value": n / t1, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
             "sample": "%d of %d images of the backbone (fp64, %.2f s)" % (n, runner.N, t1)}
@@ -1035,7 +1061,7 @@ def reference_arm(args, rank, world, inputs):
     if rank != 0:
         return 0
     import oracle
-    ref_cfg = workload_config(args.workload, inputs, args.variant, args.direction)
+    ref_cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act)
     ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
     if args.workload == "poincare":
         import numpy as np
@@ -1087,7 +1113,7 @@ def reference_arm(args, rank, world, inputs):
         return 0
     if args.workload == "backbone":
         import oracle.backbone as ob
-        layers = inputs.backbone_layers(N=1)
+        layers = inputs.backbone_layers(N=1, act=act_code(args.act))
         params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in layers]
         x = inputs.backbone_input(n_images=1)
         for _ in range(args.warmup):

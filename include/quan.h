@@ -268,6 +268,31 @@ quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const fl
                                   float eps, int act, void* out, quan_stream_t stream);
 
 /*
+ * The 4-channel stem convolution followed by a 3x3, stride-2, padding-1 max pooling of
+ * every real channel (Sec. III-D pooling rule), fused: the convolution's epilogue takes
+ * the horizontal 3-wide max of each output row and writes only that (half the bytes of
+ * the full output) to `workspace`; a second kernel takes the vertical max into `out`.
+ * The result is bit-identical to quan_qconv2d_fwd followed by quan_maxpool2d_fwd(k = 3,
+ * stride 2, pad 1) (max commutes with the monotone bf16 rounding).
+ *   arguments   those of quan_qconv2d_fwd; out is bf16 [N][Hp][Wp][Cout] with
+ *               Hp = (Ho - 1) / 2 + 1, Wp = (Wo - 1) / 2 + 1 (Ho, Wo of the convolution)
+ *   workspace   device scratch of at least quan_qconv2d_maxpool_workspace_size bytes
+ *               (N Ho (Wp + 4) Cout bf16: each pooled row and 4 side slots for the columns
+ *               whose pixels two producer warps hold), owned by the caller, overwritten
+ * Only the tensor-core pixel-pair shapes: sm_103, Cin = 4, Cout = 64, stride 2, even W,
+ * Wo <= 128, 16-byte aligned tensors; otherwise QUAN_ERR_UNSUPPORTED.
+ */
+size_t quan_qconv2d_maxpool_workspace_size(int N, int H, int W, int Cout, int kh, int kw,
+                                           int stride, int pad);
+quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void* wi,
+                                       const void* wj, const void* wk, const float* bias,
+                                       const float* iqbn_scale, const float* iqbn_shift, int N,
+                                       int H, int W, int Cin, int Cout, int kh, int kw,
+                                       int stride, int pad, int act, void* workspace,
+                                       size_t workspace_bytes, void* out,
+                                       quan_stream_t stream);
+
+/*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,
  * QSPPF), bf16 NHWC [N][H][W][C] -> [N][Ho][Wo][C], window k x k, stride, zero-size
  * padding that never wins.  C is any positive count.

@@ -18,10 +18,16 @@ class BackboneRunner:
     """Weights, activations and the per-step launch sequence of the backbone."""
 
     def __init__(self, torch, quan, inputs=_inputs, N: int = 256, H: int = 224, seed: int = 4,
-                 x_bits=None):
+                 x_bits=None, act: int = _inputs.ACT_RELU, fuse_stem_pool: bool = False):
         self.torch, self.quan, self.N, self.H = torch, quan, N, H
         dev = torch.device("cuda")
-        self.layers = inputs.backbone_layers(N=N, H=H, seed=seed)
+        self.act = act
+        self.layers = inputs.backbone_layers(N=N, H=H, seed=seed, act=act)
+        # stem + 3x3/2 max pool as one call (quan_qconv2d_maxpool_fwd): the stem's full
+        # output is never written, only its horizontally pooled rows (a workspace)
+        L0, L1 = self.layers[0], self.layers[1]
+        self.fused = (fuse_stem_pool and L0.kind == "conv" and L1.kind == "maxpool" and
+                      L1.src == 0 and (L1.k, L1.stride, L1.pad) == (3, 2, 1))
 
         def up(bits):
             return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(
@@ -38,11 +44,19 @@ class BackboneRunner:
                     "shift": torch.from_numpy(prm["shift"]).to(dev),
                     "host": prm})
                 s = L.spec
+                if self.fused and len(self.outs) == 0:
+                    # the workspace of the fused call stands in for the stem's output
+                    self.ws_bytes = quan.quan_qconv2d_maxpool_workspace_size(
+                        N, s.H, s.W, s.Cout, s.kh, s.kw, s.stride, s.pad)
+                    self.outs.append(torch.empty(self.ws_bytes // 2, dtype=torch.bfloat16,
+                                                 device=dev))
+                    self.stem_shape = (N, s.Ho, s.Wo, s.Cout)
+                    continue
                 self.outs.append(torch.empty((N, s.Ho, s.Wo, s.Cout), dtype=torch.bfloat16,
                                              device=dev))
             else:
                 src = self.outs[L.src]
-                _, Hs, Ws, C = src.shape
+                _, Hs, Ws, C = self.stem_shape if (self.fused and L.src == 0) else src.shape
                 Ho = (Hs + 2 * L.pad - L.k) // L.stride + 1
                 Wo = (Ws + 2 * L.pad - L.k) // L.stride + 1
                 self.params.append(None)
@@ -65,11 +79,19 @@ class BackboneRunner:
         x = self.layer_input(idx) if x is None else x
         out = self.outs[idx] if out is None else out
         if L.kind == "maxpool":
+            if self.fused and L.src == 0:
+                return out  # produced by the stem's fused call
             N, H, W, C = x.shape
             q.quan_maxpool2d_fwd(x, N, H, W, C, L.k, L.stride, L.pad, out, stream)
             return out
         s, prm = L.spec, self.params[idx]
         N, H, W, C = x.shape
+        if self.fused and idx == 0:
+            pooled = self.outs[1] if out is self.outs[0] else out
+            q.quan_qconv2d_maxpool_fwd(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
+                                       s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                                       self.outs[0], self.ws_bytes, pooled, stream)
+            return pooled
         if L.res is not None:
             q.quan_qconv2d_fwd_res(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
                                    s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,

@@ -751,8 +751,9 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
                           const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
-                          cudaStream_t stream, char* err, size_t errlen) {
+                          cudaStream_t stream, char* err, size_t errlen, int pool_w = 0) {
     GatherParams prm;
+    prm.pool_w = pool_w;
     prm.s = s;
     prm.ep = ep;
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
@@ -785,6 +786,11 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         return cudaErrorInvalidValue;
     }
     prm.num_tiles = static_cast<int>(tiles);
+    if (pool_w > 0 && prm.segs != 1) {
+        snprintf(err, errlen, "fused pooling needs one tile per output row (Wo <= %d)",
+                 GA_TILE_W);
+        return cudaErrorInvalidValue;
+    }
 
     const MapKey key = make_key(s, x, w, out, 1, 16, 6);
     CUtensorMap maps[6];
@@ -797,7 +803,22 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    static std::atomic<unsigned long long> done_74{0}, done_any{0};
+    static std::atomic<unsigned long long> done_74{0}, done_any{0}, done_74p{0}, done_anyp{0};
+    if (pool_w > 0) {
+        set_kernel_name("qconv_pairs_kernel<hpool>");
+        if (s.kh == 7 && prm.nsp == 4) {
+            auto kern = qconv_pairs_kernel<7, 4, true>;
+            cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74p);
+            if (e != cudaSuccess) return e;
+            return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
+                              maps[0], prm);
+        }
+        auto kern = qconv_pairs_kernel<0, 0, true>;
+        cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_anyp);
+        if (e != cudaSuccess) return e;
+        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
+                          maps[0], prm);
+    }
     set_kernel_name("qconv_pairs_kernel");
     if (s.kh == 7 && prm.nsp == 4) {  // the 7x7 stem
         auto kern = qconv_pairs_kernel<7, 4>;
@@ -1040,6 +1061,22 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
 #undef QUAN_TC_CASE
     snprintf(err, errlen, "no kernel instance for kappa=%d bnq=%d mode=%d", kappa, bnq, mode);
     return cudaErrorInvalidValue;
+}
+
+bool tc_hpool_supported(const ConvShape& s, const void* x, const void* const w[4],
+                        const void* hp, const EpilogueArgs& ep) {
+    return !s.sep && gather_ok(s) && s.Wo <= GA_TILE_W && tc_supported(s, x, w, hp, ep);
+}
+
+cudaError_t launch_qconv_tc_hpool(const ConvShape& s, const void* x, const void* const w[4],
+                                  const EpilogueArgs& ep, void* hp, int pool_w,
+                                  const TcOptions& opt, int num_sms, cudaStream_t stream,
+                                  char* err, size_t errlen) {
+    if (!load_encoders()) {
+        snprintf(err, errlen, "cuTensorMapEncodeTiled is not available");
+        return cudaErrorInvalidValue;
+    }
+    return launch_gather(s, x, w, ep, hp, opt, num_sms, stream, err, errlen, pool_w);
 }
 
 bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy) {

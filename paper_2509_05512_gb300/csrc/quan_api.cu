@@ -535,6 +535,72 @@ quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const fl
     return QUAN_OK;
 }
 
+size_t quan_qconv2d_maxpool_workspace_size(int N, int H, int W, int Cout, int kh, int kw,
+                                           int stride, int pad) {
+    quan::ConvShape s;
+    if (Cout < 4 || Cout % 4 != 0 ||
+        geometry(&s, N, H, W, 4, Cout, kh, kw, stride, pad) != QUAN_OK)
+        return 0;
+    return static_cast<size_t>(N) * s.Ho * ((s.Wo - 1) / 2 + 1 + quan::HPOOL_SIDE_SLOTS) *
+           Cout * 2;
+}
+
+quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void* wi,
+                                       const void* wj, const void* wk, const float* bias,
+                                       const float* iqbn_scale, const float* iqbn_shift, int N,
+                                       int H, int W, int Cin, int Cout, int kh, int kw,
+                                       int stride, int pad, int act, void* workspace,
+                                       size_t workspace_bytes, void* out,
+                                       quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    quan::ConvShape s;
+    // validate() checks the convolution; `out` here is the smaller pooled tensor
+    quan_status_t st = validate(&s, x, w, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                                kw, stride, pad, act, nullptr, workspace ? workspace : out, 2);
+    if (st != QUAN_OK) return st;
+    if (!out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    const int pw = (s.Wo - 1) / 2 + 1, ph = (s.Ho - 1) / 2 + 1;
+    const size_t need =
+        static_cast<size_t>(N) * s.Ho * (pw + quan::HPOOL_SIDE_SLOTS) * Cout * 2;
+    const size_t ob = static_cast<size_t>(N) * ph * pw * Cout * 2;
+    if (!workspace || workspace_bytes < need)
+        return fail(QUAN_ERR_INVALID_ARG, "workspace must hold %zu bytes (got %zu%s)", need,
+                    workspace_bytes, workspace ? "" : ", NULL");
+    if (overlaps(out, ob, workspace, need) || overlaps(out, ob, x, x_bytes(s, 2)) ||
+        overlaps(out, ob, wr, w_bytes(s, 2)) || overlaps(out, ob, wi, w_bytes(s, 2)) ||
+        overlaps(out, ob, wj, w_bytes(s, 2)) || overlaps(out, ob, wk, w_bytes(s, 2)))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input or the workspace");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    const quan::EpilogueArgs ep{bias, iqbn_scale, iqbn_shift, nullptr};
+    if (cc != 103 || !quan::tc_hpool_supported(s, x, w, workspace, ep) ||
+        reinterpret_cast<uintptr_t>(out) % 16 != 0)
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "the fused stem pooling needs sm_103, Cin = 4, Cout = 64, stride 2, an even "
+                    "W, Wo <= 128 and 16-byte aligned tensors");
+    quan::TcOptions opt;
+    opt.kappa = 0;
+    opt.bnq = 0;
+    opt.max_ctas = g_max_ctas.load();
+    opt.mode = 0;
+    opt.ws_halo = 1;
+    opt.ws_issuers = 0;
+    opt.wait_limit_ns = g_wait_limit.load();
+    opt.inject_stall = g_inject.load();
+    char err[256] = "";
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    e = quan::launch_qconv_tc_hpool(s, x, w, ep, workspace, pw, opt, num_sms, cs, err,
+                                    sizeof(err));
+    if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+    if (e != cudaSuccess) return cuda_fail(e, "qconv_pairs launch");
+    e = quan::launch_vpool_bf16(workspace, N, s.Ho, pw, quan::HPOOL_SIDE_SLOTS, Cout, out, cs);
+    if (e != cudaSuccess) return cuda_fail(e, "vpool launch");
+    t_last_path = QUAN_PATH_TC;
+    t_last_kernel = quan::last_tc_kernel();
+    return QUAN_OK;
+}
+
 quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,
                                  int pad, void* out, quan_stream_t stream) {
     if (!x || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");

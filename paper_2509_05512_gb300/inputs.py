@@ -185,16 +185,18 @@ class BackboneLayer:
     pad: int = 0
 
 
-def backbone_layers(N: int = 256, H: int = 224, seed: int = 4) -> list:
+def backbone_layers(N: int = 256, H: int = 224, seed: int = 4, act: int = ACT_RELU) -> list:
     """Layer list of the ResNet-18-style backbone: 7x7/2 stem, 3x3/2 max pool applied
     per real channel, 4 stages x 2 basic blocks at 64/128/256/512 real channels with
     1x1/2 shortcut convolutions; every convolution is a quaternion convolution with
-    fused IQBN; ReLU everywhere except on the shortcut and on the second convolution of
-    a block, which adds the block input (or shortcut) before its ReLU."""
+    fused IQBN; the activation `act` (ReLU by default, SiLU for the detector-style
+    variant) everywhere except on the shortcut, and on the second convolution of a block
+    after the block input (or shortcut) is added."""
     layers = []
     idx = [0]
+    block_act = act
 
-    def conv(src, Hin, Cin, Cout, k, s, p, act=ACT_RELU, res=None):
+    def conv(src, Hin, Cin, Cout, k, s, p, act=block_act, res=None):
         spec = LayerSpec("bb%d" % idx[0], N, Hin, Hin, Cin, Cout, k, k, s, p, act=act,
                          residual=False, seed=(seed, idx[0]),
                          x_dist="uniform" if src == -1 else "normal")

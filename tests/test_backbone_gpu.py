@@ -69,6 +69,25 @@ def test_backbone_two_images_per_layer_and_end_to_end():
     assert (got >= 0).all() and got.std() > 0.1
 
 
+def test_backbone_silu_two_images():
+    # the detector-style variant: SiLU instead of ReLU after every convolution but the
+    # shortcuts; the oracle backbone with the same layer list
+    x_bits = inputs.backbone_input(n_images=2)
+    runner = BackboneRunner(torch, quan, inputs, N=2, x_bits=x_bits, act=inputs.ACT_SILU)
+    assert all(L.spec.act in (inputs.ACT_SILU, inputs.ACT_NONE) for L in runner.layers
+               if L.kind == "conv")
+    stream = torch.cuda.current_stream().cuda_stream
+    runner.step(stream)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    params = check_layers(runner, slice(0, 2))
+    y_ref = ob.forward(inputs.backbone_layers(N=2, act=inputs.ACT_SILU), params, x_bits)
+    got = bf16_bits_to_f64(bits_of(runner.output))
+    rel_l2, _, _ = errors(got, y_ref)
+    assert rel_l2 <= E2E_REL_L2, rel_l2
+    assert (got < 0).any()  # SiLU's negative lobe survives to the output
+
+
 def test_backbone_full_batch_sampled_images():
     runner = BackboneRunner(torch, quan, inputs, N=256)
     stream = torch.cuda.current_stream().cuda_stream

@@ -39,3 +39,17 @@ def test_config_shapes_and_flops():
     assert sum(l.kind == "maxpool" for l in layers) == 1
     total = sum(l.spec.flops for l in convs)
     assert 9.0e11 < total < 1.0e12
+
+
+def test_backbone_activation_variant():
+    relu = inputs.backbone_layers(N=2, act=inputs.ACT_RELU)
+    silu = inputs.backbone_layers(N=2, act=inputs.ACT_SILU)
+    for a, b in zip(relu, silu):
+        if a.kind != "conv":
+            continue
+        # shortcuts keep no activation; every other convolution switches
+        if a.spec.act == inputs.ACT_NONE:
+            assert b.spec.act == inputs.ACT_NONE and a.spec.kh == 1
+        else:
+            assert a.spec.act == inputs.ACT_RELU and b.spec.act == inputs.ACT_SILU
+        assert a.spec.seed == b.spec.seed  # same weights

@@ -1,0 +1,115 @@
+"""The stem convolution with its 3x3/2 max pooling fused (quan_qconv2d_maxpool_fwd): bit
+for bit the two separate calls (max commutes with the monotone bf16 rounding), within the
+bf16 tolerance of the oracle's convolution followed by the oracle's pooling, and through
+the backbone."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+from paper_2509_05512_gb300 import build, inputs, quan
+from paper_2509_05512_gb300.backbone import BackboneRunner
+from tests._util import assert_bf16_close, host_f64, out_f64, to_dev, to_dev_f32
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    build.build_library()
+    yield quan.load()
+
+
+def run_both(spec, act):
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
+    N, H, W = spec.N, spec.H, spec.W
+    conv = quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, scale=sc, shift=sh, act=act)
+    ref_gpu = quan.maxpool2d(conv, k=3, stride=2, pad=1)
+    nbytes = quan.quan_qconv2d_maxpool_workspace_size(N, H, W, spec.Cout, spec.kh, spec.kw,
+                                                      spec.stride, spec.pad)
+    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    out = torch.full_like(ref_gpu, float("nan"))
+    quan.quan_qconv2d_maxpool_fwd(x, *w, None, sc, sh, N, H, W, spec.Cin, spec.Cout, spec.kh,
+                                  spec.kw, spec.stride, spec.pad, act, ws, nbytes, out)
+    torch.cuda.synchronize()
+    assert quan.quan_last_kernel() == "qconv_pairs_kernel<hpool>"
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    return d, out, ref_gpu
+
+
+STEM_CASES = [
+    # name, N, H, W: the 7x7/2 pad-3 stem, 4 -> 64 real channels
+    ("even_wo", 2, 32, 32),
+    ("odd_wo", 2, 30, 30),       # Wo = Ho = 15: the last pooled column and row are partial
+    ("wide", 1, 20, 224),        # a full 112-pixel output row
+    ("tall", 1, 41, 16),
+]
+
+
+@pytest.mark.parametrize("act", [quan.QUAN_ACT_RELU, quan.QUAN_ACT_SILU])
+@pytest.mark.parametrize("case", STEM_CASES, ids=[c[0] for c in STEM_CASES])
+def test_fused_equals_separate_calls_and_oracle(case, act):
+    name, N, H, W = case
+    spec = inputs.small_layer("stem_" + name, N, H, W, 4, 64, 7, 2, 3, seed=(900, len(name)),
+                              act=act)
+    d, out, ref_gpu = run_both(spec, act)
+    assert torch.equal(out, ref_gpu)
+    f = lambda k: host_f64(d[k], "bf16")
+    y = oracle.qconv2d(f("x"), f("wr"), f("wi"), f("wj"), f("wk"), stride=2, pad=3,
+                       scale=d["scale"], shift=d["shift"], act=act)
+    assert_bf16_close(out_f64(out), oracle.maxpool2d(y, k=3, stride=2, pad=1), name)
+
+
+def test_fused_rejects_other_shapes():
+    spec = inputs.small_layer("not_stem", 1, 16, 16, 64, 64, 3, 1, 1, seed=(901, 0))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
+    out = torch.empty((1, 8, 8, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(quan.QuanError) as ei:
+        quan.quan_qconv2d_maxpool_fwd(x, *w, None, None, None, 1, 16, 16, 64, 64, 3, 3, 1, 1,
+                                      quan.QUAN_ACT_RELU, ws, ws.numel(), out)
+    assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+
+
+def test_backbone_fused_stem_is_bit_identical():
+    x_bits = inputs.backbone_input(n_images=2)
+    stream = torch.cuda.current_stream().cuda_stream
+    outs = []
+    for fuse in (False, True):
+        runner = BackboneRunner(torch, quan, inputs, N=2, x_bits=x_bits, fuse_stem_pool=fuse)
+        assert runner.fused == fuse
+        runner.step(stream)
+        torch.cuda.synchronize()
+        assert quan.quan_device_status()[0] == quan.QUAN_OK
+        outs.append((runner.outs[1].clone(), runner.output.clone()))
+    assert torch.equal(outs[0][0], outs[1][0])  # the pooled stem output
+    assert torch.equal(outs[0][1], outs[1][1])  # the backbone output
+
+
+def test_fused_call_first_in_a_fresh_process():
+    # the fused entry point sets up everything it needs on its own (nothing else has
+    # been called in the process before it)
+    import os
+    import subprocess
+    import sys
+    code = (
+        "import torch\n"
+        "from paper_2509_05512_gb300 import inputs, quan\n"
+        "from paper_2509_05512_gb300.backbone import BackboneRunner\n"
+        "r = BackboneRunner(torch, quan, inputs, N=2, fuse_stem_pool=True)\n"
+        "r.run_layer(0, torch.cuda.current_stream().cuda_stream)\n"
+        "torch.cuda.synchronize()\n"
+        "assert quan.quan_last_kernel() == 'qconv_pairs_kernel<hpool>'\n"
+        "assert quan.quan_device_status()[0] == quan.QUAN_OK\n")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    res = subprocess.run([sys.executable, "-c", code], cwd=root, capture_output=True, text=True,
+                         timeout=300)
+    assert res.returncode == 0, res.stderr[-2000:]
