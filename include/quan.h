@@ -209,8 +209,11 @@ quan_status_t quan_qconv2d_bwd_data_static(const void* dy, const void* wr, const
                                            int Cin, int Cout, int kh, int kw, int stride,
                                            int pad, void* dx, quan_stream_t stream);
 
-/* Separable form (Eq. 8-9) of the input gradient; same arguments.  Runs on CUDA cores
- * (the workspace is checked but not used). */
+/* Separable form (Eq. 8-9) of the input gradient; same arguments.  The tensor-core path
+ * (stride 1, a square filter, pad < kh, Cin/4 and Cout/4 multiples of 16) writes the
+ * letters transposed and rotated (not conjugated) into the workspace and runs one
+ * convolution of dy whose block (q, p) is M[q][p] W'_q, M of Eq. 9; other shapes run on
+ * CUDA cores (the workspace is then checked but not used). */
 quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const void* wi,
                                         const void* wj, const void* wk, int N, int H, int W,
                                         int Cin, int Cout, int kh, int kw, int stride, int pad,
@@ -220,17 +223,21 @@ quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const vo
 /*
  * Weight gradients dwr..dwk = dL/dW_L, fp32 [Cout/4][kh][kw][Cin/4] each (device, 4-byte
  * aligned, pairwise disjoint and disjoint from x and dy): zeroed on the stream, then
- * accumulated over all N * Ho * Wo output pixels on CUDA cores (fp32 partial sums added
- * with atomics, so the summation order, and the last bits, vary from run to run).
- * x is the forward input, bf16 [N][H][W][Cin].  quan_set_path(QUAN_PATH_TC) returns
- * QUAN_ERR_UNSUPPORTED.
+ * accumulated over all N * Ho * Wo output pixels (fp32 partial sums added with atomics,
+ * so the summation order, and the last bits, vary from run to run).  Stride 1 with Cin and
+ * Cout multiples of 64 (Cout <= 256 or a multiple of 256) and 16-byte aligned x and dy
+ * runs on the tensor cores (the real weight gradient of every tap as one product over
+ * the pixels, folded into the four letters), other shapes on CUDA cores;
+ * quan_set_path(QUAN_PATH_TC) makes those fail with QUAN_ERR_UNSUPPORTED.
+ * x is the forward input, bf16 [N][H][W][Cin].
  */
 quan_status_t quan_qconv2d_bwd_weight(const void* x, const void* dy, int N, int H, int W,
                                       int Cin, int Cout, int kh, int kw, int stride, int pad,
                                       float* dwr, float* dwi, float* dwj, float* dwk,
                                       quan_stream_t stream);
 
-/* Separable form (Eq. 10) of the weight gradients; same arguments. */
+/* Separable form (Eq. 10) of the weight gradients; same arguments and paths (the
+ * tensor-core kernel folds its blocks by Eq. 7's sign table). */
 quan_status_t quan_qconv2d_sep_bwd_weight(const void* x, const void* dy, int N, int H, int W,
                                           int Cin, int Cout, int kh, int kw, int stride,
                                           int pad, float* dwr, float* dwi, float* dwj,

@@ -13,7 +13,9 @@ struct ConvShape {
     int N, H, W, Cin, Cout, kh, kw, stride, pad, act;
     int Ho, Wo, Qin, Qout;
     long long M;  // N * Ho * Wo output pixels
-    int sep;      // 1: the separable form of Eq. 7 (per-component convolutions, sign mix)
+    int sep;      // 1: the separable form of Eq. 7 (per-component convolutions, sign mix);
+                  // 2 (tensor-core path only): its transpose, the input gradient's
+                  // convolution (block (q, p) = sign(p, q) W_q)
 };
 
 struct EpilogueArgs {
@@ -87,10 +89,12 @@ cudaError_t launch_poincare(const float* rgb, long long npix, void* out, int num
 // Backward of the pre-epilogue convolution (s.sep selects the separable form, Eq. 8-10).
 // Bytes of the transformed letters bwd_transform writes: 4 x [Qin][kh][kw][Qout] bf16.
 size_t bwd_data_workspace_bytes(int Cin, int Cout, int kh, int kw);
-// out_L[ci][kh-1-dh][kw-1-dw][co] = (L == r ? +1 : -1) * w_L[co][dh][dw][ci], the four
-// letters one after the other: the forward weights of the stride-1 input gradient.
+// out_L[ci][kh-1-dh][kw-1-dw][co] = s_L * w_L[co][dh][dw][ci], the four letters one after
+// the other: the forward weights of the stride-1 input gradient; s = (+1, -1, -1, -1)
+// (the conjugate, full form) when conj, else +1 (the separable form's signs are applied
+// by the MMA table).
 cudaError_t launch_bwd_transform(int Cin, int Cout, int kh, int kw, const void* const w[4],
-                                 void* out, int num_sms, cudaStream_t stream);
+                                 bool conj, void* out, int num_sms, cudaStream_t stream);
 // dx [N][H][W][Cin] from dy [N][Ho][Wo][Cout] on CUDA cores, any stride.
 cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void* const w[4],
                                  void* dx, cudaStream_t stream);
@@ -98,7 +102,7 @@ cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void*
 // module's static device memory): its size, and its address on the current device.
 constexpr size_t BWD_STATIC_SCRATCH_BYTES = size_t(2) << 20;
 cudaError_t bwd_static_scratch_address(void** ptr);
-// Tensor-core weight gradient of the full form (stride 1, Cin and Cout multiples of 64,
+// Tensor-core weight gradient, both forms (s.sep) (stride 1, Cin and Cout multiples of 64,
 // Cout <= 256 or a multiple of 256, 16-byte aligned x and dy).  Zeroes dW_L, then adds.
 bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy);
 cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* dy,

@@ -16,7 +16,9 @@
 // Separable form (Eq. 7): Eq. 8-10 -- the output gradients are first mixed by the matrix M
 // of Eq. 9 (g_p = sum_m M[p][m] dy_m, M transposed equal to Eq. 7's sign table), then
 // dL/dx_p is the transposed convolution of g_p with W_p alone and dL/dW_p the correlation
-// of g_p with x_p alone.
+// of g_p with x_p alone.  On the tensor cores (stride 1) the input gradient is one
+// convolution of dy whose block (q, p) is M[q][p] W'_q (W' the letters transposed and
+// rotated, not conjugated): the forward kernel's transposed-separable mode.
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -39,9 +41,10 @@ __device__ __forceinline__ void mix_eq9(float dr, float di, float dj, float dk, 
     gk = -dr - di + dj + dk;
 }
 
-// out_L[ci][dh][dw][co] = s_L * W_L[co][kh-1-dh][kw-1-dw][ci], s = (+1, -1, -1, -1).
+// out_L[ci][dh][dw][co] = s_L * W_L[co][kh-1-dh][kw-1-dw][ci], s = (+1, -1, -1, -1) when
+// conj, else +1.
 __global__ void __launch_bounds__(256) bwd_transform_kernel(
-    int Qin, int Qout, int kh, int kw, const __nv_bfloat16* __restrict__ wr,
+    int Qin, int Qout, int kh, int kw, int conj, const __nv_bfloat16* __restrict__ wr,
     const __nv_bfloat16* __restrict__ wi, const __nv_bfloat16* __restrict__ wj,
     const __nv_bfloat16* __restrict__ wk, __nv_bfloat16* __restrict__ out) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -61,7 +64,7 @@ __global__ void __launch_bounds__(256) bwd_transform_kernel(
         const long long src =
             ((static_cast<long long>(co) * kh + (kh - 1 - dh)) * kw + (kw - 1 - dw)) * Qin + ci;
         const __nv_bfloat16 v = w[L][src];
-        out[i] = L == 0 ? v : __hneg(v);
+        out[i] = (L == 0 || !conj) ? v : __hneg(v);
     }
 }
 
@@ -203,13 +206,13 @@ size_t bwd_data_workspace_bytes(int Cin, int Cout, int kh, int kw) {
 }
 
 cudaError_t launch_bwd_transform(int Cin, int Cout, int kh, int kw, const void* const w[4],
-                                 void* out, int num_sms, cudaStream_t stream) {
+                                 bool conj, void* out, int num_sms, cudaStream_t stream) {
     const long long n = 4LL * (Cin / 4) * kh * kw * (Cout / 4);
     if (n == 0) return cudaSuccess;
     long long blocks = (n + 255) / 256;
     if (blocks > num_sms * 8LL) blocks = num_sms * 8LL;
     return launch_pdl(bwd_transform_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0,
-                      stream, Cin / 4, Cout / 4, kh, kw,
+                      stream, Cin / 4, Cout / 4, kh, kw, conj ? 1 : 0,
                       static_cast<const __nv_bfloat16*>(w[0]),
                       static_cast<const __nv_bfloat16*>(w[1]),
                       static_cast<const __nv_bfloat16*>(w[2]),

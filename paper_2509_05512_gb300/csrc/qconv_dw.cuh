@@ -17,6 +17,9 @@
 // ncols fp32 columns each) and one ncols-wide group of output channels, for a contiguous
 // range of pixel blocks (split K); its epilogue folds the 16 blocks into the letters and
 // adds them to the fp32 outputs with atomics (zeroed before the launch).
+// Separable form (Eq. 7, gradient Eq. 10): y_m = sum_p S[m][p] W_p conv x_p, so block
+// (m, p) goes to letter p with Eq. 7's sign S[m][p] instead (the same 16 blocks: the
+// product computes the 12 cross-component blocks the separable form does not use).
 
 namespace dwk {
 
@@ -40,6 +43,7 @@ struct DwParams {
     int a_per, pair_groups;  // pairs per CTA; groups of pairs
     int ncols, nyb;          // output channels per CTA (N of each MMA); dy boxes per stage
     int groups, splits, stages;
+    int sep;                 // 1: fold for the separable form
     uint32_t tmem_cols;
     uint32_t stage_bytes;
     unsigned long long wait_limit_ns;
@@ -222,8 +226,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int h = 0; h < 2; ++h) {
                         const int d0 = cg * p.ncols + j0 + 16 * h;
                         const int m = d0 / p.Qout, co0 = d0 - m * p.Qout;
-                        const bool neg = (NEG_MASK >> (4 * m + pc)) & 1u;
-                        float* dst = letter_ptr(p, m ^ pc) + co0 * wstride + row_off;
+                        const bool neg = ((p.sep ? SEP_NEG : NEG_MASK) >> (4 * m + pc)) & 1u;
+                        float* dst = letter_ptr(p, p.sep ? pc : (m ^ pc)) + co0 * wstride + row_off;
 #pragma unroll
                         for (int jj = 0; jj < 16; ++jj) {
                             const float val = __uint_as_float(v[16 * h + jj]);

@@ -74,6 +74,10 @@ constexpr int MODE_QUAD = 0;
 constexpr int MODE_PAIR = 1;
 constexpr int MODE_WS = 2;
 constexpr int MODE_SEP = 3;
+// The separable form's input gradient (ConvShape::sep == 2): 16 MMAs per K step like
+// MODE_QUAD, block (output q, input p) = the letter q with the sign of Eq. 7's term
+// (output p, letter q) -- the transpose of the separable block weight.
+constexpr int MODE_SEPT = 4;
 constexpr int WS_MAX_TAPS = 9;
 constexpr int MAX_STAGES = 8;
 
@@ -331,10 +335,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             } else {
 #pragma unroll
                                 for (int q = 0; q < 4; ++q) {
-                                    const int L = q ^ pc;
+                                    const int L = MODE == MODE_SEPT ? q : q ^ pc;
                                     const uint32_t b_lo =
                                         b_lo0 + ((L * C::B_TILE + ks * (UMMA_K * 2)) >> 4);
-                                    const bool neg = (NEG_MASK >> (4 * q + pc)) & 1u;
+                                    const bool neg = MODE == MODE_SEPT
+                                                         ? ((SEP_NEG >> (4 * pc + q)) & 1u)
+                                                         : ((NEG_MASK >> (4 * q + pc)) & 1u);
                                     umma_f16_w(dbase + q * BNQ, a_lo, C::DESC_HI, b_lo,
                                                C::DESC_HI, neg ? IDESC_NEG : IDESC_POS, acc);
                                 }
@@ -840,9 +846,10 @@ constexpr int DW_SMEM_MAX = 232448;  // dynamic shared memory a CTA may opt into
 
 // Tiling of the tensor-core weight gradient (see qconv_dw.cuh); false if the shape has none.
 bool dw_plan(const ConvShape& s, int num_sms, dwk::DwParams* p) {
-    if (s.sep || s.stride != 1 || s.Cin % 64 != 0 || s.Cout % 64 != 0) return false;
+    if (s.stride != 1 || s.Cin % 64 != 0 || s.Cout % 64 != 0) return false;
     if (s.Cout > 256 && s.Cout % 256 != 0) return false;
     dwk::DwParams q = {};
+    q.sep = s.sep ? 1 : 0;
     q.Ho = s.Ho; q.Wo = s.Wo; q.Qin = s.Qin; q.Qout = s.Qout;
     q.kh = s.kh; q.kw = s.kw; q.pad = s.pad; q.taps = s.kh * s.kw;
     q.nxc = s.Cin / 64;
@@ -969,7 +976,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     int kappa = pick_kappa(s.Qin, opt.kappa);
     const int bnq = pick_bnq(s.Qout, opt.bnq);
     int mode;
-    if (s.sep) mode = ws_ok ? MODE_WS : MODE_SEP;
+    if (s.sep == 2) mode = MODE_SEPT;
+    else if (s.sep) mode = ws_ok ? MODE_WS : MODE_SEP;
     else if (opt.mode == 1) mode = MODE_QUAD;
     else if (opt.mode == 2) mode = MODE_PAIR;
     else if (opt.mode == 3) mode = MODE_WS;
@@ -996,6 +1004,7 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     if (kappa == K && bnq == B)                                                    \
         fits = mode == MODE_PAIR ? cfg_fits<K, B, MODE_PAIR>()                     \
              : mode == MODE_SEP  ? cfg_fits<K, B, MODE_SEP>()                      \
+             : mode == MODE_SEPT ? cfg_fits<K, B, MODE_SEPT>()                     \
                                  : cfg_fits<K, B, MODE_QUAD>();
         QUAN_FIT_CASE(16, 16) QUAN_FIT_CASE(16, 32) QUAN_FIT_CASE(16, 64)
         QUAN_FIT_CASE(32, 16) QUAN_FIT_CASE(32, 32) QUAN_FIT_CASE(32, 64)
@@ -1039,16 +1048,18 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    set_kernel_name(mode == MODE_PAIR  ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
-                    : mode == MODE_SEP ? "qconv_tc_kernel<sep,kappa=%d,bnq=%d>"
-                                       : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
+    set_kernel_name(mode == MODE_PAIR   ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
+                    : mode == MODE_SEP  ? "qconv_tc_kernel<sep,kappa=%d,bnq=%d>"
+                    : mode == MODE_SEPT ? "qconv_tc_kernel<sep_t,kappa=%d,bnq=%d>"
+                                        : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
                     kappa, bnq);
 
 #define QUAN_TC_CASE(K, B)                                                       \
     if (kappa == K && bnq == B)                                                  \
-        return mode == MODE_PAIR  ? launch_cfg<K, B, MODE_PAIR>(maps, prm, grid, stream) \
-               : mode == MODE_SEP ? launch_cfg<K, B, MODE_SEP>(maps, prm, grid, stream)  \
-                                  : launch_cfg<K, B, MODE_QUAD>(maps, prm, grid, stream);
+        return mode == MODE_PAIR   ? launch_cfg<K, B, MODE_PAIR>(maps, prm, grid, stream)  \
+               : mode == MODE_SEP  ? launch_cfg<K, B, MODE_SEP>(maps, prm, grid, stream)   \
+               : mode == MODE_SEPT ? launch_cfg<K, B, MODE_SEPT>(maps, prm, grid, stream)  \
+                                   : launch_cfg<K, B, MODE_QUAD>(maps, prm, grid, stream);
     QUAN_TC_CASE(16, 16)
     QUAN_TC_CASE(16, 32)
     QUAN_TC_CASE(16, 64)
@@ -1119,7 +1130,8 @@ cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* 
     static std::atomic<unsigned long long> attr_done{0};
     cudaError_t e = set_smem_once(dwk::qconv_dw_kernel, DW_SMEM_MAX, attr_done);
     if (e != cudaSuccess) return e;
-    set_kernel_name("qconv_dw_kernel<pairs=%d,n=%d>", p.a_per, p.ncols);
+    set_kernel_name(p.sep ? "qconv_dw_kernel<pairs=%d,n=%d,sep>" : "qconv_dw_kernel<pairs=%d,n=%d>",
+                    p.a_per, p.ncols);
     return launch_pdl(dwk::qconv_dw_kernel, dim3(static_cast<unsigned>(p.groups * p.splits)),
                       dim3(dwk::THREADS), static_cast<size_t>(smem), stream, mx, mdy, p);
 }

@@ -232,23 +232,26 @@ quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H,
     const size_t per = need / 4;
     const void* tw[4];
     for (int L = 0; L < 4; ++L) tw[L] = static_cast<const char*>(workspace) + L * per;
-    bool tc_ok = !separable && stride == 1 && kh == kw && pad <= kh - 1 && cc == 103 &&
+    bool tc_ok = stride == 1 && kh == kw && pad <= kh - 1 && cc == 103 &&
                  geometry(&t, N, s.Ho, s.Wo, Cout, Cin, kh, kw, 1, kh - 1 - pad) == QUAN_OK &&
                  quan::tc_supported(t, dy, tw, dx, none);
+    // separable form: the transposed-separable MMA mode (Qin, Qout multiples of 16)
+    if (separable) t.sep = 2;
+    if (separable && (Cin % 64 != 0 || Cout % 64 != 0)) tc_ok = false;
     const int path = g_path.load();
     if (path == QUAN_PATH_TC && !tc_ok)
         return fail(QUAN_ERR_UNSUPPORTED,
-                    "tensor-core input gradient needs the full form, stride 1, a square filter, "
-                    "pad < kh, sm_103 and Cin/4, Cout/4 multiples of 16 with 16-byte aligned "
-                    "tensors");
+                    "tensor-core input gradient needs stride 1, a square filter, pad < kh, "
+                    "sm_103 and Cin/4, Cout/4 multiples of 16 with 16-byte aligned tensors");
     if (tc_ok && path != QUAN_PATH_SIMT) {
-        e = quan::launch_bwd_transform(Cin, Cout, kh, kw, w, workspace, num_sms, cs);
+        e = quan::launch_bwd_transform(Cin, Cout, kh, kw, w, !separable, workspace, num_sms,
+                                       cs);
         if (e != cudaSuccess) return cuda_fail(e, "bwd_transform launch");
         quan::TcOptions opt;
         opt.kappa = g_kappa.load();
         opt.bnq = g_bnq.load();
         opt.max_ctas = g_max_ctas.load();
-        opt.mode = g_mode.load();
+        opt.mode = separable ? 0 : g_mode.load();
         opt.ws_halo = g_ws_halo.load();
         opt.ws_issuers = g_ws_issuers.load();
         opt.wait_limit_ns = g_wait_limit.load();
@@ -288,14 +291,13 @@ quan_status_t run_bwd_weight(const void* x, const void* dy, int N, int H, int W,
         if (reinterpret_cast<uintptr_t>(dw[L]) % 4 != 0)
             return fail(QUAN_ERR_INVALID_ARG, "weight gradients must be 4-byte aligned");
     }
-    // tensor cores for the full form at stride 1 (the shape checks need no device)
-    const bool tc_shape = !separable && quan::bwd_weight_tc_supported(s, x, dy);
+    // tensor cores at stride 1, both forms (the shape checks need no device)
+    const bool tc_shape = quan::bwd_weight_tc_supported(s, x, dy);
     const int path = g_path.load();
     if (path == QUAN_PATH_TC && !tc_shape)
         return fail(QUAN_ERR_UNSUPPORTED,
-                    "tensor-core weight gradient needs the full form, stride 1, Cin and Cout "
-                    "multiples of 64 (Cout <= 256 or a multiple of 256) and 16-byte aligned x "
-                    "and dy");
+                    "tensor-core weight gradient needs stride 1, Cin and Cout multiples of 64 "
+                    "(Cout <= 256 or a multiple of 256) and 16-byte aligned x and dy");
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");

@@ -146,14 +146,13 @@ def test_backward_weight_invalid_arguments(lib, sep, bad):
 
 
 def test_backward_weight_tensor_core_shapes(lib):
-    # the tensor-core weight gradient takes stride 1, the full form, Cin and Cout multiples
-    # of 64: forcing it on another shape fails on the host
+    # the tensor-core weight gradient takes stride 1, Cin and Cout multiples of 64:
+    # forcing it on another shape fails on the host
     assert lib.quan_set_path(quan.QUAN_PATH_TC) == quan.QUAN_OK
     try:
         assert _bwd_weight(lib, stride=2) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, Cin=48) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, Cout=320) == quan.QUAN_ERR_UNSUPPORTED
-        assert _bwd_weight(lib, sep=True) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, x=FAKE + 8) == quan.QUAN_ERR_UNSUPPORTED  # misaligned for TMA
     finally:
         assert lib.quan_set_path(quan.QUAN_PATH_AUTO) == quan.QUAN_OK

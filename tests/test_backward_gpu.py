@@ -92,12 +92,12 @@ def tc_weight_shape(spec):
 def check_weight(d, separable=False, path=quan.QUAN_PATH_AUTO):
     got, kernel = gpu_bwd_weight(d, separable, path)
     spec = d["spec"]
-    if separable:
-        assert kernel == "bwd_weight_simt_kernel<sep>"
-    elif path != quan.QUAN_PATH_SIMT and tc_weight_shape(spec):
+    if path != quan.QUAN_PATH_SIMT and tc_weight_shape(spec):
         assert kernel.startswith("qconv_dw_kernel<"), kernel
+        assert kernel.endswith(",sep>") == separable, kernel
     else:
-        assert kernel == "bwd_weight_simt_kernel", kernel
+        assert kernel == ("bwd_weight_simt_kernel<sep>" if separable
+                          else "bwd_weight_simt_kernel"), kernel
     ref = oracle_bwd_weight(d, separable)
     for L in range(4):
         assert_f32_close(got[L], ref[L], "%s dW[%d] (%s)" % (spec.name, L, kernel))
@@ -235,6 +235,8 @@ def test_bwd_weight_paths_agree():
 
 SEP_CASES = [
     ("sep_3x3", 2, 13, 11, 64, 64, 3, 1, 1),
+    ("sep_wide", 2, 9, 10, 128, 256, 3, 1, 1),
+    ("sep_pad0_5x5", 1, 12, 11, 64, 128, 5, 1, 0),
     ("sep_stride2", 2, 15, 17, 64, 128, 3, 2, 1),
     ("sep_pointwise", 1, 10, 9, 128, 64, 1, 1, 0),
     ("sep_qin3", 1, 8, 9, 12, 16, 3, 1, 1),
@@ -246,9 +248,35 @@ def test_separable_backward(case):
     name, N, H, W, Cin, Cout, k, s, p = case
     d = layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(608, len(name))))
     got, path, kernel = gpu_bwd_data(d, separable=True)
-    assert kernel == "bwd_data_simt_kernel<sep>"
+    if s == 1 and Cin % 64 == 0 and Cout % 64 == 0:
+        assert kernel.startswith("qconv_tc_kernel<sep_t,"), kernel
+    else:
+        assert kernel == "bwd_data_simt_kernel<sep>", kernel
     assert_bf16_close(got, oracle_bwd_data(d, True), name + " sep dx")
     check_weight(d, separable=True)
+
+
+@pytest.mark.parametrize("case", [("sepw_3x3", 2, 12, 10, 64, 128, 3, 1, 1),
+                                  ("sepw_c256", 1, 9, 7, 256, 64, 3, 1, 1)],
+                         ids=lambda c: c[0])
+def test_separable_weight_gradient_paths(case):
+    # the tensor-core kernel with Eq. 7's fold against the oracle and the CUDA-core kernel
+    name, N, H, W, Cin, Cout, k, s, p = case
+    d = layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(612, len(name))))
+    tc = check_weight(d, separable=True, path=quan.QUAN_PATH_TC)
+    simt = check_weight(d, separable=True, path=quan.QUAN_PATH_SIMT)
+    for L in range(4):
+        assert_f32_close(tc[L], simt[L], "sep tc vs simt dW[%d]" % L)
+
+
+def test_separable_input_gradient_paths_agree():
+    d = layer(inputs.small_layer("sep_both", 2, 11, 9, 64, 128, 3, 1, 1, seed=(613, 0)))
+    tc, p1, k1 = gpu_bwd_data(d, separable=True, path=quan.QUAN_PATH_TC)
+    simt, p2, _ = gpu_bwd_data(d, separable=True, path=quan.QUAN_PATH_SIMT)
+    assert (p1, p2) == (quan.QUAN_PATH_TC, quan.QUAN_PATH_SIMT), k1
+    ref = oracle_bwd_data(d, True)
+    assert_bf16_close(tc, ref, "sep tc")
+    assert_bf16_close(simt, ref, "sep simt")
 
 
 def test_separable_backward_differs_from_full_form():
