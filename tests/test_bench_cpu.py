@@ -1,0 +1,53 @@
+"""bench.py's reference arm (the fp64 oracle on the host cores) on CPU: one JSON line with
+the contract's keys for the layer, backward, separable, IQBN and Poincare workloads."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+CASES = [
+    (["--workload", "c1"], "TFLOP/s"),
+    (["--pass", "bwd"], "TFLOP/s"),
+    (["--variant", "separable", "--workload", "c1"], "TFLOP/s"),
+    (["--workload", "iqbn"], "images/s"),
+    (["--workload", "poincare"], "images/s"),
+]
+
+
+@pytest.mark.parametrize("args,unit", CASES, ids=lambda a: "_".join(a) if isinstance(a, list)
+                         else None)
+def test_reference_arm_json_line(args, unit):
+    res = subprocess.run([sys.executable, "bench.py", "--impl", "reference", *args, "--steps",
+                          "1", "--warmup", "1"], cwd=ROOT, capture_output=True, text=True,
+                         timeout=600)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [ln for ln in res.stdout.splitlines() if ln.strip()]
+    assert len(lines) == 1, res.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC
+    assert d["unit"] == unit and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["steps"] == 1 and d["warmup"] == 1 and d["n_gpus"] == 1
+    assert d["e2e"] == {"value": d["value"], "unit": unit, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
+    assert isinstance(d["config"]["workload"], str) and d["vs_baseline"] is None
+    if "bwd" in args:
+        assert "backward" in d["config"]["workload"]
+    if "separable" in args:
+        assert "Eq. 7" in d["config"]["workload"]
+
+
+def test_workload_config_flops():
+    from paper_2509_05512_gb300 import inputs
+    full = bench.workload_config("c1", inputs)["flops_per_step"]
+    assert bench.workload_config("c1", inputs, "separable")["flops_per_step"] == full / 4
+    assert bench.workload_config("c1", inputs, "full", "bwd")["flops_per_step"] == 2 * full
+    bb = bench.workload_config("backbone", inputs, act="silu")
+    assert "SiLU" in bb["epilogue"] and bb["convs"] == 20
