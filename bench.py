@@ -327,8 +327,9 @@ class BwdRunner:
         self.dxs = [torch.empty_like(x0) for _ in range(self.sets)]
         wshape = (spec.Cout // 4, spec.kh, spec.kw, spec.Cin // 4)
         self.dws = [torch.empty(wshape, dtype=torch.float32, device=dev) for _ in range(4)]
-        self.ws_bytes = quan.quan_qconv2d_bwd_data_workspace_size(spec.Cin, spec.Cout,
-                                                                  spec.kh, spec.kw)
+        self.ws_bytes = quan.quan_qconv2d_bwd_data_workspace_size_ex(
+            spec.N, spec.H, spec.W, spec.Cin, spec.Cout, spec.kh, spec.kw, spec.stride,
+            spec.pad)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=dev)
         self.i = 0
         self.footprint = per_set * self.sets

@@ -165,17 +165,31 @@ quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
 size_t quan_qconv2d_bwd_data_workspace_size(int Cin, int Cout, int kh, int kw);
 
 /*
+ * Workspace that lets quan_qconv2d_bwd_data (and _sep_) run a STRIDED forward's input
+ * gradient on the tensor cores: the transformed letters, then dy with stride - 1 zeros
+ * between its pixels, [N][H + 2 pad - kh + 1][W + 2 pad - kw + 1][Cout] bf16 (256-byte
+ * aligned after the letters).  Equals quan_qconv2d_bwd_data_workspace_size for stride 1;
+ * 0 for invalid sizes.  Arguments are the forward convolution's.
+ */
+size_t quan_qconv2d_bwd_data_workspace_size_ex(int N, int H, int W, int Cin, int Cout, int kh,
+                                               int kw, int stride, int pad);
+
+/*
  * Input gradient dx = dL/dx, bf16 [N][H][W][Cin] (device), rounded to nearest even from an
  * fp32 accumulation.  N..pad are the FORWARD convolution's arguments.
  *   workspace        device scratch of at least quan_qconv2d_bwd_data_workspace_size
  *                    bytes, 16-byte aligned for the tensor-core path, owned by the caller;
  *                    NULL or too small returns QUAN_ERR_INVALID_ARG.  Its contents are
  *                    overwritten; concurrent calls need separate workspaces.
- * dx must not overlap dy, the weights or the workspace.  For stride 1, a square filter,
- * pad < kh and Cin/4, Cout/4 multiples of 16 on sm_103, the tensor-core path runs: one
- * kernel writes conj(W) with its channel axes swapped and the filter rotated by 180
- * degrees into the workspace, then the forward tensor-core kernel convolves dy with it
- * (padding kh - 1 - pad).  Other shapes run a direct CUDA-core kernel.
+ * dx must not overlap dy, the weights or the workspace.  For a square filter, pad < kh and
+ * Cin/4, Cout/4 multiples of 16 on sm_103, the tensor-core path runs: one kernel writes
+ * conj(W) with its channel axes swapped and the filter rotated by 180 degrees into the
+ * workspace, then the forward tensor-core kernel convolves dy with it (stride 1, padding
+ * kh - 1 - pad).  For a strided forward this needs the larger workspace of
+ * quan_qconv2d_bwd_data_workspace_size_ex: dy is first spread out with zeros between its
+ * pixels (stride - 1 of them), which multiplies the MMAs by stride^2 but keeps them on the
+ * tensor cores.  Other shapes, or a strided forward with the smaller workspace, run a
+ * direct CUDA-core kernel.
  * quan_set_path(QUAN_PATH_TC) makes a shape the tensor-core path cannot run fail with
  * QUAN_ERR_UNSUPPORTED.
  */
@@ -209,8 +223,8 @@ quan_status_t quan_qconv2d_bwd_data_static(const void* dy, const void* wr, const
                                            int Cin, int Cout, int kh, int kw, int stride,
                                            int pad, void* dx, quan_stream_t stream);
 
-/* Separable form (Eq. 8-9) of the input gradient; same arguments.  The tensor-core path
- * (stride 1, a square filter, pad < kh, Cin/4 and Cout/4 multiples of 16) writes the
+/* Separable form (Eq. 8-9) of the input gradient; same arguments and paths.  The
+ * tensor-core path (a square filter, pad < kh, Cin/4 and Cout/4 multiples of 16) writes the
  * letters transposed and rotated (not conjugated) into the workspace and runs one
  * convolution of dy whose block (q, p) is M[q][p] W'_q, M of Eq. 9; other shapes run on
  * CUDA cores (the workspace is then checked but not used). */
@@ -224,8 +238,8 @@ quan_status_t quan_qconv2d_sep_bwd_data(const void* dy, const void* wr, const vo
  * Weight gradients dwr..dwk = dL/dW_L, fp32 [Cout/4][kh][kw][Cin/4] each (device, 4-byte
  * aligned, pairwise disjoint and disjoint from x and dy): zeroed on the stream, then
  * accumulated over all N * Ho * Wo output pixels (fp32 partial sums added with atomics,
- * so the summation order, and the last bits, vary from run to run).  Stride 1 with Cin and
- * Cout multiples of 64 (Cout <= 256 or a multiple of 256) and 16-byte aligned x and dy
+ * so the summation order, and the last bits, vary from run to run).  Stride 1 or 2 with Cin
+ * and Cout multiples of 64 (Cout <= 256 or a multiple of 256) and 16-byte aligned x and dy
  * runs on the tensor cores (the real weight gradient of every tap as one product over
  * the pixels, folded into the four letters), other shapes on CUDA cores;
  * quan_set_path(QUAN_PATH_TC) makes those fail with QUAN_ERR_UNSUPPORTED.

@@ -95,6 +95,10 @@ size_t bwd_data_workspace_bytes(int Cin, int Cout, int kh, int kw);
 // by the MMA table).
 cudaError_t launch_bwd_transform(int Cin, int Cout, int kh, int kw, const void* const w[4],
                                  bool conj, void* out, int num_sms, cudaStream_t stream);
+// dy [N][Ho][Wo][C] with s - 1 zeros inserted between pixels, [N][Hu][Wu][C] (C % 8 == 0,
+// 16-byte aligned): the input of a strided forward's input-gradient convolution.
+cudaError_t launch_bwd_upsample(const void* dy, int N, int Ho, int Wo, int C, int s, int Hu,
+                                int Wu, void* u, int num_sms, cudaStream_t stream);
 // dx [N][H][W][Cin] from dy [N][Ho][Wo][Cout] on CUDA cores, any stride.
 cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void* const w[4],
                                  void* dx, cudaStream_t stream);
@@ -102,7 +106,7 @@ cudaError_t launch_bwd_data_simt(const ConvShape& s, const void* dy, const void*
 // module's static device memory): its size, and its address on the current device.
 constexpr size_t BWD_STATIC_SCRATCH_BYTES = size_t(2) << 20;
 cudaError_t bwd_static_scratch_address(void** ptr);
-// Tensor-core weight gradient, both forms (s.sep) (stride 1, Cin and Cout multiples of 64,
+// Tensor-core weight gradient, both forms (s.sep) (stride 1 or 2, Cin and Cout multiples of 64,
 // Cout <= 256 or a multiple of 256, 16-byte aligned x and dy).  Zeroes dW_L, then adds.
 bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy);
 cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* dy,

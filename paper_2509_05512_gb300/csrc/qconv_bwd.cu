@@ -8,8 +8,11 @@
 //   * the input gradient is itself a quaternion convolution: of dy, with the letters
 //     conjugated, their channel axes swapped and the filter rotated by 180 degrees, padding
 //     kh - 1 - pad, stride 1 (for a stride-1 forward).  bwd_transform_kernel writes those
-//     letters into a caller workspace and the forward tensor-core kernels run the rest;
-//     other strides use the direct CUDA-core kernel below;
+//     letters into a caller workspace and the forward tensor-core kernels run the rest.
+//     A stride-s forward's input gradient is the same stride-1 convolution of dy with
+//     s - 1 zero rows and columns inserted between its pixels (bwd_upsample_kernel, into
+//     the workspace after the letters), when the caller's workspace holds it; otherwise
+//     the direct CUDA-core kernel below runs;
 //   * the weight gradient is a reduction over output pixels, done on CUDA cores: every
 //     thread owns one (co, tap, ci) quaternion of dW for a chunk of pixels and adds its
 //     fp32 partial sum to the zeroed output with atomicAdd.
@@ -193,7 +196,41 @@ __global__ void __launch_bounds__(256) bwd_weight_simt_kernel(
 // not pass this name to a kernel: on the host it is a stand-in, not a device address.
 static __device__ __align__(256) unsigned char g_bwd_static_scratch[BWD_STATIC_SCRATCH_BYTES];
 
+// u[n][y][x] = dy[n][y / s][x / s] where s divides y and x (and y / s < Ho, x / s < Wo),
+// else 0: dy with s - 1 zeros between its pixels, [N][Hu][Wu][C], 16 bytes per thread.
+__global__ void __launch_bounds__(256) bwd_upsample_kernel(const uint4* __restrict__ dy, int N,
+                                                           int Ho, int Wo, int cv, int s, int Hu,
+                                                           int Wu, uint4* __restrict__ u) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const long long total = static_cast<long long>(N) * Hu * Wu * cv;
+    for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+         i += static_cast<long long>(gridDim.x) * blockDim.x) {
+        const int c = static_cast<int>(i % cv);
+        const long long pix = i / cv;
+        const int x = static_cast<int>(pix % Wu);
+        const int y = static_cast<int>((pix / Wu) % Hu);
+        const int n = static_cast<int>(pix / (static_cast<long long>(Wu) * Hu));
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (y % s == 0 && x % s == 0 && y / s < Ho && x / s < Wo)
+            v = __ldg(dy + ((static_cast<long long>(n) * Ho + y / s) * Wo + x / s) * cv + c);
+        u[i] = v;
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_bwd_upsample(const void* dy, int N, int Ho, int Wo, int C, int s, int Hu,
+                                int Wu, void* u, int num_sms, cudaStream_t stream) {
+    if (C % 8 != 0) return cudaErrorInvalidValue;
+    const long long total = static_cast<long long>(N) * Hu * Wu * (C / 8);
+    if (total == 0) return cudaSuccess;
+    long long blocks = (total + 255) / 256;
+    if (blocks > num_sms * 16LL) blocks = num_sms * 16LL;
+    return launch_pdl(bwd_upsample_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0,
+                      stream, static_cast<const uint4*>(dy), N, Ho, Wo, C / 8, s, Hu, Wu,
+                      static_cast<uint4*>(u));
+}
 
 // Device address of the scratch on the current device (called once per device, with
 // that device current, by the entry point's first call there).

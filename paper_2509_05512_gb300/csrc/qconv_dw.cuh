@@ -11,7 +11,9 @@
 //
 // Both MMA operands come straight from the NHWC tensors: a TMA box of 64 channels x P
 // pixels (P = Ht rows x Wbox columns of one image) lands as P rows of 128 bytes, the
-// MN-major SWIZZLE_128B layout (channels along M or N, pixels along K).  A holds two such
+// MN-major SWIZZLE_128B layout (channels along M or N, pixels along K).  For a strided
+// convolution the x box traverses every stride-th input pixel (the tensor map's element
+// strides), so it lands in the same layout as the dy box of the output pixels it serves.  A holds two such
 // boxes ("units": one tap's window of x, one 64-channel chunk) stacked to M = 128; B holds
 // ncols / 64 boxes of dy, N = ncols.  A CTA owns a_per unit pairs (one TMEM accumulator of
 // ncols fp32 columns each) and one ncols-wide group of output channels, for a contiguous
@@ -31,11 +33,15 @@ constexpr int BOX_ROW = 128;  // bytes of one pixel's 64 channels
 constexpr int BAR_BYTES = 256;
 // Shared memory reserved past the barriers: the MMA reads of the last stage stay inside the
 // CTA's allocation even for a descriptor whose two byte offsets were read the other way
-// round (one pixel block plus 4 KB beyond the stage).
-__host__ __device__ constexpr int tail_bytes(int P) { return P * BOX_ROW + 4096; }
+// round (one pixel block plus 4 KB beyond the stage), and a strided x box (stride s) stays
+// inside it even if the copy brought its s * s untraversed elements as well.
+__host__ __device__ constexpr int tail_bytes(int P, int stride = 1) {
+    return P * BOX_ROW + 4096 + (stride * stride - 1) * P * BOX_ROW;
+}
 
 struct DwParams {
     int Ho, Wo, Qin, Qout, kh, kw, pad, taps;
+    int stride;              // the x boxes traverse every stride-th pixel (element strides)
     int Wbox, Ht, P;         // pixel block: Ht rows x Wbox columns = P pixels
     int rblocks;             // pixel blocks per image
     long long kblocks;       // N * rblocks
@@ -148,7 +154,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const int tap = u / p.nxc, xc = u - tap * p.nxc;
                     const int dh = tap / p.kw, dw = tap - dh * p.kw;
                     tma_load_4d(dst + k * box_bytes, &tmap_x, fb, xc * 64, dw - p.pad,
-                                r0 - p.pad + dh, n, pol);
+                                r0 * p.stride - p.pad + dh, n, pol);
                 }
                 const uint32_t ydst = dst + 2 * p.a_per * box_bytes;
                 for (int c = 0; c < p.nyb; ++c)

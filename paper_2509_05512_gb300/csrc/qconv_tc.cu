@@ -846,10 +846,11 @@ constexpr int DW_SMEM_MAX = 232448;  // dynamic shared memory a CTA may opt into
 
 // Tiling of the tensor-core weight gradient (see qconv_dw.cuh); false if the shape has none.
 bool dw_plan(const ConvShape& s, int num_sms, dwk::DwParams* p) {
-    if (s.stride != 1 || s.Cin % 64 != 0 || s.Cout % 64 != 0) return false;
+    if (s.stride < 1 || s.stride > 2 || s.Cin % 64 != 0 || s.Cout % 64 != 0) return false;
     if (s.Cout > 256 && s.Cout % 256 != 0) return false;
     dwk::DwParams q = {};
     q.sep = s.sep ? 1 : 0;
+    q.stride = s.stride;
     q.Ho = s.Ho; q.Wo = s.Wo; q.Qin = s.Qin; q.Qout = s.Qout;
     q.kh = s.kh; q.kw = s.kw; q.pad = s.pad; q.taps = s.kh * s.kw;
     q.nxc = s.Cin / 64;
@@ -869,14 +870,15 @@ bool dw_plan(const ConvShape& s, int num_sms, dwk::DwParams* p) {
         const int wcand[2] = {(s.Wo + 7) / 8 * 8, (s.Wo + 15) / 16 * 16};
         for (int wc = 0; wc < 2; ++wc) {
             const int Wbox = wcand[wc];
-            if (Wbox > 256) continue;
+            if (Wbox * s.stride > 256) continue;  // the x box spans stride * Wbox columns
             for (int Ht = 1; Ht <= 8; ++Ht) {
                 const int P = Wbox * Ht;
-                if (P % 16 != 0 || P > 256) continue;
+                if (P % 16 != 0 || P > 256 || Ht * s.stride > 256) continue;
                 const long long stage =
                     static_cast<long long>(2 * a_per + q.nyb) * P * dwk::BOX_ROW;
-                long long stages =
-                    (DW_SMEM_MAX - 1024 - dwk::BAR_BYTES - dwk::tail_bytes(P)) / stage;
+                long long stages = (DW_SMEM_MAX - 1024 - dwk::BAR_BYTES -
+                                    dwk::tail_bytes(P, s.stride)) /
+                                   stage;
                 if (stages > dwk::MAX_STAGES) stages = dwk::MAX_STAGES;
                 if (stages < 2) continue;
                 const int rb = (s.Ho + Ht - 1) / Ht;
@@ -910,16 +912,20 @@ bool dw_plan(const ConvShape& s, int num_sms, dwk::DwParams* p) {
     return true;
 }
 
-// [N][H][W][C] bf16, boxes of 64 channels x Wbox columns x Ht rows of one image, SW128.
+// [N][H][W][C] bf16, boxes of 64 channels x Wbox columns x Ht rows of one image, SW128;
+// with `step` > 1 the box traverses every step-th column and row (it spans step * Wbox
+// columns and step * Ht rows, and the copy brings Wbox x Ht pixels).
 bool encode_dw_map(CUtensorMap* map, const void* t, int C, int W, int H, int N, int Wbox,
-                   int Ht) {
+                   int Ht, int step = 1) {
     const cuuint64_t dims[4] = {static_cast<cuuint64_t>(C), static_cast<cuuint64_t>(W),
                                 static_cast<cuuint64_t>(H), static_cast<cuuint64_t>(N)};
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(C) * 2,
                                    static_cast<cuuint64_t>(C) * 2 * W,
                                    static_cast<cuuint64_t>(C) * 2 * W * H};
-    const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(Wbox), static_cast<cuuint32_t>(Ht), 1};
-    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const cuuint32_t box[4] = {64, static_cast<cuuint32_t>(Wbox * step),
+                               static_cast<cuuint32_t>(Ht * step), 1};
+    const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(step), static_cast<cuuint32_t>(step),
+                                1};
     const CUresult r = g_encode_tiled(
         map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(t), dims, strides, box, estr,
         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -1110,7 +1116,7 @@ cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* 
         return cudaErrorInvalidValue;
     }
     CUtensorMap mx, mdy;
-    if (!encode_dw_map(&mx, x, s.Cin, s.W, s.H, s.N, p.Wbox, p.Ht) ||
+    if (!encode_dw_map(&mx, x, s.Cin, s.W, s.H, s.N, p.Wbox, p.Ht, s.stride) ||
         !encode_dw_map(&mdy, dy, s.Cout, s.Wo, s.Ho, s.N, p.Wbox, p.Ht)) {
         snprintf(err, errlen, "tensor-map encode failed for the weight gradient");
         return cudaErrorInvalidValue;
@@ -1126,7 +1132,7 @@ cudaError_t launch_bwd_weight_tc(const ConvShape& s, const void* x, const void* 
     p.dwj = dw[2];
     p.dwk = dw[3];
     const int smem = p.stages * static_cast<int>(p.stage_bytes) + dwk::BAR_BYTES +
-                     dwk::tail_bytes(p.P) + 1024;
+                     dwk::tail_bytes(p.P, s.stride) + 1024;
     static std::atomic<unsigned long long> attr_done{0};
     cudaError_t e = set_smem_once(dwk::qconv_dw_kernel, DW_SMEM_MAX, attr_done);
     if (e != cudaSuccess) return e;

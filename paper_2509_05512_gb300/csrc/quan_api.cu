@@ -216,37 +216,52 @@ quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H,
                     workspace_bytes, workspace ? "" : ", NULL");
     const size_t dxb = x_bytes(s, 2), dyb = y_bytes(s, 2), wb = w_bytes(s, 2);
     for (int L = 0; L < 4; ++L)
-        if (overlaps(dx, dxb, w[L], wb) || overlaps(workspace, need, w[L], wb))
+        if (overlaps(dx, dxb, w[L], wb) || overlaps(workspace, workspace_bytes, w[L], wb))
             return fail(QUAN_ERR_INVALID_ARG, "dx or workspace overlaps a weight tensor");
-    if (overlaps(dx, dxb, dy, dyb) || overlaps(workspace, need, dy, dyb) ||
-        overlaps(workspace, need, dx, dxb))
+    if (overlaps(dx, dxb, dy, dyb) || overlaps(workspace, workspace_bytes, dy, dyb) ||
+        overlaps(workspace, workspace_bytes, dx, dxb))
         return fail(QUAN_ERR_INVALID_ARG, "dx, dy and workspace must not overlap");
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
     cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
-    // The stride-1 full form is a forward convolution of dy with the transformed letters
-    // (output channels Cin, input channels Cout, padding kh - 1 - pad).
+    // The input gradient is a forward convolution of dy with the transformed letters
+    // (output channels Cin, input channels Cout, padding kh - 1 - pad, stride 1); for a
+    // strided forward, of dy with zeros inserted (u, after the letters in the workspace),
+    // when the workspace holds it.
     quan::ConvShape t;
     const quan::EpilogueArgs none{nullptr, nullptr, nullptr, nullptr};
     const size_t per = need / 4;
     const void* tw[4];
     for (int L = 0; L < 4; ++L) tw[L] = static_cast<const char*>(workspace) + L * per;
-    bool tc_ok = stride == 1 && kh == kw && pad <= kh - 1 && cc == 103 &&
-                 geometry(&t, N, s.Ho, s.Wo, Cout, Cin, kh, kw, 1, kh - 1 - pad) == QUAN_OK &&
-                 quan::tc_supported(t, dy, tw, dx, none);
+    const int Hu = H + 2 * pad - kh + 1, Wu = W + 2 * pad - kw + 1;
+    void* u = static_cast<char*>(workspace) + (need + 255) / 256 * 256;
+    const size_t ub = static_cast<size_t>(N) * Hu * Wu * Cout * 2;
+    const bool strided = stride > 1;
+    const void* src = strided ? u : dy;
+    bool tc_ok = kh == kw && pad <= kh - 1 && cc == 103 &&
+                 (!strided || workspace_bytes >= (need + 255) / 256 * 256 + ub) &&
+                 geometry(&t, N, strided ? Hu : s.Ho, strided ? Wu : s.Wo, Cout, Cin, kh, kw, 1,
+                          kh - 1 - pad) == QUAN_OK &&
+                 t.Ho == H && t.Wo == W && quan::tc_supported(t, src, tw, dx, none);
     // separable form: the transposed-separable MMA mode (Qin, Qout multiples of 16)
     if (separable) t.sep = 2;
     if (separable && (Cin % 64 != 0 || Cout % 64 != 0)) tc_ok = false;
     const int path = g_path.load();
     if (path == QUAN_PATH_TC && !tc_ok)
         return fail(QUAN_ERR_UNSUPPORTED,
-                    "tensor-core input gradient needs stride 1, a square filter, pad < kh, "
-                    "sm_103 and Cin/4, Cout/4 multiples of 16 with 16-byte aligned tensors");
+                    "tensor-core input gradient needs a square filter, pad < kh, sm_103, "
+                    "Cin/4 and Cout/4 multiples of 16 with 16-byte aligned tensors, and for "
+                    "a strided forward quan_qconv2d_bwd_data_workspace_size_ex bytes");
     if (tc_ok && path != QUAN_PATH_SIMT) {
         e = quan::launch_bwd_transform(Cin, Cout, kh, kw, w, !separable, workspace, num_sms,
                                        cs);
         if (e != cudaSuccess) return cuda_fail(e, "bwd_transform launch");
+        if (strided) {
+            e = quan::launch_bwd_upsample(dy, N, s.Ho, s.Wo, Cout, stride, Hu, Wu, u, num_sms,
+                                          cs);
+            if (e != cudaSuccess) return cuda_fail(e, "bwd_upsample launch");
+        }
         quan::TcOptions opt;
         opt.kappa = g_kappa.load();
         opt.bnq = g_bnq.load();
@@ -257,7 +272,7 @@ quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H,
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
-        e = quan::launch_qconv_tc(t, dy, tw, none, dx, opt, num_sms, cs, err, sizeof(err));
+        e = quan::launch_qconv_tc(t, src, tw, none, dx, opt, num_sms, cs, err, sizeof(err));
         if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
         if (e != cudaSuccess) return cuda_fail(e, "qconv_tc launch");
         t_last_path = QUAN_PATH_TC;
@@ -291,12 +306,12 @@ quan_status_t run_bwd_weight(const void* x, const void* dy, int N, int H, int W,
         if (reinterpret_cast<uintptr_t>(dw[L]) % 4 != 0)
             return fail(QUAN_ERR_INVALID_ARG, "weight gradients must be 4-byte aligned");
     }
-    // tensor cores at stride 1, both forms (the shape checks need no device)
+    // tensor cores at stride 1 or 2, both forms (the shape checks need no device)
     const bool tc_shape = quan::bwd_weight_tc_supported(s, x, dy);
     const int path = g_path.load();
     if (path == QUAN_PATH_TC && !tc_shape)
         return fail(QUAN_ERR_UNSUPPORTED,
-                    "tensor-core weight gradient needs stride 1, Cin and Cout multiples of 64 "
+                    "tensor-core weight gradient needs stride 1 or 2, Cin and Cout multiples of 64 "
                     "(Cout <= 256 or a multiple of 256) and 16-byte aligned x and dy");
     int num_sms = 0, cc = 0;
     cudaError_t e;
@@ -395,6 +410,17 @@ quan_status_t quan_poincare_fwd(const float* rgb, long long npix, void* out,
 size_t quan_qconv2d_bwd_data_workspace_size(int Cin, int Cout, int kh, int kw) {
     if (Cin < 4 || Cout < 4 || kh < 1 || kw < 1 || Cin % 4 || Cout % 4) return 0;
     return quan::bwd_data_workspace_bytes(Cin, Cout, kh, kw);
+}
+
+size_t quan_qconv2d_bwd_data_workspace_size_ex(int N, int H, int W, int Cin, int Cout, int kh,
+                                               int kw, int stride, int pad) {
+    quan::ConvShape s;
+    if (geometry(&s, N, H, W, Cin, Cout, kh, kw, stride, pad) != QUAN_OK) return 0;
+    const size_t letters = quan::bwd_data_workspace_bytes(Cin, Cout, kh, kw);
+    if (stride == 1) return letters;
+    const size_t Hu = static_cast<size_t>(H) + 2 * pad - kh + 1;
+    const size_t Wu = static_cast<size_t>(W) + 2 * pad - kw + 1;
+    return (letters + 255) / 256 * 256 + static_cast<size_t>(N) * Hu * Wu * Cout * 2;
 }
 
 quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* wi,

@@ -79,6 +79,8 @@ def load():
         lib.quan_qconv2d_bwd_data_static.argtypes = [_vp] * 5 + [_i] * 9 + [_vp, _vp]
         lib.quan_qconv2d_bwd_data_workspace_size.argtypes = [_i] * 4
         lib.quan_qconv2d_bwd_data_workspace_size.restype = ctypes.c_size_t
+        lib.quan_qconv2d_bwd_data_workspace_size_ex.argtypes = [_i] * 9
+        lib.quan_qconv2d_bwd_data_workspace_size_ex.restype = ctypes.c_size_t
         _bwd_weight_args = [_vp] * 2 + [_i] * 9 + [_vp] * 5
         lib.quan_qconv2d_bwd_weight.argtypes = _bwd_weight_args
         lib.quan_qconv2d_sep_bwd_weight.argtypes = _bwd_weight_args
@@ -278,6 +280,11 @@ def quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw) -> int:
     return load().quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw)
 
 
+def quan_qconv2d_bwd_data_workspace_size_ex(N, H, W, Cin, Cout, kh, kw, stride, pad) -> int:
+    return load().quan_qconv2d_bwd_data_workspace_size_ex(N, H, W, Cin, Cout, kh, kw, stride,
+                                                          pad)
+
+
 def quan_qconv2d_bwd_data(dy, wr, wi, wj, wk, N, H, W, Cin, Cout, kh, kw, stride, pad, workspace,
                           workspace_bytes, dx, stream=None) -> None:
     _check(load().quan_qconv2d_bwd_data(_ptr(dy), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), N, H,
@@ -317,13 +324,14 @@ def quan_qconv2d_sep_bwd_weight(x, dy, N, H, W, Cin, Cout, kh, kw, stride, pad, 
 def qconv2d_backward_data(dy, wr, wi, wj, wk, *, H, W, stride=1, pad=0, separable=False,
                           workspace=None, out=None, stream=None):
     """Input gradient of the pre-epilogue convolution: dy [N, Ho, Wo, Cout] (bf16, CUDA) ->
-    dx [N, H, W, Cin] bf16.  `workspace` (a uint8 CUDA tensor of at least
-    quan_qconv2d_bwd_data_workspace_size bytes) is allocated when not given."""
+    dx [N, H, W, Cin] bf16.  `workspace` (a uint8 CUDA tensor) is allocated when not given,
+    with quan_qconv2d_bwd_data_workspace_size_ex bytes (the tensor-core path of strided
+    layers included)."""
     import torch
     N, Ho, Wo, Cout = dy.shape
     Qout, kh, kw, Qin = wr.shape
     Cin = 4 * Qin
-    need = quan_qconv2d_bwd_data_workspace_size(Cin, Cout, kh, kw)
+    need = quan_qconv2d_bwd_data_workspace_size_ex(N, H, W, Cin, Cout, kh, kw, stride, pad)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=dy.device)
     if out is None:

@@ -118,6 +118,12 @@ def test_backward_workspace_size(lib):
     assert lib.quan_qconv2d_bwd_data_workspace_size(4, 64, 7, 7) == 4 * 1 * 49 * 16 * 2
     assert lib.quan_qconv2d_bwd_data_workspace_size(6, 64, 3, 3) == 0
     assert lib.quan_qconv2d_bwd_data_workspace_size(64, 64, 0, 3) == 0
+    # strided: the letters (rounded to 256 bytes) and dy spread out to H + 2 pad - kh + 1 rows
+    lt = lib.quan_qconv2d_bwd_data_workspace_size(64, 128, 3, 3)
+    assert lib.quan_qconv2d_bwd_data_workspace_size_ex(2, 8, 8, 64, 128, 3, 3, 1, 1) == lt
+    assert lib.quan_qconv2d_bwd_data_workspace_size_ex(2, 8, 8, 64, 128, 3, 3, 2, 1) == \
+        (lt + 255) // 256 * 256 + 2 * 8 * 8 * 128 * 2
+    assert lib.quan_qconv2d_bwd_data_workspace_size_ex(2, 8, 8, 64, 128, 3, 3, 0, 1) == 0
 
 
 @pytest.mark.parametrize("sep", [False, True])
@@ -146,11 +152,11 @@ def test_backward_weight_invalid_arguments(lib, sep, bad):
 
 
 def test_backward_weight_tensor_core_shapes(lib):
-    # the tensor-core weight gradient takes stride 1, Cin and Cout multiples of 64:
+    # the tensor-core weight gradient takes stride 1 or 2, Cin and Cout multiples of 64:
     # forcing it on another shape fails on the host
     assert lib.quan_set_path(quan.QUAN_PATH_TC) == quan.QUAN_OK
     try:
-        assert _bwd_weight(lib, stride=2) == quan.QUAN_ERR_UNSUPPORTED
+        assert _bwd_weight(lib, stride=3) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, Cin=48) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, Cout=320) == quan.QUAN_ERR_UNSUPPORTED
         assert _bwd_weight(lib, x=FAKE + 8) == quan.QUAN_ERR_UNSUPPORTED  # misaligned for TMA

@@ -38,17 +38,26 @@ def layer(spec):
     return d
 
 
-def gpu_bwd_data(d, separable=False, path=quan.QUAN_PATH_AUTO):
+def gpu_bwd_data(d, separable=False, path=quan.QUAN_PATH_AUTO, letters_only=False):
+    """letters_only: a workspace for the transformed letters alone (a strided layer then
+    runs on CUDA cores); else the larger one of quan_qconv2d_bwd_data_workspace_size_ex."""
     spec = d["spec"]
     dy = to_dev(d["dy"], "bf16")
     w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    if letters_only:
+        nb = quan.quan_qconv2d_bwd_data_workspace_size(spec.Cin, spec.Cout, spec.kh, spec.kw)
+    else:
+        nb = quan.quan_qconv2d_bwd_data_workspace_size_ex(spec.N, spec.H, spec.W, spec.Cin,
+                                                          spec.Cout, spec.kh, spec.kw,
+                                                          spec.stride, spec.pad)
+    ws = torch.empty(nb, dtype=torch.uint8, device="cuda")
     n = spec.N * spec.H * spec.W * spec.Cin
     pad = 4096
     buf = torch.full((n + 2 * pad,), float("nan"), dtype=torch.bfloat16, device="cuda")
     dx = buf[pad:pad + n].view(spec.N, spec.H, spec.W, spec.Cin)
     quan.quan_set_path(path)
     quan.qconv2d_backward_data(dy, *w, H=spec.H, W=spec.W, stride=spec.stride, pad=spec.pad,
-                               separable=separable, out=dx)
+                               separable=separable, workspace=ws, out=dx)
     torch.cuda.synchronize()
     assert torch.isnan(buf[:pad].float()).all() and torch.isnan(buf[pad + n:].float()).all()
     st, bits = quan.quan_device_status()
@@ -85,7 +94,7 @@ def oracle_bwd_weight(d, separable=False):
 
 
 def tc_weight_shape(spec):
-    return (spec.stride == 1 and spec.Cin % 64 == 0 and spec.Cout % 64 == 0 and
+    return (spec.stride in (1, 2) and spec.Cin % 64 == 0 and spec.Cout % 64 == 0 and
             (spec.Cout <= 256 or spec.Cout % 256 == 0))
 
 
@@ -113,6 +122,12 @@ TC_CASES = [
     ("pad0", 2, 11, 12, 64, 128, 3, 1, 0),           # transposed padding 2
     ("k5_pad2", 1, 12, 11, 64, 64, 5, 1, 2),
     ("k5_pad1", 1, 12, 11, 128, 64, 5, 1, 1),        # transposed padding 3
+    # strided: dy spread out with zeros in the workspace, then the stride-1 convolution
+    ("s2_odd", 2, 15, 17, 64, 128, 3, 2, 1),
+    ("s2_16to16", 1, 16, 16, 64, 64, 3, 2, 1),       # weight-stationary kernel
+    ("s2_shortcut", 2, 14, 14, 64, 128, 1, 2, 0),
+    ("s2_imagenet", 1, 56, 56, 256, 512, 3, 2, 1),
+    ("s2_5x5", 1, 13, 12, 64, 64, 5, 2, 2),
 ]
 
 
@@ -141,7 +156,7 @@ SIMT_CASES = [
 def test_bwd_data_cuda_cores(case):
     name, N, H, W, Cin, Cout, k, s, p = case
     d = layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(601, len(name))))
-    got, path, kernel = gpu_bwd_data(d)
+    got, path, kernel = gpu_bwd_data(d, letters_only=True)
     assert path == quan.QUAN_PATH_SIMT and kernel == "bwd_data_simt_kernel"
     assert_bf16_close(got, oracle_bwd_data(d), name + " dx")
 
@@ -164,11 +179,14 @@ def test_bwd_data_paths_agree():
     assert_bf16_close(simt, ref, "simt")
 
 
-def test_bwd_data_tc_rejects_strided():
+def test_bwd_data_tc_strided_needs_the_larger_workspace():
     d = layer(inputs.small_layer("tc_s2", 1, 9, 9, 64, 64, 3, 2, 1, seed=(604, 0)))
     with pytest.raises(quan.QuanError) as ei:
-        gpu_bwd_data(d, path=quan.QUAN_PATH_TC)
+        gpu_bwd_data(d, path=quan.QUAN_PATH_TC, letters_only=True)
     assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+    got, path, _ = gpu_bwd_data(d, path=quan.QUAN_PATH_TC)
+    assert path == quan.QUAN_PATH_TC
+    assert_bf16_close(got, oracle_bwd_data(d), "tc_s2 dx")
 
 
 def test_bwd_data_workspace_reuse():
@@ -215,6 +233,12 @@ TC_WEIGHT_CASES = [
     ("dw_cout512", 1, 6, 7, 64, 512, 3, 1, 1),       # two output-channel groups
     ("dw_tiny", 1, 1, 1, 64, 64, 3, 1, 1),
     ("dw_wide_row", 1, 3, 200, 64, 64, 3, 1, 1),     # 200 columns: one row per block
+    # stride 2: the x boxes traverse every second input pixel
+    ("dw_s2", 2, 15, 17, 64, 128, 3, 2, 1),
+    ("dw_s2_even", 1, 16, 16, 128, 64, 3, 2, 1),
+    ("dw_s2_shortcut", 2, 14, 14, 64, 128, 1, 2, 0),
+    ("dw_s2_imagenet", 1, 56, 56, 256, 512, 3, 2, 1),  # one image of the stride-2 layer
+    ("dw_s2_5x5", 1, 13, 12, 64, 64, 5, 2, 2),
 ]
 
 
@@ -248,7 +272,7 @@ def test_separable_backward(case):
     name, N, H, W, Cin, Cout, k, s, p = case
     d = layer(inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(608, len(name))))
     got, path, kernel = gpu_bwd_data(d, separable=True)
-    if s == 1 and Cin % 64 == 0 and Cout % 64 == 0:
+    if Cin % 64 == 0 and Cout % 64 == 0:
         assert kernel.startswith("qconv_tc_kernel<sep_t,"), kernel
     else:
         assert kernel == "bwd_data_simt_kernel<sep>", kernel
