@@ -6,7 +6,9 @@ contraction, bias/IQBN/activation epilogue, store) over one batch of the workloa
 Default workload: the CIFAR-shaped layer N=128, 32x32, 64->64 real channels, 3x3 s1
 p1, fused IQBN + ReLU, bf16 in / fp32 accumulate.  Other workloads: --workload
 c2a | c2b | c3a | c3b (ImageNet / detection-neck layers) | backbone (ResNet-18-style,
-images/s).
+images/s; --act silu, --no-fuse) | poincare (the Eq. 4 input mapping) | iqbn
+(training-mode IQBN); on a layer workload, --variant separable (Eq. 7) and --pass bwd
+(the input and weight gradients).
 
 Prints one JSON line.  Under torchrun every rank runs its own copy of the workload on
 its own GPU (the batch shards with no exchange step: weak scaling); the timed region
