@@ -53,3 +53,13 @@ def test_backbone_activation_variant():
         else:
             assert a.spec.act == inputs.ACT_RELU and b.spec.act == inputs.ACT_SILU
         assert a.spec.seed == b.spec.seed  # same weights
+
+
+def test_grad_output_seeded_and_prefix():
+    spec = inputs.small_layer("g", 4, 6, 5, 16, 32, 3, 2, 1, seed=(7, 3))
+    a = inputs.grad_output(spec)
+    assert a.shape == (4, spec.Ho, spec.Wo, 32) and a.dtype.name == "uint16"
+    np.testing.assert_array_equal(a, inputs.grad_output(spec))      # same seed, same bits
+    np.testing.assert_array_equal(a[:2], inputs.grad_output(spec, n_images=2))
+    other = inputs.grad_output(inputs.small_layer("g", 4, 6, 5, 16, 32, 3, 2, 1, seed=(7, 4)))
+    assert (a != other).any()
