@@ -204,11 +204,12 @@ quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* 
  * device memory: code running where cudaMalloc is off limits (its implicit device-wide
  * synchronisation would stall other work, or a framework owns all device memory through
  * its own pool), or a plain C caller with no allocator at hand.  The paper has no
- * counterpart.  The transformed letters go to a scratch buffer of 2 MiB (2097152 bytes)
- * that the library keeps in static device memory: every GPU that loads the library holds
- * it until the process exits; the call itself allocates and frees nothing.
- * Same arguments (minus the workspace), paths, results and errors as
- * quan_qconv2d_bwd_data, plus QUAN_ERR_UNSUPPORTED when
+ * counterpart.  The transformed letters (and, for a strided forward, the spread-out dy
+ * when both fit) go to a scratch buffer of 2 MiB (2097152 bytes) that the library keeps in
+ * static device memory: every GPU that loads the library holds it until the process
+ * exits; the call itself allocates and frees nothing.
+ * Same arguments (minus the workspace), results and errors as quan_qconv2d_bwd_data with
+ * a 2 MiB workspace, and the paths that workspace allows, plus QUAN_ERR_UNSUPPORTED when
  * quan_qconv2d_bwd_data_workspace_size exceeds 2 MiB (e.g. 1024 -> 1024 real channels
  * with a 3x3 filter: use quan_qconv2d_bwd_data with a workspace there).
  *   Sharing  every call on a device uses the same buffer, which keeps the last call's
