@@ -581,12 +581,16 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
                                        size_t workspace_bytes, void* out,
                                        quan_stream_t stream) {
     const void* w[4] = {wr, wi, wj, wk};
+    if (!x || !wr || !wi || !wj || !wk || !out)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
     quan::ConvShape s;
-    // validate() checks the convolution; `out` here is the smaller pooled tensor
-    quan_status_t st = validate(&s, x, w, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
-                                kw, stride, pad, act, nullptr, workspace ? workspace : out, 2);
+    quan_status_t st = geometry(&s, N, H, W, Cin, Cout, kh, kw, stride, pad);
     if (st != QUAN_OK) return st;
-    if (!out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    if ((iqbn_scale == nullptr) != (iqbn_shift == nullptr))
+        return fail(QUAN_ERR_INVALID_ARG, "iqbn_scale and iqbn_shift must both be given or both NULL");
+    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
+    s.act = act;
     const int pw = (s.Wo - 1) / 2 + 1, ph = (s.Ho - 1) / 2 + 1;
     const size_t need =
         static_cast<size_t>(N) * s.Ho * (pw + quan::HPOOL_SIDE_SLOTS) * Cout * 2;
@@ -594,10 +598,19 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
     if (!workspace || workspace_bytes < need)
         return fail(QUAN_ERR_INVALID_ARG, "workspace must hold %zu bytes (got %zu%s)", need,
                     workspace_bytes, workspace ? "" : ", NULL");
-    if (overlaps(out, ob, workspace, need) || overlaps(out, ob, x, x_bytes(s, 2)) ||
-        overlaps(out, ob, wr, w_bytes(s, 2)) || overlaps(out, ob, wi, w_bytes(s, 2)) ||
-        overlaps(out, ob, wj, w_bytes(s, 2)) || overlaps(out, ob, wk, w_bytes(s, 2)))
-        return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input or the workspace");
+    // the two tensors written (the workspace and out) against each other and every input
+    const size_t xb = x_bytes(s, 2), wb = w_bytes(s, 2), vb = static_cast<size_t>(Cout) * 4;
+    const void* written[2] = {workspace, out};
+    const size_t wsz[2] = {need, ob};
+    if (overlaps(out, ob, workspace, need))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps the workspace");
+    for (int k = 0; k < 2; ++k)
+        if (overlaps(written[k], wsz[k], x, xb) || overlaps(written[k], wsz[k], wr, wb) ||
+            overlaps(written[k], wsz[k], wi, wb) || overlaps(written[k], wsz[k], wj, wb) ||
+            overlaps(written[k], wsz[k], wk, wb) || overlaps(written[k], wsz[k], bias, vb) ||
+            overlaps(written[k], wsz[k], iqbn_scale, vb) ||
+            overlaps(written[k], wsz[k], iqbn_shift, vb))
+            return fail(QUAN_ERR_INVALID_ARG, "out or the workspace overlaps an input");
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
