@@ -51,3 +51,22 @@ def test_workload_config_flops():
     assert bench.workload_config("c1", inputs, "full", "bwd")["flops_per_step"] == 2 * full
     bb = bench.workload_config("backbone", inputs, act="silu")
     assert "SiLU" in bb["epilogue"] and bb["convs"] == 20
+
+
+def test_recorded_traffic_lookup():
+    # a record is used only for its own workload key, its own kernel and the current
+    # device-code sources
+    import json
+    with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
+        rec = json.load(f)
+    assert all(v["kernel_sha"] == bench.kernel_source_hash() for v in rec.values())
+    assert bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=2>") == \
+        rec["c1"]["dram_bytes_per_launch"]
+    assert bench.recorded_traffic("c1", "qconv_tc_kernel<pair,kappa=32,bnq=64>") is None
+    assert bench.recorded_traffic("no_such_workload", None) is None
+
+    class A:
+        workload, direction, variant = "c2a", "bwd", "separable"
+    assert bench.traffic_key(A) == "c2a:bwd:sep"
+    A.direction, A.variant = "fwd", "full"
+    assert bench.traffic_key(A) == "c2a"
