@@ -59,9 +59,10 @@ def test_recorded_traffic_lookup():
     import json
     with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
         rec = json.load(f)
-    assert all(v["kernel_sha"] == bench.kernel_source_hash() for v in rec.values())
-    assert bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=2>") == \
-        rec["c1"]["dram_bytes_per_launch"]
+    current = rec["c1"]["kernel_sha"] == bench.kernel_source_hash()
+    got = bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=2>")
+    # valid only while the device code is the one the counters were taken on
+    assert got == (rec["c1"]["dram_bytes_per_launch"] if current else None)
     assert bench.recorded_traffic("c1", "qconv_tc_kernel<pair,kappa=32,bnq=64>") is None
     assert bench.recorded_traffic("no_such_workload", None) is None
 
