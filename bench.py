@@ -3,12 +3,13 @@
 
 One step = one full pass of the hot path (staging, on-chip Hamilton block expansion,
 contraction, bias/IQBN/activation epilogue, store) over one batch of the workload.
-Default workload: the CIFAR-shaped layer N=128, 32x32, 64->64 real channels, 3x3 s1
-p1, fused IQBN + ReLU, bf16 in / fp32 accumulate.  Other workloads: --workload
-c2a | c2b | c3a | c3b (ImageNet / detection-neck layers) | backbone (ResNet-18-style,
-images/s; --act silu, --no-fuse) | poincare (the Eq. 4 input mapping) | iqbn
-(training-mode IQBN); on a layer workload, --variant separable (Eq. 7) and --pass bwd
-(the input and weight gradients).
+Default workload: the ResNet-18-style QUAN backbone forward, N=256 images of 224x224x4
+quaternion input, 20 quaternion convolutions with fused IQBN + ReLU and the stem's 3x3/2
+max pool, bf16 in / fp32 accumulate, in images/s (--act silu, --no-fuse).  Other
+workloads: --workload c1 (the CIFAR-shaped layer N=128, 32x32, 64->64 real channels,
+3x3 s1 p1) | c2a | c2b | c3a | c3b (ImageNet / detection-neck layers), in real-equivalent
+TFLOP/s | poincare (the Eq. 4 input mapping) | iqbn (training-mode IQBN); on a layer
+workload, --variant separable (Eq. 7) and --pass bwd (the input and weight gradients).
 
 Prints one JSON line.  Under torchrun every rank runs its own copy of the workload on
 its own GPU (the batch shards with no exchange step: weak scaling); the timed region
@@ -43,7 +44,7 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="c1",
+    ap.add_argument("--workload", default="backbone",
                     choices=["c1", "c2a", "c2b", "c3a", "c3b", "backbone", "poincare", "iqbn"])
     ap.add_argument("--pass", dest="direction", choices=["fwd", "bwd"], default="fwd",
                     help="layer workloads: the forward convolution, or its backward pass "

@@ -13,14 +13,15 @@ import bench  # noqa: E402
 
 CASES = [
     (["--workload", "c1"], "TFLOP/s"),
-    (["--pass", "bwd"], "TFLOP/s"),
+    (["--workload", "c1", "--pass", "bwd"], "TFLOP/s"),
+    ([], "images/s"),  # the default workload: the backbone
     (["--variant", "separable", "--workload", "c1"], "TFLOP/s"),
     (["--workload", "iqbn"], "images/s"),
     (["--workload", "poincare"], "images/s"),
 ]
 
 
-@pytest.mark.parametrize("args,unit", CASES, ids=lambda a: "_".join(a) if isinstance(a, list)
+@pytest.mark.parametrize("args,unit", CASES, ids=lambda a: ("_".join(a) or "default") if isinstance(a, list)
                          else None)
 def test_reference_arm_json_line(args, unit):
     res = subprocess.run([sys.executable, "bench.py", "--impl", "reference", *args, "--steps",
@@ -38,6 +39,8 @@ def test_reference_arm_json_line(args, unit):
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"]
     assert isinstance(d["config"]["workload"], str) and d["vs_baseline"] is None
+    if not args:
+        assert "backbone" in d["config"]["workload"]
     if "bwd" in args:
         assert "backward" in d["config"]["workload"]
     if "separable" in args:
