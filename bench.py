@@ -756,7 +756,7 @@ def workload_config(workload: str, inputs, variant: str = "full", direction: str
                 "N": c0.N, "H": c0.H, "W": c0.W, "convs": len(convs), "maxpool": 1,
                 "flops_per_step": sum(c.flops for c in convs),
                 "epilogue": "IQBN+%s (+residual)" % ("SiLU" if act == "silu" else "ReLU"),
-                "fusions": "stem conv + 3x3/2 max pool (horizontal max in the stem epilogue)"}
+                "fusions": "stem conv + 3x3/2 max pool in one kernel (only the pooled tensor is written)"}
     s = inputs.LAYERS[workload]
     cfg = {"workload": WORKLOAD_DESC[workload], "N": s.N, "H": s.H, "W": s.W, "Cin": s.Cin,
            "Cout": s.Cout, "kernel": "%dx%d" % (s.kh, s.kw), "stride": s.stride, "pad": s.pad,
@@ -1026,7 +1026,6 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
                 s0 = L.spec
                 nb += (runner.outs[1].numel() - s0.N * s0.Ho * s0.Wo * s0.Cout) * 2
                 name += " + maxpool3/2 (fused)"
-                kernels[i] = kernels[i] + " + vpool_rows_kernel"
         else:
             src = runner.outs[L.src]
             fl, nb = 0.0, src.numel() * 2 + runner.outs[i].numel() * 2

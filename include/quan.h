@@ -291,18 +291,21 @@ quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const fl
 
 /*
  * The 4-channel stem convolution followed by a 3x3, stride-2, padding-1 max pooling of
- * every real channel (Sec. III-D pooling rule), fused: the convolution's epilogue takes
- * the horizontal 3-wide max of each output row and writes only that (half the bytes of
- * the full output) to `workspace`; a second kernel takes the vertical max into `out`.
+ * every real channel (Sec. III-D pooling rule), in one kernel that writes only the pooled
+ * tensor: each CTA takes a band of pooled rows, computes the two convolution rows of each
+ * (an MMA whose rows are the signed block weight of Eq. 6 stacked for both rows and whose
+ * columns are the row's pixels) and takes the 3x3 max in registers.
  * The result is bit-identical to quan_qconv2d_fwd followed by quan_maxpool2d_fwd(k = 3,
- * stride 2, pad 1) (max commutes with the monotone bf16 rounding).
+ * stride 2, pad 1) (max commutes with the monotone bf16 rounding and, for ReLU or no
+ * activation, with the monotone affine IQBN step).
  *   arguments   those of quan_qconv2d_fwd; out is bf16 [N][Hp][Wp][Cout] with
  *               Hp = (Ho - 1) / 2 + 1, Wp = (Wo - 1) / 2 + 1 (Ho, Wo of the convolution)
- *   workspace   device scratch of at least quan_qconv2d_maxpool_workspace_size bytes
- *               (N Ho (Wp + 4) Cout bf16: each pooled row and 4 side slots for the columns
- *               whose pixels two producer warps hold), owned by the caller, overwritten
+ *   workspace   not used (may be NULL, workspace_bytes 0): quan_qconv2d_maxpool_workspace_size
+ *               returns 0 for every shape
  * Only the tensor-core pixel-pair shapes: sm_103, Cin = 4, Cout = 64, stride 2, even W,
- * Wo <= 128, 16-byte aligned tensors; otherwise QUAN_ERR_UNSUPPORTED.
+ * Wo <= 128, (kh + 2) x (filter pixel pairs per row, rounded up to even) <= 36 (the 7x7
+ * stem: 9 x 4), 16-byte aligned tensors; otherwise QUAN_ERR_UNSUPPORTED.  out must not
+ * overlap an input (QUAN_ERR_INVALID_ARG).
  */
 size_t quan_qconv2d_maxpool_workspace_size(int N, int H, int W, int Cout, int kh, int kw,
                                            int stride, int pad);

@@ -24,7 +24,7 @@ class BackboneRunner:
         self.act = act
         self.layers = inputs.backbone_layers(N=N, H=H, seed=seed, act=act)
         # stem + 3x3/2 max pool as one call (quan_qconv2d_maxpool_fwd): the stem's full
-        # output is never written, only its horizontally pooled rows (a workspace)
+        # output is never written, one kernel writes the pooled tensor
         L0, L1 = self.layers[0], self.layers[1]
         self.fused = (fuse_stem_pool and L0.kind == "conv" and L1.kind == "maxpool" and
                       L1.src == 0 and (L1.k, L1.stride, L1.pad) == (3, 2, 1))
@@ -45,7 +45,8 @@ class BackboneRunner:
                     "host": prm})
                 s = L.spec
                 if self.fused and len(self.outs) == 0:
-                    # the workspace of the fused call stands in for the stem's output
+                    # the fused call's workspace (none: 0 bytes) stands in for the stem's
+                    # output
                     self.ws_bytes = quan.quan_qconv2d_maxpool_workspace_size(
                         N, s.H, s.W, s.Cout, s.kh, s.kw, s.stride, s.pad)
                     self.outs.append(torch.empty(self.ws_bytes // 2, dtype=torch.bfloat16,

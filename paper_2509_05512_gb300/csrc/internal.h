@@ -130,20 +130,14 @@ cudaError_t launch_iqbn_apply(const void* x, long long npix, int C, const float*
                               const float* var, const float* gamma, const float* beta, float eps,
                               int act, void* out, int num_sms, cudaStream_t stream);
 
-// The 4-channel stem with the horizontal half of a 3x3/2 max pooling (padding 1) fused
-// into its epilogue: hp [N][Ho][pool_w + HPOOL_SIDE_SLOTS][64], pool_w = (Wo - 1) / 2 + 1
-// (the side slots complete the columns that straddle two TMEM quadrants).
-constexpr int HPOOL_SIDE_SLOTS = 4;
-bool tc_hpool_supported(const ConvShape& s, const void* x, const void* const w[4],
-                        const void* hp, const EpilogueArgs& ep);
-cudaError_t launch_qconv_tc_hpool(const ConvShape& s, const void* x, const void* const w[4],
-                                  const EpilogueArgs& ep, void* hp, int pool_w,
-                                  const TcOptions& opt, int num_sms, cudaStream_t stream,
-                                  char* err, size_t errlen);
-// Its vertical half: hp [N][Hin][W + side][C] -> out [N][(Hin - 1) / 2 + 1][W][C]
-// (C % 8 == 0, 16-byte aligned).
-cudaError_t launch_vpool_bf16(const void* hp, int N, int Hin, int W, int side, int C,
-                              void* out, cudaStream_t stream);
+// The 4-channel stem convolution and its 3x3/2, padding-1 max pooling in one kernel:
+// out [N][(Ho - 1) / 2 + 1][(Wo - 1) / 2 + 1][64] bf16 (Cin = 4, Cout = 64, stride 2, even W,
+// Wo <= 128).
+bool tc_stem_pool_supported(const ConvShape& s, const void* x, const void* const w[4],
+                            const void* out, const EpilogueArgs& ep);
+cudaError_t launch_qconv_stem_pool(const ConvShape& s, const void* x, const void* const w[4],
+                                   const EpilogueArgs& ep, void* out, const TcOptions& opt,
+                                   int num_sms, cudaStream_t stream, char* err, size_t errlen);
 
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,

@@ -109,73 +109,7 @@ __global__ void __launch_bounds__(512) maxpool_rows_kernel(const __nv_bfloat16* 
     }
 }
 
-// Second half of a 3x3/2 max pooling (padding 1) whose horizontal half the producing
-// convolution's epilogue already applied: out[n][r][j] = max of hp[n][y][j] over the rows
-// y = 2r - 1, 2r, 2r + 1 inside the image.  An hp row holds Wp pooled columns and `side`
-// side slots: column 16 q (q = 1 .. side - 1) also takes the max with slot q, the left
-// pixel that another warp of the producer held.  One CTA per output row; 16 bytes per
-// thread.  (Walking several output rows per thread to read each hp row once was slower:
-// fewer loads in flight.)
-template <int CV>  // 16-byte vectors per pixel (C / 8); 0: the run-time cv
-__global__ void __launch_bounds__(512) vpool_rows_kernel(const uint4* __restrict__ hp, int Hin,
-                                                         int Hout, int Wp, int side, int cv_rt,
-                                                         uint4* __restrict__ out) {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    asm volatile("griddepcontrol.wait;" ::: "memory");  // inputs from the previous kernel
-    const int cv = CV > 0 ? CV : cv_rt;
-    const int row = blockIdx.x;  // n * Hout + r
-    const int n = row / Hout, r = row - (row / Hout) * Hout;
-    const int in_vecs = (Wp + side) * cv, out_vecs = Wp * cv;
-    const uint4* src = hp + static_cast<long long>(n) * Hin * in_vecs;
-    uint4* dst = out + static_cast<long long>(row) * out_vecs;
-    for (int t = threadIdx.x; t < out_vecs; t += blockDim.x) {
-        const int j = t / cv, c = t - (t / cv) * cv;
-        const int q = j / 16;
-        const bool two = (j % 16 == 0) && q >= 1 && q < side;
-        float m[8];
-#pragma unroll
-        for (int v = 0; v < 8; ++v) m[v] = -INFINITY;
-#pragma unroll
-        for (int dy = -1; dy <= 1; ++dy) {
-            const int y = 2 * r + dy;
-            if (y < 0 || y >= Hin) continue;
-            const uint4* rowp = src + static_cast<long long>(y) * in_vecs;
-#pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                if (k == 1 && !two) break;
-                const uint4 raw = __ldg(rowp + (k == 0 ? t : (Wp + q) * cv + c));
-                const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-#pragma unroll
-                for (int v = 0; v < 4; ++v) {
-                    const float2 f = __bfloat1622float2(b2[v]);
-                    m[2 * v] = fmaxf(m[2 * v], f.x);
-                    m[2 * v + 1] = fmaxf(m[2 * v + 1], f.y);
-                }
-            }
-        }
-        uint4 raw;
-        __nv_bfloat162* b2 = reinterpret_cast<__nv_bfloat162*>(&raw);
-#pragma unroll
-        for (int v = 0; v < 4; ++v) b2[v] = __floats2bfloat162_rn(m[2 * v], m[2 * v + 1]);
-        dst[t] = raw;
-    }
-}
-
 }  // namespace
-
-cudaError_t launch_vpool_bf16(const void* hp, int N, int Hin, int W, int side, int C,
-                              void* out, cudaStream_t stream) {
-    const int Hout = (Hin - 1) / 2 + 1;
-    const long long ctas = static_cast<long long>(N) * Hout;
-    if (ctas == 0) return cudaSuccess;
-    if (ctas > 0x7fffffffLL || C % 8 != 0) return cudaErrorInvalidValue;
-    const int out_vecs = W * (C / 8);
-    const int t = out_vecs >= 512 ? 512 : ((out_vecs + 31) / 32) * 32;
-    auto kern = C == 64 ? vpool_rows_kernel<8> : vpool_rows_kernel<0>;
-    return launch_pdl(kern, dim3(static_cast<unsigned>(ctas)), dim3(t), 0, stream,
-                      static_cast<const uint4*>(hp), Hin, Hout, W, side, C / 8,
-                      static_cast<uint4*>(out));
-}
 
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream) {

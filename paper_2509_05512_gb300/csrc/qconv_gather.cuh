@@ -65,8 +65,6 @@ struct GatherParams {
     int per;          // stages owned by each issuer
     int segs;         // tiles per output row
     int num_tiles;
-    int pool_w;       // > 0: write the horizontal 3/2 max of each row, pool_w columns wide
-                      // (+ HPOOL_SIDE_SLOTS side slots)
 };
 
 struct GaCfg {
@@ -190,7 +188,7 @@ __device__ __forceinline__ void expand_block_weight(const ConvShape& s, const Ga
 // KH, NSP > 0: the filter height and pairs per filter row known at compile time, so the
 // MMA issue loop is fully unrolled with constant descriptor offsets; 0 = from the
 // parameters at run time.
-template <int KH, int NSP, bool HPOOL = false>
+template <int KH, int NSP>
 __global__ void __launch_bounds__(WIDE_THREADS, 1)
     qconv_pairs_kernel(const __grid_constant__ CUtensorMap tmap_x, const GatherParams p) {
     using C = GaCfg;
@@ -363,9 +361,8 @@ __global__ void __launch_bounds__(WIDE_THREADS, 1)
                 g.rows = left < GA_TILE_W ? left : GA_TILE_W;
                 return g;
             };
-            epilogue_direct64<decltype(geo), EPI_GROUPS, HPOOL>(
-                s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit, abort_flag, geo,
-                p.pool_w);
+            epilogue_direct64<decltype(geo), EPI_GROUPS>(
+                s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit, abort_flag, geo);
         }
     }
 

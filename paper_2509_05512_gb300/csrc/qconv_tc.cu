@@ -448,6 +448,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
 #include "qconv_ws.cuh"
 #include "qconv_gather.cuh"
+#include "qconv_stempool.cuh"
 #include "qconv_dw.cuh"
 
 // ---------------------------------------------------------------- host side
@@ -518,16 +519,17 @@ bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int chan
 }
 
 // Input of a 4-channel layer viewed as groups of G pixel pairs (16 G bytes):
-// [N][H][W/(2G)][8 G], boxes of `boxg` groups x kh input rows of one image, no swizzle
+// [N][H][W/(2G)][8 G], boxes of `boxg` groups x `rows` input rows of one image, no swizzle
 // (dense rows in shared memory).
-bool encode_x_pairs(CUtensorMap* map, const ConvShape& s, const void* x, int group, int boxg) {
+bool encode_x_pairs(CUtensorMap* map, const ConvShape& s, const void* x, int group, int boxg,
+                    int rows) {
     const cuuint64_t WG = static_cast<cuuint64_t>(s.W / (2 * group));
     const cuuint64_t eb = 16ull * group;
     const cuuint64_t dims[4] = {8ull * group, WG, static_cast<cuuint64_t>(s.H),
                                 static_cast<cuuint64_t>(s.N)};
     const cuuint64_t strides[3] = {eb, eb * WG, eb * WG * s.H};
     const cuuint32_t box[4] = {8u * group, static_cast<cuuint32_t>(boxg),
-                               static_cast<cuuint32_t>(s.kh), 1};
+                               static_cast<cuuint32_t>(rows), 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     const CUresult r = g_encode_tiled(
         map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
@@ -757,9 +759,8 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
                           const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
-                          cudaStream_t stream, char* err, size_t errlen, int pool_w = 0) {
+                          cudaStream_t stream, char* err, size_t errlen) {
     GatherParams prm;
-    prm.pool_w = pool_w;
     prm.s = s;
     prm.ep = ep;
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
@@ -792,16 +793,11 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         return cudaErrorInvalidValue;
     }
     prm.num_tiles = static_cast<int>(tiles);
-    if (pool_w > 0 && prm.segs != 1) {
-        snprintf(err, errlen, "fused pooling needs one tile per output row (Wo <= %d)",
-                 GA_TILE_W);
-        return cudaErrorInvalidValue;
-    }
 
     const MapKey key = make_key(s, x, w, out, 1, 16, 6);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        if (!encode_x_pairs(&maps[0], s, x, prm.group, prm.boxg)) {
+        if (!encode_x_pairs(&maps[0], s, x, prm.group, prm.boxg, s.kh)) {
             snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
             return cudaErrorInvalidValue;
         }
@@ -809,22 +805,7 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
-    static std::atomic<unsigned long long> done_74{0}, done_any{0}, done_74p{0}, done_anyp{0};
-    if (pool_w > 0) {
-        set_kernel_name("qconv_pairs_kernel<hpool>");
-        if (s.kh == 7 && prm.nsp == 4) {
-            auto kern = qconv_pairs_kernel<7, 4, true>;
-            cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_74p);
-            if (e != cudaSuccess) return e;
-            return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
-                              maps[0], prm);
-        }
-        auto kern = qconv_pairs_kernel<0, 0, true>;
-        cudaError_t e = set_smem_once(kern, GaCfg::SMEM_BYTES, done_anyp);
-        if (e != cudaSuccess) return e;
-        return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
-                          maps[0], prm);
-    }
+    static std::atomic<unsigned long long> done_74{0}, done_any{0};
     set_kernel_name("qconv_pairs_kernel");
     if (s.kh == 7 && prm.nsp == 4) {  // the 7x7 stem
         auto kern = qconv_pairs_kernel<7, 4>;
@@ -839,6 +820,76 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
         return launch_pdl(kern, dim3(grid), dim3(WIDE_THREADS), GaCfg::SMEM_BYTES, stream,
                           maps[0], prm);
     }
+}
+
+template <int ROWS, int NSP, int ACT>
+cudaError_t launch_stem_pool_kernel(const CUtensorMap& map, const StemPoolParams& prm, int grid,
+                                    cudaStream_t stream) {
+    auto kern = qconv_stem_pool_kernel<ROWS, NSP, ACT>;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(kern, SpCfg::SMEM_BYTES, attr_done);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(grid), dim3(SP_THREADS), SpCfg::SMEM_BYTES, stream, map, prm);
+}
+
+cudaError_t launch_stem_pool(const ConvShape& s, const void* x, const void* const w[4],
+                             const EpilogueArgs& ep, void* out, const TcOptions& opt,
+                             int num_sms, cudaStream_t stream, char* err, size_t errlen) {
+    StemPoolParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.lead = s.pad & 1;
+    prm.nsp = gather_nsp(s);
+    prm.shift = (s.pad + prm.lead) / 2;
+    const int W2 = s.W / 2;
+    prm.group = W2 % 8 == 0 ? 8 : (W2 % 4 == 0 ? 4 : (W2 % 2 == 0 ? 2 : 1));
+    prm.d0 = ((-prm.shift) % prm.group + prm.group) % prm.group;
+    prm.gx0 = (-prm.shift - prm.d0) / prm.group;  // exact: -shift - d0 is a multiple of G
+    prm.nmma = (s.Wo + 15) / 16 * 16;
+    const int boxw = prm.nmma + prm.nsp - 1;  // pairs the N rows read per input row
+    const int boxg = (prm.d0 + boxw + prm.group - 1) / prm.group;
+    prm.row_bytes = boxg * 16 * prm.group;
+    prm.rows = s.kh + 2;
+    prm.stage_bytes = (prm.rows * prm.row_bytes + 1023) & ~1023;
+    int per = SpCfg::RING_BYTES / prm.stage_bytes / SP_ISSUERS;
+    if (per > SpCfg::MAX_PER) per = SpCfg::MAX_PER;
+    if (!stem_pool_ok(s) || per < 1 || boxg > 256 || prm.rows > 256) {
+        snprintf(err, errlen, "stem pooling kernel: kh=%d kw=%d W=%d does not fit", s.kh, s.kw,
+                 s.W);
+        return cudaErrorInvalidValue;
+    }
+    prm.per = per;
+    prm.Hp = (s.Ho - 1) / 2 + 1;
+    prm.Wp = (s.Wo - 1) / 2 + 1;
+    prm.total_rows = static_cast<long long>(s.N) * prm.Hp;
+    if (prm.total_rows > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many pooled rows");
+        return cudaErrorInvalidValue;
+    }
+    const MapKey key = make_key(s, x, w, out, 1, 16, 7);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_pairs(&maps[0], s, x, prm.group, boxg, prm.rows)) {
+            snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    const int grid = grid_for(opt, num_sms, static_cast<int>(prm.total_rows));
+    set_kernel_name("qconv_stem_pool_kernel");
+    if (prm.rows == 9 && prm.nsp == 4) {  // the 7x7 stem
+        if (s.act == 1) return launch_stem_pool_kernel<9, 4, 1>(maps[0], prm, grid, stream);
+        if (s.act == 2) return launch_stem_pool_kernel<9, 4, 2>(maps[0], prm, grid, stream);
+        return launch_stem_pool_kernel<9, 4, 0>(maps[0], prm, grid, stream);
+    }
+    if (s.act == 1) return launch_stem_pool_kernel<0, 0, 1>(maps[0], prm, grid, stream);
+    if (s.act == 2) return launch_stem_pool_kernel<0, 0, 2>(maps[0], prm, grid, stream);
+    return launch_stem_pool_kernel<0, 0, 0>(maps[0], prm, grid, stream);
 }
 
 // ---------------------------------------------------------------- weight gradient
@@ -1080,20 +1131,19 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     return cudaErrorInvalidValue;
 }
 
-bool tc_hpool_supported(const ConvShape& s, const void* x, const void* const w[4],
-                        const void* hp, const EpilogueArgs& ep) {
-    return !s.sep && gather_ok(s) && s.Wo <= GA_TILE_W && tc_supported(s, x, w, hp, ep);
+bool tc_stem_pool_supported(const ConvShape& s, const void* x, const void* const w[4],
+                            const void* out, const EpilogueArgs& ep) {
+    return stem_pool_ok(s) && tc_supported(s, x, w, out, ep);
 }
 
-cudaError_t launch_qconv_tc_hpool(const ConvShape& s, const void* x, const void* const w[4],
-                                  const EpilogueArgs& ep, void* hp, int pool_w,
-                                  const TcOptions& opt, int num_sms, cudaStream_t stream,
-                                  char* err, size_t errlen) {
+cudaError_t launch_qconv_stem_pool(const ConvShape& s, const void* x, const void* const w[4],
+                                   const EpilogueArgs& ep, void* out, const TcOptions& opt,
+                                   int num_sms, cudaStream_t stream, char* err, size_t errlen) {
     if (!load_encoders()) {
         snprintf(err, errlen, "cuTensorMapEncodeTiled is not available");
         return cudaErrorInvalidValue;
     }
-    return launch_gather(s, x, w, ep, hp, opt, num_sms, stream, err, errlen, pool_w);
+    return launch_stem_pool(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
 }
 
 bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy) {

@@ -565,12 +565,8 @@ quan_status_t quan_iqbn_train_fwd(const void* x, long long npix, int C, const fl
 
 size_t quan_qconv2d_maxpool_workspace_size(int N, int H, int W, int Cout, int kh, int kw,
                                            int stride, int pad) {
-    quan::ConvShape s;
-    if (Cout < 4 || Cout % 4 != 0 ||
-        geometry(&s, N, H, W, 4, Cout, kh, kw, stride, pad) != QUAN_OK)
-        return 0;
-    return static_cast<size_t>(N) * s.Ho * ((s.Wo - 1) / 2 + 1 + quan::HPOOL_SIDE_SLOTS) *
-           Cout * 2;
+    (void)N; (void)H; (void)W; (void)Cout; (void)kh; (void)kw; (void)stride; (void)pad;
+    return 0;  // one kernel writes the pooled tensor directly
 }
 
 quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void* wi,
@@ -580,6 +576,8 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
                                        int stride, int pad, int act, void* workspace,
                                        size_t workspace_bytes, void* out,
                                        quan_stream_t stream) {
+    (void)workspace;
+    (void)workspace_bytes;
     const void* w[4] = {wr, wi, wj, wk};
     if (!x || !wr || !wi || !wj || !wk || !out)
         return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
@@ -592,34 +590,22 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
         return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
     s.act = act;
     const int pw = (s.Wo - 1) / 2 + 1, ph = (s.Ho - 1) / 2 + 1;
-    const size_t need =
-        static_cast<size_t>(N) * s.Ho * (pw + quan::HPOOL_SIDE_SLOTS) * Cout * 2;
     const size_t ob = static_cast<size_t>(N) * ph * pw * Cout * 2;
-    if (!workspace || workspace_bytes < need)
-        return fail(QUAN_ERR_INVALID_ARG, "workspace must hold %zu bytes (got %zu%s)", need,
-                    workspace_bytes, workspace ? "" : ", NULL");
-    // the two tensors written (the workspace and out) against each other and every input
+    // the written tensor against every input
     const size_t xb = x_bytes(s, 2), wb = w_bytes(s, 2), vb = static_cast<size_t>(Cout) * 4;
-    const void* written[2] = {workspace, out};
-    const size_t wsz[2] = {need, ob};
-    if (overlaps(out, ob, workspace, need))
-        return fail(QUAN_ERR_INVALID_ARG, "out overlaps the workspace");
-    for (int k = 0; k < 2; ++k)
-        if (overlaps(written[k], wsz[k], x, xb) || overlaps(written[k], wsz[k], wr, wb) ||
-            overlaps(written[k], wsz[k], wi, wb) || overlaps(written[k], wsz[k], wj, wb) ||
-            overlaps(written[k], wsz[k], wk, wb) || overlaps(written[k], wsz[k], bias, vb) ||
-            overlaps(written[k], wsz[k], iqbn_scale, vb) ||
-            overlaps(written[k], wsz[k], iqbn_shift, vb))
-            return fail(QUAN_ERR_INVALID_ARG, "out or the workspace overlaps an input");
+    if (overlaps(out, ob, x, xb) || overlaps(out, ob, wr, wb) || overlaps(out, ob, wi, wb) ||
+        overlaps(out, ob, wj, wb) || overlaps(out, ob, wk, wb) || overlaps(out, ob, bias, vb) ||
+        overlaps(out, ob, iqbn_scale, vb) || overlaps(out, ob, iqbn_shift, vb))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input");
     int num_sms = 0, cc = 0;
     cudaError_t e;
     if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
     const quan::EpilogueArgs ep{bias, iqbn_scale, iqbn_shift, nullptr};
-    if (cc != 103 || !quan::tc_hpool_supported(s, x, w, workspace, ep) ||
-        reinterpret_cast<uintptr_t>(out) % 16 != 0)
+    if (cc != 103 || !quan::tc_stem_pool_supported(s, x, w, out, ep))
         return fail(QUAN_ERR_UNSUPPORTED,
                     "the fused stem pooling needs sm_103, Cin = 4, Cout = 64, stride 2, an even "
-                    "W, Wo <= 128 and 16-byte aligned tensors");
+                    "W, Wo <= 128, (kh + 2) * ceil-even((kw + pad %% 2) / 2) <= 36 and 16-byte "
+                    "aligned tensors");
     quan::TcOptions opt;
     opt.kappa = 0;
     opt.bnq = 0;
@@ -630,13 +616,10 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
     opt.wait_limit_ns = g_wait_limit.load();
     opt.inject_stall = g_inject.load();
     char err[256] = "";
-    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
-    e = quan::launch_qconv_tc_hpool(s, x, w, ep, workspace, pw, opt, num_sms, cs, err,
-                                    sizeof(err));
+    e = quan::launch_qconv_stem_pool(s, x, w, ep, out, opt, num_sms,
+                                     reinterpret_cast<cudaStream_t>(stream), err, sizeof(err));
     if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
-    if (e != cudaSuccess) return cuda_fail(e, "qconv_pairs launch");
-    e = quan::launch_vpool_bf16(workspace, N, s.Ho, pw, quan::HPOOL_SIDE_SLOTS, Cout, out, cs);
-    if (e != cudaSuccess) return cuda_fail(e, "vpool launch");
+    if (e != cudaSuccess) return cuda_fail(e, "qconv_stem_pool launch");
     t_last_path = QUAN_PATH_TC;
     t_last_kernel = quan::last_tc_kernel();
     return QUAN_OK;

@@ -527,20 +527,11 @@ __device__ __forceinline__ void epilogue_direct_sep(const ConvShape& s, const Ep
 }
 
 // NG epilogue groups, one per MMA issuer (warps 4 + 4 NG .. 15 take no part).
-// HPOOL: instead of the tile, write its horizontal 3-wide, stride-2 max (padding 1): the
-// first half of a 3x3/2 max pooling fused into the producing convolution.  A tile must be
-// one whole output row (geo's m0 = row * Wo, rows = Wo <= 128).  y is then
-// [rows][pool_w + HPOOL_SIDE_SLOTS][64]: pooled column j covers pixels 2j - 1, 2j, 2j + 1, and a
-// lane holds 4 consecutive pixels, so each column needs at most the last pixel of the lane
-// group before it (a shuffle) -- except the first column of TMEM quadrants 1-3, whose
-// left pixel is in another warp: that warp writes it to side slot q + 1 of the row, and
-// the vertical pass takes the max with it.  No barrier and no shared memory.
-template <typename Geo, int NG = EPI_GROUPS, bool HPOOL = false>
+template <typename Geo, int NG = EPI_GROUPS>
 __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const EpilogueArgs& ep,
                                                   void* y, uint32_t tmem_base, uint32_t accf0,
                                                   uint32_t acce0, int num_tiles, uint64_t limit,
-                                                  volatile int* abort_flag, Geo geo,
-                                                  int pool_w = 0) {
+                                                  volatile int* abort_flag, Geo geo) {
     static_assert(NG >= 1 && NG <= EPI_GROUPS, "each epilogue group drains one issuer's buffers");
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int quad = warp & 3;                // TMEM lane quadrant this warp may access
@@ -606,7 +597,6 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
             chunk_transpose_stage<2, 4>(E, ci);
             chunk_transpose_stage<1, 4>(E, ci);
             // now E[k][e] = channel c0 + e of row row0 + k
-            float act_v[HPOOL ? 4 : 1][8];  // activated values of the 4 pixels (pooling)
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 float rz[8];
@@ -628,56 +618,11 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
                     const float z0 = fmaf(sc[h][2 * t], E[k][2 * t], sh[h][2 * t]) + rz[2 * t];
                     const float z1 =
                         fmaf(sc[h][2 * t + 1], E[k][2 * t + 1], sh[h][2 * t + 1]) + rz[2 * t + 1];
-                    if constexpr (HPOOL) {
-                        // pixels past the row's end never win the max
-                        const bool live = row0 + k < g.rows;
-                        act_v[k][2 * t] = live ? activate(z0, s.act) : -INFINITY;
-                        act_v[k][2 * t + 1] = live ? activate(z1, s.act) : -INFINITY;
-                    } else {
-                        w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
-                    }
+                    w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
                 }
-                if constexpr (!HPOOL) {
-                    if (row0 + k < g.rows)
-                        *reinterpret_cast<uint4*>(out + (g.m0 + row0 + k) * 64 + c0) =
-                            make_uint4(w[0], w[1], w[2], w[3]);
-                }
-            }
-            if constexpr (HPOOL) {
-                // this lane (pixels row0 .. row0 + 3, row0 a multiple of 4) writes pooled
-                // columns j = row0 / 2 (pixels row0 - 1 .. row0 + 1) and j + 1 (row0 + 1 ..
-                // row0 + 3); pixel row0 - 1 is the lane group before it, or, for rg == 0,
-                // in the quadrant before (left padding for quadrant 0): that column is
-                // written without it and completed from the side slot
-                float prev[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    prev[e] = __shfl_up_sync(0xffffffffu, act_v[3][e], 4);
-                    if (rg == 0) prev[e] = -INFINITY;
-                }
-                uint32_t wl[4], wr[4], ws[4];
-#pragma unroll
-                for (int t = 0; t < 4; ++t) {
-                    const int e0 = 2 * t, e1 = 2 * t + 1;
-                    wl[t] = pack_bf16x2(fmaxf(prev[e0], fmaxf(act_v[0][e0], act_v[1][e0])),
-                                        fmaxf(prev[e1], fmaxf(act_v[0][e1], act_v[1][e1])));
-                    wr[t] = pack_bf16x2(fmaxf(act_v[1][e0], fmaxf(act_v[2][e0], act_v[3][e0])),
-                                        fmaxf(act_v[1][e1], fmaxf(act_v[2][e1], act_v[3][e1])));
-                    ws[t] = pack_bf16x2(act_v[3][e0], act_v[3][e1]);
-                }
-                const int rowlen = pool_w + HPOOL_SIDE_SLOTS;  // 64-channel pixels per row
-                // one tile per output row: the tile index is the row (n Ho + y)
-                __nv_bfloat16* prow = out + static_cast<long long>(tile) * rowlen * 64 + c0;
-                const int j = row0 / 2;
-                if (j < pool_w)
-                    *reinterpret_cast<uint4*>(prow + j * 64) = make_uint4(wl[0], wl[1], wl[2], wl[3]);
-                if (j + 1 < pool_w)
-                    *reinterpret_cast<uint4*>(prow + (j + 1) * 64) =
-                        make_uint4(wr[0], wr[1], wr[2], wr[3]);
-                // the quadrant's last pixel, for the next quadrant's first column
-                if (rg == 7 && quad < 3 && 16 * (quad + 1) < pool_w)
-                    *reinterpret_cast<uint4*>(prow + (pool_w + quad + 1) * 64) =
-                        make_uint4(ws[0], ws[1], ws[2], ws[3]);
+                if (row0 + k < g.rows)
+                    *reinterpret_cast<uint4*>(out + (g.m0 + row0 + k) * 64 + c0) =
+                        make_uint4(w[0], w[1], w[2], w[3]);
             }
         }
     }

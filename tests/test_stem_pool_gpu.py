@@ -1,7 +1,7 @@
-"""The stem convolution with its 3x3/2 max pooling fused (quan_qconv2d_maxpool_fwd): bit
-for bit the two separate calls (max commutes with the monotone bf16 rounding), within the
-bf16 tolerance of the oracle's convolution followed by the oracle's pooling, and through
-the backbone."""
+"""The stem convolution with its 3x3/2 max pooling in one kernel (quan_qconv2d_maxpool_fwd):
+bit for bit the two separate calls (max commutes with the monotone bf16 rounding), within
+the bf16 tolerance of the oracle's convolution followed by the oracle's pooling, and
+through the backbone."""
 import numpy as np
 import pytest
 
@@ -23,22 +23,29 @@ def lib():
     yield quan.load()
 
 
-def run_both(spec, act):
+def run_both(spec, act, negate_scale=None, max_ctas=0):
     d = inputs.layer_inputs(spec)
+    if negate_scale is not None:
+        d["scale"] = np.where(negate_scale, -d["scale"], d["scale"]).astype(np.float32)
     x = to_dev(d["x"], "bf16")
     w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
     sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
     N, H, W = spec.N, spec.H, spec.W
     conv = quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, scale=sc, shift=sh, act=act)
     ref_gpu = quan.maxpool2d(conv, k=3, stride=2, pad=1)
-    nbytes = quan.quan_qconv2d_maxpool_workspace_size(N, H, W, spec.Cout, spec.kh, spec.kw,
-                                                      spec.stride, spec.pad)
-    ws = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    # one kernel writes the pooled tensor: no workspace
+    assert quan.quan_qconv2d_maxpool_workspace_size(N, H, W, spec.Cout, spec.kh, spec.kw,
+                                                    spec.stride, spec.pad) == 0
     out = torch.full_like(ref_gpu, float("nan"))
-    quan.quan_qconv2d_maxpool_fwd(x, *w, None, sc, sh, N, H, W, spec.Cin, spec.Cout, spec.kh,
-                                  spec.kw, spec.stride, spec.pad, act, ws, nbytes, out)
-    torch.cuda.synchronize()
-    assert quan.quan_last_kernel() == "qconv_pairs_kernel<hpool>"
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 0)
+    try:
+        quan.quan_qconv2d_maxpool_fwd(x, *w, None, sc, sh, N, H, W, spec.Cin, spec.Cout,
+                                      spec.kh, spec.kw, spec.stride, spec.pad, act, None, 0,
+                                      out)
+        torch.cuda.synchronize()
+    finally:
+        quan.quan_set_tc_tiles(0, 0, 0, 0)
+    assert quan.quan_last_kernel() == "qconv_stem_pool_kernel"
     assert quan.quan_device_status()[0] == quan.QUAN_OK
     return d, out, ref_gpu
 
@@ -66,16 +73,30 @@ def test_fused_equals_separate_calls_and_oracle(case, act):
     assert_bf16_close(out_f64(out), oracle.maxpool2d(y, k=3, stride=2, pad=1), name)
 
 
+@pytest.mark.parametrize("act", [quan.QUAN_ACT_RELU, quan.QUAN_ACT_NONE, quan.QUAN_ACT_SILU])
+def test_fused_negative_scales_and_bands_across_images(act):
+    # channels with a negative IQBN scale (the pooling is then a min of the accumulators,
+    # taken on negated weights); a 3-CTA grid, so that each CTA's band of pooled rows
+    # crosses image boundaries and starts inside an image (its priming tile)
+    spec = inputs.small_layer("stem_neg", 3, 38, 36, 4, 64, 7, 2, 3, seed=(902, act), act=act)
+    neg = (np.arange(64) % 3) == 1
+    d, out, ref_gpu = run_both(spec, act, negate_scale=neg, max_ctas=3)
+    assert torch.equal(out, ref_gpu)
+    f = lambda k: host_f64(d[k], "bf16")
+    y = oracle.qconv2d(f("x"), f("wr"), f("wi"), f("wj"), f("wk"), stride=2, pad=3,
+                       scale=d["scale"], shift=d["shift"], act=act)
+    assert_bf16_close(out_f64(out), oracle.maxpool2d(y, k=3, stride=2, pad=1), "stem_neg")
+
+
 def test_fused_rejects_other_shapes():
     spec = inputs.small_layer("not_stem", 1, 16, 16, 64, 64, 3, 1, 1, seed=(901, 0))
     d = inputs.layer_inputs(spec)
     x = to_dev(d["x"], "bf16")
     w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
-    ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
     out = torch.empty((1, 8, 8, 64), dtype=torch.bfloat16, device="cuda")
     with pytest.raises(quan.QuanError) as ei:
         quan.quan_qconv2d_maxpool_fwd(x, *w, None, None, None, 1, 16, 16, 64, 64, 3, 3, 1, 1,
-                                      quan.QUAN_ACT_RELU, ws, ws.numel(), out)
+                                      quan.QUAN_ACT_RELU, None, 0, out)
     assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
 
 
@@ -107,7 +128,7 @@ def test_fused_call_first_in_a_fresh_process():
         "r = BackboneRunner(torch, quan, inputs, N=2, fuse_stem_pool=True)\n"
         "r.run_layer(0, torch.cuda.current_stream().cuda_stream)\n"
         "torch.cuda.synchronize()\n"
-        "assert quan.quan_last_kernel() == 'qconv_pairs_kernel<hpool>'\n"
+        "assert quan.quan_last_kernel() == 'qconv_stem_pool_kernel'\n"
         "assert quan.quan_device_status()[0] == quan.QUAN_OK\n")
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     res = subprocess.run([sys.executable, "-c", code], cwd=root, capture_output=True, text=True,
