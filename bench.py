@@ -104,11 +104,12 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(workload: str, kernel: str | None = None):
+def recorded_traffic(workload: str, kernel: str | None = None, path: str | None = None):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or
-    None when no capture exists, it is of another kernel, or the kernel sources changed
-    since it was taken."""
-    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    None when no capture exists, it is of another kernel or template instance (the full
+    name, template arguments included, must match), or the kernel sources changed since it
+    was taken."""
+    path = path or os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f).get(workload)
@@ -116,8 +117,8 @@ def recorded_traffic(workload: str, kernel: str | None = None):
         return None
     if not rec or rec.get("kernel_sha") != kernel_source_hash():
         return None
-    if kernel is not None and not kernel.startswith(rec.get("kernel", "").split("<")[0]):
-        return None
+    if kernel is not None and kernel != rec.get("kernel"):
+        return None  # another kernel, or another template instance of it
     return rec.get("dram_bytes_per_launch")
 
 

@@ -217,7 +217,10 @@ quan_status_t quan_qconv2d_bwd_data(const void* dy, const void* wr, const void* 
  *            at zero).  Calls whose kernels overlap on the GPU (other streams, other host
  *            threads) race on it: order them (one stream, or events).
  *   Set-up   the first call on each device looks up the buffer's device address, with
- *            that device current; make that first call before any stream capture.
+ *            that device current; make that first call before any stream capture.  The
+ *            address is kept for the life of the process: do not call cudaDeviceReset on a
+ *            device between calls of this entry point (the library's module is then loaded
+ *            again and the buffer may move).
  */
 quan_status_t quan_qconv2d_bwd_data_static(const void* dy, const void* wr, const void* wi,
                                            const void* wj, const void* wk, int N, int H, int W,

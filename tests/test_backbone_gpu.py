@@ -4,10 +4,11 @@ libquan against the fp64 oracle.
 Per layer, the oracle is fed the GPU's own input (and residual) of that layer, so every
 convolution is held to the bf16 tolerance on exact inputs; max pooling is bit-exact.
 End to end, the bf16 rounding of the 20 intermediate activations accumulates, so the
-whole-network comparison uses a looser bound, relative L2 <= 2e-2: 21 layers each add
-up to half a bf16 ulp (2^-9 relative) of fresh rounding, and the residual blocks carry it
-forward, which puts the expected relative L2 near sqrt(21) * 2^-9 / sqrt(3) ~ 5e-3; the
-bound leaves a factor of four for amplification through the network."""
+whole-network comparison uses looser bounds, relative L2 <= 2e-2 and max-abs <= 0.12 RMS:
+21 layers each add up to half a bf16 ulp (2^-9 relative) of fresh rounding, and the
+residual blocks carry it forward, which puts the expected relative L2 near
+sqrt(21) * 2^-9 / sqrt(3) ~ 5e-3; both bounds leave a factor of four over the per-layer
+ones for amplification through the network."""
 import numpy as np
 import pytest
 
@@ -22,6 +23,7 @@ from tests._util import assert_bf16_close, errors
 pytestmark = pytest.mark.gpu
 
 E2E_REL_L2 = 2e-2
+E2E_MAX_ABS_RMS = 0.12  # the per-layer 3e-2 * RMS with the same factor of four
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -65,7 +67,10 @@ def test_backbone_two_images_per_layer_and_end_to_end():
     y_ref = ob.forward(inputs.backbone_layers(N=2), params, x_bits)
     got = bf16_bits_to_f64(bits_of(runner.output))
     rel_l2, max_abs, rms = errors(got, y_ref)
+    print("backbone end to end (2 images): rel-L2 %.3e, max-abs %.3e = %.3e RMS" % (
+        rel_l2, max_abs, max_abs / rms))
     assert rel_l2 <= E2E_REL_L2, rel_l2
+    assert max_abs <= E2E_MAX_ABS_RMS * rms, (max_abs, rms)
     assert (got >= 0).all() and got.std() > 0.1
 
 
@@ -83,8 +88,11 @@ def test_backbone_silu_two_images():
     params = check_layers(runner, slice(0, 2))
     y_ref = ob.forward(inputs.backbone_layers(N=2, act=inputs.ACT_SILU), params, x_bits)
     got = bf16_bits_to_f64(bits_of(runner.output))
-    rel_l2, _, _ = errors(got, y_ref)
+    rel_l2, max_abs, rms = errors(got, y_ref)
+    print("SiLU backbone end to end (2 images): rel-L2 %.3e, max-abs %.3e = %.3e RMS" % (
+        rel_l2, max_abs, max_abs / rms))
     assert rel_l2 <= E2E_REL_L2, rel_l2
+    assert max_abs <= E2E_MAX_ABS_RMS * rms, (max_abs, rms)
     assert (got < 0).any()  # SiLU's negative lobe survives to the output
 
 
@@ -94,6 +102,6 @@ def test_backbone_full_batch_sampled_images():
     runner.step(stream)
     torch.cuda.synchronize()
     assert quan.quan_device_status()[0] == quan.QUAN_OK
-    check_layers(runner, [0, 255])
+    check_layers(runner, [0, 128, 255])
     out = runner.output.float()
     assert torch.isfinite(out).all() and (out >= 0).all()

@@ -56,18 +56,22 @@ def test_workload_config_flops():
     assert "SiLU" in bb["epilogue"] and bb["convs"] == 20
 
 
-def test_recorded_traffic_lookup():
-    # a record is used only for its own workload key, its own kernel and the current
-    # device-code sources
+def test_recorded_traffic_lookup(tmp_path):
+    # a record is used only for its own workload key, its own kernel (the library's full
+    # name, template instance included) and the current device-code sources
     import json
-    with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
-        rec = json.load(f)
-    current = rec["c1"]["kernel_sha"] == bench.kernel_source_hash()
-    got = bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=2>")
-    # valid only while the device code is the one the counters were taken on
-    assert got == (rec["c1"]["dram_bytes_per_launch"] if current else None)
-    assert bench.recorded_traffic("c1", "qconv_tc_kernel<pair,kappa=32,bnq=64>") is None
-    assert bench.recorded_traffic("no_such_workload", None) is None
+    rec = {"c1": {"kernel": "qconv_ws_kernel<halo,issuers=2>", "dram_bytes_per_launch": 123,
+                  "kernel_sha": bench.kernel_source_hash()},
+           "old": {"kernel": "qconv_ws_kernel<halo,issuers=2>", "dram_bytes_per_launch": 7,
+                   "kernel_sha": "0000000000000000"}}
+    path = str(tmp_path / "traffic.json")
+    with open(path, "w") as f:
+        json.dump(rec, f)
+    assert bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=2>", path) == 123
+    assert bench.recorded_traffic("c1", "qconv_ws_kernel<halo,issuers=3>", path) is None
+    assert bench.recorded_traffic("c1", "qconv_tc_kernel<pair,kappa=32,bnq=64>", path) is None
+    assert bench.recorded_traffic("old", "qconv_ws_kernel<halo,issuers=2>", path) is None
+    assert bench.recorded_traffic("no_such_workload", None, path) is None
 
     class A:
         workload, direction, variant = "c2a", "bwd", "separable"

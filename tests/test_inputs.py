@@ -63,3 +63,20 @@ def test_grad_output_seeded_and_prefix():
     np.testing.assert_array_equal(a[:2], inputs.grad_output(spec, n_images=2))
     other = inputs.grad_output(inputs.small_layer("g", 4, 6, 5, 16, 32, 3, 2, 1, seed=(7, 4)))
     assert (a != other).any()
+
+
+def test_round_bf16_of_the_checks():
+    # the tests' fp64 -> bf16 rounding (nearest, ties to even) agrees with the input
+    # quantiser on float32 values and rounds float64 values once, directly
+    from tests._util import round_bf16
+    rng = np.random.default_rng(1)
+    a = np.concatenate([rng.standard_normal(100000).astype(np.float32) * 3,
+                        np.array([0.0, 1.0, 1e-30, -7.5], dtype=np.float32)])
+    want = (inputs.to_bf16_bits(a).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    np.testing.assert_array_equal(round_bf16(a.astype(np.float64)), want)
+    ulp = 2.0 ** -7
+    assert round_bf16(1 + ulp / 2) == 1.0                        # tie -> even (down)
+    assert round_bf16(1 + 3 * ulp / 2) == 1 + 2 * ulp            # tie -> even (up)
+    assert round_bf16(1 + ulp / 2 + 2.0 ** -40) == 1 + ulp       # just above the tie
+    assert round_bf16(-(1 + ulp / 2 + 2.0 ** -40)) == -(1 + ulp)
+    assert round_bf16(255.9) == 256.0 and round_bf16(2.0 ** -130) == 2.0 ** -130

@@ -333,6 +333,22 @@ def sample_points(spec, n_random, seed):
     return [(i // hw, (i % hw) // spec.Wo, i % spec.Wo) for i in idx]
 
 
+@pytest.mark.parametrize("name", ["c2a", "c2b", "c3a", "c3b"])
+def test_full_size_layer_whole_images(name):
+    # the full launch, compared with the oracle element by element on images 0, N/2, N - 1
+    spec = inputs.LAYERS[name]
+    d = inputs.layer_inputs(spec)
+    got, used = run_gpu(d, guard=True)
+    assert used == quan.QUAN_PATH_TC
+    images = [0, spec.N // 2, spec.N - 1]
+    w = [host_f64(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    ref = oracle.qconv2d(host_f64(d["x"][images], "bf16"), *w, stride=spec.stride,
+                         pad=spec.pad, bias=d["bias"], scale=d["scale"], shift=d["shift"],
+                         act=spec.act)
+    for k, n in enumerate(images):
+        assert_bf16_close(got[n], ref[k], "%s image %d" % (name, n))
+
+
 @pytest.mark.parametrize("name", ["c1", "c2a", "c2b", "c3a", "c3b"])
 def test_full_size_layer_sampled(name):
     spec = inputs.LAYERS[name]
