@@ -4,11 +4,12 @@ libquan against the fp64 oracle.
 Per layer, the oracle is fed the GPU's own input (and residual) of that layer, so every
 convolution is held to the bf16 tolerance on exact inputs; max pooling is bit-exact.
 End to end, the bf16 rounding of the 20 intermediate activations accumulates, so the
-whole-network comparison uses looser bounds, relative L2 <= 2e-2 and max-abs <= 0.12 RMS:
+whole-network comparison uses looser bounds, relative L2 <= 1e-2 and max-abs <= 0.12 RMS:
 21 layers each add up to half a bf16 ulp (2^-9 relative) of fresh rounding, and the
 residual blocks carry it forward, which puts the expected relative L2 near
-sqrt(21) * 2^-9 / sqrt(3) ~ 5e-3; both bounds leave a factor of four over the per-layer
-ones for amplification through the network."""
+sqrt(21) * 2^-9 / sqrt(3) ~ 5e-3 (4.7e-3 with ReLU and 5.2e-3 with SiLU measured); the
+bounds leave a factor of two over that and of four over the per-layer max-abs bound for
+amplification through the network."""
 import numpy as np
 import pytest
 
@@ -22,7 +23,7 @@ from tests._util import assert_bf16_close, errors
 
 pytestmark = pytest.mark.gpu
 
-E2E_REL_L2 = 2e-2
+E2E_REL_L2 = 1e-2
 E2E_MAX_ABS_RMS = 0.12  # the per-layer 3e-2 * RMS with the same factor of four
 
 

@@ -80,3 +80,14 @@ def test_round_bf16_of_the_checks():
     assert round_bf16(1 + ulp / 2 + 2.0 ** -40) == 1 + ulp       # just above the tie
     assert round_bf16(-(1 + ulp / 2 + 2.0 ** -40)) == -(1 + ulp)
     assert round_bf16(255.9) == 256.0 and round_bf16(2.0 ** -130) == 2.0 ** -130
+
+
+def test_bf16_reference_straddled_midpoint():
+    # the other neighbour is accepted only for an exact value within 2^-16 of a midpoint
+    from tests._util import bf16_reference
+    ulp = 2.0 ** -5                      # bf16 spacing in [4, 8)
+    mid = 4.0 + ulp / 2                  # between 4 and 4 + ulp
+    ref = np.array([mid * (1 + 2.0 ** -30), mid * (1 + 2.0 ** -10), 5.0])
+    got = np.array([4.0, 4.0, 5.0 + ulp])
+    want = np.array([4.0, 4.0 + ulp, 5.0])
+    np.testing.assert_array_equal(bf16_reference(got, ref), want)
