@@ -346,7 +346,10 @@ const char* quan_last_kernel(void);
  * in shared memory, only for Cin = Cout = 64 and at most 9 taps; 4: pixel pairs,
  * weight-stationary with the input loaded as 16-byte pairs of adjacent pixels, one TMA
  * box per filter row, only for the Cin = 4 stem shapes above; mode 0 picks it for
- * those).  Values that do not
+ * those; 5: pointwise, the MMA's rows the expanded block weight of 32 quaternion output
+ * channels and its columns 256 streamed pixels, only for 1x1 filters with pad 0, stride 1
+ * or 2 (even H and W), Cin a multiple of 64 up to 512, Cout a multiple of 128 and no
+ * residual; mode 0 picks it for those).  Values that do not
  * divide the layer, or a tile that does not fit in shared memory, make the call fail
  * with QUAN_ERR_UNSUPPORTED.
  */

@@ -449,6 +449,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #include "qconv_ws.cuh"
 #include "qconv_gather.cuh"
 #include "qconv_stempool.cuh"
+#include "qconv_pw.cuh"
 #include "qconv_dw.cuh"
 
 // ---------------------------------------------------------------- host side
@@ -822,6 +823,106 @@ cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w
     }
 }
 
+// Pointwise layer input: stride 1, [N H W][Cin] in boxes of 64 channels x `rows` pixels;
+// stride 2, [N H / 2][2][W / 2][2][Cin] in boxes of 64 channels x 1 x Wo x 1 x `rows` (the
+// sampled pixels of that many output rows).  128-byte swizzle.
+bool encode_x_pw(CUtensorMap* map, const ConvShape& s, const void* x, int rows) {
+    const cuuint64_t e = static_cast<cuuint64_t>(s.Cin) * 2;  // bytes per pixel
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    CUresult r;
+    if (s.stride == 1) {
+        const cuuint64_t dims[2] = {static_cast<cuuint64_t>(s.Cin),
+                                    static_cast<cuuint64_t>(s.N) * s.H * s.W};
+        const cuuint64_t strides[1] = {e};
+        const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(rows)};
+        r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims,
+                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    } else {
+        const cuuint64_t dims[5] = {static_cast<cuuint64_t>(s.Cin), 2,
+                                    static_cast<cuuint64_t>(s.W / 2), 2,
+                                    static_cast<cuuint64_t>(s.N) * (s.H / 2)};
+        const cuuint64_t strides[4] = {e, 2 * e, e * s.W, 2 * e * s.W};
+        const cuuint32_t box[5] = {64, 1, static_cast<cuuint32_t>(s.Wo), 1,
+                                   static_cast<cuuint32_t>(rows)};
+        r = g_encode_tiled(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(x), dims,
+                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    }
+    return r == CUDA_SUCCESS;
+}
+
+template <int STRIDE, int ACT>
+cudaError_t launch_pw_kernel(const CUtensorMap& map, const PwParams& prm, int grid,
+                             cudaStream_t stream) {
+    auto kern = qconv_pw_kernel<STRIDE, ACT>;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(kern, PwCfg::SMEM_BYTES, attr_done);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(grid), dim3(PW_THREADS), PwCfg::SMEM_BYTES, stream, map, prm);
+}
+
+cudaError_t launch_pw(const ConvShape& s, const void* x, const void* const w[4],
+                      const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
+                      cudaStream_t stream, char* err, size_t errlen) {
+    PwParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.kchunks = s.Cin / 64;
+    prm.stages = PwCfg::max_stages(prm.kchunks);
+    prm.mblocks = s.Cout / 128;
+    prm.npix = s.M;
+    // (no box extends past the tensor: tiles shrink for inputs smaller than one tile)
+    if (s.stride == 1) {
+        prm.rows_per_tile = 0;
+        prm.tile_pix = s.M < PW_NPIX ? static_cast<int>(s.M) : PW_NPIX;
+        prm.num_tiles = static_cast<int>((s.M + prm.tile_pix - 1) / prm.tile_pix);
+    } else {
+        const long long rows = static_cast<long long>(s.N) * s.Ho;
+        prm.rows_per_tile = PW_NPIX / s.Wo;
+        if (prm.rows_per_tile > rows) prm.rows_per_tile = static_cast<int>(rows);
+        prm.tile_pix = prm.rows_per_tile * s.Wo;
+        prm.num_tiles = static_cast<int>((rows + prm.rows_per_tile - 1) / prm.rows_per_tile);
+    }
+    if (prm.stages < 2 || s.M > 0x7fffffffLL) {
+        snprintf(err, errlen, "pointwise kernel: Cin=%d does not fit", s.Cin);
+        return cudaErrorInvalidValue;
+    }
+    const MapKey key = make_key(s, x, w, out, 64, 32, 8);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_pw(&maps[0], s, x,
+                         s.stride == 1 ? prm.tile_pix : prm.rows_per_tile)) {
+            snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    // every CTA keeps one channel block: the grid is a multiple of the block count
+    const long long work = static_cast<long long>(prm.mblocks) * prm.num_tiles;
+    int grid = opt.max_ctas > 0 ? opt.max_ctas : num_sms;
+    if (grid > work) grid = static_cast<int>(work);
+    grid = grid / prm.mblocks * prm.mblocks;
+    if (grid < prm.mblocks) grid = prm.mblocks;
+    set_kernel_name(s.stride == 1 ? "qconv_pw_kernel<s1>" : "qconv_pw_kernel<s2>");
+    const int act = s.act;
+    if (s.stride == 1) {
+        if (act == 1) return launch_pw_kernel<1, 1>(maps[0], prm, grid, stream);
+        if (act == 2) return launch_pw_kernel<1, 2>(maps[0], prm, grid, stream);
+        return launch_pw_kernel<1, 0>(maps[0], prm, grid, stream);
+    }
+    if (act == 1) return launch_pw_kernel<2, 1>(maps[0], prm, grid, stream);
+    if (act == 2) return launch_pw_kernel<2, 2>(maps[0], prm, grid, stream);
+    return launch_pw_kernel<2, 0>(maps[0], prm, grid, stream);
+}
+
 template <int ROWS, int NSP, int ACT>
 cudaError_t launch_stem_pool_kernel(const CUtensorMap& map, const StemPoolParams& prm, int grid,
                                     cudaStream_t stream) {
@@ -1024,6 +1125,15 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
         snprintf(err, errlen,
                  "pixel-pair gather mode needs Cin = 4, Cout = 64, stride 2, even W and at "
                  "most %d K units", GA_MAX_UNITS);
+        return cudaErrorInvalidValue;
+    }
+    if (pw_ok(s, ep) && (opt.mode == 0 || opt.mode == 5))
+        return launch_pw(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+    if (opt.mode == 5) {
+        snprintf(err, errlen,
+                 "pointwise mode needs a 1x1 filter, pad 0, stride 1 or 2 (even H and W, "
+                 "Wo <= %d), Cin a multiple of 64 up to %d, Cout a multiple of 128 and no "
+                 "residual", PW_NPIX, PW_MAX_CIN);
         return cudaErrorInvalidValue;
     }
     // Weight-stationary for 16 -> 16 quaternion channels (the whole expanded weight fits);

@@ -251,6 +251,71 @@ def test_tc_pixel_pair_gather_mode_rejects_other_shapes():
     assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
 
 
+# ------------------------------------------------------------------ pointwise (1x1) kernel
+
+PW_CASES = [
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra
+    ("pw_s1_ragged", 3, 9, 13, 64, 128, 1, 1, 0, {}),        # 351 pixels: a ragged tile
+    ("pw_s1_tiny", 1, 3, 5, 128, 256, 1, 1, 0, {}),          # 15 pixels, less than a tile
+    ("pw_s1_cin512", 2, 16, 17, 512, 256, 1, 1, 0,           # 8 K chunks through 3 stages
+     {"bias": True, "act": quan.QUAN_ACT_SILU}),
+    ("pw_s1_cout512", 1, 20, 20, 256, 512, 1, 1, 0,          # 4 channel blocks
+     {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
+    ("pw_s2_shortcut", 3, 28, 28, 64, 128, 1, 2, 0,          # 18 output rows per tile
+     {"act": quan.QUAN_ACT_NONE}),
+    ("pw_s2_wide", 2, 14, 14, 256, 512, 1, 2, 0, {"act": quan.QUAN_ACT_NONE}),  # Wo = 7
+    ("pw_s2_odd_out", 1, 30, 22, 128, 256, 1, 2, 0, {}),     # Ho = 15, Wo = 11: one short tile
+]
+
+
+@pytest.mark.parametrize("case", PW_CASES, ids=[c[0] for c in PW_CASES])
+def test_tc_pointwise_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(209, len(name)), **extra)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_pw_kernel<s%d>" % s
+
+
+@pytest.mark.parametrize("max_ctas", [2, 5])
+def test_tc_pointwise_few_ctas(max_ctas):
+    # 2 channel blocks on a grid of 2 (5 rounds down to 4): every CTA walks many pixel
+    # tiles, wrapping the stage ring and both accumulators many times
+    spec = inputs.small_layer("pw_few", 4, 32, 32, 128, 256, 1, 1, 0, seed=(210, max_ctas))
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 5)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_pw_kernel<s1>"
+
+
+def test_tc_pointwise_matches_pair_kernel():
+    # the same stride-2 shortcut on the pointwise and the pair kernel: both within the
+    # oracle's tolerance, and close to each other
+    spec = inputs.small_layer("pw_vs_pair", 2, 28, 28, 128, 256, 1, 2, 0, seed=(211, 0),
+                              act=quan.QUAN_ACT_NONE)
+    d = inputs.layer_inputs(spec)
+    ref = oracle_full(d)
+    outs = []
+    for mode, kern in ((5, "qconv_pw_kernel<s2>"), (2, None)):
+        quan.quan_set_tc_tiles(0, 0, 0, mode)
+        got, used = run_gpu(d, path=quan.QUAN_PATH_TC)
+        assert used == quan.QUAN_PATH_TC
+        if kern:
+            assert quan.quan_last_kernel() == kern
+        assert_bf16_close(got, ref, "mode %d" % mode)
+        outs.append(got)
+    assert_bf16_close(outs[0], outs[1], "pointwise vs pair")
+
+
+def test_tc_pointwise_mode_rejects_other_shapes():
+    for args in ((1, 8, 8, 64, 128, 3, 1, 1), (1, 8, 8, 64, 64, 1, 1, 0),
+                 (1, 9, 8, 64, 128, 1, 2, 0)):   # 3x3; Cout 64; odd H at stride 2
+        spec = inputs.small_layer("not_pw", *args, seed=(212, 0))
+        d = inputs.layer_inputs(spec)
+        quan.quan_set_tc_tiles(0, 0, 0, 5)
+        with pytest.raises(quan.QuanError) as ei:
+            run_gpu(d, path=quan.QUAN_PATH_TC)
+        assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+
+
 def test_tc_nonsquare_kernel():
     spec = inputs.small_layer("k3x1", 2, 9, 10, 64, 64, 3, 1, 1, kw=1, seed=(203, 0))
     # pad 1 on both sides with kw = 1 widens the output; valid for the oracle too
@@ -435,12 +500,14 @@ def test_maxpool(shape):
 
 # ------------------------------------------------------------------ failure detection
 
-@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0)])
+@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0)])
 def test_bounded_wait_timeout_every_kernel(mode, issuers):
     # the failure-injection path of the pair-mode, weight-stationary (two and three
-    # issuers) and gather kernels
+    # issuers), gather and pointwise kernels
     if mode == 4:
         spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
+    elif mode == 5:
+        spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 1, 1, 0, seed=(401, mode))
     else:
         spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
     d = inputs.layer_inputs(spec)

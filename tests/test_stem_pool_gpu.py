@@ -134,3 +134,25 @@ def test_fused_call_first_in_a_fresh_process():
     res = subprocess.run([sys.executable, "-c", code], cwd=root, capture_output=True, text=True,
                          timeout=300)
     assert res.returncode == 0, res.stderr[-2000:]
+
+
+def test_fused_bounded_wait_timeout_and_recovery():
+    # the failure-injection path: the first issuer waits on a barrier nothing arrives on;
+    # the timeout is reported and the next call on the same context is correct
+    spec = inputs.small_layer("stem_inject", 2, 32, 32, 4, 64, 7, 2, 3, seed=(903, 0))
+    quan.quan_set_wait_limit_ns(5_000_000)
+    quan.quan_set_fault_injection(True)
+    try:
+        d = inputs.layer_inputs(spec)
+        x = to_dev(d["x"], "bf16")
+        w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+        out = torch.empty((2, 8, 8, 64), dtype=torch.bfloat16, device="cuda")
+        quan.quan_qconv2d_maxpool_fwd(x, *w, None, None, None, 2, 32, 32, 4, 64, 7, 7, 2, 3,
+                                      quan.QUAN_ACT_RELU, None, 0, out)
+        st, bits = quan.quan_device_status()
+        assert st == quan.QUAN_ERR_DEVICE_TIMEOUT and bits != 0
+    finally:
+        quan.quan_set_fault_injection(False)
+        quan.quan_set_wait_limit_ns(0)
+    d, out, ref_gpu = run_both(spec, quan.QUAN_ACT_RELU)
+    assert torch.equal(out, ref_gpu)
