@@ -58,6 +58,9 @@ def parse_args():
                          "or SiLU as in YOLO-style detectors)")
     ap.add_argument("--no-fuse", action="store_true",
                     help="backbone: run the stem and its max pool as two calls")
+    ap.add_argument("--rgb", action="store_true",
+                    help="backbone: start from fp32 RGB pixels, mapped to quaternions by Eq. 4 "
+                         "inside the fused stem kernel's loader")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -737,7 +740,7 @@ def act_code(name: str) -> int:
 
 
 def workload_config(workload: str, inputs, variant: str = "full", direction: str = "fwd",
-                    act: str = "relu") -> dict:
+                    act: str = "relu", rgb: bool = False) -> dict:
     """The workload part of the JSON line's config, shared by both arms."""
     if workload == "poincare":
         N, H, W = POINCARE_SHAPE
@@ -752,8 +755,10 @@ def workload_config(workload: str, inputs, variant: str = "full", direction: str
         layers = inputs.backbone_layers(act=act_code(act))
         convs = [L.spec for L in layers if L.kind == "conv"]
         c0 = convs[0]
-        return {"workload": "%s, N=%d, %dx%dx4 quaternion input" % (
-                    WORKLOAD_DESC[workload], c0.N, c0.H, c0.W),
+        return {"workload": "%s, N=%d, %dx%d%s" % (
+                    WORKLOAD_DESC[workload], c0.N, c0.H, c0.W,
+                    " fp32 RGB input (Eq. 4 mapping in the stem kernel's loader)" if rgb
+                    else "x4 quaternion input"),
                 "N": c0.N, "H": c0.H, "W": c0.W, "convs": len(convs), "maxpool": 1,
                 "flops_per_step": sum(c.flops for c in convs),
                 "epilogue": "IQBN+%s (+residual)" % ("SiLU" if act == "silu" else "ReLU"),
@@ -818,8 +823,10 @@ def main():
     if args.workload in ("backbone", "poincare", "iqbn") and (args.variant != "full" or
                                                        args.direction != "fwd"):
         raise SystemExit("--variant and --pass apply to the convolution layer workloads")
-    if args.workload != "backbone" and args.act != "relu":
-        raise SystemExit("--act applies to the backbone workload")
+    if args.workload != "backbone" and (args.act != "relu" or args.rgb):
+        raise SystemExit("--act and --rgb apply to the backbone workload")
+    if args.rgb and args.no_fuse:
+        raise SystemExit("--rgb needs the fused stem")
     if args.workload == "poincare":
         runner = PoincareRunner(torch, quan, *POINCARE_SHAPE)
         unit, per_step_units, dtype = "images/s", runner.N, "f32->bf16"
@@ -830,7 +837,7 @@ def main():
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256,
                                          act=act_code(args.act),
-                                         fuse_stem_pool=not args.no_fuse)
+                                         fuse_stem_pool=not args.no_fuse, rgb=args.rgb)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
     else:
@@ -951,7 +958,8 @@ def main():
         dist.destroy_process_group()
     if rank != 0:
         return 0
-    cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act)
+    cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act,
+                          args.rgb)
     cfg.update({"l2": "inputs larger than L2: %d rotating buffer sets, %.0f MB" % (
                     getattr(runner, "sets", 1), runner.footprint / 1e6),
                 "parallelism": "replicas over the batch (dp%d, no collective)" % world,
@@ -1027,6 +1035,9 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
                 s0 = L.spec
                 nb += (runner.outs[1].numel() - s0.N * s0.Ho * s0.Wo * s0.Cout) * 2
                 name += " + maxpool3/2 (fused)"
+                if getattr(runner, "rgb", False):  # 12 bytes of RGB per pixel, not 8
+                    nb += s0.N * s0.H * s0.W * 4
+                    name = "poincare (Eq. 4) + " + name
         else:
             src = runner.outs[L.src]
             fl, nb = 0.0, src.numel() * 2 + runner.outs[i].numel() * 2
@@ -1050,22 +1061,31 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
 
 
 def backbone_cpu_sample(runner, seconds, inputs):
-    """The fp64 oracle backbone on a bounded number of images."""
+    """The fp64 oracle backbone on a bounded number of images (RGB input: the Eq. 4 mapping
+    first, rounded to bf16 as the stem kernel's loader stores it, inside the timing)."""
+    import numpy as np
     import oracle
     import oracle.backbone as ob
     params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in runner.layers]
-    layers = inputs.backbone_layers(N=1, H=runner.H, act=runner.act)
-    x = runner.x_host
+    rgb = getattr(runner, "rgb", False)
+
+    def run(n):
+        x = runner.x_host[:n]
+        if rgb:
+            x = inputs.to_bf16_bits(oracle.poincare(x.astype(np.float64)).astype(np.float32))
+        ob.forward(inputs.backbone_layers(N=n, H=runner.H, act=runner.act), params, x)
+
     t0 = time.perf_counter()
-    ob.forward(layers, params, x[:1])
+    run(1)
     t1 = time.perf_counter() - t0
     n = max(1, min(runner.N, int(seconds / max(t1, 1e-6))))
     if n > 1:
         t0 = time.perf_counter()
-        ob.forward(inputs.backbone_layers(N=n, H=runner.H, act=runner.act), params, x[:n])
+        run(n)
         t1 = time.perf_counter() - t0
     return {"value": n / t1, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": "%d of %d images of the backbone (fp64, %.2f s)" % (n, runner.N, t1)}
+            "sample": "%d of %d images of the backbone (fp64%s, %.2f s)" % (
+                n, runner.N, ", from RGB" if rgb else "", t1)}
 
 
 def reference_arm(args, rank, world, inputs):
@@ -1074,7 +1094,8 @@ def reference_arm(args, rank, world, inputs):
     if rank != 0:
         return 0
     import oracle
-    ref_cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act)
+    ref_cfg = workload_config(args.workload, inputs, args.variant, args.direction, args.act,
+                              args.rgb)
     ref_cfg["parallelism"] = "fp64 oracle on %d host threads" % oracle.num_threads()
     if args.workload == "poincare":
         import numpy as np
@@ -1126,14 +1147,24 @@ def reference_arm(args, rank, world, inputs):
         return 0
     if args.workload == "backbone":
         import oracle.backbone as ob
+        import numpy as np
         layers = inputs.backbone_layers(N=1, act=act_code(args.act))
         params = [inputs.backbone_params(L) if L.kind == "conv" else None for L in layers]
         x = inputs.backbone_input(n_images=1)
+        rgb = inputs.backbone_rgb(n_images=1) if args.rgb else None
+
+        def step():
+            xs = x
+            if rgb is not None:  # Eq. 4, rounded to bf16 as the stem kernel stores it
+                xs = inputs.to_bf16_bits(
+                    oracle.poincare(rgb.astype(np.float64)).astype(np.float32))
+            ob.forward(layers, params, xs)
+
         for _ in range(args.warmup):
-            ob.forward(layers, params, x)
+            step()
         t0 = time.perf_counter()
         for _ in range(args.steps):
-            ob.forward(layers, params, x)
+            step()
         dt = time.perf_counter() - t0
         value = args.steps / dt
         line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",

@@ -321,6 +321,24 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
                                        quan_stream_t stream);
 
 /*
+ * quan_qconv2d_maxpool_fwd from RGB pixels: the Poincare mapping of Eq. 4 (Sec. III-A),
+ * q = ((1 - n2), 2 r, 2 g, 2 b) / (1 + n2) with n2 = r^2 + g^2 + b^2, fused into the stem
+ * kernel's loader (each tile's input rows are loaded as fp32 RGB and turned into the bf16
+ * quaternion pixels the MMAs read; the padding around the image is zero quaternions).
+ * The result is bit-identical to quan_poincare_fwd followed by quan_qconv2d_maxpool_fwd.
+ *   rgb         fp32 [N][H][W][3], 16-byte aligned, owned by the caller
+ *   the rest    as quan_qconv2d_maxpool_fwd with Cin = 4 (no workspace)
+ * Only W a multiple of 32 (and at most 2730) on top of quan_qconv2d_maxpool_fwd's shape
+ * limits; otherwise QUAN_ERR_UNSUPPORTED.
+ */
+quan_status_t quan_qconv2d_maxpool_rgb_fwd(const float* rgb, const void* wr, const void* wi,
+                                           const void* wj, const void* wk, const float* bias,
+                                           const float* iqbn_scale, const float* iqbn_shift,
+                                           int N, int H, int W, int Cout, int kh, int kw,
+                                           int stride, int pad, int act, void* out,
+                                           quan_stream_t stream);
+
+/*
  * Max pooling of every real channel on its own (component-wise pooling of Sec. III-D,
  * QSPPF), bf16 NHWC [N][H][W][C] -> [N][Ho][Wo][C], window k x k, stride, zero-size
  * padding that never wins.  C is any positive count.

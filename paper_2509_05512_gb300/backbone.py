@@ -18,7 +18,8 @@ class BackboneRunner:
     """Weights, activations and the per-step launch sequence of the backbone."""
 
     def __init__(self, torch, quan, inputs=_inputs, N: int = 256, H: int = 224, seed: int = 4,
-                 x_bits=None, act: int = _inputs.ACT_RELU, fuse_stem_pool: bool = False):
+                 x_bits=None, act: int = _inputs.ACT_RELU, fuse_stem_pool: bool = False,
+                 rgb: bool = False, rgb_host=None):
         self.torch, self.quan, self.N, self.H = torch, quan, N, H
         dev = torch.device("cuda")
         self.act = act
@@ -28,6 +29,10 @@ class BackboneRunner:
         L0, L1 = self.layers[0], self.layers[1]
         self.fused = (fuse_stem_pool and L0.kind == "conv" and L1.kind == "maxpool" and
                       L1.src == 0 and (L1.k, L1.stride, L1.pad) == (3, 2, 1))
+        # rgb: the input is fp32 RGB, mapped by Eq. 4 inside the fused stem's loader
+        self.rgb = rgb
+        if rgb and not self.fused:
+            raise ValueError("RGB input needs the fused stem (fuse_stem_pool=True)")
 
         def up(bits):
             return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(
@@ -62,12 +67,18 @@ class BackboneRunner:
                 Wo = (Ws + 2 * L.pad - L.k) // L.stride + 1
                 self.params.append(None)
                 self.outs.append(torch.empty((N, Ho, Wo, C), dtype=torch.bfloat16, device=dev))
-        if x_bits is None:
-            x_bits = inputs.backbone_input(N=N, H=H, seed=seed)
-        self.x_host = x_bits
-        self.x = up(x_bits)
+        if rgb:
+            self.x_host = inputs.backbone_rgb(N=N, H=H, seed=seed) if rgb_host is None \
+                else rgb_host
+            self.x = torch.from_numpy(np.ascontiguousarray(self.x_host)).to(dev)
+        else:
+            if x_bits is None:
+                x_bits = inputs.backbone_input(N=N, H=H, seed=seed)
+            self.x_host = x_bits
+            self.x = up(x_bits)
         self.launches_per_step = len(self.layers)
-        self.footprint = sum(t.numel() * 2 for t in self.outs) + self.x.numel() * 2
+        self.footprint = (sum(t.numel() * 2 for t in self.outs) +
+                          self.x.numel() * self.x.element_size())
 
     # ---------------------------------------------------------------- execution
     def layer_input(self, idx: int):
@@ -87,6 +98,12 @@ class BackboneRunner:
             return out
         s, prm = L.spec, self.params[idx]
         N, H, W, C = x.shape
+        if self.rgb and idx == 0:
+            pooled = self.outs[1] if out is self.outs[0] else out
+            q.quan_qconv2d_maxpool_rgb_fwd(x, *prm["w"], None, prm["scale"], prm["shift"], N, H,
+                                           W, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                                           pooled, stream)
+            return pooled
         if self.fused and idx == 0:
             pooled = self.outs[1] if out is self.outs[0] else out
             q.quan_qconv2d_maxpool_fwd(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
@@ -133,6 +150,7 @@ class BackboneRunner:
         torch = self.torch
         self.h_x = torch.from_numpy(
             np.ascontiguousarray(self.x_host).reshape(-1).view(np.uint8)).pin_memory()
+        # (the device copy target below has the input's dtype: bf16 pixels or fp32 RGB)
         out = self.outs[-1]
         self.h_out = [torch.empty(out.numel() * 2, dtype=torch.uint8).pin_memory()
                       for _ in range(nbuf)]

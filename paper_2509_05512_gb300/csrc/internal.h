@@ -139,6 +139,15 @@ cudaError_t launch_qconv_stem_pool(const ConvShape& s, const void* x, const void
                                    const EpilogueArgs& ep, void* out, const TcOptions& opt,
                                    int num_sms, cudaStream_t stream, char* err, size_t errlen);
 
+// The same from fp32 RGB pixels [N][H][W][3] (W a multiple of 32), the Poincare mapping of
+// Eq. 4 done in the kernel's loader; s is the convolution's shape (Cin = 4).
+bool tc_stem_pool_rgb_supported(const ConvShape& s, const float* rgb, const void* const w[4],
+                                const void* out, const EpilogueArgs& ep);
+cudaError_t launch_qconv_stem_pool_rgb(const ConvShape& s, const float* rgb,
+                                       const void* const w[4], const EpilogueArgs& ep, void* out,
+                                       const TcOptions& opt, int num_sms, cudaStream_t stream,
+                                       char* err, size_t errlen);
+
 // Per-real-channel max pooling, bf16 NHWC.
 cudaError_t launch_maxpool_bf16(const void* x, int N, int H, int W, int C, int k, int stride,
                                 int pad, void* out, int num_sms, cudaStream_t stream);

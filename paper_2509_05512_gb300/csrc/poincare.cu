@@ -4,7 +4,10 @@
 // fp32 RGB [npix][3] -> bf16 [npix][4] in the component-major channel order [r|i|j|k]
 // the convolutions read (one quaternion channel: the four components of a pixel).
 // Elementwise and HBM-bound (12 bytes read, 8 written per pixel): one pixel per thread,
-// coalesced 4-byte loads, one 8-byte store.
+// coalesced 4-byte loads, one 8-byte store.  The reciprocal is the fast one (__fdividef,
+// within a few fp32 ulps: far below the bf16 result's rounding); the stem kernel's fused
+// mapping uses the same arithmetic, so mapping first and mapping in the stem agree bit for
+// bit.
 #include <cuda_bf16.h>
 
 #include "internal.h"
@@ -22,7 +25,7 @@ __global__ void __launch_bounds__(256) poincare_kernel(const float* __restrict__
          p += static_cast<long long>(gridDim.x) * blockDim.x) {
         const float r = __ldg(rgb + 3 * p), g = __ldg(rgb + 3 * p + 1), b = __ldg(rgb + 3 * p + 2);
         const float n2 = fmaf(r, r, fmaf(g, g, b * b));
-        const float inv = 1.0f / (1.0f + n2);
+        const float inv = __fdividef(1.0f, 1.0f + n2);
         const float two_inv = 2.0f * inv;
         const __nv_bfloat162 ri = __floats2bfloat162_rn((1.0f - n2) * inv, r * two_inv);
         const __nv_bfloat162 jk = __floats2bfloat162_rn(g * two_inv, b * two_inv);

@@ -269,6 +269,31 @@ __device__ __forceinline__ uint4 ld_global_na(const void* p) {
     return v;
 }
 
+// ------------------------------------------------------------------ shared-memory access
+// Explicit shared-state-space accesses by 32-bit shared address (a pointer rebuilt from an
+// integer loses its state space, and generic loads take the slower generic path).
+__device__ __forceinline__ float2 lds_f2(uint32_t addr) {
+    float2 v;
+    asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds_u4(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(addr)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void sts_u4(uint32_t addr, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
 // ------------------------------------------------------------------ shared-memory flags
 // A release store and an acquire load of one shared-memory word: the hand-off between a
 // helper warp and an MMA-issuing thread.  One acquire load costs the issuing thread about

@@ -35,6 +35,15 @@
 // channel's weights (the map is then non-decreasing in the negated accumulator, with |s|).
 // SiLU is not monotone: there every pixel is activated before the max.
 //
+// RGB input (RGB = true): the Poincare mapping of Eq. 4 (Sec. III-A) is fused into the
+// loader.  Warp 0's lane 0 loads the tile's kh + 2 rows of fp32 RGB pixels (one TMA box of
+// whole rows) into a ring of SP_RGB_SLOTS staging slots, SP_RGB_SLOTS - 1 tiles ahead;
+// warps 0 and 3 turn the rows a tile does not share with the previous one into the bf16
+// quaternion pairs of the B stage (the MMAs read the shared rows from the previous stage), q = ((1 - n2), 2 r, 2 g, 2 b) / (1 + n2)
+// with n2 = r^2 + g^2 + b^2 (the arithmetic of the stand-alone mapping kernel, so the
+// result is bit-identical to mapping first), zero pairs outside the image (the
+// convolution's zero padding of the quaternion input), and hand the stage to its issuer.
+//
 // Roles (20 warps, one CTA per SM, persistent over its band):
 //   warp 0       TMA producer: one box of (kh + 2) input rows per tile into a ring of
 //                stages (each of the two issuers owns half of the ring);
@@ -58,6 +67,7 @@ constexpr int SP_EXP_WARP0 = 2;          // warps 2..19 expand the block weight
 constexpr int SP_EXP_WARPS = 18;
 constexpr int SP_EPI_WARP0 = 4;          // warps 4..19: epilogue
 constexpr int SP_EPI_THREADS = 512;
+constexpr int SP_RGB_SLOTS = 3;          // RGB input: staging slots of kh + 2 RGB rows
 
 struct StemPoolParams {
     ConvShape s;
@@ -79,6 +89,11 @@ struct StemPoolParams {
     int nmma;         // N of the MMA: Wo rounded up to 16
     int Hp, Wp;       // pooled output size
     long long total_rows;  // N * Hp pooled rows
+    // RGB input only
+    const float* rgb;     // [N][H][W][3] fp32
+    int rgb_row_bytes;    // 12 W
+    int rgb_stage_bytes;  // rows x 12 W, rounded up to 1 KB
+    int rgb_off;          // offset of the staging slots (after the B ring)
 };
 
 struct SpCfg {
@@ -87,8 +102,9 @@ struct SpCfg {
     static constexpr int SCRATCH_BYTES = 8 * 1024;  // letters: 4 x 16 x taps x 2 bytes
     static constexpr int MAX_PER = 4;
     static constexpr int NSTAGE = SP_ISSUERS * MAX_PER;
-    // full, empty (per stage), accf, acce (per buffer), drain (per issuer), bready
-    static constexpr int NUM_BARS = 2 * NSTAGE + 2 * SP_NACC + SP_ISSUERS + 1;
+    // full, empty (per stage), accf, acce (per buffer), drain (per issuer), bready,
+    // RGB staging full and empty (per slot)
+    static constexpr int NUM_BARS = 2 * NSTAGE + 2 * SP_NACC + SP_ISSUERS + 1 + 2 * SP_RGB_SLOTS;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr int A_OFF = 0;
     static constexpr int SCRATCH_OFF = A_OFF + A_BYTES;
@@ -231,9 +247,73 @@ __device__ __forceinline__ void sp_chunk(const uint32_t (&acc)[32], float carry,
     }
 }
 
+// Eq. 4 for one pixel pair (the arithmetic of poincare.cu): 8 bf16 = [q0: r i j k | q1].
+__device__ __forceinline__ uint4 sp_poincare_pair(float2 a, float2 b, float2 c) {
+    const float px[2][3] = {{a.x, a.y, b.x}, {b.y, c.x, c.y}};  // r0 g0 b0 | r1 g1 b1
+    uint32_t w[4];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+        const float rr = px[e][0], gg = px[e][1], bb = px[e][2];
+        const float n2 = fmaf(rr, rr, fmaf(gg, gg, bb * bb));
+        const float inv = __fdividef(1.0f, 1.0f + n2);
+        const float two_inv = 2.0f * inv;
+        w[2 * e] = pack_bf16x2((1.0f - n2) * inv, rr * two_inv);
+        w[2 * e + 1] = pack_bf16x2(gg * two_inv, bb * two_inv);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Warps 0 and 3 (RGB input): rows r_begin .. rows - 1 of one tile's B stage, mapped from
+// the tile's staging slot of RGB rows (rows 0 .. 3 of a tile that continues an image are
+// rows 4 .. 7 of the previous tile: the MMAs read them from that tile's stage and they are
+// not written again; r_begin is 4 then, else 0).  ct = 0 .. 63 this thread's index among the two warps, which takes the pairs ct
+// and ct + 64 of each row; y0 = the tile's first input row; 32-bit shared addresses.  Under
+// the MMAs' operand reads shared-memory accesses take hundreds of cycles, so all of a
+// thread's loads (at most 2 pairs x MAXR rows) are issued before any pair is mapped.
+template <int MAXR>
+__device__ __forceinline__ void sp_convert_rgb(const StemPoolParams& p, uint32_t stage_sa,
+                                               int r_begin, uint32_t slot_sa, int y0, int ct) {
+    const ConvShape& s = p.s;
+    const int gp = p.row_bytes / 16;  // pairs per box row
+    const int pair0 = p.gx0 * p.group;
+    const int W2 = s.W / 2;
+    const uint32_t rb = static_cast<uint32_t>(p.row_bytes);
+    const uint32_t rgb_rb = static_cast<uint32_t>(p.rgb_row_bytes);
+    for (int r0 = r_begin; r0 < p.rows; r0 += MAXR) {
+        float2 in[MAXR][2][3];
+        bool live[MAXR][2];
+#pragma unroll
+        for (int a = 0; a < MAXR; ++a) {
+            const int r = r0 + a, y = y0 + r;
+            const bool row_in = r < p.rows && y >= 0 && y < s.H;
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const int jb = ct + 64 * c, pi = pair0 + jb;
+                live[a][c] = row_in && jb < gp && pi >= 0 && pi < W2;
+                if (live[a][c]) {
+                    const uint32_t src = slot_sa + r * rgb_rb + 24 * pi;
+                    in[a][c][0] = lds_f2(src);
+                    in[a][c][1] = lds_f2(src + 8);
+                    in[a][c][2] = lds_f2(src + 16);
+                }
+            }
+        }
+#pragma unroll
+        for (int a = 0; a < MAXR; ++a)
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const int r = r0 + a, jb = ct + 64 * c;
+                if (r >= p.rows || jb >= gp) continue;
+                sts_u4(stage_sa + r * rb + 16 * jb,
+                       live[a][c] ? sp_poincare_pair(in[a][c][0], in[a][c][1], in[a][c][2])
+                                  : make_uint4(0u, 0u, 0u, 0u));
+            }
+    }
+}
+
 // ROWS, NSP > 0: input rows per tile and pairs per filter row known at compile time (the
 // MMA issue loop is then fully unrolled with constant descriptor offsets); 0 = run time.
-template <int ROWS, int NSP, int ACT>
+template <int ROWS, int NSP, int ACT, bool RGB = false>
 __global__ void __launch_bounds__(SP_THREADS, 1)
     qconv_stem_pool_kernel(const __grid_constant__ CUtensorMap tmap_x, const StemPoolParams p) {
     using C = SpCfg;
@@ -252,6 +332,8 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
     const uint32_t acce0 = accf0 + 8u * SP_NACC;
     const uint32_t drain0 = acce0 + 8u * SP_NACC;
     const uint32_t bready_bar = drain0 + 8u * SP_ISSUERS;
+    const uint32_t rgbf0 = bready_bar + 8u;  // RGB staging slots: full, then empty
+    const uint32_t rgbe0 = rgbf0 + 8u * SP_RGB_SLOTS;
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const ConvShape& s = p.s;
@@ -269,8 +351,9 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
     griddep_launch_dependents();
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
-            mbar_init(full_bar(i), 1);
-            mbar_init(empty_bar(i), 1);
+            mbar_init(full_bar(i), RGB ? 2 : 1);  // RGB: the two converter warps
+            // RGB: a stage is also read by the next tile (the rows the two share)
+            mbar_init(empty_bar(i), RGB ? 2 : 1);
         }
         for (int b = 0; b < SP_NACC; ++b) {
             mbar_init(accf0 + 8u * b, 1);
@@ -278,6 +361,10 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
         }
         for (int i = 0; i < SP_ISSUERS; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(bready_bar, SP_EXP_WARPS);
+        for (int i = 0; i < SP_RGB_SLOTS; ++i) {
+            mbar_init(rgbf0 + 8u * i, 1);
+            mbar_init(rgbe0 + 8u * i, 2);
+        }
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -292,7 +379,80 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
     const uint32_t tmem_base = *tmem_slot;
     griddep_wait();  // the previous kernel's output (this layer's input) is complete
 
-    if (warp == 0) {
+    if (RGB && (warp == 0 || warp == 3)) {
+        // ------------------------------------------------- RGB staging and conversion
+        // (warp 3 first helps with the weight expansion)
+        if (warp == 3) sp_expand<RAW>(p, smem, (warp - SP_EXP_WARP0) * 32 + lane, lane, bready_bar);
+        const int ct = (warp == 0 ? 0 : 32) + lane;
+        const uint64_t pol_x = l2_policy_evict_first();
+        const uint32_t tx = static_cast<uint32_t>(p.rows * p.rgb_row_bytes);
+        uint32_t filled = 0, fill_parity = 0;
+        int img = static_cast<int>(rfirst / p.Hp);
+        int i = static_cast<int>(rfirst - static_cast<long long>(img) * p.Hp);
+        int nimg = img, ni = i;  // the next tile to load
+        auto load_next = [&](int k) -> bool {  // warp 0 lane 0: staging slot of tile k
+            const int sl = k % SP_RGB_SLOTS;
+            const uint32_t ph = static_cast<uint32_t>(k / SP_RGB_SLOTS) & 1u;
+            if (!wait_or_abort(rgbe0 + 8u * sl, ph ^ 1u, limit, abort_flag,
+                               STATUS_TIMEOUT_PRODUCER))
+                return false;
+            mbar_arrive_expect_tx(rgbf0 + 8u * sl, tx);
+            filled |= 1u << sl;
+            fill_parity = (fill_parity & ~(1u << sl)) | (ph << sl);
+            tma_load_4d(sbase + p.rgb_off + sl * p.rgb_stage_bytes, &tmap_x, rgbf0 + 8u * sl, 0,
+                        0, 4 * ni - s.pad, nimg, pol_x);
+            if (++ni == p.Hp) {
+                ni = 0;
+                ++nimg;
+            }
+            return true;
+        };
+        bool ok = true;
+        if (warp == 0 && lane == 0)
+            for (int k = 0; ok && k < SP_RGB_SLOTS - 1 && k < ntiles; ++k) ok = load_next(k);
+        StageCursor cur(p.per);
+        int ki = 0, prev_stage = -1;
+        for (int k = 0; k < ntiles; ++k) {
+            const int stage = cur.stage(ki);
+            const uint32_t phase = cur.phase;
+            if (++ki == SP_ISSUERS) {
+                ki = 0;
+                cur.next();
+            }
+            // rows shared with the previous tile (same image): copied, not mapped again
+            // (rows 4 .. rows - 1 of every stage are written, so the next tile's rows
+            // 0 .. rows - 6, rows 4 .. rows - 2 here, are always in this tile's stage)
+            const int r_begin = (prev_stage >= 0 && i != 0 && p.rows > 5) ? 4 : 0;
+            const int sl = k % SP_RGB_SLOTS;
+            if (warp == 0 && lane == 0 && ok && k + SP_RGB_SLOTS - 1 < ntiles)
+                ok = load_next(k + SP_RGB_SLOTS - 1);
+            if (lane == 0 && ok)
+                ok = wait_or_abort(rgbf0 + 8u * sl,
+                                   static_cast<uint32_t>(k / SP_RGB_SLOTS) & 1u, limit,
+                                   abort_flag, STATUS_TIMEOUT_PRODUCER) &&
+                     wait_or_abort(empty_bar(stage), phase ^ 1u, limit, abort_flag,
+                                   STATUS_TIMEOUT_PRODUCER);
+            ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+            // both converter warps leave together; the barrier also orders the previous
+            // tile's stage writes (of both warps) before this tile's copies from it
+            if (named_bar_or(7, 64, !ok)) break;
+            sp_convert_rgb<4>(p, sbase + C::RING_OFF + stage * p.stage_bytes, r_begin,
+                              sbase + p.rgb_off + sl * p.rgb_stage_bytes, 4 * i - s.pad, ct);
+            prev_stage = stage;
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(full_bar(stage));
+                mbar_arrive(rgbe0 + 8u * sl);
+            }
+            if (++i == p.Hp) {
+                i = 0;
+                ++img;
+            }
+        }
+        if (warp == 0 && lane == 0 && (!ok || *abort_flag))
+            drain_fills(rgbf0, SP_RGB_SLOTS, filled, fill_parity, limit);
+    } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
             const uint64_t pol_x = l2_policy_evict_normal();
@@ -350,6 +510,11 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
             const uint32_t a_lo0 = desc_lo(sbase + C::A_OFF);
             const uint32_t row_lo = static_cast<uint32_t>(p.row_bytes) >> 4;
             StageCursor cur(p.per);
+            // RGB: tile k's rows 0..3 are rows 4..7 of tile k - 1's stage unless tile k
+            // starts an image (the converters write rows 4..rows-1 of every stage); that
+            // stage is the other issuer's (the same round, or the previous one)
+            StageCursor prev_cur(p.per);
+            const int other = 1 - me;
             for (int k = me; ok && k < ntiles; k += SP_ISSUERS) {
                 int buf;
                 uint32_t use;
@@ -357,6 +522,17 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
                 const int stage = cur.stage(me);
                 const uint32_t phase = cur.phase;
                 cur.next();
+                int prev_stage = -1, r_shared = 0;
+                if constexpr (RGB) {
+                    // tile k - 1 is the other issuer's: for me = 1 the same round, for me = 0
+                    // the previous round (prev_cur lags by one round for issuer 0)
+                    if (k >= 1) {
+                        prev_stage = prev_cur.stage(other);
+                        const long long rk = rfirst + k;
+                        if (rk % p.Hp != 0 && p.rows > 5) r_shared = 4;
+                    }
+                    if (me == 1 || k >= 1) prev_cur.next();
+                }
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA) ||
                     !wait_or_abort(full_bar(stage), phase, limit, abort_flag,
@@ -368,26 +544,36 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * SP_BUF_COLS);
                 const uint32_t b_lo0 =
                     desc_lo(sbase + C::RING_OFF + stage * p.stage_bytes) + p.d0;
+                // rows below r_shared (0..3): rows r + 4 of the previous tile's stage
+                const uint32_t p_lo0 =
+                    desc_lo(sbase + C::RING_OFF + (prev_stage < 0 ? 0 : prev_stage) *
+                                                      p.stage_bytes) + p.d0 + 4 * row_lo;
                 if constexpr (ROWS > 0) {
 #pragma unroll
-                    for (int r = 0; r < ROWS; ++r)
+                    for (int r = 0; r < ROWS; ++r) {
+                        const uint32_t rlo = (RGB && r < r_shared) ? p_lo0 + r * row_lo
+                                                                   : b_lo0 + r * row_lo;
 #pragma unroll
                         for (int t = 0; t < NSP / 2; ++t) {
                             const int u = r * (NSP / 2) + t;
                             umma_f16_w(d, a_lo0 + ((u * C::CHUNK) >> 4), C::A_DESC_HI,
-                                       b_lo0 + r * row_lo + 2 * t, C::B_DESC_HI, idesc,
-                                       u != 0 ? 1u : 0u);
+                                       rlo + 2 * t, C::B_DESC_HI, idesc, u != 0 ? 1u : 0u);
                         }
+                    }
                 } else {
                     int u = 0;
-                    for (int r = 0; r < rows; ++r)
+                    for (int r = 0; r < rows; ++r) {
+                        const uint32_t rlo = (RGB && r < r_shared) ? p_lo0 + r * row_lo
+                                                                   : b_lo0 + r * row_lo;
                         for (int t = 0; t < half; ++t, ++u)
                             umma_f16_w(d, a_lo0 + ((u * C::CHUNK) >> 4), C::A_DESC_HI,
-                                       b_lo0 + r * row_lo + 2 * t, C::B_DESC_HI, idesc,
-                                       u != 0 ? 1u : 0u);
+                                       rlo + 2 * t, C::B_DESC_HI, idesc, u != 0 ? 1u : 0u);
+                    }
                 }
                 ++issued;
                 umma_commit(empty_bar(stage));
+                // RGB: the previous tile's stage is free once this tile's MMAs are done too
+                if (RGB && prev_stage >= 0) umma_commit(empty_bar(prev_stage));
                 umma_commit(accf0 + 8u * buf);
             }
             if (!ok && issued > 0) {

@@ -923,19 +923,39 @@ cudaError_t launch_pw(const ConvShape& s, const void* x, const void* const w[4],
     return launch_pw_kernel<2, 0>(maps[0], prm, grid, stream);
 }
 
-template <int ROWS, int NSP, int ACT>
+// fp32 RGB pixels [N][H][W][3] viewed as [N][H][3 W / 32][32]: boxes of `rows` whole rows
+// (128-byte elements; W a multiple of 32).
+bool encode_rgb_rows(CUtensorMap* map, const ConvShape& s, const float* rgb, int rows) {
+    const cuuint64_t rb = 12ull * s.W;  // bytes per row
+    const cuuint64_t dims[4] = {32, static_cast<cuuint64_t>(3 * s.W / 32),
+                                static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
+    const cuuint64_t strides[3] = {128, rb, rb * s.H};
+    const cuuint32_t box[4] = {32, static_cast<cuuint32_t>(3 * s.W / 32),
+                               static_cast<cuuint32_t>(rows), 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = g_encode_tiled(
+        map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<float*>(rgb), dims, strides, box,
+        estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int ROWS, int NSP, int ACT, bool RGB>
 cudaError_t launch_stem_pool_kernel(const CUtensorMap& map, const StemPoolParams& prm, int grid,
                                     cudaStream_t stream) {
-    auto kern = qconv_stem_pool_kernel<ROWS, NSP, ACT>;
+    auto kern = qconv_stem_pool_kernel<ROWS, NSP, ACT, RGB>;
     static std::atomic<unsigned long long> attr_done{0};
     cudaError_t e = set_smem_once(kern, SpCfg::SMEM_BYTES, attr_done);
     if (e != cudaSuccess) return e;
     return launch_pdl(kern, dim3(grid), dim3(SP_THREADS), SpCfg::SMEM_BYTES, stream, map, prm);
 }
 
+// x: bf16 quaternion pixels [N][H][W][4], or (rgb) fp32 RGB pixels [N][H][W][3] mapped by
+// Eq. 4 in the kernel's loader.
 cudaError_t launch_stem_pool(const ConvShape& s, const void* x, const void* const w[4],
                              const EpilogueArgs& ep, void* out, const TcOptions& opt,
-                             int num_sms, cudaStream_t stream, char* err, size_t errlen) {
+                             int num_sms, cudaStream_t stream, char* err, size_t errlen,
+                             bool rgb = false) {
     StemPoolParams prm;
     prm.s = s;
     prm.ep = ep;
@@ -956,9 +976,15 @@ cudaError_t launch_stem_pool(const ConvShape& s, const void* x, const void* cons
     prm.row_bytes = boxg * 16 * prm.group;
     prm.rows = s.kh + 2;
     prm.stage_bytes = (prm.rows * prm.row_bytes + 1023) & ~1023;
-    int per = SpCfg::RING_BYTES / prm.stage_bytes / SP_ISSUERS;
+    prm.rgb = rgb ? static_cast<const float*>(x) : nullptr;
+    prm.rgb_row_bytes = 12 * s.W;
+    prm.rgb_stage_bytes = rgb ? (prm.rows * prm.rgb_row_bytes + 1023) & ~1023 : 0;
+    int per = (SpCfg::RING_BYTES - SP_RGB_SLOTS * prm.rgb_stage_bytes) / prm.stage_bytes /
+              SP_ISSUERS;
     if (per > SpCfg::MAX_PER) per = SpCfg::MAX_PER;
-    if (!stem_pool_ok(s) || per < 1 || boxg > 256 || prm.rows > 256) {
+    prm.rgb_off = SpCfg::RING_OFF + SP_ISSUERS * per * prm.stage_bytes;
+    if (!stem_pool_ok(s) || per < 1 || boxg > 256 || prm.rows > 256 ||
+        (rgb && (s.W % 32 != 0 || 3 * s.W / 32 > 256))) {
         snprintf(err, errlen, "stem pooling kernel: kh=%d kw=%d W=%d does not fit", s.kh, s.kw,
                  s.W);
         return cudaErrorInvalidValue;
@@ -971,10 +997,12 @@ cudaError_t launch_stem_pool(const ConvShape& s, const void* x, const void* cons
         snprintf(err, errlen, "too many pooled rows");
         return cudaErrorInvalidValue;
     }
-    const MapKey key = make_key(s, x, w, out, 1, 16, 7);
+    const MapKey key = make_key(s, x, w, out, 1, 16, rgb ? 9 : 7);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        if (!encode_x_pairs(&maps[0], s, x, prm.group, boxg, prm.rows)) {
+        const bool okx = rgb ? encode_rgb_rows(&maps[0], s, static_cast<const float*>(x), prm.rows)
+                             : encode_x_pairs(&maps[0], s, x, prm.group, boxg, prm.rows);
+        if (!okx) {
             snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
             return cudaErrorInvalidValue;
         }
@@ -982,15 +1010,21 @@ cudaError_t launch_stem_pool(const ConvShape& s, const void* x, const void* cons
         cache_store(key, maps);
     }
     const int grid = grid_for(opt, num_sms, static_cast<int>(prm.total_rows));
-    set_kernel_name("qconv_stem_pool_kernel");
-    if (prm.rows == 9 && prm.nsp == 4) {  // the 7x7 stem
-        if (s.act == 1) return launch_stem_pool_kernel<9, 4, 1>(maps[0], prm, grid, stream);
-        if (s.act == 2) return launch_stem_pool_kernel<9, 4, 2>(maps[0], prm, grid, stream);
-        return launch_stem_pool_kernel<9, 4, 0>(maps[0], prm, grid, stream);
+    set_kernel_name(rgb ? "qconv_stem_pool_kernel<rgb>" : "qconv_stem_pool_kernel");
+#define QUAN_SP_LAUNCH(R)                                                                    \
+    if (prm.rows == 9 && prm.nsp == 4) { /* the 7x7 stem */                                  \
+        if (s.act == 1) return launch_stem_pool_kernel<9, 4, 1, R>(maps[0], prm, grid, stream); \
+        if (s.act == 2) return launch_stem_pool_kernel<9, 4, 2, R>(maps[0], prm, grid, stream); \
+        return launch_stem_pool_kernel<9, 4, 0, R>(maps[0], prm, grid, stream);                \
+    }                                                                                        \
+    if (s.act == 1) return launch_stem_pool_kernel<0, 0, 1, R>(maps[0], prm, grid, stream);    \
+    if (s.act == 2) return launch_stem_pool_kernel<0, 0, 2, R>(maps[0], prm, grid, stream);    \
+    return launch_stem_pool_kernel<0, 0, 0, R>(maps[0], prm, grid, stream);
+    if (rgb) {
+        QUAN_SP_LAUNCH(true)
     }
-    if (s.act == 1) return launch_stem_pool_kernel<0, 0, 1>(maps[0], prm, grid, stream);
-    if (s.act == 2) return launch_stem_pool_kernel<0, 0, 2>(maps[0], prm, grid, stream);
-    return launch_stem_pool_kernel<0, 0, 0>(maps[0], prm, grid, stream);
+    QUAN_SP_LAUNCH(false)
+#undef QUAN_SP_LAUNCH
 }
 
 // ---------------------------------------------------------------- weight gradient
@@ -1254,6 +1288,23 @@ cudaError_t launch_qconv_stem_pool(const ConvShape& s, const void* x, const void
         return cudaErrorInvalidValue;
     }
     return launch_stem_pool(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+}
+
+bool tc_stem_pool_rgb_supported(const ConvShape& s, const float* rgb, const void* const w[4],
+                                const void* out, const EpilogueArgs& ep) {
+    return stem_pool_ok(s) && s.W % 32 == 0 && 3 * s.W / 32 <= 256 &&
+           tc_supported(s, rgb, w, out, ep);
+}
+
+cudaError_t launch_qconv_stem_pool_rgb(const ConvShape& s, const float* rgb,
+                                       const void* const w[4], const EpilogueArgs& ep, void* out,
+                                       const TcOptions& opt, int num_sms, cudaStream_t stream,
+                                       char* err, size_t errlen) {
+    if (!load_encoders()) {
+        snprintf(err, errlen, "cuTensorMapEncodeTiled is not available");
+        return cudaErrorInvalidValue;
+    }
+    return launch_stem_pool(s, rgb, w, ep, out, opt, num_sms, stream, err, errlen, true);
 }
 
 bool bwd_weight_tc_supported(const ConvShape& s, const void* x, const void* dy) {

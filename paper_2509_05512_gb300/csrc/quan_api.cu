@@ -625,6 +625,59 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
     return QUAN_OK;
 }
 
+quan_status_t quan_qconv2d_maxpool_rgb_fwd(const float* rgb, const void* wr, const void* wi,
+                                           const void* wj, const void* wk, const float* bias,
+                                           const float* iqbn_scale, const float* iqbn_shift,
+                                           int N, int H, int W, int Cout, int kh, int kw,
+                                           int stride, int pad, int act, void* out,
+                                           quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    if (!rgb || !wr || !wi || !wj || !wk || !out)
+        return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");
+    quan::ConvShape s;
+    quan_status_t st = geometry(&s, N, H, W, 4, Cout, kh, kw, stride, pad);
+    if (st != QUAN_OK) return st;
+    if ((iqbn_scale == nullptr) != (iqbn_shift == nullptr))
+        return fail(QUAN_ERR_INVALID_ARG, "iqbn_scale and iqbn_shift must both be given or both NULL");
+    if (act < QUAN_ACT_NONE || act > QUAN_ACT_SILU)
+        return fail(QUAN_ERR_INVALID_ARG, "unknown activation %d", act);
+    s.act = act;
+    const int pw = (s.Wo - 1) / 2 + 1, ph = (s.Ho - 1) / 2 + 1;
+    const size_t ob = static_cast<size_t>(N) * ph * pw * Cout * 2;
+    const size_t rb = static_cast<size_t>(N) * H * W * 12, wb = w_bytes(s, 2);
+    const size_t vb = static_cast<size_t>(Cout) * 4;
+    if (overlaps(out, ob, rgb, rb) || overlaps(out, ob, wr, wb) || overlaps(out, ob, wi, wb) ||
+        overlaps(out, ob, wj, wb) || overlaps(out, ob, wk, wb) || overlaps(out, ob, bias, vb) ||
+        overlaps(out, ob, iqbn_scale, vb) || overlaps(out, ob, iqbn_shift, vb))
+        return fail(QUAN_ERR_INVALID_ARG, "out overlaps an input");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    const quan::EpilogueArgs ep{bias, iqbn_scale, iqbn_shift, nullptr};
+    if (cc != 103 || !quan::tc_stem_pool_rgb_supported(s, rgb, w, out, ep))
+        return fail(QUAN_ERR_UNSUPPORTED,
+                    "the RGB stem pooling needs sm_103, Cout = 64, stride 2, W a multiple of "
+                    "32, Wo <= 128, the stem's filter limits and 16-byte aligned tensors");
+    quan::TcOptions opt;
+    opt.kappa = 0;
+    opt.bnq = 0;
+    opt.max_ctas = g_max_ctas.load();
+    opt.mode = 0;
+    opt.ws_halo = 1;
+    opt.ws_issuers = 0;
+    opt.wait_limit_ns = g_wait_limit.load();
+    opt.inject_stall = g_inject.load();
+    char err[256] = "";
+    e = quan::launch_qconv_stem_pool_rgb(s, rgb, w, ep, out, opt, num_sms,
+                                         reinterpret_cast<cudaStream_t>(stream), err,
+                                         sizeof(err));
+    if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+    if (e != cudaSuccess) return cuda_fail(e, "qconv_stem_pool launch");
+    t_last_path = QUAN_PATH_TC;
+    t_last_kernel = quan::last_tc_kernel();
+    return QUAN_OK;
+}
+
 quan_status_t quan_maxpool2d_fwd(const void* x, int N, int H, int W, int C, int k, int stride,
                                  int pad, void* out, quan_stream_t stream) {
     if (!x || !out) return fail(QUAN_ERR_INVALID_ARG, "null tensor pointer");

@@ -232,6 +232,13 @@ def backbone_input(N: int = 256, H: int = 224, seed: int = 4, n_images: int | No
     return to_bf16_bits(x)
 
 
+def backbone_rgb(N: int = 256, H: int = 224, seed: int = 4, n_images: int | None = None):
+    """Backbone RGB image batch for the Eq. 4 input mapping, fp32 [N][H][H][3] ~ U(0, 1)."""
+    rng = np.random.default_rng((seed, 1001))
+    rgb = rng.uniform(0.0, 1.0, size=(N, H, H, 3)).astype(np.float32)
+    return rgb if n_images is None else rgb[:n_images]
+
+
 def backbone_params(layer: BackboneLayer) -> dict:
     """Weights and IQBN vectors of one backbone convolution (no activations drawn)."""
     spec = layer.spec

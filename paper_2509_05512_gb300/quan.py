@@ -68,6 +68,7 @@ def load():
         lib.quan_qconv2d_bwd_data.argtypes = _bwd_data_args
         lib.quan_qconv2d_sep_bwd_data.argtypes = _bwd_data_args
         lib.quan_qconv2d_maxpool_fwd.argtypes = _conv_args + [_vp, ctypes.c_size_t, _vp, _vp]
+        lib.quan_qconv2d_maxpool_rgb_fwd.argtypes = [_vp] * 8 + [_i] * 9 + [_vp, _vp]
         lib.quan_qconv2d_maxpool_workspace_size.argtypes = [_i] * 8
         lib.quan_qconv2d_maxpool_workspace_size.restype = ctypes.c_size_t
         lib.quan_iqbn_batch_stats.argtypes = [_vp, ctypes.c_longlong, _i, _vp, ctypes.c_size_t,
@@ -103,7 +104,7 @@ def load():
                      "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
                      "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
                      "quan_qconv2d_bwd_data_static", "quan_iqbn_batch_stats",
-                     "quan_qconv2d_maxpool_fwd",
+                     "quan_qconv2d_maxpool_fwd", "quan_qconv2d_maxpool_rgb_fwd",
                      "quan_iqbn_train_fwd",
                      "quan_qconv2d_sep_bwd_weight",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
@@ -359,6 +360,14 @@ def qconv2d_backward_weight(x, dy, *, kh, kw, stride=1, pad=0, separable=False, 
 
 def quan_qconv2d_maxpool_workspace_size(N, H, W, Cout, kh, kw, stride, pad) -> int:
     return load().quan_qconv2d_maxpool_workspace_size(N, H, W, Cout, kh, kw, stride, pad)
+
+
+def quan_qconv2d_maxpool_rgb_fwd(rgb, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W,
+                                 Cout, kh, kw, stride, pad, act, out, stream=None) -> None:
+    _check(load().quan_qconv2d_maxpool_rgb_fwd(_ptr(rgb), _ptr(wr), _ptr(wi), _ptr(wj),
+                                               _ptr(wk), _ptr(bias), _ptr(iqbn_scale),
+                                               _ptr(iqbn_shift), N, H, W, Cout, kh, kw, stride,
+                                               pad, act, _ptr(out), _stream(stream)))
 
 
 def quan_qconv2d_maxpool_fwd(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin,

@@ -156,3 +156,71 @@ def test_fused_bounded_wait_timeout_and_recovery():
         quan.quan_set_wait_limit_ns(0)
     d, out, ref_gpu = run_both(spec, quan.QUAN_ACT_RELU)
     assert torch.equal(out, ref_gpu)
+
+
+# ------------------------------------------------------------------ RGB input (Eq. 4 fused)
+
+def run_rgb(N, H, W, act, seed, max_ctas=0):
+    """The RGB stem-pool call and, for comparison, quan_poincare_fwd followed by the
+    quaternion-input call, on the same fp32 pixels and weights."""
+    spec = inputs.small_layer("stem_rgb", N, H, W, 4, 64, 7, 2, 3, seed=(904, seed), act=act)
+    d = inputs.layer_inputs(spec)
+    rgb_np = np.random.default_rng(905 + seed).uniform(0.0, 1.0, size=(N, H, W, 3))
+    rgb_np = rgb_np.astype(np.float32)
+    rgb = torch.from_numpy(rgb_np).cuda()
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    sc, sh = to_dev_f32(d["scale"]), to_dev_f32(d["shift"])
+    Ho, Wo = (H - 1) // 2 + 1, (W - 1) // 2 + 1
+    out = torch.full((N, (Ho - 1) // 2 + 1, (Wo - 1) // 2 + 1, 64), float("nan"),
+                     dtype=torch.bfloat16, device="cuda")
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 0)
+    try:
+        quan.quan_qconv2d_maxpool_rgb_fwd(rgb, *w, None, sc, sh, N, H, W, 64, 7, 7, 2, 3, act,
+                                          out)
+        torch.cuda.synchronize()
+        assert quan.quan_last_kernel() == "qconv_stem_pool_kernel<rgb>"
+        mapped = quan.poincare(rgb)
+        ref = torch.full_like(out, float("nan"))
+        quan.quan_qconv2d_maxpool_fwd(mapped, *w, None, sc, sh, N, H, W, 4, 64, 7, 7, 2, 3, act,
+                                      None, 0, ref)
+        torch.cuda.synchronize()
+    finally:
+        quan.quan_set_tc_tiles(0, 0, 0, 0)
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    return d, rgb_np, out, ref
+
+
+RGB_CASES = [
+    # name, N, H, W, act, max_ctas
+    ("square", 2, 32, 32, quan.QUAN_ACT_RELU, 0),
+    ("odd_h", 2, 35, 64, quan.QUAN_ACT_SILU, 0),      # Ho = 18, Hp = 9; 64 wide
+    ("wide", 1, 12, 224, quan.QUAN_ACT_RELU, 0),      # a full 112-pixel output row
+    ("bands", 3, 40, 32, quan.QUAN_ACT_NONE, 3),      # bands across images
+]
+
+
+@pytest.mark.parametrize("case", RGB_CASES, ids=[c[0] for c in RGB_CASES])
+def test_rgb_stem_pool_equals_mapping_then_stem_and_oracle(case):
+    name, N, H, W, act, max_ctas = case
+    d, rgb_np, out, ref = run_rgb(N, H, W, act, len(name), max_ctas)
+    assert torch.equal(out, ref)
+    # the oracle: Eq. 4 on the same fp32 pixels, rounded to bf16 as the kernel's loader
+    # stores them, then the stem convolution and the pooling in fp64
+    q = oracle.poincare(rgb_np.astype(np.float64))
+    q_bits = inputs.to_bf16_bits(q.astype(np.float32))
+    f = lambda k: host_f64(d[k], "bf16")
+    y = oracle.qconv2d(host_f64(q_bits, "bf16"), f("wr"), f("wi"), f("wj"), f("wk"), stride=2,
+                       pad=3, scale=d["scale"], shift=d["shift"], act=act)
+    assert_bf16_close(out_f64(out), oracle.maxpool2d(y, k=3, stride=2, pad=1), name)
+
+
+def test_rgb_stem_pool_rejects_width_not_multiple_of_32():
+    spec = inputs.small_layer("stem_rgb_w", 1, 16, 30, 4, 64, 7, 2, 3, seed=(906, 0))
+    d = inputs.layer_inputs(spec)
+    rgb = torch.zeros((1, 16, 30, 3), dtype=torch.float32, device="cuda")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    out = torch.empty((1, 4, 8, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(quan.QuanError) as ei:
+        quan.quan_qconv2d_maxpool_rgb_fwd(rgb, *w, None, None, None, 1, 16, 30, 64, 7, 7, 2, 3,
+                                          quan.QUAN_ACT_RELU, out)
+    assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
