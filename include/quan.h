@@ -367,7 +367,10 @@ const char* quan_last_kernel(void);
  * those; 5: pointwise, the MMA's rows the expanded block weight of 32 quaternion output
  * channels and its columns 256 streamed pixels, only for 1x1 filters with pad 0, stride 1
  * or 2 (even H and W), Cin a multiple of 64 up to 512, Cout a multiple of 128 and no
- * residual; mode 0 picks it for those).  Values that do not
+ * residual; mode 0 picks it for those; 6: CTA pairs (tcgen05 cta_group::2), M = 256 MMAs
+ * over two CTAs' pixels, each CTA keeping half of the signed block weight, only for
+ * Cout = 128, Cin a multiple of 64 and kh x kw x Cin <= 1152, and never chosen by mode 0).
+ * Values that do not
  * divide the layer, or a tile that does not fit in shared memory, make the call fail
  * with QUAN_ERR_UNSUPPORTED.
  */

@@ -1,0 +1,457 @@
+// qconv_cg2.cuh -- weight-stationary quaternion convolution on CTA pairs (tcgen05
+// cta_group::2) for 32 quaternion output channels (Cout = 128 real), the backbone's
+// second stage.  Included by qconv_tc.cu inside its anonymous namespace.
+//
+// Why a pair.  An M = 128 MMA reads its A and B operands from shared memory at 128 bytes
+// per clock, so with N = 64 (two output components of 32 channels, the pair decomposition
+// of qconv_tc.cu) it costs the reads of 6 KB for 32 clocks of work; the whole signed block
+// weight of Eq. 6 for 128 -> 128 real channels and 9 taps (288 KB) does not fit one CTA's
+// shared memory, so N = 128 would have to re-expand letters on every tile.  A CTA pair
+// runs M = 256 MMAs: each CTA holds the A operand of its own 128 output pixels and HALF of
+// the block weight (output components 0-1 in the even CTA, 2-3 in the odd one: at most
+// 64 x 1152 bf16, 144 KB), expanded once per CTA and kept, and the tensor cores of the
+// two SMs exchange the B halves.  One MMA is 256 x 128 x 16: per SM 4 KB of A and 2 KB of
+// B for 64 clocks of work, so the operand reads leave room for the pixel stream.
+//
+//   A  pixels, one im2col box of 128 output pixels x 64 input channels of one tap per
+//      stage (16 KB, 128-byte swizzle);
+//   B  rows n = 32 q + co (real output channel c = q Qout + co = n), columns k = tap Cin +
+//      p Qin + ci: B[n][k] = sign(q, p) W_{q xor p}[co][tap][ci]; the CTA of rank r keeps
+//      rows 64 r .. 64 r + 63 as K-major 64-column chunks (128-byte swizzle);
+//   D  TMEM of each CTA: its 128 pixels x the 128 output channels.
+//
+// Roles.  Both CTAs: warp 0's lane 0 loads the CTA's pixel boxes into a stage ring (the
+// stages of local pair tile k belong to issuer k mod 2); warps 2..11 expand the CTA's B
+// half; warps 4..11 are the direct epilogue of the CTA's 128 pixels (tc_common.cuh's pair
+// epilogue, with the accumulator released to the even CTA).  Even CTA: warps 1 and 2
+// (lane 0) issue the pair's MMAs for alternate pair tiles, each into its own two of four
+// 128-column accumulators; a stage is handed back to both producers and an accumulator to
+// both epilogues by multicast commits.  Odd CTA: warp 1's lane 0 relays each of its landed
+// stages to the even CTA's full barrier (a cluster-scope arrive), so the issuer waits on
+// one barrier per stage.  Both CTAs allocate TMEM together (cta_group::2) and free it
+// after a cluster barrier.  Every wait is bounded as in the other kernels.
+
+constexpr int CG_THREADS = 384;
+constexpr int CG_NI = 2;              // MMA issuers of the even CTA
+constexpr int CG_NACC = 2 * CG_NI;    // accumulators of 128 columns
+constexpr int CG_BUF_COLS = 128;
+constexpr int CG_MAX_K = 1152;        // taps x Cin of the kept weight half (144 KB)
+constexpr int CG_EXP_WARP0 = 2;       // warps 2..11 expand the B half
+constexpr int CG_EXP_WARPS = 10;
+constexpr int CG_EPI_THREADS = 256;   // warps 4..11
+
+struct Cg2Params {
+    ConvShape s;
+    EpilogueArgs ep;
+    const __nv_bfloat16* w[4];  // letter tensors [32][kh][kw][Qin]
+    void* y;                    // output [M][128]
+    unsigned long long wait_limit_ns;
+    int inject_stall;
+    int kchunks;     // taps * Cin / 64
+    int cpt;         // Cin / 64: chunks per tap
+    int per;         // stages per issuer
+    int num_ptiles;  // pair tiles of 256 output pixels
+};
+
+struct CgCfg {
+    static constexpr int BCHUNK = 64 * 128;   // 64 weight rows x 64 channels
+    static constexpr int ACHUNK = 128 * 128;  // 128 pixels x 64 channels
+    static constexpr int MAX_STAGES = 12;
+    // full, empty (per stage), accf, acce (per accumulator), drain (per issuer), bready
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * CG_NACC + CG_NI + 1;
+    static constexpr int SMEM_BYTES = 227 * 1024;
+    static constexpr uint32_t DESC_HI = desc_hi(8 * 128, desc_layout(128));
+    static constexpr uint32_t TMEM_COLS = 512;
+    static_assert(NUM_BARS * 8 + 16 <= 1024, "pair barriers");
+    // B half at 0 (kchunks x 8 KB), barriers in the next 1 KB, the stage ring after them
+    __host__ __device__ static int ring_off(int kchunks) { return kchunks * BCHUNK + 1024; }
+    static int stages(int kchunks) {
+        const int n = (SMEM_BYTES - 1024 - ring_off(kchunks)) / ACHUNK;
+        return n < MAX_STAGES ? n : MAX_STAGES;
+    }
+};
+
+// Shapes the kernel covers: the full form, 32 quaternion output channels, Cin a multiple of
+// 64, taps x Cin <= 1152.
+bool cg2_ok(const ConvShape& s) {
+    if (s.sep || s.Qout != 32 || s.Cin % 64 != 0) return false;
+    return static_cast<long long>(s.kh) * s.kw * s.Cin <= CG_MAX_K;
+}
+
+// B half of CTA `rank`: 16-byte units (8 consecutive channels of one component, one letter
+// row), four loads in flight per thread; then the even CTA's bready barrier is told.
+__device__ __forceinline__ void cg2_expand(const Cg2Params& p, uint8_t* smem, uint32_t rank,
+                                           int et, int lane, uint32_t bready_leader) {
+    constexpr int ET = CG_EXP_WARPS * 32;
+    const ConvShape& s = p.s;
+    const int Qin = s.Qin, taps = s.kh * s.kw;
+    const int upr = taps * s.Cin / 8;  // units per row
+    const int total = 64 * upr;
+    for (int i0 = et; i0 < total; i0 += 4 * ET) {
+        uint4 v[4];
+        uint32_t off[4];
+        bool live[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            const int i = i0 + t * ET;
+            live[t] = i < total;
+            if (!live[t]) continue;
+            const int nl = i & 63, U = i >> 6;  // consecutive threads: consecutive rows
+            const int n = 64 * static_cast<int>(rank) + nl;
+            const int q = n >> 5, co = n & 31;
+            const int k = 8 * U, tap = k / s.Cin, cin = k - tap * s.Cin;
+            const int pc = cin / Qin, ci = cin - pc * Qin;
+            v[t] = __ldg(reinterpret_cast<const uint4*>(
+                p.w[q ^ pc] + (static_cast<long long>(co) * taps + tap) * Qin + ci));
+            if ((NEG_MASK >> (4 * q + pc)) & 1u) v[t] = negate_bf16x8(v[t]);
+            const int kc = U >> 3, u = U & 7;
+            off[t] = static_cast<uint32_t>(kc * CgCfg::BCHUNK + nl * 128 + ((u ^ (nl & 7)) << 4));
+        }
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+            if (live[t]) *reinterpret_cast<uint4*>(smem + off[t]) = v[t];
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(bready_leader);
+}
+
+// Bounded wait with cluster-scope acquire (arrivals from the peer CTA); otherwise as
+// wait_or_abort.
+__device__ __forceinline__ bool wait_cluster_or_abort(uint32_t bar, uint32_t parity,
+                                                      uint64_t limit, volatile int* abort_flag,
+                                                      unsigned code) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+        if (mbar_try_wait_sleep(bar, parity, WAIT_SUSPEND_NS) &&
+            mbar_try_wait_cluster(bar, parity))
+            return true;
+        if (*abort_flag) return false;
+        if (global_timer_ns() - t0 > limit) {
+            atomicOr(&g_status, code);
+            *abort_flag = 1;
+            return false;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(CG_THREADS, 1)
+    qconv_cg2_kernel(const __grid_constant__ CUtensorMap tmap_x, const Cg2Params p) {
+    using C = CgCfg;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const uint32_t sbase = smem_u32(smem);
+    const int bar_off = p.kchunks * C::BCHUNK;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + bar_off);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NUM_BARS);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int st) { return bar0 + 8u * st; };
+    auto empty_bar = [&](int st) { return bar0 + 8u * (C::MAX_STAGES + st); };
+    const uint32_t accf0 = bar0 + 8u * (2 * C::MAX_STAGES);
+    const uint32_t acce0 = accf0 + 8u * CG_NACC;
+    const uint32_t drain0 = acce0 + 8u * CG_NACC;
+    const uint32_t bready_bar = drain0 + 8u * CG_NI;
+    const uint32_t ring = sbase + static_cast<uint32_t>(C::ring_off(p.kchunks));
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const ConvShape& s = p.s;
+    const uint64_t limit = p.wait_limit_ns;
+    const uint32_t rank = cluster_ctarank();  // 0: the even CTA, which issues the MMAs
+    const int STAGES = CG_NI * p.per;
+    const int pair = static_cast<int>(blockIdx.x) >> 1;
+    const int npairs = static_cast<int>(gridDim.x) >> 1;
+    // this pair's tiles: pair + k npairs, k < kt; the CTA's pixels (2 t + rank) 128 ..
+    const int kt = pair < p.num_ptiles ? (p.num_ptiles - pair + npairs - 1) / npairs : 0;
+
+    griddep_launch_dependents();
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            // even CTA: its own fill (expect_tx) and the odd CTA's relay; odd CTA: its fill
+            mbar_init(full_bar(i), rank == 0 ? 2 : 1);
+            mbar_init(empty_bar(i), 1);  // the even CTA's multicast commit
+        }
+        for (int b = 0; b < CG_NACC; ++b) {
+            mbar_init(accf0 + 8u * b, 1);                   // multicast commit
+            mbar_init(acce0 + 8u * b, 2 * CG_EPI_THREADS);  // both CTAs' epilogues (even CTA)
+        }
+        for (int i = 0; i < CG_NI; ++i) mbar_init(drain0 + 8u * i, 1);
+        mbar_init(bready_bar, 2 * CG_EXP_WARPS);  // both CTAs' expansions (even CTA)
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) tma_prefetch_desc(&tmap_x);
+    if (warp == 1) {
+        tmem_alloc_cg2(smem_u32(tmem_slot), C::TMEM_COLS);
+        tmem_relinquish_cg2();
+    }
+    tc_fence_before();
+    __syncthreads();
+    // both CTAs' barriers exist before any cluster arrive or multicast commit reaches them
+    cluster_sync_all();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const int hw = s.Ho * s.Wo;
+    griddep_wait();  // the previous kernel's output (this layer's input) is complete
+    auto tile_origin = [&](int k, int& img, int& hbase, int& wbase) {
+        const long long last = (s.M - 1) / BM * BM;  // an odd CTA past the end loads a valid tile
+        long long m0 = (2ll * (pair + static_cast<long long>(k) * npairs) + rank) * BM;
+        if (m0 > last) m0 = last;
+        img = static_cast<int>(m0 / hw);
+        const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
+        const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
+        wbase = wo * s.stride - s.pad;
+        hbase = ho * s.stride - s.pad;
+    };
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            const uint64_t pol_x = l2_policy_evict_normal();
+            uint32_t filled = 0, fill_parity = 0;
+            bool ok = true;
+            StageCursor cur(p.per);
+            for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
+                const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
+                int img[CG_NI], hbase[CG_NI], wbase[CG_NI];
+#pragma unroll
+                for (int i = 0; i < CG_NI; ++i)
+                    if (i < ng) tile_origin(g0 + i, img[i], hbase[i], wbase[i]);
+                int ch = 0, dh = 0, dw = 0;  // K chunk kc = (tap, ch), walked without divisions
+                for (int kc = 0; ok && kc < p.kchunks; ++kc, cur.next()) {
+                    if (kc > 0 && ++ch == p.cpt) {
+                        ch = 0;
+                        if (++dw == s.kw) {
+                            dw = 0;
+                            ++dh;
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < CG_NI; ++i) {
+                        if (i >= ng) break;
+                        const int stage = cur.stage(i);
+                        const uint32_t phase = cur.phase;
+                        if (!wait_cluster_or_abort(empty_bar(stage), phase ^ 1u, limit,
+                                                   abort_flag, STATUS_TIMEOUT_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t fb = full_bar(stage);
+                        mbar_arrive_expect_tx(fb, C::ACHUNK);
+                        filled |= 1u << stage;
+                        fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
+                        tma_load_im2col_4d(ring + stage * C::ACHUNK, &tmap_x, fb, 64 * ch,
+                                           wbase[i], hbase[i], img[i],
+                                           static_cast<uint16_t>(dw), static_cast<uint16_t>(dh),
+                                           pol_x);
+                    }
+                }
+            }
+            if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
+        }
+    } else if (warp <= CG_NI) {
+        if (warp >= CG_EXP_WARP0)
+            cg2_expand(p, smem, rank, (warp - CG_EXP_WARP0) * 32 + lane, lane,
+                       mapa_shared(bready_bar, 0));
+        if (rank == 0 && lane == 0) {
+            // -------------------------------------------------- MMA issuers (even CTA)
+            constexpr uint32_t IDESC = make_idesc(2 * BM, 128, 0);
+            const int me = warp - 1;
+            const uint32_t drain_bar = drain0 + 8u * me;
+            bool ok = wait_cluster_or_abort(bready_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
+            int issued = 0;
+            if (p.inject_stall && me == 0) {
+                // Failure injection: wait on a barrier nothing arrives on.
+                wait_or_abort(drain_bar, 0, limit, abort_flag, STATUS_TIMEOUT_MMA);
+                ok = false;
+            }
+            tc_fence_after();
+            const uint32_t b_lo0 = desc_lo(sbase);
+            StageCursor cur(p.per);
+            for (int k = me; ok && k < kt; k += CG_NI) {
+                int buf;
+                uint32_t use;
+                issuer_acc_n<CG_NI>(k, buf, use);
+                if (!wait_cluster_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
+                                           STATUS_TIMEOUT_MMA)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem_base + static_cast<uint32_t>(buf * CG_BUF_COLS);
+                for (int kc = 0; kc < p.kchunks; ++kc) {
+                    const int stage = cur.stage(me);
+                    const uint32_t phase = cur.phase;
+                    cur.next();
+                    if (!wait_cluster_or_abort(full_bar(stage), phase, limit, abort_flag,
+                                               STATUS_TIMEOUT_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a_lo = desc_lo(ring + stage * C::ACHUNK);
+                    const uint32_t b_lo = b_lo0 + static_cast<uint32_t>((kc * C::BCHUNK) >> 4);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)  // 16-channel steps: 32 bytes into the row
+                        umma_f16_cg2(d, a_lo + 2 * kk, C::DESC_HI, b_lo + 2 * kk, C::DESC_HI,
+                                     IDESC, (kc | kk) != 0 ? 1u : 0u);
+                    ++issued;
+                    umma_commit_cg2(empty_bar(stage), 3);  // both CTAs may refill the stage
+                }
+                if (!ok) break;
+                umma_commit_cg2(accf0 + 8u * buf, 3);  // both CTAs' accumulators are ready
+            }
+            if (!ok && issued > 0) {
+                // let this issuer's MMAs finish before TMEM is released
+                umma_commit_cg2(drain_bar, 1);
+                const uint64_t t0 = global_timer_ns();
+                while (!mbar_try_wait(drain_bar, 0u)) {
+                    if (global_timer_ns() - t0 > limit) {
+                        atomicOr(&g_status, STATUS_TIMEOUT_DRAIN);
+                        break;
+                    }
+                }
+            }
+        } else if (rank == 1 && warp == 1 && lane == 0) {
+            // ---------------------------------- relay of the odd CTA's landed stages
+            const uint32_t full_leader0 = mapa_shared(full_bar(0), 0);
+            StageCursor cur(p.per);
+            bool ok = true;
+            for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
+                const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
+                for (int kc = 0; ok && kc < p.kchunks; ++kc, cur.next()) {
+                    for (int i = 0; i < ng; ++i) {
+                        const int stage = cur.stage(i);
+                        if (!wait_or_abort(full_bar(stage), cur.phase, limit, abort_flag,
+                                           STATUS_TIMEOUT_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_cluster(full_leader0 + 8u * stage);
+                    }
+                }
+            }
+        }
+    } else {
+        cg2_expand(p, smem, rank, (warp - CG_EXP_WARP0) * 32 + lane, lane,
+                   mapa_shared(bready_bar, 0));
+        if (warp >= EPI_WARP0) {
+            // ------------------------------------------------------------ epilogue
+            // (the pair epilogue of tc_common.cuh for 32 channels per component: warps 4..7
+            // take components r and i, warps 8..11 j and k; the accumulator is released to
+            // the even CTA, whose issuer refills it)
+            constexpr int BNQ = 32, CH = 32, NCH = 4, NB = 2;
+            const int quad = warp & 3;
+            const int half = (warp - EPI_WARP0) >> 2;
+            const int ci = lane % NCH;
+            const int row0 = quad * 32 + NCH * (lane / NCH);
+            const long long Cout = s.Cout;
+            const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(p.ep.residual);
+            __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.y);
+            const uint32_t acce_leader0 = mapa_shared(acce0, 0);
+            auto load_vectors = [&](int cb, float(&sc)[8], float(&sh)[8]) {
+                float bi[8];
+                load8(p.ep.scale, cb, 1.0f, sc);
+                load8(p.ep.shift, cb, 0.0f, sh);
+                load8(p.ep.bias, cb, 0.0f, bi);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) sh[e] = fmaf(sc[e], bi[e], sh[e]);
+            };
+            for (int k = 0; k < kt; ++k) {
+                int buf;
+                uint32_t use;
+                issuer_acc_n<CG_NI>(k, buf, use);
+                bool ok = true;
+                if (lane == 0)
+                    ok = wait_cluster_or_abort(accf0 + 8u * buf, use, limit, abort_flag,
+                                               STATUS_TIMEOUT_EPILOGUE);
+                ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+                if (named_bar_or(1, CG_EPI_THREADS, !ok)) break;
+                tc_fence_after();
+                const long long m0 = (2ll * (pair + static_cast<long long>(k) * npairs) + rank) * BM;
+                const long long left = s.M - m0;
+                const int rows = left <= 0 ? 0 : (left < BM ? static_cast<int>(left) : BM);
+                const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                                       static_cast<uint32_t>(buf * CG_BUF_COLS);
+                uint32_t va[CH], vb[CH];
+                float sca[8], sha[8], scb[8], shb[8];
+                tmem_ld_32x32b_x32(taddr + (2 * half) * BNQ, va);
+                load_vectors(8 * ci + (2 * half) * s.Qout, sca, sha);
+                tmem_ld_wait();
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    uint32_t(&v)[CH] = b ? vb : va;
+                    float(&sc)[8] = b ? scb : sca;
+                    float(&sh)[8] = b ? shb : sha;
+                    const int q = 2 * half + b;
+                    const int cb = 8 * ci + q * s.Qout;
+                    if (b == 0) {
+                        tmem_ld_32x32b_x32(taddr + (2 * half + 1) * BNQ, vb);
+                        load_vectors(8 * ci + (2 * half + 1) * s.Qout, scb, shb);
+                    } else {
+                        // the tile's accumulator is in registers: hand it back
+                        tc_fence_before();
+                        mbar_arrive_cluster(acce_leader0 + 8u * buf);
+                    }
+                    uint4 r4[NCH];
+                    if (res != nullptr) {
+#pragma unroll
+                        for (int kq = 0; kq < NCH; ++kq) {
+                            r4[kq] = make_uint4(0u, 0u, 0u, 0u);
+                            if (row0 + kq < rows)
+                                r4[kq] = ld_global_na(res + (m0 + row0 + kq) * Cout + cb);
+                        }
+                    }
+                    float E[NCH][8];
+#pragma unroll
+                    for (int j = 0; j < NCH; ++j)
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) E[j][e] = __uint_as_float(v[8 * j + e]);
+                    chunk_transpose_stage<2, 4>(E, ci);
+                    chunk_transpose_stage<1, 4>(E, ci);
+#pragma unroll
+                    for (int kq = 0; kq < NCH; ++kq) {
+                        float rz[8];
+                        if (res != nullptr) {
+                            const __nv_bfloat162* rh =
+                                reinterpret_cast<const __nv_bfloat162*>(&r4[kq]);
+#pragma unroll
+                            for (int t = 0; t < 4; ++t) {
+                                const float2 f = __bfloat1622float2(rh[t]);
+                                rz[2 * t] = f.x;
+                                rz[2 * t + 1] = f.y;
+                            }
+                        } else {
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) rz[e] = 0.0f;
+                        }
+                        uint32_t wv[4];
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            const float z0 = fmaf(sc[2 * t], E[kq][2 * t], sh[2 * t]) + rz[2 * t];
+                            const float z1 =
+                                fmaf(sc[2 * t + 1], E[kq][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
+                            wv[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                        }
+                        if (row0 + kq < rows)
+                            st_global_na(out + (m0 + row0 + kq) * Cout + cb,
+                                         make_uint4(wv[0], wv[1], wv[2], wv[3]));
+                    }
+                    if (b == 0) tmem_ld_wait();
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    // the pair's MMAs into both CTAs' TMEM and both epilogues are done
+    cluster_sync_all();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc_cg2(tmem_base, C::TMEM_COLS);
+    }
+}

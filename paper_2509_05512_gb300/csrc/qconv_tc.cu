@@ -450,6 +450,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #include "qconv_gather.cuh"
 #include "qconv_stempool.cuh"
 #include "qconv_pw.cuh"
+#include "qconv_cg2.cuh"
 #include "qconv_dw.cuh"
 
 // ---------------------------------------------------------------- host side
@@ -940,6 +941,62 @@ bool encode_rgb_rows(CUtensorMap* map, const ConvShape& s, const float* rgb, int
     return r == CUDA_SUCCESS;
 }
 
+cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4],
+                       const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
+                       cudaStream_t stream, char* err, size_t errlen) {
+    Cg2Params prm;
+    prm.s = s;
+    prm.ep = ep;
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.cpt = s.Cin / 64;
+    prm.kchunks = s.kh * s.kw * prm.cpt;
+    prm.per = CgCfg::stages(prm.kchunks) / CG_NI;
+    if (prm.per > CgCfg::MAX_STAGES / CG_NI) prm.per = CgCfg::MAX_STAGES / CG_NI;
+    const long long ptiles = (s.M + 2 * BM - 1) / (2 * BM);
+    if (!cg2_ok(s) || prm.per < 1 || ptiles > 0x7fffffffLL) {
+        snprintf(err, errlen, "CTA-pair kernel: Cin=%d Cout=%d %dx%d does not fit", s.Cin,
+                 s.Cout, s.kh, s.kw);
+        return cudaErrorInvalidValue;
+    }
+    prm.num_ptiles = static_cast<int>(ptiles);
+    const MapKey key = make_key(s, x, w, out, 64, 32, 10);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_im2col(&maps[0], s, x, 64)) {
+            snprintf(err, errlen, "cuTensorMapEncodeIm2col failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    int pairs = (opt.max_ctas > 0 ? opt.max_ctas : num_sms) / 2;
+    if (pairs > prm.num_ptiles) pairs = prm.num_ptiles;
+    if (pairs < 1) pairs = 1;
+    set_kernel_name("qconv_cg2_kernel");
+    auto kern = qconv_cg2_kernel;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * pairs);
+    cfg.blockDim = dim3(CG_THREADS);
+    cfg.dynamicSmemBytes = CgCfg::SMEM_BYTES;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, kern, maps[0], prm);
+}
+
 template <int ROWS, int NSP, int ACT, bool RGB>
 cudaError_t launch_stem_pool_kernel(const CUtensorMap& map, const StemPoolParams& prm, int grid,
                                     cudaStream_t stream) {
@@ -1163,6 +1220,17 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     }
     if (pw_ok(s, ep) && (opt.mode == 0 || opt.mode == 5))
         return launch_pw(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+    // The CTA-pair kernel only on request: at the backbone's stage-2 shapes its stage ring
+    // (what the kept weight half leaves of shared memory) is too shallow for the pixel
+    // loads' latency, and the pair kernel below is faster.
+    if (!s.sep && cg2_ok(s) && opt.mode == 6)
+        return launch_cg2(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+    if (opt.mode == 6) {
+        snprintf(err, errlen,
+                 "CTA-pair mode needs the full form, Cout = 128, Cin a multiple of 64 and "
+                 "kh x kw x Cin <= %d", CG_MAX_K);
+        return cudaErrorInvalidValue;
+    }
     if (opt.mode == 5) {
         snprintf(err, errlen,
                  "pointwise mode needs a 1x1 filter, pad 0, stride 1 or 2 (even H and W, "

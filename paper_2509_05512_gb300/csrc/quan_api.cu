@@ -713,7 +713,7 @@ const char* quan_last_kernel(void) { return t_last_kernel; }
 
 quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };
-    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 5)
+    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 6)
         return fail(QUAN_ERR_INVALID_ARG,
                     "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 4");
     g_kappa.store(kappa);

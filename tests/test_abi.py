@@ -59,8 +59,8 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_maxpool2d_fwd(FAKE, 1, 4, 4, 8, 3, 2, 2, FAKE * 64, None) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_path(5) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_tiles(24, 0, 0, 0) == quan.QUAN_ERR_INVALID_ARG
-    assert lib.quan_set_tc_tiles(0, 0, 0, 6) == quan.QUAN_ERR_INVALID_ARG
-    assert lib.quan_set_tc_tiles(0, 0, 0, 5) == quan.QUAN_OK
+    assert lib.quan_set_tc_tiles(0, 0, 0, 7) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_tiles(0, 0, 0, 6) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 4) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 0) == quan.QUAN_OK
     assert lib.quan_poincare_fwd(None, 4, FAKE, None) == quan.QUAN_ERR_INVALID_ARG

@@ -316,6 +316,64 @@ def test_tc_pointwise_mode_rejects_other_shapes():
         assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
 
 
+# ------------------------------------------------------------------ CTA-pair kernel (Cout 128)
+
+CG2_CASES = [
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra
+    ("cg2_s1_res", 2, 14, 13, 128, 128, 3, 1, 1, {"residual": True}),   # 364 pixels: ragged
+    ("cg2_s2", 3, 15, 17, 64, 128, 3, 2, 1, {}),                         # 216 pixels
+    ("cg2_one_tile", 1, 8, 8, 128, 128, 3, 1, 1,                         # 64 pixels: the odd
+     {"bias": True, "act": quan.QUAN_ACT_SILU}),                         # CTA has none
+    ("cg2_no_iqbn", 2, 12, 12, 64, 128, 3, 1, 1, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
+    ("cg2_5x1", 2, 11, 9, 128, 128, 5, 1, 2, {"kw": 1}),                  # 5 taps x 128
+]
+
+
+@pytest.mark.parametrize("case", CG2_CASES, ids=[c[0] for c in CG2_CASES])
+def test_tc_cta_pair_layers(case):
+    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(213, len(name)), **extra)
+    quan.quan_set_tc_tiles(0, 0, 0, 6)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_cg2_kernel"
+
+
+@pytest.mark.parametrize("max_ctas", [4, 6])
+def test_tc_cta_pair_few_pairs(max_ctas):
+    # 2 or 3 pairs walk many pair tiles: every stage ring and all four accumulators wrap
+    spec = inputs.small_layer("cg2_few", 4, 20, 20, 128, 128, 3, 1, 1, residual=True,
+                              seed=(214, max_ctas))
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 6)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == "qconv_cg2_kernel"
+
+
+def test_tc_cta_pair_matches_pair_kernel():
+    # the stage-2 shape of the backbone on the CTA-pair and the pair kernel: both within the
+    # oracle's tolerance and close to each other
+    spec = inputs.small_layer("cg2_vs_pair", 2, 28, 28, 128, 128, 3, 1, 1, seed=(215, 0))
+    d = inputs.layer_inputs(spec)
+    ref = oracle_full(d)
+    outs = []
+    for mode in (6, 2):
+        quan.quan_set_tc_tiles(0, 0, 0, mode)
+        got, used = run_gpu(d, path=quan.QUAN_PATH_TC)
+        assert used == quan.QUAN_PATH_TC
+        assert_bf16_close(got, ref, "mode %d" % mode)
+        outs.append(got)
+    assert_bf16_close(outs[0], outs[1], "pair of CTAs vs pair kernel")
+
+
+def test_tc_cta_pair_mode_rejects_other_shapes():
+    for args in ((1, 8, 8, 64, 64, 3, 1, 1), (1, 8, 8, 192, 128, 3, 1, 1)):  # Cout 64; K > 1152
+        spec = inputs.small_layer("not_cg2", *args, seed=(216, 0))
+        d = inputs.layer_inputs(spec)
+        quan.quan_set_tc_tiles(0, 0, 0, 6)
+        with pytest.raises(quan.QuanError) as ei:
+            run_gpu(d, path=quan.QUAN_PATH_TC)
+        assert ei.value.status == quan.QUAN_ERR_UNSUPPORTED
+
+
 def test_tc_nonsquare_kernel():
     spec = inputs.small_layer("k3x1", 2, 9, 10, 64, 64, 3, 1, 1, kw=1, seed=(203, 0))
     # pad 1 on both sides with kw = 1 widens the output; valid for the oracle too
@@ -500,14 +558,16 @@ def test_maxpool(shape):
 
 # ------------------------------------------------------------------ failure detection
 
-@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0)])
+@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0), (6, 0)])
 def test_bounded_wait_timeout_every_kernel(mode, issuers):
     # the failure-injection path of the pair-mode, weight-stationary (two and three
-    # issuers), gather and pointwise kernels
+    # issuers), gather, pointwise and CTA-pair kernels
     if mode == 4:
         spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
     elif mode == 5:
         spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 1, 1, 0, seed=(401, mode))
+    elif mode == 6:
+        spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 3, 1, 1, seed=(401, mode))
     else:
         spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
     d = inputs.layer_inputs(spec)
