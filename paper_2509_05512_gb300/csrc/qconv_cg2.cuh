@@ -7,23 +7,40 @@
 // of qconv_tc.cu) it costs the reads of 6 KB for 32 clocks of work; the whole signed block
 // weight of Eq. 6 for 128 -> 128 real channels and 9 taps (288 KB) does not fit one CTA's
 // shared memory, so N = 128 would have to re-expand letters on every tile.  A CTA pair
-// runs M = 256 MMAs: each CTA holds the A operand of its own 128 output pixels and HALF of
+// runs M = 256 MMAs: each CTA holds the A operand of its own output pixels and HALF of
 // the block weight (output components 0-1 in the even CTA, 2-3 in the odd one: at most
 // 64 x 1152 bf16, 144 KB), expanded once per CTA and kept, and the tensor cores of the
 // two SMs exchange the B halves.  One MMA is 256 x 128 x 16: per SM 4 KB of A and 2 KB of
 // B for 64 clocks of work, so the operand reads leave room for the pixel stream.
 //
-//   A  pixels, one im2col box of 128 output pixels x 64 input channels of one tap per
-//      stage (16 KB, 128-byte swizzle);
+//   A  pixels, K-major rows of 64 input channels (128 bytes, 128-byte swizzle), staged in
+//      one of two ways:
+//        halo  (stride 1, 3x3, Wp = Wo + 2 <= 128): a CTA tile is R = 128 / Wp output rows
+//              of one image, and one TMA box per 64-channel chunk holds the R + 2 input rows
+//              it reads at Wp columns -pad .. Wo + 1 - pad (zero fill outside the image),
+//              row after row at a pitch of Wp pixels.  MMA row m = r Wp + c is output pixel
+//              (r, c) (c >= Wo: padding, computed and not stored), and filter tap (dh, dw)
+//              reads box row m + dh Wp + dw: every tap is the same box seen from another
+//              start row.  The MMA applies the 128-byte swizzle to absolute shared-memory
+//              addresses, as the TMA unit wrote it, so any 128-byte row offset is a valid
+//              start (the descriptor's base-offset field stays 0).  One stage feeds
+//              9 x 4 MMAs;
+//        per tap  otherwise: one im2col box of 128 consecutive output pixels x 64 input
+//              channels per (tap, chunk) stage (4 MMAs);
 //   B  rows n = 32 q + co (real output channel c = q Qout + co = n), columns k = tap Cin +
 //      p Qin + ci: B[n][k] = sign(q, p) W_{q xor p}[co][tap][ci]; the CTA of rank r keeps
 //      rows 64 r .. 64 r + 63 as K-major 64-column chunks (128-byte swizzle);
-//   D  TMEM of each CTA: its 128 pixels x the 128 output channels.
+//   D  TMEM of each CTA: its 128 MMA rows x the 128 output channels.
 //
-// Roles.  Both CTAs: warp 0's lane 0 loads the CTA's pixel boxes into a stage ring (the
-// stages of local pair tile k belong to issuer k mod 2); warps 2..11 expand the CTA's B
-// half; warps 4..11 are the direct epilogue of the CTA's 128 pixels (tc_common.cuh's pair
-// epilogue, with the accumulator released to the even CTA).  Even CTA: warps 1 and 2
+// The letters reach shared memory as four bulk copies (each letter tensor whole, into the
+// space the pixel ring takes over afterwards) and are expanded shared -> shared: each
+// 16-byte chunk of a letter is read once and written to its two places in this CTA's half
+// (q = 2 r, 2 r + 1 with p = L xor q), with Eq. 5's sign.
+//
+// Roles.  Both CTAs: warp 0's lane 0 loads the letters, then the CTA's pixel boxes into a
+// stage ring (the stages of local pair tile k belong to issuer k mod 2); warps 2..11 expand
+// the CTA's B half; warps 4..11 are the direct epilogue of the CTA's 128 rows (tc_common.cuh's
+// pair epilogue, with the accumulator released to the even CTA).  Even CTA: warps 1 and 2
 // (lane 0) issue the pair's MMAs for alternate pair tiles, each into its own two of four
 // 128-column accumulators; a stage is handed back to both producers and an accumulator to
 // both epilogues by multicast commits.  Odd CTA: warp 1's lane 0 relays each of its landed
@@ -39,6 +56,7 @@ constexpr int CG_MAX_K = 1152;        // taps x Cin of the kept weight half (144
 constexpr int CG_EXP_WARP0 = 2;       // warps 2..11 expand the B half
 constexpr int CG_EXP_WARPS = 10;
 constexpr int CG_EPI_THREADS = 256;   // warps 4..11
+constexpr int CG_HALO_MAX_WP = 128;   // halo tiles: at least one padded output row per tile
 
 struct Cg2Params {
     ConvShape s;
@@ -47,73 +65,93 @@ struct Cg2Params {
     void* y;                    // output [M][128]
     unsigned long long wait_limit_ns;
     int inject_stall;
-    int kchunks;     // taps * Cin / 64
-    int cpt;         // Cin / 64: chunks per tap
-    int per;         // stages per issuer
-    int num_ptiles;  // pair tiles of 256 output pixels
+    int kchunks;       // taps * Cin / 64: 64-column chunks of the kept weight half
+    int cpt;           // Cin / 64: chunks per tap
+    int nst;           // stages per tile: cpt (halo) or kchunks (per tap)
+    int per;           // stages per issuer
+    int stage_bytes;   // one stage of the pixel ring (a multiple of 1024)
+    int box_bytes;     // bytes one stage's box delivers
+    int letter_bytes;  // one letter tensor, 32 x taps x Qin bf16
+    int num_tiles;     // CTA tiles
+    int num_ptiles;    // pair tiles: two consecutive CTA tiles
+    // halo staging
+    int Wp;            // Wo + 2: row pitch of a stage, in pixels
+    int R;             // output rows per tile: 128 / Wp
+    int tpi;           // tiles per image: ceil(Ho / R)
 };
 
 struct CgCfg {
     static constexpr int BCHUNK = 64 * 128;   // 64 weight rows x 64 channels
     static constexpr int ACHUNK = 128 * 128;  // 128 pixels x 64 channels
     static constexpr int MAX_STAGES = 12;
-    // full, empty (per stage), accf, acce (per accumulator), drain (per issuer), bready
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * CG_NACC + CG_NI + 1;
+    // full, empty (per stage), accf, acce (per accumulator), drain (per issuer), bready,
+    // letters landed, letters read
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * CG_NACC + CG_NI + 3;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr uint32_t DESC_HI = desc_hi(8 * 128, desc_layout(128));
     static constexpr uint32_t TMEM_COLS = 512;
     static_assert(NUM_BARS * 8 + 16 <= 1024, "pair barriers");
     // B half at 0 (kchunks x 8 KB), barriers in the next 1 KB, the stage ring after them
     __host__ __device__ static int ring_off(int kchunks) { return kchunks * BCHUNK + 1024; }
-    static int stages(int kchunks) {
-        const int n = (SMEM_BYTES - 1024 - ring_off(kchunks)) / ACHUNK;
-        return n < MAX_STAGES ? n : MAX_STAGES;
-    }
+    static int ring_bytes(int kchunks) { return SMEM_BYTES - 1024 - ring_off(kchunks); }
 };
 
 // Shapes the kernel covers: the full form, 32 quaternion output channels, Cin a multiple of
-// 64, taps x Cin <= 1152.
+// 64, taps x Cin <= 1152 (the four staged letters, 64 taps Cin bytes, then fit the ring).
 bool cg2_ok(const ConvShape& s) {
     if (s.sep || s.Qout != 32 || s.Cin % 64 != 0) return false;
     return static_cast<long long>(s.kh) * s.kw * s.Cin <= CG_MAX_K;
 }
 
-// B half of CTA `rank`: 16-byte units (8 consecutive channels of one component, one letter
-// row), four loads in flight per thread; then the even CTA's bready barrier is told.
-__device__ __forceinline__ void cg2_expand(const Cg2Params& p, uint8_t* smem, uint32_t rank,
-                                           int et, int lane, uint32_t bready_leader) {
+// Halo staging: stride 1, a 3x3 filter, output rows narrow enough for one per tile.
+bool cg2_halo_ok(const ConvShape& s) {
+    return cg2_ok(s) && s.stride == 1 && s.kh == 3 && s.kw == 3 && s.Wo + 2 <= CG_HALO_MAX_WP;
+}
+
+// This CTA's B half from the letters staged at `lsm` (letter L at L * letter_bytes, in the
+// global layout [32][taps][Qin]): chunk i (16 bytes) of letter L holds
+// W_L[co][tap][8 c8 .. 8 c8 + 7] with i = (co taps + tap) Qin / 8 + c8.  TAPS > 0: the tap
+// count known at compile time and Qin / 8 a power of two (1 << cpr_log2), so the chunk
+// index splits without run-time divisions.
+template <int TAPS>
+__device__ __forceinline__ void cg2_expand(const Cg2Params& p, uint32_t sbase, uint32_t lsm,
+                                           uint32_t rank, int et, int cpr_log2) {
     constexpr int ET = CG_EXP_WARPS * 32;
     const ConvShape& s = p.s;
-    const int Qin = s.Qin, taps = s.kh * s.kw;
-    const int upr = taps * s.Cin / 8;  // units per row
-    const int total = 64 * upr;
-    for (int i0 = et; i0 < total; i0 += 4 * ET) {
-        uint4 v[4];
-        uint32_t off[4];
-        bool live[4];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            const int i = i0 + t * ET;
-            live[t] = i < total;
-            if (!live[t]) continue;
-            const int nl = i & 63, U = i >> 6;  // consecutive threads: consecutive rows
-            const int n = 64 * static_cast<int>(rank) + nl;
-            const int q = n >> 5, co = n & 31;
-            const int k = 8 * U, tap = k / s.Cin, cin = k - tap * s.Cin;
-            const int pc = cin / Qin, ci = cin - pc * Qin;
-            v[t] = __ldg(reinterpret_cast<const uint4*>(
-                p.w[q ^ pc] + (static_cast<long long>(co) * taps + tap) * Qin + ci));
-            if ((NEG_MASK >> (4 * q + pc)) & 1u) v[t] = negate_bf16x8(v[t]);
-            const int kc = U >> 3, u = U & 7;
-            off[t] = static_cast<uint32_t>(kc * CgCfg::BCHUNK + nl * 128 + ((u ^ (nl & 7)) << 4));
+    const int Qin = s.Qin, taps = TAPS > 0 ? TAPS : s.kh * s.kw;
+    const int cpr = Qin >> 3;  // chunks per (co, tap)
+    const int per_letter = 32 * taps * cpr;
+    const int total = 4 * per_letter;
+    for (int i = et; i < total; i += ET) {
+        int L, co, tap, c8;
+        if constexpr (TAPS > 0) {
+            const int j = i >> cpr_log2;  // (32 L + co) TAPS + tap
+            c8 = i - (j << cpr_log2);
+            const int lc = j / TAPS;
+            tap = j - lc * TAPS;
+            L = lc >> 5;
+            co = lc & 31;
+        } else {
+            L = i / per_letter;
+            const int off = i - L * per_letter;
+            const int ct = off / cpr;
+            c8 = off - ct * cpr;
+            co = ct / taps;
+            tap = ct - co * taps;
         }
+        const uint4 v = lds_u4(lsm + static_cast<uint32_t>(i) * 16u);
 #pragma unroll
-        for (int t = 0; t < 4; ++t)
-            if (live[t]) *reinterpret_cast<uint4*>(smem + off[t]) = v[t];
+        for (int b = 0; b < 2; ++b) {
+            const int q = 2 * static_cast<int>(rank) + b, pc = L ^ q;
+            const uint4 u = ((NEG_MASK >> (4 * q + pc)) & 1u) ? negate_bf16x8(v) : v;
+            const int nl = 32 * b + co;
+            const int k = tap * s.Cin + pc * Qin + 8 * c8;
+            const int kc = k >> 6, uu = (k >> 3) & 7;
+            sts_u4(sbase + static_cast<uint32_t>(kc * CgCfg::BCHUNK + nl * 128 +
+                                                 ((uu ^ (nl & 7)) << 4)),
+                   u);
+        }
     }
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(bready_leader);
 }
 
 // Bounded wait with cluster-scope acquire (arrivals from the peer CTA); otherwise as
@@ -136,6 +174,31 @@ __device__ __forceinline__ bool wait_cluster_or_abort(uint32_t bar, uint32_t par
     }
 }
 
+// One expansion warp: wait for the staged letters, expand this CTA's share, make the stores
+// visible to the tensor cores, then tell the producer (the letters may be overwritten) and
+// the even CTA's issuers (this part of the B half is ready).
+template <bool HALO>
+__device__ __forceinline__ void cg2_expand_warp(const Cg2Params& p, uint32_t sbase,
+                                                uint32_t ring, uint32_t rank, int warp,
+                                                int lane, uint32_t lbar, uint32_t lfree,
+                                                uint32_t bready_bar, uint64_t limit,
+                                                volatile int* abort_flag) {
+    const int et = (warp - CG_EXP_WARP0) * 32 + lane;
+    if (wait_or_abort(lbar, 0, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE)) {
+        if constexpr (HALO)
+            cg2_expand<9>(p, sbase, ring, rank, et, 31 - __clz(p.s.Qin >> 3));
+        else
+            cg2_expand<0>(p, sbase, ring, rank, et, 0);
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+        mbar_arrive(lfree);
+        mbar_arrive_cluster(mapa_shared(bready_bar, 0));
+    }
+}
+
+template <bool HALO>
 __global__ void __launch_bounds__(CG_THREADS, 1)
     qconv_cg2_kernel(const __grid_constant__ CUtensorMap tmap_x, const Cg2Params p) {
     using C = CgCfg;
@@ -154,6 +217,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     const uint32_t acce0 = accf0 + 8u * CG_NACC;
     const uint32_t drain0 = acce0 + 8u * CG_NACC;
     const uint32_t bready_bar = drain0 + 8u * CG_NI;
+    const uint32_t lbar = bready_bar + 8u;  // the four letter copies have landed
+    const uint32_t lfree = lbar + 8u;       // every expansion warp has read the letters
     const uint32_t ring = sbase + static_cast<uint32_t>(C::ring_off(p.kchunks));
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -163,7 +228,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     const int STAGES = CG_NI * p.per;
     const int pair = static_cast<int>(blockIdx.x) >> 1;
     const int npairs = static_cast<int>(gridDim.x) >> 1;
-    // this pair's tiles: pair + k npairs, k < kt; the CTA's pixels (2 t + rank) 128 ..
+    // this pair's tiles: pair + k npairs, k < kt; the CTA's own tile is 2 (that) + rank
     const int kt = pair < p.num_ptiles ? (p.num_ptiles - pair + npairs - 1) / npairs : 0;
 
     griddep_launch_dependents();
@@ -179,6 +244,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
         }
         for (int i = 0; i < CG_NI; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(bready_bar, 2 * CG_EXP_WARPS);  // both CTAs' expansions (even CTA)
+        mbar_init(lbar, 1);
+        mbar_init(lfree, CG_EXP_WARPS);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -193,17 +260,30 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     cluster_sync_all();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    const int hw = s.Ho * s.Wo;
     griddep_wait();  // the previous kernel's output (this layer's input) is complete
+
+    // CTA tile of local pair tile k
+    auto cta_tile = [&](int k) { return 2 * (pair + k * npairs) + static_cast<int>(rank); };
+    // image, first input row and first input column a tile reads (an odd CTA past the last
+    // tile loads the last one and stores nothing)
     auto tile_origin = [&](int k, int& img, int& hbase, int& wbase) {
-        const long long last = (s.M - 1) / BM * BM;  // an odd CTA past the end loads a valid tile
-        long long m0 = (2ll * (pair + static_cast<long long>(k) * npairs) + rank) * BM;
-        if (m0 > last) m0 = last;
-        img = static_cast<int>(m0 / hw);
-        const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
-        const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
-        wbase = wo * s.stride - s.pad;
-        hbase = ho * s.stride - s.pad;
+        if constexpr (HALO) {
+            int t = cta_tile(k);
+            if (t >= p.num_tiles) t = p.num_tiles - 1;
+            img = t / p.tpi;
+            hbase = (t - img * p.tpi) * p.R - s.pad;
+            wbase = -s.pad;
+        } else {
+            const int hw = s.Ho * s.Wo;
+            const long long last = (s.M - 1) / BM * BM;
+            long long m0 = static_cast<long long>(cta_tile(k)) * BM;
+            if (m0 > last) m0 = last;
+            img = static_cast<int>(m0 / hw);
+            const int rem = static_cast<int>(m0 - static_cast<long long>(img) * hw);
+            const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
+            wbase = wo * s.stride - s.pad;
+            hbase = ho * s.stride - s.pad;
+        }
     };
 
     if (warp == 0) {
@@ -211,7 +291,12 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
         if (lane == 0) {
             const uint64_t pol_x = l2_policy_evict_normal();
             uint32_t filled = 0, fill_parity = 0;
-            bool ok = true;
+            // the letters into the ring's space; the pixels once the letters have been read
+            mbar_arrive_expect_tx(lbar, 4u * static_cast<uint32_t>(p.letter_bytes));
+            for (int l = 0; l < 4; ++l)
+                bulk_load(ring + static_cast<uint32_t>(l * p.letter_bytes), p.w[l],
+                          static_cast<uint32_t>(p.letter_bytes), lbar);
+            bool ok = wait_or_abort(lfree, 0, limit, abort_flag, STATUS_TIMEOUT_PRODUCER);
             StageCursor cur(p.per);
             for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
                 const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
@@ -219,9 +304,11 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
 #pragma unroll
                 for (int i = 0; i < CG_NI; ++i)
                     if (i < ng) tile_origin(g0 + i, img[i], hbase[i], wbase[i]);
-                int ch = 0, dh = 0, dw = 0;  // K chunk kc = (tap, ch), walked without divisions
-                for (int kc = 0; ok && kc < p.kchunks; ++kc, cur.next()) {
-                    if (kc > 0 && ++ch == p.cpt) {
+                int ch = 0, dh = 0, dw = 0;  // per tap: stage kc = (tap, ch), no divisions
+                for (int kc = 0; ok && kc < p.nst; ++kc, cur.next()) {
+                    if constexpr (HALO) {
+                        ch = kc;
+                    } else if (kc > 0 && ++ch == p.cpt) {
                         ch = 0;
                         if (++dw == s.kw) {
                             dw = 0;
@@ -239,22 +326,29 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                             break;
                         }
                         const uint32_t fb = full_bar(stage);
-                        mbar_arrive_expect_tx(fb, C::ACHUNK);
+                        const uint32_t dst = ring + static_cast<uint32_t>(stage * p.stage_bytes);
+                        mbar_arrive_expect_tx(fb, static_cast<uint32_t>(p.box_bytes));
                         filled |= 1u << stage;
                         fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
-                        tma_load_im2col_4d(ring + stage * C::ACHUNK, &tmap_x, fb, 64 * ch,
-                                           wbase[i], hbase[i], img[i],
-                                           static_cast<uint16_t>(dw), static_cast<uint16_t>(dh),
-                                           pol_x);
+                        if constexpr (HALO)
+                            tma_load_4d(dst, &tmap_x, fb, 64 * ch, wbase[i], hbase[i], img[i],
+                                        pol_x);
+                        else
+                            tma_load_im2col_4d(dst, &tmap_x, fb, 64 * ch, wbase[i], hbase[i],
+                                               img[i], static_cast<uint16_t>(dw),
+                                               static_cast<uint16_t>(dh), pol_x);
                     }
                 }
             }
-            if (!ok || *abort_flag) drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
+            if (!ok || *abort_flag) {
+                drain_fills(full_bar(0), STAGES, filled, fill_parity, limit);
+                drain_fills(lbar, 1, 1u, 0u, limit);  // the letter copies, if still landing
+            }
         }
     } else if (warp <= CG_NI) {
         if (warp >= CG_EXP_WARP0)
-            cg2_expand(p, smem, rank, (warp - CG_EXP_WARP0) * 32 + lane, lane,
-                       mapa_shared(bready_bar, 0));
+            cg2_expand_warp<HALO>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar,
+                                  limit, abort_flag);
         if (rank == 0 && lane == 0) {
             // -------------------------------------------------- MMA issuers (even CTA)
             constexpr uint32_t IDESC = make_idesc(2 * BM, 128, 0);
@@ -269,6 +363,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             }
             tc_fence_after();
             const uint32_t b_lo0 = desc_lo(sbase);
+            // halo: descriptor offset (16-byte units) of filter row dh = 1
+            const uint32_t row1 = static_cast<uint32_t>(p.Wp * 8);
             StageCursor cur(p.per);
             for (int k = me; ok && k < kt; k += CG_NI) {
                 int buf;
@@ -281,7 +377,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t d = tmem_base + static_cast<uint32_t>(buf * CG_BUF_COLS);
-                for (int kc = 0; kc < p.kchunks; ++kc) {
+                for (int kc = 0; kc < p.nst; ++kc) {
                     const int stage = cur.stage(me);
                     const uint32_t phase = cur.phase;
                     cur.next();
@@ -291,12 +387,32 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a_lo = desc_lo(ring + stage * C::ACHUNK);
-                    const uint32_t b_lo = b_lo0 + static_cast<uint32_t>((kc * C::BCHUNK) >> 4);
+                    const uint32_t a_lo =
+                        desc_lo(ring + static_cast<uint32_t>(stage * p.stage_bytes));
+                    if constexpr (HALO) {
+                        // stage kc holds input channels 64 kc .. 64 kc + 63; tap (dh, dw)
+                        // starts dh Wp + dw rows into the box and uses weight chunk
+                        // tap cpt + kc
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)  // 16-channel steps: 32 bytes into the row
-                        umma_f16_cg2(d, a_lo + 2 * kk, C::DESC_HI, b_lo + 2 * kk, C::DESC_HI,
-                                     IDESC, (kc | kk) != 0 ? 1u : 0u);
+                        for (int t = 0; t < 9; ++t) {
+                            const int dh = t / 3, dw = t % 3;
+                            const uint32_t a_t = a_lo + static_cast<uint32_t>(dh) * row1 +
+                                                 static_cast<uint32_t>(dw * 8);
+                            const uint32_t b_t =
+                                b_lo0 + static_cast<uint32_t>(((t * p.cpt + kc) * C::BCHUNK) >> 4);
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk)  // 16 channels: 32 bytes into a row
+                                umma_f16_cg2(d, a_t + 2 * kk, C::DESC_HI, b_t + 2 * kk,
+                                             C::DESC_HI, IDESC, (kc | t | kk) != 0 ? 1u : 0u);
+                        }
+                    } else {
+                        const uint32_t b_lo =
+                            b_lo0 + static_cast<uint32_t>((kc * C::BCHUNK) >> 4);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk)
+                            umma_f16_cg2(d, a_lo + 2 * kk, C::DESC_HI, b_lo + 2 * kk,
+                                         C::DESC_HI, IDESC, (kc | kk) != 0 ? 1u : 0u);
+                    }
                     ++issued;
                     umma_commit_cg2(empty_bar(stage), 3);  // both CTAs may refill the stage
                 }
@@ -321,7 +437,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             bool ok = true;
             for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
                 const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
-                for (int kc = 0; ok && kc < p.kchunks; ++kc, cur.next()) {
+                for (int kc = 0; ok && kc < p.nst; ++kc, cur.next()) {
                     for (int i = 0; i < ng; ++i) {
                         const int stage = cur.stage(i);
                         if (!wait_or_abort(full_bar(stage), cur.phase, limit, abort_flag,
@@ -335,8 +451,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             }
         }
     } else {
-        cg2_expand(p, smem, rank, (warp - CG_EXP_WARP0) * 32 + lane, lane,
-                   mapa_shared(bready_bar, 0));
+        cg2_expand_warp<HALO>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar, limit,
+                              abort_flag);
         if (warp >= EPI_WARP0) {
             // ------------------------------------------------------------ epilogue
             // (the pair epilogue of tc_common.cuh for 32 channels per component: warps 4..7
@@ -351,6 +467,24 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             const __nv_bfloat16* res = static_cast<const __nv_bfloat16*>(p.ep.residual);
             __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.y);
             const uint32_t acce_leader0 = mapa_shared(acce0, 0);
+            // the thread's MMA rows row0 + kq as output pixels of a tile: offset from the
+            // tile's first pixel, row within the tile, and whether the row is an output
+            int pix[NCH], prow[NCH];
+            bool pval[NCH];
+#pragma unroll
+            for (int kq = 0; kq < NCH; ++kq) {
+                const int m = row0 + kq;
+                if constexpr (HALO) {
+                    const int r = m / p.Wp, c = m - r * p.Wp;
+                    pix[kq] = r * s.Wo + c;
+                    prow[kq] = r;
+                    pval[kq] = c < s.Wo && r < p.R;
+                } else {
+                    pix[kq] = m;
+                    prow[kq] = m;
+                    pval[kq] = true;
+                }
+            }
             auto load_vectors = [&](int cb, float(&sc)[8], float(&sh)[8]) {
                 float bi[8];
                 load8(p.ep.scale, cb, 1.0f, sc);
@@ -370,9 +504,22 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                 ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
                 if (named_bar_or(1, CG_EPI_THREADS, !ok)) break;
                 tc_fence_after();
-                const long long m0 = (2ll * (pair + static_cast<long long>(k) * npairs) + rank) * BM;
-                const long long left = s.M - m0;
-                const int rows = left <= 0 ? 0 : (left < BM ? static_cast<int>(left) : BM);
+                // the tile's first output pixel and how many of its rows exist
+                const int t = cta_tile(k);
+                long long base;
+                int lim;
+                if constexpr (HALO) {
+                    const int img = t / p.tpi, h0 = (t - img * p.tpi) * p.R;
+                    base = (static_cast<long long>(img) * s.Ho + h0) * s.Wo;
+                    lim = t < p.num_tiles ? s.Ho - h0 : 0;
+                } else {
+                    base = static_cast<long long>(t) * BM;
+                    const long long left = s.M - base;
+                    lim = left <= 0 ? 0 : (left < BM ? static_cast<int>(left) : BM);
+                }
+                bool st[NCH];
+#pragma unroll
+                for (int kq = 0; kq < NCH; ++kq) st[kq] = pval[kq] && prow[kq] < lim;
                 const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                        static_cast<uint32_t>(buf * CG_BUF_COLS);
                 uint32_t va[CH], vb[CH];
@@ -400,8 +547,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
 #pragma unroll
                         for (int kq = 0; kq < NCH; ++kq) {
                             r4[kq] = make_uint4(0u, 0u, 0u, 0u);
-                            if (row0 + kq < rows)
-                                r4[kq] = ld_global_na(res + (m0 + row0 + kq) * Cout + cb);
+                            if (st[kq])
+                                r4[kq] = ld_global_na(res + (base + pix[kq]) * Cout + cb);
                         }
                     }
                     float E[NCH][8];
@@ -418,10 +565,10 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                             const __nv_bfloat162* rh =
                                 reinterpret_cast<const __nv_bfloat162*>(&r4[kq]);
 #pragma unroll
-                            for (int t = 0; t < 4; ++t) {
-                                const float2 f = __bfloat1622float2(rh[t]);
-                                rz[2 * t] = f.x;
-                                rz[2 * t + 1] = f.y;
+                            for (int t2 = 0; t2 < 4; ++t2) {
+                                const float2 f = __bfloat1622float2(rh[t2]);
+                                rz[2 * t2] = f.x;
+                                rz[2 * t2 + 1] = f.y;
                             }
                         } else {
 #pragma unroll
@@ -429,14 +576,16 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         }
                         uint32_t wv[4];
 #pragma unroll
-                        for (int t = 0; t < 4; ++t) {
-                            const float z0 = fmaf(sc[2 * t], E[kq][2 * t], sh[2 * t]) + rz[2 * t];
+                        for (int t2 = 0; t2 < 4; ++t2) {
+                            const float z0 =
+                                fmaf(sc[2 * t2], E[kq][2 * t2], sh[2 * t2]) + rz[2 * t2];
                             const float z1 =
-                                fmaf(sc[2 * t + 1], E[kq][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
-                            wv[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                                fmaf(sc[2 * t2 + 1], E[kq][2 * t2 + 1], sh[2 * t2 + 1]) +
+                                rz[2 * t2 + 1];
+                            wv[t2] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
                         }
-                        if (row0 + kq < rows)
-                            st_global_na(out + (m0 + row0 + kq) * Cout + cb,
+                        if (st[kq])
+                            st_global_na(out + (base + pix[kq]) * Cout + cb,
                                          make_uint4(wv[0], wv[1], wv[2], wv[3]));
                     }
                     if (b == 0) tmem_ld_wait();

@@ -502,15 +502,17 @@ bool encode_x_im2col(CUtensorMap* map, const ConvShape& s, const void* x, int ch
     return r == CUDA_SUCCESS;
 }
 
-// Activation tiled map for halo boxes: `channels` x Wo columns x `rows` rows of one image.
+// Activation tiled map for halo boxes: `channels` x `cols` columns (Wo if 0) x `rows` rows
+// of one image.
 bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int channels,
-                   int rows) {
+                   int rows, int cols = 0) {
     const cuuint64_t dims[4] = {static_cast<cuuint64_t>(s.Cin), static_cast<cuuint64_t>(s.W),
                                 static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(s.Cin) * 2,
                                    static_cast<cuuint64_t>(s.Cin) * 2 * s.W,
                                    static_cast<cuuint64_t>(s.Cin) * 2 * s.W * s.H};
-    const cuuint32_t box[4] = {static_cast<cuuint32_t>(channels), static_cast<cuuint32_t>(s.Wo),
+    const cuuint32_t box[4] = {static_cast<cuuint32_t>(channels),
+                               static_cast<cuuint32_t>(cols > 0 ? cols : s.Wo),
                                static_cast<cuuint32_t>(rows), 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     const CUresult r = g_encode_tiled(
@@ -941,32 +943,70 @@ bool encode_rgb_rows(CUtensorMap* map, const ConvShape& s, const float* rgb, int
     return r == CUDA_SUCCESS;
 }
 
+// Sizes of the CTA-pair kernel for shape s (halo or per-tap staging); false if its stage
+// ring or the staged letters do not fit.
+bool cg2_plan(const ConvShape& s, bool halo, Cg2Params* prm) {
+    if (!cg2_ok(s) || (halo && !cg2_halo_ok(s))) return false;
+    prm->cpt = s.Cin / 64;
+    prm->kchunks = s.kh * s.kw * prm->cpt;
+    prm->letter_bytes = 32 * s.kh * s.kw * s.Qin * 2;
+    long long tiles;
+    if (halo) {
+        // R output rows of Wp = Wo + 2 pixels per tile; a stage holds the R + 2 input rows
+        // of the box and every row an MMA of the last tap reads (128 + 2 Wp + 2)
+        prm->Wp = s.Wo + 2;
+        prm->R = BM / prm->Wp;
+        prm->tpi = (s.Ho + prm->R - 1) / prm->R;
+        const int box_rows = prm->R + 2;
+        const int rows = box_rows * prm->Wp > BM + 2 * prm->Wp + 2 ? box_rows * prm->Wp
+                                                                     : BM + 2 * prm->Wp + 2;
+        prm->stage_bytes = (rows * 128 + 1023) / 1024 * 1024;
+        prm->box_bytes = box_rows * prm->Wp * 128;
+        prm->nst = prm->cpt;
+        tiles = static_cast<long long>(s.N) * prm->tpi;
+    } else {
+        prm->stage_bytes = CgCfg::ACHUNK;
+        prm->box_bytes = CgCfg::ACHUNK;
+        prm->nst = prm->kchunks;
+        tiles = (s.M + BM - 1) / BM;
+    }
+    const int ring = CgCfg::ring_bytes(prm->kchunks);
+    prm->per = ring / prm->stage_bytes / CG_NI;
+    if (prm->per > CgCfg::MAX_STAGES / CG_NI) prm->per = CgCfg::MAX_STAGES / CG_NI;
+    if (prm->per < 1 || 4 * prm->letter_bytes > ring || tiles > 0x7ffffffeLL) return false;
+    prm->num_tiles = static_cast<int>(tiles);
+    prm->num_ptiles = static_cast<int>((tiles + 1) / 2);
+    return true;
+}
+
+bool cg2_halo_fits(const ConvShape& s) {
+    Cg2Params prm = {};
+    return cg2_plan(s, true, &prm);
+}
+
 cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4],
                        const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
                        cudaStream_t stream, char* err, size_t errlen) {
-    Cg2Params prm;
+    Cg2Params prm = {};
+    const bool halo = cg2_halo_fits(s);
+    if (!cg2_plan(s, halo, &prm)) {
+        snprintf(err, errlen, "CTA-pair kernel: Cin=%d Cout=%d %dx%d does not fit", s.Cin,
+                 s.Cout, s.kh, s.kw);
+        return cudaErrorInvalidValue;
+    }
     prm.s = s;
     prm.ep = ep;
     for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
     prm.y = out;
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
-    prm.cpt = s.Cin / 64;
-    prm.kchunks = s.kh * s.kw * prm.cpt;
-    prm.per = CgCfg::stages(prm.kchunks) / CG_NI;
-    if (prm.per > CgCfg::MAX_STAGES / CG_NI) prm.per = CgCfg::MAX_STAGES / CG_NI;
-    const long long ptiles = (s.M + 2 * BM - 1) / (2 * BM);
-    if (!cg2_ok(s) || prm.per < 1 || ptiles > 0x7fffffffLL) {
-        snprintf(err, errlen, "CTA-pair kernel: Cin=%d Cout=%d %dx%d does not fit", s.Cin,
-                 s.Cout, s.kh, s.kw);
-        return cudaErrorInvalidValue;
-    }
-    prm.num_ptiles = static_cast<int>(ptiles);
-    const MapKey key = make_key(s, x, w, out, 64, 32, 10);
+    const MapKey key = make_key(s, x, w, out, 64, 32, halo ? 11 : 10);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        if (!encode_x_im2col(&maps[0], s, x, 64)) {
-            snprintf(err, errlen, "cuTensorMapEncodeIm2col failed for the activation tensor");
+        const bool okx = halo ? encode_x_halo(&maps[0], s, x, 64, prm.R + 2, prm.Wp)
+                              : encode_x_im2col(&maps[0], s, x, 64);
+        if (!okx) {
+            snprintf(err, errlen, "tensor map encoding failed for the activation tensor");
             return cudaErrorInvalidValue;
         }
         for (int l = 1; l < 6; ++l) maps[l] = maps[0];
@@ -975,10 +1015,10 @@ cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4]
     int pairs = (opt.max_ctas > 0 ? opt.max_ctas : num_sms) / 2;
     if (pairs > prm.num_ptiles) pairs = prm.num_ptiles;
     if (pairs < 1) pairs = 1;
-    set_kernel_name("qconv_cg2_kernel");
-    auto kern = qconv_cg2_kernel;
-    static std::atomic<unsigned long long> attr_done{0};
-    cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done);
+    set_kernel_name(halo ? "qconv_cg2_kernel<halo>" : "qconv_cg2_kernel");
+    auto kern = halo ? qconv_cg2_kernel<true> : qconv_cg2_kernel<false>;
+    static std::atomic<unsigned long long> attr_done[2];
+    cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done[halo ? 1 : 0]);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * pairs);
@@ -1220,10 +1260,11 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     }
     if (pw_ok(s, ep) && (opt.mode == 0 || opt.mode == 5))
         return launch_pw(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
-    // The CTA-pair kernel only on request: at the backbone's stage-2 shapes its stage ring
-    // (what the kept weight half leaves of shared memory) is too shallow for the pixel
-    // loads' latency, and the pair kernel below is faster.
-    if (!s.sep && cg2_ok(s) && opt.mode == 6)
+    // The CTA-pair kernel: by default for stride-1 3x3 layers with 128 output channels,
+    // whose halo stages feed 36 MMAs each; with per-tap stages (other shapes) only on
+    // request, since four MMAs per stage leave the pixel loads' latency exposed and the
+    // pair kernel below is faster there.
+    if (!s.sep && cg2_ok(s) && (opt.mode == 6 || (opt.mode == 0 && cg2_halo_fits(s))))
         return launch_cg2(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     if (opt.mode == 6) {
         snprintf(err, errlen,

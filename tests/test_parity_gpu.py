@@ -318,24 +318,33 @@ def test_tc_pointwise_mode_rejects_other_shapes():
 
 # ------------------------------------------------------------------ CTA-pair kernel (Cout 128)
 
+HALO, PER_TAP = "qconv_cg2_kernel<halo>", "qconv_cg2_kernel"
 CG2_CASES = [
-    # name, N, H, W, Cin, Cout, k, stride, pad, extra
-    ("cg2_s1_res", 2, 14, 13, 128, 128, 3, 1, 1, {"residual": True}),   # 364 pixels: ragged
-    ("cg2_s2", 3, 15, 17, 64, 128, 3, 2, 1, {}),                         # 216 pixels
-    ("cg2_one_tile", 1, 8, 8, 128, 128, 3, 1, 1,                         # 64 pixels: the odd
-     {"bias": True, "act": quan.QUAN_ACT_SILU}),                         # CTA has none
-    ("cg2_no_iqbn", 2, 12, 12, 64, 128, 3, 1, 1, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),
-    ("cg2_5x1", 2, 11, 9, 128, 128, 5, 1, 2, {"kw": 1}),                  # 5 taps x 128
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra, kernel
+    # halo staging (stride 1, 3x3): 8 rows of 15 per tile, the image's second tile 6 rows
+    ("cg2_s1_res", 2, 14, 13, 128, 128, 3, 1, 1, {"residual": True}, HALO),
+    ("cg2_one_tile", 1, 8, 8, 128, 128, 3, 1, 1,                         # one tile: the odd
+     {"bias": True, "act": quan.QUAN_ACT_SILU}, HALO),                   # CTA has none
+    ("cg2_no_iqbn", 2, 12, 12, 64, 128, 3, 1, 1,                         # one 64-channel chunk
+     {"iqbn": False, "act": quan.QUAN_ACT_NONE}, HALO),
+    ("cg2h_wide", 1, 6, 90, 128, 128, 3, 1, 1, {}, HALO),    # 92-pixel pitch: one row per tile
+    ("cg2h_pad0", 2, 10, 12, 128, 128, 3, 1, 0, {}, HALO),   # box from column 0
+    ("cg2h_pad2", 1, 9, 7, 64, 128, 3, 1, 2, {"residual": True}, HALO),  # box from column -2
+    ("cg2h_deep", 3, 28, 28, 128, 128, 3, 1, 1, {"residual": True}, HALO),  # the stage-2 shape
+    # per-tap staging: stride 2, other filters, rows too wide for two halo stages
+    ("cg2_s2", 3, 15, 17, 64, 128, 3, 2, 1, {}, PER_TAP),                # 216 pixels
+    ("cg2_5x1", 2, 11, 9, 128, 128, 5, 1, 2, {"kw": 1}, PER_TAP),        # 5 taps x 128
+    ("cg2_too_wide", 1, 3, 100, 128, 128, 3, 1, 1, {}, PER_TAP),         # 102-pixel pitch
 ]
 
 
 @pytest.mark.parametrize("case", CG2_CASES, ids=[c[0] for c in CG2_CASES])
 def test_tc_cta_pair_layers(case):
-    name, N, H, W, Cin, Cout, k, s, p, extra = case
+    name, N, H, W, Cin, Cout, k, s, p, extra, kernel = case
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(213, len(name)), **extra)
     quan.quan_set_tc_tiles(0, 0, 0, 6)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
-    assert quan.quan_last_kernel() == "qconv_cg2_kernel"
+    assert quan.quan_last_kernel() == kernel
 
 
 @pytest.mark.parametrize("max_ctas", [4, 6])
@@ -345,20 +354,30 @@ def test_tc_cta_pair_few_pairs(max_ctas):
                               seed=(214, max_ctas))
     quan.quan_set_tc_tiles(0, 0, max_ctas, 6)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
-    assert quan.quan_last_kernel() == "qconv_cg2_kernel"
+    assert quan.quan_last_kernel() == HALO
+
+
+@pytest.mark.parametrize("max_ctas", [4, 6])
+def test_tc_cta_pair_per_tap_few_pairs(max_ctas):
+    # the per-tap staging's ring (12 stages) wraps many times
+    spec = inputs.small_layer("cg2_few_s2", 4, 30, 30, 64, 128, 3, 2, 1, seed=(217, max_ctas))
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 6)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == PER_TAP
 
 
 def test_tc_cta_pair_matches_pair_kernel():
-    # the stage-2 shape of the backbone on the CTA-pair and the pair kernel: both within the
-    # oracle's tolerance and close to each other
+    # the stage-2 shape of the backbone on the CTA-pair kernel (the default choice for it)
+    # and on the pair kernel: both within the oracle's tolerance and close to each other
     spec = inputs.small_layer("cg2_vs_pair", 2, 28, 28, 128, 128, 3, 1, 1, seed=(215, 0))
     d = inputs.layer_inputs(spec)
     ref = oracle_full(d)
     outs = []
-    for mode in (6, 2):
+    for mode, kern in ((0, HALO), (2, "qconv_tc_kernel<pair,kappa=32,bnq=32>")):
         quan.quan_set_tc_tiles(0, 0, 0, mode)
         got, used = run_gpu(d, path=quan.QUAN_PATH_TC)
         assert used == quan.QUAN_PATH_TC
+        assert quan.quan_last_kernel() == kern
         assert_bf16_close(got, ref, "mode %d" % mode)
         outs.append(got)
     assert_bf16_close(outs[0], outs[1], "pair of CTAs vs pair kernel")
@@ -558,16 +577,20 @@ def test_maxpool(shape):
 
 # ------------------------------------------------------------------ failure detection
 
-@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0), (6, 0)])
+@pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0), (6, 0),
+                                          (6, 1)])
 def test_bounded_wait_timeout_every_kernel(mode, issuers):
     # the failure-injection path of the pair-mode, weight-stationary (two and three
-    # issuers), gather, pointwise and CTA-pair kernels
+    # issuers), gather, pointwise and CTA-pair kernels (halo staging, and per-tap staging
+    # for the strided layer marked by issuers = 1, which the CTA-pair kernel ignores)
     if mode == 4:
         spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
     elif mode == 5:
         spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 1, 1, 0, seed=(401, mode))
     elif mode == 6:
-        spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 3, 1, 1, seed=(401, mode))
+        spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 3, 1 + issuers, 1,
+                                  seed=(401, mode))
+        issuers = 0
     else:
         spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
     d = inputs.layer_inputs(spec)
