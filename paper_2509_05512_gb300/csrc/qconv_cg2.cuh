@@ -38,19 +38,22 @@
 // (q = 2 r, 2 r + 1 with p = L xor q), with Eq. 5's sign.
 //
 // Roles.  Both CTAs: warp 0's lane 0 loads the letters, then the CTA's pixel boxes into a
-// stage ring (the stages of local pair tile k belong to issuer k mod 2); warps 2..11 expand
-// the CTA's B half; warps 4..11 are the direct epilogue of the CTA's 128 rows (tc_common.cuh's
-// pair epilogue, with the accumulator released to the even CTA).  Even CTA: warps 1 and 2
-// (lane 0) issue the pair's MMAs for alternate pair tiles, each into its own two of four
-// 128-column accumulators; a stage is handed back to both producers and an accumulator to
+// stage ring; warps 2..11 expand the CTA's B half; warps 4..11 are the direct epilogue of
+// the CTA's 128 rows (tc_common.cuh's pair epilogue, with the per-channel vectors kept in
+// registers, the residual read ahead of the accumulator, and the accumulator released to
+// the even CTA).  Even CTA, per-tap staging: warps 1 and 2 (lane 0) issue the pair's MMAs
+// for alternate pair tiles, each from its own share of the ring into its own two of four
+// 128-column accumulators (a stage's four MMAs leave a single issuer's waits exposed);
+// halo staging: warp 1 alone, through the whole ring (three stages of 36 MMAs) and the four
+// accumulators in order.  A stage is handed back to both producers and an accumulator to
 // both epilogues by multicast commits.  Odd CTA: warp 1's lane 0 relays each of its landed
 // stages to the even CTA's full barrier (a cluster-scope arrive), so the issuer waits on
 // one barrier per stage.  Both CTAs allocate TMEM together (cta_group::2) and free it
 // after a cluster barrier.  Every wait is bounded as in the other kernels.
 
 constexpr int CG_THREADS = 384;
-constexpr int CG_NI = 2;              // MMA issuers of the even CTA
-constexpr int CG_NACC = 2 * CG_NI;    // accumulators of 128 columns
+constexpr int CG_MAX_NI = 2;          // MMA issuers of the even CTA: 1 (halo) or 2 (per tap)
+constexpr int CG_NACC = 4;            // accumulators of 128 columns
 constexpr int CG_BUF_COLS = 128;
 constexpr int CG_MAX_K = 1152;        // taps x Cin of the kept weight half (144 KB)
 constexpr int CG_EXP_WARP0 = 2;       // warps 2..11 expand the B half
@@ -86,7 +89,7 @@ struct CgCfg {
     static constexpr int MAX_STAGES = 12;
     // full, empty (per stage), accf, acce (per accumulator), drain (per issuer), bready,
     // letters landed, letters read
-    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * CG_NACC + CG_NI + 3;
+    static constexpr int NUM_BARS = 2 * MAX_STAGES + 2 * CG_NACC + CG_MAX_NI + 3;
     static constexpr int SMEM_BYTES = 227 * 1024;
     static constexpr uint32_t DESC_HI = desc_hi(8 * 128, desc_layout(128));
     static constexpr uint32_t TMEM_COLS = 512;
@@ -198,7 +201,22 @@ __device__ __forceinline__ void cg2_expand_warp(const Cg2Params& p, uint32_t sba
     }
 }
 
-template <bool HALO>
+// Accumulator buffer and its use count for local pair tile k: with two issuers, issuer
+// k mod 2 alternates between its own two buffers; with one, the four buffers in turn.
+template <int NI>
+__device__ __forceinline__ void cg2_acc(int k, int& buf, uint32_t& use) {
+    if constexpr (NI == 1) {
+        buf = k & 3;
+        use = static_cast<uint32_t>(k >> 2) & 1u;
+    } else {
+        issuer_acc_n<NI>(k, buf, use);
+    }
+}
+
+// NI: MMA issuers (one for halo staging, whose stages carry 36 MMAs each and are consumed
+// in order from one ring of three; two for per-tap staging, whose four-MMA stages would
+// leave a single issuer's waits exposed).
+template <bool HALO, int NI>
 __global__ void __launch_bounds__(CG_THREADS, 1)
     qconv_cg2_kernel(const __grid_constant__ CUtensorMap tmap_x, const Cg2Params p) {
     using C = CgCfg;
@@ -216,7 +234,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     const uint32_t accf0 = bar0 + 8u * (2 * C::MAX_STAGES);
     const uint32_t acce0 = accf0 + 8u * CG_NACC;
     const uint32_t drain0 = acce0 + 8u * CG_NACC;
-    const uint32_t bready_bar = drain0 + 8u * CG_NI;
+    const uint32_t bready_bar = drain0 + 8u * CG_MAX_NI;
     const uint32_t lbar = bready_bar + 8u;  // the four letter copies have landed
     const uint32_t lfree = lbar + 8u;       // every expansion warp has read the letters
     const uint32_t ring = sbase + static_cast<uint32_t>(C::ring_off(p.kchunks));
@@ -225,7 +243,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     const ConvShape& s = p.s;
     const uint64_t limit = p.wait_limit_ns;
     const uint32_t rank = cluster_ctarank();  // 0: the even CTA, which issues the MMAs
-    const int STAGES = CG_NI * p.per;
+    const int STAGES = NI * p.per;
     const int pair = static_cast<int>(blockIdx.x) >> 1;
     const int npairs = static_cast<int>(gridDim.x) >> 1;
     // this pair's tiles: pair + k npairs, k < kt; the CTA's own tile is 2 (that) + rank
@@ -242,7 +260,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             mbar_init(accf0 + 8u * b, 1);                   // multicast commit
             mbar_init(acce0 + 8u * b, 2 * CG_EPI_THREADS);  // both CTAs' epilogues (even CTA)
         }
-        for (int i = 0; i < CG_NI; ++i) mbar_init(drain0 + 8u * i, 1);
+        for (int i = 0; i < NI; ++i) mbar_init(drain0 + 8u * i, 1);
         mbar_init(bready_bar, 2 * CG_EXP_WARPS);  // both CTAs' expansions (even CTA)
         mbar_init(lbar, 1);
         mbar_init(lfree, CG_EXP_WARPS);
@@ -298,11 +316,11 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                           static_cast<uint32_t>(p.letter_bytes), lbar);
             bool ok = wait_or_abort(lfree, 0, limit, abort_flag, STATUS_TIMEOUT_PRODUCER);
             StageCursor cur(p.per);
-            for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
-                const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
-                int img[CG_NI], hbase[CG_NI], wbase[CG_NI];
+            for (int g0 = 0; ok && g0 < kt; g0 += NI) {
+                const int ng = kt - g0 < NI ? kt - g0 : NI;
+                int img[NI], hbase[NI], wbase[NI];
 #pragma unroll
-                for (int i = 0; i < CG_NI; ++i)
+                for (int i = 0; i < NI; ++i)
                     if (i < ng) tile_origin(g0 + i, img[i], hbase[i], wbase[i]);
                 int ch = 0, dh = 0, dw = 0;  // per tap: stage kc = (tap, ch), no divisions
                 for (int kc = 0; ok && kc < p.nst; ++kc, cur.next()) {
@@ -316,7 +334,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         }
                     }
 #pragma unroll
-                    for (int i = 0; i < CG_NI; ++i) {
+                    for (int i = 0; i < NI; ++i) {
                         if (i >= ng) break;
                         const int stage = cur.stage(i);
                         const uint32_t phase = cur.phase;
@@ -345,11 +363,11 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                 drain_fills(lbar, 1, 1u, 0u, limit);  // the letter copies, if still landing
             }
         }
-    } else if (warp <= CG_NI) {
+    } else if (warp <= CG_MAX_NI) {
         if (warp >= CG_EXP_WARP0)
             cg2_expand_warp<HALO>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar,
                                   limit, abort_flag);
-        if (rank == 0 && lane == 0) {
+        if (rank == 0 && lane == 0 && warp <= NI) {
             // -------------------------------------------------- MMA issuers (even CTA)
             constexpr uint32_t IDESC = make_idesc(2 * BM, 128, 0);
             const int me = warp - 1;
@@ -366,10 +384,10 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             // halo: descriptor offset (16-byte units) of filter row dh = 1
             const uint32_t row1 = static_cast<uint32_t>(p.Wp * 8);
             StageCursor cur(p.per);
-            for (int k = me; ok && k < kt; k += CG_NI) {
+            for (int k = me; ok && k < kt; k += NI) {
                 int buf;
                 uint32_t use;
-                issuer_acc_n<CG_NI>(k, buf, use);
+                cg2_acc<NI>(k, buf, use);
                 if (!wait_cluster_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                            STATUS_TIMEOUT_MMA)) {
                     ok = false;
@@ -435,8 +453,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             const uint32_t full_leader0 = mapa_shared(full_bar(0), 0);
             StageCursor cur(p.per);
             bool ok = true;
-            for (int g0 = 0; ok && g0 < kt; g0 += CG_NI) {
-                const int ng = kt - g0 < CG_NI ? kt - g0 : CG_NI;
+            for (int g0 = 0; ok && g0 < kt; g0 += NI) {
+                const int ng = kt - g0 < NI ? kt - g0 : NI;
                 for (int kc = 0; ok && kc < p.nst; ++kc, cur.next()) {
                     for (int i = 0; i < ng; ++i) {
                         const int stage = cur.stage(i);
@@ -485,26 +503,25 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                     pval[kq] = true;
                 }
             }
-            auto load_vectors = [&](int cb, float(&sc)[8], float(&sh)[8]) {
+            // the per-channel vectors of the thread's two channel blocks (components
+            // 2 half + b, channels 8 ci .. 8 ci + 7), for the whole run
+            float sc[2][8], sh[2][8];
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                const int cb = 8 * ci + (2 * half + b) * s.Qout;
                 float bi[8];
-                load8(p.ep.scale, cb, 1.0f, sc);
-                load8(p.ep.shift, cb, 0.0f, sh);
+                load8(p.ep.scale, cb, 1.0f, sc[b]);
+                load8(p.ep.shift, cb, 0.0f, sh[b]);
                 load8(p.ep.bias, cb, 0.0f, bi);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) sh[e] = fmaf(sc[e], bi[e], sh[e]);
-            };
+                for (int e = 0; e < 8; ++e) sh[b][e] = fmaf(sc[b][e], bi[e], sh[b][e]);
+            }
             for (int k = 0; k < kt; ++k) {
                 int buf;
                 uint32_t use;
-                issuer_acc_n<CG_NI>(k, buf, use);
-                bool ok = true;
-                if (lane == 0)
-                    ok = wait_cluster_or_abort(accf0 + 8u * buf, use, limit, abort_flag,
-                                               STATUS_TIMEOUT_EPILOGUE);
-                ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-                if (named_bar_or(1, CG_EPI_THREADS, !ok)) break;
-                tc_fence_after();
-                // the tile's first output pixel and how many of its rows exist
+                cg2_acc<NI>(k, buf, use);
+                // the tile's first output pixel and how many of its rows exist (known before
+                // the accumulator is: the residual of block 0 is read while it is computed)
                 const int t = cta_tile(k);
                 long long base;
                 int lim;
@@ -520,36 +537,40 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                 bool st[NCH];
 #pragma unroll
                 for (int kq = 0; kq < NCH; ++kq) st[kq] = pval[kq] && prow[kq] < lim;
+                uint4 r4[NB][NCH];
+                auto load_res = [&](int b) {
+                    const int cb = 8 * ci + (2 * half + b) * s.Qout;
+#pragma unroll
+                    for (int kq = 0; kq < NCH; ++kq) {
+                        r4[b][kq] = make_uint4(0u, 0u, 0u, 0u);
+                        if (st[kq]) r4[b][kq] = ld_global_na(res + (base + pix[kq]) * Cout + cb);
+                    }
+                };
+                if (res != nullptr) load_res(0);
+                bool ok = true;
+                if (lane == 0)
+                    ok = wait_cluster_or_abort(accf0 + 8u * buf, use, limit, abort_flag,
+                                               STATUS_TIMEOUT_EPILOGUE);
+                ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+                if (named_bar_or(1, CG_EPI_THREADS, !ok)) break;
+                tc_fence_after();
                 const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                        static_cast<uint32_t>(buf * CG_BUF_COLS);
                 uint32_t va[CH], vb[CH];
-                float sca[8], sha[8], scb[8], shb[8];
                 tmem_ld_32x32b_x32(taddr + (2 * half) * BNQ, va);
-                load_vectors(8 * ci + (2 * half) * s.Qout, sca, sha);
                 tmem_ld_wait();
 #pragma unroll
                 for (int b = 0; b < NB; ++b) {
                     uint32_t(&v)[CH] = b ? vb : va;
-                    float(&sc)[8] = b ? scb : sca;
-                    float(&sh)[8] = b ? shb : sha;
                     const int q = 2 * half + b;
                     const int cb = 8 * ci + q * s.Qout;
                     if (b == 0) {
                         tmem_ld_32x32b_x32(taddr + (2 * half + 1) * BNQ, vb);
-                        load_vectors(8 * ci + (2 * half + 1) * s.Qout, scb, shb);
+                        if (res != nullptr) load_res(1);
                     } else {
                         // the tile's accumulator is in registers: hand it back
                         tc_fence_before();
                         mbar_arrive_cluster(acce_leader0 + 8u * buf);
-                    }
-                    uint4 r4[NCH];
-                    if (res != nullptr) {
-#pragma unroll
-                        for (int kq = 0; kq < NCH; ++kq) {
-                            r4[kq] = make_uint4(0u, 0u, 0u, 0u);
-                            if (st[kq])
-                                r4[kq] = ld_global_na(res + (base + pix[kq]) * Cout + cb);
-                        }
                     }
                     float E[NCH][8];
 #pragma unroll
@@ -563,7 +584,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         float rz[8];
                         if (res != nullptr) {
                             const __nv_bfloat162* rh =
-                                reinterpret_cast<const __nv_bfloat162*>(&r4[kq]);
+                                reinterpret_cast<const __nv_bfloat162*>(&r4[b][kq]);
 #pragma unroll
                             for (int t2 = 0; t2 < 4; ++t2) {
                                 const float2 f = __bfloat1622float2(rh[t2]);
@@ -577,10 +598,10 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         uint32_t wv[4];
 #pragma unroll
                         for (int t2 = 0; t2 < 4; ++t2) {
-                            const float z0 =
-                                fmaf(sc[2 * t2], E[kq][2 * t2], sh[2 * t2]) + rz[2 * t2];
+                            const float z0 = fmaf(sc[b][2 * t2], E[kq][2 * t2], sh[b][2 * t2]) +
+                                             rz[2 * t2];
                             const float z1 =
-                                fmaf(sc[2 * t2 + 1], E[kq][2 * t2 + 1], sh[2 * t2 + 1]) +
+                                fmaf(sc[b][2 * t2 + 1], E[kq][2 * t2 + 1], sh[b][2 * t2 + 1]) +
                                 rz[2 * t2 + 1];
                             wv[t2] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
                         }

@@ -971,9 +971,12 @@ bool cg2_plan(const ConvShape& s, bool halo, Cg2Params* prm) {
         tiles = (s.M + BM - 1) / BM;
     }
     const int ring = CgCfg::ring_bytes(prm->kchunks);
-    prm->per = ring / prm->stage_bytes / CG_NI;
-    if (prm->per > CgCfg::MAX_STAGES / CG_NI) prm->per = CgCfg::MAX_STAGES / CG_NI;
-    if (prm->per < 1 || 4 * prm->letter_bytes > ring || tiles > 0x7ffffffeLL) return false;
+    const int ni = halo ? 1 : 2;  // MMA issuers (the kernel's NI)
+    prm->per = ring / prm->stage_bytes / ni;
+    if (prm->per > CgCfg::MAX_STAGES / ni) prm->per = CgCfg::MAX_STAGES / ni;
+    // halo: at least two stages, so one lands while the other's MMAs run
+    if (prm->per < (halo ? 2 : 1) || 4 * prm->letter_bytes > ring || tiles > 0x7ffffffeLL)
+        return false;
     prm->num_tiles = static_cast<int>(tiles);
     prm->num_ptiles = static_cast<int>((tiles + 1) / 2);
     return true;
@@ -1016,7 +1019,7 @@ cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4]
     if (pairs > prm.num_ptiles) pairs = prm.num_ptiles;
     if (pairs < 1) pairs = 1;
     set_kernel_name(halo ? "qconv_cg2_kernel<halo>" : "qconv_cg2_kernel");
-    auto kern = halo ? qconv_cg2_kernel<true> : qconv_cg2_kernel<false>;
+    auto kern = halo ? qconv_cg2_kernel<true, 1> : qconv_cg2_kernel<false, 2>;
     static std::atomic<unsigned long long> attr_done[2];
     cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done[halo ? 1 : 0]);
     if (e != cudaSuccess) return e;
