@@ -369,8 +369,12 @@ const char* quan_last_kernel(void);
  * or 2 (even H and W), Cin a multiple of 64 up to 512, Cout a multiple of 128 and no
  * residual; mode 0 picks it for those; 6: CTA pairs (tcgen05 cta_group::2), M = 256 MMAs
  * over two CTAs' pixels, each CTA keeping half of the signed block weight, only for
- * Cout = 128, Cin a multiple of 64 and kh x kw x Cin <= 1152, and never chosen by mode 0).
- * Values that do not
+ * Cout = 128, Cin a multiple of 64 and kh x kw x Cin <= 1152, and never chosen by mode 0;
+ * 7: vertical taps stacked, for 3x3 stride-1 layers with Cin = Cout = 64 (pad <= 2): one
+ * MMA multiplies a row of input pixels by the block weights of the three vertical taps of
+ * one horizontal tap (N = 192), its three results going to three consecutive output rows
+ * kept side by side in the accumulator; mode 0 picks it for those shapes, mode 3 keeps the
+ * older weight-stationary kernel).  Values that do not
  * divide the layer, or a tile that does not fit in shared memory, make the call fail
  * with QUAN_ERR_UNSUPPORTED.
  */
@@ -393,6 +397,13 @@ quan_status_t quan_set_tc_halo(int enable);
  * the other tile options.
  */
 quan_status_t quan_set_tc_issuers(int issuers);
+
+/*
+ * Output rows per band of the vertical-tap kernel (mode 7): 0 (default) picks the height
+ * with the fewest estimated MMA clocks over the grid's waves; 1 to 4 force it.  Any other
+ * value returns QUAN_ERR_INVALID_ARG.  Results do not depend on it.  Process-wide.
+ */
+quan_status_t quan_set_tc_band_rows(int rows);
 
 /* Time limit of every bounded wait inside the tensor-core kernel, in nanoseconds
  * (default 2e9).  0 restores the default. */

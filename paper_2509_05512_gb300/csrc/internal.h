@@ -42,6 +42,7 @@ struct TcOptions {
     int ws_halo;                  // weight-stationary: stage row blocks with halos (1) when
                                   // the shape allows it, else one im2col box per tap (0)
     int ws_issuers;               // weight-stationary MMA issuers: 0 auto, 2 or 3
+    int vs_rows;                  // vertical-tap kernel: output rows per band, 0 auto, 1..4
     unsigned long long wait_limit_ns;
     int inject_stall;             // failure-injection: the MMA role never consumes
 };

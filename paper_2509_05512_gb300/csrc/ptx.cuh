@@ -67,6 +67,11 @@ __device__ __forceinline__ void tma_prefetch_desc(const void* map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// Bring the line holding `p` into L2 (no register result; the later load hits L2).
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(p)) : "memory");
+}
+
 // 4-D im2col load: coordinates (c, w, h, n) of the first pixel's filter origin and the
 // filter-tap offsets (w, h).  Fills pixelsPerColumn x channelsPerPixel elements.
 __device__ __forceinline__ void tma_load_im2col_4d(uint32_t dst, const void* map, uint32_t bar,

@@ -447,6 +447,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 }
 
 #include "qconv_ws.cuh"
+#include "qconv_vs.cuh"
 #include "qconv_gather.cuh"
 #include "qconv_stempool.cuh"
 #include "qconv_pw.cuh"
@@ -759,6 +760,92 @@ cudaError_t launch_ws(const ConvShape& s, const void* x, const void* const w[4],
     const bool k3x3 = s.kh == 3 && s.kw == 3;
     return s.sep ? launch_ws_form<true>(maps[0], prm, grid, halo, k3x3, ni, stream)
                  : launch_ws_form<false>(maps[0], prm, grid, halo, k3x3, ni, stream);
+}
+
+// Activation map of the vertical-tap kernel: boxes of 64 channels x P columns x 1 row x E
+// images (one input row of E images, lane e P + c at shared-memory row e P + c).
+bool encode_x_vs(CUtensorMap* map, const ConvShape& s, const void* x, int P, int E) {
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(s.Cin), static_cast<cuuint64_t>(s.W),
+                                static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
+    const cuuint64_t strides[3] = {static_cast<cuuint64_t>(s.Cin) * 2,
+                                   static_cast<cuuint64_t>(s.Cin) * 2 * s.W,
+                                   static_cast<cuuint64_t>(s.Cin) * 2 * s.W * s.H};
+    const cuuint32_t box[4] = {static_cast<cuuint32_t>(s.Cin), static_cast<cuuint32_t>(P), 1u,
+                               static_cast<cuuint32_t>(E)};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = g_encode_tiled(
+        map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
+        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int NBOX, bool SEP>
+cudaError_t launch_vs_kernel(const CUtensorMap& map, const VsParams& prm, int grid,
+                             cudaStream_t stream) {
+    auto kern = qconv_vs_kernel<NBOX, SEP>;
+    static std::atomic<unsigned long long> attr_done{0};
+    cudaError_t e = set_smem_once(kern, VsCfg::SMEM_BYTES, attr_done);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(grid), dim3(VS_THREADS), VsCfg::SMEM_BYTES, stream, map, prm);
+}
+
+cudaError_t launch_vs(const ConvShape& s, const void* x, const void* const w[4],
+                      const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
+                      cudaStream_t stream, char* err, size_t errlen) {
+    VsParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    for (int l = 0; l < 4; ++l) prm.w[l] = static_cast<const __nv_bfloat16*>(w[l]);
+    prm.y = out;
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    int nbox = 0;
+    if (!vs_ok(s) || !vs_layout(s.Wo, &nbox, &prm.E, &prm.P)) {
+        snprintf(err, errlen,
+                 "vertical-tap mode needs a 3x3 filter, stride 1, pad <= 2, Cin = Cout = 64 and "
+                 "Wo + 2 <= %d or Wo dividing %d", BM, BM);
+        return cudaErrorInvalidValue;
+    }
+    prm.box_bytes = prm.E * prm.P * 128;
+    prm.row_bytes = (nbox * prm.box_bytes + 1023) & ~1023;
+    prm.stage_bytes = (nbox == 1 ? 3 : 1) * prm.row_bytes;  // input rows per stage: 3 or 1
+    prm.nst = VsCfg::RING_BYTES / prm.stage_bytes;
+    if (prm.nst > VS_MAX_STAGES) prm.nst = VS_MAX_STAGES;
+    if (prm.nst < 2) {
+        snprintf(err, errlen, "vertical-tap stage of %d bytes does not fit", prm.stage_bytes);
+        return cudaErrorInvalidValue;
+    }
+    const long long groups = (s.N + prm.E - 1) / prm.E;
+    const int grid0 = opt.max_ctas > 0 ? opt.max_ctas : num_sms;
+    prm.bh = opt.vs_rows >= 1 && opt.vs_rows <= VS_BH ? opt.vs_rows : vs_pick_bh(s, prm.E, grid0);
+    prm.nbands = (s.Ho + prm.bh - 1) / prm.bh;
+    const long long units = groups * prm.nbands;
+    if (units > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many work units");
+        return cudaErrorInvalidValue;
+    }
+    prm.num_units = static_cast<int>(units);
+
+    const MapKey key = make_key(s, x, w, out, prm.P, prm.E, 12);
+    CUtensorMap maps[6];
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_vs(&maps[0], s, x, prm.P, prm.E)) {
+            snprintf(err, errlen, "tensor-map encode failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 1; l < 6; ++l) maps[l] = maps[0];
+        cache_store(key, maps);
+    }
+    const int grid = grid_for(opt, num_sms, prm.num_units);
+    set_kernel_name(s.sep ? "qconv_vs_kernel<boxes=%d,rows=%d,sep>"
+                          : "qconv_vs_kernel<boxes=%d,rows=%d>",
+                    nbox, prm.bh);
+    if (nbox == 3)
+        return s.sep ? launch_vs_kernel<3, true>(maps[0], prm, grid, stream)
+                     : launch_vs_kernel<3, false>(maps[0], prm, grid, stream);
+    return s.sep ? launch_vs_kernel<1, true>(maps[0], prm, grid, stream)
+                 : launch_vs_kernel<1, false>(maps[0], prm, grid, stream);
 }
 
 cudaError_t launch_gather(const ConvShape& s, const void* x, const void* const w[4],
@@ -1267,6 +1354,15 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     // whose halo stages feed 36 MMAs each; with per-tap stages (other shapes) only on
     // request, since four MMAs per stage leave the pixel loads' latency exposed and the
     // pair kernel below is faster there.
+    // 3x3 stride-1 layers of 16 -> 16 quaternion channels: the vertical taps stacked along N
+    if (s.sep != 2 && vs_ok(s) && (opt.mode == 0 || opt.mode == 7))
+        return launch_vs(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
+    if (opt.mode == 7) {
+        snprintf(err, errlen,
+                 "vertical-tap mode needs a 3x3 filter, stride 1, pad <= 2, Cin = Cout = 64 and "
+                 "Wo + 2 <= %d or Wo dividing %d", BM, BM);
+        return cudaErrorInvalidValue;
+    }
     if (!s.sep && cg2_ok(s) && (opt.mode == 6 || (opt.mode == 0 && cg2_halo_fits(s))))
         return launch_cg2(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     if (opt.mode == 6) {

@@ -18,7 +18,8 @@ thread_local char t_errmsg[512] = "";
 thread_local int t_last_path = 0;
 thread_local const char* t_last_kernel = "";
 std::atomic<int> g_path{QUAN_PATH_AUTO};
-std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1}, g_ws_issuers{0};
+std::atomic<int> g_kappa{0}, g_bnq{0}, g_max_ctas{0}, g_mode{0}, g_ws_halo{1}, g_ws_issuers{0},
+    g_vs_rows{0};
 std::atomic<unsigned long long> g_wait_limit{2000000000ull};
 std::atomic<int> g_inject{0};
 
@@ -182,6 +183,7 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         opt.mode = g_mode.load();
         opt.ws_halo = g_ws_halo.load();
         opt.ws_issuers = g_ws_issuers.load();
+        opt.vs_rows = g_vs_rows.load();
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -269,6 +271,7 @@ quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H,
         opt.mode = separable ? 0 : g_mode.load();
         opt.ws_halo = g_ws_halo.load();
         opt.ws_issuers = g_ws_issuers.load();
+        opt.vs_rows = g_vs_rows.load();
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -613,6 +616,7 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
     opt.mode = 0;
     opt.ws_halo = 1;
     opt.ws_issuers = 0;
+    opt.vs_rows = 0;
     opt.wait_limit_ns = g_wait_limit.load();
     opt.inject_stall = g_inject.load();
     char err[256] = "";
@@ -665,6 +669,7 @@ quan_status_t quan_qconv2d_maxpool_rgb_fwd(const float* rgb, const void* wr, con
     opt.mode = 0;
     opt.ws_halo = 1;
     opt.ws_issuers = 0;
+    opt.vs_rows = 0;
     opt.wait_limit_ns = g_wait_limit.load();
     opt.inject_stall = g_inject.load();
     char err[256] = "";
@@ -713,9 +718,9 @@ const char* quan_last_kernel(void) { return t_last_kernel; }
 
 quan_status_t quan_set_tc_tiles(int kappa, int bnq, int max_ctas, int mode) {
     auto okv = [](int v) { return v == 0 || v == 16 || v == 32 || v == 64; };
-    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 6)
+    if (!okv(kappa) || !okv(bnq) || max_ctas < 0 || mode < 0 || mode > 7)
         return fail(QUAN_ERR_INVALID_ARG,
-                    "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 4");
+                    "kappa and bnq must be 0, 16, 32 or 64; max_ctas >= 0; mode 0 to 7");
     g_kappa.store(kappa);
     g_bnq.store(bnq);
     g_max_ctas.store(max_ctas);
@@ -732,6 +737,13 @@ quan_status_t quan_set_tc_issuers(int issuers) {
     if (issuers != 0 && issuers != 2 && issuers != 3)
         return fail(QUAN_ERR_INVALID_ARG, "issuers must be 0 (automatic), 2 or 3");
     g_ws_issuers.store(issuers);
+    return QUAN_OK;
+}
+
+quan_status_t quan_set_tc_band_rows(int rows) {
+    if (rows < 0 || rows > 4)
+        return fail(QUAN_ERR_INVALID_ARG, "band rows must be 0 (automatic) or 1 to 4");
+    g_vs_rows.store(rows);
     return QUAN_OK;
 }
 

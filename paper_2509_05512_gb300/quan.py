@@ -93,6 +93,7 @@ def load():
         lib.quan_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
         lib.quan_set_tc_halo.argtypes = [_i]
         lib.quan_set_tc_issuers.argtypes = [_i]
+        lib.quan_set_tc_band_rows.argtypes = [_i]
         lib.quan_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_uint)]
         lib.quan_set_fault_injection.argtypes = [_i]
         lib.quan_status_string.argtypes = [_i]
@@ -109,7 +110,7 @@ def load():
                      "quan_qconv2d_sep_bwd_weight",
                      "quan_maxpool2d_fwd", "quan_set_path", "quan_set_tc_tiles",
                      "quan_set_wait_limit_ns", "quan_device_status", "quan_set_fault_injection",
-                     "quan_set_tc_halo", "quan_set_tc_issuers"):
+                     "quan_set_tc_halo", "quan_set_tc_issuers", "quan_set_tc_band_rows"):
             getattr(lib, name).restype = _i
         lib.quan_last_path.restype = _i
         lib.quan_version.restype = _i
@@ -190,6 +191,10 @@ def quan_set_tc_halo(enable: bool) -> None:
 
 def quan_set_tc_issuers(issuers: int = 0) -> None:
     _check(load().quan_set_tc_issuers(issuers))
+
+
+def quan_set_tc_band_rows(rows: int = 0) -> None:
+    _check(load().quan_set_tc_band_rows(rows))
 
 
 def quan_set_wait_limit_ns(ns: int) -> None:

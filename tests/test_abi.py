@@ -59,7 +59,8 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_maxpool2d_fwd(FAKE, 1, 4, 4, 8, 3, 2, 2, FAKE * 64, None) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_path(5) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_tiles(24, 0, 0, 0) == quan.QUAN_ERR_INVALID_ARG
-    assert lib.quan_set_tc_tiles(0, 0, 0, 7) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_tiles(0, 0, 0, 8) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_tiles(0, 0, 0, 7) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 6) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 4) == quan.QUAN_OK
     assert lib.quan_set_tc_tiles(0, 0, 0, 0) == quan.QUAN_OK
@@ -72,6 +73,10 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_set_tc_issuers(4) == quan.QUAN_ERR_INVALID_ARG
     assert lib.quan_set_tc_issuers(2) == quan.QUAN_OK
     assert lib.quan_set_tc_issuers(0) == quan.QUAN_OK
+    assert lib.quan_set_tc_band_rows(-1) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_band_rows(5) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_set_tc_band_rows(3) == quan.QUAN_OK
+    assert lib.quan_set_tc_band_rows(0) == quan.QUAN_OK
     assert lib.quan_set_path(0) == quan.QUAN_OK
     assert lib.quan_set_wait_limit_ns(0) == quan.QUAN_OK
 

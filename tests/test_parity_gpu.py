@@ -40,6 +40,7 @@ def _reset_paths():
     quan.quan_set_wait_limit_ns(0)
     quan.quan_set_tc_halo(True)
     quan.quan_set_tc_issuers(0)
+    quan.quan_set_tc_band_rows(0)
 
 
 def run_gpu(d, path=quan.QUAN_PATH_AUTO, guard=True):
@@ -96,7 +97,7 @@ def test_config1_full(path):
     check(inputs.LAYERS["c1"], path=path, expect_path=path)
 
 
-@pytest.mark.parametrize("mode", [1, 2, 3])
+@pytest.mark.parametrize("mode", [1, 2, 3, 7])
 def test_config1_full_every_mode(mode):
     quan.quan_set_tc_tiles(0, 0, 0, mode)
     check(inputs.LAYERS["c1"], path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
@@ -152,6 +153,59 @@ def test_config1_weight_stationary_staging(halo, issuers):
     quan.quan_set_tc_halo(bool(halo))
     quan.quan_set_tc_issuers(issuers)
     check(inputs.LAYERS["c1"], path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+
+
+# vertical-tap kernel (3x3 stride 1, 16 -> 16 quaternion channels): one box per input row
+# (P = Wo + 2 lanes per image) or three (P = Wo, Wo dividing 128), bands of 1 to 4 output
+# rows, image groups with a ragged last group, padding 0 and 2, the epilogue's options
+VS_CASES = [
+    # name, N, H, W, pad, extra
+    ("vs_56", 3, 56, 56, 1, {"residual": True}),              # 1 box, E = 2, ragged groups
+    ("vs_32", 5, 32, 32, 1, {}),                               # 3 boxes, E = 4
+    ("vs_13x11", 3, 13, 11, 1, {"bias": True, "act": quan.QUAN_ACT_SILU}),  # 1 box, E = 9
+    ("vs_16", 9, 16, 16, 1, {"residual": True}),               # 3 boxes, E = 8
+    ("vs_valid", 2, 18, 18, 0, {"iqbn": False, "act": quan.QUAN_ACT_NONE}),  # Wo = 16
+    ("vs_pad2", 3, 10, 6, 2, {}),                              # Wo = 8: 3 boxes, E = 16
+    ("vs_wide", 2, 5, 126, 1, {}),                             # P = 128, one image
+    ("vs_tiny", 2, 1, 1, 1, {}),                               # Wo = 1: E = 128
+    ("vs_24", 2, 24, 24, 1, {"residual": True}),               # 1 box, E = 4
+]
+
+
+@pytest.mark.parametrize("rows", [0, 1, 2, 3, 4])
+@pytest.mark.parametrize("case", VS_CASES, ids=[c[0] for c in VS_CASES])
+def test_tc_vertical_tap_layers(case, rows):
+    name, N, H, W, p, extra = case
+    spec = inputs.small_layer(name, N, H, W, 64, 64, 3, 1, p, seed=(206, len(name)), **extra)
+    quan.quan_set_tc_band_rows(rows)
+    try:
+        check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    finally:
+        quan.quan_set_tc_band_rows(0)
+    kernel = quan.quan_last_kernel()
+    assert kernel.startswith("qconv_vs_kernel<"), kernel
+    if rows:
+        assert ",rows=%d" % rows in kernel, kernel
+
+
+@pytest.mark.parametrize("rows", [1, 4])
+def test_tc_vertical_tap_few_ctas(rows):
+    # 2 CTAs: the stage ring and both band buffers wrap many times
+    spec = inputs.small_layer("vs_few", 7, 32, 32, 64, 64, 3, 1, 1, residual=True,
+                              seed=(207, rows))
+    quan.quan_set_tc_tiles(0, 0, 2, 7)
+    quan.quan_set_tc_band_rows(rows)
+    try:
+        check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    finally:
+        quan.quan_set_tc_band_rows(0)
+
+
+def test_tc_vertical_tap_mode_rejects_other_shapes():
+    spec = inputs.small_layer("vs_reject", 1, 9, 9, 64, 64, 3, 2, 1, seed=(208, 0))
+    quan.quan_set_tc_tiles(0, 0, 0, 7)
+    with pytest.raises(quan.QuanError):
+        run_gpu(inputs.layer_inputs(spec), quan.QUAN_PATH_TC, guard=False)
 
 
 # ------------------------------------------------------------------ tensor-core small layers
@@ -578,7 +632,7 @@ def test_maxpool(shape):
 # ------------------------------------------------------------------ failure detection
 
 @pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0), (6, 0),
-                                          (6, 1)])
+                                          (6, 1), (7, 0)])
 def test_bounded_wait_timeout_every_kernel(mode, issuers):
     # the failure-injection path of the pair-mode, weight-stationary (two and three
     # issuers), gather, pointwise and CTA-pair kernels (halo staging, and per-tap staging
