@@ -1354,8 +1354,12 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     // whose halo stages feed 36 MMAs each; with per-tap stages (other shapes) only on
     // request, since four MMAs per stage leave the pixel loads' latency exposed and the
     // pair kernel below is faster there.
-    // 3x3 stride-1 layers of 16 -> 16 quaternion channels: the vertical taps stacked along N
-    if (s.sep != 2 && vs_ok(s) && (opt.mode == 0 || opt.mode == 7))
+    // 3x3 stride-1 layers of 16 -> 16 quaternion channels: the vertical taps stacked along N,
+    // by default where one box per input row serves (Wo + 2 lanes per image); with three
+    // boxes per row (Wo dividing 128) the weight-stationary kernel below is faster
+    int vs_nbox = 0, vs_e = 0, vs_p = 0;
+    const bool vs_one_box = vs_ok(s) && vs_layout(s.Wo, &vs_nbox, &vs_e, &vs_p) && vs_nbox == 1;
+    if (s.sep != 2 && vs_ok(s) && (opt.mode == 7 || (opt.mode == 0 && vs_one_box)))
         return launch_vs(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     if (opt.mode == 7) {
         snprintf(err, errlen,

@@ -40,9 +40,10 @@
 // loop body between MMAs costs more than the MMAs); a partial band (the last of an image
 // when bh does not divide Ho, or bh < 4) skips rows outside the image and is issued with
 // run-time row parameters.  Roles (20 warps):
-//   warp 0       TMA producer (three boxes: warps 0, 2, 3, one box each), through a ring of
-//                up to 12 stages of three input rows (one box) or one (three boxes), so the
-//                issuer waits once per 36 or 12 MMAs;
+//   warps 0,2,3  TMA producers (lane 0 of each), through a ring of up to 12 stages of three
+//                input rows (one box: each producer loads one of a stage's rows) or one
+//                (three boxes: each loads one dw box), so the issuer waits once per 36 or
+//                12 MMAs and the loads of a stage are issued by three threads at once;
 //   warp 1       owns TMEM (two band buffers of 256 columns); lane 0 issues the MMAs, unit
 //                after unit, into alternate buffers;
 //   warps 4..19  expand the signed block weight once per CTA (72 KB, tap order (dw, dh)),
@@ -63,6 +64,7 @@ constexpr int VS_MAX_STAGES = 12;
 constexpr int VS_EPI_WARP0 = 4;      // warps 4..19: expansion, then the epilogue
 constexpr int VS_EPI_THREADS = 512;
 constexpr int VS_TAP_BYTES = 64 * 128;  // expanded weight of one tap: 64 rows x 64 channels
+constexpr int VS_PRODUCERS = 3;      // TMA-issuing threads: lane 0 of warps 0, 2, 3
 
 struct VsParams {
     ConvShape s;
@@ -277,7 +279,7 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
     griddep_launch_dependents();
     if (threadIdx.x == 0) {
         for (int i = 0; i < nst; ++i) {
-            mbar_init(full_bar(i), NBOX);
+            mbar_init(full_bar(i), VS_PRODUCERS);
             mbar_init(empty_bar(i), 1);
         }
         for (int b = 0; b < 2; ++b) {
@@ -316,13 +318,15 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
     };
     const int pid = warp == 0 ? 0 : warp - 1;  // producer index (warps 0, 2, 3)
 
-    if ((warp == 0 || (NBOX == 3 && (warp == 2 || warp == 3))) && lane == 0) {
+    if ((warp == 0 || warp == 2 || warp == 3) && lane == 0) {
         // ------------------------------------------------------------ TMA producers
         const uint64_t pol = l2_policy_evict_normal();
         uint32_t filled = 0, fill_parity = 0;
         int idx = 0;
         uint32_t phase = 0;
         bool ok = true;
+        // three boxes: producer pid loads box dw = pid of every row; one box: producer pid loads
+        // row pid of every stage (the TMA unit takes several threads' copies at once)
         const int x0 = (NBOX == 3 ? pid : 0) - s.pad;
         for (int u = blockIdx.x; ok && u < p.num_units; u += gridDim.x) {
             int n0, h0, r;
@@ -340,12 +344,15 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
                     int nr = 1;
                     for (int t2 = t + 1; nr < RPS && t2 <= r + 1; ++t2)
                         if (row_staged(h0, r, t2)) ++nr;
-                    mbar_arrive_expect_tx(full_bar(idx), nr * p.box_bytes);
+                    const int mine = NBOX == 3 ? nr : (pid < nr ? 1 : 0);
+                    mbar_arrive_expect_tx(full_bar(idx), mine * p.box_bytes);
                     filled |= 1u << idx;
                     fill_parity = (fill_parity & ~(1u << idx)) | (phase << idx);
                 }
-                tma_load_4d(sbase + idx * p.stage_bytes + q * p.row_bytes + pid * p.box_bytes,
-                            &tmap_x, full_bar(idx), 0, x0, h0 - s.pad + t, n0, pol);
+                if (NBOX == 3 || q == pid)
+                    tma_load_4d(sbase + idx * p.stage_bytes + q * p.row_bytes +
+                                    (NBOX == 3 ? pid * p.box_bytes : 0),
+                                &tmap_x, full_bar(idx), 0, x0, h0 - s.pad + t, n0, pol);
                 if (++q == RPS) {
                     q = 0;
                     if (++idx == nst) {

@@ -177,6 +177,7 @@ VS_CASES = [
 def test_tc_vertical_tap_layers(case, rows):
     name, N, H, W, p, extra = case
     spec = inputs.small_layer(name, N, H, W, 64, 64, 3, 1, p, seed=(206, len(name)), **extra)
+    quan.quan_set_tc_tiles(0, 0, 0, 7)
     quan.quan_set_tc_band_rows(rows)
     try:
         check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
@@ -199,6 +200,18 @@ def test_tc_vertical_tap_few_ctas(rows):
         check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
     finally:
         quan.quan_set_tc_band_rows(0)
+
+
+@pytest.mark.parametrize("case", [("vs_auto_56", 2, 56, 56, True), ("vs_auto_32", 2, 32, 32, False),
+                                  ("vs_auto_13x11", 2, 13, 11, True)], ids=lambda c: c[0])
+def test_tc_vertical_tap_default_choice(case):
+    # mode 0 takes the vertical-tap kernel where one box per input row serves, the
+    # weight-stationary kernel where the row needs three boxes
+    name, N, H, W, vs = case
+    spec = inputs.small_layer(name, N, H, W, 64, 64, 3, 1, 1, seed=(210, len(name)))
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    kernel = quan.quan_last_kernel()
+    assert kernel.startswith("qconv_vs_kernel<boxes=1" if vs else "qconv_ws_kernel<"), kernel
 
 
 def test_tc_vertical_tap_mode_rejects_other_shapes():

@@ -87,13 +87,12 @@ def test_separable_tc_layers(case):
     spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, s, p, seed=(500, len(name)), **extra)
     check_sep(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
     kernel = quan.quan_last_kernel()
-    if Cin == Cout == 64 and k == 3 and s == 1:
-        # 16 -> 16 quaternion channels, 3x3 stride 1: the vertical-tap kernel with the
-        # separable block weight expanded on chip
-        assert kernel.startswith("qconv_vs_kernel<") and kernel.endswith(",sep>"), kernel
-    elif Cin == Cout == 64 and k * k <= 9:
-        # other 16 -> 16 filters: the weight-stationary kernel, same block weight
-        assert kernel.startswith("qconv_ws_kernel<") and kernel.endswith(",sep>"), kernel
+    if Cin == Cout == 64 and k * k <= 9:
+        # 16 -> 16 quaternion channels: the vertical-tap (3x3 stride 1, one box per input
+        # row) or the weight-stationary kernel, with the separable block weight expanded
+        # on chip
+        assert kernel.startswith(("qconv_vs_kernel<", "qconv_ws_kernel<")), kernel
+        assert kernel.endswith(",sep>"), kernel
     else:
         assert kernel.startswith("qconv_tc_kernel<sep,"), kernel
 
