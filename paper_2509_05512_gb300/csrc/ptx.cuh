@@ -361,6 +361,15 @@ __device__ __forceinline__ void st_global_na(void* p, uint4 v) {
                  : "memory");
 }
 
+// One bf16 store that does not allocate in L1.  Stores that do allocate, issued by epilogue
+// warps while MMAs run, slow the tensor cores' shared-memory operand reads (measured: a
+// stream of 2-byte stores cost the MMAs ~45%, the same stream without L1 allocation ~5%).
+__device__ __forceinline__ void st_global_na_bf16(void* p, __nv_bfloat16 v) {
+    asm volatile("st.global.L1::no_allocate.b16 [%0], %1;" ::"l"(p),
+                 "h"(*reinterpret_cast<const unsigned short*>(&v))
+                 : "memory");
+}
+
 __device__ __forceinline__ uint4 ld_global_na(const void* p) {
     uint4 v;
     asm volatile("ld.global.nc.L1::no_allocate.v4.b32 {%0, %1, %2, %3}, [%4];"

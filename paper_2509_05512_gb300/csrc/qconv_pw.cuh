@@ -298,25 +298,25 @@ __global__ void __launch_bounds__(PW_THREADS, 1)
 #pragma unroll
                     for (int k = 0; k < 32; ++k) {
                         const float z = activate(fmaf(sc, __uint_as_float(v0[k]), sh), ACT);
-                        op[k * Cout] = __float2bfloat16_rn(z);
+                        st_global_na_bf16(op + k * Cout, __float2bfloat16_rn(z));
                     }
 #pragma unroll
                     for (int k = 0; k < 32; ++k) {
                         const float z = activate(fmaf(sc, __uint_as_float(v1[k]), sh), ACT);
-                        op[(32 + k) * Cout] = __float2bfloat16_rn(z);
+                        st_global_na_bf16(op + (32 + k) * Cout, __float2bfloat16_rn(z));
                     }
                 } else {
 #pragma unroll
                     for (int k = 0; k < 32; ++k)
                         if (n0 + k < left) {
                             const float z = activate(fmaf(sc, __uint_as_float(v0[k]), sh), ACT);
-                            op[k * Cout] = __float2bfloat16_rn(z);
+                            st_global_na_bf16(op + k * Cout, __float2bfloat16_rn(z));
                         }
 #pragma unroll
                     for (int k = 0; k < 32; ++k)
                         if (n0 + 32 + k < left) {
                             const float z = activate(fmaf(sc, __uint_as_float(v1[k]), sh), ACT);
-                            op[(32 + k) * Cout] = __float2bfloat16_rn(z);
+                            st_global_na_bf16(op + (32 + k) * Cout, __float2bfloat16_rn(z));
                         }
                 }
             }

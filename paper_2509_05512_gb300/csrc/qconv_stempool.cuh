@@ -239,11 +239,11 @@ __device__ __forceinline__ void sp_chunk(const uint32_t (&acc)[32], float carry,
         if constexpr (RAW) m[u] = activate(fmaf(sc, m[u], sh) + 0.0f, ACT);
     if (j0 + 16 <= Wp) {  // warp-uniform
 #pragma unroll
-        for (int u = 0; u < 8; ++u) op[u * 128] = __float2bfloat16_rn(m[u]);
+        for (int u = 0; u < 8; ++u) st_global_na_bf16(op + u * 128, __float2bfloat16_rn(m[u]));
     } else {
 #pragma unroll
         for (int u = 0; u < 8; ++u)
-            if (j0 + 2 * u + v < Wp) op[u * 128] = __float2bfloat16_rn(m[u]);
+            if (j0 + 2 * u + v < Wp) st_global_na_bf16(op + u * 128, __float2bfloat16_rn(m[u]));
     }
 }
 
