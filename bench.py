@@ -61,6 +61,10 @@ def parse_args():
     ap.add_argument("--rgb", action="store_true",
                     help="backbone: start from fp32 RGB pixels, mapped to quaternions by Eq. 4 "
                          "inside the fused stem kernel's loader")
+    ap.add_argument("--no-overlap", action="store_true",
+                    help="backbone: run every layer on one stream (by default each 1x1/2 "
+                         "shortcut runs on a second stream beside the block's 3x3/2 "
+                         "convolution, forked and joined by events)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -837,7 +841,8 @@ def main():
         from paper_2509_05512_gb300 import backbone
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256,
                                          act=act_code(args.act),
-                                         fuse_stem_pool=not args.no_fuse, rgb=args.rgb)
+                                         fuse_stem_pool=not args.no_fuse, rgb=args.rgb,
+                                         overlap_shortcuts=not args.no_overlap)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
     else:
@@ -967,6 +972,9 @@ def main():
                 else "plain launch loop"})
     if args.workload == "backbone" and not getattr(runner, "fused", False):
         cfg["fusions"] = "none"
+    if args.workload == "backbone":
+        cfg["streams"] = ("the 1x1/2 shortcuts on a second stream beside their block's 3x3/2 "
+                          "convolution" if getattr(runner, "side", None) else "one stream")
     if args.workload not in ("backbone", "poincare", "iqbn") and args.direction == "fwd":
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     if args.direction == "bwd":

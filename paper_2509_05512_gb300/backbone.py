@@ -19,7 +19,7 @@ class BackboneRunner:
 
     def __init__(self, torch, quan, inputs=_inputs, N: int = 256, H: int = 224, seed: int = 4,
                  x_bits=None, act: int = _inputs.ACT_RELU, fuse_stem_pool: bool = False,
-                 rgb: bool = False, rgb_host=None):
+                 rgb: bool = False, rgb_host=None, overlap_shortcuts: bool = False):
         self.torch, self.quan, self.N, self.H = torch, quan, N, H
         dev = torch.device("cuda")
         self.act = act
@@ -77,6 +77,18 @@ class BackboneRunner:
             self.x_host = x_bits
             self.x = up(x_bits)
         self.launches_per_step = len(self.layers)
+        # overlap_shortcuts: a downsampling block's 1x1/2 shortcut (the layer after the
+        # block's 3x3/2 convolution, reading the same input) runs on a second stream, forked
+        # before the 3x3/2 convolution and joined before the block's second convolution,
+        # so its CTAs can take the SMs the convolution's last wave leaves idle
+        self.side = {}
+        if overlap_shortcuts:
+            for i, L in enumerate(self.layers):
+                P = self.layers[i - 1] if i > 0 else None
+                if (L.kind == "conv" and P is not None and P.kind == "conv" and L.src == P.src
+                        and L.spec.kh == 1 and P.spec.kh > 1):
+                    self.side[i] = (torch.cuda.Event(), torch.cuda.Event())
+            self.side_stream = torch.cuda.Stream() if self.side else None
         self.footprint = (sum(t.numel() * 2 for t in self.outs) +
                           self.x.numel() * self.x.element_size())
 
@@ -120,8 +132,30 @@ class BackboneRunner:
         return out
 
     def step(self, stream):
+        if not self.side:
+            for i in range(len(self.layers)):
+                self.run_layer(i, stream)
+            return
+        torch = self.torch
+        main = torch.cuda.ExternalStream(stream)
+        side = self.side_stream
+        pending = None  # the join of a shortcut whose output the next main-stream layer reads
         for i in range(len(self.layers)):
+            if i + 1 in self.side:  # fork just before the block's 3x3/2 convolution
+                self.side[i + 1][0].record(main)
+            if i in self.side:
+                fork, join = self.side[i]
+                side.wait_event(fork)
+                self.run_layer(i, side.cuda_stream)
+                join.record(side)
+                pending = join
+                continue
+            if pending is not None:
+                main.wait_event(pending)
+                pending = None
             self.run_layer(i, stream)
+        if pending is not None:
+            main.wait_event(pending)
 
     @property
     def output(self):

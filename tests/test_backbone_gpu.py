@@ -106,3 +106,30 @@ def test_backbone_full_batch_sampled_images():
     check_layers(runner, [0, 128, 255])
     out = runner.output.float()
     assert torch.isfinite(out).all() and (out >= 0).all()
+
+
+def test_backbone_shortcuts_on_a_second_stream_bit_identical():
+    # the default bench layout: each 1x1/2 shortcut on a second stream (fork before the
+    # block's 3x3/2 convolution, join before the block's second convolution), captured in
+    # a CUDA graph like the bench's timed region; every activation equals the one-stream
+    # run bit for bit
+    x_bits = inputs.backbone_input(n_images=3)
+    ref = BackboneRunner(torch, quan, inputs, N=3, x_bits=x_bits, fuse_stem_pool=True)
+    ovl = BackboneRunner(torch, quan, inputs, N=3, x_bits=x_bits, fuse_stem_pool=True,
+                         overlap_shortcuts=True)
+    assert sorted(ovl.side) == [7, 12, 17]
+    stream = torch.cuda.current_stream().cuda_stream
+    ref.step(stream)
+    cap = torch.cuda.Stream()
+    cap.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=cap):
+        ovl.step(cap.cuda_stream)
+    torch.cuda.synchronize()
+    for rep in range(2):
+        graph.replay()
+        torch.cuda.synchronize()
+        assert quan.quan_device_status()[0] == quan.QUAN_OK
+        for i in range(1, len(ref.layers)):
+            np.testing.assert_array_equal(bits_of(ovl.outs[i]), bits_of(ref.outs[i]),
+                                          err_msg="layer %d, replay %d" % (i, rep))
