@@ -61,6 +61,9 @@ def parse_args():
     ap.add_argument("--rgb", action="store_true",
                     help="backbone: start from fp32 RGB pixels, mapped to quaternions by Eq. 4 "
                          "inside the fused stem kernel's loader")
+    ap.add_argument("--no-split", action="store_true",
+                    help="backbone: run the convolutions without the split-K workspace "
+                         "(quan_qconv2d_fwd / _res instead of quan_qconv2d_fwd_ex)")
     ap.add_argument("--no-overlap", action="store_true",
                     help="backbone: run every layer on one stream (by default each 1x1/2 "
                          "shortcut runs on a second stream beside the block's 3x3/2 "
@@ -842,7 +845,8 @@ def main():
         runner = backbone.BackboneRunner(torch, quan, inputs, N=args.batch or 256,
                                          act=act_code(args.act),
                                          fuse_stem_pool=not args.no_fuse, rgb=args.rgb,
-                                         overlap_shortcuts=not args.no_overlap)
+                                         overlap_shortcuts=not args.no_overlap,
+                                         split_k=not args.no_split)
         runner.sets = 1
         unit, per_step_units, dtype = "images/s", runner.N, "bf16"
     else:
@@ -975,6 +979,7 @@ def main():
     if args.workload == "backbone":
         cfg["streams"] = ("the 1x1/2 shortcuts on a second stream beside their block's 3x3/2 "
                           "convolution" if getattr(runner, "side", None) else "one stream")
+        cfg["split_k"] = getattr(runner, "workspace", None) is not None
     if args.workload not in ("backbone", "poincare", "iqbn") and args.direction == "fwd":
         cfg["path"] = {1: "tc", 2: "simt"}.get(quan.quan_last_path(), "?")
     if args.direction == "bwd":
@@ -1019,11 +1024,11 @@ def backbone_roofline(runner, torch, stream, peaks, peak_src):
     for i, L in enumerate(runner.layers):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         for _ in range(2):
-            runner.run_layer(i, sh)
+            runner.run_layer(i, sh, workspace=getattr(runner, "workspace", None))
         kernels.append(runner.quan.quan_last_kernel() if L.kind == "conv" else "maxpool_kernel")
         e0.record(stream)
         for _ in range(5):
-            runner.run_layer(i, sh)
+            runner.run_layer(i, sh, workspace=getattr(runner, "workspace", None))
         e1.record(stream)
         torch.cuda.synchronize()
         times.append(e0.elapsed_time(e1) / 5 / 1e3)

@@ -113,6 +113,35 @@ quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi
                                    const void* residual, void* out, quan_stream_t stream);
 
 /*
+ * quan_qconv2d_fwd (residual NULL) or quan_qconv2d_fwd_res (residual given) with a caller
+ * workspace that lets the tensor-core kernel split its work evenly over the SMs (Eq. 5/6,
+ * the same convolution and epilogue).  A layer whose output tiles make between one and two
+ * waves of CTAs (the backbone's 7 x 7 layers: 196 tiles on 152 SMs) otherwise leaves most
+ * SMs idle in its second wave; with the workspace each CTA takes an equal contiguous range
+ * of the (tile, K block) iterations, a tile shared by two CTAs being finished by one of
+ * them after adding the other's fp32 partial sums from the workspace.  Other layers run as
+ * without the workspace.
+ * The summation order differs from quan_qconv2d_fwd's, so results agree within rounding,
+ * not bit for bit.
+ *   workspace        device memory of at least quan_qconv2d_fwd_workspace_size() bytes,
+ *                    256-byte aligned, owned by the caller, overlapping no tensor of the
+ *                    call; ZERO-FILLED before its first use: every call leaves it as zero
+ *                    again (after a QUAN_ERR_DEVICE_TIMEOUT, zero it once more).  Calls that
+ *                    may run at the same time on the GPU need separate workspaces.  NULL
+ *                    (with workspace_bytes 0) or a smaller workspace: no split, the call runs
+ *                    as quan_qconv2d_fwd / quan_qconv2d_fwd_res.
+ * Errors as quan_qconv2d_fwd; a NULL workspace with workspace_bytes > 0 or a workspace not
+ * 256-byte aligned is QUAN_ERR_INVALID_ARG.
+ */
+size_t quan_qconv2d_fwd_workspace_size(void);
+quan_status_t quan_qconv2d_fwd_ex(const void* x, const void* wr, const void* wi, const void* wj,
+                                  const void* wk, const float* bias, const float* iqbn_scale,
+                                  const float* iqbn_shift, int N, int H, int W, int Cin,
+                                  int Cout, int kh, int kw, int stride, int pad, int act,
+                                  const void* residual, void* workspace, size_t workspace_bytes,
+                                  void* out, quan_stream_t stream);
+
+/*
  * The separable QUAN convolution of Eq. 7 (Sec. III-B), bf16, same arguments, layouts,
  * epilogue and errors as quan_qconv2d_fwd.  Each output component is a signed sum of the
  * four per-component convolutions c_p = W_p (*) x_p (p = r, i, j, k):

@@ -19,7 +19,8 @@ class BackboneRunner:
 
     def __init__(self, torch, quan, inputs=_inputs, N: int = 256, H: int = 224, seed: int = 4,
                  x_bits=None, act: int = _inputs.ACT_RELU, fuse_stem_pool: bool = False,
-                 rgb: bool = False, rgb_host=None, overlap_shortcuts: bool = False):
+                 rgb: bool = False, rgb_host=None, overlap_shortcuts: bool = False,
+                 split_k: bool = False):
         self.torch, self.quan, self.N, self.H = torch, quan, N, H
         dev = torch.device("cuda")
         self.act = act
@@ -77,6 +78,11 @@ class BackboneRunner:
             self.x_host = x_bits
             self.x = up(x_bits)
         self.launches_per_step = len(self.layers)
+        # split_k: the convolutions run through quan_qconv2d_fwd_ex with one workspace (the
+        # layers run one after another on the main stream; the shortcuts on the side stream
+        # run without one), so layers whose tiles leave a partial last wave of CTAs spread
+        # their work evenly over the SMs
+        self.workspace = quan.fwd_workspace() if split_k else None
         # overlap_shortcuts: a downsampling block's 1x1/2 shortcut (the layer after the
         # block's 3x3/2 convolution, reading the same input) runs on a second stream, forked
         # before the 3x3/2 convolution and joined before the block's second convolution,
@@ -97,7 +103,7 @@ class BackboneRunner:
         src = self.layers[idx].src
         return self.x if src == -1 else self.outs[src]
 
-    def run_layer(self, idx: int, stream, x=None, out=None):
+    def run_layer(self, idx: int, stream, x=None, out=None, workspace=None):
         L = self.layers[idx]
         q = self.quan
         x = self.layer_input(idx) if x is None else x
@@ -122,7 +128,12 @@ class BackboneRunner:
                                        s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
                                        self.outs[0], self.ws_bytes, pooled, stream)
             return pooled
-        if L.res is not None:
+        if workspace is not None:
+            q.quan_qconv2d_fwd_ex(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
+                                  s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
+                                  self.outs[L.res] if L.res is not None else None, workspace,
+                                  workspace.numel(), out, stream)
+        elif L.res is not None:
             q.quan_qconv2d_fwd_res(x, *prm["w"], None, prm["scale"], prm["shift"], N, H, W,
                                    s.Cin, s.Cout, s.kh, s.kw, s.stride, s.pad, s.act,
                                    self.outs[L.res], out, stream)
@@ -132,9 +143,10 @@ class BackboneRunner:
         return out
 
     def step(self, stream):
+        ws = self.workspace
         if not self.side:
             for i in range(len(self.layers)):
-                self.run_layer(i, stream)
+                self.run_layer(i, stream, workspace=ws)
             return
         torch = self.torch
         main = torch.cuda.ExternalStream(stream)
@@ -153,7 +165,7 @@ class BackboneRunner:
             if pending is not None:
                 main.wait_event(pending)
                 pending = None
-            self.run_layer(i, stream)
+            self.run_layer(i, stream, workspace=ws)
         if pending is not None:
             main.wait_event(pending)
 
@@ -203,4 +215,5 @@ class BackboneRunner:
         last = len(self.layers) - 1
         for i in range(len(self.layers)):
             x = self.e_x[b] if self.layers[i].src == -1 else None
-            self.run_layer(i, stream, x=x, out=self.e_out[b] if i == last else None)
+            self.run_layer(i, stream, x=x, out=self.e_out[b] if i == last else None,
+                           workspace=self.workspace)

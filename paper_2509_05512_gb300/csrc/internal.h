@@ -43,6 +43,8 @@ struct TcOptions {
                                   // the shape allows it, else one im2col box per tap (0)
     int ws_issuers;               // weight-stationary MMA issuers: 0 auto, 2 or 3
     int vs_rows;                  // vertical-tap kernel: output rows per band, 0 auto, 1..4
+    void* sk_ws;                  // caller workspace for K ranges split over the CTAs (the
+    size_t sk_ws_bytes;           // quad/pair kernel's partial tiles and flags), or null
     unsigned long long wait_limit_ns;
     int inject_stall;             // failure-injection: the MMA role never consumes
 };
@@ -54,6 +56,9 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                             const EpilogueArgs& ep, void* out, const TcOptions& opt,
                             int num_sms, cudaStream_t stream, char* err, size_t errlen);
 cudaError_t read_and_clear_status(unsigned* status, cudaStream_t stream);
+// Workspace bytes that let a quad/pair-kernel launch on a device of num_sms SMs split its
+// K ranges evenly over its CTAs (one fp32 partial tile and one flag per CTA).
+size_t tc_split_workspace_bytes(int num_sms);
 // Name of the tensor-core kernel the calling thread's last launch_qconv_tc used.
 const char* last_tc_kernel();
 

@@ -53,6 +53,7 @@
 
 #include <atomic>
 #include <cstdio>
+#include <cstring>
 #include <mutex>
 
 #include "internal.h"
@@ -91,6 +92,7 @@ struct TcParams {
     void* y;          // output [M][Cout]
     unsigned long long wait_limit_ns;
     int inject_stall;
+    SplitK sk;        // K ranges split evenly over the CTAs (QUAD/PAIR modes, caller workspace)
 };
 
 template <int KAPPA, int BNQ, int MODE>
@@ -197,7 +199,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t phase = 0;
             uint32_t filled = 0, fill_parity = 0;  // per stage: ever filled, parity of last fill
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
+            UnitIter units(p.sk.on, p.num_tiles, p.ktiles);
+            Unit unit;
+            while (ok && units.next(unit)) {
+                const int tile = unit.tile;
                 const int m_tile = tile / p.num_n_tiles;
                 const int n_tile = tile - m_tile * p.num_n_tiles;
                 const long long m0 = static_cast<long long>(m_tile) * BM;
@@ -206,9 +211,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const int ho = rem / s.Wo, wo = rem - (rem / s.Wo) * s.Wo;
                 const int wbase = wo * s.stride - s.pad, hbase = ho * s.stride - s.pad;
                 // K block kt = (tap, chunk), tap = dh * kw + dw: walked without divisions
-                int chunk = 0, tap = 0, dh = 0, dw = 0;
-                for (int kt = 0; kt < p.ktiles; ++kt) {
-                    if (kt > 0 && ++chunk == p.kchunks) {
+                // from the unit's first block
+                int tap = unit.k0 / p.kchunks;
+                int chunk = unit.k0 - tap * p.kchunks;
+                int dh = tap / s.kw, dw = tap - (tap / s.kw) * s.kw;
+                for (int kt = unit.k0; kt < unit.k1; ++kt) {
+                    if (kt > unit.k0 && ++chunk == p.kchunks) {
                         chunk = 0;
                         ++tap;
                         if (++dw == s.kw) {
@@ -282,9 +290,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 ok = false;
             }
             int local = 0;
-            for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x, ++local) {
+            UnitIter units(p.sk.on, p.num_tiles, p.ktiles);
+            Unit unit;
+            while (ok && units.next(unit)) {
                 const int buf = local & 1;
                 const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+                ++local;
                 if (!wait_or_abort(acce0 + 8u * buf, use ^ 1u, limit, abort_flag,
                                    STATUS_TIMEOUT_MMA)) {
                     ok = false;
@@ -292,7 +303,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t dbase = tmem_base + static_cast<uint32_t>(buf * 4 * BNQ);
-                for (int kt = 0; kt < p.ktiles; ++kt) {
+                for (int kt = unit.k0; kt < unit.k1; ++kt) {
                     // pixels and letter tiles landed (pair mode: with the negated copies)
                     if (!flag_wait_or_abort(ready_word(stage), round + 1u, limit, abort_flag,
                                             STATUS_TIMEOUT_MMA)) {
@@ -304,7 +315,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     // sub-MMA below only adds a compile-time offset to them
                     const uint32_t a_lo0 = desc_lo(sbase + stage * C::STAGE_BYTES);
                     const uint32_t b_lo0 = a_lo0 + (4 * C::A_TILE >> 4);
-                    const uint32_t first = kt != 0 ? 1u : 0u;
+                    const uint32_t first = kt != unit.k0 ? 1u : 0u;
 #pragma unroll
                     for (int pc = 0; pc < 4; ++pc) {
 #pragma unroll
@@ -381,8 +392,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         int stage = 0;
         uint32_t phase = 0, round = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < p.num_tiles; tile += gridDim.x) {
-            for (int kt = 0; kt < p.ktiles; ++kt) {
+        UnitIter units(p.sk.on, p.num_tiles, p.ktiles);
+        Unit unit;
+        while (ok && units.next(unit)) {
+            for (int kt = unit.k0; kt < unit.k1; ++kt) {
                 if (!wait_or_abort(fullw_bar(stage), phase, limit, abort_flag,
                                    STATUS_TIMEOUT_PRODUCER)) {
                     ok = false;
@@ -433,8 +446,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             epilogue_direct_sep<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit,
                                      abort_flag, geo);
         else
-            epilogue_direct_pair<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit,
-                                      abort_flag, geo);
+            epilogue_direct_pair<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles,
+                                      p.ktiles, p.sk, limit, abort_flag, geo);
     }
 
     tc_fence_before();
@@ -1308,6 +1321,13 @@ bool encode_dw_map(CUtensorMap* map, const void* t, int C, int W, int H, int N, 
 
 }  // namespace
 
+size_t tc_split_workspace_bytes(int num_sms) {
+    // a partial tile of the widest tile (bnq = 64: 4 x 64 fp32 columns x 128 rows) and a
+    // flag per CTA of a full-width grid
+    const size_t n = num_sms > 0 ? static_cast<size_t>(num_sms) : 0;
+    return (n * 512 * 64 * sizeof(float) + n * 4 + 255) / 256 * 256;
+}
+
 bool tc_supported(const ConvShape& s, const void* x, const void* const w[4], const void* out,
                   const EpilogueArgs& ep) {
     auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
@@ -1461,11 +1481,38 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
     const int grid = grid_for(opt, num_sms, prm.num_tiles);
+    // K ranges split evenly over the CTAs when the tiles make between one and two waves
+    // (the second one partial: at 196 tiles on 152 CTAs the whole-tile schedule runs two
+    // full tile times where 1.3 would do) and the caller gave a workspace for the partial
+    // tiles (full form only).  With more waves the contiguous ranges cost more, in the L2
+    // reuse between neighbouring tiles the strided schedule keeps, than the last wave's
+    // idle CTAs (measured: the backbone's 14 x 14 layers at 5.2 waves 6% slower, its 7 x 7
+    // layers at 1.3 waves 13% faster)
+    prm.sk.on = 0;
+    prm.sk.partial = nullptr;
+    prm.sk.flags = nullptr;
+    const size_t slot_bytes = static_cast<size_t>(512) * bnq * sizeof(float);
+    const size_t sk_need = static_cast<size_t>(grid) * slot_bytes + static_cast<size_t>(grid) * 4;
+    if (opt.sk_ws != nullptr && opt.sk_ws_bytes >= sk_need &&
+        (mode == MODE_PAIR || mode == MODE_QUAD) && prm.num_tiles > grid &&
+        prm.num_tiles < 2 * grid) {
+        prm.sk.on = 1;
+        prm.sk.partial = static_cast<float*>(opt.sk_ws);
+        prm.sk.flags = reinterpret_cast<unsigned*>(static_cast<char*>(opt.sk_ws) +
+                                                   static_cast<size_t>(grid) * slot_bytes);
+    }
     set_kernel_name(mode == MODE_PAIR   ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d>"
                     : mode == MODE_SEP  ? "qconv_tc_kernel<sep,kappa=%d,bnq=%d>"
                     : mode == MODE_SEPT ? "qconv_tc_kernel<sep_t,kappa=%d,bnq=%d>"
                                         : "qconv_tc_kernel<quad,kappa=%d,bnq=%d>",
                     kappa, bnq);
+    if (prm.sk.on) {  // the name records the split
+        const size_t len = strlen(t_kernel_name);
+        if (len > 0 && len + 10 < sizeof(t_kernel_name)) {
+            t_kernel_name[len - 1] = '\0';
+            strcat(t_kernel_name, ",splitk>");
+        }
+    }
 
 #define QUAN_TC_CASE(K, B)                                                       \
     if (kappa == K && bnq == B)                                                  \

@@ -147,7 +147,7 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
                        const void* wk, const float* bias, const float* scale, const float* shift,
                        int N, int H, int W, int Cin, int Cout, int kh, int kw, int stride, int pad,
                        int act, const void* residual, void* out, quan_stream_t stream,
-                       bool separable = false) {
+                       bool separable = false, void* sk_ws = nullptr, size_t sk_ws_bytes = 0) {
     const void* w[4] = {wr, wi, wj, wk};
     quan::ConvShape s;
     quan_status_t st = validate(&s, x, w, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
@@ -184,6 +184,8 @@ quan_status_t run_bf16(const void* x, const void* wr, const void* wi, const void
         opt.ws_halo = g_ws_halo.load();
         opt.ws_issuers = g_ws_issuers.load();
         opt.vs_rows = g_vs_rows.load();
+        opt.sk_ws = sk_ws;
+        opt.sk_ws_bytes = sk_ws_bytes;
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -272,6 +274,8 @@ quan_status_t run_bwd_data(const void* dy, const void* const w[4], int N, int H,
         opt.ws_halo = g_ws_halo.load();
         opt.ws_issuers = g_ws_issuers.load();
         opt.vs_rows = g_vs_rows.load();
+        opt.sk_ws = nullptr;
+        opt.sk_ws_bytes = 0;
         opt.wait_limit_ns = g_wait_limit.load();
         opt.inject_stall = g_inject.load();
         char err[256] = "";
@@ -350,6 +354,27 @@ quan_status_t quan_qconv2d_fwd(const void* x, const void* wr, const void* wi, co
                                quan_stream_t stream) {
     return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
                     stride, pad, act, nullptr, out, stream);
+}
+
+size_t quan_qconv2d_fwd_workspace_size(void) {
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return 0;
+    return quan::tc_split_workspace_bytes(num_sms);
+}
+
+quan_status_t quan_qconv2d_fwd_ex(const void* x, const void* wr, const void* wi, const void* wj,
+                                  const void* wk, const float* bias, const float* iqbn_scale,
+                                  const float* iqbn_shift, int N, int H, int W, int Cin,
+                                  int Cout, int kh, int kw, int stride, int pad, int act,
+                                  const void* residual, void* workspace, size_t workspace_bytes,
+                                  void* out, quan_stream_t stream) {
+    if (workspace_bytes > 0 && workspace == nullptr)
+        return fail(QUAN_ERR_INVALID_ARG, "workspace is NULL with workspace_bytes > 0");
+    if (workspace != nullptr && (reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+        return fail(QUAN_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                    stride, pad, act, residual, out, stream, false, workspace, workspace_bytes);
 }
 
 quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi, const void* wj,
@@ -617,6 +642,8 @@ quan_status_t quan_qconv2d_maxpool_fwd(const void* x, const void* wr, const void
     opt.ws_halo = 1;
     opt.ws_issuers = 0;
     opt.vs_rows = 0;
+    opt.sk_ws = nullptr;
+    opt.sk_ws_bytes = 0;
     opt.wait_limit_ns = g_wait_limit.load();
     opt.inject_stall = g_inject.load();
     char err[256] = "";
@@ -670,6 +697,8 @@ quan_status_t quan_qconv2d_maxpool_rgb_fwd(const float* rgb, const void* wr, con
     opt.ws_halo = 1;
     opt.ws_issuers = 0;
     opt.vs_rows = 0;
+    opt.sk_ws = nullptr;
+    opt.sk_ws_bytes = 0;
     opt.wait_limit_ns = g_wait_limit.load();
     opt.inject_stall = g_inject.load();
     char err[256] = "";

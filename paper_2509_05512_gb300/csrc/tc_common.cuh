@@ -275,6 +275,83 @@ __device__ __forceinline__ void load8(const float* p, int c, float fill, float (
     v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 
+// Work units of a persistent CTA of the QUAD/PAIR kernel.  Without a split (sk = 0) a unit
+// is a whole tile, the CTA taking tiles blockIdx.x + k gridDim.x.  With a split, the
+// num_tiles x ktiles (tile, K block) iterations are cut into gridDim.x equal contiguous
+// ranges, one per CTA (used only when num_tiles >= gridDim.x, so a range spans at least one
+// tile and a tile is shared by at most two CTAs), so that every CTA does the same work
+// whatever the tile count (the whole-tile schedule leaves most CTAs idle in a partial last
+// wave).  A range then starts with the tail part of a tile (a HEAD unit: its accumulator
+// goes to the CTA's partial slot in the caller's workspace and is flagged ready), runs
+// whole tiles, and ends with the first part of a tile (a TAIL unit: the epilogue waits for
+// the next CTA's flag, adds that CTA's partial and finishes the tile).  The head comes
+// first in its CTA's run and the tail last in the other's, so the wait is normally over
+// before it starts.
+struct SplitK {
+    int on;
+    float* partial;      // workspace: one slot of 512 BNQ floats per CTA
+    unsigned* flags;     // one flag per CTA: 1 while its partial is ready; the reader clears it
+};
+enum : int { UNIT_WHOLE = 0, UNIT_HEAD = 1, UNIT_TAIL = 2 };
+struct Unit {
+    int tile, k0, k1, kind;
+};
+struct UnitIter {
+    int on, ktiles, num_tiles, tile;
+    long long cur, hi;
+    __device__ __forceinline__ UnitIter(int on_, int num_tiles_, int ktiles_)
+        : on(on_), ktiles(ktiles_), num_tiles(num_tiles_), tile(static_cast<int>(blockIdx.x)) {
+        const long long total = static_cast<long long>(num_tiles_) * ktiles_;
+        cur = total * blockIdx.x / gridDim.x;
+        hi = total * (blockIdx.x + 1) / gridDim.x;
+    }
+    __device__ __forceinline__ bool next(Unit& u) {
+        if (!on) {
+            if (tile >= num_tiles) return false;
+            u.tile = tile;
+            u.k0 = 0;
+            u.k1 = ktiles;
+            u.kind = UNIT_WHOLE;
+            tile += static_cast<int>(gridDim.x);
+            return true;
+        }
+        if (cur >= hi) return false;
+        u.tile = static_cast<int>(cur / ktiles);
+        u.k0 = static_cast<int>(cur - static_cast<long long>(u.tile) * ktiles);
+        const long long left = hi - cur;
+        u.k1 = left < ktiles - u.k0 ? u.k0 + static_cast<int>(left) : ktiles;
+        u.kind = u.k0 > 0 ? UNIT_HEAD : (u.k1 < ktiles ? UNIT_TAIL : UNIT_WHOLE);
+        cur += u.k1 - u.k0;
+        return true;
+    }
+};
+
+// Global-memory flag handshake between the CTAs sharing a tile (all CTAs of the grid are
+// resident: one per SM), every wait bounded like the mbarrier waits.
+__device__ __forceinline__ void st_release_gpu(unsigned* p, unsigned v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ bool gflag_wait_or_abort(const unsigned* flag, uint64_t limit,
+                                                    volatile int* abort_flag, unsigned code) {
+    if (ld_acquire_gpu(flag) != 0u) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (true) {
+        __nanosleep(256);
+        if (ld_acquire_gpu(flag) != 0u) return true;
+        if (*abort_flag) return false;
+        if (global_timer_ns() - t0 > limit) {
+            atomicOr(&g_status, code);
+            *abort_flag = 1;
+            return false;
+        }
+    }
+}
+
 // Direct epilogue of the QUAD/PAIR kernel (warps 4..11, two per TMEM lane quadrant;
 // warps 4..7 take output components r and i of every tile, warps 8..11 components j and k).
 // Accumulator buffer b (of two, used round robin over the CTA's tiles) lives at TMEM
@@ -298,7 +375,8 @@ template <int BNQ, typename Geo>
 __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const EpilogueArgs& ep,
                                                      void* y, uint32_t tmem_base,
                                                      uint32_t accf0, uint32_t acce0,
-                                                     int num_tiles, uint64_t limit,
+                                                     int num_tiles, int ktiles, const SplitK& sk,
+                                                     uint64_t limit,
                                                      volatile int* abort_flag, Geo geo) {
     constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
     constexpr int NCH = CH / 8;              // 8-channel chunks per load: 2 or 4
@@ -329,16 +407,37 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
 #pragma unroll
         for (int e = 0; e < 8; ++e) sh[e] = fmaf(sc[e], bi[e], sh[e]);
     };
+    // this thread's floats in a partial slot: block b, 4-float group j -> lanes contiguous
+    const int ew = warp - EPI_WARP0;  // 0..7
+    auto pslot = [&](const float* slot, int b, int j) {
+        return reinterpret_cast<float4*>(const_cast<float*>(slot)) +
+               ((ew * NB + b) * (CH / 4) + j) * 32 + lane;
+    };
     int local = 0;
-    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+    UnitIter units(sk.on, num_tiles, ktiles);
+    Unit unit;
+    while (units.next(unit)) {
+        const int tile = unit.tile;
         const int buf = local & 1;
         const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        ++local;
         bool ok = true;
         if (lane == 0)
             ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         // leave together: a warp that gave up must not strand the others at a barrier
         if (named_bar_or(1, 256, !ok)) break;
+        if (unit.kind == UNIT_TAIL) {
+            // the rest of this tile's K blocks were done by the next CTA: wait for its partial
+            bool ready = true;
+            if (threadIdx.x == EPI_WARP0 * 32) {
+                ready = gflag_wait_or_abort(sk.flags + blockIdx.x + 1, limit, abort_flag,
+                                            STATUS_TIMEOUT_EPILOGUE);
+                // cleared for the next call (whose writer runs only after this grid ends)
+                if (ready) sk.flags[blockIdx.x + 1] = 0u;
+            }
+            if (named_bar_or(1, 256, !ready)) break;
+        }
         tc_fence_after();
         const EpiTile g = geo(tile);
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
@@ -369,6 +468,30 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
                 // the tile's accumulator is in registers: hand the buffer back
                 tc_fence_before();
                 mbar_arrive(acce0 + 8u * buf);
+            }
+            if (unit.kind == UNIT_HEAD) {
+                // this CTA's share of the tile: the raw accumulator to the partial slot (L2)
+                float* my_slot = sk.partial + static_cast<size_t>(blockIdx.x) * (512 * BNQ);
+#pragma unroll
+                for (int j = 0; j < CH / 4; ++j)
+                    __stcg(pslot(my_slot, b, j),
+                           make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                       __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3])));
+                if (b + 1 < NB) tmem_ld_wait();
+                continue;
+            }
+            if (unit.kind == UNIT_TAIL) {
+                // the next CTA's share, read from L2 (never from this SM's L1)
+                const float* next_slot =
+                    sk.partial + static_cast<size_t>(blockIdx.x + 1) * (512 * BNQ);
+#pragma unroll
+                for (int j = 0; j < CH / 4; ++j) {
+                    const float4 q4 = __ldcg(pslot(next_slot, b, j));
+                    v[4 * j] = __float_as_uint(__uint_as_float(v[4 * j]) + q4.x);
+                    v[4 * j + 1] = __float_as_uint(__uint_as_float(v[4 * j + 1]) + q4.y);
+                    v[4 * j + 2] = __float_as_uint(__uint_as_float(v[4 * j + 2]) + q4.z);
+                    v[4 * j + 3] = __float_as_uint(__uint_as_float(v[4 * j + 3]) + q4.w);
+                }
             }
             uint4 r4[NCH];
             if (res != nullptr) {
@@ -419,6 +542,12 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
                                  make_uint4(w[0], w[1], w[2], w[3]));
             }
             if (b + 1 < NB) tmem_ld_wait();
+        }
+        if (unit.kind == UNIT_HEAD) {
+            // every epilogue thread's partial stores are visible device-wide before the flag
+            __threadfence();
+            named_bar_sync(2, 256);
+            if (threadIdx.x == EPI_WARP0 * 32) st_release_gpu(sk.flags + blockIdx.x, 1u);
         }
     }
 }

@@ -61,6 +61,9 @@ def load():
         lib.quan_qconv2d_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_qconv2d_fwd_f32.argtypes = _conv_args + [_vp, _vp]
         lib.quan_qconv2d_fwd_res.argtypes = _conv_args + [_vp, _vp, _vp]
+        lib.quan_qconv2d_fwd_ex.argtypes = _conv_args + [_vp, _vp, ctypes.c_size_t, _vp, _vp]
+        lib.quan_qconv2d_fwd_workspace_size.argtypes = []
+        lib.quan_qconv2d_fwd_workspace_size.restype = ctypes.c_size_t
         lib.quan_qconv2d_sep_fwd.argtypes = _conv_args + [_vp, _vp]
         lib.quan_maxpool2d_fwd.argtypes = [_vp] + [_i] * 7 + [_vp, _vp]
         lib.quan_poincare_fwd.argtypes = [_vp, ctypes.c_longlong, _vp, _vp]
@@ -102,6 +105,7 @@ def load():
         lib.quan_last_error_message.restype = ctypes.c_char_p
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
+                     "quan_qconv2d_fwd_ex",
                      "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
                      "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
                      "quan_qconv2d_bwd_data_static", "quan_iqbn_batch_stats",
@@ -162,6 +166,27 @@ def quan_qconv2d_fwd_res(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, 
                                        _ptr(bias), _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W,
                                        Cin, Cout, kh, kw, stride, pad, act, _ptr(residual),
                                        _ptr(out), _stream(stream)))
+
+
+def quan_qconv2d_fwd_ex(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                        kw, stride, pad, act, residual, workspace, workspace_bytes, out,
+                        stream=None) -> None:
+    _check(load().quan_qconv2d_fwd_ex(_ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk),
+                                      _ptr(bias), _ptr(iqbn_scale), _ptr(iqbn_shift), N, H, W,
+                                      Cin, Cout, kh, kw, stride, pad, act, _ptr(residual),
+                                      _ptr(workspace), workspace_bytes, _ptr(out),
+                                      _stream(stream)))
+
+
+def quan_qconv2d_fwd_workspace_size() -> int:
+    return int(load().quan_qconv2d_fwd_workspace_size())
+
+
+def fwd_workspace(device=None):
+    """A zero-filled workspace (uint8 CUDA tensor) for quan_qconv2d_fwd_ex."""
+    import torch
+    return torch.zeros(quan_qconv2d_fwd_workspace_size(), dtype=torch.uint8,
+                       device=device or "cuda")
 
 
 def quan_maxpool2d_fwd(x, N, H, W, C, k, stride, pad, out, stream=None) -> None:
@@ -237,10 +262,13 @@ def out_size(n: int, k: int, stride: int, pad: int) -> int:
 
 
 def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=None,
-            act=QUAN_ACT_NONE, residual=None, out=None, stream=None, separable=False):
+            act=QUAN_ACT_NONE, residual=None, out=None, stream=None, separable=False,
+            workspace=None):
     """Allocate the output (torch, same dtype/device as x) and run the convolution.
     x: [N, H, W, Cin] (bf16 or fp32, CUDA); w*: [Cout/4, kh, kw, Cin/4].  separable=True
-    runs the separable form of Eq. 7 (bf16 only, no residual)."""
+    runs the separable form of Eq. 7 (bf16 only, no residual).  workspace (a zero-filled
+    uint8 CUDA tensor, see fwd_workspace) runs the bf16 full form through
+    quan_qconv2d_fwd_ex."""
     import torch
     N, H, W, Cin = x.shape
     Qout, kh, kw, _ = wr.shape
@@ -258,6 +286,10 @@ def qconv2d(x, wr, wi, wj, wk, *, stride=1, pad=0, bias=None, scale=None, shift=
             raise ValueError("the fp32 entry point has no residual input")
         quan_qconv2d_fwd_f32(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
                              stride, pad, act, out, stream)
+    elif workspace is not None:
+        quan_qconv2d_fwd_ex(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
+                            stride, pad, act, residual, workspace,
+                            workspace.numel() * workspace.element_size(), out, stream)
     elif residual is not None:
         quan_qconv2d_fwd_res(x, wr, wi, wj, wk, bias, scale, shift, N, H, W, Cin, Cout, kh, kw,
                              stride, pad, act, residual, out, stream)

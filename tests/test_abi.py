@@ -79,6 +79,12 @@ def test_maxpool_and_setters_validate(lib):
     assert lib.quan_set_tc_band_rows(0) == quan.QUAN_OK
     assert lib.quan_set_path(0) == quan.QUAN_OK
     assert lib.quan_set_wait_limit_ns(0) == quan.QUAN_OK
+    # quan_qconv2d_fwd_ex: the workspace arguments are checked before anything else
+    conv = [FAKE] * 8 + [1, 8, 8, 64, 64, 3, 3, 1, 1, 1]
+    assert lib.quan_qconv2d_fwd_ex(*conv, None, None, 64, FAKE * 64, None) == \
+        quan.QUAN_ERR_INVALID_ARG  # workspace NULL with bytes > 0
+    assert lib.quan_qconv2d_fwd_ex(*conv, None, FAKE + 16, 4096, FAKE * 64, None) == \
+        quan.QUAN_ERR_INVALID_ARG  # not 256-byte aligned
 
 
 def test_f32_entry_point_validates(lib):

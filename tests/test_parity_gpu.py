@@ -221,6 +221,79 @@ def test_tc_vertical_tap_mode_rejects_other_shapes():
         run_gpu(inputs.layer_inputs(spec), quan.QUAN_PATH_TC, guard=False)
 
 
+# split K (quan_qconv2d_fwd_ex): the (tile, K block) iterations cut evenly over a grid that
+# the tile count does not divide, tiles shared by two CTAs finished through the workspace
+SPLITK_CASES = [
+    # name, N, H, W, Cin, Cout, k, stride, pad, extra, grid, (kappa, bnq, mode)
+    ("sk_pair_res", 4, 12, 12, 128, 256, 3, 1, 1, {"residual": True}, 3, (0, 0, 0)),  # 5 tiles
+    ("sk_quad", 4, 12, 12, 128, 256, 3, 1, 1, {}, 4, (0, 0, 1)),
+    ("sk_two_ntiles", 3, 11, 13, 128, 256, 3, 1, 1, {"bias": True, "act": quan.QUAN_ACT_SILU},
+     5, (32, 32, 2)),                                        # 8 tiles (2 channel blocks)
+    ("sk_kappa16", 4, 10, 12, 64, 128, 3, 1, 1, {}, 3, (16, 32, 2)),  # 4 tiles
+    ("sk_stride2", 5, 15, 17, 128, 256, 3, 2, 1, {}, 2, (0, 0, 0)),   # 3 tiles
+    ("sk_5x5", 2, 11, 12, 64, 256, 5, 1, 2, {"residual": True}, 2, (0, 0, 0)),  # 3 tiles
+]
+
+
+def run_split(d, ws, grid, tiles):
+    kappa, bnq, mode = tiles
+    quan.quan_set_tc_tiles(kappa, bnq, grid, mode)
+    spec = d["spec"]
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    bias, scale, shift = (to_dev_f32(d[k]) for k in ("bias", "scale", "shift"))
+    res = to_dev(d["residual"], "bf16") if d["residual"] is not None else None
+    quan.quan_set_path(quan.QUAN_PATH_TC)
+    y = quan.qconv2d(x, *w, stride=spec.stride, pad=spec.pad, bias=bias, scale=scale,
+                     shift=shift, act=spec.act, residual=res, workspace=ws)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    return y, quan.quan_last_kernel()
+
+
+@pytest.mark.parametrize("case", SPLITK_CASES, ids=[c[0] for c in SPLITK_CASES])
+def test_tc_split_k_layers(case):
+    name, N, H, W, Cin, Cout, k, st, p, extra, grid, tiles = case
+    spec = inputs.small_layer(name, N, H, W, Cin, Cout, k, st, p, seed=(211, len(name)), **extra)
+    d = inputs.layer_inputs(spec)
+    ws = quan.fwd_workspace()
+    y1, kernel = run_split(d, ws, grid, tiles)
+    assert kernel.endswith(",splitk>"), kernel
+    ref = oracle_full(d)
+    assert_bf16_close(out_f64(y1), ref, name)
+    # a second call on the same workspace: the same result (the split is deterministic), and
+    # every flag is clear again afterwards
+    y2, _ = run_split(d, ws, grid, tiles)
+    assert torch.equal(y1, y2)
+    flags = ws.view(torch.uint8)[grid * 512 * (tiles[1] or 64) * 4:]
+    assert int(flags[:grid * 4].count_nonzero()) == 0
+    # no workspace: the unsplit kernel, within rounding of the split one
+    y0, kernel0 = run_split(d, None, grid, tiles)
+    assert not kernel0.endswith(",splitk>")
+    assert_bf16_close(out_f64(y0), ref, name + "-unsplit")
+
+
+def test_tc_split_k_full_size_stage4():
+    # the backbone's 7x7 512 -> 512 residual layer on the full grid (196 tiles on the SMs)
+    spec = inputs.small_layer("sk_stage4", 256, 7, 7, 512, 512, 3, 1, 1, residual=True,
+                              seed=(212, 0))
+    d = inputs.layer_inputs(spec)
+    ws = quan.fwd_workspace()
+    y1, kernel = run_split(d, ws, 0, (0, 0, 0))
+    assert kernel.endswith(",splitk>"), kernel
+    y0, kernel0 = run_split(d, None, 0, (0, 0, 0))
+    a, b = out_f64(y1), out_f64(y0)
+    rel = float(np.linalg.norm(a - b) / np.linalg.norm(b))
+    assert rel < 2e-3, rel
+    # images 0, N/2, N-1 against the oracle
+    for n in (0, 128, 255):
+        dn = dict(d)
+        dn["x"] = d["x"][n:n + 1]
+        dn["residual"] = d["residual"][n:n + 1]
+        dn["spec"] = dataclasses.replace(spec, N=1)
+        assert_bf16_close(a[n:n + 1], oracle_full(dn), "sk_stage4 image %d" % n)
+
+
 # ------------------------------------------------------------------ tensor-core small layers
 
 SMALL_TC = [
