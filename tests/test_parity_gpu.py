@@ -753,6 +753,32 @@ def test_bounded_wait_timeout_every_kernel(mode, issuers):
     assert_bf16_close(out_f64(y), oracle_full(d2), "after-timeout-%d" % mode)
 
 
+def test_bounded_wait_timeout_split_k():
+    # failure injection on a split launch: the waits end with a timeout status, the
+    # context stays usable, and after zeroing the workspace again the split call is right
+    spec = inputs.small_layer("inject_sk", 4, 12, 12, 128, 256, 3, 1, 1, seed=(402, 0))
+    d = inputs.layer_inputs(spec)
+    x = to_dev(d["x"], "bf16")
+    w = [to_dev(d[k], "bf16") for k in ("wr", "wi", "wj", "wk")]
+    ws = quan.fwd_workspace()
+    quan.quan_set_path(quan.QUAN_PATH_TC)
+    quan.quan_set_tc_tiles(0, 0, 3, 0)
+    quan.quan_set_wait_limit_ns(5_000_000)
+    quan.quan_set_fault_injection(True)
+    quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act, workspace=ws)
+    st, bits = quan.quan_device_status()
+    assert st == quan.QUAN_ERR_DEVICE_TIMEOUT and bits != 0
+    quan.quan_set_fault_injection(False)
+    quan.quan_set_wait_limit_ns(0)
+    ws.zero_()
+    y = quan.qconv2d(x, *w, stride=1, pad=1, act=spec.act, workspace=ws)
+    torch.cuda.synchronize()
+    assert quan.quan_device_status()[0] == quan.QUAN_OK
+    assert quan.quan_last_kernel().endswith(",splitk>")
+    d2 = dict(d); d2["scale"] = d2["shift"] = None
+    assert_bf16_close(out_f64(y), oracle_full(d2), "after-timeout-splitk")
+
+
 def test_bounded_wait_timeout_reports_status_and_context_survives():
     spec = inputs.small_layer("inject", 1, 16, 16, 64, 64, 3, 1, 1, seed=(400, 0))
     d = inputs.layer_inputs(spec)
