@@ -398,7 +398,9 @@ const char* quan_last_kernel(void);
  * or 2 (even H and W), Cin a multiple of 64 up to 512, Cout a multiple of 128 and no
  * residual; mode 0 picks it for those; 6: CTA pairs (tcgen05 cta_group::2), M = 256 MMAs
  * over two CTAs' pixels, each CTA keeping half of the signed block weight, only for
- * Cout = 128, Cin a multiple of 64 and kh x kw x Cin <= 1152, and never chosen by mode 0;
+ * Cout = 128, Cin a multiple of 64 and kh x kw x Cin <= 1152; mode 0 picks it for 3x3
+ * filters of stride 1 or 2 where a tile of whole output rows and its input rows (stride 2:
+ * four boxes, one per parity of the input row and column) fit twice in shared memory;
  * 7: vertical taps stacked, for 3x3 stride-1 layers with Cin = Cout = 64 (pad <= 2): one
  * MMA multiplies a row of input pixels by the block weights of the three vertical taps of
  * one horizontal tap (N = 192), its three results going to three consecutive output rows

@@ -25,6 +25,16 @@
 //              addresses, as the TMA unit wrote it, so any 128-byte row offset is a valid
 //              start (the descriptor's base-offset field stays 0).  One stage feeds
 //              9 x 4 MMAs;
+//        halo2 (stride 2, 3x3, Wp = Wo + 1 <= 128): the tile is R = 128 / Wp output rows
+//              again, and a stage holds four boxes per 64-channel chunk, one per parity of
+//              the input row and column (TMA element strides of 2): box (a, b) holds input
+//              pixels (2 (h0 + i) - pad + a, 2 j - pad + b) for i = 0 .. R, j < Wp, at a row
+//              pitch of Wp pixels.  Output pixel (r, c) reads input (2 r + dh - pad,
+//              2 c + dw - pad), which is row (r + dh / 2) Wp + c + dw / 2 of box
+//              (dh mod 2, dw mod 2), so tap (dh, dw) is again one box seen from a start row.
+//              Each box starts on a 1024-byte boundary; a padding row past the end of a box
+//              reads into the next box of the same stage (no box's MMAs reach past the
+//              stage);
 //        per tap  otherwise: one im2col box of 128 consecutive output pixels x 64 input
 //              channels per (tap, chunk) stage (4 MMAs);
 //   B  rows n = 32 q + co (real output channel c = q Qout + co = n), columns k = tap Cin +
@@ -44,8 +54,8 @@
 // the even CTA).  Even CTA, per-tap staging: warps 1 and 2 (lane 0) issue the pair's MMAs
 // for alternate pair tiles, each from its own share of the ring into its own two of four
 // 128-column accumulators (a stage's four MMAs leave a single issuer's waits exposed);
-// halo staging: warp 1 alone, through the whole ring (three stages of 36 MMAs) and the four
-// accumulators in order.  A stage is handed back to both producers and an accumulator to
+// halo staging (either stride): warp 1 alone, through the whole ring (stages of 36 MMAs)
+// and the four accumulators in order.  A stage is handed back to both producers and an accumulator to
 // both epilogues by multicast commits.  Odd CTA: warp 1's lane 0 relays each of its landed
 // stages to the even CTA's full barrier (a cluster-scope arrive), so the issuer waits on
 // one barrier per stage.  Both CTAs allocate TMEM together (cta_group::2) and free it
@@ -60,6 +70,10 @@ constexpr int CG_EXP_WARP0 = 2;       // warps 2..11 expand the B half
 constexpr int CG_EXP_WARPS = 10;
 constexpr int CG_EPI_THREADS = 256;   // warps 4..11
 constexpr int CG_HALO_MAX_WP = 128;   // halo tiles: at least one padded output row per tile
+// pixel staging of the kernel (its STG template argument)
+constexpr int CG_PER_TAP = 0;
+constexpr int CG_HALO = 1;            // stride 1: one box of R + 2 input rows per chunk
+constexpr int CG_HALO2 = 2;           // stride 2: four parity boxes of R + 1 rows per chunk
 
 struct Cg2Params {
     ConvShape s;
@@ -78,9 +92,10 @@ struct Cg2Params {
     int num_tiles;     // CTA tiles
     int num_ptiles;    // pair tiles: two consecutive CTA tiles
     // halo staging
-    int Wp;            // Wo + 2: row pitch of a stage, in pixels
+    int Wp;            // row pitch of a box, in pixels: Wo + 2 (stride 1) or Wo + 1 (stride 2)
     int R;             // output rows per tile: 128 / Wp
     int tpi;           // tiles per image: ceil(Ho / R)
+    int box_stride;    // stride 2: bytes from one parity box of a stage to the next
 };
 
 struct CgCfg {
@@ -106,9 +121,12 @@ bool cg2_ok(const ConvShape& s) {
     return static_cast<long long>(s.kh) * s.kw * s.Cin <= CG_MAX_K;
 }
 
-// Halo staging: stride 1, a 3x3 filter, output rows narrow enough for one per tile.
+// Halo staging: a 3x3 filter, stride 1 or 2, output rows narrow enough for one per tile.
 bool cg2_halo_ok(const ConvShape& s) {
     return cg2_ok(s) && s.stride == 1 && s.kh == 3 && s.kw == 3 && s.Wo + 2 <= CG_HALO_MAX_WP;
+}
+bool cg2_halo2_ok(const ConvShape& s) {
+    return cg2_ok(s) && s.stride == 2 && s.kh == 3 && s.kw == 3 && s.Wo + 1 <= CG_HALO_MAX_WP;
 }
 
 // This CTA's B half from the letters staged at `lsm` (letter L at L * letter_bytes, in the
@@ -180,7 +198,7 @@ __device__ __forceinline__ bool wait_cluster_or_abort(uint32_t bar, uint32_t par
 // One expansion warp: wait for the staged letters, expand this CTA's share, make the stores
 // visible to the tensor cores, then tell the producer (the letters may be overwritten) and
 // the even CTA's issuers (this part of the B half is ready).
-template <bool HALO>
+template <int STG>
 __device__ __forceinline__ void cg2_expand_warp(const Cg2Params& p, uint32_t sbase,
                                                 uint32_t ring, uint32_t rank, int warp,
                                                 int lane, uint32_t lbar, uint32_t lfree,
@@ -188,7 +206,7 @@ __device__ __forceinline__ void cg2_expand_warp(const Cg2Params& p, uint32_t sba
                                                 volatile int* abort_flag) {
     const int et = (warp - CG_EXP_WARP0) * 32 + lane;
     if (wait_or_abort(lbar, 0, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE)) {
-        if constexpr (HALO)
+        if constexpr (STG != CG_PER_TAP)
             cg2_expand<9>(p, sbase, ring, rank, et, 31 - __clz(p.s.Qin >> 3));
         else
             cg2_expand<0>(p, sbase, ring, rank, et, 0);
@@ -213,13 +231,15 @@ __device__ __forceinline__ void cg2_acc(int k, int& buf, uint32_t& use) {
     }
 }
 
-// NI: MMA issuers (one for halo staging, whose stages carry 36 MMAs each and are consumed
-// in order from one ring of three; two for per-tap staging, whose four-MMA stages would
-// leave a single issuer's waits exposed).
-template <bool HALO, int NI>
+// STG: the pixel staging (CG_PER_TAP, CG_HALO or CG_HALO2).  NI: MMA issuers (one for
+// halo staging, whose stages carry 36 MMAs each and are consumed in order from one ring;
+// two for per-tap staging, whose four-MMA stages would leave a single issuer's waits
+// exposed).
+template <int STG, int NI>
 __global__ void __launch_bounds__(CG_THREADS, 1)
     qconv_cg2_kernel(const __grid_constant__ CUtensorMap tmap_x, const Cg2Params p) {
     using C = CgCfg;
+    constexpr bool HALO = STG != CG_PER_TAP;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -289,7 +309,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             int t = cta_tile(k);
             if (t >= p.num_tiles) t = p.num_tiles - 1;
             img = t / p.tpi;
-            hbase = (t - img * p.tpi) * p.R - s.pad;
+            hbase = (t - img * p.tpi) * p.R * s.stride - s.pad;
             wbase = -s.pad;
         } else {
             const int hw = s.Ho * s.Wo;
@@ -348,13 +368,22 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         mbar_arrive_expect_tx(fb, static_cast<uint32_t>(p.box_bytes));
                         filled |= 1u << stage;
                         fill_parity = (fill_parity & ~(1u << stage)) | (phase << stage);
-                        if constexpr (HALO)
+                        if constexpr (STG == CG_HALO2) {
+                            // the four parity boxes (row parity a, column parity b) at
+                            // 2 a + b box strides
+#pragma unroll
+                            for (int ab = 0; ab < 4; ++ab)
+                                tma_load_4d(dst + static_cast<uint32_t>(ab * p.box_stride),
+                                            &tmap_x, fb, 64 * ch, wbase[i] + (ab & 1),
+                                            hbase[i] + (ab >> 1), img[i], pol_x);
+                        } else if constexpr (HALO) {
                             tma_load_4d(dst, &tmap_x, fb, 64 * ch, wbase[i], hbase[i], img[i],
                                         pol_x);
-                        else
+                        } else {
                             tma_load_im2col_4d(dst, &tmap_x, fb, 64 * ch, wbase[i], hbase[i],
                                                img[i], static_cast<uint16_t>(dw),
                                                static_cast<uint16_t>(dh), pol_x);
+                        }
                     }
                 }
             }
@@ -365,8 +394,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
         }
     } else if (warp <= CG_MAX_NI) {
         if (warp >= CG_EXP_WARP0)
-            cg2_expand_warp<HALO>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar,
-                                  limit, abort_flag);
+            cg2_expand_warp<STG>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar,
+                                 limit, abort_flag);
         if (rank == 0 && lane == 0 && warp <= NI) {
             // -------------------------------------------------- MMA issuers (even CTA)
             constexpr uint32_t IDESC = make_idesc(2 * BM, 128, 0);
@@ -381,8 +410,10 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             }
             tc_fence_after();
             const uint32_t b_lo0 = desc_lo(sbase);
-            // halo: descriptor offset (16-byte units) of filter row dh = 1
+            // halo: descriptor offset (16-byte units) of one box row of Wp pixels, and
+            // (stride 2) of one parity box
             const uint32_t row1 = static_cast<uint32_t>(p.Wp * 8);
+            const uint32_t box1 = static_cast<uint32_t>(p.box_stride >> 4);
             StageCursor cur(p.per);
             for (int k = me; ok && k < kt; k += NI) {
                 int buf;
@@ -409,13 +440,20 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                         desc_lo(ring + static_cast<uint32_t>(stage * p.stage_bytes));
                     if constexpr (HALO) {
                         // stage kc holds input channels 64 kc .. 64 kc + 63; tap (dh, dw)
-                        // starts dh Wp + dw rows into the box and uses weight chunk
-                        // tap cpt + kc
+                        // starts dh Wp + dw rows into the box (stride 1), or
+                        // (dh / 2) Wp + dw / 2 rows into parity box (dh mod 2, dw mod 2)
+                        // (stride 2), and uses weight chunk tap cpt + kc
 #pragma unroll
                         for (int t = 0; t < 9; ++t) {
                             const int dh = t / 3, dw = t % 3;
-                            const uint32_t a_t = a_lo + static_cast<uint32_t>(dh) * row1 +
-                                                 static_cast<uint32_t>(dw * 8);
+                            uint32_t a_t;
+                            if constexpr (STG == CG_HALO2)
+                                a_t = a_lo + static_cast<uint32_t>(2 * (dh & 1) + (dw & 1)) * box1 +
+                                      static_cast<uint32_t>(dh >> 1) * row1 +
+                                      static_cast<uint32_t>((dw >> 1) * 8);
+                            else
+                                a_t = a_lo + static_cast<uint32_t>(dh) * row1 +
+                                      static_cast<uint32_t>(dw * 8);
                             const uint32_t b_t =
                                 b_lo0 + static_cast<uint32_t>(((t * p.cpt + kc) * C::BCHUNK) >> 4);
 #pragma unroll
@@ -469,8 +507,8 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
             }
         }
     } else {
-        cg2_expand_warp<HALO>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar, limit,
-                              abort_flag);
+        cg2_expand_warp<STG>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar, limit,
+                             abort_flag);
         if (warp >= EPI_WARP0) {
             // ------------------------------------------------------------ epilogue
             // (the pair epilogue of tc_common.cuh for 32 channels per component: warps 4..7
@@ -570,7 +608,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                     } else {
                         // the tile's accumulator is in registers: hand it back
                         tc_fence_before();
-                        mbar_arrive_cluster(acce_leader0 + 8u * buf);
+                        mbar_arrive_cluster_relaxed(acce_leader0 + 8u * buf);
                     }
                     float E[NCH][8];
 #pragma unroll

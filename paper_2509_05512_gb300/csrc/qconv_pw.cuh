@@ -288,7 +288,7 @@ __global__ void __launch_bounds__(PW_THREADS, 1)
                 tmem_ld_wait();
                 // the accumulator is in registers: hand the buffer back to the issuer
                 tc_fence_before();
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
                 const long long pix0 = static_cast<long long>(t) * p.tile_pix;
                 long long left = p.npix - pix0;
                 if (left > p.tile_pix) left = p.tile_pix;

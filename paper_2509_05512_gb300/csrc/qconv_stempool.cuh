@@ -630,7 +630,7 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
                 }
                 // the accumulator is in registers: hand the buffer back to its issuer
                 tc_fence_before();
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
                 if (active) {
                     if (i == 0) {  // the first pooled row of an image: no row above
 #pragma unroll

@@ -517,18 +517,20 @@ bool encode_x_im2col(CUtensorMap* map, const ConvShape& s, const void* x, int ch
 }
 
 // Activation tiled map for halo boxes: `channels` x `cols` columns (Wo if 0) x `rows` rows
-// of one image.
+// of one image; with `step` > 1 the box takes every step-th column and row (it spans
+// step * cols columns and step * rows rows).
 bool encode_x_halo(CUtensorMap* map, const ConvShape& s, const void* x, int channels,
-                   int rows, int cols = 0) {
+                   int rows, int cols = 0, int step = 1) {
     const cuuint64_t dims[4] = {static_cast<cuuint64_t>(s.Cin), static_cast<cuuint64_t>(s.W),
                                 static_cast<cuuint64_t>(s.H), static_cast<cuuint64_t>(s.N)};
     const cuuint64_t strides[3] = {static_cast<cuuint64_t>(s.Cin) * 2,
                                    static_cast<cuuint64_t>(s.Cin) * 2 * s.W,
                                    static_cast<cuuint64_t>(s.Cin) * 2 * s.W * s.H};
     const cuuint32_t box[4] = {static_cast<cuuint32_t>(channels),
-                               static_cast<cuuint32_t>(cols > 0 ? cols : s.Wo),
-                               static_cast<cuuint32_t>(rows), 1};
-    const cuuint32_t estr[4] = {1, 1, 1, 1};
+                               static_cast<cuuint32_t>((cols > 0 ? cols : s.Wo) * step),
+                               static_cast<cuuint32_t>(rows * step), 1};
+    const cuuint32_t estr[4] = {1, static_cast<cuuint32_t>(step), static_cast<cuuint32_t>(step),
+                                1};
     const CUresult r = g_encode_tiled(
         map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(x), dims, strides, box, estr,
         CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for_row(channels * 2),
@@ -1043,15 +1045,34 @@ bool encode_rgb_rows(CUtensorMap* map, const ConvShape& s, const float* rgb, int
     return r == CUDA_SUCCESS;
 }
 
-// Sizes of the CTA-pair kernel for shape s (halo or per-tap staging); false if its stage
-// ring or the staged letters do not fit.
-bool cg2_plan(const ConvShape& s, bool halo, Cg2Params* prm) {
-    if (!cg2_ok(s) || (halo && !cg2_halo_ok(s))) return false;
+// Sizes of the CTA-pair kernel for shape s with pixel staging stg (CG_PER_TAP, CG_HALO or
+// CG_HALO2); false if the staging does not apply or its stage ring or the staged letters do
+// not fit.
+bool cg2_plan(const ConvShape& s, int stg, Cg2Params* prm) {
+    if (!cg2_ok(s) || (stg == CG_HALO && !cg2_halo_ok(s)) ||
+        (stg == CG_HALO2 && !cg2_halo2_ok(s)))
+        return false;
+    const bool halo = stg != CG_PER_TAP;
     prm->cpt = s.Cin / 64;
     prm->kchunks = s.kh * s.kw * prm->cpt;
     prm->letter_bytes = 32 * s.kh * s.kw * s.Qin * 2;
     long long tiles;
-    if (halo) {
+    if (stg == CG_HALO2) {
+        // R output rows of Wp = Wo + 1 pixels per tile; four parity boxes of R + 1 rows of
+        // Wp pixels per stage, each from a 1024-byte boundary.  A padding MMA row reads at
+        // most Wp + 1 rows past the 128th row of box (0, 0) and Wp rows past that of box
+        // (0, 1), both inside the following boxes; boxes (1, 0) and (1, 1) are read at
+        // offsets of at most one row, within their (R + 1) Wp > 128 rows plus the next box.
+        prm->Wp = s.Wo + 1;
+        prm->R = BM / prm->Wp;
+        prm->tpi = (s.Ho + prm->R - 1) / prm->R;
+        const int box_rows = (prm->R + 1) * prm->Wp;
+        prm->box_stride = (box_rows * 128 + 1023) / 1024 * 1024;
+        prm->stage_bytes = 4 * prm->box_stride;
+        prm->box_bytes = 4 * box_rows * 128;
+        prm->nst = prm->cpt;
+        tiles = static_cast<long long>(s.N) * prm->tpi;
+    } else if (halo) {
         // R output rows of Wp = Wo + 2 pixels per tile; a stage holds the R + 2 input rows
         // of the box and every row an MMA of the last tap reads (128 + 2 Wp + 2)
         prm->Wp = s.Wo + 2;
@@ -1082,17 +1103,20 @@ bool cg2_plan(const ConvShape& s, bool halo, Cg2Params* prm) {
     return true;
 }
 
-bool cg2_halo_fits(const ConvShape& s) {
+// The halo staging that fits shape s (CG_HALO or CG_HALO2), else CG_PER_TAP.
+int cg2_halo_staging(const ConvShape& s) {
     Cg2Params prm = {};
-    return cg2_plan(s, true, &prm);
+    if (cg2_plan(s, CG_HALO, &prm)) return CG_HALO;
+    if (cg2_plan(s, CG_HALO2, &prm)) return CG_HALO2;
+    return CG_PER_TAP;
 }
 
 cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4],
                        const EpilogueArgs& ep, void* out, const TcOptions& opt, int num_sms,
                        cudaStream_t stream, char* err, size_t errlen) {
     Cg2Params prm = {};
-    const bool halo = cg2_halo_fits(s);
-    if (!cg2_plan(s, halo, &prm)) {
+    const int stg = cg2_halo_staging(s);
+    if (!cg2_plan(s, stg, &prm)) {
         snprintf(err, errlen, "CTA-pair kernel: Cin=%d Cout=%d %dx%d does not fit", s.Cin,
                  s.Cout, s.kh, s.kw);
         return cudaErrorInvalidValue;
@@ -1103,11 +1127,12 @@ cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4]
     prm.y = out;
     prm.wait_limit_ns = opt.wait_limit_ns;
     prm.inject_stall = opt.inject_stall;
-    const MapKey key = make_key(s, x, w, out, 64, 32, halo ? 11 : 10);
+    const MapKey key = make_key(s, x, w, out, 64, 32, 10 + stg);
     CUtensorMap maps[6];
     if (!cache_lookup(key, maps)) {
-        const bool okx = halo ? encode_x_halo(&maps[0], s, x, 64, prm.R + 2, prm.Wp)
-                              : encode_x_im2col(&maps[0], s, x, 64);
+        const bool okx = stg == CG_HALO2 ? encode_x_halo(&maps[0], s, x, 64, prm.R + 1, prm.Wp, 2)
+                         : stg == CG_HALO ? encode_x_halo(&maps[0], s, x, 64, prm.R + 2, prm.Wp)
+                                          : encode_x_im2col(&maps[0], s, x, 64);
         if (!okx) {
             snprintf(err, errlen, "tensor map encoding failed for the activation tensor");
             return cudaErrorInvalidValue;
@@ -1118,10 +1143,14 @@ cudaError_t launch_cg2(const ConvShape& s, const void* x, const void* const w[4]
     int pairs = (opt.max_ctas > 0 ? opt.max_ctas : num_sms) / 2;
     if (pairs > prm.num_ptiles) pairs = prm.num_ptiles;
     if (pairs < 1) pairs = 1;
-    set_kernel_name(halo ? "qconv_cg2_kernel<halo>" : "qconv_cg2_kernel");
-    auto kern = halo ? qconv_cg2_kernel<true, 1> : qconv_cg2_kernel<false, 2>;
-    static std::atomic<unsigned long long> attr_done[2];
-    cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done[halo ? 1 : 0]);
+    set_kernel_name(stg == CG_HALO2  ? "qconv_cg2_kernel<halo2>"
+                    : stg == CG_HALO ? "qconv_cg2_kernel<halo>"
+                                     : "qconv_cg2_kernel");
+    auto kern = stg == CG_HALO2  ? qconv_cg2_kernel<CG_HALO2, 1>
+                : stg == CG_HALO ? qconv_cg2_kernel<CG_HALO, 1>
+                                 : qconv_cg2_kernel<CG_PER_TAP, 2>;
+    static std::atomic<unsigned long long> attr_done[3];
+    cudaError_t e = set_smem_once(kern, CgCfg::SMEM_BYTES, attr_done[stg]);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * pairs);
@@ -1387,7 +1416,8 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                  "Wo + 2 <= %d or Wo dividing %d", BM, BM);
         return cudaErrorInvalidValue;
     }
-    if (!s.sep && cg2_ok(s) && (opt.mode == 6 || (opt.mode == 0 && cg2_halo_fits(s))))
+    if (!s.sep && cg2_ok(s) &&
+        (opt.mode == 6 || (opt.mode == 0 && cg2_halo_staging(s) != CG_PER_TAP)))
         return launch_cg2(s, x, w, ep, out, opt, num_sms, stream, err, errlen);
     if (opt.mode == 6) {
         snprintf(err, errlen,

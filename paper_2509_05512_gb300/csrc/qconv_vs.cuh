@@ -566,7 +566,7 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
             if (__shfl_sync(0xffffffffu, ok ? 1 : 0, 0) == 0) break;
             tc_fence_after();
             if (!mine) {
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
                 continue;
             }
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
@@ -586,7 +586,7 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
                 } else {
                     // the band row is in registers: hand the buffer back to the issuer
                     tc_fence_before();
-                    mbar_arrive(acce0 + 8u * buf);
+                    mbar_arrive_relaxed(acce0 + 8u * buf);
                 }
                 float E[2][8];  // E[jj][e]: channel 16 b + 8 jj + e of this lane's row
 #pragma unroll

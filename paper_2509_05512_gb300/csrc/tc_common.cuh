@@ -467,7 +467,7 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
             } else {
                 // the tile's accumulator is in registers: hand the buffer back
                 tc_fence_before();
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
             }
             if (unit.kind == UNIT_HEAD) {
                 // this CTA's share of the tile: the raw accumulator to the partial slot (L2)
@@ -608,7 +608,7 @@ __device__ __forceinline__ void epilogue_direct_sep(const ConvShape& s, const Ep
             if (sub == NSUB - 1) {
                 // the tile's accumulator is in registers: hand the buffer back
                 tc_fence_before();
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
             }
 #pragma unroll
             for (int m = 0; m < 4; ++m) {
@@ -705,7 +705,7 @@ __device__ __forceinline__ void epilogue_direct64(const ConvShape& s, const Epil
             if (h == 1) {
                 // the accumulator is in registers: hand the buffer back to the MMA issuer
                 tc_fence_before();
-                mbar_arrive(acce0 + 8u * buf);
+                mbar_arrive_relaxed(acce0 + 8u * buf);
             }
             const int c0 = 32 * h + 8 * ci;
             uint4 r4[4];

@@ -458,7 +458,7 @@ def test_tc_pointwise_mode_rejects_other_shapes():
 
 # ------------------------------------------------------------------ CTA-pair kernel (Cout 128)
 
-HALO, PER_TAP = "qconv_cg2_kernel<halo>", "qconv_cg2_kernel"
+HALO, HALO2, PER_TAP = "qconv_cg2_kernel<halo>", "qconv_cg2_kernel<halo2>", "qconv_cg2_kernel"
 CG2_CASES = [
     # name, N, H, W, Cin, Cout, k, stride, pad, extra, kernel
     # halo staging (stride 1, 3x3): 8 rows of 15 per tile, the image's second tile 6 rows
@@ -471,10 +471,21 @@ CG2_CASES = [
     ("cg2h_pad0", 2, 10, 12, 128, 128, 3, 1, 0, {}, HALO),   # box from column 0
     ("cg2h_pad2", 1, 9, 7, 64, 128, 3, 1, 2, {"residual": True}, HALO),  # box from column -2
     ("cg2h_deep", 3, 28, 28, 128, 128, 3, 1, 1, {"residual": True}, HALO),  # the stage-2 shape
-    # per-tap staging: stride 2, other filters, rows too wide for two halo stages
-    ("cg2_s2", 3, 15, 17, 64, 128, 3, 2, 1, {}, PER_TAP),                # 216 pixels
+    # stride-2 halo staging (four parity boxes per stage): odd input sizes, one tile of
+    # 8 rows of 10 per image
+    ("cg2h2_odd", 3, 15, 17, 64, 128, 3, 2, 1, {}, HALO2),
+    ("cg2h2_stage2", 3, 56, 56, 64, 128, 3, 2, 1, {"residual": True}, HALO2),  # 7 tiles of 4 rows
+    ("cg2h2_ragged", 2, 20, 58, 64, 128, 3, 2, 1,                # 29 columns, 10 rows: the
+     {"bias": True, "act": quan.QUAN_ACT_SILU}, HALO2),          # third tile has 2 of 4 rows
+    ("cg2h2_pad0", 2, 13, 13, 64, 128, 3, 2, 0, {}, HALO2),      # boxes from column 0 and 1
+    ("cg2h2_pad2", 1, 11, 11, 64, 128, 3, 2, 2, {"residual": True}, HALO2),  # from -2 and -1
+    ("cg2h2_one_col", 2, 9, 2, 64, 128, 3, 2, 1, {}, HALO2),     # Wo = 1: 64 rows per tile
+    # per-tap staging: other filters, rows too wide for two halo stages, or a block weight
+    # that leaves room for one stride-2 stage only
+    ("cg2_s2_wide_k", 3, 15, 17, 128, 128, 3, 2, 1, {}, PER_TAP),        # 216 pixels
     ("cg2_5x1", 2, 11, 9, 128, 128, 5, 1, 2, {"kw": 1}, PER_TAP),        # 5 taps x 128
     ("cg2_too_wide", 1, 3, 100, 128, 128, 3, 1, 1, {}, PER_TAP),         # 102-pixel pitch
+    ("cg2_s2_too_wide", 1, 5, 120, 64, 128, 3, 2, 1, {}, PER_TAP),       # 61-pixel pitch
 ]
 
 
@@ -500,10 +511,29 @@ def test_tc_cta_pair_few_pairs(max_ctas):
 @pytest.mark.parametrize("max_ctas", [4, 6])
 def test_tc_cta_pair_per_tap_few_pairs(max_ctas):
     # the per-tap staging's ring (12 stages) wraps many times
-    spec = inputs.small_layer("cg2_few_s2", 4, 30, 30, 64, 128, 3, 2, 1, seed=(217, max_ctas))
+    spec = inputs.small_layer("cg2_few_s2", 4, 30, 30, 128, 128, 3, 2, 1, seed=(217, max_ctas))
     quan.quan_set_tc_tiles(0, 0, max_ctas, 6)
     check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
     assert quan.quan_last_kernel() == PER_TAP
+
+
+@pytest.mark.parametrize("max_ctas", [2, 6])
+def test_tc_cta_pair_stride2_few_pairs(max_ctas):
+    # one or three pairs: the two-stage ring of parity boxes and the four accumulators wrap
+    # many times (6 images of 2 tiles of 8 rows)
+    spec = inputs.small_layer("cg2h2_few", 6, 30, 30, 64, 128, 3, 2, 1, residual=True,
+                              seed=(218, max_ctas))
+    quan.quan_set_tc_tiles(0, 0, max_ctas, 6)
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == HALO2
+
+
+def test_tc_cta_pair_stride2_default_choice():
+    # the backbone's first stage-2 convolution (3x3 / 2, 64 -> 128) takes the CTA-pair
+    # kernel with parity boxes by default
+    spec = inputs.small_layer("cg2h2_default", 2, 56, 56, 64, 128, 3, 2, 1, seed=(219, 0))
+    check(spec, path=quan.QUAN_PATH_TC, expect_path=quan.QUAN_PATH_TC)
+    assert quan.quan_last_kernel() == HALO2
 
 
 def test_tc_cta_pair_matches_pair_kernel():
@@ -718,18 +748,18 @@ def test_maxpool(shape):
 # ------------------------------------------------------------------ failure detection
 
 @pytest.mark.parametrize("mode,issuers", [(2, 0), (3, 2), (3, 3), (4, 0), (5, 0), (6, 0),
-                                          (6, 1), (7, 0)])
+                                          (6, 1), (6, 2), (7, 0)])
 def test_bounded_wait_timeout_every_kernel(mode, issuers):
     # the failure-injection path of the pair-mode, weight-stationary (two and three
-    # issuers), gather, pointwise and CTA-pair kernels (halo staging, and per-tap staging
-    # for the strided layer marked by issuers = 1, which the CTA-pair kernel ignores)
+    # issuers), gather, pointwise and CTA-pair kernels (the CTA-pair kernel ignores the
+    # issuer count, which selects its staging here: halo, stride-2 halo, per tap)
     if mode == 4:
         spec = inputs.small_layer("inject_m", 2, 32, 32, 4, 64, 7, 2, 3, seed=(401, mode))
     elif mode == 5:
         spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 1, 1, 0, seed=(401, mode))
     elif mode == 6:
-        spec = inputs.small_layer("inject_m", 2, 16, 16, 64, 128, 3, 1 + issuers, 1,
-                                  seed=(401, mode))
+        spec = inputs.small_layer("inject_m", 2, 16, 16, 128 if issuers == 2 else 64, 128, 3,
+                                  1 if issuers == 0 else 2, 1, seed=(401, mode))
         issuers = 0
     else:
         spec = inputs.small_layer("inject_m", 1, 16, 16, 64, 64, 3, 1, 1, seed=(401, mode))
