@@ -31,7 +31,14 @@
  *               keeps no reference after the call and allocates nothing per call.
  *               `out` must not overlap any input.
  *   Streams     calls are asynchronous on `stream` (a cudaStream_t; NULL is the legacy
- *               default stream) and do not synchronise.
+ *               default stream) and do not synchronise.  Kernels are launched with
+ *               programmatic stream serialization: a convolution kernel may start while
+ *               the preceding library kernel on the stream finishes, and waits for it
+ *               before touching activations (input, residual, output).  Its weights and
+ *               per-channel vectors may be read before that wait, so they must not be
+ *               written by the immediately preceding call on the stream when that call is
+ *               a forward convolution or quan_qconv2d_bwd_weight (any other producer, e.g.
+ *               a framework kernel or a copy, completes before the call's kernels start).
  *   Errors      argument errors are detected on the host before anything is launched and
  *               return QUAN_ERR_INVALID_ARG or QUAN_ERR_UNSUPPORTED; a launch failure
  *               returns QUAN_ERR_CUDA.  quan_last_error_message() describes the last error

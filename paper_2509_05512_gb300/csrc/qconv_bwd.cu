@@ -45,12 +45,13 @@ __device__ __forceinline__ void mix_eq9(float dr, float di, float dj, float dk, 
 }
 
 // out_L[ci][dh][dw][co] = s_L * W_L[co][kh-1-dh][kw-1-dw][ci], s = (+1, -1, -1, -1) when
-// conj, else +1.
+// conj, else +1.  Its output is the next kernel's weight operand, which the forward
+// tensor-core kernels read before their dependency wait: this kernel does not trigger its
+// dependents early, so the next one starts only once it has completed.
 __global__ void __launch_bounds__(256) bwd_transform_kernel(
     int Qin, int Qout, int kh, int kw, int conj, const __nv_bfloat16* __restrict__ wr,
     const __nv_bfloat16* __restrict__ wi, const __nv_bfloat16* __restrict__ wj,
     const __nv_bfloat16* __restrict__ wk, __nv_bfloat16* __restrict__ out) {
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     asm volatile("griddepcontrol.wait;" ::: "memory");
     const long long per = static_cast<long long>(Qin) * kh * kw * Qout;
     const __nv_bfloat16* w[4] = {wr, wi, wj, wk};

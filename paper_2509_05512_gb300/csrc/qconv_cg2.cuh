@@ -298,7 +298,9 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     cluster_sync_all();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    griddep_wait();  // the previous kernel's output (this layer's input) is complete
+    // The letters are staged and expanded before the dependency wait, overlapping the
+    // previous kernel's last CTAs; every thread that touches activations (the pixel
+    // producer, the epilogue) waits for that kernel before its first access.
 
     // CTA tile of local pair tile k
     auto cta_tile = [&](int k) { return 2 * (pair + k * npairs) + static_cast<int>(rank); };
@@ -335,6 +337,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
                 bulk_load(ring + static_cast<uint32_t>(l * p.letter_bytes), p.w[l],
                           static_cast<uint32_t>(p.letter_bytes), lbar);
             bool ok = wait_or_abort(lfree, 0, limit, abort_flag, STATUS_TIMEOUT_PRODUCER);
+            griddep_wait();  // the previous kernel's output (this layer's input) is complete
             StageCursor cur(p.per);
             for (int g0 = 0; ok && g0 < kt; g0 += NI) {
                 const int ng = kt - g0 < NI ? kt - g0 : NI;
@@ -509,6 +512,7 @@ __global__ void __launch_bounds__(CG_THREADS, 1)
     } else {
         cg2_expand_warp<STG>(p, sbase, ring, rank, warp, lane, lbar, lfree, bready_bar, limit,
                              abort_flag);
+        griddep_wait();  // the residual complete, the output buffer no longer read
         if (warp >= EPI_WARP0) {
             // ------------------------------------------------------------ epilogue
             // (the pair epilogue of tc_common.cuh for 32 channels per component: warps 4..7

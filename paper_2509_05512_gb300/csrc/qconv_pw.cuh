@@ -163,11 +163,14 @@ __global__ void __launch_bounds__(PW_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    griddep_wait();  // the previous kernel's output (this layer's input) is complete
+    // The block weight is expanded before the dependency wait, overlapping the previous
+    // kernel's last CTAs; the producer and the epilogue wait for that kernel before their
+    // first access to activations.
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
+            griddep_wait();  // the previous kernel's output (this layer's input) is complete
             const uint64_t pol = l2_policy_evict_normal();
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
@@ -260,6 +263,7 @@ __global__ void __launch_bounds__(PW_THREADS, 1)
         }
     } else {
         pw_expand(p, smem, mb, (warp - PW_EXP_WARP0) * 32 + lane, lane, bready_bar);
+        griddep_wait();  // the output buffer no longer read by the previous kernel
         if (warp >= PW_EPI_WARP0) {
             // -------------------------------------------------------- epilogue
             const int qd = warp & 3;                     // TMEM lane quadrant: component

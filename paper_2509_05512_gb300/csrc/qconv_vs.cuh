@@ -300,7 +300,9 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    griddep_wait();  // the previous kernel's output (this layer's input) is complete
+    // The block weight is expanded before the dependency wait, overlapping the previous
+    // kernel's last CTAs; the producers and the epilogue wait for that kernel before their
+    // first access to activations.
 
     // unit u: image group u / nbands, band u % nbands
     auto unit_geo = [&](int u, int& n0, int& h0, int& r) {
@@ -328,6 +330,7 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
         // three boxes: producer pid loads box dw = pid of every row; one box: producer pid loads
         // row pid of every stage (the TMA unit takes several threads' copies at once)
         const int x0 = (NBOX == 3 ? pid : 0) - s.pad;
+        griddep_wait();  // the previous kernel's output (this layer's input) is complete
         for (int u = blockIdx.x; ok && u < p.num_units; u += gridDim.x) {
             int n0, h0, r;
             unit_geo(u, n0, h0, r);
@@ -501,6 +504,7 @@ __global__ void __launch_bounds__(VS_THREADS, 1)
             vec[64 + et] = fmaf(sc, b, p.ep.scale ? __ldg(p.ep.shift + et) : 0.0f);
         }
         named_bar_sync(1, VS_EPI_THREADS);
+        griddep_wait();  // the residual complete, the output buffer no longer read
         // ------------------------------------------------------------ epilogue
         // Per band row, four blocks of 16 columns; a block's 32 lanes x 2 chunks of 8 channels
         // are transposed across lane pairs, so lane 2 m + c holds chunk c of lanes row0 and
