@@ -218,7 +218,7 @@ __device__ __forceinline__ void sp_chunk(const uint32_t (&acc)[32], float carry,
     float hm[16];  // horizontal 3-wide stride-2 max of this lane's row
 #pragma unroll
     for (int t = 0; t < 16; ++t)
-        hm[t] = fmaxf(fmaxf(t == 0 ? carry : a[2 * t - 1], a[2 * t]), a[2 * t + 1]);
+        hm[t] = fmax3(t == 0 ? carry : a[2 * t - 1], a[2 * t], a[2 * t + 1]);
     if (!rows_ok) {  // warp-uniform: output row 2 i + 1 is past the end (odd Ho)
 #pragma unroll
         for (int t = 0; t < 16; ++t) hm[t] = v_ok ? hm[t] : -INFINITY;
@@ -230,7 +230,7 @@ __device__ __forceinline__ void sp_chunk(const uint32_t (&acc)[32], float carry,
         const float mine = v ? hm[2 * u + 1] : hm[2 * u];
         const float send = v ? hm[2 * u] : hm[2 * u + 1];
         const float recv = __shfl_xor_sync(0xffffffffu, send, 1);
-        m[u] = fmaxf(fmaxf(mine, recv), prev1[u]);
+        m[u] = fmax3(mine, recv, prev1[u]);
         prev1[u] = v ? mine : recv;  // output row 2 i + 1 at this lane's column
     }
     if (!store) return;  // warp-uniform (the priming tile)
@@ -377,12 +377,15 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    griddep_wait();  // the previous kernel's output (this layer's input) is complete
+    // The block weight is expanded before the dependency wait, overlapping the previous
+    // kernel's last CTAs; the input loaders and the epilogue wait for that kernel before
+    // their first access to activations.
 
     if (RGB && (warp == 0 || warp == 3)) {
         // ------------------------------------------------- RGB staging and conversion
         // (warp 3 first helps with the weight expansion)
         if (warp == 3) sp_expand<RAW>(p, smem, (warp - SP_EXP_WARP0) * 32 + lane, lane, bready_bar);
+        griddep_wait();  // the previous kernel's output (this layer's input) is complete
         const int ct = (warp == 0 ? 0 : 32) + lane;
         const uint64_t pol_x = l2_policy_evict_first();
         const uint32_t tx = static_cast<uint32_t>(p.rows * p.rgb_row_bytes);
@@ -455,6 +458,7 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
     } else if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
         if (lane == 0) {
+            griddep_wait();  // the previous kernel's output (this layer's input) is complete
             const uint64_t pol_x = l2_policy_evict_normal();
             uint32_t filled = 0, fill_parity = 0;
             bool ok = true;
@@ -590,6 +594,7 @@ __global__ void __launch_bounds__(SP_THREADS, 1)
         }
     } else {
         sp_expand<RAW>(p, smem, (warp - SP_EXP_WARP0) * 32 + lane, lane, bready_bar);
+        griddep_wait();  // the output buffer no longer read by earlier kernels
         if (warp >= SP_EPI_WARP0) {
             // -------------------------------------------------------- epilogue
             const int qd = warp & 3;                    // TMEM lane quadrant
