@@ -99,15 +99,38 @@ def load_peaks():
 HOST_ONLY_SOURCES = ("quan_api.cu",)
 
 
-def kernel_source_hash() -> str:
-    """Hash of the device-code sources under csrc (every file but the host-only front
-    end): a recorded ncu traffic figure stays valid while it is unchanged."""
+# Device-code sources each kernel is built from, beyond the shared ones: an ncu traffic
+# figure stays valid while these are unchanged.  qconv_tc.cu holds the tensor-core kernels'
+# host launch code (grid, tiles, tensor maps) and includes every .cuh listed here.
+SHARED_DEVICE_SOURCES = ("ptx.cuh", "tc_common.cuh", "internal.h")
+KERNEL_SOURCES = {
+    "qconv_stem_pool_kernel": ("qconv_tc.cu", "qconv_stempool.cuh", "qconv_gather.cuh"),
+    "qconv_pairs_kernel": ("qconv_tc.cu", "qconv_gather.cuh"),
+    "qconv_vs_kernel": ("qconv_tc.cu", "qconv_vs.cuh"),
+    "qconv_ws_kernel": ("qconv_tc.cu", "qconv_ws.cuh"),
+    "qconv_cg2_kernel": ("qconv_tc.cu", "qconv_cg2.cuh"),
+    "qconv_pw_kernel": ("qconv_tc.cu", "qconv_pw.cuh"),
+    "qconv_tc_kernel": ("qconv_tc.cu",),
+    "qconv_dw_kernel": ("qconv_tc.cu", "qconv_dw.cuh"),
+    "iqbn_apply_kernel": ("iqbn.cu",),
+    "iqbn_stats_kernel": ("iqbn.cu",),
+    "poincare_kernel": ("poincare.cu",),
+}
+
+
+def kernel_source_hash(kernel: str | None = None) -> str:
+    """Hash of the device-code sources of `kernel` (the library's kernel name; its base
+    name before '<' selects the files), or of every source under csrc but the host-only
+    front end for an unknown or absent name."""
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2509_05512_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name in HOST_ONLY_SOURCES:
-            continue
+    base = (kernel or "").split("<")[0].split()[0] if kernel else ""
+    if base in KERNEL_SOURCES:
+        names = sorted(SHARED_DEVICE_SOURCES + KERNEL_SOURCES[base])
+    else:
+        names = [n for n in sorted(os.listdir(csrc)) if n not in HOST_ONLY_SOURCES]
+    for name in names:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode())
             h.update(f.read())
@@ -117,15 +140,15 @@ def kernel_source_hash() -> str:
 def recorded_traffic(workload: str, kernel: str | None = None, path: str | None = None):
     """DRAM bytes per launch of the dominant kernel from the committed ncu summary, or
     None when no capture exists, it is of another kernel or template instance (the full
-    name, template arguments included, must match), or the kernel sources changed since it
-    was taken."""
+    name, template arguments included, must match), or that kernel's device sources
+    changed since it was taken."""
     path = path or os.path.join(ROOT, "profiles", "ncu_traffic.json")
     try:
         with open(path) as f:
             rec = json.load(f).get(workload)
     except (OSError, ValueError):
         return None
-    if not rec or rec.get("kernel_sha") != kernel_source_hash():
+    if not rec or rec.get("kernel_sha") != kernel_source_hash(rec.get("kernel")):
         return None
     if kernel is not None and kernel != rec.get("kernel"):
         return None  # another kernel, or another template instance of it

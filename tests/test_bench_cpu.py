@@ -61,7 +61,7 @@ def test_recorded_traffic_lookup(tmp_path):
     # name, template instance included) and the current device-code sources
     import json
     rec = {"c1": {"kernel": "qconv_ws_kernel<halo,issuers=2>", "dram_bytes_per_launch": 123,
-                  "kernel_sha": bench.kernel_source_hash()},
+                  "kernel_sha": bench.kernel_source_hash("qconv_ws_kernel<halo,issuers=2>")},
            "old": {"kernel": "qconv_ws_kernel<halo,issuers=2>", "dram_bytes_per_launch": 7,
                    "kernel_sha": "0000000000000000"}}
     path = str(tmp_path / "traffic.json")
@@ -72,6 +72,13 @@ def test_recorded_traffic_lookup(tmp_path):
     assert bench.recorded_traffic("c1", "qconv_tc_kernel<pair,kappa=32,bnq=64>", path) is None
     assert bench.recorded_traffic("old", "qconv_ws_kernel<halo,issuers=2>", path) is None
     assert bench.recorded_traffic("no_such_workload", None, path) is None
+
+    # the hash follows the kernel's own sources: another kernel's file does not enter it
+    assert bench.kernel_source_hash("qconv_ws_kernel<x>") != bench.kernel_source_hash(
+        "qconv_vs_kernel<x>")
+    assert bench.kernel_source_hash("qconv_ws_kernel<a>") == bench.kernel_source_hash(
+        "qconv_ws_kernel<b>")
+    assert bench.kernel_source_hash(None) == bench.kernel_source_hash("unknown_kernel")
 
     class A:
         workload, direction, variant = "c2a", "bwd", "separable"
