@@ -149,6 +149,33 @@ quan_status_t quan_qconv2d_fwd_ex(const void* x, const void* wr, const void* wi,
                                   void* out, quan_stream_t stream);
 
 /*
+ * A convolution (Eq. 5/6, as quan_qconv2d_fwd: x, its letters, bias / IQBN scale / shift,
+ * act -> out) and a 1x1 quaternion convolution of the same input x with the same stride and
+ * no padding (the residual shortcut of a downsampling block, Sec. III-D: letters sc_w*
+ * [Cout_sc/4][1][1][Cin/4], its own bias / IQBN scale / shift and activation -> out_sc
+ * [N][Ho][Wo][Cout_sc]), both bf16, in one call.  The shortcut reads x at (ho stride,
+ * wo stride), the pixel the convolution's filter tap (pad, pad) reads, so on the tensor
+ * path the two run as one launch: the shortcut's output-channel tiles follow the
+ * convolution's and run the K blocks of that tap only, with their own letters and
+ * epilogue (quan_last_kernel() then names a "shortcut" instance).  Shapes without that form
+ * (or the CUDA-core path) run as the two separate calls.  Each output equals, within
+ * rounding, what quan_qconv2d_fwd gives for its layer; with the same tile overrides the
+ * fused launch is bit-identical to separate calls on the quad/pair kernel.
+ *   Requirements: pad < kh and pad < kw; (H - 1) / stride + 1 == Ho and likewise for W
+ *   (the two outputs have one size); out and out_sc disjoint from each other and from every
+ *   input.  No residual input, no split workspace.
+ * Errors: QUAN_ERR_INVALID_ARG for argument errors of either layer or mismatched output
+ * sizes; otherwise as quan_qconv2d_fwd.
+ */
+quan_status_t quan_qconv2d_fwd_shortcut(
+    const void* x, const void* wr, const void* wi, const void* wj, const void* wk,
+    const float* bias, const float* iqbn_scale, const float* iqbn_shift, int N, int H, int W,
+    int Cin, int Cout, int kh, int kw, int stride, int pad, int act, const void* sc_wr,
+    const void* sc_wi, const void* sc_wj, const void* sc_wk, const float* sc_bias,
+    const float* sc_iqbn_scale, const float* sc_iqbn_shift, int Cout_sc, int sc_act, void* out,
+    void* out_sc, quan_stream_t stream);
+
+/*
  * The separable QUAN convolution of Eq. 7 (Sec. III-B), bf16, same arguments, layouts,
  * epilogue and errors as quan_qconv2d_fwd.  Each output component is a signed sum of the
  * four per-component convolutions c_p = W_p (*) x_p (p = r, i, j, k):

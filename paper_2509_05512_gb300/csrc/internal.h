@@ -59,6 +59,19 @@ cudaError_t read_and_clear_status(unsigned* status, cudaStream_t stream);
 // Workspace bytes that let a quad/pair-kernel launch on a device of num_sms SMs split its
 // K ranges evenly over its CTAs (one fp32 partial tile and one flag per CTA).
 size_t tc_split_workspace_bytes(int num_sms);
+// The convolution s and a 1x1 shortcut (Qout_sc quaternion output channels, no padding, the
+// same stride) on the same input x in one tensor-core launch; its own letters, epilogue
+// vectors (no residual), activation and output.
+bool tc_shortcut_supported(const ConvShape& s, const void* x, const void* const w[4],
+                           const void* out, const EpilogueArgs& ep, const void* const wsc[4],
+                           int qout_sc, const EpilogueArgs& ep_sc, const void* out_sc,
+                           const TcOptions& opt);
+cudaError_t launch_qconv_tc_shortcut(const ConvShape& s, const void* x, const void* const w[4],
+                                     const EpilogueArgs& ep, void* out,
+                                     const void* const wsc[4], int qout_sc, int act_sc,
+                                     const EpilogueArgs& ep_sc, void* out_sc,
+                                     const TcOptions& opt, int num_sms, cudaStream_t stream,
+                                     char* err, size_t errlen);
 // Name of the tensor-core kernel the calling thread's last launch_qconv_tc used.
 const char* last_tc_kernel();
 

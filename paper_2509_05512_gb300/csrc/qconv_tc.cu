@@ -93,6 +93,12 @@ struct TcParams {
     unsigned long long wait_limit_ns;
     int inject_stall;
     SplitK sk;        // K ranges split evenly over the CTAs (QUAD/PAIR modes, caller workspace)
+    ScParams sc;      // the fused 1x1 shortcut (the SC form of the kernel)
+};
+
+// The fused shortcut's four letter maps (SC form; unused otherwise).
+struct ScMaps {
+    CUtensorMap w[4];
 };
 
 template <int KAPPA, int BNQ, int MODE>
@@ -125,13 +131,18 @@ struct Cfg {
     static_assert(BNQ == 16 || BNQ == 32 || BNQ == 64, "BNQ");
 };
 
-template <int KAPPA, int BNQ, int MODE>
+// SC: N tiles from p.sc.n_conv on belong to a 1x1 shortcut on the same input, fused into
+// the launch (ScParams): their K blocks are the filter tap p.sc.tap's only, their letters
+// come from `scm`, and the epilogue writes them to the shortcut's output.
+template <int KAPPA, int BNQ, int MODE, bool SC = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     qconv_tc_kernel(const __grid_constant__ CUtensorMap tmap_x,
                     const __grid_constant__ CUtensorMap tmap_wr,
                     const __grid_constant__ CUtensorMap tmap_wi,
                     const __grid_constant__ CUtensorMap tmap_wj,
-                    const __grid_constant__ CUtensorMap tmap_wk, const TcParams p) {
+                    const __grid_constant__ CUtensorMap tmap_wk, const TcParams p,
+                    const __grid_constant__ ScMaps scm) {
+    static_assert(!SC || MODE == MODE_PAIR || MODE == MODE_QUAD, "fused shortcut modes");
     using C = Cfg<KAPPA, BNQ, MODE>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ uint8_t smem_raw[];
@@ -177,6 +188,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         tma_prefetch_desc(&tmap_wi);
         tma_prefetch_desc(&tmap_wj);
         tma_prefetch_desc(&tmap_wk);
+        if constexpr (SC)
+            for (int l = 0; l < 4; ++l) tma_prefetch_desc(&scm.w[l]);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
@@ -215,8 +228,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 int tap = unit.k0 / p.kchunks;
                 int chunk = unit.k0 - tap * p.kchunks;
                 int dh = tap / s.kw, dw = tap - (tap / s.kw) * s.kw;
-                for (int kt = unit.k0; kt < unit.k1; ++kt) {
-                    if (kt > unit.k0 && ++chunk == p.kchunks) {
+                int k1 = unit.k1;
+                bool sct = false;  // a fused shortcut's tile: one tap, its own letters
+                if constexpr (SC) {
+                    sct = n_tile >= p.sc.n_conv;
+                    if (sct) {
+                        k1 = p.sc.ktiles;
+                        tap = p.sc.tap;
+                        dh = p.sc.dh;
+                        dw = p.sc.dw;
+                        chunk = 0;
+                    }
+                }
+                for (int kt = unit.k0; kt < k1; ++kt) {
+                    if (SC && sct) {
+                        if (kt > unit.k0) ++chunk;
+                    } else if (kt > unit.k0 && ++chunk == p.kchunks) {
                         chunk = 0;
                         ++tap;
                         if (++dw == s.kw) {
@@ -246,7 +273,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                                static_cast<uint16_t>(dh), pol_x);
                     } else {
                         const int wcol = tap * s.Qin + cin0, wrow = n_tile * BNQ;
-                        if constexpr (MODE == MODE_PAIR) {
+                        if (SC && sct) {
+                            // the shortcut's 1x1 letters [Qout_sc][Qin]
+                            const int wr2 = (n_tile - p.sc.n_conv) * BNQ;
+                            if constexpr (MODE == MODE_PAIR) {
+                                tma_load_2d(b0 + 1 * C::B_TILE, &scm.w[0], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 2 * C::B_TILE, &scm.w[1], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 3 * C::B_TILE, &scm.w[2], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 4 * C::B_TILE, &scm.w[3], fb, cin0, wr2, pol_w);
+                            } else {
+                                tma_load_2d(b0 + 0 * C::B_TILE, &scm.w[0], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 1 * C::B_TILE, &scm.w[1], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 2 * C::B_TILE, &scm.w[2], fb, cin0, wr2, pol_w);
+                                tma_load_2d(b0 + 3 * C::B_TILE, &scm.w[3], fb, cin0, wr2, pol_w);
+                            }
+                        } else if constexpr (MODE == MODE_PAIR) {
                             // slots: [-W_i | W_r | W_i] [W_j | W_k | -W_j]; the sign-flip
                             // warp writes slots 0 and 5 from slots 2 and 3
                             tma_load_2d(b0 + 1 * C::B_TILE, &tmap_wr, fb, wcol, wrow, pol_w);
@@ -303,7 +344,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t dbase = tmem_base + static_cast<uint32_t>(buf * 4 * BNQ);
-                for (int kt = unit.k0; kt < unit.k1; ++kt) {
+                int k1 = unit.k1;
+                if constexpr (SC)
+                    if (unit.tile % p.num_n_tiles >= p.sc.n_conv) k1 = p.sc.ktiles;
+                for (int kt = unit.k0; kt < k1; ++kt) {
                     // pixels and letter tiles landed (pair mode: with the negated copies)
                     if (!flag_wait_or_abort(ready_word(stage), round + 1u, limit, abort_flag,
                                             STATUS_TIMEOUT_MMA)) {
@@ -395,7 +439,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         UnitIter units(p.sk.on, p.num_tiles, p.ktiles);
         Unit unit;
         while (ok && units.next(unit)) {
-            for (int kt = unit.k0; kt < unit.k1; ++kt) {
+            int k1 = unit.k1;
+            if constexpr (SC)
+                if (unit.tile % p.num_n_tiles >= p.sc.n_conv) k1 = p.sc.ktiles;
+            for (int kt = unit.k0; kt < k1; ++kt) {
                 if (!wait_or_abort(fullw_bar(stage), phase, limit, abort_flag,
                                    STATUS_TIMEOUT_PRODUCER)) {
                     ok = false;
@@ -445,6 +492,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         if constexpr (MODE == MODE_SEP)
             epilogue_direct_sep<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles, limit,
                                      abort_flag, geo);
+        else if constexpr (SC)
+            epilogue_direct_pair_sc<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles,
+                                         p.ktiles, p.sk, limit, abort_flag, geo, &p.sc);
         else
             epilogue_direct_pair<BNQ>(s, p.ep, p.y, tmem_base, accf0, acce0, p.num_tiles,
                                       p.ktiles, p.sk, limit, abort_flag, geo);
@@ -587,19 +637,21 @@ cudaError_t set_smem_once(K kern, int bytes, std::atomic<unsigned long long>& do
     return cudaSuccess;
 }
 
-template <int KAPPA, int BNQ, int MODE>
+template <int KAPPA, int BNQ, int MODE, bool SC = false>
 cudaError_t launch_cfg(const CUtensorMap maps[6], const TcParams& prm, int grid,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, const ScMaps* scm = nullptr) {
     using C = Cfg<KAPPA, BNQ, MODE>;
-    if constexpr (!C::FITS) {
+    if constexpr (!C::FITS || (SC && MODE != MODE_PAIR && MODE != MODE_QUAD)) {
         return cudaErrorInvalidValue;
     } else {
-        auto kern = qconv_tc_kernel<KAPPA, BNQ, MODE>;
+        auto kern = qconv_tc_kernel<KAPPA, BNQ, MODE, SC>;
         static std::atomic<unsigned long long> attr_done{0};
         cudaError_t e = set_smem_once(kern, C::SMEM_BYTES, attr_done);
         if (e != cudaSuccess) return e;
+        ScMaps none;
+        memset(&none, 0, sizeof(none));
         return launch_pdl(kern, dim3(grid), dim3(NUM_THREADS), C::SMEM_BYTES, stream, maps[0],
-                          maps[1], maps[2], maps[3], maps[4], prm);
+                          maps[1], maps[2], maps[3], maps[4], prm, scm != nullptr ? *scm : none);
     }
 }
 
@@ -1550,6 +1602,158 @@ cudaError_t launch_qconv_tc(const ConvShape& s, const void* x, const void* const
                : mode == MODE_SEP  ? launch_cfg<K, B, MODE_SEP>(maps, prm, grid, stream)   \
                : mode == MODE_SEPT ? launch_cfg<K, B, MODE_SEPT>(maps, prm, grid, stream)  \
                                    : launch_cfg<K, B, MODE_QUAD>(maps, prm, grid, stream);
+    QUAN_TC_CASE(16, 16)
+    QUAN_TC_CASE(16, 32)
+    QUAN_TC_CASE(16, 64)
+    QUAN_TC_CASE(32, 16)
+    QUAN_TC_CASE(32, 32)
+    QUAN_TC_CASE(32, 64)
+    QUAN_TC_CASE(64, 16)
+    QUAN_TC_CASE(64, 32)
+    QUAN_TC_CASE(64, 64)
+#undef QUAN_TC_CASE
+    snprintf(err, errlen, "no kernel instance for kappa=%d bnq=%d mode=%d", kappa, bnq, mode);
+    return cudaErrorInvalidValue;
+}
+
+// The convolution and a 1x1 shortcut on the same input in one QUAD/PAIR launch (the
+// shortcut's N tiles after the convolution's, on the K blocks of the filter tap that reads
+// x at (ho stride, wo stride)): the tile sizes, or false when the shapes do not allow it.
+bool tc_shortcut_plan(const ConvShape& s, int qout_sc, const TcOptions& opt, int* kappa_out,
+                      int* bnq_out, int* mode_out) {
+    if (s.sep || s.Qin % 16 != 0 || s.Qout % 16 != 0 || qout_sc <= 0 || qout_sc % 16 != 0)
+        return false;
+    if (s.pad >= s.kh || s.pad >= s.kw) return false;
+    // the 1x1 / stride shortcut without padding has the convolution's output size
+    if ((s.H - 1) / s.stride + 1 != s.Ho || (s.W - 1) / s.stride + 1 != s.Wo) return false;
+    int kappa = pick_kappa(s.Qin, opt.kappa);
+    const int bnq = pick_bnq(s.Qout, opt.bnq);
+    if (kappa == 0 || bnq == 0 || qout_sc % bnq != 0) return false;
+    int mode;
+    if (opt.mode == 1) mode = MODE_QUAD;
+    else if (opt.mode == 2) mode = MODE_PAIR;
+    else if (opt.mode == 0) mode = bnq >= 32 ? MODE_PAIR : MODE_QUAD;
+    else return false;
+    if (mode == MODE_PAIR && kappa == 64 && bnq == 64 && opt.kappa == 0) kappa = 32;
+    bool fits = false;
+#define QUAN_FIT_CASE(K, B)                                                          \
+    if (kappa == K && bnq == B)                                                      \
+        fits = mode == MODE_PAIR ? cfg_fits<K, B, MODE_PAIR>() : cfg_fits<K, B, MODE_QUAD>();
+    QUAN_FIT_CASE(16, 16) QUAN_FIT_CASE(16, 32) QUAN_FIT_CASE(16, 64)
+    QUAN_FIT_CASE(32, 16) QUAN_FIT_CASE(32, 32) QUAN_FIT_CASE(32, 64)
+    QUAN_FIT_CASE(64, 16) QUAN_FIT_CASE(64, 32) QUAN_FIT_CASE(64, 64)
+#undef QUAN_FIT_CASE
+    if (!fits) return false;
+    *kappa_out = kappa;
+    *bnq_out = bnq;
+    *mode_out = mode;
+    return true;
+}
+
+bool tc_shortcut_supported(const ConvShape& s, const void* x, const void* const w[4],
+                           const void* out, const EpilogueArgs& ep, const void* const wsc[4],
+                           int qout_sc, const EpilogueArgs& ep_sc, const void* out_sc,
+                           const TcOptions& opt) {
+    int kappa, bnq, mode;
+    if (!tc_shortcut_plan(s, qout_sc, opt, &kappa, &bnq, &mode)) return false;
+    if (!tc_supported(s, x, w, out, ep)) return false;
+    ConvShape s1 = s;  // the shortcut as a layer of its own, for the alignment checks
+    s1.kh = s1.kw = 1;
+    s1.pad = 0;
+    s1.Qout = qout_sc;
+    s1.Cout = 4 * qout_sc;
+    EpilogueArgs e1 = ep_sc;
+    e1.residual = nullptr;
+    return ep_sc.residual == nullptr && tc_supported(s1, x, wsc, out_sc, e1);
+}
+
+cudaError_t launch_qconv_tc_shortcut(const ConvShape& s, const void* x, const void* const w[4],
+                                     const EpilogueArgs& ep, void* out,
+                                     const void* const wsc[4], int qout_sc, int act_sc,
+                                     const EpilogueArgs& ep_sc, void* out_sc,
+                                     const TcOptions& opt, int num_sms, cudaStream_t stream,
+                                     char* err, size_t errlen) {
+    if (!load_encoders()) {
+        snprintf(err, errlen, "tensor-map encoders unavailable from the CUDA driver");
+        return cudaErrorNotSupported;
+    }
+    int kappa, bnq, mode;
+    if (!tc_shortcut_plan(s, qout_sc, opt, &kappa, &bnq, &mode)) {
+        snprintf(err, errlen, "no fused shortcut form for this layer");
+        return cudaErrorInvalidValue;
+    }
+    ConvShape s1 = s;  // the shortcut's 1x1 letters [Qout_sc][1][1][Qin]
+    s1.kh = s1.kw = 1;
+    s1.pad = 0;
+    s1.Qout = qout_sc;
+    s1.Cout = 4 * qout_sc;
+    CUtensorMap maps[6];
+    const MapKey key = make_key(s, x, w, out, kappa, bnq, 20);
+    if (!cache_lookup(key, maps)) {
+        if (!encode_x_im2col(&maps[0], s, x, kappa)) {
+            snprintf(err, errlen, "cuTensorMapEncodeIm2col failed for the activation tensor");
+            return cudaErrorInvalidValue;
+        }
+        for (int l = 0; l < 4; ++l)
+            if (!encode_w(&maps[1 + l], s, w[l], kappa, bnq)) {
+                snprintf(err, errlen, "cuTensorMapEncodeTiled failed for weight letter %d", l);
+                return cudaErrorInvalidValue;
+            }
+        maps[5] = maps[0];
+        cache_store(key, maps);
+    }
+    ScMaps scm;
+    {
+        CUtensorMap m2[6];
+        const MapKey key2 = make_key(s1, x, wsc, out_sc, kappa, bnq, 21);
+        if (!cache_lookup(key2, m2)) {
+            for (int l = 0; l < 4; ++l)
+                if (!encode_w(&m2[l], s1, wsc[l], kappa, bnq)) {
+                    snprintf(err, errlen, "cuTensorMapEncodeTiled failed for shortcut letter %d",
+                             l);
+                    return cudaErrorInvalidValue;
+                }
+            m2[4] = m2[5] = m2[0];
+            cache_store(key2, m2);
+        }
+        for (int l = 0; l < 4; ++l) scm.w[l] = m2[l];
+    }
+    TcParams prm;
+    prm.s = s;
+    prm.ep = ep;
+    prm.kchunks = s.Qin / kappa;
+    prm.ktiles = s.kh * s.kw * prm.kchunks;
+    prm.sc.n_conv = s.Qout / bnq;
+    prm.num_n_tiles = prm.sc.n_conv + qout_sc / bnq;
+    prm.y = out;
+    prm.sc.ktiles = prm.kchunks;
+    prm.sc.dh = prm.sc.dw = s.pad;
+    prm.sc.tap = s.pad * s.kw + s.pad;
+    prm.sc.Qout = qout_sc;
+    prm.sc.act = act_sc;
+    prm.sc.y = out_sc;
+    prm.sc.ep = ep_sc;
+    prm.sc.ep.residual = nullptr;
+    const long long tiles = (s.M + BM - 1) / BM * prm.num_n_tiles;
+    if (tiles > 0x7fffffffLL) {
+        snprintf(err, errlen, "too many tiles");
+        return cudaErrorInvalidValue;
+    }
+    prm.num_tiles = static_cast<int>(tiles);
+    prm.wait_limit_ns = opt.wait_limit_ns;
+    prm.inject_stall = opt.inject_stall;
+    prm.sk.on = 0;  // whole tiles: a split would cut shortcut and convolution tiles alike
+    prm.sk.partial = nullptr;
+    prm.sk.flags = nullptr;
+    const int grid = grid_for(opt, num_sms, prm.num_tiles);
+    set_kernel_name(mode == MODE_PAIR ? "qconv_tc_kernel<pair,kappa=%d,bnq=%d,shortcut>"
+                                      : "qconv_tc_kernel<quad,kappa=%d,bnq=%d,shortcut>",
+                    kappa, bnq);
+#define QUAN_TC_CASE(K, B)                                                               \
+    if (kappa == K && bnq == B)                                                          \
+        return mode == MODE_PAIR                                                         \
+                   ? launch_cfg<K, B, MODE_PAIR, true>(maps, prm, grid, stream, &scm)    \
+                   : launch_cfg<K, B, MODE_QUAD, true>(maps, prm, grid, stream, &scm);
     QUAN_TC_CASE(16, 16)
     QUAN_TC_CASE(16, 32)
     QUAN_TC_CASE(16, 64)

@@ -377,6 +377,69 @@ quan_status_t quan_qconv2d_fwd_ex(const void* x, const void* wr, const void* wi,
                     stride, pad, act, residual, out, stream, false, workspace, workspace_bytes);
 }
 
+quan_status_t quan_qconv2d_fwd_shortcut(
+    const void* x, const void* wr, const void* wi, const void* wj, const void* wk,
+    const float* bias, const float* iqbn_scale, const float* iqbn_shift, int N, int H, int W,
+    int Cin, int Cout, int kh, int kw, int stride, int pad, int act, const void* sc_wr,
+    const void* sc_wi, const void* sc_wj, const void* sc_wk, const float* sc_bias,
+    const float* sc_iqbn_scale, const float* sc_iqbn_shift, int Cout_sc, int sc_act, void* out,
+    void* out_sc, quan_stream_t stream) {
+    const void* w[4] = {wr, wi, wj, wk};
+    const void* wsc[4] = {sc_wr, sc_wi, sc_wj, sc_wk};
+    quan::ConvShape s, s1;
+    quan_status_t st = validate(&s, x, w, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh,
+                                kw, stride, pad, act, nullptr, out, 2);
+    if (st != QUAN_OK) return st;
+    st = validate(&s1, x, wsc, sc_bias, sc_iqbn_scale, sc_iqbn_shift, N, H, W, Cin, Cout_sc, 1,
+                  1, stride, 0, sc_act, nullptr, out_sc, 2);
+    if (st != QUAN_OK) return st;
+    if (s1.Ho != s.Ho || s1.Wo != s.Wo)
+        return fail(QUAN_ERR_INVALID_ARG,
+                    "the 1x1 shortcut's output (%dx%d) differs from the convolution's (%dx%d)",
+                    s1.Ho, s1.Wo, s.Ho, s.Wo);
+    if (overlaps(out, y_bytes(s, 2), out_sc, y_bytes(s1, 2)))
+        return fail(QUAN_ERR_INVALID_ARG, "out and out_sc overlap");
+    const size_t wb = w_bytes(s1, 2);
+    for (int L = 0; L < 4; ++L)
+        if (overlaps(out, y_bytes(s, 2), wsc[L], wb))
+            return fail(QUAN_ERR_INVALID_ARG, "out overlaps a shortcut weight tensor");
+    int num_sms = 0, cc = 0;
+    cudaError_t e;
+    if (!device_info(&num_sms, &cc, &e)) return cuda_fail(e, "device query");
+    const quan::EpilogueArgs ep{bias, iqbn_scale, iqbn_shift, nullptr};
+    const quan::EpilogueArgs ep_sc{sc_bias, sc_iqbn_scale, sc_iqbn_shift, nullptr};
+    quan::TcOptions opt;
+    opt.kappa = g_kappa.load();
+    opt.bnq = g_bnq.load();
+    opt.max_ctas = g_max_ctas.load();
+    opt.mode = g_mode.load();
+    opt.ws_halo = g_ws_halo.load();
+    opt.ws_issuers = g_ws_issuers.load();
+    opt.vs_rows = g_vs_rows.load();
+    opt.sk_ws = nullptr;
+    opt.sk_ws_bytes = 0;
+    opt.wait_limit_ns = g_wait_limit.load();
+    opt.inject_stall = g_inject.load();
+    if (g_path.load() != QUAN_PATH_SIMT && cc == 103 &&
+        quan::tc_shortcut_supported(s, x, w, out, ep, wsc, s1.Qout, ep_sc, out_sc, opt)) {
+        char err[256] = "";
+        e = quan::launch_qconv_tc_shortcut(s, x, w, ep, out, wsc, s1.Qout, sc_act, ep_sc, out_sc,
+                                           opt, num_sms, reinterpret_cast<cudaStream_t>(stream),
+                                           err, sizeof(err));
+        if (err[0] != '\0') return fail(QUAN_ERR_UNSUPPORTED, "%s", err);
+        if (e != cudaSuccess) return cuda_fail(e, "qconv_tc shortcut launch");
+        t_last_path = QUAN_PATH_TC;
+        t_last_kernel = quan::last_tc_kernel();
+        return QUAN_OK;
+    }
+    // no fused form for these shapes, path or device: the two layers as separate calls
+    st = run_bf16(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin, Cout, kh, kw,
+                  stride, pad, act, nullptr, out, stream);
+    if (st != QUAN_OK) return st;
+    return run_bf16(x, sc_wr, sc_wi, sc_wj, sc_wk, sc_bias, sc_iqbn_scale, sc_iqbn_shift, N, H,
+                    W, Cin, Cout_sc, 1, 1, stride, 0, sc_act, nullptr, out_sc, stream);
+}
+
 quan_status_t quan_qconv2d_fwd_res(const void* x, const void* wr, const void* wi, const void* wj,
                                    const void* wk, const float* bias, const float* iqbn_scale,
                                    const float* iqbn_shift, int N, int H, int W, int Cin,

@@ -292,6 +292,19 @@ struct SplitK {
     float* partial;      // workspace: one slot of 512 BNQ floats per CTA
     unsigned* flags;     // one flag per CTA: 1 while its partial is ready; the reader clears it
 };
+// A 1x1 shortcut fused into the convolution (the QUAD/PAIR kernel's SC form): its input is
+// the convolution's filter tap (dh, dw) = (pad, pad) on the same input (x at (ho stride,
+// wo stride)), so its N tiles n_conv .. num_n_tiles - 1 run the K blocks of that tap only,
+// with their own letters, and write their own output tensor with their own epilogue.
+struct ScParams {
+    int n_conv;        // N tiles of the convolution; the rest are the shortcut's
+    int ktiles;        // K blocks of a shortcut tile: Qin / KAPPA
+    int tap, dh, dw;   // the convolution's filter tap that is the shortcut's input pixel
+    int Qout;          // the shortcut's quaternion output channels
+    int act;
+    void* y;           // the shortcut's output [M][4 Qout]
+    EpilogueArgs ep;   // its bias / IQBN scale and shift (no residual)
+};
 enum : int { UNIT_WHOLE = 0, UNIT_HEAD = 1, UNIT_TAIL = 2 };
 struct Unit {
     int tile, k0, k1, kind;
@@ -536,6 +549,214 @@ __device__ __forceinline__ void epilogue_direct_pair(const ConvShape& s, const E
                     const float z1 =
                         fmaf(sc[2 * t + 1], E[k][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
                     w[t] = pack_bf16x2(activate(z0, s.act), activate(z1, s.act));
+                }
+                if (row0 + k < g.rows)
+                    st_global_na(out + (g.m0 + row0 + k) * Cout + cb,
+                                 make_uint4(w[0], w[1], w[2], w[3]));
+            }
+            if (b + 1 < NB) tmem_ld_wait();
+        }
+        if (unit.kind == UNIT_HEAD) {
+            // every epilogue thread's partial stores are visible device-wide before the flag
+            __threadfence();
+            named_bar_sync(2, 256);
+            if (threadIdx.x == EPI_WARP0 * 32) st_release_gpu(sk.flags + blockIdx.x, 1u);
+        }
+    }
+}
+
+// The same for the fused shortcut form of the QUAD/PAIR kernel (whole tiles): tiles from N
+// tile sc->n_conv on are the shortcut's (ScParams), written with its own output, channel
+// count, per-channel vectors and activation.
+template <int BNQ, typename Geo>
+__device__ __forceinline__ void epilogue_direct_pair_sc(const ConvShape& s, const EpilogueArgs& ep,
+                                                     void* y, uint32_t tmem_base,
+                                                     uint32_t accf0, uint32_t acce0,
+                                                     int num_tiles, int ktiles, const SplitK& sk,
+                                                     uint64_t limit,
+                                                     volatile int* abort_flag, Geo geo,
+                                                     const ScParams* sc) {
+    constexpr int CH = BNQ < 32 ? BNQ : 32;  // columns per TMEM load
+    constexpr int NCH = CH / 8;              // 8-channel chunks per load: 2 or 4
+    constexpr int SLICES = BNQ / CH;
+    constexpr int NB = 2 * SLICES;           // blocks per warp and tile
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
+    const int half = (warp - EPI_WARP0) >> 2;  // output components 2 half, 2 half + 1
+    const int ci = lane % NCH;                 // this lane's chunk after the transpose
+    const int row0 = quad * 32 + NCH * (lane / NCH);  // its rows: row0 .. row0 + NCH - 1
+    const long long Cout0 = s.Cout;
+    const __nv_bfloat16* res0 = static_cast<const __nv_bfloat16*>(ep.residual);
+    __nv_bfloat16* out0 = static_cast<__nv_bfloat16*>(y);
+    // the tile's output parameters (the convolution's or the shortcut's)
+    const EpilogueArgs* epp = &ep;
+    // block b of this warp: component 2 half + b / SLICES, columns (b % SLICES) CH ..
+    auto tmem_col = [&](int b) { return (2 * half + b / SLICES) * BNQ + (b % SLICES) * CH; };
+    auto load_block = [&](uint32_t taddr, int b, uint32_t(&v)[CH]) {
+        if constexpr (CH == 32)
+            tmem_ld_32x32b_x32(taddr + tmem_col(b), v);
+        else
+            tmem_ld_32x32b_x16(taddr + tmem_col(b), v);
+    };
+    // the per-channel vectors of this lane's 8 channels of block b
+    auto load_vectors = [&](int cb, float(&scv)[8], float(&sh)[8]) {
+        const EpilogueArgs* e = &ep;
+        e = epp;
+        float bi[8];
+        load8(e->scale, cb, 1.0f, scv);
+        load8(e->shift, cb, 0.0f, sh);
+        load8(e->bias, cb, 0.0f, bi);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) sh[e] = fmaf(scv[e], bi[e], sh[e]);
+    };
+    // this thread's floats in a partial slot: block b, 4-float group j -> lanes contiguous
+    const int ew = warp - EPI_WARP0;  // 0..7
+    auto pslot = [&](const float* slot, int b, int j) {
+        return reinterpret_cast<float4*>(const_cast<float*>(slot)) +
+               ((ew * NB + b) * (CH / 4) + j) * 32 + lane;
+    };
+    int local = 0;
+    UnitIter units(sk.on, num_tiles, ktiles);
+    Unit unit;
+    while (units.next(unit)) {
+        const int tile = unit.tile;
+        const int buf = local & 1;
+        const uint32_t use = static_cast<uint32_t>(local >> 1) & 1u;
+        ++local;
+        bool ok = true;
+        if (lane == 0)
+            ok = wait_or_abort(accf0 + 8u * buf, use, limit, abort_flag, STATUS_TIMEOUT_EPILOGUE);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        // leave together: a warp that gave up must not strand the others at a barrier
+        if (named_bar_or(1, 256, !ok)) break;
+        if (unit.kind == UNIT_TAIL) {
+            // the rest of this tile's K blocks were done by the next CTA: wait for its partial
+            bool ready = true;
+            if (threadIdx.x == EPI_WARP0 * 32) {
+                ready = gflag_wait_or_abort(sk.flags + blockIdx.x + 1, limit, abort_flag,
+                                            STATUS_TIMEOUT_EPILOGUE);
+                // cleared for the next call (whose writer runs only after this grid ends)
+                if (ready) sk.flags[blockIdx.x + 1] = 0u;
+            }
+            if (named_bar_or(1, 256, !ready)) break;
+        }
+        tc_fence_after();
+        EpiTile g = geo(tile);
+        long long Cout = Cout0;
+        int Qout = s.Qout, act = s.act;
+        const __nv_bfloat16* res = res0;
+        __nv_bfloat16* out = out0;
+        {
+            // this tile's output: the convolution's or the fused shortcut's
+            const bool sct = g.n_tile >= sc->n_conv;
+            if (sct) {
+                g.n_tile -= sc->n_conv;
+                Qout = sc->Qout;
+                act = sc->act;
+                Cout = 4LL * Qout;
+                epp = &sc->ep;
+                res = nullptr;
+                out = static_cast<__nv_bfloat16*>(sc->y);
+            } else {
+                epp = &ep;
+            }
+        }
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                               static_cast<uint32_t>(buf * 4 * BNQ);
+        const int c_tile = g.n_tile * BNQ + 8 * ci;  // + q Qout + slice offset: lane's channel
+        uint32_t va[CH], vb[CH];
+        float sca[8], sha[8], scb[8], shb[8];
+        load_block(taddr, 0, va);
+        load_vectors(c_tile + (2 * half) * Qout, sca, sha);
+        tmem_ld_wait();
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            uint32_t(&v)[CH] = (b & 1) ? vb : va;
+            uint32_t(&vn)[CH] = (b & 1) ? va : vb;
+            float(&sc)[8] = (b & 1) ? scb : sca;
+            float(&sh)[8] = (b & 1) ? shb : sha;
+            float(&scn)[8] = (b & 1) ? sca : scb;
+            float(&shn)[8] = (b & 1) ? sha : shb;
+            const int q = 2 * half + b / SLICES;
+            const int cb = c_tile + q * Qout + (b % SLICES) * CH;
+            if (b + 1 < NB) {
+                // next block in flight while this one is processed
+                load_block(taddr, b + 1, vn);
+                load_vectors(c_tile + (2 * half + (b + 1) / SLICES) * Qout +
+                                 ((b + 1) % SLICES) * CH,
+                             scn, shn);
+            } else {
+                // the tile's accumulator is in registers: hand the buffer back
+                tc_fence_before();
+                mbar_arrive_relaxed(acce0 + 8u * buf);
+            }
+            if (unit.kind == UNIT_HEAD) {
+                // this CTA's share of the tile: the raw accumulator to the partial slot (L2)
+                float* my_slot = sk.partial + static_cast<size_t>(blockIdx.x) * (512 * BNQ);
+#pragma unroll
+                for (int j = 0; j < CH / 4; ++j)
+                    __stcg(pslot(my_slot, b, j),
+                           make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                       __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3])));
+                if (b + 1 < NB) tmem_ld_wait();
+                continue;
+            }
+            if (unit.kind == UNIT_TAIL) {
+                // the next CTA's share, read from L2 (never from this SM's L1)
+                const float* next_slot =
+                    sk.partial + static_cast<size_t>(blockIdx.x + 1) * (512 * BNQ);
+#pragma unroll
+                for (int j = 0; j < CH / 4; ++j) {
+                    const float4 q4 = __ldcg(pslot(next_slot, b, j));
+                    v[4 * j] = __float_as_uint(__uint_as_float(v[4 * j]) + q4.x);
+                    v[4 * j + 1] = __float_as_uint(__uint_as_float(v[4 * j + 1]) + q4.y);
+                    v[4 * j + 2] = __float_as_uint(__uint_as_float(v[4 * j + 2]) + q4.z);
+                    v[4 * j + 3] = __float_as_uint(__uint_as_float(v[4 * j + 3]) + q4.w);
+                }
+            }
+            uint4 r4[NCH];
+            if (res != nullptr) {
+#pragma unroll
+                for (int k = 0; k < NCH; ++k) {
+                    r4[k] = make_uint4(0u, 0u, 0u, 0u);
+                    if (row0 + k < g.rows)
+                        r4[k] = ld_global_na(res + (g.m0 + row0 + k) * Cout + cb);
+                }
+            }
+            float E[NCH][8];  // E[j][e]: channel 8 j + e of this lane's row
+#pragma unroll
+            for (int j = 0; j < NCH; ++j)
+#pragma unroll
+                for (int e = 0; e < 8; ++e) E[j][e] = __uint_as_float(v[8 * j + e]);
+            if constexpr (NCH == 4) {
+                chunk_transpose_stage<2, 4>(E, ci);
+                chunk_transpose_stage<1, 4>(E, ci);
+            } else {
+                chunk_transpose_stage<1, 2>(E, ci);
+            }
+            // now E[k][e] = channel cb + e of row row0 + k
+#pragma unroll
+            for (int k = 0; k < NCH; ++k) {
+                float rz[8];
+                if (res != nullptr) {
+                    const __nv_bfloat162* rh = reinterpret_cast<const __nv_bfloat162*>(&r4[k]);
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {
+                        const float2 f = __bfloat1622float2(rh[t]);
+                        rz[2 * t] = f.x;
+                        rz[2 * t + 1] = f.y;
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) rz[e] = 0.0f;
+                }
+                uint32_t w[4];
+#pragma unroll
+                for (int t = 0; t < 4; ++t) {
+                    const float z0 = fmaf(sc[2 * t], E[k][2 * t], sh[2 * t]) + rz[2 * t];
+                    const float z1 =
+                        fmaf(sc[2 * t + 1], E[k][2 * t + 1], sh[2 * t + 1]) + rz[2 * t + 1];
+                    w[t] = pack_bf16x2(activate(z0, act), activate(z1, act));
                 }
                 if (row0 + k < g.rows)
                     st_global_na(out + (g.m0 + row0 + k) * Cout + cb,

@@ -62,6 +62,8 @@ def load():
         lib.quan_qconv2d_fwd_f32.argtypes = _conv_args + [_vp, _vp]
         lib.quan_qconv2d_fwd_res.argtypes = _conv_args + [_vp, _vp, _vp]
         lib.quan_qconv2d_fwd_ex.argtypes = _conv_args + [_vp, _vp, ctypes.c_size_t, _vp, _vp]
+        lib.quan_qconv2d_fwd_shortcut.argtypes = (_conv_args + [_vp] * 7 + [_i, _i] +
+                                                  [_vp, _vp, _vp])
         lib.quan_qconv2d_fwd_workspace_size.argtypes = []
         lib.quan_qconv2d_fwd_workspace_size.restype = ctypes.c_size_t
         lib.quan_qconv2d_sep_fwd.argtypes = _conv_args + [_vp, _vp]
@@ -105,7 +107,7 @@ def load():
         lib.quan_last_error_message.restype = ctypes.c_char_p
         lib.quan_version.argtypes = []
         for name in ("quan_qconv2d_fwd", "quan_qconv2d_fwd_f32", "quan_qconv2d_fwd_res",
-                     "quan_qconv2d_fwd_ex",
+                     "quan_qconv2d_fwd_ex", "quan_qconv2d_fwd_shortcut",
                      "quan_qconv2d_sep_fwd", "quan_poincare_fwd", "quan_qconv2d_bwd_data",
                      "quan_qconv2d_sep_bwd_data", "quan_qconv2d_bwd_weight",
                      "quan_qconv2d_bwd_data_static", "quan_iqbn_batch_stats",
@@ -176,6 +178,38 @@ def quan_qconv2d_fwd_ex(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W
                                       Cin, Cout, kh, kw, stride, pad, act, _ptr(residual),
                                       _ptr(workspace), workspace_bytes, _ptr(out),
                                       _stream(stream)))
+
+
+def quan_qconv2d_fwd_shortcut(x, wr, wi, wj, wk, bias, iqbn_scale, iqbn_shift, N, H, W, Cin,
+                              Cout, kh, kw, stride, pad, act, sc_wr, sc_wi, sc_wj, sc_wk,
+                              sc_bias, sc_iqbn_scale, sc_iqbn_shift, Cout_sc, sc_act, out,
+                              out_sc, stream=None) -> None:
+    _check(load().quan_qconv2d_fwd_shortcut(
+        _ptr(x), _ptr(wr), _ptr(wi), _ptr(wj), _ptr(wk), _ptr(bias), _ptr(iqbn_scale),
+        _ptr(iqbn_shift), N, H, W, Cin, Cout, kh, kw, stride, pad, act, _ptr(sc_wr),
+        _ptr(sc_wi), _ptr(sc_wj), _ptr(sc_wk), _ptr(sc_bias), _ptr(sc_iqbn_scale),
+        _ptr(sc_iqbn_shift), Cout_sc, sc_act, _ptr(out), _ptr(out_sc), _stream(stream)))
+
+
+def qconv2d_shortcut(x, w, sc_w, *, stride=2, pad=1, bias=None, scale=None, shift=None,
+                     act=QUAN_ACT_NONE, sc_bias=None, sc_scale=None, sc_shift=None,
+                     sc_act=QUAN_ACT_NONE, out=None, out_sc=None, stream=None):
+    """A convolution (letters w = (wr, wi, wj, wk)) and the 1x1 shortcut of the same input
+    (letters sc_w, same stride, no padding) in one call: returns (out, out_sc), allocated
+    like qconv2d's when not given (bf16 CUDA tensors)."""
+    import torch
+    N, H, W, Cin = x.shape
+    Qout, kh, kw, _ = w[0].shape
+    Cout, Cout_sc = 4 * Qout, 4 * sc_w[0].shape[0]
+    Ho, Wo = out_size(H, kh, stride, pad), out_size(W, kw, stride, pad)
+    if out is None:
+        out = torch.empty((N, Ho, Wo, Cout), dtype=x.dtype, device=x.device)
+    if out_sc is None:
+        out_sc = torch.empty((N, Ho, Wo, Cout_sc), dtype=x.dtype, device=x.device)
+    quan_qconv2d_fwd_shortcut(x, *w, bias, scale, shift, N, H, W, Cin, Cout, kh, kw, stride, pad,
+                              act, *sc_w, sc_bias, sc_scale, sc_shift, Cout_sc, sc_act, out,
+                              out_sc, stream)
+    return out, out_sc
 
 
 def quan_qconv2d_fwd_workspace_size() -> int:

@@ -216,3 +216,34 @@ def test_fused_stem_pool_validates(lib):
     assert f(*args(None)) == bad                           # no output
     assert f(*args(FAKE + 0x10)) == bad                    # output overlaps the input
     assert f(*args(0x9000000, x=None)) == bad              # no input
+
+
+def _call_sc(lib, **kw):
+    # quan_qconv2d_fwd_shortcut: the downsampling block's 3x3/2 convolution and its 1x1/2
+    # shortcut of the same input
+    a = dict(x=FAKE, w=FAKE + 0x1000, bias=None, scale=None, shift=None, N=1, H=8, W=8,
+             Cin=64, Cout=128, kh=3, kw=3, stride=2, pad=1, act=1, sw=FAKE + 0x100000,
+             sbias=None, sscale=None, sshift=None, Cout_sc=128, sact=0, out=0x7000000,
+             out_sc=0x8000000, stream=None)
+    a.update(kw)
+    at = lambda base, k: None if base is None else base + k
+    return lib.quan_qconv2d_fwd_shortcut(
+        a["x"], a["w"], at(a["w"], 0x10000), at(a["w"], 0x20000), at(a["w"], 0x30000),
+        a["bias"], a["scale"], a["shift"], a["N"], a["H"], a["W"], a["Cin"], a["Cout"],
+        a["kh"], a["kw"], a["stride"], a["pad"], a["act"], a["sw"], at(a["sw"], 0x10000),
+        at(a["sw"], 0x20000), at(a["sw"], 0x30000), a["sbias"], a["sscale"], a["sshift"],
+        a["Cout_sc"], a["sact"], a["out"], a["out_sc"], a["stream"])
+
+
+@pytest.mark.parametrize("bad", [
+    dict(x=None), dict(sw=None), dict(out_sc=None),
+    dict(Cout_sc=10),                 # not a multiple of 4
+    dict(sact=7),
+    dict(sscale=0x9000000),           # shortcut scale without shift
+    dict(pad=0),                      # 3x3/2 without padding: 3x3 output, the 1x1/2 one 4x4
+    dict(out_sc=0x7000000 + 64),      # out_sc overlaps out
+    dict(out_sc=FAKE),                # out_sc overlaps x
+])
+def test_fused_shortcut_invalid_arguments(lib, bad):
+    assert _call_sc(lib, **bad) == quan.QUAN_ERR_INVALID_ARG
+    assert lib.quan_last_error_message()
