@@ -609,12 +609,6 @@ __device__ __forceinline__ void epilogue_direct_pair_sc(const ConvShape& s, cons
 #pragma unroll
         for (int e = 0; e < 8; ++e) sh[e] = fmaf(scv[e], bi[e], sh[e]);
     };
-    // this thread's floats in a partial slot: block b, 4-float group j -> lanes contiguous
-    const int ew = warp - EPI_WARP0;  // 0..7
-    auto pslot = [&](const float* slot, int b, int j) {
-        return reinterpret_cast<float4*>(const_cast<float*>(slot)) +
-               ((ew * NB + b) * (CH / 4) + j) * 32 + lane;
-    };
     int local = 0;
     UnitIter units(sk.on, num_tiles, ktiles);
     Unit unit;
@@ -629,17 +623,6 @@ __device__ __forceinline__ void epilogue_direct_pair_sc(const ConvShape& s, cons
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         // leave together: a warp that gave up must not strand the others at a barrier
         if (named_bar_or(1, 256, !ok)) break;
-        if (unit.kind == UNIT_TAIL) {
-            // the rest of this tile's K blocks were done by the next CTA: wait for its partial
-            bool ready = true;
-            if (threadIdx.x == EPI_WARP0 * 32) {
-                ready = gflag_wait_or_abort(sk.flags + blockIdx.x + 1, limit, abort_flag,
-                                            STATUS_TIMEOUT_EPILOGUE);
-                // cleared for the next call (whose writer runs only after this grid ends)
-                if (ready) sk.flags[blockIdx.x + 1] = 0u;
-            }
-            if (named_bar_or(1, 256, !ready)) break;
-        }
         tc_fence_after();
         EpiTile g = geo(tile);
         long long Cout = Cout0;
@@ -690,30 +673,6 @@ __device__ __forceinline__ void epilogue_direct_pair_sc(const ConvShape& s, cons
                 tc_fence_before();
                 mbar_arrive_relaxed(acce0 + 8u * buf);
             }
-            if (unit.kind == UNIT_HEAD) {
-                // this CTA's share of the tile: the raw accumulator to the partial slot (L2)
-                float* my_slot = sk.partial + static_cast<size_t>(blockIdx.x) * (512 * BNQ);
-#pragma unroll
-                for (int j = 0; j < CH / 4; ++j)
-                    __stcg(pslot(my_slot, b, j),
-                           make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                       __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3])));
-                if (b + 1 < NB) tmem_ld_wait();
-                continue;
-            }
-            if (unit.kind == UNIT_TAIL) {
-                // the next CTA's share, read from L2 (never from this SM's L1)
-                const float* next_slot =
-                    sk.partial + static_cast<size_t>(blockIdx.x + 1) * (512 * BNQ);
-#pragma unroll
-                for (int j = 0; j < CH / 4; ++j) {
-                    const float4 q4 = __ldcg(pslot(next_slot, b, j));
-                    v[4 * j] = __float_as_uint(__uint_as_float(v[4 * j]) + q4.x);
-                    v[4 * j + 1] = __float_as_uint(__uint_as_float(v[4 * j + 1]) + q4.y);
-                    v[4 * j + 2] = __float_as_uint(__uint_as_float(v[4 * j + 2]) + q4.z);
-                    v[4 * j + 3] = __float_as_uint(__uint_as_float(v[4 * j + 3]) + q4.w);
-                }
-            }
             uint4 r4[NCH];
             if (res != nullptr) {
 #pragma unroll
@@ -763,12 +722,6 @@ __device__ __forceinline__ void epilogue_direct_pair_sc(const ConvShape& s, cons
                                  make_uint4(w[0], w[1], w[2], w[3]));
             }
             if (b + 1 < NB) tmem_ld_wait();
-        }
-        if (unit.kind == UNIT_HEAD) {
-            // every epilogue thread's partial stores are visible device-wide before the flag
-            __threadfence();
-            named_bar_sync(2, 256);
-            if (threadIdx.x == EPI_WARP0 * 32) st_release_gpu(sk.flags + blockIdx.x, 1u);
         }
     }
 }
