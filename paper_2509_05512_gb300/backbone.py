@@ -77,7 +77,8 @@ class BackboneRunner:
                 x_bits = inputs.backbone_input(N=N, H=H, seed=seed)
             self.x_host = x_bits
             self.x = up(x_bits)
-        self.launches_per_step = len(self.layers)
+        # one launch per layer; the fused stem + max pool is one launch for two layers
+        self.launches_per_step = len(self.layers) - (1 if self.fused else 0)
         # split_k: the convolutions run through quan_qconv2d_fwd_ex with one workspace (the
         # layers run one after another on the main stream; the shortcuts on the side stream
         # run without one), so layers whose tiles leave a partial last wave of CTAs spread

@@ -118,6 +118,8 @@ def test_backbone_shortcuts_on_a_second_stream_bit_identical():
     ovl = BackboneRunner(torch, quan, inputs, N=3, x_bits=x_bits, fuse_stem_pool=True,
                          overlap_shortcuts=True)
     assert sorted(ovl.side) == [7, 12, 17]
+    # the bench's gpu_launches: 19 convolutions and the fused stem + max pool per step
+    assert ovl.launches_per_step == 20
     stream = torch.cuda.current_stream().cuda_stream
     ref.step(stream)
     cap = torch.cuda.Stream()
