@@ -85,3 +85,20 @@ def test_recorded_traffic_lookup(tmp_path):
     assert bench.traffic_key(A) == "c2a:bwd:sep"
     A.direction, A.variant = "fwd", "full"
     assert bench.traffic_key(A) == "c2a"
+
+
+def test_kernel_sources_table_names_existing_files():
+    # the traffic hash of a kernel covers the files of its KERNEL_SOURCES entry and the
+    # shared headers: each must exist, or an edit to the kernel would go unnoticed
+    import os
+    csrc = os.path.join(bench.ROOT, "paper_2509_05512_gb300", "csrc")
+    for kernel, files in bench.KERNEL_SOURCES.items():
+        for name in files + bench.SHARED_DEVICE_SOURCES:
+            assert os.path.isfile(os.path.join(csrc, name)), (kernel, name)
+        assert name not in bench.HOST_ONLY_SOURCES
+    # the dominant kernel of the default bench line has a record taken on its current
+    # sources (the kernel name is the library's, without template arguments)
+    import json
+    with open(os.path.join(bench.ROOT, "profiles", "ncu_traffic.json")) as f:
+        rec = json.load(f)["backbone"]
+    assert rec["kernel"].split("<")[0] in bench.KERNEL_SOURCES
