@@ -70,8 +70,10 @@ def parse_args():
                          "convolution, forked and joined by events)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0,
-                    help="target duration of the bounded oracle sample")
+    ap.add_argument("--cpu-seconds", type=float, default=24.0,
+                    help="target of the bounded oracle sample, sized from a one-image run "
+                         "(the oracle's threads scale better on many images, so the sample "
+                         "itself takes about half of it: ~10-12 s)")
     ap.add_argument("--profile", action="store_true",
                     help="for ncu: exactly W + K plain launches, no clock sampling, no e2e "
                          "or CPU legs")
